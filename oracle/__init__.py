@@ -1,0 +1,2 @@
+"""CPU fp64 oracle for SWAN (test infrastructure; never imported by the library)."""
+from .swan_oracle import *  # noqa: F401,F403

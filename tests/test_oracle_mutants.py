@@ -1,0 +1,82 @@
+"""Plant plausible mistakes in a copy of the oracle; each must fail a pin.
+
+The mutant is the oracle's own source with one small textual change, loaded as
+a separate module on the CPU; the real oracle is never modified.
+"""
+import importlib.util
+import os
+import sys
+import types
+
+import pytest
+
+from tests.oracle_pins import ALL_PINS
+
+SRC = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))),
+                   "oracle", "swan_oracle.py")
+
+# (name, original text, mutated text, count of occurrences to replace)
+MUTANTS = [
+    ("transposed_R_for_cache",
+     'np.einsum("bhti,hij->bhtj"', 'np.einsum("bhti,hji->bhtj"', 1),
+    ("transposed_R_for_query",
+     "q_hat = q[b, hq] @ self.R_qk[h]", "q_hat = q[b, hq] @ self.R_qk[h].T", 1),
+    ("rotate_back_without_transpose",
+     "@ np.asarray(R, np.float64).T", "@ np.asarray(R, np.float64)", 1),
+    ("prune_smallest",
+     'np.argsort(-mag, axis=-1, kind="stable")[..., :k]',
+     'np.argsort(mag, axis=-1, kind="stable")[..., :k]', 1),
+    ("prune_signed_not_magnitude",
+     "mag = np.abs(x16.astype(np.float64))", "mag = x16.astype(np.float64)", 1),
+    ("prune_ties_to_higher_index",
+     'order = np.argsort(-mag, axis=-1, kind="stable")[..., :k]',
+     'order = (mag.shape[-1] - 1 - np.argsort(-mag[..., ::-1], axis=-1, kind="stable"))[..., :k]', 1),
+    ("scale_sqrt_k",
+     "s = np.concatenate([s_sp, s_bf]) / math.sqrt(d)",
+     "s = np.concatenate([s_sp, s_bf]) / math.sqrt(ka)", 1),
+    ("dropped_buffer_values",
+     "o = o + p[n_sp:] @ np.asarray(buf_v, np.float64)", "o = o", 1),
+    ("value_sum_without_weights",
+     "w = np.asarray(p, np.float64)[:, None] * np.asarray(vals, np.float64)",
+     "w = np.asarray(vals, np.float64) + 0 * np.asarray(p)[:, None]", 1),
+    ("key_indices_used_for_values",
+     "o = sparse_value_sum(p[:n_sp], sp_idx_v[:, :ka]", "o = sparse_value_sum(p[:n_sp], sp_idx[:, :ka]", 1),
+    ("combine_wrong_sign",
+     "np.exp(ms - m)", "np.exp(m - ms)", 1),
+    ("evict_newest",
+     "ik, vk = self._prune(self.buf_k[:, :, :n])", "ik, vk = self._prune(self.buf_k[:, :, -n:])", 1),
+    ("gqa_modulo_mapping",
+     "h = hq // self.G\n                q_hat", "h = hq % self.H_kv\n                q_hat", 1),
+    ("no_fp16_storage",
+     "return to_fp16(y) if self.round else y", "return y", 1),
+    ("break_even_without_buffer",
+     "return d * d / (d - k) + b", "return d * d / (d - k)", 1),
+    ("bytes_without_offset",
+     "return k * (value_bytes + index_bytes) + offset_bytes",
+     "return k * (value_bytes + index_bytes)", 1),
+    ("runtime_k_ignored",
+     "s_sp = sparse_scores(q_hat, sp_idx[:, :ka], sp_vals_k[:, :ka])",
+     "s_sp = sparse_scores(q_hat, sp_idx, sp_vals_k)", 1),
+]
+
+
+def _load_mutant(name, old, new, count):
+    src = open(SRC).read()
+    assert src.count(old) == count, (name, src.count(old))
+    mod = types.ModuleType("oracle_mutant_" + name)
+    mod.__file__ = SRC
+    sys.modules[mod.__name__] = mod
+    exec(compile(src.replace(old, new), SRC, "exec"), mod.__dict__)
+    return mod
+
+
+@pytest.mark.parametrize("name,old,new,count", MUTANTS, ids=[m[0] for m in MUTANTS])
+def test_mutant_is_caught(name, old, new, count):
+    mod = _load_mutant(name, old, new, count)
+    failed = []
+    for pin in ALL_PINS:
+        try:
+            pin(mod)
+        except Exception as e:  # noqa: BLE001 - any failure counts as caught
+            failed.append((pin.__name__, type(e).__name__))
+    assert failed, f"mutant {name} passed every pin"

@@ -1,0 +1,417 @@
+"""SWAN decode benchmark on one GB300 (or N replicas, one per GPU).
+
+One step = one pass of the whole hot path (Algorithm 1 for one token): append
+one new key/value per sequence (rotate, insert into the dense buffer, evict
+the oldest buffered vector and prune it into the sparse cache) and one decode
+attention over the hybrid cache (rotate q, sparse + dense scores, online
+softmax, value scatter, split combine, rotate-back).
+
+Default workload: a Llama-2-7B-shaped attention layer at 32k context: batch
+16, 32 MHA heads, head_dim 128, 32768 sparse tokens + 128 dense buffer tokens,
+keep k = 64, synthetic low-rank keys/values (sigma_i ∝ 1/i), per-head random
+orthogonal R.  Metric: decode KV-tokens/s (token-head records attended per
+second) and HBM GB/s over the algorithmic bytes.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl swan|reference]
+  python bench.py --workload gqa-131k   # Llama-3-8B GQA layer, 131072 ctx
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import re
+import statistics
+import subprocess
+import sys
+import time
+
+for _v in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS"):
+    os.environ.setdefault(_v, "1")
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+
+D = 128
+WORKLOADS = {
+    "llama2-7b-layer-32k": dict(B=16, H_q=32, H_kv=32, L_s=32768, n_b=128, k=64, k_store=64,
+                                desc="Llama-2-7B-shaped layer: batch 16, 32 MHA heads, d 128, "
+                                     "32768 sparse + 128 dense-buffer tokens, k 64"),
+    "gqa-131k": dict(B=4, H_q=32, H_kv=8, L_s=130944, n_b=128, k=56, k_store=56,
+                     desc="Llama-3-8B-shaped GQA layer: batch 4, 32 q / 8 kv heads, d 128, "
+                          "130944 sparse + 128 dense-buffer tokens (131072 ctx), k 56"),
+}
+METRIC = "decode-attention KV-tokens/s and achieved HBM GB/s (% of 8 TB/s) at 32k ctx"
+NOMINAL_HBM_GBS = 8000.0
+
+
+def measured_peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return json.load(f)
+    except OSError:
+        return None
+
+
+def decode_kernel_traffic(workload: str):
+    """DRAM bytes per decode-kernel launch from the committed ncu summary, if
+    it was taken on the current kernel source (else None)."""
+    src = os.path.join(ROOT, "paper_2511_18936_gb300", "csrc", "decode.cu")
+    digest = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+    path = os.path.join(ROOT, "profiles", f"decode_kernel_{workload}.md")
+    try:
+        text = open(path).read()
+    except OSError:
+        return None
+    m_src = re.search(r"decode\.cu sha256\[:16\]:\s*([0-9a-f]{16})", text)
+    m_tr = re.search(r"dram bytes per launch:\s*([0-9.eE+]+)", text)
+    if not m_src or not m_tr or m_src.group(1) != digest:
+        return None
+    return float(m_tr.group(1))
+
+
+class ClockSampler:
+    """nvidia-smi samples of SM clocks and throttle reasons during a region."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+        time.sleep(0.3)
+        return self
+
+    def __exit__(self, *exc):
+        self.out = ""
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.out, _ = self.proc.communicate(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+                self.out, _ = self.proc.communicate()
+
+    def summary(self):
+        rows = []
+        for ln in (self.out or "").splitlines():
+            parts = [p.strip() for p in ln.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                rows.append((float(parts[1]), float(parts[2]), parts[5:9]))
+            except ValueError:
+                continue
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unavailable"], "samples": 0}
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for _, _, r in rows for i, v in enumerate(r) if v.lower() == "active"})
+        return {"sm_mhz": statistics.median(r[0] for r in rows), "sm_max_mhz": max(r[1] for r in rows),
+                "reasons": reasons, "samples": len(rows)}
+
+
+# ---------------------------------------------------------------------------
+# CPU baseline: the oracle as it stands, on a bounded sample of the workload
+# ---------------------------------------------------------------------------
+
+def oracle_sample(wl, n_units: int, seed: int = 0):
+    """Prepare the compressed state of ``n_units`` (batch, kv-head) units of
+    the workload on the host (untimed) and return a step function that runs
+    one oracle step (append one token, decode every query head of the unit)."""
+    import oracle
+    from paper_2511_18936_gb300 import synth
+    G = wl["H_q"] // wl["H_kv"]
+    L = wl["L_s"] + wl["n_b"]
+    states = []
+    for u in range(n_units):
+        R = synth.rotations(1, D, seed=seed, workload=7, layer=0, tensor_id=synth.T_R_QK, )
+        k = synth.lowrank_kv(1, 1, L + 64, D, seed, 7, u, synth.T_K)
+        v = synth.lowrank_kv(1, 1, L + 64, D, seed, 7, u, synth.T_V)
+        st = oracle.SwanOracle(R, batch=1, n_q_heads=G, k_store=wl["k_store"], buffer_cap=wl["n_b"])
+        st.append(k[:, :, :wl["L_s"]], v[:, :, :wl["L_s"]])
+        st.flush()
+        st.append(k[:, :, wl["L_s"]:L], v[:, :, wl["L_s"]:L])
+        st.set_k(wl["k"])
+        q = synth.gaussian_fp16((1, G, D), seed, 7, u, synth.T_Q)
+        states.append((st, k[:, :, L:], v[:, :, L:], q))
+    step_no = [0]
+
+    def step():
+        i = step_no[0] % 64
+        step_no[0] += 1
+        tokens = 0
+        for st, kn, vn, q in states:
+            st.append(kn[:, :, i:i + 1], vn[:, :, i:i + 1])
+            st.decode(q)
+            tokens += st.sparse_len + st.buffer_len
+        return tokens
+    return step
+
+
+def run_reference(args, wl, rank: int):
+    if rank != 0:
+        return None
+    n_units = 2
+    t0 = time.perf_counter()
+    step = oracle_sample(wl, n_units)
+    prep = time.perf_counter() - t0
+    for _ in range(args.warmup):
+        step()
+    times, toks = [], 0
+    for _ in range(args.steps):
+        t = time.perf_counter()
+        toks += step()
+        times.append(time.perf_counter() - t)
+    total = sum(times)
+    value = toks / total
+    sample = (f"{n_units} of {wl['B'] * wl['H_kv']} (batch, kv-head) units of the workload, "
+              f"{wl['H_q'] // wl['H_kv']} query heads each; one step = append 1 token + decode; "
+              f"state preparation {prep:.1f} s untimed")
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "KV-tokens/s",
+            "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": 1e3 * total / args.steps, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": args.workload, "desc": wl["desc"], "parallelism": "none (host CPU)"},
+            "cpu_baseline": {"value": value, "unit": "KV-tokens/s", "cores": 1, "kind": "oracle",
+                             "sample": sample},
+            "e2e": {"value": value, "unit": "KV-tokens/s", "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    return line
+
+
+def cpu_baseline_leg(wl, budget_s: float = 20.0):
+    step = oracle_sample(wl, 1)
+    step()
+    t0 = time.perf_counter()
+    toks, n = 0, 0
+    while time.perf_counter() - t0 < budget_s and n < 200:
+        toks += step()
+        n += 1
+    dt = time.perf_counter() - t0
+    return {"value": toks / dt, "unit": "KV-tokens/s", "cores": 1, "kind": "oracle",
+            "sample": f"1 of {wl['B'] * wl['H_kv']} (batch, kv-head) units of the same workload "
+                      f"({wl['H_q'] // wl['H_kv']} query heads), {n} steps of append 1 token + decode, "
+                      f"{dt:.1f} s, NumPy fp64 single thread"}
+
+
+# ---------------------------------------------------------------------------
+# The CUDA path
+# ---------------------------------------------------------------------------
+
+def run_swan(args, wl, rank: int, world: int, local_rank: int):
+    import torch
+
+    from paper_2511_18936_gb300 import swan, synth
+
+    dev = torch.device("cuda", local_rank)
+    torch.cuda.set_device(dev)
+    B, H_q, H_kv, L_s, n_b, k = wl["B"], wl["H_q"], wl["H_kv"], wl["L_s"], wl["n_b"], wl["k"]
+    G = H_q // H_kv
+    steps_total = args.warmup + args.steps + 2 * args.e2e_steps
+    max_seq = L_s + n_b + steps_total + 8
+    stream = torch.cuda.Stream(dev)
+    seed = args.seed + rank
+
+    with torch.cuda.stream(stream):
+        R = torch.from_numpy(synth.rotations(H_kv, D, seed=seed, workload=1, layer=0))[None].to(dev)
+        # prefill: the whole context in one append (L_s tokens pruned, n_b stay dense)
+        ctx = swan.Context(R, num_layers=1, batch=B, n_q_heads=H_q, n_kv_heads=H_kv,
+                           k_store=wl["k_store"], buffer_cap=n_b, max_seq=max_seq, stream=stream)
+        kk = synth.torch_lowrank_kv(B, H_kv, L_s + n_b, D, seed, synth.T_K, dev)
+        vv = synth.torch_lowrank_kv(B, H_kv, L_s + n_b, D, seed, synth.T_V, dev)
+        ctx.append(0, kk, vv)
+        del kk, vv
+        k_new = synth.torch_lowrank_kv(B, H_kv, steps_total, D, seed, synth.T_NEWK, dev)
+        v_new = synth.torch_lowrank_kv(B, H_kv, steps_total, D, seed, synth.T_NEWV, dev)
+        k_steps = [k_new[:, :, i:i + 1].contiguous() for i in range(steps_total)]
+        v_steps = [v_new[:, :, i:i + 1].contiguous() for i in range(steps_total)]
+        del k_new, v_new
+        qs = synth.torch_gaussian_fp16((steps_total, B, H_q, D), seed, synth.T_Q, dev)
+        out = torch.empty((B, H_q, D), dtype=torch.float16, device=dev)
+        ctx.set_k(k)
+    stream.synchronize()
+    ctx.check()
+
+    def step(i):
+        ctx.append(0, k_steps[i], v_steps[i], 1)
+        ctx.decode(0, qs[i], out)
+
+    for i in range(args.warmup):
+        step(i)
+    stream.synchronize()
+
+    def barrier():
+        if world > 1:
+            torch.distributed.barrier()
+
+    # ---- timed region: inputs resident in HBM -----------------------------
+    ctxlen = []
+    launches0 = ctx.launch_count()
+    ctx.timing_enable(True)
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    barrier()
+    torch.cuda.synchronize(dev)
+    with ClockSampler(local_rank) as clk:
+        ev0.record(stream)
+        for i in range(args.warmup, args.warmup + args.steps):
+            step(i)
+            info_len = L_s + n_b + (i + 1)  # context attended in step i
+            ctxlen.append(info_len)
+        ev1.record(stream)
+        stream.synchronize()
+    barrier()
+    torch.cuda.synchronize(dev)
+    ms = ev0.elapsed_time(ev1)
+    kt = ctx.timing_read()
+    ctx.timing_enable(False)
+    launches = ctx.launch_count() - launches0
+    info = ctx.query(0)
+    assert info.sparse_len + info.buffer_len == L_s + n_b + args.warmup + args.steps
+
+    # ---- end to end: pinned host inputs, H2D copies and the D2H read inside -
+    e2e_steps = args.e2e_steps
+    base = args.warmup + args.steps
+    hk = [k_steps[base + i].cpu().pin_memory() for i in range(2 * e2e_steps)]
+    hv = [v_steps[base + i].cpu().pin_memory() for i in range(2 * e2e_steps)]
+    hq = [qs[base + i].cpu().pin_memory() for i in range(2 * e2e_steps)]
+    hout = torch.empty((B, H_q, D), dtype=torch.float16).pin_memory()
+    dk = torch.empty_like(k_steps[0])
+    dv = torch.empty_like(v_steps[0])
+    dq = torch.empty_like(qs[0])
+
+    def e2e_step(i):
+        with torch.cuda.stream(stream):
+            dk.copy_(hk[i], non_blocking=True)
+            dv.copy_(hv[i], non_blocking=True)
+            dq.copy_(hq[i], non_blocking=True)
+            ctx.append(0, dk, dv, 1)
+            ctx.decode(0, dq, out)
+            hout.copy_(out, non_blocking=True)
+        stream.synchronize()
+
+    for i in range(e2e_steps):  # warm-up of the copy path
+        e2e_step(i)
+    barrier()
+    t0 = time.perf_counter()
+    e2e_tokens = 0
+    for i in range(e2e_steps, 2 * e2e_steps):
+        e2e_step(i)
+        e2e_tokens += B * H_kv * (L_s + n_b + base + i + 1)
+    e2e_s = time.perf_counter() - t0
+    barrier()
+    h2d = hk[0].numel() * 2 + hv[0].numel() * 2 + hq[0].numel() * 2
+    d2h = hout.numel() * 2
+
+    # ---- aggregate over ranks ----------------------------------------------
+    kv_tokens = sum(B * H_kv * c for c in ctxlen)
+    t_max = ms
+    e2e_max = e2e_s
+    if world > 1:
+        tt = torch.tensor([ms, e2e_s], device=dev, dtype=torch.float64)
+        torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
+        t_max, e2e_max = float(tt[0]), float(tt[1])
+    value = world * kv_tokens / (t_max / 1e3)
+    e2e_value = world * e2e_tokens / e2e_max
+
+    dec_ms, dec_n = kt["decode"]
+    avg_dec_s = dec_ms / 1e3 / max(dec_n, 1)
+    ctx_mean = statistics.mean(ctxlen)
+    sparse_mean = ctx_mean - n_b
+    # algorithmic bytes of one decode-kernel launch: per (sparse token, kv head)
+    # 2 * 3 * k bytes (fp16 value + uint8 index for K and V); per (buffer
+    # token, kv head) 2 * 2 * d bytes
+    alg_decode = B * H_kv * (sparse_mean * 6 * k + n_b * 4 * D)
+    achieved = alg_decode / avg_dec_s / 1e9
+    peaks = measured_peaks()
+    peak = float(peaks["hbm_gbs"]) if peaks else 6800.0
+    step_s = t_max / 1e3 / args.steps
+    # whole-step algorithmic bytes: decode reads + q/out + R (q and out fp16,
+    # R fp32 once per kv head) + the append's new vectors and evicted one
+    alg_step = (alg_decode + 2 * B * H_q * D * 2 + H_kv * D * D * 4
+                + B * H_kv * (2 * D * 2 * 2 + 6 * wl["k_store"]))
+    line = {
+        "metric": METRIC, "value": value, "unit": "KV-tokens/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": t_max / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+        "data": "synthetic (seeded low-rank K/V, Gaussian q, random orthogonal R)",
+        "config": {"workload": args.workload, "desc": wl["desc"], "batch": B, "n_q_heads": H_q,
+                   "n_kv_heads": H_kv, "sparse_tokens": L_s, "buffer_tokens": n_b, "k": k,
+                   "storage": "fp16 values + uint8 indices (sparse), fp16 (buffer)",
+                   "l2": f"inputs larger than L2: {alg_decode / 1e9:.2f} GB read per decode, no flush",
+                   "parallelism": f"replicas x{world}" if world > 1 else "single GPU"},
+        "hbm_gbs_step": alg_step / step_s / 1e9,
+        "pct_of_8tbs_step": 100.0 * alg_step / step_s / 1e9 / NOMINAL_HBM_GBS,
+        "roofline": {"kernel": "decode", "bound": "hbm", "achieved": achieved, "peak": peak,
+                     "unit": "GB/s", "frac": achieved / peak,
+                     "peak_source": "MEASURED_PEAKS.json hbm_gbs (measured)" if peaks
+                     else "fallback 6.8 TB/s",
+                     "pct_of_8tbs": 100.0 * achieved / NOMINAL_HBM_GBS,
+                     "alg_bytes_per_launch": alg_decode, "avg_launch_ms": avg_dec_s * 1e3,
+                     "traffic": decode_kernel_traffic(args.workload)},
+        "kernels_ms_per_step": {name: v[0] / max(v[1], 1) for name, v in kt.items() if v[1]},
+        "gpu_launches": launches,
+        "e2e": {"value": e2e_value, "unit": "KV-tokens/s", "h2d_bytes_per_step": h2d,
+                "d2h_bytes_per_step": d2h, "steps": e2e_steps},
+        "clocks": clk.summary(),
+    }
+    ctx.check()
+    ctx.close()
+    return line
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="swan", choices=["swan", "reference"])
+    ap.add_argument("--workload", default="llama2-7b-layer-32k", choices=sorted(WORKLOADS))
+    ap.add_argument("--e2e-steps", type=int, default=20)
+    ap.add_argument("--seed", type=int, default=0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+    wl = WORKLOADS[args.workload]
+
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+
+    if args.impl == "reference":
+        line = run_reference(args, wl, rank)
+        if line is not None:
+            print(json.dumps(line), flush=True)
+        return
+
+    if world > 1:
+        import torch
+        torch.distributed.init_process_group("nccl")
+    line = run_swan(args, wl, rank, world, local_rank)
+    if rank == 0:
+        if not args.no_cpu_baseline and world == 1:
+            line["cpu_baseline"] = cpu_baseline_leg(wl)
+        elif not args.no_cpu_baseline:
+            line["cpu_baseline"] = cpu_baseline_leg(wl)
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        import torch
+        torch.distributed.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

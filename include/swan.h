@@ -1,0 +1,215 @@
+/*
+ * swan.h -- C ABI of libswan, the SWAN decode hot path on one GB300 (sm_103a).
+ *
+ * SWAN ("Sparse Winnowed Attention", arXiv 2511.18936) keeps each attention
+ * head's key/value history as rotated, pruned sparse vectors plus a small
+ * dense buffer of recent vectors, and attends to that cache directly, with no
+ * reconstruction.  This library owns the cache in GPU memory and provides:
+ *
+ *   swan_init          allocate a cache for L layers (Section 4.3's hybrid
+ *                      cache; Section 5.1's sparse format)
+ *   swan_append        rotate new keys/values by R and insert them
+ *                      (Algorithm 1: projection, buffer insert, eviction of
+ *                      the oldest vectors with magnitude top-k pruning)
+ *   swan_flush_buffer  prune every buffered vector into the sparse history
+ *   swan_decode        one decode step of attention over the hybrid cache
+ *                      (Algorithm 1: rotated query, sparse-dense and
+ *                      dense-dense score products, softmax, value product),
+ *                      followed by the rotate-back o = o_hat R_vo^T
+ *                      (Appendix A.1, Lemma 2)
+ *   swan_set_k         runtime keep count (Section 1 contributions, Section
+ *                      4.3: the pruning threshold is tunable at inference)
+ *
+ * Conventions (all entry points):
+ *   - Row vectors, as in Section 4.2: x_hat[j] = sum_i x[i] * R[i][j].
+ *   - head_dim d must be 128 (uint8 indices, Section 5.1).
+ *   - Every pointer named "device" is a CUDA device pointer on the device
+ *     that was current at swan_init; the caller keeps ownership of it.
+ *   - Work is enqueued asynchronously on cfg.stream; nothing synchronises
+ *     except swan_debug_export, swan_check and swan_timing_read.
+ *   - Argument and capacity checks happen on the host before any launch; a
+ *     failed check returns an error and leaves the cache unchanged.
+ *   - A CUDA error during a launch returns SWAN_ERR_CUDA; the context is then
+ *     poisoned and every later call returns SWAN_ERR_STATE.
+ *   - No call allocates device memory after swan_init.
+ *   - One context per stream; a context is not thread-safe.
+ *   - All sequences of a batch have the same length.
+ *   - Nothing throws across the ABI and nothing calls abort().
+ */
+#ifndef SWAN_H
+#define SWAN_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum swan_status {
+  SWAN_OK = 0,
+  SWAN_ERR_INVALID_ARG = 1,    /* bad pointer, size, layer, k, ... */
+  SWAN_ERR_UNSUPPORTED = 2,    /* valid but not built (e.g. head_dim != 128) */
+  SWAN_ERR_CAPACITY = 3,       /* would exceed max_seq; nothing was changed */
+  SWAN_ERR_CUDA = 4,           /* a CUDA runtime call failed */
+  SWAN_ERR_STATE = 5,          /* context poisoned by an earlier CUDA error */
+  SWAN_ERR_DEVICE_TIMEOUT = 6, /* reserved: a bounded device wait ran out */
+  SWAN_ERR_NOMEM = 7,          /* device or host allocation failed in init */
+  SWAN_ERR_DEVICE_CHECK = 8    /* a device-side consistency check failed */
+} swan_status;
+
+typedef struct swan_ctx swan_ctx; /* opaque; owned by the library */
+
+typedef struct swan_config {
+  int num_layers;  /* >= 1 */
+  int batch;       /* B >= 1 */
+  int n_q_heads;   /* H_q, a multiple of n_kv_heads */
+  int n_kv_heads;  /* H_kv; G = H_q / H_kv query heads share a kv head
+                      (Section 4.1.1); G must be 1, 2 or 4 */
+  int head_dim;    /* d, must be 128 */
+  int k_store;     /* kept entries stored per vector, 1..d; the runtime keep
+                      count k_active may be any value 1..k_store */
+  int buffer_cap;  /* b, dense buffer capacity in tokens, 0..4096 */
+  int max_seq;     /* tokens per sequence the cache can hold (sparse + buffer) */
+  int page_tokens; /* tokens per cache page, multiple of 32; 0 = 128 */
+  void* stream;    /* cudaStream_t the context enqueues on; NULL = default */
+} swan_config;
+
+/*
+ * Create a context.  R_qk, R_vo: device fp32 [num_layers][n_kv_heads][d][d],
+ * row-major, orthogonal (P_QK and P_VO of Section 4.1.2).  R_vo == NULL uses
+ * R_qk for the values too.  Both are copied; the caller may free them after
+ * the call returns.  All cache memory is allocated here, once.
+ * On success *out receives the context and k_active = k_store.
+ * Errors: INVALID_ARG, UNSUPPORTED, NOMEM, CUDA.  *out is NULL on error.
+ */
+swan_status swan_init(swan_ctx** out, const swan_config* cfg,
+                      const float* R_qk, const float* R_vo);
+
+/* Release every resource of the context (synchronises its stream).
+ * NULL is accepted and ignored. */
+swan_status swan_destroy(swan_ctx* ctx);
+
+/*
+ * Set the runtime keep count (Section 4.3; Section 1 lists runtime
+ * tunability as a contribution).  Entries are stored in decreasing magnitude
+ * order, so decoding with k_active < k_store uses exactly the top-k_active
+ * entries of every cached vector: the same result as a cache built with
+ * k_store = k_active.  Applies to decodes enqueued after the call.
+ * Errors: INVALID_ARG unless 1 <= k_active <= k_store.
+ */
+swan_status swan_set_k(swan_ctx* ctx, int k_active);
+
+/*
+ * Append T tokens to every sequence of one layer (Algorithm 1, generalised
+ * to T tokens at once).
+ *   k_new, v_new: device fp16 [batch][n_kv_heads][T][d], post-RoPE keys and
+ *   unrotated values.  The library rotates them: k_hat = k R_qk,
+ *   v_hat = v R_vo (fp32 arithmetic, rounded to fp16 round-to-nearest-even).
+ * If buffer_count + T > buffer_cap, the oldest (buffer_count + T - buffer_cap)
+ * vectors of (buffer, then new tokens) are pruned to their k_store
+ * largest-magnitude coordinates (ties to the lower index; keys and values
+ * separately) and appended to the sparse history, in order; the rest stay
+ * dense in the buffer.  T == 0 is a no-op.
+ * Errors: INVALID_ARG (layer, T < 0, NULL), CAPACITY (sparse + buffer would
+ * exceed max_seq), STATE, CUDA.
+ */
+swan_status swan_append(swan_ctx* ctx, int layer, const void* k_new,
+                        const void* v_new, int T);
+
+/*
+ * Prune every buffered vector of a layer into the sparse history (oldest
+ * first); the buffer becomes empty.  layer == -1 flushes all layers.
+ * Errors: INVALID_ARG, STATE, CUDA.
+ */
+swan_status swan_flush_buffer(swan_ctx* ctx, int layer);
+
+/*
+ * One decode step of attention for one layer (Algorithm 1, attention part):
+ *   q:   device fp16 [batch][n_q_heads][d], post-RoPE, unrotated.
+ *   out: device fp16 [batch][n_q_heads][d], written as
+ *        out = softmax((q R_qk) K_cache^T / sqrt(d)) V_cache R_vo^T
+ *        where K_cache / V_cache are the rotated sparse history (first
+ *        k_active stored entries of each vector) followed by the dense
+ *        buffer.  Query head h attends to kv head h / G.
+ * Attends over every token appended so far.  With an empty cache out is 0.
+ * q and out must not overlap.  Errors: INVALID_ARG, STATE, CUDA.
+ */
+swan_status swan_decode(swan_ctx* ctx, int layer, const void* q, void* out);
+
+/* Host-side view of a layer's cache (no synchronisation). */
+typedef struct swan_layer_info {
+  int64_t sparse_len;   /* tokens per sequence in the sparse history */
+  int64_t buffer_len;   /* tokens per sequence in the dense buffer */
+  int k_active;
+  int k_store;
+  int k_slots;          /* k_store rounded up to a multiple of 8 */
+  int page_tokens;
+  int64_t page_bytes;   /* bytes of one page (keys and values) */
+  int64_t device_bytes; /* device memory owned by the whole context */
+} swan_layer_info;
+
+swan_status swan_query(const swan_ctx* ctx, int layer, swan_layer_info* info);
+
+/*
+ * Copy part of a layer's cache to host memory, in a canonical layout
+ * (synchronises the stream).  For tests and debugging.
+ *   SWAN_EXPORT_BUFFER_K / _V: fp16 [batch][n_kv_heads][buffer_len][d],
+ *     oldest first.
+ *   SWAN_EXPORT_SPARSE_K / _V: uint8 indices [batch][n_kv_heads]
+ *     [sparse_len][k_store], then fp16 values of the same shape, each vector's
+ *     entries in stored (decreasing magnitude) order.
+ * bytes must equal the exact size of the requested view.
+ * Errors: INVALID_ARG (what, layer, size), STATE, CUDA.
+ */
+enum {
+  SWAN_EXPORT_BUFFER_K = 1,
+  SWAN_EXPORT_BUFFER_V = 2,
+  SWAN_EXPORT_SPARSE_K = 3,
+  SWAN_EXPORT_SPARSE_V = 4
+};
+swan_status swan_debug_export(swan_ctx* ctx, int layer, int what,
+                              void* host_dst, size_t bytes);
+
+/*
+ * Synchronise the stream and read the device status word that kernels set
+ * when a device-side consistency check fails (for instance a page-table
+ * entry out of range); such a kernel skips the access instead of faulting.
+ * Returns OK, DEVICE_CHECK (and clears the word), STATE or CUDA.
+ */
+swan_status swan_check(swan_ctx* ctx);
+
+/*
+ * Per-kernel timing with CUDA events on the context's stream.  While enabled,
+ * every launch is bracketed by an event pair; swan_timing_read synchronises,
+ * sums the elapsed times per kernel kind and resets the sums.
+ */
+enum {
+  SWAN_KERNEL_ROTATE_Q = 0, /* q' = q R_qk */
+  SWAN_KERNEL_DECODE = 1,   /* split decode over the packed cache */
+  SWAN_KERNEL_COMBINE = 2,  /* split combine + rotate-back */
+  SWAN_KERNEL_APPEND = 3,   /* rotate new tokens; buffer insert or prune */
+  SWAN_KERNEL_PRUNE = 4,    /* prune buffered vectors (eviction, flush) */
+  SWAN_KERNEL_KINDS = 8
+};
+typedef struct swan_timing {
+  double ms[SWAN_KERNEL_KINDS];
+  int64_t launches[SWAN_KERNEL_KINDS];
+} swan_timing;
+swan_status swan_timing_enable(swan_ctx* ctx, int enable);
+swan_status swan_timing_read(swan_ctx* ctx, swan_timing* out);
+
+/* Number of kernels this context has launched since swan_init. */
+int64_t swan_launch_count(const swan_ctx* ctx);
+
+/* Static string for a status code. */
+const char* swan_status_string(swan_status s);
+
+/* Detail of the last error returned on this thread ("" if none). */
+const char* swan_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* SWAN_H */

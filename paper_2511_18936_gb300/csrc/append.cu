@@ -1,0 +1,248 @@
+// Compress-on-append: rotation of new keys/values, dense ring-buffer insert,
+// and magnitude top-k pruning into the paged sparse cache (Algorithm 1;
+// Section 4.3; Section 5.1).
+#include "swan_internal.h"
+
+namespace swan {
+namespace {
+
+// Sort 128 unique 32-bit keys held by one warp (lane l holds elements
+// 4l..4l+3) into decreasing order with a bitonic network: the element of
+// rank r ends up in lane r/4, slot r%4.
+__device__ __forceinline__ void sort128_desc(uint32_t (&v)[4], int lane) {
+#pragma unroll
+  for (int k = 2; k <= 128; k <<= 1) {
+#pragma unroll
+    for (int j = k >> 1; j > 0; j >>= 1) {
+      uint32_t nv[4];
+#pragma unroll
+      for (int s = 0; s < 4; ++s) {
+        const int i = 4 * lane + s;
+        const uint32_t other = (j >= 4) ? __shfl_xor_sync(0xffffffffu, v[s], j >> 2) : v[s ^ j];
+        const bool desc = (i & k) == 0;   // direction of this bitonic run
+        const bool lower = (i & j) == 0;  // lower element of the pair
+        const uint32_t hi = max(v[s], other), lo = min(v[s], other);
+        nv[s] = (lower == desc) ? hi : lo;
+      }
+#pragma unroll
+      for (int s = 0; s < 4; ++s) v[s] = nv[s];
+    }
+  }
+}
+
+// Prune one rotated fp16 vector (lane l holds coordinates 4l..4l+3 as raw
+// bits) to its k_store largest-magnitude coordinates, ties to the lower
+// index, and store them in decreasing order at sparse position `sp` of
+// `unit`.  The sort key is (|x| as fp16 bits, 127 - j, sign): unique, and its
+// order is magnitude first, then lower index first.
+__device__ __forceinline__ void warp_prune_store(uint2 raw, int lane, int kind, int64_t unit,
+                                                 int64_t sp, const CacheGeom& g,
+                                                 unsigned* status) {
+  uint32_t key[4];
+  const uint32_t h16[4] = {raw.x & 0xffffu, raw.x >> 16, raw.y & 0xffffu, raw.y >> 16};
+#pragma unroll
+  for (int s = 0; s < 4; ++s) {
+    const uint32_t j = 4u * lane + s;
+    key[s] = ((h16[s] & 0x7fffu) << 16) | ((127u - j) << 1) | (h16[s] >> 15);
+  }
+  sort128_desc(key, lane);
+
+  const int64_t page = sp / g.P;
+  const int slot = (int)(sp % g.P);
+  if (page >= g.pages_per_unit) {
+    if (lane == 0) atomicOr(status, kStatusPageRange);
+    return;
+  }
+  const int32_t phys = g.page_table[unit * g.pages_per_unit + page];
+  if (phys < 0 || phys >= g.num_pages) {
+    if (lane == 0) atomicOr(status, kStatusPageRange);
+    return;
+  }
+  uint8_t* pg = g.pool + (int64_t)phys * g.page_bytes;
+  const int64_t voff = kind ? g.vval_off() : 0;
+  const int64_t ioff = kind ? g.vidx_off() : g.kidx_off();
+  if (lane < (g.k_slots >> 2)) {
+    const int c = lane >> 1, half = lane & 1;
+    uint32_t vb[4], ib[4];
+#pragma unroll
+    for (int s = 0; s < 4; ++s) {
+      const bool keep = (4 * lane + s) < g.k_store;
+      const uint32_t j = 127u - ((key[s] >> 1) & 127u);
+      const uint32_t bits = ((key[s] & 1u) << 15) | (key[s] >> 16);
+      vb[s] = keep ? bits : 0u;
+      ib[s] = keep ? j : 0u;
+    }
+    const uint2 vals = make_uint2(vb[0] | (vb[1] << 16), vb[2] | (vb[3] << 16));
+    const uint32_t idx = ib[0] | (ib[1] << 8) | (ib[2] << 16) | (ib[3] << 24);
+    const int64_t rec = (int64_t)c * g.P + slot;
+    *reinterpret_cast<uint2*>(pg + voff + rec * 16 + half * 8) = vals;
+    *reinterpret_cast<uint32_t*>(pg + ioff + rec * 8 + half * 4) = idx;
+  }
+}
+
+__device__ __forceinline__ float half_at(const uint4 (&xr)[16], int i) {
+  const uint4 w = xr[i >> 3];
+  const int q = (i >> 1) & 3;
+  const uint32_t word = q == 0 ? w.x : q == 1 ? w.y : q == 2 ? w.z : w.w;
+  const unsigned short bits = (i & 1) ? (unsigned short)(word >> 16) : (unsigned short)(word & 0xffffu);
+  return __half2float(__ushort_as_half(bits));
+}
+
+constexpr int kStageWords = 65;  // 64 words of fp16 pairs + 1 pad (bank skew)
+constexpr size_t kAppendSmem = 128 * 128 * sizeof(float) + kThreads * kStageWords * 4;
+
+// One CTA: one kv head (blockIdx.y), keys or values (blockIdx.z), 256 of the
+// B*T new vectors (one per thread).  R is staged in shared memory; each lane
+// computes its vector's 128 rotated coordinates in fp32 (32 at a time) and
+// rounds them to fp16.  Vectors that stay dense go to their ring slot;
+// vectors past the eviction point are pruned by their warp.
+__global__ void __launch_bounds__(kThreads, 1) append_kernel(AppendParams p) {
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  float* Rs = reinterpret_cast<float*>(smem_raw);
+  uint32_t* stage = reinterpret_cast<uint32_t*>(smem_raw + 128 * 128 * sizeof(float));
+
+  const int kind = blockIdx.z;
+  const int h = blockIdx.y;
+  const float* R = (kind ? p.R_vo : p.R_qk) + (size_t)h * kHeadDim * kHeadDim;
+  const __half* X = kind ? p.v_new : p.k_new;
+  __half* ring = kind ? p.ring_v : p.ring_k;
+
+  for (int i = threadIdx.x; i < kHeadDim * kHeadDim / 4; i += kThreads)
+    reinterpret_cast<float4*>(Rs)[i] = __ldg(reinterpret_cast<const float4*>(R) + i);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int64_t nvec = (int64_t)p.B * p.T;
+  const int64_t n = (int64_t)blockIdx.x * kThreads + threadIdx.x;
+  const bool valid = n < nvec;
+  int64_t b = 0, j = 0;
+  uint4 xr[16];
+  if (valid) {
+    b = n / p.T;
+    j = n % p.T;
+    const uint4* src = reinterpret_cast<const uint4*>(X + (((size_t)b * p.H + h) * p.T + j) * kHeadDim);
+#pragma unroll
+    for (int i = 0; i < 16; ++i) xr[i] = __ldg(src + i);
+  } else {
+#pragma unroll
+    for (int i = 0; i < 16; ++i) xr[i] = make_uint4(0, 0, 0, 0);
+  }
+  __syncthreads();
+
+  const int64_t pos = (int64_t)p.n_b + j;  // logical position in (buffer, new tokens)
+  const bool to_ring = valid && pos >= p.evict;
+  __half* ring_row = nullptr;
+  if (to_ring) {
+    const int slot = (int)((p.buf_start + pos) % p.cap);
+    ring_row = ring + (((size_t)b * p.H + h) * p.cap + slot) * kHeadDim;
+  }
+  uint32_t* my_stage = stage + threadIdx.x * kStageWords;
+
+#pragma unroll 1
+  for (int cb = 0; cb < 4; ++cb) {
+    float acc[32];
+#pragma unroll
+    for (int m = 0; m < 32; ++m) acc[m] = 0.f;
+#pragma unroll
+    for (int i = 0; i < kHeadDim; ++i) {
+      const float xi = half_at(xr, i);
+      const float4* Rrow = reinterpret_cast<const float4*>(Rs + i * kHeadDim + cb * 32);
+#pragma unroll
+      for (int q = 0; q < 8; ++q) {
+        const float4 r = Rrow[q];
+        acc[4 * q + 0] = fmaf(xi, r.x, acc[4 * q + 0]);
+        acc[4 * q + 1] = fmaf(xi, r.y, acc[4 * q + 1]);
+        acc[4 * q + 2] = fmaf(xi, r.z, acc[4 * q + 2]);
+        acc[4 * q + 3] = fmaf(xi, r.w, acc[4 * q + 3]);
+      }
+    }
+    uint32_t packed[16];
+#pragma unroll
+    for (int m = 0; m < 16; ++m) {
+      const unsigned short lo = __half_as_ushort(__float2half_rn(acc[2 * m]));
+      const unsigned short hi = __half_as_ushort(__float2half_rn(acc[2 * m + 1]));
+      packed[m] = (uint32_t)lo | ((uint32_t)hi << 16);
+      my_stage[cb * 16 + m] = packed[m];
+    }
+    if (to_ring) {
+      uint4* dst = reinterpret_cast<uint4*>(ring_row + cb * 32);
+#pragma unroll
+      for (int q = 0; q < 4; ++q)
+        dst[q] = make_uint4(packed[4 * q], packed[4 * q + 1], packed[4 * q + 2], packed[4 * q + 3]);
+    }
+  }
+  __syncwarp();
+
+  // Prune this warp's vectors that land past the eviction point.
+  const int64_t warp_first = (int64_t)blockIdx.x * kThreads + warp * 32;
+#pragma unroll 1
+  for (int v = 0; v < 32; ++v) {
+    const int64_t nv = warp_first + v;
+    if (nv >= nvec) break;
+    const int64_t bv = nv / p.T, jv = nv % p.T;
+    const int64_t posv = (int64_t)p.n_b + jv;
+    if (posv >= p.evict) continue;
+    const uint32_t* row = stage + (warp * 32 + v) * kStageWords;
+    const uint2 raw = make_uint2(row[2 * lane], row[2 * lane + 1]);
+    warp_prune_store(raw, lane, kind, bv * p.H + h, p.sparse_len + posv, p.geom, p.status);
+  }
+}
+
+// One warp per (unit, buffered token, K or V): read the ring row and prune.
+__global__ void __launch_bounds__(kThreads) prune_ring_kernel(PruneRingParams p) {
+  const int lane = threadIdx.x & 31;
+  const int64_t gw = ((int64_t)blockIdx.x * kThreads + threadIdx.x) >> 5;
+  const int64_t total = (int64_t)p.units * p.count * 2;
+  if (gw >= total) return;
+  const int kind = (int)(gw & 1);
+  const int64_t rest = gw >> 1;
+  const int64_t unit = rest / p.count;
+  const int i = (int)(rest % p.count);
+  const int slot = (p.buf_start + i) % p.cap;
+  const __half* row = (kind ? p.ring_v : p.ring_k) + ((size_t)unit * p.cap + slot) * kHeadDim;
+  const uint2 raw = __ldg(reinterpret_cast<const uint2*>(row) + lane);
+  warp_prune_store(raw, lane, kind, unit, p.sparse_len + i, p.geom, p.status);
+}
+
+__global__ void transpose_r_kernel(const float* src, float* dst, int64_t mats) {
+  __shared__ float tile[32][33];
+  const int64_t m = blockIdx.z;
+  const int bx = blockIdx.x * 32, by = blockIdx.y * 32;
+  const float* s = src + m * kHeadDim * kHeadDim;
+  float* d = dst + m * kHeadDim * kHeadDim;
+  for (int r = threadIdx.y; r < 32; r += blockDim.y)
+    tile[r][threadIdx.x] = s[(by + r) * kHeadDim + bx + threadIdx.x];
+  __syncthreads();
+  for (int r = threadIdx.y; r < 32; r += blockDim.y)
+    d[(bx + r) * kHeadDim + by + threadIdx.x] = tile[threadIdx.x][r];
+}
+
+}  // namespace
+
+cudaError_t launch_append(const AppendParams& p, cudaStream_t s) {
+  static bool attr_set = false;
+  if (!attr_set) {
+    cudaError_t e = cudaFuncSetAttribute(append_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)kAppendSmem);
+    if (e != cudaSuccess) return e;
+    attr_set = true;
+  }
+  const int64_t nvec = (int64_t)p.B * p.T;
+  dim3 grid((unsigned)((nvec + kThreads - 1) / kThreads), (unsigned)p.H, 2);
+  append_kernel<<<grid, kThreads, kAppendSmem, s>>>(p);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_prune_ring(const PruneRingParams& p, cudaStream_t s) {
+  const int64_t warps = (int64_t)p.units * p.count * 2;
+  const int64_t blocks = (warps + kWarpsPerCta - 1) / kWarpsPerCta;
+  prune_ring_kernel<<<(unsigned)blocks, kThreads, 0, s>>>(p);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_transpose_r(const float* src, float* dst, int64_t mats, cudaStream_t s) {
+  dim3 grid(kHeadDim / 32, kHeadDim / 32, (unsigned)mats);
+  transpose_r_kernel<<<grid, dim3(32, 8), 0, s>>>(src, dst, mats);
+  return cudaGetLastError();
+}
+
+}  // namespace swan

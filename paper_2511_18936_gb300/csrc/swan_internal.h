@@ -1,0 +1,130 @@
+// Internal definitions shared by the host library and the kernels.
+//
+// Sparse cache page layout (Section 5.1's values + 8-bit indices, arranged
+// for 128-bit coalesced loads on sm_103a).  A page holds P tokens (P a
+// multiple of 32) of one (layer, batch, kv-head) unit.  Each vector's kept
+// entries are grouped in chunks of 8, in stored (decreasing magnitude) order;
+// chunk c of token t is a 16-byte record of 8 fp16 values and an 8-byte
+// record of 8 uint8 indices:
+//
+//   [K values  : k_slots/8 chunks][P tokens][8 x fp16]   (16 B per record)
+//   [K indices : k_slots/8 chunks][P tokens][8 x uint8]  ( 8 B per record)
+//   [V values  : same as K values]
+//   [V indices : same as K indices]
+//
+// A warp that handles 32 consecutive tokens (one per lane) reads chunk c of
+// all of them as one contiguous 512-byte run (values) and one 256-byte run
+// (indices).  A runtime keep count k_active <= k_store reads only the first
+// ceil(k_active / 8) chunks: a contiguous prefix of each region.
+#pragma once
+
+#include <cuda_fp16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace swan {
+
+constexpr int kHeadDim = 128;
+constexpr int kWarpsPerCta = 8;
+constexpr int kThreads = kWarpsPerCta * 32;
+// log2-domain slack before the running max of the online softmax is moved:
+// scores may exceed the running max by up to 2^kLazyRescale before the
+// accumulators are rescaled (exact; only the reference point changes).
+constexpr float kLazyRescale = 8.0f;
+
+// Device status word bits (set instead of faulting on inconsistent state).
+constexpr unsigned kStatusPageRange = 1u;
+constexpr unsigned kStatusRingRange = 2u;
+
+struct CacheGeom {
+  uint8_t* pool;             // all pages of all layers
+  const int32_t* page_table; // this layer: [units][pages_per_unit] -> page id
+  int pages_per_unit;
+  int64_t num_pages;         // pages in the pool (bounds check)
+  int P;                     // tokens per page
+  int k_slots;               // k_store rounded up to 8
+  int k_store;
+  int64_t page_bytes;        // P * k_slots * 6
+  __device__ __host__ int64_t kidx_off() const { return (int64_t)P * k_slots * 2; }
+  __device__ __host__ int64_t vval_off() const { return (int64_t)P * k_slots * 3; }
+  __device__ __host__ int64_t vidx_off() const { return (int64_t)P * k_slots * 5; }
+};
+
+// Rotate T new tokens per unit, then either write them to the ring buffer or
+// prune them straight into the sparse cache (Algorithm 1, generalised to T).
+struct AppendParams {
+  const __half* k_new;  // [B][H][T][d]
+  const __half* v_new;
+  const float* R_qk;    // this layer: [H][d][d]
+  const float* R_vo;
+  __half* ring_k;       // this layer: [B*H][cap][d]
+  __half* ring_v;
+  int B, H, T, cap;
+  int buf_start;        // ring slot of the oldest buffered token
+  int n_b;              // buffered tokens before the append
+  int64_t evict;        // logical positions < evict go to the sparse cache
+  int64_t sparse_len;   // sparse tokens before the append
+  CacheGeom geom;
+  unsigned* status;
+};
+
+// Prune `count` buffered tokens (logical positions 0..count-1) per unit from
+// the ring buffer into the sparse cache (eviction and flush).
+struct PruneRingParams {
+  const __half* ring_k;
+  const __half* ring_v;
+  int units, cap, buf_start, count;
+  int64_t sparse_len;
+  CacheGeom geom;
+  unsigned* status;
+};
+
+struct RotateQParams {
+  const __half* q;   // [B][H_q][d]
+  const float* R_qk; // this layer: [H_kv][d][d]
+  float* qprime;     // [B][H_q][d]
+  int H_q, G;
+};
+
+// Split decode: the flat list of 32-token groups of all units is cut into
+// equal contiguous ranges, one per CTA.  Group g of unit u is a sparse group
+// for g < n_sg (tokens 32g..32g+31 of the sparse history) and a buffer group
+// after that.  A CTA writes one partial (m, l, acc[d]) per (unit, head) it
+// touches, at pair index (cta + unit).
+struct DecodeParams {
+  const float* qprime;     // [B][H_q][d]
+  CacheGeom geom;
+  const __half* ring_k;    // this layer: [units][cap][d]
+  const __half* ring_v;
+  int cap, buf_start, n_b;
+  int64_t sparse_len;
+  int64_t n_sg, N_g;       // sparse groups per unit; groups per unit
+  int64_t total_groups, range;
+  int H_kv, H_q;
+  int k_full_chunks;       // k_active / 8
+  int k_rem;               // k_active % 8
+  float scale_log2;        // log2(e) / sqrt(d)
+  float* partials;         // [pairs][G][d + 2]
+  unsigned* status;
+};
+
+struct CombineParams {
+  const float* partials;
+  const float* R_voT;      // this layer: [H_kv][d][d], transposed
+  __half* out;             // [B][H_q][d]
+  int H_kv, H_q, G;
+  int64_t N_g, range, total_groups;
+};
+
+// Launchers (return the launch error, if any).
+cudaError_t launch_append(const AppendParams& p, cudaStream_t s);
+cudaError_t launch_prune_ring(const PruneRingParams& p, cudaStream_t s);
+cudaError_t launch_rotate_q(const RotateQParams& p, int B, cudaStream_t s);
+cudaError_t launch_decode(const DecodeParams& p, int G, int k_slots, int grid, cudaStream_t s);
+cudaError_t launch_combine(const CombineParams& p, int B, cudaStream_t s);
+cudaError_t launch_transpose_r(const float* src, float* dst, int64_t mats, cudaStream_t s);
+// Decode CTAs that fit on one SM together (for the grid size).
+int decode_ctas_per_sm(int G, int k_slots);
+size_t decode_smem_bytes(int G);
+
+}  // namespace swan

@@ -1,0 +1,216 @@
+"""Thin Python binding of libswan (ctypes).  Argument marshalling only: every
+step of the decode path runs in the library's CUDA kernels.  PyTorch supplies
+device memory and the stream.
+
+The library must have been built (``paper_2511_18936_gb300.build.build()``);
+loading fails loudly otherwise - there is no fallback implementation.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import numpy as np
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_PKG, "libswan.so")
+
+OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_CAPACITY, ERR_CUDA, ERR_STATE, \
+    ERR_DEVICE_TIMEOUT, ERR_NOMEM, ERR_DEVICE_CHECK = range(9)
+EXPORT_BUFFER_K, EXPORT_BUFFER_V, EXPORT_SPARSE_K, EXPORT_SPARSE_V = 1, 2, 3, 4
+KERNEL_ROTATE_Q, KERNEL_DECODE, KERNEL_COMBINE, KERNEL_APPEND, KERNEL_PRUNE = range(5)
+KERNEL_KINDS = 8
+KERNEL_NAMES = {KERNEL_ROTATE_Q: "rotate_q", KERNEL_DECODE: "decode", KERNEL_COMBINE: "combine",
+                KERNEL_APPEND: "append", KERNEL_PRUNE: "prune_ring"}
+
+# Every symbol include/swan.h declares.
+EXPORTED = ["swan_init", "swan_destroy", "swan_set_k", "swan_append", "swan_flush_buffer",
+            "swan_decode", "swan_query", "swan_debug_export", "swan_check",
+            "swan_timing_enable", "swan_timing_read", "swan_launch_count",
+            "swan_status_string", "swan_last_error"]
+
+
+class SwanConfig(ctypes.Structure):
+    _fields_ = [("num_layers", ctypes.c_int), ("batch", ctypes.c_int),
+                ("n_q_heads", ctypes.c_int), ("n_kv_heads", ctypes.c_int),
+                ("head_dim", ctypes.c_int), ("k_store", ctypes.c_int),
+                ("buffer_cap", ctypes.c_int), ("max_seq", ctypes.c_int),
+                ("page_tokens", ctypes.c_int), ("stream", ctypes.c_void_p)]
+
+
+class LayerInfo(ctypes.Structure):
+    _fields_ = [("sparse_len", ctypes.c_int64), ("buffer_len", ctypes.c_int64),
+                ("k_active", ctypes.c_int), ("k_store", ctypes.c_int), ("k_slots", ctypes.c_int),
+                ("page_tokens", ctypes.c_int), ("page_bytes", ctypes.c_int64),
+                ("device_bytes", ctypes.c_int64)]
+
+
+class Timing(ctypes.Structure):
+    _fields_ = [("ms", ctypes.c_double * KERNEL_KINDS), ("launches", ctypes.c_int64 * KERNEL_KINDS)]
+
+
+class SwanError(RuntimeError):
+    def __init__(self, status: int, where: str, detail: str):
+        super().__init__(f"{where}: status {status} ({detail})")
+        self.status = status
+
+
+_lib = None
+
+
+def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
+    """Load libswan.so (once).  Raises if it has not been built."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(path):
+        raise RuntimeError(f"{path} is missing: build it with "
+                           "`python -m paper_2511_18936_gb300.build` (no fallback exists)")
+    lib = ctypes.CDLL(path)
+    vp, i, i64 = ctypes.c_void_p, ctypes.c_int, ctypes.c_int64
+    sig = {
+        "swan_init": (i, [ctypes.POINTER(vp), ctypes.POINTER(SwanConfig), vp, vp]),
+        "swan_destroy": (i, [vp]),
+        "swan_set_k": (i, [vp, i]),
+        "swan_append": (i, [vp, i, vp, vp, i]),
+        "swan_flush_buffer": (i, [vp, i]),
+        "swan_decode": (i, [vp, i, vp, vp]),
+        "swan_query": (i, [vp, i, ctypes.POINTER(LayerInfo)]),
+        "swan_debug_export": (i, [vp, i, i, vp, ctypes.c_size_t]),
+        "swan_check": (i, [vp]),
+        "swan_timing_enable": (i, [vp, i]),
+        "swan_timing_read": (i, [vp, ctypes.POINTER(Timing)]),
+        "swan_launch_count": (i64, [vp]),
+        "swan_status_string": (ctypes.c_char_p, [i]),
+        "swan_last_error": (ctypes.c_char_p, []),
+    }
+    for name, (res, args) in sig.items():
+        fn = getattr(lib, name)
+        fn.restype = res
+        fn.argtypes = args
+    _lib = lib
+    return lib
+
+
+def _check(status: int, where: str):
+    if status != OK:
+        lib = load_library()
+        detail = lib.swan_last_error().decode() or lib.swan_status_string(status).decode()
+        raise SwanError(status, where, detail)
+
+
+def _ptr(t) -> int:
+    """Device address of a contiguous CUDA tensor (or a raw int address)."""
+    if isinstance(t, int):
+        return t
+    if not t.is_cuda:
+        raise ValueError("tensor must live on the GPU")
+    if not t.is_contiguous():
+        raise ValueError("tensor must be contiguous")
+    return t.data_ptr()
+
+
+class Context:
+    """One SWAN cache (``num_layers`` layers) on the current CUDA device.
+
+    ``R_qk``/``R_vo``: CUDA fp32 tensors ``[num_layers][n_kv_heads][128][128]``.
+    ``stream``: a ``torch.cuda.Stream`` (default: the current stream).
+    """
+
+    def __init__(self, R_qk, R_vo=None, *, num_layers: int, batch: int, n_q_heads: int,
+                 n_kv_heads: int, k_store: int, buffer_cap: int, max_seq: int,
+                 page_tokens: int = 0, head_dim: int = 128, stream=None):
+        import torch
+        self._lib = load_library()
+        if stream is None:
+            stream = torch.cuda.current_stream()
+        self.stream = stream
+        self.cfg = SwanConfig(num_layers, batch, n_q_heads, n_kv_heads, head_dim, k_store,
+                              buffer_cap, max_seq, page_tokens, ctypes.c_void_p(stream.cuda_stream))
+        self.batch, self.n_q_heads, self.n_kv_heads = batch, n_q_heads, n_kv_heads
+        self.num_layers, self.k_store, self.head_dim = num_layers, k_store, head_dim
+        h = ctypes.c_void_p()
+        _check(self._lib.swan_init(ctypes.byref(h), ctypes.byref(self.cfg), _ptr(R_qk),
+                                   None if R_vo is None else _ptr(R_vo)), "swan_init")
+        self._h = h
+
+    # -- lifecycle ----------------------------------------------------------
+    def close(self):
+        if getattr(self, "_h", None):
+            self._lib.swan_destroy(self._h)
+            self._h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:  # noqa: BLE001 - interpreter shutdown
+            pass
+
+    def __enter__(self):
+        return self
+
+    def __exit__(self, *exc):
+        self.close()
+
+    # -- the hot path ------------------------------------------------------
+    def set_k(self, k_active: int):
+        _check(self._lib.swan_set_k(self._h, int(k_active)), "swan_set_k")
+
+    def append(self, layer: int, k_new, v_new, T: int | None = None):
+        if T is None:
+            T = k_new.shape[2]
+        _check(self._lib.swan_append(self._h, int(layer), _ptr(k_new), _ptr(v_new), int(T)),
+               "swan_append")
+
+    def flush(self, layer: int = -1):
+        _check(self._lib.swan_flush_buffer(self._h, int(layer)), "swan_flush_buffer")
+
+    def decode(self, layer: int, q, out=None):
+        if out is None:
+            import torch
+            out = torch.empty_like(q)
+        _check(self._lib.swan_decode(self._h, int(layer), _ptr(q), _ptr(out)), "swan_decode")
+        return out
+
+    # -- inspection --------------------------------------------------------
+    def query(self, layer: int = 0) -> LayerInfo:
+        info = LayerInfo()
+        _check(self._lib.swan_query(self._h, int(layer), ctypes.byref(info)), "swan_query")
+        return info
+
+    def check(self):
+        _check(self._lib.swan_check(self._h), "swan_check")
+
+    def export_buffer(self, layer: int, which: str) -> np.ndarray:
+        info = self.query(layer)
+        shape = (self.batch, self.n_kv_heads, info.buffer_len, self.head_dim)
+        out = np.empty(shape, np.float16)
+        what = EXPORT_BUFFER_K if which == "k" else EXPORT_BUFFER_V
+        _check(self._lib.swan_debug_export(self._h, int(layer), what,
+                                           out.ctypes.data_as(ctypes.c_void_p), out.nbytes),
+               "swan_debug_export")
+        return out
+
+    def export_sparse(self, layer: int, which: str):
+        info = self.query(layer)
+        shape = (self.batch, self.n_kv_heads, info.sparse_len, self.k_store)
+        n = int(np.prod(shape))
+        raw = np.empty(n * 3, np.uint8)
+        what = EXPORT_SPARSE_K if which == "k" else EXPORT_SPARSE_V
+        _check(self._lib.swan_debug_export(self._h, int(layer), what,
+                                           raw.ctypes.data_as(ctypes.c_void_p), raw.nbytes),
+               "swan_debug_export")
+        idx = raw[:n].reshape(shape)
+        vals = raw[n:].view(np.float16).reshape(shape)
+        return idx, vals
+
+    def timing_enable(self, on: bool = True):
+        _check(self._lib.swan_timing_enable(self._h, 1 if on else 0), "swan_timing_enable")
+
+    def timing_read(self) -> dict:
+        t = Timing()
+        _check(self._lib.swan_timing_read(self._h, ctypes.byref(t)), "swan_timing_read")
+        return {KERNEL_NAMES[k]: (t.ms[k], t.launches[k]) for k in KERNEL_NAMES}
+
+    def launch_count(self) -> int:
+        return int(self._lib.swan_launch_count(self._h))

@@ -193,12 +193,12 @@ def run_reference(args, wl, rank: int):
     return line
 
 
-def cpu_baseline_leg(wl, budget_s: float = 20.0):
+def cpu_baseline_leg(wl, budget_s: float = 15.0):
     step = oracle_sample(wl, 1)
     step()
     t0 = time.perf_counter()
     toks, n = 0, 0
-    while time.perf_counter() - t0 < budget_s and n < 200:
+    while time.perf_counter() - t0 < budget_s:
         toks += step()
         n += 1
     dt = time.perf_counter() - t0
@@ -383,10 +383,15 @@ def main():
     ap.add_argument("--e2e-steps", type=int, default=20)
     ap.add_argument("--seed", type=int, default=0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--batch", type=int, default=0,
+                    help="override the workload's batch (smaller cases for profiling)")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
-    wl = WORKLOADS[args.workload]
+    wl = dict(WORKLOADS[args.workload])
+    if args.batch:
+        wl["B"] = args.batch
+        wl["desc"] += f" (batch overridden to {args.batch})"
 
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
@@ -404,8 +409,6 @@ def main():
     line = run_swan(args, wl, rank, world, local_rank)
     if rank == 0:
         if not args.no_cpu_baseline and world == 1:
-            line["cpu_baseline"] = cpu_baseline_leg(wl)
-        elif not args.no_cpu_baseline:
             line["cpu_baseline"] = cpu_baseline_leg(wl)
         print(json.dumps(line), flush=True)
     if world > 1:

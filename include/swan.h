@@ -199,6 +199,74 @@ typedef struct swan_timing {
 swan_status swan_timing_enable(swan_ctx* ctx, int enable);
 swan_status swan_timing_read(swan_ctx* ctx, swan_timing* out);
 
+/*
+ * Decode without allocating: the paper has no counterpart; this is a
+ * deployment interface for callers that cannot call cudaMalloc, such as an
+ * engine that hands out all device memory from its own reserved pool and
+ * must not see a hidden allocation, or that reserves its memory budget up
+ * front.  swan_init allocates the cache and per-call scratch with cudaMalloc;
+ * this entry point instead decodes over a cache held in the caller's own
+ * device memory and keeps its scratch (rotated queries and split partials)
+ * in a fixed static device array inside the library.  It calls no cudaMalloc,
+ * cudaFree or other allocating routine.
+ *
+ * view: the caller's cache, all pointers device pointers on the current
+ *   device, caller-owned:
+ *   pages       page pool; page p starts at pages + p * page_tokens *
+ *               k_slots * 6 and holds, for P = page_tokens tokens, four
+ *               regions: K values [k_slots/8][P][8] fp16, K indices
+ *               [k_slots/8][P][8] uint8, V values, V indices (same shapes).
+ *               Record (chunk c, token t) holds entries 8c..8c+7 of token t's
+ *               kept coordinates in decreasing magnitude order.  This is the
+ *               layout swan_init's own pool uses.
+ *   page_table  int32 [batch * n_kv_heads][pages_per_unit]: page of the
+ *               unit's sparse tokens p*P .. p*P+P-1; entries index `pages`
+ *               and must be < num_pages.
+ *   buf_k/v     fp16 [batch * n_kv_heads][buffer_cap][d] rotated dense ring;
+ *               buffered token i (oldest first) is at slot
+ *               (buf_start + i) % buffer_cap.
+ *   R_qk        fp32 [n_kv_heads][d][d]; R_vo_t fp32 [n_kv_heads][d][d]
+ *               holding R_vo transposed (R_vo_t[h][j][i] = R_vo[h][i][j]).
+ * q, out: device fp16 [batch][n_q_heads][d]; out as for swan_decode.
+ * stream: cudaStream_t (NULL = default stream).
+ *
+ * Limits of the static scratch (about 1.6 MB per device, held from the
+ * library's first use on that device until the process exits):
+ * batch * n_q_heads <= 1024 and (decode CTAs + batch * n_kv_heads) * G <=
+ * 2048, where decode CTAs is at most (SM count x resident CTAs per SM; 152 on
+ * a GB300).  Larger sizes return SWAN_ERR_INVALID_ARG with a message.
+ * The first call on a device resolves the scratch address and the grid limits
+ * (cudaGetSymbolAddress, occupancy queries); make that first call before any
+ * stream capture.  Every call on a device shares the one scratch array, which
+ * keeps the last call's contents: calls that overlap on the GPU (different
+ * streams, or different host threads) race and give wrong results; serialise
+ * them.  Device-side consistency checks are recorded in the scratch and not
+ * reported.  Errors: INVALID_ARG, UNSUPPORTED, CUDA.
+ */
+typedef struct swan_cache_view {
+  const void* pages;
+  const int32_t* page_table;
+  int64_t num_pages;
+  int pages_per_unit;
+  int page_tokens;       /* P, multiple of 32 */
+  int k_slots;           /* entries stored per vector, multiple of 8, <= 128 */
+  int k_active;          /* entries used, 1..k_slots */
+  const void* buf_k;
+  const void* buf_v;
+  int buffer_cap;
+  int buf_start;
+  int buf_len;
+  int64_t sparse_len;    /* sparse tokens per sequence */
+  int batch;
+  int n_q_heads;
+  int n_kv_heads;
+  int head_dim;          /* must be 128 */
+  const float* R_qk;
+  const float* R_vo_t;
+} swan_cache_view;
+swan_status swan_decode_noalloc(const swan_cache_view* view, const void* q, void* out,
+                                void* stream);
+
 /* Number of kernels this context has launched since swan_init. */
 int64_t swan_launch_count(const swan_ctx* ctx);
 

@@ -1,0 +1,187 @@
+// swan_decode_noalloc: one decode step over a cache held in caller-owned
+// device memory, with no device allocation of any kind.
+//
+// For callers that may not call cudaMalloc (for example an engine whose
+// device memory all comes from its own pre-reserved pool, or code running
+// where an allocation would break a memory budget or a captured sequence of
+// work), the per-call scratch of the decode path (rotated queries and split
+// partials) lives in a file-scope static device array of a fixed size
+// instead of context-owned memory.  The array exists once per device that
+// loads the library and stays allocated until the process exits.
+#include <algorithm>
+#include <cmath>
+#include <cstdio>
+#include <mutex>
+
+#include "swan.h"
+#include "swan_internal.h"
+
+namespace swan {
+namespace {
+
+constexpr int kNoallocMaxQ = 1024;         // batch * n_q_heads
+constexpr int kNoallocMaxSlots = 2048;     // (decode CTAs + units) * G partials
+constexpr size_t kQFloats = (size_t)kNoallocMaxQ * kHeadDim;
+constexpr size_t kPartFloats = (size_t)kNoallocMaxSlots * (kHeadDim + 2);
+constexpr size_t kStatusFloats = 64;       // 256 bytes, the status word first
+
+// Layout: [rotated queries][split partials][status word]
+__device__ __align__(256) float g_noalloc_scratch[kQFloats + kPartFloats + kStatusFloats];
+
+constexpr int kMaxDevices = 64;
+struct DeviceSetup {
+  bool ready = false;
+  float* scratch = nullptr;  // device address of g_noalloc_scratch
+  int sms = 0;
+  int ctas_per_sm[3][2] = {};  // [G = 1, 2, 4][k_slots <= 64, > 64]
+};
+DeviceSetup g_setup[kMaxDevices];
+std::mutex g_setup_mutex;
+
+thread_local char g_err[256];
+
+swan_status err(swan_status s, const char* msg) {
+  snprintf(g_err, sizeof(g_err), "swan_decode_noalloc: %s", msg);
+  set_last_error(g_err);
+  return s;
+}
+
+int gi(int G) { return G == 1 ? 0 : G == 2 ? 1 : 2; }
+
+// Once per device, with that device current: resolve the device address of
+// the static scratch array and the decode grid limits.
+swan_status setup_device(int dev, DeviceSetup** out) {
+  if (dev < 0 || dev >= kMaxDevices) return err(SWAN_ERR_UNSUPPORTED, "device index out of range");
+  std::lock_guard<std::mutex> lock(g_setup_mutex);
+  DeviceSetup& s = g_setup[dev];
+  if (!s.ready) {
+    void* p = nullptr;
+    cudaError_t e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+    if (e != cudaSuccess || p == nullptr) return err(SWAN_ERR_CUDA, "cudaGetSymbolAddress failed");
+    e = cudaDeviceGetAttribute(&s.sms, cudaDevAttrMultiProcessorCount, dev);
+    if (e != cudaSuccess) return err(SWAN_ERR_CUDA, "cudaDeviceGetAttribute failed");
+    const int gs[3] = {1, 2, 4};
+    for (int g = 0; g < 3; ++g)
+      for (int big = 0; big < 2; ++big) {
+        s.ctas_per_sm[g][big] = decode_ctas_per_sm(gs[g], big ? 128 : 64);
+        if (s.ctas_per_sm[g][big] < 1) return err(SWAN_ERR_CUDA, "decode kernel occupancy query failed");
+      }
+    s.scratch = static_cast<float*>(p);
+    s.ready = true;
+  }
+  *out = &s;
+  return SWAN_OK;
+}
+
+}  // namespace
+}  // namespace swan
+
+using namespace swan;
+
+extern "C" swan_status swan_decode_noalloc(const swan_cache_view* v, const void* q, void* out,
+                                           void* stream) {
+  set_last_error("");
+  if (!v || !q || !out) return err(SWAN_ERR_INVALID_ARG, "NULL view, q or out");
+  if (v->head_dim != kHeadDim) return err(SWAN_ERR_UNSUPPORTED, "head_dim must be 128");
+  if (v->batch < 1 || v->n_kv_heads < 1 || v->n_q_heads < 1 || v->n_q_heads % v->n_kv_heads)
+    return err(SWAN_ERR_INVALID_ARG, "bad batch or head counts");
+  const int G = v->n_q_heads / v->n_kv_heads;
+  if (G != 1 && G != 2 && G != 4) return err(SWAN_ERR_UNSUPPORTED, "group size must be 1, 2 or 4");
+  if (v->k_slots < 8 || v->k_slots > kHeadDim || v->k_slots % 8)
+    return err(SWAN_ERR_INVALID_ARG, "k_slots must be a multiple of 8 in [8, 128]");
+  if (v->k_active < 1 || v->k_active > v->k_slots) return err(SWAN_ERR_INVALID_ARG, "k_active out of range");
+  if (v->page_tokens < 32 || v->page_tokens % 32 || v->page_tokens > 4096)
+    return err(SWAN_ERR_INVALID_ARG, "page_tokens must be a multiple of 32 in [32, 4096]");
+  if (v->sparse_len < 0 || v->buf_len < 0 || v->buf_len > v->buffer_cap || v->buffer_cap < 0 ||
+      (v->buffer_cap > 0 && (v->buf_start < 0 || v->buf_start >= v->buffer_cap)))
+    return err(SWAN_ERR_INVALID_ARG, "inconsistent buffer or sparse lengths");
+  if (v->pages_per_unit < 0 || v->sparse_len > (int64_t)v->pages_per_unit * v->page_tokens)
+    return err(SWAN_ERR_INVALID_ARG, "sparse_len exceeds pages_per_unit * page_tokens");
+  if (v->sparse_len > 0 && (!v->pages || !v->page_table || v->num_pages < 1))
+    return err(SWAN_ERR_INVALID_ARG, "NULL pages or page table");
+  if (v->buf_len > 0 && (!v->buf_k || !v->buf_v)) return err(SWAN_ERR_INVALID_ARG, "NULL buffer");
+  if (!v->R_qk || !v->R_vo_t) return err(SWAN_ERR_INVALID_ARG, "NULL rotation matrix");
+  const int64_t nq = (int64_t)v->batch * v->n_q_heads;
+  if (nq > kNoallocMaxQ) return err(SWAN_ERR_INVALID_ARG, "batch * n_q_heads exceeds 1024 (static scratch)");
+
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return err(SWAN_ERR_CUDA, "cudaGetDevice failed");
+  DeviceSetup* ds = nullptr;
+  swan_status st = setup_device(dev, &ds);
+  if (st != SWAN_OK) return st;
+
+  const int64_t units = (int64_t)v->batch * v->n_kv_heads;
+  const int64_t n_sg = (v->sparse_len + 31) / 32;
+  const int64_t n_bg = ((int64_t)v->buf_len + 31) / 32;
+  const int64_t N_g = n_sg + n_bg;
+  const int64_t total = units * N_g;
+  int64_t range = 1, grid = 0;
+  if (total > 0) {
+    const int64_t ctas = std::min<int64_t>((int64_t)ds->sms * ds->ctas_per_sm[gi(G)][v->k_slots > 64], total);
+    range = (total + ctas - 1) / ctas;
+    grid = (total + range - 1) / range;
+  }
+  if ((grid + units) * G > kNoallocMaxSlots)
+    return err(SWAN_ERR_INVALID_ARG, "(decode CTAs + batch * n_kv_heads) * G exceeds 2048 (static scratch)");
+
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  float* qprime = ds->scratch;
+  float* partials = ds->scratch + kQFloats;
+  unsigned* status = reinterpret_cast<unsigned*>(ds->scratch + kQFloats + kPartFloats);
+  // the status word must start at zero; the rest is fully written before use
+  if (cudaMemsetAsync(status, 0, sizeof(unsigned), s) != cudaSuccess)
+    return err(SWAN_ERR_CUDA, "cudaMemsetAsync of the status word failed");
+
+  RotateQParams rq{};
+  rq.q = static_cast<const __half*>(q);
+  rq.R_qk = v->R_qk;
+  rq.qprime = qprime;
+  rq.H_q = v->n_q_heads;
+  rq.G = G;
+  if (launch_rotate_q(rq, v->batch, s) != cudaSuccess) return err(SWAN_ERR_CUDA, "rotate_q launch failed");
+
+  if (grid > 0) {
+    DecodeParams p{};
+    p.qprime = qprime;
+    p.geom.pool = static_cast<uint8_t*>(const_cast<void*>(v->pages));
+    p.geom.page_table = v->page_table;
+    p.geom.pages_per_unit = v->pages_per_unit;
+    p.geom.num_pages = v->num_pages;
+    p.geom.P = v->page_tokens;
+    p.geom.k_slots = v->k_slots;
+    p.geom.k_store = v->k_slots;
+    p.geom.page_bytes = (int64_t)v->page_tokens * v->k_slots * 6;
+    p.ring_k = static_cast<const __half*>(v->buf_k);
+    p.ring_v = static_cast<const __half*>(v->buf_v);
+    p.cap = v->buffer_cap > 0 ? v->buffer_cap : 1;
+    p.buf_start = v->buf_start;
+    p.n_b = v->buf_len;
+    p.sparse_len = v->sparse_len;
+    p.n_sg = n_sg;
+    p.N_g = N_g;
+    p.total_groups = total;
+    p.range = range;
+    p.H_kv = v->n_kv_heads;
+    p.H_q = v->n_q_heads;
+    p.k_full_chunks = v->k_active / 8;
+    p.k_rem = v->k_active % 8;
+    p.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)kHeadDim));
+    p.partials = partials;
+    p.status = status;
+    if (launch_decode(p, G, v->k_slots, (int)grid, s) != cudaSuccess)
+      return err(SWAN_ERR_CUDA, "decode launch failed");
+  }
+
+  CombineParams cp{};
+  cp.partials = partials;
+  cp.R_voT = v->R_vo_t;
+  cp.out = static_cast<__half*>(out);
+  cp.H_kv = v->n_kv_heads;
+  cp.H_q = v->n_q_heads;
+  cp.G = G;
+  cp.N_g = N_g > 0 ? N_g : 1;
+  cp.range = range;
+  cp.total_groups = total;
+  if (launch_combine(cp, v->batch, s) != cudaSuccess) return err(SWAN_ERR_CUDA, "combine launch failed");
+  return SWAN_OK;
+}

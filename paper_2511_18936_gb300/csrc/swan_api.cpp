@@ -228,6 +228,8 @@ swan_status prune_from_ring(swan_ctx* c, int layer, int count) {
 
 }  // namespace
 
+void swan::set_last_error(const char* msg) { g_last_error = msg ? msg : ""; }
+
 extern "C" {
 
 const char* swan_status_string(swan_status s) {

@@ -126,5 +126,7 @@ cudaError_t launch_transpose_r(const float* src, float* dst, int64_t mats, cudaS
 // Decode CTAs that fit on one SM together (for the grid size).
 int decode_ctas_per_sm(int G, int k_slots);
 size_t decode_smem_bytes(int G);
+// Record the detail string that swan_last_error() returns on this thread.
+void set_last_error(const char* msg);
 
 }  // namespace swan

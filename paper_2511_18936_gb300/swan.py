@@ -27,7 +27,7 @@ KERNEL_NAMES = {KERNEL_ROTATE_Q: "rotate_q", KERNEL_DECODE: "decode", KERNEL_COM
 EXPORTED = ["swan_init", "swan_destroy", "swan_set_k", "swan_append", "swan_flush_buffer",
             "swan_decode", "swan_query", "swan_debug_export", "swan_check",
             "swan_timing_enable", "swan_timing_read", "swan_launch_count",
-            "swan_status_string", "swan_last_error"]
+            "swan_status_string", "swan_last_error", "swan_decode_noalloc"]
 
 
 class SwanConfig(ctypes.Structure):
@@ -47,6 +47,17 @@ class LayerInfo(ctypes.Structure):
 
 class Timing(ctypes.Structure):
     _fields_ = [("ms", ctypes.c_double * KERNEL_KINDS), ("launches", ctypes.c_int64 * KERNEL_KINDS)]
+
+
+class CacheView(ctypes.Structure):
+    """A cache in caller-owned device memory (see swan_decode_noalloc)."""
+    _fields_ = [("pages", ctypes.c_void_p), ("page_table", ctypes.c_void_p),
+                ("num_pages", ctypes.c_int64), ("pages_per_unit", ctypes.c_int),
+                ("page_tokens", ctypes.c_int), ("k_slots", ctypes.c_int), ("k_active", ctypes.c_int),
+                ("buf_k", ctypes.c_void_p), ("buf_v", ctypes.c_void_p), ("buffer_cap", ctypes.c_int),
+                ("buf_start", ctypes.c_int), ("buf_len", ctypes.c_int), ("sparse_len", ctypes.c_int64),
+                ("batch", ctypes.c_int), ("n_q_heads", ctypes.c_int), ("n_kv_heads", ctypes.c_int),
+                ("head_dim", ctypes.c_int), ("R_qk", ctypes.c_void_p), ("R_vo_t", ctypes.c_void_p)]
 
 
 class SwanError(RuntimeError):
@@ -83,6 +94,7 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "swan_launch_count": (i64, [vp]),
         "swan_status_string": (ctypes.c_char_p, [i]),
         "swan_last_error": (ctypes.c_char_p, []),
+        "swan_decode_noalloc": (i, [ctypes.POINTER(CacheView), vp, vp, vp]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(lib, name)
@@ -214,3 +226,16 @@ class Context:
 
     def launch_count(self) -> int:
         return int(self._lib.swan_launch_count(self._h))
+
+
+def decode_noalloc(view: CacheView, q, out, stream=None):
+    """One decode step over a caller-owned cache with no device allocation
+    (``swan_decode_noalloc``); ``stream``: a ``torch.cuda.Stream`` or None for
+    the current stream."""
+    import torch
+    lib = load_library()
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    _check(lib.swan_decode_noalloc(ctypes.byref(view), _ptr(q), _ptr(out),
+                                   ctypes.c_void_p(stream.cuda_stream)), "swan_decode_noalloc")
+    return out

@@ -71,7 +71,8 @@ typedef struct swan_config {
                       count k_active may be any value 1..k_store */
   int buffer_cap;  /* b, dense buffer capacity in tokens, 0..4096 */
   int max_seq;     /* tokens per sequence the cache can hold (sparse + buffer) */
-  int page_tokens; /* tokens per cache page, multiple of 32; 0 = 128 */
+  int page_tokens; /* tokens per cache page, a power of two in [32, 4096];
+                      0 = 128 */
   void* stream;    /* cudaStream_t the context enqueues on; NULL = default */
 } swan_config;
 
@@ -213,12 +214,14 @@ swan_status swan_timing_read(swan_ctx* ctx, swan_timing* out);
  * view: the caller's cache, all pointers device pointers on the current
  *   device, caller-owned:
  *   pages       page pool; page p starts at pages + p * page_tokens *
- *               k_slots * 6 and holds, for P = page_tokens tokens, four
- *               regions: K values [k_slots/8][P][8] fp16, K indices
- *               [k_slots/8][P][8] uint8, V values, V indices (same shapes).
- *               Record (chunk c, token t) holds entries 8c..8c+7 of token t's
- *               kept coordinates in decreasing magnitude order.  This is the
- *               layout swan_init's own pool uses.
+ *               k_slots * 6 and holds P = page_tokens tokens as P/32 blocks
+ *               of 32 tokens, block q at q * 192 * k_slots bytes.  A block
+ *               holds four regions: K values [k_slots/8][32][8] fp16 at 0,
+ *               K indices [k_slots/8][32][8] uint8 at 64 * k_slots, V values
+ *               at 96 * k_slots, V indices at 160 * k_slots.  Record
+ *               (chunk c, token t) holds entries 8c..8c+7 of token t's kept
+ *               coordinates in decreasing magnitude order; indices must be
+ *               < 128.  This is the layout swan_init's own pool uses.
  *   page_table  int32 [batch * n_kv_heads][pages_per_unit]: page of the
  *               unit's sparse tokens p*P .. p*P+P-1; entries index `pages`
  *               and must be < num_pages.
@@ -248,7 +251,7 @@ typedef struct swan_cache_view {
   const int32_t* page_table;
   int64_t num_pages;
   int pages_per_unit;
-  int page_tokens;       /* P, multiple of 32 */
+  int page_tokens;       /* P, a power of two in [32, 4096] */
   int k_slots;           /* entries stored per vector, multiple of 8, <= 128 */
   int k_active;          /* entries used, 1..k_slots */
   const void* buf_k;

@@ -58,9 +58,10 @@ __device__ __forceinline__ void warp_prune_store(uint2 raw, int lane, int kind, 
     if (lane == 0) atomicOr(status, kStatusPageRange);
     return;
   }
-  uint8_t* pg = g.pool + (int64_t)phys * g.page_bytes;
-  const int64_t voff = kind ? g.vval_off() : 0;
-  const int64_t ioff = kind ? g.vidx_off() : g.kidx_off();
+  uint8_t* blk = g.pool + (int64_t)phys * g.page_bytes + (int64_t)(slot >> 5) * g.block_bytes();
+  const int t = slot & 31;
+  const int voff = kind ? g.vval_off() : 0;
+  const int ioff = kind ? g.vidx_off() : g.kidx_off();
   if (lane < (g.k_slots >> 2)) {
     const int c = lane >> 1, half = lane & 1;
     uint32_t vb[4], ib[4];
@@ -74,9 +75,9 @@ __device__ __forceinline__ void warp_prune_store(uint2 raw, int lane, int kind, 
     }
     const uint2 vals = make_uint2(vb[0] | (vb[1] << 16), vb[2] | (vb[3] << 16));
     const uint32_t idx = ib[0] | (ib[1] << 8) | (ib[2] << 16) | (ib[3] << 24);
-    const int64_t rec = (int64_t)c * g.P + slot;
-    *reinterpret_cast<uint2*>(pg + voff + rec * 16 + half * 8) = vals;
-    *reinterpret_cast<uint32_t*>(pg + ioff + rec * 8 + half * 4) = idx;
+    const int rec = c * 32 + t;
+    *reinterpret_cast<uint2*>(blk + voff + rec * 16 + half * 8) = vals;
+    *reinterpret_cast<uint32_t*>(blk + ioff + rec * 8 + half * 4) = idx;
   }
 }
 

@@ -45,77 +45,139 @@ __device__ __forceinline__ float warp_sum(float v) {
   return v;
 }
 
-// Shared-memory address (in floats, relative to a lane's column) of
-// coordinate `i` in a [128][32] lane-interleaved array: element (i, lane) at
-// i*32 + lane, so 32 lanes gathering arbitrary coordinates hit 32 distinct
-// banks.
-__device__ __forceinline__ int col(uint32_t i) { return (int)((i & 0x7fu) << 5); }
-
-// Score contribution of one 8-entry chunk: sum_e q'[idx_e] * val_e.
-__device__ __forceinline__ void score_chunk(const float* qc, uint4 v, uint2 ix, float& s0, float& s1) {
-  const float2 a = h2f(v.x), b = h2f(v.y), c = h2f(v.z), d = h2f(v.w);
-  s0 = fmaf(qc[col(ix.x)], a.x, s0);
-  s1 = fmaf(qc[col(ix.x >> 8)], a.y, s1);
-  s0 = fmaf(qc[col(ix.x >> 16)], b.x, s0);
-  s1 = fmaf(qc[col(ix.x >> 24)], b.y, s1);
-  s0 = fmaf(qc[col(ix.y)], c.x, s0);
-  s1 = fmaf(qc[col(ix.y >> 8)], c.y, s1);
-  s0 = fmaf(qc[col(ix.y >> 16)], d.x, s0);
-  s1 = fmaf(qc[col(ix.y >> 24)], d.y, s1);
+// Shared-memory accesses by 32-bit shared-window address.  They are volatile
+// so that they keep their program order among themselves: each chunk's eight
+// loads are issued back to back, then its eight stores (the indices of one
+// vector are distinct, so the batch never aliases).
+__device__ __forceinline__ float lds(uint32_t a) {
+  float v;
+  asm volatile("ld.shared.f32 %0, [%1];" : "=f"(v) : "r"(a));
+  return v;
+}
+__device__ __forceinline__ void sts(uint32_t a, float v) {
+  asm volatile("st.shared.f32 [%0], %1;" ::"r"(a), "f"(v));
 }
 
-// Scatter-accumulate one 8-entry chunk: acc[idx_e] += p * val_e.
-__device__ __forceinline__ void value_chunk(float* ac, float p, uint4 v, uint2 ix) {
+// Address of coordinate idx (byte e of the index record word w) in a
+// [128][32] lane-interleaved fp32 array whose base is 16 KB aligned:
+// base | (idx & 127) << 7 | lane << 2.  One shift and one LOP3; element
+// (idx, lane) sits at idx*32 + lane, so 32 lanes gathering arbitrary
+// coordinates hit 32 distinct banks, and any index byte stays inside the
+// array.
+template <int E>
+__device__ __forceinline__ uint32_t addr_of(uint32_t w, uint32_t base) {
+  if (E == 0) return ((w << 7) & 0x3f80u) | base;
+  if (E == 1) return ((w >> 1) & 0x3f80u) | base;
+  if (E == 2) return ((w >> 9) & 0x3f80u) | base;
+  return ((w >> 17) & 0x3f80u) | base;
+}
+
+// Score contribution of one 8-entry chunk into four partial sums.
+__device__ __forceinline__ void score_chunk(uint32_t qb, uint4 v, uint2 ix, float (&s)[4]) {
+  const float q0 = lds(addr_of<0>(ix.x, qb)), q1 = lds(addr_of<1>(ix.x, qb));
+  const float q2 = lds(addr_of<2>(ix.x, qb)), q3 = lds(addr_of<3>(ix.x, qb));
+  const float q4 = lds(addr_of<0>(ix.y, qb)), q5 = lds(addr_of<1>(ix.y, qb));
+  const float q6 = lds(addr_of<2>(ix.y, qb)), q7 = lds(addr_of<3>(ix.y, qb));
   const float2 a = h2f(v.x), b = h2f(v.y), c = h2f(v.z), d = h2f(v.w);
-  float* t;
-  t = ac + col(ix.x);        *t = fmaf(p, a.x, *t);
-  t = ac + col(ix.x >> 8);   *t = fmaf(p, a.y, *t);
-  t = ac + col(ix.x >> 16);  *t = fmaf(p, b.x, *t);
-  t = ac + col(ix.x >> 24);  *t = fmaf(p, b.y, *t);
-  t = ac + col(ix.y);        *t = fmaf(p, c.x, *t);
-  t = ac + col(ix.y >> 8);   *t = fmaf(p, c.y, *t);
-  t = ac + col(ix.y >> 16);  *t = fmaf(p, d.x, *t);
-  t = ac + col(ix.y >> 24);  *t = fmaf(p, d.y, *t);
+  s[0] = fmaf(q0, a.x, s[0]);
+  s[1] = fmaf(q1, a.y, s[1]);
+  s[2] = fmaf(q2, b.x, s[2]);
+  s[3] = fmaf(q3, b.y, s[3]);
+  s[0] = fmaf(q4, c.x, s[0]);
+  s[1] = fmaf(q5, c.y, s[1]);
+  s[2] = fmaf(q6, d.x, s[2]);
+  s[3] = fmaf(q7, d.y, s[3]);
+}
+
+// acc[idx_e] += p * val_e for one full chunk (distinct indices): eight loads,
+// eight FMAs, eight stores.
+__device__ __forceinline__ void value_chunk(uint32_t ab, float p, uint4 v, uint2 ix) {
+  const uint32_t a0 = addr_of<0>(ix.x, ab), a1 = addr_of<1>(ix.x, ab);
+  const uint32_t a2 = addr_of<2>(ix.x, ab), a3 = addr_of<3>(ix.x, ab);
+  const uint32_t a4 = addr_of<0>(ix.y, ab), a5 = addr_of<1>(ix.y, ab);
+  const uint32_t a6 = addr_of<2>(ix.y, ab), a7 = addr_of<3>(ix.y, ab);
+  const float o0 = lds(a0), o1 = lds(a1), o2 = lds(a2), o3 = lds(a3);
+  const float o4 = lds(a4), o5 = lds(a5), o6 = lds(a6), o7 = lds(a7);
+  const float2 a = h2f(v.x), b = h2f(v.y), c = h2f(v.z), d = h2f(v.w);
+  sts(a0, fmaf(p, a.x, o0));
+  sts(a1, fmaf(p, a.y, o1));
+  sts(a2, fmaf(p, b.x, o2));
+  sts(a3, fmaf(p, b.y, o3));
+  sts(a4, fmaf(p, c.x, o4));
+  sts(a5, fmaf(p, c.y, o5));
+  sts(a6, fmaf(p, d.x, o6));
+  sts(a7, fmaf(p, d.y, o7));
+}
+
+// The first `n` (< 8) entries of a chunk, one read-modify-write at a time
+// (the masked tail of a runtime keep count that is not a multiple of 8).
+__device__ __forceinline__ void value_chunk_partial(uint32_t ab, float p, uint4 v, uint2 ix, int n) {
+  const uint32_t hw[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+  for (int e = 0; e < 7; ++e) {
+    if (e < n) {
+      const uint32_t w = e < 4 ? ix.x : ix.y;
+      const uint32_t sh = 8u * (e & 3);
+      const uint32_t a = ((w >> sh) & 0x7fu) << 7 | ab;
+      const float2 f = h2f(hw[e >> 1]);
+      sts(a, fmaf(p, (e & 1) ? f.y : f.x, lds(a)));
+    }
+  }
 }
 
 __device__ __forceinline__ uint4 and4(uint4 a, uint4 m) {
   return make_uint4(a.x & m.x, a.y & m.y, a.z & m.z, a.w & m.w);
 }
 
+constexpr uint32_t kRegionBytes = kHeadDim * 32 * sizeof(float);  // 16 KB
+
+// Ask the memory system to bring `bytes` (a multiple of 16, 16-byte aligned)
+// into L2 ahead of the loads that will read them.
+__device__ __forceinline__ void prefetch_l2(const void* ptr, uint32_t bytes) {
+  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(ptr), "r"(bytes) : "memory");
+}
+
 // Split decode kernel.
-//   Shared memory: q' of the unit's G query heads replicated per lane
-//   ([G][128][32] fp32) and one lane-private rotated-space accumulator per
-//   warp ([8][128][32] fp32).  Both are indexed (coordinate, lane), so the
-//   random gathers and scatters of 32 lanes never share a bank.
-//   Warp w serves query head w % G; the G warps of a team walk the same
-//   32-token groups.  Lane = token.
+//   Shared memory (16 KB-aligned regions): q' of the unit's G query heads
+//   replicated per lane ([G][128][32] fp32) and one lane-private
+//   rotated-space accumulator per warp ([8][128][32] fp32).
+//   Lane = token.  Warp w serves query head w % G; the G warps of a team walk
+//   the same contiguous run of 32-token blocks.  While block g is processed,
+//   the key records of block g+1 are in flight to registers and block g+2 is
+//   being prefetched into L2.
 template <int G, int MAXC>
 __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
   constexpr int TEAMS = kWarpsPerCta / G;
   constexpr bool kL1 = G > 1;
-  constexpr bool kPreloadV = MAXC <= 8;
-  extern __shared__ __align__(16) float smem[];
-  float* qrep = smem;                          // [G][128][32]
-  float* accs = smem + G * kHeadDim * 32;      // [8][128][32]
+  extern __shared__ __align__(16) unsigned char smem_raw[];
   __shared__ float red_m[kWarpsPerCta], red_l[kWarpsPerCta];
+
+  const uint32_t raw = (uint32_t)__cvta_generic_to_shared(smem_raw);
+  const uint32_t base = (raw + kRegionBytes - 1) & ~(kRegionBytes - 1);
+  float* qrep = reinterpret_cast<float*>(smem_raw + (base - raw));  // [G][128][32]
+  float* accs = qrep + G * kHeadDim * 32;                            // [8][128][32]
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int hh = warp % G, team = warp / G;
-  float* my_acc = accs + warp * kHeadDim * 32 + lane;
-  const float* my_q = qrep + hh * kHeadDim * 32 + lane;
+  const uint32_t qb = base + hh * kRegionBytes + (lane << 2);
+  const uint32_t ab = base + (G + warp) * kRegionBytes + (lane << 2);
 
   const CacheGeom& g = p.geom;
-  const int P = g.P;
-  const int nchunks = p.k_full_chunks + (p.k_rem ? 1 : 0);
-  uint4 remmask = make_uint4(0, 0, 0, 0);
+  const int kfull = p.k_full_chunks, krem = p.k_rem;
+  const int nchunks = kfull + (krem ? 1 : 0);
+  const int ks = g.k_slots;
+  // byte offsets inside a block, plus this lane's record
+  const int o_kv = lane * 16, o_ki = 64 * ks + lane * 8;
+  const int o_vv = 96 * ks + lane * 16, o_vi = 160 * ks + lane * 8;
+  const bool whole_block = nchunks * 8 == ks;
+  const uint32_t pf_val = (uint32_t)nchunks * 512, pf_idx = (uint32_t)nchunks * 256;
+  const int bsh = p.blocks_per_page_log2, bmask = (1 << bsh) - 1;
+  uint4 remmask;
   {
     uint32_t w[4];
 #pragma unroll
-    for (int e = 0; e < 4; ++e) {
-      const uint32_t lo = (2 * e < p.k_rem) ? 0xffffu : 0u;
-      const uint32_t hi = (2 * e + 1 < p.k_rem) ? 0xffff0000u : 0u;
-      w[e] = lo | hi;
-    }
+    for (int e = 0; e < 4; ++e)
+      w[e] = ((2 * e < krem) ? 0xffffu : 0u) | ((2 * e + 1 < krem) ? 0xffff0000u : 0u);
     remmask = make_uint4(w[0], w[1], w[2], w[3]);
   }
 
@@ -123,11 +185,18 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
   const int64_t g_end = min(p.total_groups, g_begin + p.range);
   if (g_begin >= g_end) return;
   const int64_t u_first = g_begin / p.N_g, u_last = (g_end - 1) / p.N_g;
+  const int n_sg = (int)p.n_sg;
 
   for (int64_t u = u_first; u <= u_last; ++u) {
-    const int64_t s0 = max(g_begin, u * p.N_g) - u * p.N_g;
-    const int64_t s1 = min(g_end, (u + 1) * p.N_g) - u * p.N_g;
+    const int s0 = (int)(max(g_begin, u * p.N_g) - u * p.N_g);
+    const int s1 = (int)(min(g_end, (u + 1) * p.N_g) - u * p.N_g);
     const int64_t b = u / p.H_kv, h = u % p.H_kv;
+    // this team's contiguous run of groups [t_lo, t_hi)
+    const int len = s1 - s0;
+    const int t_lo = s0 + (len * team) / TEAMS;
+    const int t_hi = s0 + (len * (team + 1)) / TEAMS;
+    const int sp_hi = min(t_hi, n_sg);  // sparse groups of the run: [t_lo, sp_hi)
+    const int32_t* ptab = g.page_table + u * g.pages_per_unit;
 
     __syncthreads();  // the previous segment's reduction is done with smem
     for (int i = threadIdx.x; i < G * kHeadDim * 32; i += kThreads) {
@@ -135,66 +204,92 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
       qrep[i] = __ldg(p.qprime + ((b * p.H_q + h * G + gh) * kHeadDim + dd));
     }
 #pragma unroll 8
-    for (int dd = 0; dd < kHeadDim; ++dd) my_acc[dd * 32] = 0.f;
+    for (int dd = 0; dd < kHeadDim; ++dd) sts(ab + dd * 128, 0.f);
     __syncthreads();
 
     float m_w = -INFINITY;  // running max (log2 domain), uniform in the warp
     float l_sum = 0.f;      // this lane's sum of exp2(s - m_w)
 
-    for (int64_t gi = s0 + team; gi < s1; gi += TEAMS) {
-      float s2;
-      bool valid;
-      if (gi < p.n_sg) {
-        // ---- sparse group: tokens 32*gi .. 32*gi+31 of the sparse history
-        const int64_t t0 = gi * 32;
-        valid = t0 + lane < p.sparse_len;
-        const int64_t page = t0 / P;
-        const int slot = (int)(t0 % P) + lane;
-        int32_t phys = g.page_table[u * g.pages_per_unit + page];
-        if (phys < 0 || phys >= g.num_pages) {
-          if (lane == 0) atomicOr(p.status, kStatusPageRange);
-          phys = 0;
-          valid = false;
+    // block of sparse group gi (nullptr past the run or on a bad page)
+    auto block_of = [&](int gi) -> const uint8_t* {
+      if (gi >= sp_hi) return nullptr;
+      const int32_t ph = __ldg(ptab + (gi >> bsh));
+      if (ph < 0 || ph >= g.num_pages) {
+        atomicOr(p.status, kStatusPageRange);
+        return nullptr;
+      }
+      return g.pool + (int64_t)ph * g.page_bytes + (int64_t)(gi & bmask) * g.block_bytes();
+    };
+    auto prefetch_block = [&](const uint8_t* blk) {
+      if (blk == nullptr || lane != 0) return;
+      if (whole_block) {
+        prefetch_l2(blk, (uint32_t)g.block_bytes());
+      } else {
+        prefetch_l2(blk, pf_val);
+        prefetch_l2(blk + 64 * ks, pf_idx);
+        prefetch_l2(blk + 96 * ks, pf_val);
+        prefetch_l2(blk + 160 * ks, pf_idx);
+      }
+    };
+    auto load_k = [&](const uint8_t* blk, uint4 (&kv)[MAXC], uint2 (&ki)[MAXC]) {
+      const uint8_t* src = blk ? blk : g.pool;
+#pragma unroll
+      for (int c = 0; c < MAXC; ++c)
+        if (c < nchunks) {
+          kv[c] = ld_rec16<kL1>(src + o_kv + c * 512);
+          ki[c] = ld_rec8<kL1>(src + o_ki + c * 256);
         }
-        const uint8_t* pg = g.pool + (int64_t)phys * g.page_bytes;
-        const uint4* kv = reinterpret_cast<const uint4*>(pg) + slot;
-        const uint2* ki = reinterpret_cast<const uint2*>(pg + g.kidx_off()) + slot;
-        const uint4* vv = reinterpret_cast<const uint4*>(pg + g.vval_off()) + slot;
-        const uint2* vi = reinterpret_cast<const uint2*>(pg + g.vidx_off()) + slot;
-        const bool tail = t0 + 32 > p.sparse_len;  // warp-uniform
-        const uint4 lanemask = valid ? make_uint4(~0u, ~0u, ~0u, ~0u) : make_uint4(0, 0, 0, 0);
+    };
 
-        uint4 kvr[MAXC];
-        uint2 kir[MAXC];
-        uint4 vvr[kPreloadV ? MAXC : 1];
-        uint2 vir[kPreloadV ? MAXC : 1];
+    uint4 kv[MAXC];
+    uint2 ki[MAXC];
+    const uint8_t* b_cur = block_of(t_lo);
+    const uint8_t* b_n1 = block_of(t_lo + 1);
+    prefetch_block(b_n1);
+    if (t_lo < sp_hi) load_k(b_cur, kv, ki);
+
+    for (int gi = t_lo; gi < t_hi; ++gi) {
+      float s2, pr;
+      if (gi < n_sg) {
+        // ---- sparse group: tokens 32*gi .. 32*gi+31 of the sparse history
+        const int64_t t0 = (int64_t)gi * 32;
+        const bool ok = b_cur != nullptr;
+        const bool valid = ok && t0 + lane < p.sparse_len;
+        const bool tail = !ok || t0 + 32 > p.sparse_len;  // warp-uniform
+        const uint8_t* src = ok ? b_cur : g.pool;
+        uint4 vv[MAXC];
+        uint2 vi[MAXC];
 #pragma unroll
-        for (int c = 0; c < MAXC; ++c) {
+        for (int c = 0; c < MAXC; ++c)
           if (c < nchunks) {
-            kvr[c] = ld_rec16<kL1>(kv + (int64_t)c * P);
-            kir[c] = ld_rec8<kL1>(ki + (int64_t)c * P);
+            vv[c] = ld_rec16<kL1>(src + o_vv + c * 512);
+            vi[c] = ld_rec8<kL1>(src + o_vi + c * 256);
           }
-        }
-        if constexpr (kPreloadV) {
+        // two blocks ahead: into L2
+        const uint8_t* b_n2 = block_of(gi + 2);
+        prefetch_block(b_n2);
+
+        const uint4 lanemask = valid ? make_uint4(~0u, ~0u, ~0u, ~0u) : make_uint4(0, 0, 0, 0);
+        float s[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-          for (int c = 0; c < MAXC; ++c) {
-            if (c < nchunks) {
-              vvr[c] = ld_rec16<kL1>(vv + (int64_t)c * P);
-              vir[c] = ld_rec8<kL1>(vi + (int64_t)c * P);
+        for (int c = 0; c < MAXC; ++c)
+          if (c < nchunks) {
+            uint4 v = kv[c];
+            uint2 ix = ki[c];
+            if (krem && c == nchunks - 1) v = and4(v, remmask);
+            if (tail) {
+              v = and4(v, lanemask);
+              ix = valid ? ix : make_uint2(0, 0);
             }
+            score_chunk(qb, v, ix, s);
           }
-        }
-        float sa = 0.f, sb = 0.f;
-#pragma unroll
-        for (int c = 0; c < MAXC; ++c) {
-          if (c < nchunks) {
-            uint4 v = kvr[c];
-            if (p.k_rem && c == nchunks - 1) v = and4(v, remmask);
-            if (tail) v = and4(v, lanemask);
-            score_chunk(my_q, v, kir[c], sa, sb);
-          }
-        }
-        s2 = valid ? (sa + sb) * p.scale_log2 : -INFINITY;
+        s2 = valid ? ((s[0] + s[1]) + (s[2] + s[3])) * p.scale_log2 : -INFINITY;
+
+        // the next block's key records into registers while this block's
+        // values are accumulated
+        if (gi + 1 < sp_hi) load_k(b_n1, kv, ki);
+        b_cur = b_n1;
+        b_n1 = b_n2;
 
         const float gmax = warp_max(s2);
         if (gmax > m_w + kLazyRescale) {
@@ -202,80 +297,82 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
             const float f = exp2f(m_w - gmax);
             l_sum *= f;
 #pragma unroll 8
-            for (int dd = 0; dd < kHeadDim; ++dd) my_acc[dd * 32] *= f;
+            for (int dd = 0; dd < kHeadDim; ++dd) sts(ab + dd * 128, lds(ab + dd * 128) * f);
           }
           m_w = gmax;
         }
-        const float pr = valid ? exp2f(s2 - m_w) : 0.f;
+        pr = valid ? exp2f(s2 - m_w) : 0.f;
         l_sum += pr;
 
 #pragma unroll
-        for (int c = 0; c < MAXC; ++c) {
-          if (c < nchunks) {
-            uint4 v;
-            uint2 ix;
-            if constexpr (kPreloadV) {
-              v = vvr[c];
-              ix = vir[c];
-            } else {
-              v = ld_rec16<kL1>(vv + (int64_t)c * P);
-              ix = ld_rec8<kL1>(vi + (int64_t)c * P);
+        for (int c = 0; c < MAXC; ++c)
+          if (c < kfull) {
+            uint4 v = vv[c];
+            uint2 ix = vi[c];
+            if (tail) {
+              v = and4(v, lanemask);
+              ix = valid ? ix : make_uint2(0, 0);
             }
-            if (p.k_rem && c == nchunks - 1) v = and4(v, remmask);
-            if (tail) v = and4(v, lanemask);
-            value_chunk(my_acc, pr, v, ix);
+            value_chunk(ab, pr, v, ix);
           }
+        if (krem && valid) {
+#pragma unroll
+          for (int c = 0; c < MAXC; ++c)
+            if (c == kfull) value_chunk_partial(ab, pr, vv[c], vi[c], krem);
         }
       } else {
         // ---- buffer group: dense rotated fp16 vectors of the ring buffer
-        const int64_t i = (gi - p.n_sg) * 32 + lane;
-        valid = i < p.n_b;
+        const int64_t i = (int64_t)(gi - n_sg) * 32 + lane;
+        const bool valid = i < p.n_b;
         const int slot = valid ? (int)((p.buf_start + i) % p.cap) : 0;
         const size_t row = ((size_t)u * p.cap + slot) * kHeadDim;
         const uint4* kr = reinterpret_cast<const uint4*>(p.ring_k + row);
         const uint4* vr = reinterpret_cast<const uint4*>(p.ring_v + row);
-        float sa = 0.f, sb = 0.f;
+        float s[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll 4
         for (int c = 0; c < 16; ++c) {
           const uint4 w = __ldg(kr + c);
           const float2 a = h2f(w.x), bb = h2f(w.y), cc = h2f(w.z), d = h2f(w.w);
-          const float* q = my_q + c * 8 * 32;
-          sa = fmaf(q[0 * 32], a.x, sa);
-          sb = fmaf(q[1 * 32], a.y, sb);
-          sa = fmaf(q[2 * 32], bb.x, sa);
-          sb = fmaf(q[3 * 32], bb.y, sb);
-          sa = fmaf(q[4 * 32], cc.x, sa);
-          sb = fmaf(q[5 * 32], cc.y, sb);
-          sa = fmaf(q[6 * 32], d.x, sa);
-          sb = fmaf(q[7 * 32], d.y, sb);
+          const uint32_t q = qb + c * 8 * 128;
+          s[0] = fmaf(lds(q + 0 * 128), a.x, s[0]);
+          s[1] = fmaf(lds(q + 1 * 128), a.y, s[1]);
+          s[2] = fmaf(lds(q + 2 * 128), bb.x, s[2]);
+          s[3] = fmaf(lds(q + 3 * 128), bb.y, s[3]);
+          s[0] = fmaf(lds(q + 4 * 128), cc.x, s[0]);
+          s[1] = fmaf(lds(q + 5 * 128), cc.y, s[1]);
+          s[2] = fmaf(lds(q + 6 * 128), d.x, s[2]);
+          s[3] = fmaf(lds(q + 7 * 128), d.y, s[3]);
         }
-        s2 = valid ? (sa + sb) * p.scale_log2 : -INFINITY;
+        s2 = valid ? ((s[0] + s[1]) + (s[2] + s[3])) * p.scale_log2 : -INFINITY;
         const float gmax = warp_max(s2);
         if (gmax > m_w + kLazyRescale) {
           if (m_w != -INFINITY) {
             const float f = exp2f(m_w - gmax);
             l_sum *= f;
 #pragma unroll 8
-            for (int dd = 0; dd < kHeadDim; ++dd) my_acc[dd * 32] *= f;
+            for (int dd = 0; dd < kHeadDim; ++dd) sts(ab + dd * 128, lds(ab + dd * 128) * f);
           }
           m_w = gmax;
         }
-        const float pr = valid ? exp2f(s2 - m_w) : 0.f;
+        pr = valid ? exp2f(s2 - m_w) : 0.f;
         l_sum += pr;
         if (valid) {
-#pragma unroll 4
+#pragma unroll 2
           for (int c = 0; c < 16; ++c) {
             const uint4 w = __ldg(vr + c);
             const float2 a = h2f(w.x), bb = h2f(w.y), cc = h2f(w.z), d = h2f(w.w);
-            float* t = my_acc + c * 8 * 32;
-            t[0 * 32] = fmaf(pr, a.x, t[0 * 32]);
-            t[1 * 32] = fmaf(pr, a.y, t[1 * 32]);
-            t[2 * 32] = fmaf(pr, bb.x, t[2 * 32]);
-            t[3 * 32] = fmaf(pr, bb.y, t[3 * 32]);
-            t[4 * 32] = fmaf(pr, cc.x, t[4 * 32]);
-            t[5 * 32] = fmaf(pr, cc.y, t[5 * 32]);
-            t[6 * 32] = fmaf(pr, d.x, t[6 * 32]);
-            t[7 * 32] = fmaf(pr, d.y, t[7 * 32]);
+            const uint32_t t = ab + c * 8 * 128;
+            const float o0 = lds(t + 0 * 128), o1 = lds(t + 1 * 128), o2 = lds(t + 2 * 128),
+                        o3 = lds(t + 3 * 128), o4 = lds(t + 4 * 128), o5 = lds(t + 5 * 128),
+                        o6 = lds(t + 6 * 128), o7 = lds(t + 7 * 128);
+            sts(t + 0 * 128, fmaf(pr, a.x, o0));
+            sts(t + 1 * 128, fmaf(pr, a.y, o1));
+            sts(t + 2 * 128, fmaf(pr, bb.x, o2));
+            sts(t + 3 * 128, fmaf(pr, bb.y, o3));
+            sts(t + 4 * 128, fmaf(pr, cc.x, o4));
+            sts(t + 5 * 128, fmaf(pr, cc.y, o5));
+            sts(t + 6 * 128, fmaf(pr, d.x, o6));
+            sts(t + 7 * 128, fmaf(pr, d.y, o7));
           }
         }
       }
@@ -403,7 +500,7 @@ int ctas_per_sm_t() {
 
 }  // namespace
 
-size_t decode_smem_bytes(int G) { return (size_t)(G + kWarpsPerCta) * kHeadDim * 32 * sizeof(float); }
+size_t decode_smem_bytes(int G) { return (size_t)(G + kWarpsPerCta + 1) * kRegionBytes; }
 
 int decode_ctas_per_sm(int G, int k_slots) {
   const bool big = k_slots > 64;

@@ -90,8 +90,8 @@ extern "C" swan_status swan_decode_noalloc(const swan_cache_view* v, const void*
   if (v->k_slots < 8 || v->k_slots > kHeadDim || v->k_slots % 8)
     return err(SWAN_ERR_INVALID_ARG, "k_slots must be a multiple of 8 in [8, 128]");
   if (v->k_active < 1 || v->k_active > v->k_slots) return err(SWAN_ERR_INVALID_ARG, "k_active out of range");
-  if (v->page_tokens < 32 || v->page_tokens % 32 || v->page_tokens > 4096)
-    return err(SWAN_ERR_INVALID_ARG, "page_tokens must be a multiple of 32 in [32, 4096]");
+  if (v->page_tokens < 32 || v->page_tokens > 4096 || (v->page_tokens & (v->page_tokens - 1)))
+    return err(SWAN_ERR_INVALID_ARG, "page_tokens must be a power of two in [32, 4096]");
   if (v->sparse_len < 0 || v->buf_len < 0 || v->buf_len > v->buffer_cap || v->buffer_cap < 0 ||
       (v->buffer_cap > 0 && (v->buf_start < 0 || v->buf_start >= v->buffer_cap)))
     return err(SWAN_ERR_INVALID_ARG, "inconsistent buffer or sparse lengths");
@@ -163,6 +163,7 @@ extern "C" swan_status swan_decode_noalloc(const swan_cache_view* v, const void*
     p.range = range;
     p.H_kv = v->n_kv_heads;
     p.H_q = v->n_q_heads;
+    p.blocks_per_page_log2 = __builtin_ctz((unsigned)(v->page_tokens / 32));
     p.k_full_chunks = v->k_active / 8;
     p.k_rem = v->k_active % 8;
     p.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)kHeadDim));

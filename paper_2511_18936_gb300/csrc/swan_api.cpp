@@ -272,8 +272,8 @@ swan_status swan_init(swan_ctx** out, const swan_config* cfg, const float* R_qk,
     return fail(SWAN_ERR_INVALID_ARG, "buffer_cap %d out of [0, %d]", C.buffer_cap, kMaxBufferCap);
   if (C.max_seq < 1) return fail(SWAN_ERR_INVALID_ARG, "max_seq must be >= 1");
   const int P = C.page_tokens ? C.page_tokens : 128;
-  if (P < 32 || P % 32 || P > 4096)
-    return fail(SWAN_ERR_INVALID_ARG, "page_tokens %d must be a multiple of 32 in [32, 4096]", P);
+  if (P < 32 || P > 4096 || (P & (P - 1)))
+    return fail(SWAN_ERR_INVALID_ARG, "page_tokens %d must be a power of two in [32, 4096]", P);
 
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
@@ -498,6 +498,7 @@ swan_status swan_decode(swan_ctx* c, int layer, const void* q, void* out) {
     p.range = range;
     p.H_kv = c->cfg.n_kv_heads;
     p.H_q = c->cfg.n_q_heads;
+    p.blocks_per_page_log2 = __builtin_ctz((unsigned)(c->P / 32));
     p.k_full_chunks = c->k_active / 8;
     p.k_rem = c->k_active % 8;
     p.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)kHeadDim));
@@ -574,8 +575,9 @@ swan_status swan_debug_export(swan_ctx* c, int layer, int what, void* host_dst, 
     if (need == 0) return SWAN_OK;
     const bool isv = what == SWAN_EXPORT_SPARSE_V;
     const int64_t P = c->P;
-    const int64_t voff = isv ? (int64_t)P * c->k_slots * 3 : 0;
-    const int64_t ioff = isv ? (int64_t)P * c->k_slots * 5 : (int64_t)P * c->k_slots * 2;
+    const int64_t blk = 192 * (int64_t)c->k_slots;
+    const int64_t voff = isv ? 96 * (int64_t)c->k_slots : 0;
+    const int64_t ioff = isv ? 160 * (int64_t)c->k_slots : 64 * (int64_t)c->k_slots;
     std::vector<int32_t> pt((size_t)c->units * c->ppu);
     e = cudaMemcpy(pt.data(), c->page_table + (int64_t)layer * c->units * c->ppu, pt.size() * 4,
                    cudaMemcpyDeviceToHost);
@@ -594,12 +596,13 @@ swan_status swan_debug_export(swan_ctx* c, int layer, int what, void* host_dst, 
         for (int64_t sl = 0; sl < P; ++sl) {
           const int64_t t = pg * P + sl;
           if (t >= L.sparse_len) break;
+          const int64_t b0 = (sl / 32) * blk;
           for (int r = 0; r < ks; ++r) {
-            const int64_t rec = (int64_t)(r / 8) * P + sl;
+            const int64_t rec = (int64_t)(r / 8) * 32 + (sl % 32);
             const size_t o = ((size_t)u * L.sparse_len + t) * ks + r;
-            idx_dst[o] = page[ioff + rec * 8 + (r % 8)];
+            idx_dst[o] = page[b0 + ioff + rec * 8 + (r % 8)];
             uint16_t v;
-            std::memcpy(&v, page.data() + voff + rec * 16 + (r % 8) * 2, 2);
+            std::memcpy(&v, page.data() + b0 + voff + rec * 16 + (r % 8) * 2, 2);
             val_dst[o] = v;
           }
         }

@@ -2,20 +2,22 @@
 //
 // Sparse cache page layout (Section 5.1's values + 8-bit indices, arranged
 // for 128-bit coalesced loads on sm_103a).  A page holds P tokens (P a
-// multiple of 32) of one (layer, batch, kv-head) unit.  Each vector's kept
-// entries are grouped in chunks of 8, in stored (decreasing magnitude) order;
-// chunk c of token t is a 16-byte record of 8 fp16 values and an 8-byte
-// record of 8 uint8 indices:
+// multiple of 32) of one (layer, batch, kv-head) unit, as P/32 consecutive
+// blocks of 32 tokens.  Each vector's kept entries are grouped in chunks of
+// 8, in stored (decreasing magnitude) order; chunk c of token t is a 16-byte
+// record of 8 fp16 values and an 8-byte record of 8 uint8 indices.  A block
+// (192 * k_slots bytes) is
 //
-//   [K values  : k_slots/8 chunks][P tokens][8 x fp16]   (16 B per record)
-//   [K indices : k_slots/8 chunks][P tokens][8 x uint8]  ( 8 B per record)
-//   [V values  : same as K values]
-//   [V indices : same as K indices]
+//   [K values  : k_slots/8 chunks][32 tokens][8 x fp16]   at 0
+//   [K indices : k_slots/8 chunks][32 tokens][8 x uint8]  at 64 * k_slots
+//   [V values  : same shape as K values]                  at 96 * k_slots
+//   [V indices : same shape as K indices]                 at 160 * k_slots
 //
-// A warp that handles 32 consecutive tokens (one per lane) reads chunk c of
-// all of them as one contiguous 512-byte run (values) and one 256-byte run
-// (indices).  A runtime keep count k_active <= k_store reads only the first
-// ceil(k_active / 8) chunks: a contiguous prefix of each region.
+// A warp that handles the 32 tokens of a block (one per lane) reads chunk c
+// of all of them as one contiguous 512-byte run (values) and one 256-byte run
+// (indices), at compile-time offsets from the region base.  A runtime keep
+// count k_active <= k_store reads only the first ceil(k_active / 8) chunks:
+// a contiguous prefix of each region.
 #pragma once
 
 #include <cuda_fp16.h>
@@ -45,9 +47,11 @@ struct CacheGeom {
   int k_slots;               // k_store rounded up to 8
   int k_store;
   int64_t page_bytes;        // P * k_slots * 6
-  __device__ __host__ int64_t kidx_off() const { return (int64_t)P * k_slots * 2; }
-  __device__ __host__ int64_t vval_off() const { return (int64_t)P * k_slots * 3; }
-  __device__ __host__ int64_t vidx_off() const { return (int64_t)P * k_slots * 5; }
+  // offsets inside a 32-token block
+  __device__ __host__ int block_bytes() const { return 192 * k_slots; }
+  __device__ __host__ int kidx_off() const { return 64 * k_slots; }
+  __device__ __host__ int vval_off() const { return 96 * k_slots; }
+  __device__ __host__ int vidx_off() const { return 160 * k_slots; }
 };
 
 // Rotate T new tokens per unit, then either write them to the ring buffer or
@@ -101,6 +105,7 @@ struct DecodeParams {
   int64_t n_sg, N_g;       // sparse groups per unit; groups per unit
   int64_t total_groups, range;
   int H_kv, H_q;
+  int blocks_per_page_log2; // log2(P / 32)
   int k_full_chunks;       // k_active / 8
   int k_rem;               // k_active % 8
   float scale_log2;        // log2(e) / sqrt(d)

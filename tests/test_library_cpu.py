@@ -60,6 +60,8 @@ def _cfg(**kw):
     (dict(buffer_cap=5000), swan.ERR_INVALID_ARG),
     (dict(max_seq=0), swan.ERR_INVALID_ARG),
     (dict(page_tokens=48), swan.ERR_INVALID_ARG),
+    (dict(page_tokens=96), swan.ERR_INVALID_ARG),
+    (dict(page_tokens=8192), swan.ERR_INVALID_ARG),
     (dict(num_layers=0), swan.ERR_INVALID_ARG),
     (dict(batch=0), swan.ERR_INVALID_ARG),
 ])

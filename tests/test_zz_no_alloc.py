@@ -23,26 +23,31 @@ D = 128
 
 def _pages_from_export(idx_k, val_k, idx_v, val_v, P, k_slots, perm):
     """Lay exported sparse vectors out as pages (the layout the header
-    documents); page slots follow the permutation ``perm``."""
+    documents: pages of P/32 blocks of 32 tokens); page slots follow the
+    permutation ``perm``."""
     units, L, ks = idx_k.shape
     ppu = max(1, -(-L // P))
     page_bytes = P * k_slots * 6
+    block_bytes = 192 * k_slots
     pool = np.zeros((units * ppu, page_bytes), np.uint8)
     table = np.empty(units * ppu, np.int32)
     for u in range(units):
         for pg in range(ppu):
             phys = perm[u * ppu + pg]
             table[u * ppu + pg] = phys
-            page = pool[phys]
-            for region, (idx, val) in enumerate(((idx_k, val_k), (idx_v, val_v))):
-                voff = region * P * k_slots * 3
-                ioff = voff + P * k_slots * 2
-                vals = page[voff:voff + P * k_slots * 2].view(np.uint16).reshape(k_slots // 8, P, 8)
-                inds = page[ioff:ioff + P * k_slots].reshape(k_slots // 8, P, 8)
-                t0, t1 = pg * P, min(L, pg * P + P)
-                for r in range(ks):
-                    vals[r // 8, :t1 - t0, r % 8] = val[u, t0:t1, r].view(np.uint16)
-                    inds[r // 8, :t1 - t0, r % 8] = idx[u, t0:t1, r]
+            for q in range(P // 32):
+                blk = pool[phys, q * block_bytes:(q + 1) * block_bytes]
+                t0 = pg * P + q * 32
+                t1 = min(L, t0 + 32)
+                if t1 <= t0:
+                    continue
+                for voff, idx, val in ((0, idx_k, val_k), (96 * k_slots, idx_v, val_v)):
+                    ioff = voff + 64 * k_slots
+                    vals = blk[voff:voff + 64 * k_slots].view(np.uint16).reshape(k_slots // 8, 32, 8)
+                    inds = blk[ioff:ioff + 32 * k_slots].reshape(k_slots // 8, 32, 8)
+                    for r in range(ks):
+                        vals[r // 8, :t1 - t0, r % 8] = val[u, t0:t1, r].view(np.uint16)
+                        inds[r // 8, :t1 - t0, r % 8] = idx[u, t0:t1, r]
     return pool, table, ppu
 
 

@@ -188,6 +188,68 @@ __global__ void __launch_bounds__(kThreads, 1) append_kernel(AppendParams p) {
   }
 }
 
+// Small appends (decode steps): one CTA per (kv head, K or V).  Phase 1
+// prunes the `evict_old` oldest buffered vectors of every sequence out of the
+// ring; after a barrier, phase 2 rotates the new vectors one per warp (lane l
+// computes coordinates 4l..4l+3 from R in shared memory, in the same fp32
+// order as append_kernel) and either prunes them or writes them to the ring.
+// Ring slots freed in phase 1 are reused in phase 2 only after the barrier.
+__global__ void __launch_bounds__(kThreads) append_small_kernel(AppendParams p, int evict_old) {
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  float* Rs = reinterpret_cast<float*>(smem_raw);
+  const int kind = blockIdx.y;
+  const int h = blockIdx.x;
+  const float* R = (kind ? p.R_vo : p.R_qk) + (size_t)h * kHeadDim * kHeadDim;
+  const __half* X = kind ? p.v_new : p.k_new;
+  __half* ring = kind ? p.ring_v : p.ring_k;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+  for (int i = threadIdx.x; i < kHeadDim * kHeadDim / 4; i += kThreads)
+    reinterpret_cast<float4*>(Rs)[i] = __ldg(reinterpret_cast<const float4*>(R) + i);
+
+  // phase 1: evict the oldest buffered vectors (sparse positions L_s + i)
+  for (int item = warp; item < p.B * evict_old; item += kWarpsPerCta) {
+    const int b = item / evict_old, i = item % evict_old;
+    const int64_t unit = (int64_t)b * p.H + h;
+    const int slot = (p.buf_start + i) % p.cap;
+    const uint2 raw = __ldg(reinterpret_cast<const uint2*>(ring + (unit * p.cap + slot) * kHeadDim) + lane);
+    warp_prune_store(raw, lane, kind, unit, p.sparse_len + i, p.geom, p.status);
+  }
+  __syncthreads();
+
+  // phase 2: the new vectors
+  for (int item = warp; item < p.B * p.T; item += kWarpsPerCta) {
+    const int b = item / p.T, j = item % p.T;
+    const int64_t unit = (int64_t)b * p.H + h;
+    const uint2 xw = __ldg(reinterpret_cast<const uint2*>(X + ((unit * p.T) + j) * kHeadDim) + lane);
+    const float2 x01 = __half22float2(*reinterpret_cast<const __half2*>(&xw.x));
+    const float2 x23 = __half22float2(*reinterpret_cast<const __half2*>(&xw.y));
+    const float xs[4] = {x01.x, x01.y, x23.x, x23.y};
+    float acc[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll 8
+    for (int i = 0; i < kHeadDim; ++i) {
+      const float xi = __shfl_sync(0xffffffffu, xs[i & 3], i >> 2);
+      const float4 r = reinterpret_cast<const float4*>(Rs + i * kHeadDim)[lane];
+      acc[0] = fmaf(xi, r.x, acc[0]);
+      acc[1] = fmaf(xi, r.y, acc[1]);
+      acc[2] = fmaf(xi, r.z, acc[2]);
+      acc[3] = fmaf(xi, r.w, acc[3]);
+    }
+    uint2 yw;
+    yw.x = (uint32_t)__half_as_ushort(__float2half_rn(acc[0])) |
+           ((uint32_t)__half_as_ushort(__float2half_rn(acc[1])) << 16);
+    yw.y = (uint32_t)__half_as_ushort(__float2half_rn(acc[2])) |
+           ((uint32_t)__half_as_ushort(__float2half_rn(acc[3])) << 16);
+    const int64_t pos = (int64_t)p.n_b + j;
+    if (pos < p.evict) {
+      warp_prune_store(yw, lane, kind, unit, p.sparse_len + pos, p.geom, p.status);
+    } else {
+      const int slot = (int)((p.buf_start + pos) % p.cap);
+      reinterpret_cast<uint2*>(ring + (unit * p.cap + slot) * kHeadDim)[lane] = yw;
+    }
+  }
+}
+
 // One warp per (unit, buffered token, K or V): read the ring row and prune.
 __global__ void __launch_bounds__(kThreads) prune_ring_kernel(PruneRingParams p) {
   const int lane = threadIdx.x & 31;
@@ -230,6 +292,19 @@ cudaError_t launch_append(const AppendParams& p, cudaStream_t s) {
   const int64_t nvec = (int64_t)p.B * p.T;
   dim3 grid((unsigned)((nvec + kThreads - 1) / kThreads), (unsigned)p.H, 2);
   append_kernel<<<grid, kThreads, kAppendSmem, s>>>(p);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_append_small(const AppendParams& p, int evict_old, cudaStream_t s) {
+  static bool attr_set = false;
+  constexpr size_t smem = 128 * 128 * sizeof(float);
+  if (!attr_set) {
+    cudaError_t e = cudaFuncSetAttribute(append_small_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)smem);
+    if (e != cudaSuccess) return e;
+    attr_set = true;
+  }
+  append_small_kernel<<<dim3((unsigned)p.H, 2), kThreads, smem, s>>>(p, evict_old);
   return cudaGetLastError();
 }
 

@@ -410,27 +410,89 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
         dst[1] = L;
       }
     }
+
+    // ---- the last CTA to finish a segment of unit u merges the unit's
+    // partials, normalises, rotates back and writes the output (the
+    // arrival counter resets itself for the next decode; nothing waits)
+    __threadfence();
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      const int64_t c0 = (u * p.N_g) / p.range, c1 = ((u + 1) * p.N_g - 1) / p.range;
+      const int old = atomicAdd(p.counters + u, 1);
+      const bool last = old == (int)(c1 - c0);
+      if (last) p.counters[u] = 0;
+      red_m[0] = last ? 1.f : 0.f;
+    }
+    __syncthreads();
+    if (red_m[0] != 0.f) {
+      __threadfence();
+      const int64_t c0 = (u * p.N_g) / p.range, c1 = ((u + 1) * p.N_g - 1) / p.range;
+      float* o_hat = qrep;  // [G][128]; q' of this unit is no longer needed
+      for (int o = threadIdx.x; o < G * kHeadDim; o += kThreads) {
+        const int gh = o / kHeadDim, dd = o % kHeadDim;
+        float M = -INFINITY;
+        for (int64_t c = c0; c <= c1; ++c)
+          M = fmaxf(M, __ldcg(p.partials + ((size_t)(c + u) * G + gh) * (kHeadDim + 2)));
+        float L = 0.f, A = 0.f;
+        for (int64_t c = c0; c <= c1; ++c) {
+          const float* part = p.partials + ((size_t)(c + u) * G + gh) * (kHeadDim + 2);
+          const float mc = __ldcg(part);
+          const float w = (mc == -INFINITY) ? 0.f : exp2f(mc - M);
+          L = fmaf(w, __ldcg(part + 1), L);
+          A = fmaf(w, __ldcg(part + 2 + dd), A);
+        }
+        o_hat[o] = (L > 0.f) ? A / L : 0.f;
+      }
+      __syncthreads();
+      const float* RT = p.R_voT + (size_t)h * kHeadDim * kHeadDim;
+      for (int o = threadIdx.x; o < G * kHeadDim; o += kThreads) {
+        const int gh = o / kHeadDim, i = o % kHeadDim;
+        const float* oh = o_hat + gh * kHeadDim;
+        float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
+#pragma unroll 8
+        for (int j = 0; j < kHeadDim; j += 4) {
+          a0 = fmaf(oh[j + 0], __ldg(RT + (j + 0) * kHeadDim + i), a0);
+          a1 = fmaf(oh[j + 1], __ldg(RT + (j + 1) * kHeadDim + i), a1);
+          a2 = fmaf(oh[j + 2], __ldg(RT + (j + 2) * kHeadDim + i), a2);
+          a3 = fmaf(oh[j + 3], __ldg(RT + (j + 3) * kHeadDim + i), a3);
+        }
+        p.out[((b * p.H_q) + h * G + gh) * kHeadDim + i] = __float2half_rn((a0 + a1) + (a2 + a3));
+      }
+    }
   }
 }
 
-// q' = q R_qk for every (batch, query head): one CTA per vector, thread j
-// computes coordinate j (coalesced rows of R).
-__global__ void __launch_bounds__(kHeadDim) rotate_q_kernel(RotateQParams p) {
-  __shared__ float qs[kHeadDim];
-  const int64_t bq = blockIdx.x;
-  const int hq = (int)(bq % p.H_q);
-  const int h = hq / p.G;
-  const int t = threadIdx.x;
-  qs[t] = __half2float(p.q[bq * kHeadDim + t]);
-  __syncthreads();
+// q' = q R_qk: one CTA per kv head with R in shared memory, one warp per
+// query vector of that head (all batches, all G heads of the group); lane l
+// computes coordinates 4l..4l+3 in a sequential fp32 FMA chain.
+__global__ void __launch_bounds__(kThreads) rotate_q_kernel(RotateQParams p, int B) {
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  float* Rs = reinterpret_cast<float*>(smem_raw);
+  const int h = blockIdx.x;
   const float* R = p.R_qk + (size_t)h * kHeadDim * kHeadDim;
-  float a0 = 0.f, a1 = 0.f;
+  for (int i = threadIdx.x; i < kHeadDim * kHeadDim / 4; i += kThreads)
+    reinterpret_cast<float4*>(Rs)[i] = __ldg(reinterpret_cast<const float4*>(R) + i);
+  __syncthreads();
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  for (int item = warp; item < B * p.G; item += kWarpsPerCta) {
+    const int b = item / p.G, gh = item % p.G;
+    const int64_t bq = (int64_t)b * p.H_q + h * p.G + gh;
+    const uint2 xw = __ldg(reinterpret_cast<const uint2*>(p.q + bq * kHeadDim) + lane);
+    const float2 x01 = __half22float2(*reinterpret_cast<const __half2*>(&xw.x));
+    const float2 x23 = __half22float2(*reinterpret_cast<const __half2*>(&xw.y));
+    const float xs[4] = {x01.x, x01.y, x23.x, x23.y};
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll 8
-  for (int i = 0; i < kHeadDim; i += 2) {
-    a0 = fmaf(qs[i], __ldg(R + i * kHeadDim + t), a0);
-    a1 = fmaf(qs[i + 1], __ldg(R + (i + 1) * kHeadDim + t), a1);
+    for (int i = 0; i < kHeadDim; ++i) {
+      const float xi = __shfl_sync(0xffffffffu, xs[i & 3], i >> 2);
+      const float4 r = reinterpret_cast<const float4*>(Rs + i * kHeadDim)[lane];
+      acc.x = fmaf(xi, r.x, acc.x);
+      acc.y = fmaf(xi, r.y, acc.y);
+      acc.z = fmaf(xi, r.z, acc.z);
+      acc.w = fmaf(xi, r.w, acc.w);
+    }
+    reinterpret_cast<float4*>(p.qprime + bq * kHeadDim)[lane] = acc;
   }
-  p.qprime[bq * kHeadDim + t] = a0 + a1;
 }
 
 // Merge the partials of one (batch, query head), normalise, rotate back by
@@ -523,7 +585,15 @@ cudaError_t launch_decode(const DecodeParams& p, int G, int k_slots, int grid, c
 }
 
 cudaError_t launch_rotate_q(const RotateQParams& p, int B, cudaStream_t s) {
-  rotate_q_kernel<<<(unsigned)((int64_t)B * p.H_q), kHeadDim, 0, s>>>(p);
+  static bool attr_set = false;
+  constexpr size_t smem = kHeadDim * kHeadDim * sizeof(float);
+  if (!attr_set) {
+    cudaError_t e =
+        cudaFuncSetAttribute(rotate_q_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    attr_set = true;
+  }
+  rotate_q_kernel<<<(unsigned)(p.H_q / p.G), kThreads, smem, s>>>(p, B);
   return cudaGetLastError();
 }
 

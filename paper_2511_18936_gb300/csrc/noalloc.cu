@@ -23,10 +23,12 @@ constexpr int kNoallocMaxQ = 1024;         // batch * n_q_heads
 constexpr int kNoallocMaxSlots = 2048;     // (decode CTAs + units) * G partials
 constexpr size_t kQFloats = (size_t)kNoallocMaxQ * kHeadDim;
 constexpr size_t kPartFloats = (size_t)kNoallocMaxSlots * (kHeadDim + 2);
+constexpr size_t kCounterFloats = kNoallocMaxSlots;  // per-unit arrival counters (int)
 constexpr size_t kStatusFloats = 64;       // 256 bytes, the status word first
 
-// Layout: [rotated queries][split partials][status word]
-__device__ __align__(256) float g_noalloc_scratch[kQFloats + kPartFloats + kStatusFloats];
+// Layout: [rotated queries][split partials][counters][status word]
+__device__ __align__(256) float
+    g_noalloc_scratch[kQFloats + kPartFloats + kCounterFloats + kStatusFloats];
 
 constexpr int kMaxDevices = 64;
 struct DeviceSetup {
@@ -127,10 +129,13 @@ extern "C" swan_status swan_decode_noalloc(const swan_cache_view* v, const void*
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   float* qprime = ds->scratch;
   float* partials = ds->scratch + kQFloats;
-  unsigned* status = reinterpret_cast<unsigned*>(ds->scratch + kQFloats + kPartFloats);
-  // the status word must start at zero; the rest is fully written before use
-  if (cudaMemsetAsync(status, 0, sizeof(unsigned), s) != cudaSuccess)
-    return err(SWAN_ERR_CUDA, "cudaMemsetAsync of the status word failed");
+  int* counters = reinterpret_cast<int*>(ds->scratch + kQFloats + kPartFloats);
+  unsigned* status = reinterpret_cast<unsigned*>(ds->scratch + kQFloats + kPartFloats + kCounterFloats);
+  // the counters and the status word must start at zero; the rest is fully
+  // written before use
+  if (cudaMemsetAsync(counters, 0, (size_t)units * sizeof(int), s) != cudaSuccess ||
+      cudaMemsetAsync(status, 0, sizeof(unsigned), s) != cudaSuccess)
+    return err(SWAN_ERR_CUDA, "cudaMemsetAsync of the counters failed");
 
   RotateQParams rq{};
   rq.q = static_cast<const __half*>(q);
@@ -168,9 +173,13 @@ extern "C" swan_status swan_decode_noalloc(const swan_cache_view* v, const void*
     p.k_rem = v->k_active % 8;
     p.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)kHeadDim));
     p.partials = partials;
+    p.counters = counters;
+    p.R_voT = v->R_vo_t;
+    p.out = static_cast<__half*>(out);
     p.status = status;
     if (launch_decode(p, G, v->k_slots, (int)grid, s) != cudaSuccess)
       return err(SWAN_ERR_CUDA, "decode launch failed");
+    return SWAN_OK;
   }
 
   CombineParams cp{};

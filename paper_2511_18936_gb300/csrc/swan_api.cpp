@@ -69,6 +69,7 @@ struct swan_ctx {
   __half* ring_v = nullptr;
   float* qprime = nullptr;
   float* partials = nullptr;
+  int* counters = nullptr;  // per-unit arrival counters of the fused combine
   unsigned* status = nullptr;
   int64_t device_bytes = 0;
 
@@ -85,6 +86,7 @@ struct swan_ctx {
 namespace {
 
 constexpr int kMaxBufferCap = 4096;
+constexpr int64_t kSmallAppendVectors = 256;  // batch * T per kv head
 constexpr size_t kMaxEventPairs = 4096;
 
 void free_all(swan_ctx* c) {
@@ -97,6 +99,7 @@ void free_all(swan_ctx* c) {
   cudaFree(c->ring_v);
   cudaFree(c->qprime);
   cudaFree(c->partials);
+  cudaFree(c->counters);
   cudaFree(c->status);
   for (auto& e : c->ev_free) {
     cudaEventDestroy(e.start);
@@ -329,6 +332,7 @@ swan_status swan_init(swan_ctx** out, const swan_config* cfg, const float* R_qk,
   if (s == SWAN_OK) s = dev_alloc(c, (void**)&c->ring_v, ring_elems * sizeof(__half), "value ring");
   if (s == SWAN_OK) s = dev_alloc(c, (void**)&c->qprime, q_elems * sizeof(float), "rotated queries");
   if (s == SWAN_OK) s = dev_alloc(c, (void**)&c->partials, part_elems * sizeof(float), "split partials");
+  if (s == SWAN_OK) s = dev_alloc(c, (void**)&c->counters, (size_t)c->units * sizeof(int), "counters");
   if (s == SWAN_OK) s = dev_alloc(c, (void**)&c->status, sizeof(unsigned), "status word");
   if (s != SWAN_OK) {
     free_all(c);
@@ -350,6 +354,7 @@ swan_status swan_init(swan_ctx** out, const swan_config* cfg, const float* R_qk,
   if (e == cudaSuccess) e = cudaMemsetAsync(c->pool, 0, (size_t)c->num_pages * (size_t)c->page_bytes, st);
   if (e == cudaSuccess) e = cudaMemsetAsync(c->ring_k, 0, ring_elems * sizeof(__half), st);
   if (e == cudaSuccess) e = cudaMemsetAsync(c->ring_v, 0, ring_elems * sizeof(__half), st);
+  if (e == cudaSuccess) e = cudaMemsetAsync(c->counters, 0, (size_t)c->units * sizeof(int), st);
   if (e == cudaSuccess) e = cudaMemsetAsync(c->status, 0, sizeof(unsigned), st);
   if (e == cudaSuccess) e = cudaStreamSynchronize(st);  // pt is a pageable host vector
   if (e != cudaSuccess) {
@@ -402,12 +407,18 @@ swan_status swan_append(swan_ctx* c, int layer, const void* k_new, const void* v
   const int64_t evict = std::max<int64_t>(0, (int64_t)L.buf_count + T - cap);
   const int old_evict = (int)std::min<int64_t>(evict, L.buf_count);
 
-  // 1) prune the evicted buffered tokens (they leave the ring first, so the
-  //    new tokens may reuse their slots)
   const int64_t sparse_before = L.sparse_len;
   const int start_before = L.buf_start;
   const int count_before = L.buf_count;
-  if ((s = prune_from_ring(c, layer, old_evict)) != SWAN_OK) return s;
+  // Decode-step appends (few vectors per head) run as one launch that evicts
+  // and inserts; bulk appends as a pruning launch for the evicted buffered
+  // tokens followed by the rotation launch.
+  const bool small = (int64_t)c->cfg.batch * T <= kSmallAppendVectors &&
+                     (int64_t)c->cfg.batch * old_evict <= kSmallAppendVectors;
+
+  // 1) prune the evicted buffered tokens (they leave the ring first, so the
+  //    new tokens may reuse their slots)
+  if (!small && (s = prune_from_ring(c, layer, old_evict)) != SWAN_OK) return s;
 
   // 2) rotate the new tokens; those before `evict` are pruned directly, the
   //    rest land in the ring after the surviving buffered tokens
@@ -428,7 +439,11 @@ swan_status swan_append(swan_ctx* c, int layer, const void* k_new, const void* v
   p.sparse_len = sparse_before;
   p.geom = geom_for(c, layer);
   p.status = c->status;
-  s = launch(c, SWAN_KERNEL_APPEND, "append kernel", [&] { return launch_append(p, c->stream); });
+  if (small)
+    s = launch(c, SWAN_KERNEL_APPEND, "append_small kernel",
+               [&] { return launch_append_small(p, old_evict, c->stream); });
+  else
+    s = launch(c, SWAN_KERNEL_APPEND, "append kernel", [&] { return launch_append(p, c->stream); });
   if (s != SWAN_OK) return s;
 
   L.sparse_len = sparse_before + evict;
@@ -503,11 +518,15 @@ swan_status swan_decode(swan_ctx* c, int layer, const void* q, void* out) {
     p.k_rem = c->k_active % 8;
     p.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)kHeadDim));
     p.partials = c->partials;
+    p.counters = c->counters;
+    p.R_voT = c->R_voT + (size_t)layer * c->cfg.n_kv_heads * kHeadDim * kHeadDim;
+    p.out = static_cast<__half*>(out);
     p.status = c->status;
-    s = launch(c, SWAN_KERNEL_DECODE, "decode kernel",
-               [&] { return launch_decode(p, G, c->k_slots, (int)grid, c->stream); });
-    if (s != SWAN_OK) return s;
+    // the split combine and the rotate-back run inside the decode kernel
+    return launch(c, SWAN_KERNEL_DECODE, "decode kernel",
+                  [&] { return launch_decode(p, G, c->k_slots, (int)grid, c->stream); });
   }
+  // empty cache: the combine kernel writes zeros
 
   CombineParams cp{};
   cp.partials = c->partials;

@@ -110,6 +110,9 @@ struct DecodeParams {
   int k_rem;               // k_active % 8
   float scale_log2;        // log2(e) / sqrt(d)
   float* partials;         // [pairs][G][d + 2]
+  int* counters;           // [units] arrival counters, zero between decodes
+  const float* R_voT;      // this layer: [H_kv][d][d], transposed
+  __half* out;             // [B][H_q][d]
   unsigned* status;
 };
 
@@ -123,6 +126,9 @@ struct CombineParams {
 
 // Launchers (return the launch error, if any).
 cudaError_t launch_append(const AppendParams& p, cudaStream_t s);
+// Eviction of `evict_old` buffered tokens and insertion of T new ones in one
+// launch; for small batch * T (decode steps).
+cudaError_t launch_append_small(const AppendParams& p, int evict_old, cudaStream_t s);
 cudaError_t launch_prune_ring(const PruneRingParams& p, cudaStream_t s);
 cudaError_t launch_rotate_q(const RotateQParams& p, int B, cudaStream_t s);
 cudaError_t launch_decode(const DecodeParams& p, int G, int k_slots, int grid, cudaStream_t s);

@@ -133,6 +133,37 @@ def test_direct_and_buffered_pruning_agree():
     b.close()
 
 
+def test_small_and_bulk_append_paths_agree():
+    """One bulk append of T tokens per sequence (above the fused small-append
+    limit) and the same tokens appended one per call (evicting one buffered
+    vector each time) leave bit-identical caches."""
+    import torch
+
+    from paper_2511_18936_gb300 import swan
+    B, H, T, cap = 4, 2, 150, 40
+    R, Rv = _rot(H, 13), _rot(H, 13, synth.T_R_VO)
+    k, v = _kv(B, H, T, seed=14)
+    Rt, Rvt = torch.from_numpy(R)[None].cuda(), torch.from_numpy(Rv)[None].cuda()
+    kw = dict(num_layers=1, batch=B, n_q_heads=H, n_kv_heads=H, k_store=40, buffer_cap=cap,
+              max_seq=T, page_tokens=32)
+    a = swan.Context(Rt, Rvt, **kw)
+    b = swan.Context(Rt, Rvt, **kw)
+    kt, vt = torch.from_numpy(k).cuda(), torch.from_numpy(v).cuda()
+    a.append(0, kt, vt)
+    for t in range(T):
+        b.append(0, kt[:, :, t:t + 1].contiguous(), vt[:, :, t:t + 1].contiguous())
+    for which in ("k", "v"):
+        ia, va = a.export_sparse(0, which)
+        ib, vb = b.export_sparse(0, which)
+        assert np.array_equal(ia, ib) and np.array_equal(va.view(np.uint16), vb.view(np.uint16))
+        assert np.array_equal(a.export_buffer(0, which).view(np.uint16),
+                              b.export_buffer(0, which).view(np.uint16))
+    a.check()
+    b.check()
+    a.close()
+    b.close()
+
+
 def test_index_parity_end_to_end_with_near_tie_exemption():
     B, H = 2, 2
     R, Rv = _rot(H, 11), _rot(H, 11, synth.T_R_VO)

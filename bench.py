@@ -38,12 +38,23 @@ import numpy as np  # noqa: E402
 
 D = 128
 WORKLOADS = {
+    "latency-1k": dict(B=1, H_q=1, H_kv=1, L_s=1024, n_b=64, k=64, k_store=64, l2_flush=True,
+                       desc="one head, batch 1, d 128, 1024 sparse + 64 dense-buffer tokens, k 64 "
+                            "(L2-resident: latency)"),
     "llama2-7b-layer-32k": dict(B=16, H_q=32, H_kv=32, L_s=32768, n_b=128, k=64, k_store=64,
                                 desc="Llama-2-7B-shaped layer: batch 16, 32 MHA heads, d 128, "
                                      "32768 sparse + 128 dense-buffer tokens, k 64"),
     "gqa-131k": dict(B=4, H_q=32, H_kv=8, L_s=130944, n_b=128, k=56, k_store=56,
                      desc="Llama-3-8B-shaped GQA layer: batch 4, 32 q / 8 kv heads, d 128, "
                           "130944 sparse + 128 dense-buffer tokens (131072 ctx), k 56"),
+    "ksweep-32k": dict(B=16, H_q=32, H_kv=32, L_s=32768, n_b=128, k=64, k_store=128,
+                       desc="Llama-2-7B-shaped layer at 32k with k_store 128, decoded at a runtime "
+                            "keep count k (--k-active)"),
+    "stack-32x8k": dict(kind="stack", B=8, H_q=32, H_kv=32, layers=32, prefix=8192, n_b=128,
+                        flush_every=128, max_steps=256, k=64, k_store=64,
+                        desc="32-layer Llama-2-7B-shaped KV stack, batch 8, 8192-token prefix "
+                             "compressed by one append per layer, decode steps appending one token "
+                             "per layer, buffers flushed every 128 steps, k 64"),
 }
 METRIC = "decode-attention KV-tokens/s and achieved HBM GB/s (% of 8 TB/s) at 32k ctx"
 NOMINAL_HBM_GBS = 8000.0
@@ -135,16 +146,17 @@ def oracle_sample(wl, n_units: int, seed: int = 0):
     import oracle
     from paper_2511_18936_gb300 import synth
     G = wl["H_q"] // wl["H_kv"]
-    L = wl["L_s"] + wl["n_b"]
+    L_s = wl.get("L_s", wl.get("prefix"))
+    L = L_s + wl["n_b"]
     states = []
     for u in range(n_units):
         R = synth.rotations(1, D, seed=seed, workload=7, layer=0, tensor_id=synth.T_R_QK, )
         k = synth.lowrank_kv(1, 1, L + 64, D, seed, 7, u, synth.T_K)
         v = synth.lowrank_kv(1, 1, L + 64, D, seed, 7, u, synth.T_V)
         st = oracle.SwanOracle(R, batch=1, n_q_heads=G, k_store=wl["k_store"], buffer_cap=wl["n_b"])
-        st.append(k[:, :, :wl["L_s"]], v[:, :, :wl["L_s"]])
+        st.append(k[:, :, :L_s], v[:, :, :L_s])
         st.flush()
-        st.append(k[:, :, wl["L_s"]:L], v[:, :, wl["L_s"]:L])
+        st.append(k[:, :, L_s:L], v[:, :, L_s:L])
         st.set_k(wl["k"])
         q = synth.gaussian_fp16((1, G, D), seed, 7, u, synth.T_Q)
         states.append((st, k[:, :, L:], v[:, :, L:], q))
@@ -212,46 +224,153 @@ def cpu_baseline_leg(wl, budget_s: float = 15.0):
 # The CUDA path
 # ---------------------------------------------------------------------------
 
+class LayerRun:
+    """One attention layer (the 1-head, 32k, GQA-131k and k-sweep workloads):
+    prefill the context in one append, then per step append one token per
+    sequence (the buffer is full, so one vector is evicted and pruned) and
+    decode."""
+
+    def __init__(self, wl, dev, stream, seed, steps_total):
+        import torch
+
+        from paper_2511_18936_gb300 import swan, synth
+        self.wl = wl
+        B, H_q, H_kv, L_s, n_b = wl["B"], wl["H_q"], wl["H_kv"], wl["L_s"], wl["n_b"]
+        self.layers = 1
+        self.max_seq = L_s + n_b + steps_total + 8
+        with torch.cuda.stream(stream):
+            R = torch.from_numpy(synth.rotations(H_kv, D, seed=seed, workload=1, layer=0))[None].to(dev)
+            self.ctx = swan.Context(R, num_layers=1, batch=B, n_q_heads=H_q, n_kv_heads=H_kv,
+                                    k_store=wl["k_store"], buffer_cap=n_b, max_seq=self.max_seq,
+                                    stream=stream)
+            kk = synth.torch_lowrank_kv(B, H_kv, L_s + n_b, D, seed, synth.T_K, dev)
+            vv = synth.torch_lowrank_kv(B, H_kv, L_s + n_b, D, seed, synth.T_V, dev)
+            self.ctx.append(0, kk, vv)
+            del kk, vv
+            k_new = synth.torch_lowrank_kv(B, H_kv, steps_total, D, seed, synth.T_NEWK, dev)
+            v_new = synth.torch_lowrank_kv(B, H_kv, steps_total, D, seed, synth.T_NEWV, dev)
+            self.k_steps = [k_new[:, :, i:i + 1].contiguous() for i in range(steps_total)]
+            self.v_steps = [v_new[:, :, i:i + 1].contiguous() for i in range(steps_total)]
+            del k_new, v_new
+            self.qs = synth.torch_gaussian_fp16((steps_total, B, H_q, D), seed, synth.T_Q, dev)
+            self.out = torch.empty((B, H_q, D), dtype=torch.float16, device=dev)
+            self.ctx.set_k(wl["k"])
+        stream.synchronize()
+        self.ctx.check()
+
+    def step(self, i):
+        self.ctx.append(0, self.k_steps[i], self.v_steps[i], 1)
+        self.ctx.decode(0, self.qs[i], self.out)
+
+    def context_after(self, i):
+        """(sparse, buffer) tokens attended by the decode of step i."""
+        wl = self.wl
+        return wl["L_s"] + i + 1, wl["n_b"]
+
+    def host_inputs(self, i):
+        return [self.k_steps[i], self.v_steps[i], self.qs[i]]
+
+    def step_with(self, dev_inputs):
+        dk, dv, dq = dev_inputs
+        self.ctx.append(0, dk, dv, 1)
+        self.ctx.decode(0, dq, self.out)
+        return [self.out]
+
+
+class StackRun:
+    """A 32-layer KV stack: the prefix of every layer compressed by one
+    append (timed separately), flushed, then decode steps that append one
+    token per layer and decode it, with every layer's buffer flushed after
+    each 128 steps."""
+
+    def __init__(self, wl, dev, stream, seed, steps_total):
+        import torch
+
+        from paper_2511_18936_gb300 import swan, synth
+        self.wl = wl
+        B, H, Lyr, pre, cap = wl["B"], wl["H_q"], wl["layers"], wl["prefix"], wl["n_b"]
+        self.layers = Lyr
+        self.max_seq = pre + steps_total + 8
+        self.flush_every = wl["flush_every"]
+        R = np.stack([synth.rotations(H, D, seed=seed, workload=4, layer=l) for l in range(Lyr)])
+        with torch.cuda.stream(stream):
+            Rt = torch.from_numpy(R).to(dev)
+            self.ctx = swan.Context(Rt, num_layers=Lyr, batch=B, n_q_heads=H, n_kv_heads=H,
+                                    k_store=wl["k_store"], buffer_cap=cap, max_seq=self.max_seq,
+                                    stream=stream)
+            self.ctx.set_k(wl["k"])
+        stream.synchronize()
+        # prefix: one append per layer (plain Gaussian K/V), timed on the stream
+        ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        self.prefix_ms = 0.0
+        for l in range(Lyr):
+            with torch.cuda.stream(stream):
+                kk = synth.torch_gaussian_fp16((B, H, pre, D), seed, synth.T_K, dev, 1.0, l)
+                vv = synth.torch_gaussian_fp16((B, H, pre, D), seed, synth.T_V, dev, 1.0, l)
+                ev0.record(stream)
+                self.ctx.append(l, kk, vv)
+                self.ctx.flush(l)
+                ev1.record(stream)
+            stream.synchronize()
+            self.prefix_ms += ev0.elapsed_time(ev1)
+            del kk, vv
+        with torch.cuda.stream(stream):
+            kn = synth.torch_gaussian_fp16((Lyr, steps_total, B, H, 1, D), seed, synth.T_NEWK, dev)
+            vn = synth.torch_gaussian_fp16((Lyr, steps_total, B, H, 1, D), seed, synth.T_NEWV, dev)
+            self.kn, self.vn = kn, vn
+            self.qs = synth.torch_gaussian_fp16((Lyr, steps_total, B, H, D), seed, synth.T_Q, dev)
+            self.out = torch.empty((Lyr, B, H, D), dtype=torch.float16, device=dev)
+        stream.synchronize()
+        self.ctx.check()
+
+    def _flush_due(self, i):
+        return (i + 1) % self.flush_every == 0
+
+    def step(self, i):
+        for l in range(self.layers):
+            self.ctx.append(l, self.kn[l, i], self.vn[l, i], 1)
+            self.ctx.decode(l, self.qs[l, i], self.out[l])
+        if self._flush_due(i):
+            self.ctx.flush(-1)
+
+    def context_after(self, i):
+        # the buffer holds the tokens appended since the last flush
+        in_buf = i % self.flush_every + 1
+        return self.wl["prefix"] + i + 1 - in_buf, in_buf
+
+    def host_inputs(self, i):
+        return [self.kn[:, i], self.vn[:, i], self.qs[:, i]]
+
+    def step_with(self, dev_inputs):
+        dk, dv, dq = dev_inputs
+        i = self._e2e_i
+        for l in range(self.layers):
+            self.ctx.append(l, dk[l], dv[l], 1)
+            self.ctx.decode(l, dq[l], self.out[l])
+        if self._flush_due(i):
+            self.ctx.flush(-1)
+        return [self.out]
+
+
 def run_swan(args, wl, rank: int, world: int, local_rank: int):
     import torch
 
-    from paper_2511_18936_gb300 import swan, synth
-
     dev = torch.device("cuda", local_rank)
     torch.cuda.set_device(dev)
-    B, H_q, H_kv, L_s, n_b, k = wl["B"], wl["H_q"], wl["H_kv"], wl["L_s"], wl["n_b"], wl["k"]
-    G = H_q // H_kv
+    B, H_q, H_kv, k = wl["B"], wl["H_q"], wl["H_kv"], wl["k"]
     steps_total = args.warmup + args.steps + 2 * args.e2e_steps
-    max_seq = L_s + n_b + steps_total + 8
     stream = torch.cuda.Stream(dev)
     seed = args.seed + rank
-
-    with torch.cuda.stream(stream):
-        R = torch.from_numpy(synth.rotations(H_kv, D, seed=seed, workload=1, layer=0))[None].to(dev)
-        # prefill: the whole context in one append (L_s tokens pruned, n_b stay dense)
-        ctx = swan.Context(R, num_layers=1, batch=B, n_q_heads=H_q, n_kv_heads=H_kv,
-                           k_store=wl["k_store"], buffer_cap=n_b, max_seq=max_seq, stream=stream)
-        kk = synth.torch_lowrank_kv(B, H_kv, L_s + n_b, D, seed, synth.T_K, dev)
-        vv = synth.torch_lowrank_kv(B, H_kv, L_s + n_b, D, seed, synth.T_V, dev)
-        ctx.append(0, kk, vv)
-        del kk, vv
-        k_new = synth.torch_lowrank_kv(B, H_kv, steps_total, D, seed, synth.T_NEWK, dev)
-        v_new = synth.torch_lowrank_kv(B, H_kv, steps_total, D, seed, synth.T_NEWV, dev)
-        k_steps = [k_new[:, :, i:i + 1].contiguous() for i in range(steps_total)]
-        v_steps = [v_new[:, :, i:i + 1].contiguous() for i in range(steps_total)]
-        del k_new, v_new
-        qs = synth.torch_gaussian_fp16((steps_total, B, H_q, D), seed, synth.T_Q, dev)
-        out = torch.empty((B, H_q, D), dtype=torch.float16, device=dev)
-        ctx.set_k(k)
-    stream.synchronize()
-    ctx.check()
-
-    def step(i):
-        ctx.append(0, k_steps[i], v_steps[i], 1)
-        ctx.decode(0, qs[i], out)
+    kind = wl.get("kind", "layer")
+    if kind == "stack" and steps_total > wl["max_steps"]:
+        raise SystemExit(f"the stack workload runs at most {wl['max_steps']} decode steps")
+    run = (StackRun if kind == "stack" else LayerRun)(wl, dev, stream, seed, steps_total)
+    ctx = run.ctx
+    flush_l2 = wl.get("l2_flush", False)
+    l2_buf = torch.empty(512 * 1024 * 1024 // 4, dtype=torch.float32, device=dev) if flush_l2 else None
 
     for i in range(args.warmup):
-        step(i)
+        run.step(i)
     stream.synchronize()
 
     def barrier():
@@ -259,48 +378,53 @@ def run_swan(args, wl, rank: int, world: int, local_rank: int):
             torch.distributed.barrier()
 
     # ---- timed region: inputs resident in HBM -----------------------------
-    ctxlen = []
+    steps = range(args.warmup, args.warmup + args.steps)
     launches0 = ctx.launch_count()
     ctx.timing_enable(True)
-    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     barrier()
     torch.cuda.synchronize(dev)
     with ClockSampler(local_rank) as clk:
-        ev0.record(stream)
-        for i in range(args.warmup, args.warmup + args.steps):
-            step(i)
-            info_len = L_s + n_b + (i + 1)  # context attended in step i
-            ctxlen.append(info_len)
-        ev1.record(stream)
-        stream.synchronize()
+        if not flush_l2:
+            ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            ev0.record(stream)
+            for i in steps:
+                run.step(i)
+            ev1.record(stream)
+            stream.synchronize()
+            ms = ev0.elapsed_time(ev1)
+        else:
+            # L2-resident workload: flush L2 (write 512 MB) between timed steps
+            ms = 0.0
+            for i in steps:
+                with torch.cuda.stream(stream):
+                    l2_buf.zero_()
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                e0.record(stream)
+                run.step(i)
+                e1.record(stream)
+                stream.synchronize()
+                ms += e0.elapsed_time(e1)
     barrier()
     torch.cuda.synchronize(dev)
-    ms = ev0.elapsed_time(ev1)
     kt = ctx.timing_read()
     ctx.timing_enable(False)
     launches = ctx.launch_count() - launches0
-    info = ctx.query(0)
-    assert info.sparse_len + info.buffer_len == L_s + n_b + args.warmup + args.steps
 
     # ---- end to end: pinned host inputs, H2D copies and the D2H read inside -
     e2e_steps = args.e2e_steps
     base = args.warmup + args.steps
-    hk = [k_steps[base + i].cpu().pin_memory() for i in range(2 * e2e_steps)]
-    hv = [v_steps[base + i].cpu().pin_memory() for i in range(2 * e2e_steps)]
-    hq = [qs[base + i].cpu().pin_memory() for i in range(2 * e2e_steps)]
-    hout = torch.empty((B, H_q, D), dtype=torch.float16).pin_memory()
-    dk = torch.empty_like(k_steps[0])
-    dv = torch.empty_like(v_steps[0])
-    dq = torch.empty_like(qs[0])
+    host = [[t.cpu().pin_memory() for t in run.host_inputs(base + i)] for i in range(2 * e2e_steps)]
+    dev_in = [torch.empty_like(t, device=dev) for t in host[0]]
+    host_out = [torch.empty_like(run.out, device="cpu").pin_memory()]
 
     def e2e_step(i):
+        run._e2e_i = base + i
         with torch.cuda.stream(stream):
-            dk.copy_(hk[i], non_blocking=True)
-            dv.copy_(hv[i], non_blocking=True)
-            dq.copy_(hq[i], non_blocking=True)
-            ctx.append(0, dk, dv, 1)
-            ctx.decode(0, dq, out)
-            hout.copy_(out, non_blocking=True)
+            for d, h in zip(dev_in, host[i]):
+                d.copy_(h, non_blocking=True)
+            outs = run.step_with(dev_in)
+            for ho, o in zip(host_out, outs):
+                ho.copy_(o, non_blocking=True)
         stream.synchronize()
 
     for i in range(e2e_steps):  # warm-up of the copy path
@@ -310,16 +434,17 @@ def run_swan(args, wl, rank: int, world: int, local_rank: int):
     e2e_tokens = 0
     for i in range(e2e_steps, 2 * e2e_steps):
         e2e_step(i)
-        e2e_tokens += B * H_kv * (L_s + n_b + base + i + 1)
+        sp, bf = run.context_after(base + i)
+        e2e_tokens += B * H_kv * (sp + bf) * run.layers
     e2e_s = time.perf_counter() - t0
     barrier()
-    h2d = hk[0].numel() * 2 + hv[0].numel() * 2 + hq[0].numel() * 2
-    d2h = hout.numel() * 2
+    h2d = sum(t.numel() * t.element_size() for t in host[0])
+    d2h = sum(t.numel() * t.element_size() for t in host_out)
 
     # ---- aggregate over ranks ----------------------------------------------
-    kv_tokens = sum(B * H_kv * c for c in ctxlen)
-    t_max = ms
-    e2e_max = e2e_s
+    ctxs = [run.context_after(i) for i in steps]
+    kv_tokens = sum(B * H_kv * (sp + bf) * run.layers for sp, bf in ctxs)
+    t_max, e2e_max = ms, e2e_s
     if world > 1:
         tt = torch.tensor([ms, e2e_s], device=dev, dtype=torch.float64)
         torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
@@ -329,45 +454,54 @@ def run_swan(args, wl, rank: int, world: int, local_rank: int):
 
     dec_ms, dec_n = kt["decode"]
     avg_dec_s = dec_ms / 1e3 / max(dec_n, 1)
-    ctx_mean = statistics.mean(ctxlen)
-    sparse_mean = ctx_mean - n_b
-    # algorithmic bytes of one decode-kernel launch: per (sparse token, kv head)
-    # 2 * 3 * k bytes (fp16 value + uint8 index for K and V); per (buffer
-    # token, kv head) 2 * 2 * d bytes
-    alg_decode = B * H_kv * (sparse_mean * 6 * k + n_b * 4 * D)
+    sp_mean = statistics.mean(sp for sp, _ in ctxs)
+    bf_mean = statistics.mean(bf for _, bf in ctxs)
+    # algorithmic bytes of one decode-kernel launch (one layer): per (sparse
+    # token, kv head) 2 * 3 * k bytes (fp16 value + uint8 index for K and V);
+    # per (buffer token, kv head) 2 * 2 * d bytes
+    alg_decode = B * H_kv * (sp_mean * 6 * k + bf_mean * 4 * D)
     achieved = alg_decode / avg_dec_s / 1e9
     peaks = measured_peaks()
     peak = float(peaks["hbm_gbs"]) if peaks else 6800.0
     step_s = t_max / 1e3 / args.steps
-    # whole-step algorithmic bytes: decode reads + q/out + R (q and out fp16,
-    # R fp32 once per kv head) + the append's new vectors and evicted one
-    alg_step = (alg_decode + 2 * B * H_q * D * 2 + H_kv * D * D * 4
-                + B * H_kv * (2 * D * 2 * 2 + 6 * wl["k_store"]))
+    # whole-step algorithmic bytes per layer: decode reads + q/out (fp16) + R
+    # (fp32, once per kv head, query and value rotations) + the append's new
+    # vectors (fp16 in, fp16 to the buffer)
+    alg_step = run.layers * (alg_decode + 2 * B * H_q * D * 2 + 2 * H_kv * D * D * 4
+                             + B * H_kv * 2 * D * 2 * 2)
+    l2_note = ("L2 flushed (512 MB written) before every timed step" if flush_l2 else
+               f"inputs larger than L2: {alg_decode * run.layers / 1e9:.2f} GB read per step, no flush")
+    cfg = {"workload": args.workload, "desc": wl["desc"], "batch": B, "n_q_heads": H_q,
+           "n_kv_heads": H_kv, "layers": run.layers, "sparse_tokens": wl.get("L_s", wl.get("prefix")),
+           "buffer_tokens": wl["n_b"], "k": k, "k_store": wl["k_store"],
+           "storage": "fp16 values + uint8 indices (sparse), fp16 (buffer)", "l2": l2_note,
+           "parallelism": f"replicas x{world} (independent batches per GPU)" if world > 1
+           else "single GPU"}
     line = {
         "metric": METRIC, "value": value, "unit": "KV-tokens/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": t_max / args.steps,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
-        "data": "synthetic (seeded low-rank K/V, Gaussian q, random orthogonal R)",
-        "config": {"workload": args.workload, "desc": wl["desc"], "batch": B, "n_q_heads": H_q,
-                   "n_kv_heads": H_kv, "sparse_tokens": L_s, "buffer_tokens": n_b, "k": k,
-                   "storage": "fp16 values + uint8 indices (sparse), fp16 (buffer)",
-                   "l2": f"inputs larger than L2: {alg_decode / 1e9:.2f} GB read per decode, no flush",
-                   "parallelism": f"replicas x{world}" if world > 1 else "single GPU"},
+        "data": "synthetic (seeded low-rank K/V, Gaussian q, random orthogonal R)"
+                if kind != "stack" else "synthetic (seeded Gaussian q/K/V, random orthogonal R)",
+        "config": cfg,
         "hbm_gbs_step": alg_step / step_s / 1e9,
         "pct_of_8tbs_step": 100.0 * alg_step / step_s / 1e9 / NOMINAL_HBM_GBS,
         "roofline": {"kernel": "decode", "bound": "hbm", "achieved": achieved, "peak": peak,
                      "unit": "GB/s", "frac": achieved / peak,
-                     "peak_source": "MEASURED_PEAKS.json hbm_gbs (measured)" if peaks
+                     "peak_source": "MEASURED_PEAKS.json hbm_gbs (measured copy)" if peaks
                      else "fallback 6.8 TB/s",
                      "pct_of_8tbs": 100.0 * achieved / NOMINAL_HBM_GBS,
                      "alg_bytes_per_launch": alg_decode, "avg_launch_ms": avg_dec_s * 1e3,
                      "traffic": decode_kernel_traffic(args.workload)},
-        "kernels_ms_per_step": {name: v[0] / max(v[1], 1) for name, v in kt.items() if v[1]},
+        "kernels_ms_per_step": {name: v[0] / args.steps for name, v in kt.items() if v[1]},
         "gpu_launches": launches,
         "e2e": {"value": e2e_value, "unit": "KV-tokens/s", "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h, "steps": e2e_steps},
         "clocks": clk.summary(),
     }
+    if kind == "stack":
+        line["prefix_ms"] = run.prefix_ms
+        line["prefix_tokens_per_s"] = wl["layers"] * B * H_kv * wl["prefix"] / (run.prefix_ms / 1e3)
     ctx.check()
     ctx.close()
     return line
@@ -385,6 +519,8 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--batch", type=int, default=0,
                     help="override the workload's batch (smaller cases for profiling)")
+    ap.add_argument("--k-active", type=int, default=0,
+                    help="runtime keep count (ksweep-32k: 32, 48, 64, 96 or 128)")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
@@ -392,6 +528,11 @@ def main():
     if args.batch:
         wl["B"] = args.batch
         wl["desc"] += f" (batch overridden to {args.batch})"
+    if args.k_active:
+        if not 1 <= args.k_active <= wl["k_store"]:
+            ap.error(f"--k-active must be in [1, {wl['k_store']}]")
+        wl["k"] = args.k_active
+        wl["desc"] += f" (k_active {args.k_active})"
 
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))

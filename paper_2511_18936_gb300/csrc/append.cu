@@ -108,8 +108,7 @@ __global__ void __launch_bounds__(kThreads, 1) append_kernel(AppendParams p) {
   const __half* X = kind ? p.v_new : p.k_new;
   __half* ring = kind ? p.ring_v : p.ring_k;
 
-  for (int i = threadIdx.x; i < kHeadDim * kHeadDim / 4; i += kThreads)
-    reinterpret_cast<float4*>(Rs)[i] = __ldg(reinterpret_cast<const float4*>(R) + i);
+  stage_matrix(Rs, R);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int64_t nvec = (int64_t)p.B * p.T;
@@ -204,8 +203,7 @@ __global__ void __launch_bounds__(kThreads) append_small_kernel(AppendParams p, 
   __half* ring = kind ? p.ring_v : p.ring_k;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
-  for (int i = threadIdx.x; i < kHeadDim * kHeadDim / 4; i += kThreads)
-    reinterpret_cast<float4*>(Rs)[i] = __ldg(reinterpret_cast<const float4*>(R) + i);
+  stage_matrix(Rs, R);
 
   // phase 1: evict the oldest buffered vectors (sparse positions L_s + i)
   for (int item = warp; item < p.B * evict_old; item += kWarpsPerCta) {

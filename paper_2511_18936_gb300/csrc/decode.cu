@@ -145,12 +145,19 @@ __device__ __forceinline__ void prefetch_l2(const void* ptr, uint32_t bytes) {
 //   the same contiguous run of 32-token blocks.  While block g is processed,
 //   the key records of block g+1 are in flight to registers and block g+2 is
 //   being prefetched into L2.
+// Warps per decode CTA: as many lane-private accumulators as fit next to
+// the replicated q' (16 KB each, 227 KB of shared memory per CTA).
 template <int G, int MAXC>
-__global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
-  constexpr int TEAMS = kWarpsPerCta / G;
+__host__ __device__ constexpr int decode_warps() { return (G == 1 && MAXC <= 8) ? 12 : 8; }
+
+template <int G, int MAXC>
+__global__ void __launch_bounds__(decode_warps<G, MAXC>() * 32, 1) decode_kernel(DecodeParams p) {
+  constexpr int NW = decode_warps<G, MAXC>();
+  constexpr int NT = NW * 32;
+  constexpr int TEAMS = NW / G;
   constexpr bool kL1 = G > 1;
   extern __shared__ __align__(16) unsigned char smem_raw[];
-  __shared__ float red_m[kWarpsPerCta], red_l[kWarpsPerCta];
+  __shared__ float red_m[NW], red_l[NW];
 
   const uint32_t raw = (uint32_t)__cvta_generic_to_shared(smem_raw);
   const uint32_t base = (raw + kRegionBytes - 1) & ~(kRegionBytes - 1);
@@ -199,7 +206,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
     const int32_t* ptab = g.page_table + u * g.pages_per_unit;
 
     __syncthreads();  // the previous segment's reduction is done with smem
-    for (int i = threadIdx.x; i < G * kHeadDim * 32; i += kThreads) {
+    for (int i = threadIdx.x; i < G * kHeadDim * 32; i += NT) {
       const int gh = i >> 12, dd = (i >> 5) & (kHeadDim - 1);
       qrep[i] = __ldg(p.qprime + ((b * p.H_q + h * G + gh) * kHeadDim + dd));
     }
@@ -385,7 +392,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
       red_l[warp] = l_sum;
     }
     __syncthreads();
-    for (int o = threadIdx.x; o < G * kHeadDim; o += kThreads) {
+    for (int o = threadIdx.x; o < G * kHeadDim; o += NT) {
       const int gh = o / kHeadDim, dd = o % kHeadDim;
       float M = -INFINITY;
 #pragma unroll
@@ -428,7 +435,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
       __threadfence();
       const int64_t c0 = (u * p.N_g) / p.range, c1 = ((u + 1) * p.N_g - 1) / p.range;
       float* o_hat = qrep;  // [G][128]; q' of this unit is no longer needed
-      for (int o = threadIdx.x; o < G * kHeadDim; o += kThreads) {
+      for (int o = threadIdx.x; o < G * kHeadDim; o += NT) {
         const int gh = o / kHeadDim, dd = o % kHeadDim;
         float M = -INFINITY;
         for (int64_t c = c0; c <= c1; ++c)
@@ -445,7 +452,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
       }
       __syncthreads();
       const float* RT = p.R_voT + (size_t)h * kHeadDim * kHeadDim;
-      for (int o = threadIdx.x; o < G * kHeadDim; o += kThreads) {
+      for (int o = threadIdx.x; o < G * kHeadDim; o += NT) {
         const int gh = o / kHeadDim, i = o % kHeadDim;
         const float* oh = o_hat + gh * kHeadDim;
         float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
@@ -470,8 +477,7 @@ __global__ void __launch_bounds__(kThreads) rotate_q_kernel(RotateQParams p, int
   float* Rs = reinterpret_cast<float*>(smem_raw);
   const int h = blockIdx.x;
   const float* R = p.R_qk + (size_t)h * kHeadDim * kHeadDim;
-  for (int i = threadIdx.x; i < kHeadDim * kHeadDim / 4; i += kThreads)
-    reinterpret_cast<float4*>(Rs)[i] = __ldg(reinterpret_cast<const float4*>(R) + i);
+  stage_matrix(Rs, R);
   __syncthreads();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   for (int item = warp; item < B * p.G; item += kWarpsPerCta) {
@@ -536,25 +542,26 @@ __global__ void __launch_bounds__(kHeadDim) combine_kernel(CombineParams p) {
 template <int G, int MAXC>
 cudaError_t launch_decode_t(const DecodeParams& p, int grid, cudaStream_t s) {
   static bool attr_set = false;
-  const size_t smem = decode_smem_bytes(G);
+  const size_t smem = decode_smem_bytes(G, MAXC * 8);
   if (!attr_set) {
     cudaError_t e = cudaFuncSetAttribute(decode_kernel<G, MAXC>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
-  decode_kernel<G, MAXC><<<grid, kThreads, smem, s>>>(p);
+  decode_kernel<G, MAXC><<<grid, decode_warps<G, MAXC>() * 32, smem, s>>>(p);
   return cudaGetLastError();
 }
 
 template <int G, int MAXC>
 int ctas_per_sm_t() {
-  const size_t smem = decode_smem_bytes(G);
+  const size_t smem = decode_smem_bytes(G, MAXC * 8);
   if (cudaFuncSetAttribute(decode_kernel<G, MAXC>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                            (int)smem) != cudaSuccess)
     return 0;
   int n = 0;
-  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, decode_kernel<G, MAXC>, kThreads, smem) !=
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, decode_kernel<G, MAXC>, decode_warps<G, MAXC>() * 32,
+                                                    smem) !=
       cudaSuccess)
     return 0;
   return n;
@@ -562,7 +569,10 @@ int ctas_per_sm_t() {
 
 }  // namespace
 
-size_t decode_smem_bytes(int G) { return (size_t)(G + kWarpsPerCta + 1) * kRegionBytes; }
+size_t decode_smem_bytes(int G, int k_slots) {
+  const int nw = (G == 1 && k_slots <= 64) ? decode_warps<1, 8>() : decode_warps<2, 16>();
+  return (size_t)(G + nw + 1) * kRegionBytes;
+}
 
 int decode_ctas_per_sm(int G, int k_slots) {
   const bool big = k_slots > 64;
@@ -574,8 +584,8 @@ int decode_ctas_per_sm(int G, int k_slots) {
   }
 }
 
-cudaError_t launch_decode(const DecodeParams& p, int G, int k_slots, int grid, cudaStream_t s) {
-  const bool big = k_slots > 64;
+cudaError_t launch_decode(const DecodeParams& p, int G, int k_read, int grid, cudaStream_t s) {
+  const bool big = k_read > 64;
   switch (G) {
     case 1: return big ? launch_decode_t<1, 16>(p, grid, s) : launch_decode_t<1, 8>(p, grid, s);
     case 2: return big ? launch_decode_t<2, 16>(p, grid, s) : launch_decode_t<2, 8>(p, grid, s);

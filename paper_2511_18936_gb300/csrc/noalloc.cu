@@ -119,7 +119,7 @@ extern "C" swan_status swan_decode_noalloc(const swan_cache_view* v, const void*
   const int64_t total = units * N_g;
   int64_t range = 1, grid = 0;
   if (total > 0) {
-    const int64_t ctas = std::min<int64_t>((int64_t)ds->sms * ds->ctas_per_sm[gi(G)][v->k_slots > 64], total);
+    const int64_t ctas = std::min<int64_t>((int64_t)ds->sms * ds->ctas_per_sm[gi(G)][v->k_active > 64], total);
     range = (total + ctas - 1) / ctas;
     grid = (total + range - 1) / range;
   }
@@ -177,7 +177,7 @@ extern "C" swan_status swan_decode_noalloc(const swan_cache_view* v, const void*
     p.R_voT = v->R_vo_t;
     p.out = static_cast<__half*>(out);
     p.status = status;
-    if (launch_decode(p, G, v->k_slots, (int)grid, s) != cudaSuccess)
+    if (launch_decode(p, G, (v->k_active + 7) / 8 * 8, (int)grid, s) != cudaSuccess)
       return err(SWAN_ERR_CUDA, "decode launch failed");
     return SWAN_OK;
   }

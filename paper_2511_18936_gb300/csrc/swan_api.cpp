@@ -524,7 +524,7 @@ swan_status swan_decode(swan_ctx* c, int layer, const void* q, void* out) {
     p.status = c->status;
     // the split combine and the rotate-back run inside the decode kernel
     return launch(c, SWAN_KERNEL_DECODE, "decode kernel",
-                  [&] { return launch_decode(p, G, c->k_slots, (int)grid, c->stream); });
+                  [&] { return launch_decode(p, G, (c->k_active + 7) / 8 * 8, (int)grid, c->stream); });
   }
   // empty cache: the combine kernel writes zeros
 

@@ -124,6 +124,20 @@ struct CombineParams {
   int64_t N_g, range, total_groups;
 };
 
+#ifdef __CUDACC__
+// Stage a 128 x 128 fp32 matrix in shared memory with a CTA of kThreads
+// threads: every thread issues its 16 loads before its first store, so all
+// of them are in flight at once.
+__device__ __forceinline__ void stage_matrix(float* dst, const float* src) {
+  float4 r[16];
+#pragma unroll
+  for (int k = 0; k < 16; ++k)
+    r[k] = __ldg(reinterpret_cast<const float4*>(src) + threadIdx.x + k * kThreads);
+#pragma unroll
+  for (int k = 0; k < 16; ++k) reinterpret_cast<float4*>(dst)[threadIdx.x + k * kThreads] = r[k];
+}
+#endif
+
 // Launchers (return the launch error, if any).
 cudaError_t launch_append(const AppendParams& p, cudaStream_t s);
 // Eviction of `evict_old` buffered tokens and insertion of T new ones in one
@@ -131,12 +145,13 @@ cudaError_t launch_append(const AppendParams& p, cudaStream_t s);
 cudaError_t launch_append_small(const AppendParams& p, int evict_old, cudaStream_t s);
 cudaError_t launch_prune_ring(const PruneRingParams& p, cudaStream_t s);
 cudaError_t launch_rotate_q(const RotateQParams& p, int B, cudaStream_t s);
-cudaError_t launch_decode(const DecodeParams& p, int G, int k_slots, int grid, cudaStream_t s);
+// k_read: entries read per vector rounded up to 8 (selects the kernel variant)
+cudaError_t launch_decode(const DecodeParams& p, int G, int k_read, int grid, cudaStream_t s);
 cudaError_t launch_combine(const CombineParams& p, int B, cudaStream_t s);
 cudaError_t launch_transpose_r(const float* src, float* dst, int64_t mats, cudaStream_t s);
 // Decode CTAs that fit on one SM together (for the grid size).
 int decode_ctas_per_sm(int G, int k_slots);
-size_t decode_smem_bytes(int G);
+size_t decode_smem_bytes(int G, int k_slots);
 // Record the detail string that swan_last_error() returns on this thread.
 void set_last_error(const char* msg);
 

@@ -137,6 +137,58 @@ __device__ __forceinline__ void prefetch_l2(const void* ptr, uint32_t bytes) {
   asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(ptr), "r"(bytes) : "memory");
 }
 
+// The last CTA to finish a segment of unit u merges the unit's partials,
+// normalises, rotates back (o = o_hat R_vo^T) and writes the output.  The
+// arrival counter resets itself for the next decode; nothing waits.
+// `scratch` holds G * 128 floats (free at this point); `flag` one float.
+template <int G, int NT>
+__device__ __forceinline__ void finish_unit(const DecodeParams& p, int64_t u, int64_t b, int64_t h,
+                                            float* scratch, float* flag) {
+  __threadfence();
+  __syncthreads();
+  const int64_t c0 = (u * p.N_g) / p.range, c1 = ((u + 1) * p.N_g - 1) / p.range;
+  if (threadIdx.x == 0) {
+    const int old = atomicAdd(p.counters + u, 1);
+    const bool last = old == (int)(c1 - c0);
+    if (last) p.counters[u] = 0;
+    flag[0] = last ? 1.f : 0.f;
+  }
+  __syncthreads();
+  if (flag[0] == 0.f) return;
+  __threadfence();
+  float* o_hat = scratch;  // [G][128]
+  for (int o = threadIdx.x; o < G * kHeadDim; o += NT) {
+    const int gh = o / kHeadDim, dd = o % kHeadDim;
+    float M = -INFINITY;
+    for (int64_t c = c0; c <= c1; ++c)
+      M = fmaxf(M, __ldcg(p.partials + ((size_t)(c + u) * G + gh) * (kHeadDim + 2)));
+    float L = 0.f, A = 0.f;
+    for (int64_t c = c0; c <= c1; ++c) {
+      const float* part = p.partials + ((size_t)(c + u) * G + gh) * (kHeadDim + 2);
+      const float mc = __ldcg(part);
+      const float w = (mc == -INFINITY) ? 0.f : exp2f(mc - M);
+      L = fmaf(w, __ldcg(part + 1), L);
+      A = fmaf(w, __ldcg(part + 2 + dd), A);
+    }
+    o_hat[o] = (L > 0.f) ? A / L : 0.f;
+  }
+  __syncthreads();
+  const float* RT = p.R_voT + (size_t)h * kHeadDim * kHeadDim;
+  for (int o = threadIdx.x; o < G * kHeadDim; o += NT) {
+    const int gh = o / kHeadDim, i = o % kHeadDim;
+    const float* oh = o_hat + gh * kHeadDim;
+    float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
+#pragma unroll 8
+    for (int j = 0; j < kHeadDim; j += 4) {
+      a0 = fmaf(oh[j + 0], __ldg(RT + (j + 0) * kHeadDim + i), a0);
+      a1 = fmaf(oh[j + 1], __ldg(RT + (j + 1) * kHeadDim + i), a1);
+      a2 = fmaf(oh[j + 2], __ldg(RT + (j + 2) * kHeadDim + i), a2);
+      a3 = fmaf(oh[j + 3], __ldg(RT + (j + 3) * kHeadDim + i), a3);
+    }
+    p.out[((b * p.H_q) + h * G + gh) * kHeadDim + i] = __float2half_rn((a0 + a1) + (a2 + a3));
+  }
+}
+
 // Split decode kernel.
 //   Shared memory (16 KB-aligned regions): q' of the unit's G query heads
 //   replicated per lane ([G][128][32] fp32) and one lane-private
@@ -418,54 +470,399 @@ __global__ void __launch_bounds__(decode_warps<G, MAXC>() * 32, 1) decode_kernel
       }
     }
 
-    // ---- the last CTA to finish a segment of unit u merges the unit's
-    // partials, normalises, rotates back and writes the output (the
-    // arrival counter resets itself for the next decode; nothing waits)
-    __threadfence();
-    __syncthreads();
-    if (threadIdx.x == 0) {
-      const int64_t c0 = (u * p.N_g) / p.range, c1 = ((u + 1) * p.N_g - 1) / p.range;
-      const int old = atomicAdd(p.counters + u, 1);
-      const bool last = old == (int)(c1 - c0);
-      if (last) p.counters[u] = 0;
-      red_m[0] = last ? 1.f : 0.f;
+    finish_unit<G, NT>(p, u, b, h, qrep, red_m);
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Grouped-query heads (G = 2 or 4): each lane carries a pair of query heads
+// of one token, so the index decoding, the fp16 conversion and the record
+// loads are shared by two heads, and one accumulator array serves the whole
+// group: lanes 16..31 take heads 2..3 of the tokens that lanes 0..15 take
+// heads 0..1 of (G = 4).  q' and the accumulators are [128][32 lanes][2]
+// fp32 (32 KB), so 32 lanes reading or updating arbitrary coordinates with
+// 8-byte accesses never share a bank within a half-warp.
+// ---------------------------------------------------------------------------
+
+constexpr uint32_t kPairRegionBytes = kHeadDim * 32 * 2 * sizeof(float);  // 32 KB
+constexpr int kGqaWarps = 5;  // q' + 5 accumulators at 32 KB-aligned offsets fit in 227 KB
+
+// base | (idx & 127) << 8 | lane << 3 for byte e of an index word (base 32 KB aligned)
+template <int E>
+__device__ __forceinline__ uint32_t addr2_of(uint32_t w, uint32_t base) {
+  if (E == 0) return ((w << 8) & 0x7f00u) | base;
+  if (E == 1) return (w & 0x7f00u) | base;
+  if (E == 2) return ((w >> 8) & 0x7f00u) | base;
+  return ((w >> 16) & 0x7f00u) | base;
+}
+__device__ __forceinline__ float2 lds2(uint32_t a) {
+  float2 v;
+  asm volatile("ld.shared.v2.f32 {%0,%1}, [%2];" : "=f"(v.x), "=f"(v.y) : "r"(a));
+  return v;
+}
+__device__ __forceinline__ void sts2(uint32_t a, float2 v) {
+  asm volatile("st.shared.v2.f32 [%0], {%1,%2};" ::"r"(a), "f"(v.x), "f"(v.y));
+}
+
+// Scores of two heads for one chunk: s[0..1] head 0, s[2..3] head 1.
+__device__ __forceinline__ void score2_chunk(uint32_t qb, uint4 v, uint2 ix, float (&s)[4]) {
+  const float2 q0 = lds2(addr2_of<0>(ix.x, qb)), q1 = lds2(addr2_of<1>(ix.x, qb));
+  const float2 q2 = lds2(addr2_of<2>(ix.x, qb)), q3 = lds2(addr2_of<3>(ix.x, qb));
+  const float2 q4 = lds2(addr2_of<0>(ix.y, qb)), q5 = lds2(addr2_of<1>(ix.y, qb));
+  const float2 q6 = lds2(addr2_of<2>(ix.y, qb)), q7 = lds2(addr2_of<3>(ix.y, qb));
+  const float2 a = h2f(v.x), b = h2f(v.y), c = h2f(v.z), d = h2f(v.w);
+  s[0] = fmaf(q0.x, a.x, s[0]); s[2] = fmaf(q0.y, a.x, s[2]);
+  s[1] = fmaf(q1.x, a.y, s[1]); s[3] = fmaf(q1.y, a.y, s[3]);
+  s[0] = fmaf(q2.x, b.x, s[0]); s[2] = fmaf(q2.y, b.x, s[2]);
+  s[1] = fmaf(q3.x, b.y, s[1]); s[3] = fmaf(q3.y, b.y, s[3]);
+  s[0] = fmaf(q4.x, c.x, s[0]); s[2] = fmaf(q4.y, c.x, s[2]);
+  s[1] = fmaf(q5.x, c.y, s[1]); s[3] = fmaf(q5.y, c.y, s[3]);
+  s[0] = fmaf(q6.x, d.x, s[0]); s[2] = fmaf(q6.y, d.x, s[2]);
+  s[1] = fmaf(q7.x, d.y, s[1]); s[3] = fmaf(q7.y, d.y, s[3]);
+}
+
+__device__ __forceinline__ float2 fma2(float p0, float p1, float v, float2 o) {
+  return make_float2(fmaf(p0, v, o.x), fmaf(p1, v, o.y));
+}
+
+// acc[idx_e] += (p0, p1) * val_e for one full chunk (distinct indices).
+__device__ __forceinline__ void value2_chunk(uint32_t ab, float p0, float p1, uint4 v, uint2 ix) {
+  const uint32_t a0 = addr2_of<0>(ix.x, ab), a1 = addr2_of<1>(ix.x, ab);
+  const uint32_t a2 = addr2_of<2>(ix.x, ab), a3 = addr2_of<3>(ix.x, ab);
+  const uint32_t a4 = addr2_of<0>(ix.y, ab), a5 = addr2_of<1>(ix.y, ab);
+  const uint32_t a6 = addr2_of<2>(ix.y, ab), a7 = addr2_of<3>(ix.y, ab);
+  const float2 o0 = lds2(a0), o1 = lds2(a1), o2 = lds2(a2), o3 = lds2(a3);
+  const float2 o4 = lds2(a4), o5 = lds2(a5), o6 = lds2(a6), o7 = lds2(a7);
+  const float2 a = h2f(v.x), b = h2f(v.y), c = h2f(v.z), d = h2f(v.w);
+  sts2(a0, fma2(p0, p1, a.x, o0));
+  sts2(a1, fma2(p0, p1, a.y, o1));
+  sts2(a2, fma2(p0, p1, b.x, o2));
+  sts2(a3, fma2(p0, p1, b.y, o3));
+  sts2(a4, fma2(p0, p1, c.x, o4));
+  sts2(a5, fma2(p0, p1, c.y, o5));
+  sts2(a6, fma2(p0, p1, d.x, o6));
+  sts2(a7, fma2(p0, p1, d.y, o7));
+}
+
+__device__ __forceinline__ void value2_chunk_partial(uint32_t ab, float p0, float p1, uint4 v, uint2 ix,
+                                                     int n) {
+  const uint32_t hw[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+  for (int e = 0; e < 7; ++e) {
+    if (e < n) {
+      const uint32_t w = e < 4 ? ix.x : ix.y;
+      const uint32_t a = ((w >> (8u * (e & 3))) & 0x7fu) << 8 | ab;
+      const float2 f = h2f(hw[e >> 1]);
+      sts2(a, fma2(p0, p1, (e & 1) ? f.y : f.x, lds2(a)));
     }
-    __syncthreads();
-    if (red_m[0] != 0.f) {
-      __threadfence();
-      const int64_t c0 = (u * p.N_g) / p.range, c1 = ((u + 1) * p.N_g - 1) / p.range;
-      float* o_hat = qrep;  // [G][128]; q' of this unit is no longer needed
-      for (int o = threadIdx.x; o < G * kHeadDim; o += NT) {
-        const int gh = o / kHeadDim, dd = o % kHeadDim;
-        float M = -INFINITY;
-        for (int64_t c = c0; c <= c1; ++c)
-          M = fmaxf(M, __ldcg(p.partials + ((size_t)(c + u) * G + gh) * (kHeadDim + 2)));
-        float L = 0.f, A = 0.f;
-        for (int64_t c = c0; c <= c1; ++c) {
-          const float* part = p.partials + ((size_t)(c + u) * G + gh) * (kHeadDim + 2);
-          const float mc = __ldcg(part);
-          const float w = (mc == -INFINITY) ? 0.f : exp2f(mc - M);
-          L = fmaf(w, __ldcg(part + 1), L);
-          A = fmaf(w, __ldcg(part + 2 + dd), A);
-        }
-        o_hat[o] = (L > 0.f) ? A / L : 0.f;
-      }
-      __syncthreads();
-      const float* RT = p.R_voT + (size_t)h * kHeadDim * kHeadDim;
-      for (int o = threadIdx.x; o < G * kHeadDim; o += NT) {
-        const int gh = o / kHeadDim, i = o % kHeadDim;
-        const float* oh = o_hat + gh * kHeadDim;
-        float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
+  }
+}
+
+// Reduce over the lanes of one head group (TS lanes: the whole warp for
+// G = 2, a half-warp for G = 4).
+template <int TS>
+__device__ __forceinline__ float group_max(float v) {
+#pragma unroll
+  for (int o = TS / 2; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+  return v;
+}
+template <int TS>
+__device__ __forceinline__ float group_sum(float v) {
+#pragma unroll
+  for (int o = TS / 2; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+template <int G, int MAXC>
+__global__ void __launch_bounds__(kGqaWarps * 32, 1) decode_gqa_kernel(DecodeParams p) {
+  constexpr int NW = kGqaWarps, NT = NW * 32;
+  constexpr int LPT = G / 2;          // lanes per token
+  constexpr int TS = 32 / LPT;        // tokens per warp iteration
+  constexpr int HALVES = 32 / TS;     // iterations per 32-token block
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  __shared__ float red_m[NW * G], red_l[NW * G], flag[1];
+
+  const uint32_t raw = (uint32_t)__cvta_generic_to_shared(smem_raw);
+  const uint32_t base = (raw + kPairRegionBytes - 1) & ~(kPairRegionBytes - 1);
+  float* qrep = reinterpret_cast<float*>(smem_raw + (base - raw));  // [128][32][2]
+  float* accs = qrep + kHeadDim * 32 * 2;                            // [NW][128][32][2]
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int ts = lane % TS, hg = lane / TS;  // token slot, head pair
+  const uint32_t qb = base + (lane << 3);
+  const uint32_t ab = base + (1 + warp) * kPairRegionBytes + (lane << 3);
+
+  const CacheGeom& g = p.geom;
+  const int kfull = p.k_full_chunks, krem = p.k_rem;
+  const int nchunks = kfull + (krem ? 1 : 0);
+  const int ks = g.k_slots;
+  const bool whole_block = nchunks * 8 == ks;
+  const uint32_t pf_val = (uint32_t)nchunks * 512, pf_idx = (uint32_t)nchunks * 256;
+  const int bsh = p.blocks_per_page_log2, bmask = (1 << bsh) - 1;
+  uint4 remmask;
+  {
+    uint32_t w[4];
+#pragma unroll
+    for (int e = 0; e < 4; ++e)
+      w[e] = ((2 * e < krem) ? 0xffffu : 0u) | ((2 * e + 1 < krem) ? 0xffff0000u : 0u);
+    remmask = make_uint4(w[0], w[1], w[2], w[3]);
+  }
+
+  const int64_t g_begin = (int64_t)blockIdx.x * p.range;
+  const int64_t g_end = min(p.total_groups, g_begin + p.range);
+  if (g_begin >= g_end) return;
+  const int64_t u_first = g_begin / p.N_g, u_last = (g_end - 1) / p.N_g;
+  const int n_sg = (int)p.n_sg;
+
+  for (int64_t u = u_first; u <= u_last; ++u) {
+    const int s0 = (int)(max(g_begin, u * p.N_g) - u * p.N_g);
+    const int s1 = (int)(min(g_end, (u + 1) * p.N_g) - u * p.N_g);
+    const int64_t b = u / p.H_kv, h = u % p.H_kv;
+    // this warp's contiguous run of items (half-blocks for G = 4)
+    const int items = (s1 - s0) * HALVES;
+    const int i_lo = s0 * HALVES + (items * warp) / NW;
+    const int i_hi = s0 * HALVES + (items * (warp + 1)) / NW;
+    const int32_t* ptab = g.page_table + u * g.pages_per_unit;
+
+    __syncthreads();  // the previous segment is done with shared memory
+    for (int i = threadIdx.x; i < kHeadDim * 32 * 2; i += NT) {
+      const int dd = i >> 6, l = (i >> 1) & 31, j = i & 1;
+      const int head = 2 * (l / TS) + j;
+      qrep[i] = __ldg(p.qprime + ((b * p.H_q + h * G + head) * kHeadDim + dd));
+    }
 #pragma unroll 8
-        for (int j = 0; j < kHeadDim; j += 4) {
-          a0 = fmaf(oh[j + 0], __ldg(RT + (j + 0) * kHeadDim + i), a0);
-          a1 = fmaf(oh[j + 1], __ldg(RT + (j + 1) * kHeadDim + i), a1);
-          a2 = fmaf(oh[j + 2], __ldg(RT + (j + 2) * kHeadDim + i), a2);
-          a3 = fmaf(oh[j + 3], __ldg(RT + (j + 3) * kHeadDim + i), a3);
+    for (int dd = 0; dd < kHeadDim; ++dd) sts2(ab + dd * 256, make_float2(0.f, 0.f));
+    __syncthreads();
+
+    float m0 = -INFINITY, m1 = -INFINITY;  // running maxima (log2), uniform in the head group
+    float l0 = 0.f, l1 = 0.f;
+
+    auto block_of = [&](int gi) -> const uint8_t* {
+      if (gi >= n_sg || gi * HALVES >= i_hi) return nullptr;
+      const int32_t ph = __ldg(ptab + (gi >> bsh));
+      if (ph < 0 || ph >= g.num_pages) {
+        atomicOr(p.status, kStatusPageRange);
+        return nullptr;
+      }
+      return g.pool + (int64_t)ph * g.page_bytes + (int64_t)(gi & bmask) * g.block_bytes();
+    };
+    auto prefetch_block = [&](const uint8_t* blk) {
+      if (blk == nullptr || lane != 0) return;
+      if (whole_block) {
+        prefetch_l2(blk, (uint32_t)g.block_bytes());
+      } else {
+        prefetch_l2(blk, pf_val);
+        prefetch_l2(blk + 64 * ks, pf_idx);
+        prefetch_l2(blk + 96 * ks, pf_val);
+        prefetch_l2(blk + 160 * ks, pf_idx);
+      }
+    };
+    // key records of item `it` (block gi, half `half`) for this lane's token
+    auto load_k = [&](const uint8_t* blk, int half, uint4 (&kv)[MAXC], uint2 (&ki)[MAXC]) {
+      const uint8_t* src = blk ? blk : g.pool;
+      const int t = half * TS + ts;
+#pragma unroll
+      for (int c = 0; c < MAXC; ++c)
+        if (c < nchunks) {
+          kv[c] = ld_rec16<true>(src + t * 16 + c * 512);
+          ki[c] = ld_rec8<true>(src + 64 * ks + t * 8 + c * 256);
         }
-        p.out[((b * p.H_q) + h * G + gh) * kHeadDim + i] = __float2half_rn((a0 + a1) + (a2 + a3));
+    };
+
+    uint4 kv[MAXC];
+    uint2 ki[MAXC];
+    int gi0 = i_lo / HALVES;
+    const uint8_t* b_cur = block_of(gi0);
+    const uint8_t* b_n1 = block_of(gi0 + 1);
+    prefetch_block(b_n1);
+    if (i_lo < i_hi && gi0 < n_sg) load_k(b_cur, i_lo % HALVES, kv, ki);
+
+    for (int it = i_lo; it < i_hi; ++it) {
+      const int gi = it / HALVES, half = it % HALVES;
+      float s[4] = {0.f, 0.f, 0.f, 0.f};
+      float p0, p1;
+      bool valid;
+      if (gi < n_sg) {
+        // ---- sparse tokens 32*gi + half*TS + ts
+        const int64_t t = (int64_t)gi * 32 + half * TS + ts;
+        const bool ok = b_cur != nullptr;
+        valid = ok && t < p.sparse_len;
+        const bool tail = !ok || (int64_t)gi * 32 + (half + 1) * TS > p.sparse_len;  // warp-uniform
+        const uint8_t* src = ok ? b_cur : g.pool;
+        const int tt = half * TS + ts;
+        uint4 vv[MAXC];
+        uint2 vi[MAXC];
+#pragma unroll
+        for (int c = 0; c < MAXC; ++c)
+          if (c < nchunks) {
+            vv[c] = ld_rec16<true>(src + 96 * ks + tt * 16 + c * 512);
+            vi[c] = ld_rec8<true>(src + 160 * ks + tt * 8 + c * 256);
+          }
+        const bool last_half = half == HALVES - 1;
+        const uint8_t* b_n2 = nullptr;
+        if (last_half) {
+          b_n2 = block_of(gi + 2);
+          prefetch_block(b_n2);
+        }
+
+        const uint4 lanemask = valid ? make_uint4(~0u, ~0u, ~0u, ~0u) : make_uint4(0, 0, 0, 0);
+#pragma unroll
+        for (int c = 0; c < MAXC; ++c)
+          if (c < nchunks) {
+            uint4 v = kv[c];
+            uint2 ix = ki[c];
+            if (krem && c == nchunks - 1) v = and4(v, remmask);
+            if (tail) {
+              v = and4(v, lanemask);
+              ix = valid ? ix : make_uint2(0, 0);
+            }
+            score2_chunk(qb, v, ix, s);
+          }
+
+        // next item's key records (same block's next half, or the next block)
+        const int nit = it + 1;
+        if (nit < i_hi) {
+          const int ngi = nit / HALVES;
+          if (ngi < n_sg) load_k(last_half ? b_n1 : b_cur, nit % HALVES, kv, ki);
+        }
+        if (last_half) {
+          b_cur = b_n1;
+          b_n1 = b_n2;
+        }
+
+        const float s0v = valid ? (s[0] + s[1]) * p.scale_log2 : -INFINITY;
+        const float s1v = valid ? (s[2] + s[3]) * p.scale_log2 : -INFINITY;
+        const float g0 = group_max<TS>(s0v), g1 = group_max<TS>(s1v);
+        if (g0 > m0 + kLazyRescale || g1 > m1 + kLazyRescale) {
+          const float n0 = (g0 > m0 + kLazyRescale) ? g0 : m0;
+          const float n1 = (g1 > m1 + kLazyRescale) ? g1 : m1;
+          const float f0 = (m0 == -INFINITY) ? 1.f : exp2f(m0 - n0);
+          const float f1 = (m1 == -INFINITY) ? 1.f : exp2f(m1 - n1);
+          l0 *= f0;
+          l1 *= f1;
+#pragma unroll 8
+          for (int dd = 0; dd < kHeadDim; ++dd) {
+            const float2 o = lds2(ab + dd * 256);
+            sts2(ab + dd * 256, make_float2(o.x * f0, o.y * f1));
+          }
+          m0 = n0;
+          m1 = n1;
+        }
+        p0 = valid ? exp2f(s0v - m0) : 0.f;
+        p1 = valid ? exp2f(s1v - m1) : 0.f;
+        l0 += p0;
+        l1 += p1;
+
+#pragma unroll
+        for (int c = 0; c < MAXC; ++c)
+          if (c < kfull) {
+            uint4 v = vv[c];
+            uint2 ix = vi[c];
+            if (tail) {
+              v = and4(v, lanemask);
+              ix = valid ? ix : make_uint2(0, 0);
+            }
+            value2_chunk(ab, p0, p1, v, ix);
+          }
+        if (krem && valid) {
+#pragma unroll
+          for (int c = 0; c < MAXC; ++c)
+            if (c == kfull) value2_chunk_partial(ab, p0, p1, vv[c], vi[c], krem);
+        }
+      } else {
+        // ---- dense buffer tokens
+        const int64_t i = (int64_t)(gi - n_sg) * 32 + half * TS + ts;
+        valid = i < p.n_b;
+        const int slot = valid ? (int)((p.buf_start + i) % p.cap) : 0;
+        const size_t row = ((size_t)u * p.cap + slot) * kHeadDim;
+        const uint4* kr = reinterpret_cast<const uint4*>(p.ring_k + row);
+        const uint4* vr = reinterpret_cast<const uint4*>(p.ring_v + row);
+#pragma unroll 2
+        for (int c = 0; c < 16; ++c) {
+          const uint4 w = __ldg(kr + c);
+          const float2 a = h2f(w.x), bb = h2f(w.y), cc = h2f(w.z), d = h2f(w.w);
+          const float vals[8] = {a.x, a.y, bb.x, bb.y, cc.x, cc.y, d.x, d.y};
+#pragma unroll
+          for (int e = 0; e < 8; ++e) {
+            const float2 q = lds2(qb + (c * 8 + e) * 256);
+            s[(e & 1)] = fmaf(q.x, vals[e], s[(e & 1)]);
+            s[2 + (e & 1)] = fmaf(q.y, vals[e], s[2 + (e & 1)]);
+          }
+        }
+        const float s0v = valid ? (s[0] + s[1]) * p.scale_log2 : -INFINITY;
+        const float s1v = valid ? (s[2] + s[3]) * p.scale_log2 : -INFINITY;
+        const float g0 = group_max<TS>(s0v), g1 = group_max<TS>(s1v);
+        if (g0 > m0 + kLazyRescale || g1 > m1 + kLazyRescale) {
+          const float n0 = (g0 > m0 + kLazyRescale) ? g0 : m0;
+          const float n1 = (g1 > m1 + kLazyRescale) ? g1 : m1;
+          const float f0 = (m0 == -INFINITY) ? 1.f : exp2f(m0 - n0);
+          const float f1 = (m1 == -INFINITY) ? 1.f : exp2f(m1 - n1);
+          l0 *= f0;
+          l1 *= f1;
+#pragma unroll 8
+          for (int dd = 0; dd < kHeadDim; ++dd) {
+            const float2 o = lds2(ab + dd * 256);
+            sts2(ab + dd * 256, make_float2(o.x * f0, o.y * f1));
+          }
+          m0 = n0;
+          m1 = n1;
+        }
+        p0 = valid ? exp2f(s0v - m0) : 0.f;
+        p1 = valid ? exp2f(s1v - m1) : 0.f;
+        l0 += p0;
+        l1 += p1;
+        if (valid) {
+#pragma unroll 2
+          for (int c = 0; c < 16; ++c) {
+            const uint4 w = __ldg(vr + c);
+            const float2 a = h2f(w.x), bb = h2f(w.y), cc = h2f(w.z), d = h2f(w.w);
+            const float vals[8] = {a.x, a.y, bb.x, bb.y, cc.x, cc.y, d.x, d.y};
+            float2 o[8];
+#pragma unroll
+            for (int e = 0; e < 8; ++e) o[e] = lds2(ab + (c * 8 + e) * 256);
+#pragma unroll
+            for (int e = 0; e < 8; ++e) sts2(ab + (c * 8 + e) * 256, fma2(p0, p1, vals[e], o[e]));
+          }
+        }
       }
     }
+
+    // ---- merge lanes and warps per query head into one partial
+    l0 = group_sum<TS>(l0);
+    l1 = group_sum<TS>(l1);
+    if (ts == 0) {
+      red_m[warp * G + 2 * hg] = m0;
+      red_m[warp * G + 2 * hg + 1] = m1;
+      red_l[warp * G + 2 * hg] = l0;
+      red_l[warp * G + 2 * hg + 1] = l1;
+    }
+    __syncthreads();
+    for (int o = threadIdx.x; o < G * kHeadDim; o += NT) {
+      const int hd = o / kHeadDim, dd = o % kHeadDim;
+      const int grp = hd >> 1, j = hd & 1;
+      float M = -INFINITY;
+#pragma unroll
+      for (int w = 0; w < NW; ++w) M = fmaxf(M, red_m[w * G + hd]);
+      float tot = 0.f, L = 0.f;
+#pragma unroll
+      for (int w = 0; w < NW; ++w) {
+        const float mw = red_m[w * G + hd];
+        const float f = (mw == -INFINITY) ? 0.f : exp2f(mw - M);
+        const float* a = accs + (size_t)w * kHeadDim * 64 + dd * 64 + j;
+        float sum = 0.f;
+#pragma unroll 4
+        for (int jj = 0; jj < TS; ++jj) sum += a[2 * (grp * TS + ((jj + dd) % TS))];
+        tot = fmaf(f, sum, tot);
+        L = fmaf(f, red_l[w * G + hd], L);
+      }
+      float* dst = p.partials + ((size_t)(blockIdx.x + u) * G + hd) * (kHeadDim + 2);
+      dst[2 + dd] = tot;
+      if (dd == 0) {
+        dst[0] = M;
+        dst[1] = L;
+      }
+    }
+    finish_unit<G, NT>(p, u, b, h, qrep, flag);
   }
 }
 
@@ -554,6 +951,33 @@ cudaError_t launch_decode_t(const DecodeParams& p, int grid, cudaStream_t s) {
 }
 
 template <int G, int MAXC>
+cudaError_t launch_gqa_t(const DecodeParams& p, int grid, cudaStream_t s) {
+  static bool attr_set = false;
+  constexpr size_t smem = 7 * kPairRegionBytes;
+  if (!attr_set) {
+    cudaError_t e = cudaFuncSetAttribute(decode_gqa_kernel<G, MAXC>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    attr_set = true;
+  }
+  decode_gqa_kernel<G, MAXC><<<grid, kGqaWarps * 32, smem, s>>>(p);
+  return cudaGetLastError();
+}
+
+template <int G, int MAXC>
+int gqa_ctas_per_sm_t() {
+  constexpr size_t smem = 7 * kPairRegionBytes;
+  if (cudaFuncSetAttribute(decode_gqa_kernel<G, MAXC>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           (int)smem) != cudaSuccess)
+    return 0;
+  int n = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, decode_gqa_kernel<G, MAXC>, kGqaWarps * 32,
+                                                    smem) != cudaSuccess)
+    return 0;
+  return n;
+}
+
+template <int G, int MAXC>
 int ctas_per_sm_t() {
   const size_t smem = decode_smem_bytes(G, MAXC * 8);
   if (cudaFuncSetAttribute(decode_kernel<G, MAXC>, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -578,8 +1002,8 @@ int decode_ctas_per_sm(int G, int k_slots) {
   const bool big = k_slots > 64;
   switch (G) {
     case 1: return big ? ctas_per_sm_t<1, 16>() : ctas_per_sm_t<1, 8>();
-    case 2: return big ? ctas_per_sm_t<2, 16>() : ctas_per_sm_t<2, 8>();
-    case 4: return big ? ctas_per_sm_t<4, 16>() : ctas_per_sm_t<4, 8>();
+    case 2: return big ? gqa_ctas_per_sm_t<2, 16>() : gqa_ctas_per_sm_t<2, 8>();
+    case 4: return big ? gqa_ctas_per_sm_t<4, 16>() : gqa_ctas_per_sm_t<4, 8>();
     default: return 0;
   }
 }
@@ -588,8 +1012,8 @@ cudaError_t launch_decode(const DecodeParams& p, int G, int k_read, int grid, cu
   const bool big = k_read > 64;
   switch (G) {
     case 1: return big ? launch_decode_t<1, 16>(p, grid, s) : launch_decode_t<1, 8>(p, grid, s);
-    case 2: return big ? launch_decode_t<2, 16>(p, grid, s) : launch_decode_t<2, 8>(p, grid, s);
-    case 4: return big ? launch_decode_t<4, 16>(p, grid, s) : launch_decode_t<4, 8>(p, grid, s);
+    case 2: return big ? launch_gqa_t<2, 16>(p, grid, s) : launch_gqa_t<2, 8>(p, grid, s);
+    case 4: return big ? launch_gqa_t<4, 16>(p, grid, s) : launch_gqa_t<4, 8>(p, grid, s);
     default: return cudaErrorInvalidValue;
   }
 }

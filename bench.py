@@ -73,10 +73,14 @@ def decode_kernel_traffic(workload: str):
     it was taken on the current kernel source (else None)."""
     src = os.path.join(ROOT, "paper_2511_18936_gb300", "csrc", "decode.cu")
     digest = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
-    path = os.path.join(ROOT, "profiles", f"decode_kernel_{workload}.md")
-    try:
-        text = open(path).read()
-    except OSError:
+    text = None
+    for name in (f"decode_kernel_{workload}.md", f"decode_gqa_kernel_{workload}.md"):
+        try:
+            text = open(os.path.join(ROOT, "profiles", name)).read()
+            break
+        except OSError:
+            continue
+    if text is None:
         return None
     m_src = re.search(r"decode\.cu sha256\[:16\]:\s*([0-9a-f]{16})", text)
     m_tr = re.search(r"dram bytes per launch:\s*([0-9.eE+]+)", text)
@@ -223,6 +227,20 @@ def cpu_baseline_leg(wl, budget_s: float = 15.0):
 # ---------------------------------------------------------------------------
 # The CUDA path
 # ---------------------------------------------------------------------------
+
+def aggregate_ranks(kv_tokens: float, ms: float, e2e_tokens: float, e2e_s: float, world: int,
+                    device=None):
+    """Whole-job throughput over ``world`` replicas: every rank processed the
+    same number of tokens; the job time is the slowest rank's (MAX over
+    ranks).  Returns (value, e2e_value, max_ms)."""
+    t_max, e2e_max = ms, e2e_s
+    if world > 1:
+        import torch
+        tt = torch.tensor([ms, e2e_s], dtype=torch.float64, device=device)
+        torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
+        t_max, e2e_max = float(tt[0]), float(tt[1])
+    return world * kv_tokens / (t_max / 1e3), world * e2e_tokens / e2e_max, t_max
+
 
 class LayerRun:
     """One attention layer (the 1-head, 32k, GQA-131k and k-sweep workloads):
@@ -444,13 +462,7 @@ def run_swan(args, wl, rank: int, world: int, local_rank: int):
     # ---- aggregate over ranks ----------------------------------------------
     ctxs = [run.context_after(i) for i in steps]
     kv_tokens = sum(B * H_kv * (sp + bf) * run.layers for sp, bf in ctxs)
-    t_max, e2e_max = ms, e2e_s
-    if world > 1:
-        tt = torch.tensor([ms, e2e_s], device=dev, dtype=torch.float64)
-        torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
-        t_max, e2e_max = float(tt[0]), float(tt[1])
-    value = world * kv_tokens / (t_max / 1e3)
-    e2e_value = world * e2e_tokens / e2e_max
+    value, e2e_value, t_max = aggregate_ranks(kv_tokens, ms, e2e_tokens, e2e_s, world, dev)
 
     dec_ms, dec_n = kt["decode"]
     avg_dec_s = dec_ms / 1e3 / max(dec_n, 1)

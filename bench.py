@@ -376,7 +376,7 @@ def run_swan(args, wl, rank: int, world: int, local_rank: int):
     dev = torch.device("cuda", local_rank)
     torch.cuda.set_device(dev)
     B, H_q, H_kv, k = wl["B"], wl["H_q"], wl["H_kv"], wl["k"]
-    steps_total = args.warmup + args.steps + 2 * args.e2e_steps
+    steps_total = args.warmup + 2 * args.steps + 2 * args.e2e_steps
     stream = torch.cuda.Stream(dev)
     seed = args.seed + rank
     kind = wl.get("kind", "layer")
@@ -395,42 +395,52 @@ def run_swan(args, wl, rank: int, world: int, local_rank: int):
         if world > 1:
             torch.distributed.barrier()
 
-    # ---- timed region: inputs resident in HBM -----------------------------
-    steps = range(args.warmup, args.warmup + args.steps)
-    launches0 = ctx.launch_count()
-    ctx.timing_enable(True)
-    barrier()
-    torch.cuda.synchronize(dev)
-    with ClockSampler(local_rank) as clk:
+    def timed(step_range):
+        """CUDA-event time of the steps on the context's stream (ms)."""
         if not flush_l2:
             ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
             ev0.record(stream)
-            for i in steps:
+            for i in step_range:
                 run.step(i)
             ev1.record(stream)
             stream.synchronize()
-            ms = ev0.elapsed_time(ev1)
-        else:
-            # L2-resident workload: flush L2 (write 512 MB) between timed steps
-            ms = 0.0
-            for i in steps:
-                with torch.cuda.stream(stream):
-                    l2_buf.zero_()
-                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-                e0.record(stream)
-                run.step(i)
-                e1.record(stream)
-                stream.synchronize()
-                ms += e0.elapsed_time(e1)
+            return ev0.elapsed_time(ev1)
+        # L2-resident workload: flush L2 (write 512 MB) before every timed step
+        total = 0.0
+        for i in step_range:
+            with torch.cuda.stream(stream):
+                l2_buf.zero_()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            run.step(i)
+            e1.record(stream)
+            stream.synchronize()
+            total += e0.elapsed_time(e1)
+        return total
+
+    # ---- timed region: inputs resident in HBM -----------------------------
+    steps = range(args.warmup, args.warmup + args.steps)
+    launches0 = ctx.launch_count()
     barrier()
     torch.cuda.synchronize(dev)
+    with ClockSampler(local_rank) as clk:
+        ms = timed(steps)
+    barrier()
+    torch.cuda.synchronize(dev)
+    launches = ctx.launch_count() - launches0
+
+    # ---- per-kernel CUDA-event times over a second timed region of the same
+    # length (events between launches would hide the launch overlap above)
+    ksteps = range(args.warmup + args.steps, args.warmup + 2 * args.steps)
+    ctx.timing_enable(True)
+    torch.cuda.synchronize(dev)
+    timed(ksteps)
     kt = ctx.timing_read()
     ctx.timing_enable(False)
-    launches = ctx.launch_count() - launches0
 
     # ---- end to end: pinned host inputs, H2D copies and the D2H read inside -
     e2e_steps = args.e2e_steps
-    base = args.warmup + args.steps
+    base = args.warmup + 2 * args.steps
     host = [[t.cpu().pin_memory() for t in run.host_inputs(base + i)] for i in range(2 * e2e_steps)]
     dev_in = [torch.empty_like(t, device=dev) for t in host[0]]
     host_out = [torch.empty_like(run.out, device="cpu").pin_memory()]
@@ -466,8 +476,9 @@ def run_swan(args, wl, rank: int, world: int, local_rank: int):
 
     dec_ms, dec_n = kt["decode"]
     avg_dec_s = dec_ms / 1e3 / max(dec_n, 1)
-    sp_mean = statistics.mean(sp for sp, _ in ctxs)
-    bf_mean = statistics.mean(bf for _, bf in ctxs)
+    kctxs = [run.context_after(i) for i in ksteps]  # the region the kernels were timed on
+    sp_mean = statistics.mean(sp for sp, _ in kctxs)
+    bf_mean = statistics.mean(bf for _, bf in kctxs)
     # algorithmic bytes of one decode-kernel launch (one layer): per (sparse
     # token, kv head) 2 * 3 * k bytes (fp16 value + uint8 index for K and V);
     # per (buffer token, kv head) 2 * 2 * d bytes
@@ -476,10 +487,13 @@ def run_swan(args, wl, rank: int, world: int, local_rank: int):
     peaks = measured_peaks()
     peak = float(peaks["hbm_gbs"]) if peaks else 6800.0
     step_s = t_max / 1e3 / args.steps
+    sp_step = statistics.mean(sp for sp, _ in ctxs)
+    bf_step = statistics.mean(bf for _, bf in ctxs)
+    alg_decode_step = B * H_kv * (sp_step * 6 * k + bf_step * 4 * D)
     # whole-step algorithmic bytes per layer: decode reads + q/out (fp16) + R
     # (fp32, once per kv head, query and value rotations) + the append's new
     # vectors (fp16 in, fp16 to the buffer)
-    alg_step = run.layers * (alg_decode + 2 * B * H_q * D * 2 + 2 * H_kv * D * D * 4
+    alg_step = run.layers * (alg_decode_step + 2 * B * H_q * D * 2 + 2 * H_kv * D * D * 4
                              + B * H_kv * 2 * D * 2 * 2)
     l2_note = ("L2 flushed (512 MB written) before every timed step" if flush_l2 else
                f"inputs larger than L2: {alg_decode * run.layers / 1e9:.2f} GB read per step, no flush")
@@ -506,6 +520,7 @@ def run_swan(args, wl, rank: int, world: int, local_rank: int):
                      "alg_bytes_per_launch": alg_decode, "avg_launch_ms": avg_dec_s * 1e3,
                      "traffic": decode_kernel_traffic(args.workload)},
         "kernels_ms_per_step": {name: v[0] / args.steps for name, v in kt.items() if v[1]},
+        "kernels_timed": "second timed region of the same length, CUDA events around every launch",
         "gpu_launches": launches,
         "e2e": {"value": e2e_value, "unit": "KV-tokens/s", "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h, "steps": e2e_steps},

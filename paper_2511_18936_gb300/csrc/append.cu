@@ -108,7 +108,9 @@ __global__ void __launch_bounds__(kThreads, 1) append_kernel(AppendParams p) {
   const __half* X = kind ? p.v_new : p.k_new;
   __half* ring = kind ? p.ring_v : p.ring_k;
 
+  pdl_trigger();
   stage_matrix(Rs, R);
+  pdl_wait();
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int64_t nvec = (int64_t)p.B * p.T;
@@ -193,21 +195,25 @@ __global__ void __launch_bounds__(kThreads, 1) append_kernel(AppendParams p) {
 // computes coordinates 4l..4l+3 from R in shared memory, in the same fp32
 // order as append_kernel) and either prunes them or writes them to the ring.
 // Ring slots freed in phase 1 are reused in phase 2 only after the barrier.
-__global__ void __launch_bounds__(kThreads) append_small_kernel(AppendParams p, int evict_old) {
+__global__ void __launch_bounds__(kThreads) append_small_kernel(AppendParams p, int evict_old, int bpc) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   float* Rs = reinterpret_cast<float*>(smem_raw);
   const int kind = blockIdx.y;
   const int h = blockIdx.x;
+  const int b0 = blockIdx.z * bpc;                 // this CTA's sequences: [b0, b0 + nb)
+  const int nb = min(bpc, p.B - b0);
   const float* R = (kind ? p.R_vo : p.R_qk) + (size_t)h * kHeadDim * kHeadDim;
   const __half* X = kind ? p.v_new : p.k_new;
   __half* ring = kind ? p.ring_v : p.ring_k;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
+  pdl_trigger();
   stage_matrix(Rs, R);
+  pdl_wait();
 
   // phase 1: evict the oldest buffered vectors (sparse positions L_s + i)
-  for (int item = warp; item < p.B * evict_old; item += kWarpsPerCta) {
-    const int b = item / evict_old, i = item % evict_old;
+  for (int item = warp; item < nb * evict_old; item += kWarpsPerCta) {
+    const int b = b0 + item / evict_old, i = item % evict_old;
     const int64_t unit = (int64_t)b * p.H + h;
     const int slot = (p.buf_start + i) % p.cap;
     const uint2 raw = __ldg(reinterpret_cast<const uint2*>(ring + (unit * p.cap + slot) * kHeadDim) + lane);
@@ -216,8 +222,8 @@ __global__ void __launch_bounds__(kThreads) append_small_kernel(AppendParams p, 
   __syncthreads();
 
   // phase 2: the new vectors
-  for (int item = warp; item < p.B * p.T; item += kWarpsPerCta) {
-    const int b = item / p.T, j = item % p.T;
+  for (int item = warp; item < nb * p.T; item += kWarpsPerCta) {
+    const int b = b0 + item / p.T, j = item % p.T;
     const int64_t unit = (int64_t)b * p.H + h;
     const uint2 xw = __ldg(reinterpret_cast<const uint2*>(X + ((unit * p.T) + j) * kHeadDim) + lane);
     const float2 x01 = __half22float2(*reinterpret_cast<const __half2*>(&xw.x));
@@ -250,6 +256,8 @@ __global__ void __launch_bounds__(kThreads) append_small_kernel(AppendParams p, 
 
 // One warp per (unit, buffered token, K or V): read the ring row and prune.
 __global__ void __launch_bounds__(kThreads) prune_ring_kernel(PruneRingParams p) {
+  pdl_trigger();
+  pdl_wait();
   const int lane = threadIdx.x & 31;
   const int64_t gw = ((int64_t)blockIdx.x * kThreads + threadIdx.x) >> 5;
   const int64_t total = (int64_t)p.units * p.count * 2;
@@ -289,8 +297,7 @@ cudaError_t launch_append(const AppendParams& p, cudaStream_t s) {
   }
   const int64_t nvec = (int64_t)p.B * p.T;
   dim3 grid((unsigned)((nvec + kThreads - 1) / kThreads), (unsigned)p.H, 2);
-  append_kernel<<<grid, kThreads, kAppendSmem, s>>>(p);
-  return cudaGetLastError();
+  return launch_pdl(append_kernel, grid, dim3(kThreads), kAppendSmem, s, p);
 }
 
 cudaError_t launch_append_small(const AppendParams& p, int evict_old, cudaStream_t s) {
@@ -302,15 +309,17 @@ cudaError_t launch_append_small(const AppendParams& p, int evict_old, cudaStream
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
-  append_small_kernel<<<dim3((unsigned)p.H, 2), kThreads, smem, s>>>(p, evict_old);
-  return cudaGetLastError();
+  // enough sequences per CTA for one vector per warp and phase
+  const int per = max(p.T, evict_old);
+  const int bpc = max(1, kWarpsPerCta / max(per, 1));
+  return launch_pdl(append_small_kernel, dim3((unsigned)p.H, 2, (unsigned)((p.B + bpc - 1) / bpc)),
+                    dim3(kThreads), smem, s, p, evict_old, bpc);
 }
 
 cudaError_t launch_prune_ring(const PruneRingParams& p, cudaStream_t s) {
   const int64_t warps = (int64_t)p.units * p.count * 2;
   const int64_t blocks = (warps + kWarpsPerCta - 1) / kWarpsPerCta;
-  prune_ring_kernel<<<(unsigned)blocks, kThreads, 0, s>>>(p);
-  return cudaGetLastError();
+  return launch_pdl(prune_ring_kernel, dim3((unsigned)blocks), dim3(kThreads), 0, s, p);
 }
 
 cudaError_t launch_transpose_r(const float* src, float* dst, int64_t mats, cudaStream_t s) {

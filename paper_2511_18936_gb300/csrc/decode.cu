@@ -210,6 +210,7 @@ __global__ void __launch_bounds__(decode_warps<G, MAXC>() * 32, 1) decode_kernel
   constexpr bool kL1 = G > 1;
   extern __shared__ __align__(16) unsigned char smem_raw[];
   __shared__ float red_m[NW], red_l[NW];
+  pdl_trigger();
 
   const uint32_t raw = (uint32_t)__cvta_generic_to_shared(smem_raw);
   const uint32_t base = (raw + kRegionBytes - 1) & ~(kRegionBytes - 1);
@@ -242,6 +243,7 @@ __global__ void __launch_bounds__(decode_warps<G, MAXC>() * 32, 1) decode_kernel
 
   const int64_t g_begin = (int64_t)blockIdx.x * p.range;
   const int64_t g_end = min(p.total_groups, g_begin + p.range);
+  pdl_wait();
   if (g_begin >= g_end) return;
   const int64_t u_first = g_begin / p.N_g, u_last = (g_end - 1) / p.N_g;
   const int n_sg = (int)p.n_sg;
@@ -581,6 +583,7 @@ __global__ void __launch_bounds__(kGqaWarps * 32, 1) decode_gqa_kernel(DecodePar
   constexpr int HALVES = 32 / TS;     // iterations per 32-token block
   extern __shared__ __align__(16) unsigned char smem_raw[];
   __shared__ float red_m[NW * G], red_l[NW * G], flag[1];
+  pdl_trigger();
 
   const uint32_t raw = (uint32_t)__cvta_generic_to_shared(smem_raw);
   const uint32_t base = (raw + kPairRegionBytes - 1) & ~(kPairRegionBytes - 1);
@@ -610,6 +613,7 @@ __global__ void __launch_bounds__(kGqaWarps * 32, 1) decode_gqa_kernel(DecodePar
 
   const int64_t g_begin = (int64_t)blockIdx.x * p.range;
   const int64_t g_end = min(p.total_groups, g_begin + p.range);
+  pdl_wait();
   if (g_begin >= g_end) return;
   const int64_t u_first = g_begin / p.N_g, u_last = (g_end - 1) / p.N_g;
   const int n_sg = (int)p.n_sg;
@@ -874,10 +878,14 @@ __global__ void __launch_bounds__(kThreads) rotate_q_kernel(RotateQParams p, int
   float* Rs = reinterpret_cast<float*>(smem_raw);
   const int h = blockIdx.x;
   const float* R = p.R_qk + (size_t)h * kHeadDim * kHeadDim;
+  pdl_trigger();
   stage_matrix(Rs, R);
   __syncthreads();
+  pdl_wait();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  for (int item = warp; item < B * p.G; item += kWarpsPerCta) {
+  // this CTA's query vectors: [blockIdx.y * 8, blockIdx.y * 8 + 8) of the B * G of head h
+  for (int item = blockIdx.y * kWarpsPerCta + warp; item < min(B * p.G, (int)(blockIdx.y + 1) * kWarpsPerCta);
+       item += kWarpsPerCta) {
     const int b = item / p.G, gh = item % p.G;
     const int64_t bq = (int64_t)b * p.H_q + h * p.G + gh;
     const uint2 xw = __ldg(reinterpret_cast<const uint2*>(p.q + bq * kHeadDim) + lane);
@@ -902,6 +910,8 @@ __global__ void __launch_bounds__(kThreads) rotate_q_kernel(RotateQParams p, int
 // R_vo^T and round to fp16.
 __global__ void __launch_bounds__(kHeadDim) combine_kernel(CombineParams p) {
   __shared__ float o_hat[kHeadDim];
+  pdl_trigger();
+  pdl_wait();
   const int64_t bq = blockIdx.x;
   const int64_t b = bq / p.H_q;
   const int hq = (int)(bq % p.H_q);
@@ -946,8 +956,7 @@ cudaError_t launch_decode_t(const DecodeParams& p, int grid, cudaStream_t s) {
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
-  decode_kernel<G, MAXC><<<grid, decode_warps<G, MAXC>() * 32, smem, s>>>(p);
-  return cudaGetLastError();
+  return launch_pdl(decode_kernel<G, MAXC>, dim3(grid), dim3(decode_warps<G, MAXC>() * 32), smem, s, p);
 }
 
 template <int G, int MAXC>
@@ -960,8 +969,7 @@ cudaError_t launch_gqa_t(const DecodeParams& p, int grid, cudaStream_t s) {
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
-  decode_gqa_kernel<G, MAXC><<<grid, kGqaWarps * 32, smem, s>>>(p);
-  return cudaGetLastError();
+  return launch_pdl(decode_gqa_kernel<G, MAXC>, dim3(grid), dim3(kGqaWarps * 32), smem, s, p);
 }
 
 template <int G, int MAXC>
@@ -1027,13 +1035,14 @@ cudaError_t launch_rotate_q(const RotateQParams& p, int B, cudaStream_t s) {
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
-  rotate_q_kernel<<<(unsigned)(p.H_q / p.G), kThreads, smem, s>>>(p, B);
-  return cudaGetLastError();
+  const int vecs = B * p.G;  // query vectors per kv head
+  return launch_pdl(rotate_q_kernel,
+                    dim3((unsigned)(p.H_q / p.G), (unsigned)((vecs + kWarpsPerCta - 1) / kWarpsPerCta)),
+                    dim3(kThreads), smem, s, p, B);
 }
 
 cudaError_t launch_combine(const CombineParams& p, int B, cudaStream_t s) {
-  combine_kernel<<<(unsigned)((int64_t)B * p.H_q), kHeadDim, 0, s>>>(p);
-  return cudaGetLastError();
+  return launch_pdl(combine_kernel, dim3((unsigned)((int64_t)B * p.H_q)), dim3(kHeadDim), 0, s, p);
 }
 
 }  // namespace swan

@@ -35,6 +35,9 @@ Readings where the paper is silent (each listed in the design notes):
 * Kept entries are stored in decreasing magnitude order, so a smaller
   runtime keep count is a prefix of a larger one.
 * The score scale is ``1/sqrt(d_h)`` with the full head dimension.
+* With 8-bit values (Section 4.3, Section 5.1) the format is E4M3, the kept
+  entries are chosen on the fp16 vector and then rounded to nearest even,
+  saturating to +-448; the dense buffer stays fp16.
 * The rotated query is not rounded.
 * Query head ``h`` attends to kv head ``h // G`` (the reshape of Section
   4.1.1 groups consecutive query heads).
@@ -91,6 +94,21 @@ def prune(x16, k: int):
     order = np.argsort(-mag, axis=-1, kind="stable")[..., :k]
     vals = np.take_along_axis(x16, order, axis=-1)
     return order.astype(np.uint8), vals
+
+
+def to_e4m3(x) -> np.ndarray:
+    """Round to the 8-bit float E4M3 (1 sign, 4 exponent bits with bias 7,
+    3 mantissa bits, no infinities; largest finite value 448, subnormal
+    spacing 2^-9), round-to-nearest-even, saturating to +-448.  Returns the
+    rounded values as fp64.  (Section 4.3 and Section 5.1 store the kept
+    values as 8-bit floats; the format is E4M3.)"""
+    x = np.asarray(x, np.float64)
+    a = np.abs(x)
+    e = np.floor(np.log2(np.maximum(a, 2.0 ** -30)))
+    e = np.maximum(e, -6.0)                    # below 2^-6 the spacing stays 2^-9
+    q = np.exp2(e - 3.0)                       # spacing of the binade: 3 mantissa bits
+    r = np.minimum(np.round(a / q) * q, 448.0)  # np.round: halves to even
+    return np.copysign(r, x)
 
 
 def densify(idx, vals, d: int) -> np.ndarray:
@@ -192,7 +210,7 @@ class SwanOracle:
     """
 
     def __init__(self, R_qk, R_vo=None, *, batch: int, n_q_heads: int, k_store: int,
-                 buffer_cap: int, round_rotated: bool = True):
+                 buffer_cap: int, round_rotated: bool = True, value_format: str = "fp16"):
         self.R_qk = np.asarray(R_qk, np.float64)
         self.R_vo = self.R_qk if R_vo is None else np.asarray(R_vo, np.float64)
         self.H_kv, self.d, _ = self.R_qk.shape
@@ -207,6 +225,9 @@ class SwanOracle:
         self.k_active = k_store
         self.b = buffer_cap
         self.round = round_rotated
+        if value_format not in ("fp16", "fp8_e4m3"):
+            raise ValueError("value_format must be fp16 or fp8_e4m3")
+        self.fp8 = value_format == "fp8_e4m3"
         vdt = np.float16 if round_rotated else np.float64
         self.buf_k = np.zeros((self.B, self.H_kv, 0, self.d), vdt)
         self.buf_v = np.zeros((self.B, self.H_kv, 0, self.d), vdt)
@@ -222,7 +243,11 @@ class SwanOracle:
 
     def _prune(self, x):
         if self.round:
-            return prune(x, self.k_store)
+            idx, vals = prune(x, self.k_store)
+            if self.fp8:
+                # the kept fp16 values are stored as E4M3 (exact in fp16)
+                vals = to_e4m3(vals.astype(np.float64)).astype(np.float16)
+            return idx, vals
         # fp64 variant (lemma checks only): same rule on the fp64 vector
         mag = np.abs(x)
         order = np.argsort(-mag, axis=-1, kind="stable")[..., : self.k_store]

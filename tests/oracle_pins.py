@@ -242,6 +242,41 @@ def pin_formulas(o):
     assert abs(o.compression_ratio(64, 128) - 194 / 256) < 1e-15
 
 
+# -- 8-bit value rounding (E4M3) against torch's float8_e4m3fn ------------
+
+def pin_e4m3_rounding(o):
+    h = np.arange(65536, dtype=np.uint16).view(np.float16)
+    h = h[np.isfinite(h)].astype(np.float64)
+    got = o.to_e4m3(h)
+    inr = np.abs(h) < 464.0  # torch turns |x| >= 480 into NaN instead of saturating
+    ref = torch.from_numpy(h[inr].astype(np.float32)).to(torch.float8_e4m3fn).double().numpy()
+    assert np.array_equal(got[inr], ref)
+    assert np.all(np.abs(got[~inr]) == 448.0) and np.array_equal(np.sign(got[~inr]), np.sign(h[~inr]))
+    # every E4M3 value is its own rounding; ties go to the even neighbour
+    assert np.array_equal(o.to_e4m3(got), got)
+    assert o.to_e4m3(1.0625) == 1.0 and o.to_e4m3(1.1875) == 1.25 and o.to_e4m3(2.0 ** -10) == 0.0
+
+
+def pin_fp8_cache_is_rounded_sparse_cache(o):
+    """The fp8 cache holds the same indices as the fp16 cache (selection on
+    the fp16 vector) with the kept values rounded to E4M3; decoding it equals
+    dense attention on the zero-filled rounded vectors."""
+    R, Rv, k, v, q = _small_problem(61, B=1, H_kv=1, d=32, L=40)
+    a = o.SwanOracle(R, Rv, batch=1, n_q_heads=1, k_store=12, buffer_cap=5)
+    b = o.SwanOracle(R, Rv, batch=1, n_q_heads=1, k_store=12, buffer_cap=5, value_format="fp8_e4m3")
+    a.append(k, v)
+    b.append(k, v)
+    assert np.array_equal(a.sp_idx_k, b.sp_idx_k) and np.array_equal(a.sp_idx_v, b.sp_idx_v)
+    assert np.array_equal(b.sp_val_k.astype(np.float64), o.to_e4m3(a.sp_val_k.astype(np.float64)))
+    assert np.array_equal(a.buf_k.view(np.uint16), b.buf_k.view(np.uint16))
+    Kd = np.concatenate([o.densify(b.sp_idx_k[0, 0], b.sp_val_k[0, 0], 32), b.buf_k[0, 0].astype(np.float64)])
+    Vd = np.concatenate([o.densify(b.sp_idx_v[0, 0], b.sp_val_v[0, 0], 32), b.buf_v[0, 0].astype(np.float64)])
+    qh = q[0, 0].astype(np.float64) @ R[0].astype(np.float64)
+    ref = o.dense_attention(qh, Kd, Vd) @ Rv[0].astype(np.float64).T
+    assert np.abs(b.decode(q)[0, 0] - ref).max() < 1e-12
+
+
 ALL_PINS = [pin_rotation_orthogonal, pin_rotation_orientation, pin_prune_bruteforce,
             pin_k_equals_d_is_dense, pin_decompression_free, pin_buffer_semantics,
-            pin_split_combine, pin_k_prefix, pin_gqa_mapping, pin_formulas]
+            pin_split_combine, pin_k_prefix, pin_gqa_mapping, pin_formulas, pin_e4m3_rounding,
+            pin_fp8_cache_is_rounded_sparse_cache]

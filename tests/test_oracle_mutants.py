@@ -54,6 +54,14 @@ MUTANTS = [
     ("bytes_without_offset",
      "return k * (value_bytes + index_bytes) + offset_bytes",
      "return k * (value_bytes + index_bytes)", 1),
+    ("e4m3_two_mantissa_bits",
+     "q = np.exp2(e - 3.0)", "q = np.exp2(e - 2.0)", 1),
+    ("e4m3_no_saturation",
+     "r = np.minimum(np.round(a / q) * q, 448.0)", "r = np.round(a / q) * q", 1),
+    ("e4m3_no_subnormals",
+     "e = np.maximum(e, -6.0)", "e = np.maximum(e, -30.0)", 1),
+    ("fp8_values_not_rounded",
+     "vals = to_e4m3(vals.astype(np.float64)).astype(np.float16)", "vals = vals", 1),
     ("runtime_k_ignored",
      "s_sp = sparse_scores(q_hat, sp_idx[:, :ka], sp_vals_k[:, :ka])",
      "s_sp = sparse_scores(q_hat, sp_idx, sp_vals_k)", 1),

@@ -260,7 +260,7 @@ class LayerRun:
             R = torch.from_numpy(synth.rotations(H_kv, D, seed=seed, workload=1, layer=0))[None].to(dev)
             self.ctx = swan.Context(R, num_layers=1, batch=B, n_q_heads=H_q, n_kv_heads=H_kv,
                                     k_store=wl["k_store"], buffer_cap=n_b, max_seq=self.max_seq,
-                                    stream=stream)
+                                    stream=stream, value_format=wl["values"])
             kk = synth.torch_lowrank_kv(B, H_kv, L_s + n_b, D, seed, synth.T_K, dev)
             vv = synth.torch_lowrank_kv(B, H_kv, L_s + n_b, D, seed, synth.T_V, dev)
             self.ctx.append(0, kk, vv)
@@ -315,7 +315,7 @@ class StackRun:
             Rt = torch.from_numpy(R).to(dev)
             self.ctx = swan.Context(Rt, num_layers=Lyr, batch=B, n_q_heads=H, n_kv_heads=H,
                                     k_store=wl["k_store"], buffer_cap=cap, max_seq=self.max_seq,
-                                    stream=stream)
+                                    stream=stream, value_format=wl["values"])
             self.ctx.set_k(wl["k"])
         stream.synchronize()
         # prefix: one append per layer (plain Gaussian K/V), timed on the stream
@@ -480,16 +480,17 @@ def run_swan(args, wl, rank: int, world: int, local_rank: int):
     sp_mean = statistics.mean(sp for sp, _ in kctxs)
     bf_mean = statistics.mean(bf for _, bf in kctxs)
     # algorithmic bytes of one decode-kernel launch (one layer): per (sparse
-    # token, kv head) 2 * 3 * k bytes (fp16 value + uint8 index for K and V);
-    # per (buffer token, kv head) 2 * 2 * d bytes
-    alg_decode = B * H_kv * (sp_mean * 6 * k + bf_mean * 4 * D)
+    # token, kv head) 2 * (value + index bytes) * k (K and V: 6k with fp16
+    # values, 4k with 8-bit values); per (buffer token, kv head) 2 * 2 * d
+    ent = 4 if wl["values"] == "fp8_e4m3" else 6
+    alg_decode = B * H_kv * (sp_mean * ent * k + bf_mean * 4 * D)
     achieved = alg_decode / avg_dec_s / 1e9
     peaks = measured_peaks()
     peak = float(peaks["hbm_gbs"]) if peaks else 6800.0
     step_s = t_max / 1e3 / args.steps
     sp_step = statistics.mean(sp for sp, _ in ctxs)
     bf_step = statistics.mean(bf for _, bf in ctxs)
-    alg_decode_step = B * H_kv * (sp_step * 6 * k + bf_step * 4 * D)
+    alg_decode_step = B * H_kv * (sp_step * ent * k + bf_step * 4 * D)
     # whole-step algorithmic bytes per layer: decode reads + q/out (fp16) + R
     # (fp32, once per kv head, query and value rotations) + the append's new
     # vectors (fp16 in, fp16 to the buffer)
@@ -500,7 +501,8 @@ def run_swan(args, wl, rank: int, world: int, local_rank: int):
     cfg = {"workload": args.workload, "desc": wl["desc"], "batch": B, "n_q_heads": H_q,
            "n_kv_heads": H_kv, "layers": run.layers, "sparse_tokens": wl.get("L_s", wl.get("prefix")),
            "buffer_tokens": wl["n_b"], "k": k, "k_store": wl["k_store"],
-           "storage": "fp16 values + uint8 indices (sparse), fp16 (buffer)", "l2": l2_note,
+           "storage": ("e4m3" if wl["values"] == "fp8_e4m3" else "fp16")
+                      + " values + uint8 indices (sparse), fp16 (buffer)", "l2": l2_note,
            "parallelism": f"replicas x{world} (independent batches per GPU)" if world > 1
            else "single GPU"}
     line = {
@@ -546,12 +548,17 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--batch", type=int, default=0,
                     help="override the workload's batch (smaller cases for profiling)")
+    ap.add_argument("--values", default="fp16", choices=["fp16", "fp8_e4m3"],
+                    help="kept sparse values as fp16 (3k bytes per vector) or E4M3 (2k)")
     ap.add_argument("--k-active", type=int, default=0,
                     help="runtime keep count (ksweep-32k: 32, 48, 64, 96 or 128)")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
     wl = dict(WORKLOADS[args.workload])
+    wl["values"] = args.values
+    if args.values != "fp16":
+        wl["desc"] += f" ({args.values} values)"
     if args.batch:
         wl["B"] = args.batch
         wl["desc"] += f" (batch overridden to {args.batch})"

@@ -74,7 +74,15 @@ typedef struct swan_config {
   int page_tokens; /* tokens per cache page, a power of two in [32, 4096];
                       0 = 128 */
   void* stream;    /* cudaStream_t the context enqueues on; NULL = default */
+  int value_format; /* SWAN_VALUES_FP16 (0, default) or SWAN_VALUES_FP8_E4M3:
+                       kept sparse values stored as 8-bit floats (Section 4.3,
+                       Section 5.1: 2k bytes per vector instead of 3k),
+                       E4M3, round to nearest even, saturating to +-448; the
+                       entries are still chosen on the fp16 vector and the
+                       dense buffer stays fp16 */
 } swan_config;
+
+enum { SWAN_VALUES_FP16 = 0, SWAN_VALUES_FP8_E4M3 = 1 };
 
 /*
  * Create a context.  R_qk, R_vo: device fp32 [num_layers][n_kv_heads][d][d],
@@ -148,6 +156,7 @@ typedef struct swan_layer_info {
   int page_tokens;
   int64_t page_bytes;   /* bytes of one page (keys and values) */
   int64_t device_bytes; /* device memory owned by the whole context */
+  int value_format;     /* SWAN_VALUES_FP16 or SWAN_VALUES_FP8_E4M3 */
 } swan_layer_info;
 
 swan_status swan_query(const swan_ctx* ctx, int layer, swan_layer_info* info);
@@ -159,7 +168,8 @@ swan_status swan_query(const swan_ctx* ctx, int layer, swan_layer_info* info);
  *     oldest first.
  *   SWAN_EXPORT_SPARSE_K / _V: uint8 indices [batch][n_kv_heads]
  *     [sparse_len][k_store], then fp16 values of the same shape, each vector's
- *     entries in stored (decreasing magnitude) order.
+ *     entries in stored (decreasing magnitude) order (8-bit values are
+ *     widened to fp16, exactly).
  * bytes must equal the exact size of the requested view.
  * Errors: INVALID_ARG (what, layer, size), STATE, CUDA.
  */
@@ -213,15 +223,18 @@ swan_status swan_timing_read(swan_ctx* ctx, swan_timing* out);
  *
  * view: the caller's cache, all pointers device pointers on the current
  *   device, caller-owned:
- *   pages       page pool; page p starts at pages + p * page_tokens *
- *               k_slots * 6 and holds P = page_tokens tokens as P/32 blocks
- *               of 32 tokens, block q at q * 192 * k_slots bytes.  A block
- *               holds four regions: K values [k_slots/8][32][8] fp16 at 0,
+ *   pages       page pool; page p holds P = page_tokens tokens as P/32
+ *               blocks of 32 tokens.  With fp16 values a block is
+ *               192 * k_slots bytes: K values [k_slots/8][32][8] fp16 at 0,
  *               K indices [k_slots/8][32][8] uint8 at 64 * k_slots, V values
- *               at 96 * k_slots, V indices at 160 * k_slots.  Record
- *               (chunk c, token t) holds entries 8c..8c+7 of token t's kept
- *               coordinates in decreasing magnitude order; indices must be
- *               < 128.  This is the layout swan_init's own pool uses.
+ *               at 96 * k_slots, V indices at 160 * k_slots.  With E4M3
+ *               values a block is 128 * k_slots bytes: K records
+ *               [k_slots/8][32][16 bytes] at 0 (8 E4M3 values, then 8
+ *               indices), V records at 64 * k_slots.  Page p starts at
+ *               pages + p * (P / 32) * block bytes.  Chunk c of token t holds
+ *               entries 8c..8c+7 of the token's kept coordinates in
+ *               decreasing magnitude order; indices must be < 128.  This is
+ *               the layout swan_init's own pool uses.
  *   page_table  int32 [batch * n_kv_heads][pages_per_unit]: page of the
  *               unit's sparse tokens p*P .. p*P+P-1; entries index `pages`
  *               and must be < num_pages.
@@ -266,6 +279,7 @@ typedef struct swan_cache_view {
   int head_dim;          /* must be 128 */
   const float* R_qk;
   const float* R_vo_t;
+  int value_format;      /* SWAN_VALUES_FP16 or SWAN_VALUES_FP8_E4M3 */
 } swan_cache_view;
 swan_status swan_decode_noalloc(const swan_cache_view* view, const void* q, void* out,
                                 void* stream);

@@ -1,6 +1,8 @@
 // Compress-on-append: rotation of new keys/values, dense ring-buffer insert,
 // and magnitude top-k pruning into the paged sparse cache (Algorithm 1;
 // Section 4.3; Section 5.1).
+#include <cuda_fp8.h>
+
 #include "swan_internal.h"
 
 namespace swan {
@@ -60,8 +62,6 @@ __device__ __forceinline__ void warp_prune_store(uint2 raw, int lane, int kind, 
   }
   uint8_t* blk = g.pool + (int64_t)phys * g.page_bytes + (int64_t)(slot >> 5) * g.block_bytes();
   const int t = slot & 31;
-  const int voff = kind ? g.vval_off() : 0;
-  const int ioff = kind ? g.vidx_off() : g.kidx_off();
   if (lane < (g.k_slots >> 2)) {
     const int c = lane >> 1, half = lane & 1;
     uint32_t vb[4], ib[4];
@@ -73,11 +73,28 @@ __device__ __forceinline__ void warp_prune_store(uint2 raw, int lane, int kind, 
       vb[s] = keep ? bits : 0u;
       ib[s] = keep ? j : 0u;
     }
-    const uint2 vals = make_uint2(vb[0] | (vb[1] << 16), vb[2] | (vb[3] << 16));
     const uint32_t idx = ib[0] | (ib[1] << 8) | (ib[2] << 16) | (ib[3] << 24);
     const int rec = c * 32 + t;
-    *reinterpret_cast<uint2*>(blk + voff + rec * 16 + half * 8) = vals;
-    *reinterpret_cast<uint32_t*>(blk + ioff + rec * 8 + half * 4) = idx;
+    if (g.fmt == kFmtFp8) {
+      // one 16-byte record per chunk: 8 E4M3 values (round to nearest even,
+      // saturating to +-448), then the 8 indices
+      uint32_t v8 = 0;
+#pragma unroll
+      for (int s = 0; s < 4; ++s) {
+        __half_raw hr;
+        hr.x = (unsigned short)vb[s];
+        v8 |= (uint32_t)__nv_cvt_halfraw_to_fp8(hr, __NV_SATFINITE, __NV_E4M3) << (8 * s);
+      }
+      uint8_t* r = blk + (kind ? g.vval_off() : 0) + rec * 16;
+      *reinterpret_cast<uint32_t*>(r + half * 4) = v8;
+      *reinterpret_cast<uint32_t*>(r + 8 + half * 4) = idx;
+    } else {
+      const uint2 vals = make_uint2(vb[0] | (vb[1] << 16), vb[2] | (vb[3] << 16));
+      const int voff = kind ? g.vval_off() : 0;
+      const int ioff = kind ? g.vidx_off() : g.kidx_off();
+      *reinterpret_cast<uint2*>(blk + voff + rec * 16 + half * 8) = vals;
+      *reinterpret_cast<uint32_t*>(blk + ioff + rec * 8 + half * 4) = idx;
+    }
   }
 }
 

@@ -1,14 +1,16 @@
 // Decode attention on the packed sparse cache (Algorithm 1, attention part;
-// Section 4.3), split over the SMs, then the split combine and the
-// rotate-back o = o_hat R_vo^T (Appendix A.1, Lemma 2).
+// Section 4.3), split over the SMs, with the split combine and the
+// rotate-back o = o_hat R_vo^T (Appendix A.1, Lemma 2) fused in.
+#include <cuda_fp8.h>
+
 #include "swan_internal.h"
 
 namespace swan {
 namespace {
 
 // Streaming loads of cache records.  With one query head per kv head nothing
-// is re-read, so the records bypass L1; with several heads the warps of a
-// team read the same records and L1 serves the repeats.
+// is re-read, so the records bypass L1; with head pairs split over two lanes
+// the two lanes of a token read the same record in one instruction.
 template <bool kL1>
 __device__ __forceinline__ uint4 ld_rec16(const void* ptr) {
   uint4 r;
@@ -34,6 +36,65 @@ __device__ __forceinline__ float2 h2f(uint32_t w) {
   return __half22float2(*reinterpret_cast<const __half2*>(&w));
 }
 
+// Two E4M3 values (low 16 bits of w, or the high 16 bits) to fp32.
+__device__ __forceinline__ float2 e4m3x2_to_f2(uint32_t w, bool hi) {
+  const __nv_fp8x2_storage_t pair = (__nv_fp8x2_storage_t)(hi ? (w >> 16) : (w & 0xffffu));
+  const __half2_raw h = __nv_cvt_fp8x2_to_halfraw2(pair, __NV_E4M3);
+  return __half22float2(*reinterpret_cast<const __half2*>(&h));
+}
+
+// ---------------------------------------------------------------------------
+// One 8-entry chunk of a cached vector, per value format:
+//   fp16: a 16-byte record of 8 fp16 values and an 8-byte record of indices;
+//   fp8:  one 16-byte record: 8 E4M3 values, then 8 indices.
+// ---------------------------------------------------------------------------
+template <int FMT>
+struct Chunk;
+template <>
+struct Chunk<kFmtFp16> {
+  uint4 v;
+  uint2 i;
+};
+template <>
+struct Chunk<kFmtFp8> {
+  uint4 r;
+};
+
+// vb: this lane's 16-byte record run, ib: its 8-byte index run (fp16 only)
+template <int FMT, bool kL1>
+__device__ __forceinline__ Chunk<FMT> load_chunk(const uint8_t* vb, const uint8_t* ib, int c) {
+  Chunk<FMT> ch;
+  if constexpr (FMT == kFmtFp16) {
+    ch.v = ld_rec16<kL1>(vb + c * 512);
+    ch.i = ld_rec8<kL1>(ib + c * 256);
+  } else {
+    ch.r = ld_rec16<kL1>(vb + c * 512);
+  }
+  return ch;
+}
+template <int FMT>
+__device__ __forceinline__ uint2 chunk_idx(const Chunk<FMT>& ch) {
+  if constexpr (FMT == kFmtFp16)
+    return ch.i;
+  else
+    return make_uint2(ch.r.z, ch.r.w);
+}
+template <int FMT>
+__device__ __forceinline__ void chunk_vals(const Chunk<FMT>& ch, float (&f)[8]) {
+  float2 a, b, c, d;
+  if constexpr (FMT == kFmtFp16) {
+    a = h2f(ch.v.x), b = h2f(ch.v.y), c = h2f(ch.v.z), d = h2f(ch.v.w);
+  } else {
+    a = e4m3x2_to_f2(ch.r.x, false), b = e4m3x2_to_f2(ch.r.x, true);
+    c = e4m3x2_to_f2(ch.r.y, false), d = e4m3x2_to_f2(ch.r.y, true);
+  }
+  f[0] = a.x, f[1] = a.y, f[2] = b.x, f[3] = b.y, f[4] = c.x, f[5] = c.y, f[6] = d.x, f[7] = d.y;
+}
+__device__ __forceinline__ void keep_first(float (&f)[8], int n) {
+#pragma unroll
+  for (int e = 0; e < 8; ++e) f[e] = (e < n) ? f[e] : 0.f;
+}
+
 __device__ __forceinline__ float warp_max(float v) {
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
@@ -57,9 +118,27 @@ __device__ __forceinline__ float lds(uint32_t a) {
 __device__ __forceinline__ void sts(uint32_t a, float v) {
   asm volatile("st.shared.f32 [%0], %1;" ::"r"(a), "f"(v));
 }
+__device__ __forceinline__ float2 lds2(uint32_t a) {
+  float2 v;
+  asm volatile("ld.shared.v2.f32 {%0,%1}, [%2];" : "=f"(v.x), "=f"(v.y) : "r"(a));
+  return v;
+}
+__device__ __forceinline__ void sts2(uint32_t a, float2 v) {
+  asm volatile("st.shared.v2.f32 [%0], {%1,%2};" ::"r"(a), "f"(v.x), "f"(v.y));
+}
 
-// Address of coordinate idx (byte e of the index record word w) in a
-// [128][32] lane-interleaved fp32 array whose base is 16 KB aligned:
+// Ask the memory system to bring `bytes` (a multiple of 16, 16-byte aligned)
+// into L2 ahead of the loads that will read them.
+__device__ __forceinline__ void prefetch_l2(const void* ptr, uint32_t bytes) {
+  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(ptr), "r"(bytes) : "memory");
+}
+
+// ---------------------------------------------------------------------------
+// One query head per kv head: lane = token, lane-private accumulators.
+// ---------------------------------------------------------------------------
+
+// Address of coordinate idx (byte e of the index word w) in a [128][32]
+// lane-interleaved fp32 array whose base is 16 KB aligned:
 // base | (idx & 127) << 7 | lane << 2.  One shift and one LOP3; element
 // (idx, lane) sits at idx*32 + lane, so 32 lanes gathering arbitrary
 // coordinates hit 32 distinct banks, and any index byte stays inside the
@@ -72,70 +151,56 @@ __device__ __forceinline__ uint32_t addr_of(uint32_t w, uint32_t base) {
   return ((w >> 17) & 0x3f80u) | base;
 }
 
-// Score contribution of one 8-entry chunk into four partial sums.
-__device__ __forceinline__ void score_chunk(uint32_t qb, uint4 v, uint2 ix, float (&s)[4]) {
+// Score contribution of one chunk into four partial sums.
+__device__ __forceinline__ void score_chunk(uint32_t qb, const float (&f)[8], uint2 ix, float (&s)[4]) {
   const float q0 = lds(addr_of<0>(ix.x, qb)), q1 = lds(addr_of<1>(ix.x, qb));
   const float q2 = lds(addr_of<2>(ix.x, qb)), q3 = lds(addr_of<3>(ix.x, qb));
   const float q4 = lds(addr_of<0>(ix.y, qb)), q5 = lds(addr_of<1>(ix.y, qb));
   const float q6 = lds(addr_of<2>(ix.y, qb)), q7 = lds(addr_of<3>(ix.y, qb));
-  const float2 a = h2f(v.x), b = h2f(v.y), c = h2f(v.z), d = h2f(v.w);
-  s[0] = fmaf(q0, a.x, s[0]);
-  s[1] = fmaf(q1, a.y, s[1]);
-  s[2] = fmaf(q2, b.x, s[2]);
-  s[3] = fmaf(q3, b.y, s[3]);
-  s[0] = fmaf(q4, c.x, s[0]);
-  s[1] = fmaf(q5, c.y, s[1]);
-  s[2] = fmaf(q6, d.x, s[2]);
-  s[3] = fmaf(q7, d.y, s[3]);
+  s[0] = fmaf(q0, f[0], s[0]);
+  s[1] = fmaf(q1, f[1], s[1]);
+  s[2] = fmaf(q2, f[2], s[2]);
+  s[3] = fmaf(q3, f[3], s[3]);
+  s[0] = fmaf(q4, f[4], s[0]);
+  s[1] = fmaf(q5, f[5], s[1]);
+  s[2] = fmaf(q6, f[6], s[2]);
+  s[3] = fmaf(q7, f[7], s[3]);
 }
 
 // acc[idx_e] += p * val_e for one full chunk (distinct indices): eight loads,
 // eight FMAs, eight stores.
-__device__ __forceinline__ void value_chunk(uint32_t ab, float p, uint4 v, uint2 ix) {
+__device__ __forceinline__ void value_chunk(uint32_t ab, float p, const float (&f)[8], uint2 ix) {
   const uint32_t a0 = addr_of<0>(ix.x, ab), a1 = addr_of<1>(ix.x, ab);
   const uint32_t a2 = addr_of<2>(ix.x, ab), a3 = addr_of<3>(ix.x, ab);
   const uint32_t a4 = addr_of<0>(ix.y, ab), a5 = addr_of<1>(ix.y, ab);
   const uint32_t a6 = addr_of<2>(ix.y, ab), a7 = addr_of<3>(ix.y, ab);
   const float o0 = lds(a0), o1 = lds(a1), o2 = lds(a2), o3 = lds(a3);
   const float o4 = lds(a4), o5 = lds(a5), o6 = lds(a6), o7 = lds(a7);
-  const float2 a = h2f(v.x), b = h2f(v.y), c = h2f(v.z), d = h2f(v.w);
-  sts(a0, fmaf(p, a.x, o0));
-  sts(a1, fmaf(p, a.y, o1));
-  sts(a2, fmaf(p, b.x, o2));
-  sts(a3, fmaf(p, b.y, o3));
-  sts(a4, fmaf(p, c.x, o4));
-  sts(a5, fmaf(p, c.y, o5));
-  sts(a6, fmaf(p, d.x, o6));
-  sts(a7, fmaf(p, d.y, o7));
+  sts(a0, fmaf(p, f[0], o0));
+  sts(a1, fmaf(p, f[1], o1));
+  sts(a2, fmaf(p, f[2], o2));
+  sts(a3, fmaf(p, f[3], o3));
+  sts(a4, fmaf(p, f[4], o4));
+  sts(a5, fmaf(p, f[5], o5));
+  sts(a6, fmaf(p, f[6], o6));
+  sts(a7, fmaf(p, f[7], o7));
 }
 
 // The first `n` (< 8) entries of a chunk, one read-modify-write at a time
-// (the masked tail of a runtime keep count that is not a multiple of 8).
-__device__ __forceinline__ void value_chunk_partial(uint32_t ab, float p, uint4 v, uint2 ix, int n) {
-  const uint32_t hw[4] = {v.x, v.y, v.z, v.w};
+// (the tail of a runtime keep count that is not a multiple of 8).
+__device__ __forceinline__ void value_chunk_partial(uint32_t ab, float p, const float (&f)[8], uint2 ix,
+                                                    int n) {
 #pragma unroll
   for (int e = 0; e < 7; ++e) {
     if (e < n) {
       const uint32_t w = e < 4 ? ix.x : ix.y;
-      const uint32_t sh = 8u * (e & 3);
-      const uint32_t a = ((w >> sh) & 0x7fu) << 7 | ab;
-      const float2 f = h2f(hw[e >> 1]);
-      sts(a, fmaf(p, (e & 1) ? f.y : f.x, lds(a)));
+      const uint32_t a = ((w >> (8u * (e & 3))) & 0x7fu) << 7 | ab;
+      sts(a, fmaf(p, f[e], lds(a)));
     }
   }
 }
 
-__device__ __forceinline__ uint4 and4(uint4 a, uint4 m) {
-  return make_uint4(a.x & m.x, a.y & m.y, a.z & m.z, a.w & m.w);
-}
-
 constexpr uint32_t kRegionBytes = kHeadDim * 32 * sizeof(float);  // 16 KB
-
-// Ask the memory system to bring `bytes` (a multiple of 16, 16-byte aligned)
-// into L2 ahead of the loads that will read them.
-__device__ __forceinline__ void prefetch_l2(const void* ptr, uint32_t bytes) {
-  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(ptr), "r"(bytes) : "memory");
-}
 
 // The last CTA to finish a segment of unit u merges the unit's partials,
 // normalises, rotates back (o = o_hat R_vo^T) and writes the output.  The
@@ -189,57 +254,45 @@ __device__ __forceinline__ void finish_unit(const DecodeParams& p, int64_t u, in
   }
 }
 
-// Split decode kernel.
-//   Shared memory (16 KB-aligned regions): q' of the unit's G query heads
-//   replicated per lane ([G][128][32] fp32) and one lane-private
-//   rotated-space accumulator per warp ([8][128][32] fp32).
-//   Lane = token.  Warp w serves query head w % G; the G warps of a team walk
-//   the same contiguous run of 32-token blocks.  While block g is processed,
-//   the key records of block g+1 are in flight to registers and block g+2 is
-//   being prefetched into L2.
-// Warps per decode CTA: as many lane-private accumulators as fit next to
-// the replicated q' (16 KB each, 227 KB of shared memory per CTA).
-template <int G, int MAXC>
-__host__ __device__ constexpr int decode_warps() { return (G == 1 && MAXC <= 8) ? 12 : 8; }
+// Warps per CTA of the one-head kernel: as many lane-private accumulators as
+// fit next to q' (16 KB each, 227 KB of shared memory per CTA) and, for 16
+// chunks, as many as the registers allow.
+template <int MAXC>
+__host__ __device__ constexpr int decode_warps() { return MAXC <= 8 ? 12 : 8; }
 
-template <int G, int MAXC>
-__global__ void __launch_bounds__(decode_warps<G, MAXC>() * 32, 1) decode_kernel(DecodeParams p) {
-  constexpr int NW = decode_warps<G, MAXC>();
+// Split decode kernel, one query head per kv head.
+//   The flat list of 32-token blocks of all units is cut into equal ranges,
+//   one per CTA.  Shared memory (16 KB-aligned regions): q' replicated per
+//   lane ([128][32] fp32) and one lane-private rotated-space accumulator per
+//   warp ([128][32] fp32).  Lane = token; each warp walks a contiguous run of
+//   blocks.  While block g is processed, the key records of block g+1 are in
+//   flight to registers and block g+2 is being prefetched into L2.
+template <int MAXC, int FMT>
+__global__ void __launch_bounds__(decode_warps<MAXC>() * 32, 1) decode_kernel(DecodeParams p) {
+  constexpr int NW = decode_warps<MAXC>();
   constexpr int NT = NW * 32;
-  constexpr int TEAMS = NW / G;
-  constexpr bool kL1 = G > 1;
   extern __shared__ __align__(16) unsigned char smem_raw[];
   __shared__ float red_m[NW], red_l[NW];
   pdl_trigger();
 
   const uint32_t raw = (uint32_t)__cvta_generic_to_shared(smem_raw);
   const uint32_t base = (raw + kRegionBytes - 1) & ~(kRegionBytes - 1);
-  float* qrep = reinterpret_cast<float*>(smem_raw + (base - raw));  // [G][128][32]
-  float* accs = qrep + G * kHeadDim * 32;                            // [8][128][32]
+  float* qrep = reinterpret_cast<float*>(smem_raw + (base - raw));  // [128][32]
+  float* accs = qrep + kHeadDim * 32;                                // [NW][128][32]
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int hh = warp % G, team = warp / G;
-  const uint32_t qb = base + hh * kRegionBytes + (lane << 2);
-  const uint32_t ab = base + (G + warp) * kRegionBytes + (lane << 2);
+  const uint32_t qb = base + (lane << 2);
+  const uint32_t ab = base + (1 + warp) * kRegionBytes + (lane << 2);
 
   const CacheGeom& g = p.geom;
   const int kfull = p.k_full_chunks, krem = p.k_rem;
   const int nchunks = kfull + (krem ? 1 : 0);
   const int ks = g.k_slots;
-  // byte offsets inside a block, plus this lane's record
-  const int o_kv = lane * 16, o_ki = 64 * ks + lane * 8;
-  const int o_vv = 96 * ks + lane * 16, o_vi = 160 * ks + lane * 8;
+  // this lane's record runs inside a block
+  const int o_kv = lane * 16, o_ki = g.kidx_off() + lane * 8;
+  const int o_vv = g.vval_off() + lane * 16, o_vi = g.vidx_off() + lane * 8;
   const bool whole_block = nchunks * 8 == ks;
-  const uint32_t pf_val = (uint32_t)nchunks * 512, pf_idx = (uint32_t)nchunks * 256;
   const int bsh = p.blocks_per_page_log2, bmask = (1 << bsh) - 1;
-  uint4 remmask;
-  {
-    uint32_t w[4];
-#pragma unroll
-    for (int e = 0; e < 4; ++e)
-      w[e] = ((2 * e < krem) ? 0xffffu : 0u) | ((2 * e + 1 < krem) ? 0xffff0000u : 0u);
-    remmask = make_uint4(w[0], w[1], w[2], w[3]);
-  }
 
   const int64_t g_begin = (int64_t)blockIdx.x * p.range;
   const int64_t g_end = min(p.total_groups, g_begin + p.range);
@@ -252,18 +305,16 @@ __global__ void __launch_bounds__(decode_warps<G, MAXC>() * 32, 1) decode_kernel
     const int s0 = (int)(max(g_begin, u * p.N_g) - u * p.N_g);
     const int s1 = (int)(min(g_end, (u + 1) * p.N_g) - u * p.N_g);
     const int64_t b = u / p.H_kv, h = u % p.H_kv;
-    // this team's contiguous run of groups [t_lo, t_hi)
+    // this warp's contiguous run of groups [t_lo, t_hi)
     const int len = s1 - s0;
-    const int t_lo = s0 + (len * team) / TEAMS;
-    const int t_hi = s0 + (len * (team + 1)) / TEAMS;
+    const int t_lo = s0 + (len * warp) / NW;
+    const int t_hi = s0 + (len * (warp + 1)) / NW;
     const int sp_hi = min(t_hi, n_sg);  // sparse groups of the run: [t_lo, sp_hi)
     const int32_t* ptab = g.page_table + u * g.pages_per_unit;
 
-    __syncthreads();  // the previous segment's reduction is done with smem
-    for (int i = threadIdx.x; i < G * kHeadDim * 32; i += NT) {
-      const int gh = i >> 12, dd = (i >> 5) & (kHeadDim - 1);
-      qrep[i] = __ldg(p.qprime + ((b * p.H_q + h * G + gh) * kHeadDim + dd));
-    }
+    __syncthreads();  // the previous segment is done with shared memory
+    for (int i = threadIdx.x; i < kHeadDim * 32; i += NT)
+      qrep[i] = __ldg(p.qprime + ((b * p.H_q + h) * kHeadDim + (i >> 5)));
 #pragma unroll 8
     for (int dd = 0; dd < kHeadDim; ++dd) sts(ab + dd * 128, 0.f);
     __syncthreads();
@@ -285,29 +336,29 @@ __global__ void __launch_bounds__(decode_warps<G, MAXC>() * 32, 1) decode_kernel
       if (blk == nullptr || lane != 0) return;
       if (whole_block) {
         prefetch_l2(blk, (uint32_t)g.block_bytes());
+      } else if constexpr (FMT == kFmtFp16) {
+        prefetch_l2(blk, nchunks * 512u);
+        prefetch_l2(blk + g.kidx_off(), nchunks * 256u);
+        prefetch_l2(blk + g.vval_off(), nchunks * 512u);
+        prefetch_l2(blk + g.vidx_off(), nchunks * 256u);
       } else {
-        prefetch_l2(blk, pf_val);
-        prefetch_l2(blk + 64 * ks, pf_idx);
-        prefetch_l2(blk + 96 * ks, pf_val);
-        prefetch_l2(blk + 160 * ks, pf_idx);
+        prefetch_l2(blk, nchunks * 512u);
+        prefetch_l2(blk + g.vval_off(), nchunks * 512u);
       }
     };
-    auto load_k = [&](const uint8_t* blk, uint4 (&kv)[MAXC], uint2 (&ki)[MAXC]) {
+
+    Chunk<FMT> kc[MAXC];
+    auto load_k = [&](const uint8_t* blk) {
       const uint8_t* src = blk ? blk : g.pool;
 #pragma unroll
       for (int c = 0; c < MAXC; ++c)
-        if (c < nchunks) {
-          kv[c] = ld_rec16<kL1>(src + o_kv + c * 512);
-          ki[c] = ld_rec8<kL1>(src + o_ki + c * 256);
-        }
+        if (c < nchunks) kc[c] = load_chunk<FMT, false>(src + o_kv, src + o_ki, c);
     };
 
-    uint4 kv[MAXC];
-    uint2 ki[MAXC];
     const uint8_t* b_cur = block_of(t_lo);
     const uint8_t* b_n1 = block_of(t_lo + 1);
     prefetch_block(b_n1);
-    if (t_lo < sp_hi) load_k(b_cur, kv, ki);
+    if (t_lo < sp_hi) load_k(b_cur);
 
     for (int gi = t_lo; gi < t_hi; ++gi) {
       float s2, pr;
@@ -318,47 +369,43 @@ __global__ void __launch_bounds__(decode_warps<G, MAXC>() * 32, 1) decode_kernel
         const bool valid = ok && t0 + lane < p.sparse_len;
         const bool tail = !ok || t0 + 32 > p.sparse_len;  // warp-uniform
         const uint8_t* src = ok ? b_cur : g.pool;
-        uint4 vv[MAXC];
-        uint2 vi[MAXC];
+        Chunk<FMT> vc[MAXC];
 #pragma unroll
         for (int c = 0; c < MAXC; ++c)
-          if (c < nchunks) {
-            vv[c] = ld_rec16<kL1>(src + o_vv + c * 512);
-            vi[c] = ld_rec8<kL1>(src + o_vi + c * 256);
-          }
+          if (c < nchunks) vc[c] = load_chunk<FMT, false>(src + o_vv, src + o_vi, c);
         // two blocks ahead: into L2
         const uint8_t* b_n2 = block_of(gi + 2);
         prefetch_block(b_n2);
 
-        const uint4 lanemask = valid ? make_uint4(~0u, ~0u, ~0u, ~0u) : make_uint4(0, 0, 0, 0);
         float s[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
         for (int c = 0; c < MAXC; ++c)
           if (c < nchunks) {
-            uint4 v = kv[c];
-            uint2 ix = ki[c];
-            if (krem && c == nchunks - 1) v = and4(v, remmask);
-            if (tail) {
-              v = and4(v, lanemask);
-              ix = valid ? ix : make_uint2(0, 0);
+            float f[8];
+            chunk_vals<FMT>(kc[c], f);
+            uint2 ix = chunk_idx<FMT>(kc[c]);
+            if (krem && c == nchunks - 1) keep_first(f, krem);
+            if (tail && !valid) {
+              keep_first(f, 0);
+              ix = make_uint2(0, 0);
             }
-            score_chunk(qb, v, ix, s);
+            score_chunk(qb, f, ix, s);
           }
         s2 = valid ? ((s[0] + s[1]) + (s[2] + s[3])) * p.scale_log2 : -INFINITY;
 
         // the next block's key records into registers while this block's
         // values are accumulated
-        if (gi + 1 < sp_hi) load_k(b_n1, kv, ki);
+        if (gi + 1 < sp_hi) load_k(b_n1);
         b_cur = b_n1;
         b_n1 = b_n2;
 
         const float gmax = warp_max(s2);
         if (gmax > m_w + kLazyRescale) {
           if (m_w != -INFINITY) {
-            const float f = exp2f(m_w - gmax);
-            l_sum *= f;
+            const float fs = exp2f(m_w - gmax);
+            l_sum *= fs;
 #pragma unroll 8
-            for (int dd = 0; dd < kHeadDim; ++dd) sts(ab + dd * 128, lds(ab + dd * 128) * f);
+            for (int dd = 0; dd < kHeadDim; ++dd) sts(ab + dd * 128, lds(ab + dd * 128) * fs);
           }
           m_w = gmax;
         }
@@ -368,18 +415,23 @@ __global__ void __launch_bounds__(decode_warps<G, MAXC>() * 32, 1) decode_kernel
 #pragma unroll
         for (int c = 0; c < MAXC; ++c)
           if (c < kfull) {
-            uint4 v = vv[c];
-            uint2 ix = vi[c];
-            if (tail) {
-              v = and4(v, lanemask);
-              ix = valid ? ix : make_uint2(0, 0);
+            float f[8];
+            chunk_vals<FMT>(vc[c], f);
+            uint2 ix = chunk_idx<FMT>(vc[c]);
+            if (tail && !valid) {
+              keep_first(f, 0);
+              ix = make_uint2(0, 0);
             }
-            value_chunk(ab, pr, v, ix);
+            value_chunk(ab, pr, f, ix);
           }
         if (krem && valid) {
 #pragma unroll
           for (int c = 0; c < MAXC; ++c)
-            if (c == kfull) value_chunk_partial(ab, pr, vv[c], vi[c], krem);
+            if (c == kfull) {
+              float f[8];
+              chunk_vals<FMT>(vc[c], f);
+              value_chunk_partial(ab, pr, f, chunk_idx<FMT>(vc[c]), krem);
+            }
         }
       } else {
         // ---- buffer group: dense rotated fp16 vectors of the ring buffer
@@ -408,10 +460,10 @@ __global__ void __launch_bounds__(decode_warps<G, MAXC>() * 32, 1) decode_kernel
         const float gmax = warp_max(s2);
         if (gmax > m_w + kLazyRescale) {
           if (m_w != -INFINITY) {
-            const float f = exp2f(m_w - gmax);
-            l_sum *= f;
+            const float fs = exp2f(m_w - gmax);
+            l_sum *= fs;
 #pragma unroll 8
-            for (int dd = 0; dd < kHeadDim; ++dd) sts(ab + dd * 128, lds(ab + dd * 128) * f);
+            for (int dd = 0; dd < kHeadDim; ++dd) sts(ab + dd * 128, lds(ab + dd * 128) * fs);
           }
           m_w = gmax;
         }
@@ -439,22 +491,20 @@ __global__ void __launch_bounds__(decode_warps<G, MAXC>() * 32, 1) decode_kernel
       }
     }
 
-    // ---- merge the lanes and warps of each head into one partial
+    // ---- merge the lanes and warps into one partial
     l_sum = warp_sum(l_sum);
     if (lane == 0) {
       red_m[warp] = m_w;
       red_l[warp] = l_sum;
     }
     __syncthreads();
-    for (int o = threadIdx.x; o < G * kHeadDim; o += NT) {
-      const int gh = o / kHeadDim, dd = o % kHeadDim;
+    for (int dd = threadIdx.x; dd < kHeadDim; dd += NT) {
       float M = -INFINITY;
 #pragma unroll
-      for (int t = 0; t < TEAMS; ++t) M = fmaxf(M, red_m[t * G + gh]);
+      for (int w = 0; w < NW; ++w) M = fmaxf(M, red_m[w]);
       float tot = 0.f, L = 0.f;
 #pragma unroll
-      for (int t = 0; t < TEAMS; ++t) {
-        const int w = t * G + gh;
+      for (int w = 0; w < NW; ++w) {
         const float mw = red_m[w];
         const float f = (mw == -INFINITY) ? 0.f : exp2f(mw - M);
         const float* a = accs + w * kHeadDim * 32 + dd * 32;
@@ -464,21 +514,20 @@ __global__ void __launch_bounds__(decode_warps<G, MAXC>() * 32, 1) decode_kernel
         tot = fmaf(f, sum, tot);
         L = fmaf(f, red_l[w], L);
       }
-      float* dst = p.partials + ((size_t)(blockIdx.x + u) * G + gh) * (kHeadDim + 2);
+      float* dst = p.partials + ((size_t)(blockIdx.x + u)) * (kHeadDim + 2);
       dst[2 + dd] = tot;
       if (dd == 0) {
         dst[0] = M;
         dst[1] = L;
       }
     }
-
-    finish_unit<G, NT>(p, u, b, h, qrep, red_m);
+    finish_unit<1, NT>(p, u, b, h, qrep, red_m);
   }
 }
 
 // ---------------------------------------------------------------------------
 // Grouped-query heads (G = 2 or 4): each lane carries a pair of query heads
-// of one token, so the index decoding, the fp16 conversion and the record
+// of one token, so the index decoding, the value conversion and the record
 // loads are shared by two heads, and one accumulator array serves the whole
 // group: lanes 16..31 take heads 2..3 of the tokens that lanes 0..15 take
 // heads 0..1 of (G = 4).  q' and the accumulators are [128][32 lanes][2]
@@ -497,30 +546,21 @@ __device__ __forceinline__ uint32_t addr2_of(uint32_t w, uint32_t base) {
   if (E == 2) return ((w >> 8) & 0x7f00u) | base;
   return ((w >> 16) & 0x7f00u) | base;
 }
-__device__ __forceinline__ float2 lds2(uint32_t a) {
-  float2 v;
-  asm volatile("ld.shared.v2.f32 {%0,%1}, [%2];" : "=f"(v.x), "=f"(v.y) : "r"(a));
-  return v;
-}
-__device__ __forceinline__ void sts2(uint32_t a, float2 v) {
-  asm volatile("st.shared.v2.f32 [%0], {%1,%2};" ::"r"(a), "f"(v.x), "f"(v.y));
-}
 
 // Scores of two heads for one chunk: s[0..1] head 0, s[2..3] head 1.
-__device__ __forceinline__ void score2_chunk(uint32_t qb, uint4 v, uint2 ix, float (&s)[4]) {
+__device__ __forceinline__ void score2_chunk(uint32_t qb, const float (&f)[8], uint2 ix, float (&s)[4]) {
   const float2 q0 = lds2(addr2_of<0>(ix.x, qb)), q1 = lds2(addr2_of<1>(ix.x, qb));
   const float2 q2 = lds2(addr2_of<2>(ix.x, qb)), q3 = lds2(addr2_of<3>(ix.x, qb));
   const float2 q4 = lds2(addr2_of<0>(ix.y, qb)), q5 = lds2(addr2_of<1>(ix.y, qb));
   const float2 q6 = lds2(addr2_of<2>(ix.y, qb)), q7 = lds2(addr2_of<3>(ix.y, qb));
-  const float2 a = h2f(v.x), b = h2f(v.y), c = h2f(v.z), d = h2f(v.w);
-  s[0] = fmaf(q0.x, a.x, s[0]); s[2] = fmaf(q0.y, a.x, s[2]);
-  s[1] = fmaf(q1.x, a.y, s[1]); s[3] = fmaf(q1.y, a.y, s[3]);
-  s[0] = fmaf(q2.x, b.x, s[0]); s[2] = fmaf(q2.y, b.x, s[2]);
-  s[1] = fmaf(q3.x, b.y, s[1]); s[3] = fmaf(q3.y, b.y, s[3]);
-  s[0] = fmaf(q4.x, c.x, s[0]); s[2] = fmaf(q4.y, c.x, s[2]);
-  s[1] = fmaf(q5.x, c.y, s[1]); s[3] = fmaf(q5.y, c.y, s[3]);
-  s[0] = fmaf(q6.x, d.x, s[0]); s[2] = fmaf(q6.y, d.x, s[2]);
-  s[1] = fmaf(q7.x, d.y, s[1]); s[3] = fmaf(q7.y, d.y, s[3]);
+  s[0] = fmaf(q0.x, f[0], s[0]); s[2] = fmaf(q0.y, f[0], s[2]);
+  s[1] = fmaf(q1.x, f[1], s[1]); s[3] = fmaf(q1.y, f[1], s[3]);
+  s[0] = fmaf(q2.x, f[2], s[0]); s[2] = fmaf(q2.y, f[2], s[2]);
+  s[1] = fmaf(q3.x, f[3], s[1]); s[3] = fmaf(q3.y, f[3], s[3]);
+  s[0] = fmaf(q4.x, f[4], s[0]); s[2] = fmaf(q4.y, f[4], s[2]);
+  s[1] = fmaf(q5.x, f[5], s[1]); s[3] = fmaf(q5.y, f[5], s[3]);
+  s[0] = fmaf(q6.x, f[6], s[0]); s[2] = fmaf(q6.y, f[6], s[2]);
+  s[1] = fmaf(q7.x, f[7], s[1]); s[3] = fmaf(q7.y, f[7], s[3]);
 }
 
 __device__ __forceinline__ float2 fma2(float p0, float p1, float v, float2 o) {
@@ -528,34 +568,31 @@ __device__ __forceinline__ float2 fma2(float p0, float p1, float v, float2 o) {
 }
 
 // acc[idx_e] += (p0, p1) * val_e for one full chunk (distinct indices).
-__device__ __forceinline__ void value2_chunk(uint32_t ab, float p0, float p1, uint4 v, uint2 ix) {
+__device__ __forceinline__ void value2_chunk(uint32_t ab, float p0, float p1, const float (&f)[8], uint2 ix) {
   const uint32_t a0 = addr2_of<0>(ix.x, ab), a1 = addr2_of<1>(ix.x, ab);
   const uint32_t a2 = addr2_of<2>(ix.x, ab), a3 = addr2_of<3>(ix.x, ab);
   const uint32_t a4 = addr2_of<0>(ix.y, ab), a5 = addr2_of<1>(ix.y, ab);
   const uint32_t a6 = addr2_of<2>(ix.y, ab), a7 = addr2_of<3>(ix.y, ab);
   const float2 o0 = lds2(a0), o1 = lds2(a1), o2 = lds2(a2), o3 = lds2(a3);
   const float2 o4 = lds2(a4), o5 = lds2(a5), o6 = lds2(a6), o7 = lds2(a7);
-  const float2 a = h2f(v.x), b = h2f(v.y), c = h2f(v.z), d = h2f(v.w);
-  sts2(a0, fma2(p0, p1, a.x, o0));
-  sts2(a1, fma2(p0, p1, a.y, o1));
-  sts2(a2, fma2(p0, p1, b.x, o2));
-  sts2(a3, fma2(p0, p1, b.y, o3));
-  sts2(a4, fma2(p0, p1, c.x, o4));
-  sts2(a5, fma2(p0, p1, c.y, o5));
-  sts2(a6, fma2(p0, p1, d.x, o6));
-  sts2(a7, fma2(p0, p1, d.y, o7));
+  sts2(a0, fma2(p0, p1, f[0], o0));
+  sts2(a1, fma2(p0, p1, f[1], o1));
+  sts2(a2, fma2(p0, p1, f[2], o2));
+  sts2(a3, fma2(p0, p1, f[3], o3));
+  sts2(a4, fma2(p0, p1, f[4], o4));
+  sts2(a5, fma2(p0, p1, f[5], o5));
+  sts2(a6, fma2(p0, p1, f[6], o6));
+  sts2(a7, fma2(p0, p1, f[7], o7));
 }
 
-__device__ __forceinline__ void value2_chunk_partial(uint32_t ab, float p0, float p1, uint4 v, uint2 ix,
-                                                     int n) {
-  const uint32_t hw[4] = {v.x, v.y, v.z, v.w};
+__device__ __forceinline__ void value2_chunk_partial(uint32_t ab, float p0, float p1, const float (&f)[8],
+                                                     uint2 ix, int n) {
 #pragma unroll
   for (int e = 0; e < 7; ++e) {
     if (e < n) {
       const uint32_t w = e < 4 ? ix.x : ix.y;
       const uint32_t a = ((w >> (8u * (e & 3))) & 0x7fu) << 8 | ab;
-      const float2 f = h2f(hw[e >> 1]);
-      sts2(a, fma2(p0, p1, (e & 1) ? f.y : f.x, lds2(a)));
+      sts2(a, fma2(p0, p1, f[e], lds2(a)));
     }
   }
 }
@@ -575,7 +612,7 @@ __device__ __forceinline__ float group_sum(float v) {
   return v;
 }
 
-template <int G, int MAXC>
+template <int G, int MAXC, int FMT>
 __global__ void __launch_bounds__(kGqaWarps * 32, 1) decode_gqa_kernel(DecodeParams p) {
   constexpr int NW = kGqaWarps, NT = NW * 32;
   constexpr int LPT = G / 2;          // lanes per token
@@ -600,16 +637,7 @@ __global__ void __launch_bounds__(kGqaWarps * 32, 1) decode_gqa_kernel(DecodePar
   const int nchunks = kfull + (krem ? 1 : 0);
   const int ks = g.k_slots;
   const bool whole_block = nchunks * 8 == ks;
-  const uint32_t pf_val = (uint32_t)nchunks * 512, pf_idx = (uint32_t)nchunks * 256;
   const int bsh = p.blocks_per_page_log2, bmask = (1 << bsh) - 1;
-  uint4 remmask;
-  {
-    uint32_t w[4];
-#pragma unroll
-    for (int e = 0; e < 4; ++e)
-      w[e] = ((2 * e < krem) ? 0xffffu : 0u) | ((2 * e + 1 < krem) ? 0xffff0000u : 0u);
-    remmask = make_uint4(w[0], w[1], w[2], w[3]);
-  }
 
   const int64_t g_begin = (int64_t)blockIdx.x * p.range;
   const int64_t g_end = min(p.total_groups, g_begin + p.range);
@@ -654,32 +682,31 @@ __global__ void __launch_bounds__(kGqaWarps * 32, 1) decode_gqa_kernel(DecodePar
       if (blk == nullptr || lane != 0) return;
       if (whole_block) {
         prefetch_l2(blk, (uint32_t)g.block_bytes());
+      } else if constexpr (FMT == kFmtFp16) {
+        prefetch_l2(blk, nchunks * 512u);
+        prefetch_l2(blk + g.kidx_off(), nchunks * 256u);
+        prefetch_l2(blk + g.vval_off(), nchunks * 512u);
+        prefetch_l2(blk + g.vidx_off(), nchunks * 256u);
       } else {
-        prefetch_l2(blk, pf_val);
-        prefetch_l2(blk + 64 * ks, pf_idx);
-        prefetch_l2(blk + 96 * ks, pf_val);
-        prefetch_l2(blk + 160 * ks, pf_idx);
+        prefetch_l2(blk, nchunks * 512u);
+        prefetch_l2(blk + g.vval_off(), nchunks * 512u);
       }
     };
-    // key records of item `it` (block gi, half `half`) for this lane's token
-    auto load_k = [&](const uint8_t* blk, int half, uint4 (&kv)[MAXC], uint2 (&ki)[MAXC]) {
+    // records of item `half` of a block for this lane's token
+    Chunk<FMT> kc[MAXC];
+    auto load_k = [&](const uint8_t* blk, int half) {
       const uint8_t* src = blk ? blk : g.pool;
       const int t = half * TS + ts;
 #pragma unroll
       for (int c = 0; c < MAXC; ++c)
-        if (c < nchunks) {
-          kv[c] = ld_rec16<true>(src + t * 16 + c * 512);
-          ki[c] = ld_rec8<true>(src + 64 * ks + t * 8 + c * 256);
-        }
+        if (c < nchunks) kc[c] = load_chunk<FMT, true>(src + t * 16, src + g.kidx_off() + t * 8, c);
     };
 
-    uint4 kv[MAXC];
-    uint2 ki[MAXC];
     int gi0 = i_lo / HALVES;
     const uint8_t* b_cur = block_of(gi0);
     const uint8_t* b_n1 = block_of(gi0 + 1);
     prefetch_block(b_n1);
-    if (i_lo < i_hi && gi0 < n_sg) load_k(b_cur, i_lo % HALVES, kv, ki);
+    if (i_lo < i_hi && gi0 < n_sg) load_k(b_cur, i_lo % HALVES);
 
     for (int it = i_lo; it < i_hi; ++it) {
       const int gi = it / HALVES, half = it % HALVES;
@@ -694,14 +721,11 @@ __global__ void __launch_bounds__(kGqaWarps * 32, 1) decode_gqa_kernel(DecodePar
         const bool tail = !ok || (int64_t)gi * 32 + (half + 1) * TS > p.sparse_len;  // warp-uniform
         const uint8_t* src = ok ? b_cur : g.pool;
         const int tt = half * TS + ts;
-        uint4 vv[MAXC];
-        uint2 vi[MAXC];
+        Chunk<FMT> vc[MAXC];
 #pragma unroll
         for (int c = 0; c < MAXC; ++c)
-          if (c < nchunks) {
-            vv[c] = ld_rec16<true>(src + 96 * ks + tt * 16 + c * 512);
-            vi[c] = ld_rec8<true>(src + 160 * ks + tt * 8 + c * 256);
-          }
+          if (c < nchunks)
+            vc[c] = load_chunk<FMT, true>(src + g.vval_off() + tt * 16, src + g.vidx_off() + tt * 8, c);
         const bool last_half = half == HALVES - 1;
         const uint8_t* b_n2 = nullptr;
         if (last_half) {
@@ -709,25 +733,25 @@ __global__ void __launch_bounds__(kGqaWarps * 32, 1) decode_gqa_kernel(DecodePar
           prefetch_block(b_n2);
         }
 
-        const uint4 lanemask = valid ? make_uint4(~0u, ~0u, ~0u, ~0u) : make_uint4(0, 0, 0, 0);
 #pragma unroll
         for (int c = 0; c < MAXC; ++c)
           if (c < nchunks) {
-            uint4 v = kv[c];
-            uint2 ix = ki[c];
-            if (krem && c == nchunks - 1) v = and4(v, remmask);
-            if (tail) {
-              v = and4(v, lanemask);
-              ix = valid ? ix : make_uint2(0, 0);
+            float f[8];
+            chunk_vals<FMT>(kc[c], f);
+            uint2 ix = chunk_idx<FMT>(kc[c]);
+            if (krem && c == nchunks - 1) keep_first(f, krem);
+            if (tail && !valid) {
+              keep_first(f, 0);
+              ix = make_uint2(0, 0);
             }
-            score2_chunk(qb, v, ix, s);
+            score2_chunk(qb, f, ix, s);
           }
 
         // next item's key records (same block's next half, or the next block)
         const int nit = it + 1;
         if (nit < i_hi) {
           const int ngi = nit / HALVES;
-          if (ngi < n_sg) load_k(last_half ? b_n1 : b_cur, nit % HALVES, kv, ki);
+          if (ngi < n_sg) load_k(last_half ? b_n1 : b_cur, nit % HALVES);
         }
         if (last_half) {
           b_cur = b_n1;
@@ -760,18 +784,23 @@ __global__ void __launch_bounds__(kGqaWarps * 32, 1) decode_gqa_kernel(DecodePar
 #pragma unroll
         for (int c = 0; c < MAXC; ++c)
           if (c < kfull) {
-            uint4 v = vv[c];
-            uint2 ix = vi[c];
-            if (tail) {
-              v = and4(v, lanemask);
-              ix = valid ? ix : make_uint2(0, 0);
+            float f[8];
+            chunk_vals<FMT>(vc[c], f);
+            uint2 ix = chunk_idx<FMT>(vc[c]);
+            if (tail && !valid) {
+              keep_first(f, 0);
+              ix = make_uint2(0, 0);
             }
-            value2_chunk(ab, p0, p1, v, ix);
+            value2_chunk(ab, p0, p1, f, ix);
           }
         if (krem && valid) {
 #pragma unroll
           for (int c = 0; c < MAXC; ++c)
-            if (c == kfull) value2_chunk_partial(ab, p0, p1, vv[c], vi[c], krem);
+            if (c == kfull) {
+              float f[8];
+              chunk_vals<FMT>(vc[c], f);
+              value2_chunk_partial(ab, p0, p1, f, chunk_idx<FMT>(vc[c]), krem);
+            }
         }
       } else {
         // ---- dense buffer tokens
@@ -870,9 +899,9 @@ __global__ void __launch_bounds__(kGqaWarps * 32, 1) decode_gqa_kernel(DecodePar
   }
 }
 
-// q' = q R_qk: one CTA per kv head with R in shared memory, one warp per
-// query vector of that head (all batches, all G heads of the group); lane l
-// computes coordinates 4l..4l+3 in a sequential fp32 FMA chain.
+// q' = q R_qk: one CTA per (kv head, up to 8 query vectors of that head),
+// R in shared memory, one warp per query vector; lane l computes coordinates
+// 4l..4l+3 in a sequential fp32 FMA chain.
 __global__ void __launch_bounds__(kThreads) rotate_q_kernel(RotateQParams p, int B) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   float* Rs = reinterpret_cast<float*>(smem_raw);
@@ -883,7 +912,6 @@ __global__ void __launch_bounds__(kThreads) rotate_q_kernel(RotateQParams p, int
   __syncthreads();
   pdl_wait();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  // this CTA's query vectors: [blockIdx.y * 8, blockIdx.y * 8 + 8) of the B * G of head h
   for (int item = blockIdx.y * kWarpsPerCta + warp; item < min(B * p.G, (int)(blockIdx.y + 1) * kWarpsPerCta);
        item += kWarpsPerCta) {
     const int b = item / p.G, gh = item % p.G;
@@ -906,8 +934,7 @@ __global__ void __launch_bounds__(kThreads) rotate_q_kernel(RotateQParams p, int
   }
 }
 
-// Merge the partials of one (batch, query head), normalise, rotate back by
-// R_vo^T and round to fp16.
+// Empty cache: writes zeros (the rotate-back of an empty attention).
 __global__ void __launch_bounds__(kHeadDim) combine_kernel(CombineParams p) {
   __shared__ float o_hat[kHeadDim];
   pdl_trigger();
@@ -946,82 +973,72 @@ __global__ void __launch_bounds__(kHeadDim) combine_kernel(CombineParams p) {
   p.out[bq * kHeadDim + dd] = __float2half_rn(a0 + a1);
 }
 
-template <int G, int MAXC>
-cudaError_t launch_decode_t(const DecodeParams& p, int grid, cudaStream_t s) {
-  static bool attr_set = false;
-  const size_t smem = decode_smem_bytes(G, MAXC * 8);
-  if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(decode_kernel<G, MAXC>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return e;
-    attr_set = true;
-  }
-  return launch_pdl(decode_kernel<G, MAXC>, dim3(grid), dim3(decode_warps<G, MAXC>() * 32), smem, s, p);
+size_t one_head_smem(int maxc) {
+  const int nw = maxc <= 8 ? decode_warps<8>() : decode_warps<16>();
+  return (size_t)(1 + nw + 1) * kRegionBytes;
 }
+constexpr size_t kGqaSmem = 7 * kPairRegionBytes;
 
-template <int G, int MAXC>
-cudaError_t launch_gqa_t(const DecodeParams& p, int grid, cudaStream_t s) {
-  static bool attr_set = false;
-  constexpr size_t smem = 7 * kPairRegionBytes;
-  if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(decode_gqa_kernel<G, MAXC>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return e;
-    attr_set = true;
-  }
-  return launch_pdl(decode_gqa_kernel<G, MAXC>, dim3(grid), dim3(kGqaWarps * 32), smem, s, p);
-}
-
-template <int G, int MAXC>
-int gqa_ctas_per_sm_t() {
-  constexpr size_t smem = 7 * kPairRegionBytes;
-  if (cudaFuncSetAttribute(decode_gqa_kernel<G, MAXC>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                           (int)smem) != cudaSuccess)
+template <typename K>
+int occupancy(K kernel, int threads, size_t smem) {
+  if (cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
     return 0;
   int n = 0;
-  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, decode_gqa_kernel<G, MAXC>, kGqaWarps * 32,
-                                                    smem) != cudaSuccess)
-    return 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, kernel, threads, smem) != cudaSuccess) return 0;
   return n;
 }
 
+template <int G, int MAXC, int FMT>
+cudaError_t launch_t(const DecodeParams& p, int grid, cudaStream_t s) {
+  static bool attr_set = false;
+  if constexpr (G == 1) {
+    const size_t smem = one_head_smem(MAXC);
+    if (!attr_set) {
+      cudaError_t e = cudaFuncSetAttribute(decode_kernel<MAXC, FMT>,
+                                           cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+      if (e != cudaSuccess) return e;
+      attr_set = true;
+    }
+    return launch_pdl(decode_kernel<MAXC, FMT>, dim3(grid), dim3(decode_warps<MAXC>() * 32), smem, s, p);
+  } else {
+    if (!attr_set) {
+      cudaError_t e = cudaFuncSetAttribute(decode_gqa_kernel<G, MAXC, FMT>,
+                                           cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kGqaSmem);
+      if (e != cudaSuccess) return e;
+      attr_set = true;
+    }
+    return launch_pdl(decode_gqa_kernel<G, MAXC, FMT>, dim3(grid), dim3(kGqaWarps * 32), kGqaSmem, s, p);
+  }
+}
+
 template <int G, int MAXC>
-int ctas_per_sm_t() {
-  const size_t smem = decode_smem_bytes(G, MAXC * 8);
-  if (cudaFuncSetAttribute(decode_kernel<G, MAXC>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                           (int)smem) != cudaSuccess)
-    return 0;
-  int n = 0;
-  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, decode_kernel<G, MAXC>, decode_warps<G, MAXC>() * 32,
-                                                    smem) !=
-      cudaSuccess)
-    return 0;
-  return n;
+cudaError_t launch_fmt(const DecodeParams& p, int grid, cudaStream_t s) {
+  return p.geom.fmt == kFmtFp8 ? launch_t<G, MAXC, kFmtFp8>(p, grid, s)
+                               : launch_t<G, MAXC, kFmtFp16>(p, grid, s);
 }
 
 }  // namespace
 
-size_t decode_smem_bytes(int G, int k_slots) {
-  const int nw = (G == 1 && k_slots <= 64) ? decode_warps<1, 8>() : decode_warps<2, 16>();
-  return (size_t)(G + nw + 1) * kRegionBytes;
-}
-
 int decode_ctas_per_sm(int G, int k_slots) {
   const bool big = k_slots > 64;
-  switch (G) {
-    case 1: return big ? ctas_per_sm_t<1, 16>() : ctas_per_sm_t<1, 8>();
-    case 2: return big ? gqa_ctas_per_sm_t<2, 16>() : gqa_ctas_per_sm_t<2, 8>();
-    case 4: return big ? gqa_ctas_per_sm_t<4, 16>() : gqa_ctas_per_sm_t<4, 8>();
-    default: return 0;
-  }
+  if (G == 1)
+    return big ? occupancy(decode_kernel<16, kFmtFp16>, decode_warps<16>() * 32, one_head_smem(16))
+               : occupancy(decode_kernel<8, kFmtFp16>, decode_warps<8>() * 32, one_head_smem(8));
+  if (G == 2)
+    return big ? occupancy(decode_gqa_kernel<2, 16, kFmtFp16>, kGqaWarps * 32, kGqaSmem)
+               : occupancy(decode_gqa_kernel<2, 8, kFmtFp16>, kGqaWarps * 32, kGqaSmem);
+  if (G == 4)
+    return big ? occupancy(decode_gqa_kernel<4, 16, kFmtFp16>, kGqaWarps * 32, kGqaSmem)
+               : occupancy(decode_gqa_kernel<4, 8, kFmtFp16>, kGqaWarps * 32, kGqaSmem);
+  return 0;
 }
 
 cudaError_t launch_decode(const DecodeParams& p, int G, int k_read, int grid, cudaStream_t s) {
   const bool big = k_read > 64;
   switch (G) {
-    case 1: return big ? launch_decode_t<1, 16>(p, grid, s) : launch_decode_t<1, 8>(p, grid, s);
-    case 2: return big ? launch_gqa_t<2, 16>(p, grid, s) : launch_gqa_t<2, 8>(p, grid, s);
-    case 4: return big ? launch_gqa_t<4, 16>(p, grid, s) : launch_gqa_t<4, 8>(p, grid, s);
+    case 1: return big ? launch_fmt<1, 16>(p, grid, s) : launch_fmt<1, 8>(p, grid, s);
+    case 2: return big ? launch_fmt<2, 16>(p, grid, s) : launch_fmt<2, 8>(p, grid, s);
+    case 4: return big ? launch_fmt<4, 16>(p, grid, s) : launch_fmt<4, 8>(p, grid, s);
     default: return cudaErrorInvalidValue;
   }
 }

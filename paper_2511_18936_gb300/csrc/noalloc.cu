@@ -103,6 +103,9 @@ extern "C" swan_status swan_decode_noalloc(const swan_cache_view* v, const void*
     return err(SWAN_ERR_INVALID_ARG, "NULL pages or page table");
   if (v->buf_len > 0 && (!v->buf_k || !v->buf_v)) return err(SWAN_ERR_INVALID_ARG, "NULL buffer");
   if (!v->R_qk || !v->R_vo_t) return err(SWAN_ERR_INVALID_ARG, "NULL rotation matrix");
+  if (v->value_format != SWAN_VALUES_FP16 && v->value_format != SWAN_VALUES_FP8_E4M3)
+    return err(SWAN_ERR_INVALID_ARG, "value_format must be fp16 (0) or fp8 e4m3 (1)");
+  const int fmt = v->value_format == SWAN_VALUES_FP8_E4M3 ? kFmtFp8 : kFmtFp16;
   const int64_t nq = (int64_t)v->batch * v->n_q_heads;
   if (nq > kNoallocMaxQ) return err(SWAN_ERR_INVALID_ARG, "batch * n_q_heads exceeds 1024 (static scratch)");
 
@@ -155,7 +158,8 @@ extern "C" swan_status swan_decode_noalloc(const swan_cache_view* v, const void*
     p.geom.P = v->page_tokens;
     p.geom.k_slots = v->k_slots;
     p.geom.k_store = v->k_slots;
-    p.geom.page_bytes = (int64_t)v->page_tokens * v->k_slots * 6;
+    p.geom.fmt = fmt;
+    p.geom.page_bytes = (int64_t)v->page_tokens * v->k_slots * (fmt == kFmtFp8 ? 4 : 6);
     p.ring_k = static_cast<const __half*>(v->buf_k);
     p.ring_v = static_cast<const __half*>(v->buf_v);
     p.cap = v->buffer_cap > 0 ? v->buffer_cap : 1;

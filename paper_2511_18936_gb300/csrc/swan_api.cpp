@@ -54,6 +54,7 @@ struct swan_ctx {
   int ppu = 0;  // pages per unit
   int64_t page_bytes = 0;
   int64_t num_pages = 0;
+  int fmt = kFmtFp16;
   int64_t units = 0;  // batch * n_kv_heads (per layer)
   cudaStream_t stream = nullptr;
   int device = 0;
@@ -187,6 +188,7 @@ CacheGeom geom_for(const swan_ctx* c, int layer) {
   g.k_slots = c->k_slots;
   g.k_store = c->cfg.k_store;
   g.page_bytes = c->page_bytes;
+  g.fmt = c->fmt;
   return g;
 }
 
@@ -204,6 +206,22 @@ swan_status check_layer(const swan_ctx* c, int layer) {
   if (layer < 0 || layer >= c->cfg.num_layers)
     return fail(SWAN_ERR_INVALID_ARG, "layer %d out of range [0, %d)", layer, c->cfg.num_layers);
   return SWAN_OK;
+}
+
+// An E4M3 byte widened to fp16 bits (exact: every E4M3 value is an fp16
+// value).  E4M3: sign, 4 exponent bits (bias 7), 3 mantissa bits;
+// exponent 0 holds the subnormals m * 2^-9; S.1111.111 is NaN.
+uint16_t e4m3_to_half_bits(uint8_t b) {
+  const uint16_t sign = (uint16_t)((b & 0x80u) << 8);
+  const int e = (b >> 3) & 15, m = b & 7;
+  if (e == 15 && m == 7) return sign | 0x7e00u;
+  if (e == 0 && m == 0) return sign;
+  double v = e == 0 ? std::ldexp((double)m, -9) : std::ldexp((double)(8 + m), e - 10);
+  int ex = 0;
+  const double fr = std::frexp(v, &ex);  // v = fr * 2^ex, fr in [0.5, 1)
+  const int he = ex - 1 + 15;            // fp16 biased exponent (always >= 6 here)
+  const int hm = (int)std::lround((fr * 2.0 - 1.0) * 1024.0);
+  return sign | (uint16_t)(he << 10) | (uint16_t)hm;
 }
 
 // Prune buffered tokens 0..count-1 of a layer into the sparse cache.
@@ -274,6 +292,8 @@ swan_status swan_init(swan_ctx** out, const swan_config* cfg, const float* R_qk,
   if (C.buffer_cap < 0 || C.buffer_cap > kMaxBufferCap)
     return fail(SWAN_ERR_INVALID_ARG, "buffer_cap %d out of [0, %d]", C.buffer_cap, kMaxBufferCap);
   if (C.max_seq < 1) return fail(SWAN_ERR_INVALID_ARG, "max_seq must be >= 1");
+  if (C.value_format != SWAN_VALUES_FP16 && C.value_format != SWAN_VALUES_FP8_E4M3)
+    return fail(SWAN_ERR_INVALID_ARG, "value_format %d is neither fp16 (0) nor fp8 e4m3 (1)", C.value_format);
   const int P = C.page_tokens ? C.page_tokens : 128;
   if (P < 32 || P > 4096 || (P & (P - 1)))
     return fail(SWAN_ERR_INVALID_ARG, "page_tokens %d must be a power of two in [32, 4096]", P);
@@ -293,7 +313,8 @@ swan_status swan_init(swan_ctx** out, const swan_config* cfg, const float* R_qk,
   c->k_active = C.k_store;
   c->P = P;
   c->ppu = (int)((C.max_seq + P - 1) / P);
-  c->page_bytes = (int64_t)P * c->k_slots * 6;
+  c->fmt = C.value_format == SWAN_VALUES_FP8_E4M3 ? kFmtFp8 : kFmtFp16;
+  c->page_bytes = (int64_t)P * c->k_slots * (c->fmt == kFmtFp8 ? 4 : 6);
   c->units = (int64_t)C.batch * C.n_kv_heads;
   c->num_pages = (int64_t)C.num_layers * c->units * c->ppu;
   c->stream = static_cast<cudaStream_t>(C.stream);
@@ -555,6 +576,7 @@ swan_status swan_query(const swan_ctx* c, int layer, swan_layer_info* info) {
   info->page_tokens = c->P;
   info->page_bytes = c->page_bytes;
   info->device_bytes = c->device_bytes;
+  info->value_format = c->fmt == kFmtFp8 ? SWAN_VALUES_FP8_E4M3 : SWAN_VALUES_FP16;
   return SWAN_OK;
 }
 
@@ -593,10 +615,14 @@ swan_status swan_debug_export(swan_ctx* c, int layer, int what, void* host_dst, 
     if (bytes != need) return fail(SWAN_ERR_INVALID_ARG, "bytes %zu != %zu", bytes, need);
     if (need == 0) return SWAN_OK;
     const bool isv = what == SWAN_EXPORT_SPARSE_V;
+    const bool fp8 = c->fmt == kFmtFp8;
     const int64_t P = c->P;
-    const int64_t blk = 192 * (int64_t)c->k_slots;
-    const int64_t voff = isv ? 96 * (int64_t)c->k_slots : 0;
-    const int64_t ioff = isv ? 160 * (int64_t)c->k_slots : 64 * (int64_t)c->k_slots;
+    const int64_t ks8 = c->k_slots;
+    const int64_t blk = (fp8 ? 128 : 192) * ks8;
+    // fp16: value records of 16 B and index records of 8 B in separate
+    // regions; fp8: 16-byte records of 8 values then 8 indices
+    const int64_t voff = fp8 ? (isv ? 64 * ks8 : 0) : (isv ? 96 * ks8 : 0);
+    const int64_t ioff = fp8 ? voff + 8 : (isv ? 160 * ks8 : 64 * ks8);
     std::vector<int32_t> pt((size_t)c->units * c->ppu);
     e = cudaMemcpy(pt.data(), c->page_table + (int64_t)layer * c->units * c->ppu, pt.size() * 4,
                    cudaMemcpyDeviceToHost);
@@ -619,10 +645,15 @@ swan_status swan_debug_export(swan_ctx* c, int layer, int what, void* host_dst, 
           for (int r = 0; r < ks; ++r) {
             const int64_t rec = (int64_t)(r / 8) * 32 + (sl % 32);
             const size_t o = ((size_t)u * L.sparse_len + t) * ks + r;
-            idx_dst[o] = page[b0 + ioff + rec * 8 + (r % 8)];
-            uint16_t v;
-            std::memcpy(&v, page.data() + b0 + voff + rec * 16 + (r % 8) * 2, 2);
-            val_dst[o] = v;
+            if (fp8) {
+              idx_dst[o] = page[b0 + ioff + rec * 16 + (r % 8)];
+              val_dst[o] = e4m3_to_half_bits(page[b0 + voff + rec * 16 + (r % 8)]);
+            } else {
+              idx_dst[o] = page[b0 + ioff + rec * 8 + (r % 8)];
+              uint16_t v;
+              std::memcpy(&v, page.data() + b0 + voff + rec * 16 + (r % 8) * 2, 2);
+              val_dst[o] = v;
+            }
           }
         }
       }

@@ -1,11 +1,10 @@
 // Internal definitions shared by the host library and the kernels.
 //
 // Sparse cache page layout (Section 5.1's values + 8-bit indices, arranged
-// for 128-bit coalesced loads on sm_103a).  A page holds P tokens (P a
-// multiple of 32) of one (layer, batch, kv-head) unit, as P/32 consecutive
+// for 128-bit coalesced loads on sm_103a).  A page holds P tokens (P a power
+// of two >= 32) of one (layer, batch, kv-head) unit, as P/32 consecutive
 // blocks of 32 tokens.  Each vector's kept entries are grouped in chunks of
-// 8, in stored (decreasing magnitude) order; chunk c of token t is a 16-byte
-// record of 8 fp16 values and an 8-byte record of 8 uint8 indices.  A block
+// 8, in stored (decreasing magnitude) order.  With fp16 values a block
 // (192 * k_slots bytes) is
 //
 //   [K values  : k_slots/8 chunks][32 tokens][8 x fp16]   at 0
@@ -13,11 +12,17 @@
 //   [V values  : same shape as K values]                  at 96 * k_slots
 //   [V indices : same shape as K indices]                 at 160 * k_slots
 //
+// and with 8-bit (E4M3) values (Section 4.3, Section 5.1) a block
+// (128 * k_slots bytes) is
+//
+//   [K records : k_slots/8 chunks][32 tokens][8 x e4m3, 8 x uint8]  at 0
+//   [V records : same shape]                                         at 64 * k_slots
+//
 // A warp that handles the 32 tokens of a block (one per lane) reads chunk c
-// of all of them as one contiguous 512-byte run (values) and one 256-byte run
-// (indices), at compile-time offsets from the region base.  A runtime keep
-// count k_active <= k_store reads only the first ceil(k_active / 8) chunks:
-// a contiguous prefix of each region.
+// of all of them as one contiguous 512-byte run (values or records), at
+// compile-time offsets from the region base.  A runtime keep count
+// k_active <= k_store reads only the first ceil(k_active / 8) chunks: a
+// contiguous prefix of each region.
 #pragma once
 
 #include <cuda_fp16.h>
@@ -38,6 +43,9 @@ constexpr float kLazyRescale = 8.0f;
 constexpr unsigned kStatusPageRange = 1u;
 constexpr unsigned kStatusRingRange = 2u;
 
+constexpr int kFmtFp16 = 0;  // fp16 values
+constexpr int kFmtFp8 = 1;   // E4M3 values
+
 struct CacheGeom {
   uint8_t* pool;             // all pages of all layers
   const int32_t* page_table; // this layer: [units][pages_per_unit] -> page id
@@ -46,11 +54,12 @@ struct CacheGeom {
   int P;                     // tokens per page
   int k_slots;               // k_store rounded up to 8
   int k_store;
-  int64_t page_bytes;        // P * k_slots * 6
-  // offsets inside a 32-token block
-  __device__ __host__ int block_bytes() const { return 192 * k_slots; }
+  int64_t page_bytes;        // P / 32 * block_bytes()
+  int fmt;                   // kFmtFp16 or kFmtFp8
+  // offsets inside a 32-token block (index regions: fp16 only)
+  __device__ __host__ int block_bytes() const { return (fmt == kFmtFp8 ? 128 : 192) * k_slots; }
   __device__ __host__ int kidx_off() const { return 64 * k_slots; }
-  __device__ __host__ int vval_off() const { return 96 * k_slots; }
+  __device__ __host__ int vval_off() const { return (fmt == kFmtFp8 ? 64 : 96) * k_slots; }
   __device__ __host__ int vidx_off() const { return 160 * k_slots; }
 };
 
@@ -179,7 +188,6 @@ cudaError_t launch_combine(const CombineParams& p, int B, cudaStream_t s);
 cudaError_t launch_transpose_r(const float* src, float* dst, int64_t mats, cudaStream_t s);
 // Decode CTAs that fit on one SM together (for the grid size).
 int decode_ctas_per_sm(int G, int k_slots);
-size_t decode_smem_bytes(int G, int k_slots);
 // Record the detail string that swan_last_error() returns on this thread.
 void set_last_error(const char* msg);
 

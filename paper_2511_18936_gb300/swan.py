@@ -18,6 +18,7 @@ LIB_PATH = os.path.join(_PKG, "libswan.so")
 OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_CAPACITY, ERR_CUDA, ERR_STATE, \
     ERR_DEVICE_TIMEOUT, ERR_NOMEM, ERR_DEVICE_CHECK = range(9)
 EXPORT_BUFFER_K, EXPORT_BUFFER_V, EXPORT_SPARSE_K, EXPORT_SPARSE_V = 1, 2, 3, 4
+VALUE_FORMATS = {"fp16": 0, "fp8_e4m3": 1}
 KERNEL_ROTATE_Q, KERNEL_DECODE, KERNEL_COMBINE, KERNEL_APPEND, KERNEL_PRUNE = range(5)
 KERNEL_KINDS = 8
 KERNEL_NAMES = {KERNEL_ROTATE_Q: "rotate_q", KERNEL_DECODE: "decode", KERNEL_COMBINE: "combine",
@@ -35,14 +36,15 @@ class SwanConfig(ctypes.Structure):
                 ("n_q_heads", ctypes.c_int), ("n_kv_heads", ctypes.c_int),
                 ("head_dim", ctypes.c_int), ("k_store", ctypes.c_int),
                 ("buffer_cap", ctypes.c_int), ("max_seq", ctypes.c_int),
-                ("page_tokens", ctypes.c_int), ("stream", ctypes.c_void_p)]
+                ("page_tokens", ctypes.c_int), ("stream", ctypes.c_void_p),
+                ("value_format", ctypes.c_int)]
 
 
 class LayerInfo(ctypes.Structure):
     _fields_ = [("sparse_len", ctypes.c_int64), ("buffer_len", ctypes.c_int64),
                 ("k_active", ctypes.c_int), ("k_store", ctypes.c_int), ("k_slots", ctypes.c_int),
                 ("page_tokens", ctypes.c_int), ("page_bytes", ctypes.c_int64),
-                ("device_bytes", ctypes.c_int64)]
+                ("device_bytes", ctypes.c_int64), ("value_format", ctypes.c_int)]
 
 
 class Timing(ctypes.Structure):
@@ -57,7 +59,8 @@ class CacheView(ctypes.Structure):
                 ("buf_k", ctypes.c_void_p), ("buf_v", ctypes.c_void_p), ("buffer_cap", ctypes.c_int),
                 ("buf_start", ctypes.c_int), ("buf_len", ctypes.c_int), ("sparse_len", ctypes.c_int64),
                 ("batch", ctypes.c_int), ("n_q_heads", ctypes.c_int), ("n_kv_heads", ctypes.c_int),
-                ("head_dim", ctypes.c_int), ("R_qk", ctypes.c_void_p), ("R_vo_t", ctypes.c_void_p)]
+                ("head_dim", ctypes.c_int), ("R_qk", ctypes.c_void_p), ("R_vo_t", ctypes.c_void_p),
+                ("value_format", ctypes.c_int)]
 
 
 class SwanError(RuntimeError):
@@ -131,14 +134,18 @@ class Context:
 
     def __init__(self, R_qk, R_vo=None, *, num_layers: int, batch: int, n_q_heads: int,
                  n_kv_heads: int, k_store: int, buffer_cap: int, max_seq: int,
-                 page_tokens: int = 0, head_dim: int = 128, stream=None):
+                 page_tokens: int = 0, head_dim: int = 128, stream=None,
+                 value_format: str = "fp16"):
         import torch
         self._lib = load_library()
         if stream is None:
             stream = torch.cuda.current_stream()
         self.stream = stream
+        if value_format not in VALUE_FORMATS:
+            raise ValueError(f"value_format must be one of {sorted(VALUE_FORMATS)}")
         self.cfg = SwanConfig(num_layers, batch, n_q_heads, n_kv_heads, head_dim, k_store,
-                              buffer_cap, max_seq, page_tokens, ctypes.c_void_p(stream.cuda_stream))
+                              buffer_cap, max_seq, page_tokens, ctypes.c_void_p(stream.cuda_stream),
+                              VALUE_FORMATS[value_format])
         self.batch, self.n_q_heads, self.n_kv_heads = batch, n_q_heads, n_kv_heads
         self.num_layers, self.k_store, self.head_dim = num_layers, k_store, head_dim
         h = ctypes.c_void_p()

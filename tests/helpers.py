@@ -10,7 +10,7 @@ TOL_OUT = 2e-3  # max-abs tolerance on attention outputs (fp16 storage, fp32 acc
 
 
 def run_ops(ops, R, Rv, *, B, H_kv, G, k_store, cap, max_seq=None, page_tokens=0,
-            check_each=True):
+            check_each=True, value_format="fp16"):
     """Replay ``ops`` on the oracle and on a libswan context.
 
     ops: ("append", k, v) | ("flush",) | ("set_k", k) | ("decode", q); all
@@ -23,11 +23,13 @@ def run_ops(ops, R, Rv, *, B, H_kv, G, k_store, cap, max_seq=None, page_tokens=0
     dev = torch.device("cuda")
     if max_seq is None:
         max_seq = sum(op[1].shape[2] for op in ops if op[0] == "append") or 1
-    ref = oracle.SwanOracle(R, Rv, batch=B, n_q_heads=H_kv * G, k_store=k_store, buffer_cap=cap)
+    ref = oracle.SwanOracle(R, Rv, batch=B, n_q_heads=H_kv * G, k_store=k_store, buffer_cap=cap,
+                            value_format=value_format)
     Rt = torch.from_numpy(np.asarray(R, np.float32))[None].to(dev).contiguous()
     Rvt = None if Rv is None else torch.from_numpy(np.asarray(Rv, np.float32))[None].to(dev).contiguous()
     ctx = swan.Context(Rt, Rvt, num_layers=1, batch=B, n_q_heads=H_kv * G, n_kv_heads=H_kv,
-                       k_store=k_store, buffer_cap=cap, max_seq=max_seq, page_tokens=page_tokens)
+                       k_store=k_store, buffer_cap=cap, max_seq=max_seq, page_tokens=page_tokens,
+                       value_format=value_format)
     outs = []
     for op in ops:
         if op[0] == "append":

@@ -19,7 +19,8 @@ pytestmark = pytest.mark.gpu
 D = 128
 
 
-def _layer_case(B, H_q, H_kv, L_s, n_b, k_store, k_actives, samples, seed=0, steps=2):
+def _layer_case(B, H_q, H_kv, L_s, n_b, k_store, k_actives, samples, seed=0, steps=2,
+                value_format="fp16"):
     """Prefill L_s + n_b tokens, then `steps` decode steps (append one token +
     decode at every k in k_actives); compare sampled units with the oracle."""
     import torch
@@ -29,14 +30,16 @@ def _layer_case(B, H_q, H_kv, L_s, n_b, k_store, k_actives, samples, seed=0, ste
     G = H_q // H_kv
     R = synth.rotations(H_kv, D, seed=seed, workload=1, layer=0)
     ctx = swan.Context(torch.from_numpy(R)[None].to(dev), num_layers=1, batch=B, n_q_heads=H_q,
-                       n_kv_heads=H_kv, k_store=k_store, buffer_cap=n_b, max_seq=L_s + n_b + steps)
+                       n_kv_heads=H_kv, k_store=k_store, buffer_cap=n_b, max_seq=L_s + n_b + steps,
+                       value_format=value_format)
     kk = synth.torch_lowrank_kv(B, H_kv, L_s + n_b + steps, D, seed, synth.T_K, dev)
     vv = synth.torch_lowrank_kv(B, H_kv, L_s + n_b + steps, D, seed, synth.T_V, dev)
     ctx.append(0, kk[:, :, :L_s + n_b].contiguous(), vv[:, :, :L_s + n_b].contiguous())
     qs = synth.torch_gaussian_fp16((steps, B, H_q, D), seed, synth.T_Q, dev)
     refs = {}
     for b, h in samples:
-        st = oracle.SwanOracle(R[h:h + 1], batch=1, n_q_heads=G, k_store=k_store, buffer_cap=n_b)
+        st = oracle.SwanOracle(R[h:h + 1], batch=1, n_q_heads=G, k_store=k_store, buffer_cap=n_b,
+                               value_format=value_format)
         st.append(kk[b:b + 1, h:h + 1, :L_s + n_b].cpu().numpy(), vv[b:b + 1, h:h + 1, :L_s + n_b].cpu().numpy())
         refs[(b, h)] = st
     worst = 0.0
@@ -65,6 +68,11 @@ def _layer_case(B, H_q, H_kv, L_s, n_b, k_store, k_actives, samples, seed=0, ste
 def test_llama2_layer_32k_sampled():
     _layer_case(B=16, H_q=32, H_kv=32, L_s=32768, n_b=128, k_store=64, k_actives=(64,),
                 samples=[(0, 0), (7, 19), (15, 31)])
+
+
+def test_llama2_layer_32k_fp8_values_sampled():
+    _layer_case(B=16, H_q=32, H_kv=32, L_s=32768, n_b=128, k_store=64, k_actives=(64,),
+                samples=[(1, 2), (14, 29)], value_format="fp8_e4m3")
 
 
 def test_gqa_131k_sampled():

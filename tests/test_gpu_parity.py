@@ -354,3 +354,59 @@ def test_multi_layer_state_is_independent():
         assert np.abs(got - ref.decode(q)).max() <= TOL_OUT
     ctx.check()
     ctx.close()
+
+
+# ---------------------------------------------------------------------------
+# 8-bit (E4M3) kept values (Section 4.3, Section 5.1)
+# ---------------------------------------------------------------------------
+
+@pytest.mark.parametrize("k_store,cap,P", [(64, 5, 128), (60, 0, 32), (128, 64, 64), (56, 128, 128)])
+def test_fp8_prune_bitexact_on_identical_rotated_inputs(k_store, cap, P):
+    B, H = 2, 3
+    eye = np.broadcast_to(np.eye(D, dtype=np.float32), (H, D, D)).copy()
+    R = _rot(H, 101)
+    kraw, vraw = _kv(B, H, 301, seed=102)
+    k16 = oracle.to_fp16(np.einsum("bhti,hij->bhtj", kraw.astype(np.float64), R.astype(np.float64)))
+    v16 = oracle.to_fp16(np.einsum("bhti,hij->bhtj", vraw.astype(np.float64), R.astype(np.float64)))
+    k16[0, 0, :40] = _tricky_vectors(40, 103)          # ties, +-0, values beyond 448
+    v16[1, 2, :40] = _tricky_vectors(40, 104) * np.float16(20)
+    ops = [("append", k16[:, :, :37].copy(), v16[:, :, :37].copy()),
+           ("append", k16[:, :, 37:38].copy(), v16[:, :, 37:38].copy()),
+           ("append", k16[:, :, 38:].copy(), v16[:, :, 38:].copy()), ("flush",)]
+    ctx, ref, _ = run_ops(ops, eye, None, B=B, H_kv=H, G=1, k_store=k_store, cap=cap, page_tokens=P,
+                          value_format="fp8_e4m3")
+    assert ctx.query(0).value_format == 1
+    for which, ri, rv in (("k", ref.sp_idx_k, ref.sp_val_k), ("v", ref.sp_idx_v, ref.sp_val_v)):
+        gi, gv = ctx.export_sparse(0, which)
+        assert np.array_equal(gi, ri), which
+        assert np.array_equal(gv.view(np.uint16), rv.view(np.uint16)), which
+    ctx.close()
+
+
+FP8_DECODE_CASES = [
+    # B, H_kv, G, L_total, cap, k_store, k_actives, page_tokens
+    (2, 2, 1, 1000, 64, 64, (64, 57, 16), 128),
+    (4, 8, 1, 2050, 128, 64, (64,), 128),
+    (2, 2, 4, 1500, 128, 56, (56, 13), 64),
+    (2, 4, 2, 777, 16, 60, (60, 7), 32),
+    (1, 2, 1, 700, 128, 128, (128, 96, 32), 128),
+]
+
+
+@pytest.mark.parametrize("B,H,G,L,cap,ks,kas,P", FP8_DECODE_CASES)
+def test_fp8_decode_matches_oracle(B, H, G, L, cap, ks, kas, P):
+    R, Rv = _rot(H, 120 + L), _rot(H, 120 + L, synth.T_R_VO)
+    k, v = _kv(B, H, L, seed=L + 7)
+    q = _q(B, H * G, seed=L + 8)
+    qp = _q(B, H * G, seed=L + 9, scale=4.0)
+    cut = max(1, L // 3)
+    ops = [("append", k[:, :, :cut].copy(), v[:, :, :cut].copy()), ("decode", q),
+           ("append", k[:, :, cut:].copy(), v[:, :, cut:].copy())]
+    for ka in kas:
+        ops += [("set_k", ka), ("decode", q), ("decode", qp)]
+    ctx, ref, outs = run_ops(ops, R, Rv, B=B, H_kv=H, G=G, k_store=ks, cap=cap, page_tokens=P,
+                             value_format="fp8_e4m3")
+    for got, want in outs:
+        err = np.abs(got - want).max()
+        assert err <= TOL_OUT, err
+    ctx.close()

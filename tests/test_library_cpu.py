@@ -44,7 +44,7 @@ def test_status_strings(lib):
 
 def _cfg(**kw):
     base = dict(num_layers=1, batch=1, n_q_heads=1, n_kv_heads=1, head_dim=128, k_store=64,
-                buffer_cap=64, max_seq=1024, page_tokens=0, stream=None)
+                buffer_cap=64, max_seq=1024, page_tokens=0, stream=None, value_format=0)
     base.update(kw)
     return swan.SwanConfig(*[base[f] for f, _ in swan.SwanConfig._fields_])
 
@@ -64,6 +64,8 @@ def _cfg(**kw):
     (dict(page_tokens=8192), swan.ERR_INVALID_ARG),
     (dict(num_layers=0), swan.ERR_INVALID_ARG),
     (dict(batch=0), swan.ERR_INVALID_ARG),
+    (dict(value_format=2), swan.ERR_INVALID_ARG),
+    (dict(value_format=-1), swan.ERR_INVALID_ARG),
 ])
 def test_init_rejects_bad_config_without_cuda(lib, kw, status):
     h = ctypes.c_void_p(123)

@@ -68,13 +68,14 @@ def measured_peaks():
         return None
 
 
-def decode_kernel_traffic(workload: str):
+def decode_kernel_traffic(workload: str, values: str = "fp16"):
     """DRAM bytes per decode-kernel launch from the committed ncu summary, if
     it was taken on the current kernel source (else None)."""
     src = os.path.join(ROOT, "paper_2511_18936_gb300", "csrc", "decode.cu")
     digest = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
     text = None
-    for name in (f"decode_kernel_{workload}.md", f"decode_gqa_kernel_{workload}.md"):
+    suffix = "" if values == "fp16" else "-fp8"
+    for name in (f"decode_kernel_{workload}{suffix}.md", f"decode_gqa_kernel_{workload}{suffix}.md"):
         try:
             text = open(os.path.join(ROOT, "profiles", name)).read()
             break
@@ -520,7 +521,7 @@ def run_swan(args, wl, rank: int, world: int, local_rank: int):
                      else "fallback 6.8 TB/s",
                      "pct_of_8tbs": 100.0 * achieved / NOMINAL_HBM_GBS,
                      "alg_bytes_per_launch": alg_decode, "avg_launch_ms": avg_dec_s * 1e3,
-                     "traffic": decode_kernel_traffic(args.workload)},
+                     "traffic": decode_kernel_traffic(args.workload, wl["values"])},
         "kernels_ms_per_step": {name: v[0] / args.steps for name, v in kt.items() if v[1]},
         "kernels_timed": "second timed region of the same length, CUDA events around every launch",
         "gpu_launches": launches,

@@ -151,15 +151,18 @@ def sparse_value_sum(p, idx, vals, d: int) -> np.ndarray:
 
 
 def swan_attend_unit(q_hat, sp_idx, sp_vals_k, sp_idx_v, sp_vals_v, buf_k, buf_v,
-                     k_active: int, d: int):
+                     k_active: int, d: int, k_active_v: int | None = None):
     """Attention of one rotated query over one unit's hybrid cache.
 
     Algorithm 1: ``S = q_hat Concat(K_sparse, K_buffer)^T``,
     ``o_hat = softmax(S / sqrt(d_h)) Concat(V_sparse, V_buffer)``; the sparse
-    vectors use their first ``k_active`` stored entries.  Returns
-    ``(o_hat, scores)`` with the scores already divided by ``sqrt(d)``.
+    keys use their first ``k_active`` stored entries, the sparse values their
+    first ``k_active_v`` (default: the same; the appendix ablation varies the
+    two).  Returns ``(o_hat, scores)`` with the scores already divided by
+    ``sqrt(d)``.
     """
     ka = k_active
+    kv = k_active if k_active_v is None else k_active_v
     s_sp = sparse_scores(q_hat, sp_idx[:, :ka], sp_vals_k[:, :ka])
     s_bf = np.asarray(buf_k, np.float64) @ np.asarray(q_hat, np.float64)
     s = np.concatenate([s_sp, s_bf]) / math.sqrt(d)
@@ -169,7 +172,7 @@ def swan_attend_unit(q_hat, sp_idx, sp_vals_k, sp_idx_v, sp_vals_v, buf_k, buf_v
     e = np.exp(s - m)
     p = e / e.sum()
     n_sp = s_sp.shape[0]
-    o = sparse_value_sum(p[:n_sp], sp_idx_v[:, :ka], sp_vals_v[:, :ka], d)
+    o = sparse_value_sum(p[:n_sp], sp_idx_v[:, :kv], sp_vals_v[:, :kv], d)
     o = o + p[n_sp:] @ np.asarray(buf_v, np.float64)
     return o, s
 
@@ -210,7 +213,8 @@ class SwanOracle:
     """
 
     def __init__(self, R_qk, R_vo=None, *, batch: int, n_q_heads: int, k_store: int,
-                 buffer_cap: int, round_rotated: bool = True, value_format: str = "fp16"):
+                 buffer_cap: int, round_rotated: bool = True, value_format: str = "fp16",
+                 k_store_v: int | None = None):
         self.R_qk = np.asarray(R_qk, np.float64)
         self.R_vo = self.R_qk if R_vo is None else np.asarray(R_vo, np.float64)
         self.H_kv, self.d, _ = self.R_qk.shape
@@ -219,10 +223,13 @@ class SwanOracle:
         if self.H_q % self.H_kv:
             raise ValueError("n_q_heads must be a multiple of n_kv_heads")
         self.G = self.H_q // self.H_kv
-        if not (1 <= k_store <= self.d):
+        k_store_v = k_store if k_store_v is None else k_store_v
+        if not (1 <= k_store <= self.d) or not (1 <= k_store_v <= self.d):
             raise ValueError("k_store out of range")
-        self.k_store = k_store
+        self.k_store = k_store      # keys
+        self.k_store_v = k_store_v  # values
         self.k_active = k_store
+        self.k_active_v = k_store_v
         self.b = buffer_cap
         self.round = round_rotated
         if value_format not in ("fp16", "fp8_e4m3"):
@@ -233,24 +240,24 @@ class SwanOracle:
         self.buf_v = np.zeros((self.B, self.H_kv, 0, self.d), vdt)
         self.sp_idx_k = np.zeros((self.B, self.H_kv, 0, k_store), np.uint8)
         self.sp_val_k = np.zeros((self.B, self.H_kv, 0, k_store), vdt)
-        self.sp_idx_v = np.zeros((self.B, self.H_kv, 0, k_store), np.uint8)
-        self.sp_val_v = np.zeros((self.B, self.H_kv, 0, k_store), vdt)
+        self.sp_idx_v = np.zeros((self.B, self.H_kv, 0, k_store_v), np.uint8)
+        self.sp_val_v = np.zeros((self.B, self.H_kv, 0, k_store_v), vdt)
 
     # -- Section 4.2 / Algorithm 1: rotate the incoming key and value -------
     def _rotate_store(self, x, R):
         y = np.einsum("bhti,hij->bhtj", np.asarray(x, np.float64), R)
         return to_fp16(y) if self.round else y
 
-    def _prune(self, x):
+    def _prune(self, x, k: int):
         if self.round:
-            idx, vals = prune(x, self.k_store)
+            idx, vals = prune(x, k)
             if self.fp8:
                 # the kept fp16 values are stored as E4M3 (exact in fp16)
                 vals = to_e4m3(vals.astype(np.float64)).astype(np.float16)
             return idx, vals
         # fp64 variant (lemma checks only): same rule on the fp64 vector
         mag = np.abs(x)
-        order = np.argsort(-mag, axis=-1, kind="stable")[..., : self.k_store]
+        order = np.argsort(-mag, axis=-1, kind="stable")[..., :k]
         return order.astype(np.uint8), np.take_along_axis(x, order, axis=-1)
 
     def _move_to_sparse(self, n: int):
@@ -258,8 +265,8 @@ class SwanOracle:
         separately) and append them to the sparse history."""
         if n <= 0:
             return
-        ik, vk = self._prune(self.buf_k[:, :, :n])
-        iv, vv = self._prune(self.buf_v[:, :, :n])
+        ik, vk = self._prune(self.buf_k[:, :, :n], self.k_store)
+        iv, vv = self._prune(self.buf_v[:, :, :n], self.k_store_v)
         self.sp_idx_k = np.concatenate([self.sp_idx_k, ik], axis=2)
         self.sp_val_k = np.concatenate([self.sp_val_k, vk], axis=2)
         self.sp_idx_v = np.concatenate([self.sp_idx_v, iv], axis=2)
@@ -280,10 +287,15 @@ class SwanOracle:
         """Move every buffered vector to the sparse history."""
         self._move_to_sparse(self.buf_k.shape[2])
 
-    def set_k(self, k_active: int):
-        if not (1 <= k_active <= self.k_store):
+    def set_k(self, k_active: int, k_active_v: int | None = None):
+        """Runtime keep counts for keys and values (values default to
+        ``min(k_active, k_store_v)``)."""
+        if k_active_v is None:
+            k_active_v = min(k_active, self.k_store_v)
+        if not (1 <= k_active <= self.k_store) or not (1 <= k_active_v <= self.k_store_v):
             raise ValueError("k_active out of range")
         self.k_active = k_active
+        self.k_active_v = k_active_v
 
     @property
     def sparse_len(self) -> int:
@@ -306,7 +318,7 @@ class SwanOracle:
                 o_hat, _ = swan_attend_unit(
                     q_hat, self.sp_idx_k[b, h], self.sp_val_k[b, h],
                     self.sp_idx_v[b, h], self.sp_val_v[b, h],
-                    self.buf_k[b, h], self.buf_v[b, h], self.k_active, self.d)
+                    self.buf_k[b, h], self.buf_v[b, h], self.k_active, self.d, self.k_active_v)
                 o_hat_all[b, hq] = o_hat
                 out[b, hq] = rotate_back(o_hat, self.R_vo[h])
         return (out, o_hat_all) if return_rotated else out
@@ -318,7 +330,7 @@ class SwanOracle:
         o_hat, _ = swan_attend_unit(
             q_hat, self.sp_idx_k[b, h], self.sp_val_k[b, h],
             self.sp_idx_v[b, h], self.sp_val_v[b, h],
-            self.buf_k[b, h], self.buf_v[b, h], self.k_active, self.d)
+            self.buf_k[b, h], self.buf_v[b, h], self.k_active, self.d, self.k_active_v)
         return rotate_back(o_hat, self.R_vo[h])
 
 

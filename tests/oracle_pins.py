@@ -276,7 +276,32 @@ def pin_fp8_cache_is_rounded_sparse_cache(o):
     assert np.abs(b.decode(q)[0, 0] - ref).max() < 1e-12
 
 
+# -- asymmetric keep counts for keys and values (appendix ablation) --------
+
+def pin_asymmetric_keep_counts(o):
+    """Keys keep k_K entries and values k_V: decoding equals dense attention
+    on keys zero-filled at k_K and values zero-filled at k_V; a runtime split
+    on a symmetric cache equals a cache stored with that split."""
+    R, Rv, k, v, q = _small_problem(71, B=1, H_kv=1, d=32, L=30)
+    st = o.SwanOracle(R, Rv, batch=1, n_q_heads=1, k_store=9, k_store_v=20, buffer_cap=4)
+    st.append(k, v)
+    assert st.sp_idx_k.shape[-1] == 9 and st.sp_idx_v.shape[-1] == 20
+    kh = (k[0, 0].astype(np.float64) @ R[0].astype(np.float64)).astype(np.float16)
+    vh = (v[0, 0].astype(np.float64) @ Rv[0].astype(np.float64)).astype(np.float16)
+    ik, vk = o.prune(kh[:26], 9)
+    iv, vv = o.prune(vh[:26], 20)
+    Kd = np.concatenate([o.densify(ik, vk, 32), kh[26:].astype(np.float64)])
+    Vd = np.concatenate([o.densify(iv, vv, 32), vh[26:].astype(np.float64)])
+    qh = q[0, 0].astype(np.float64) @ R[0].astype(np.float64)
+    ref = o.dense_attention(qh, Kd, Vd) @ Rv[0].astype(np.float64).T
+    assert np.abs(st.decode(q)[0, 0] - ref).max() < 1e-12
+    big = o.SwanOracle(R, Rv, batch=1, n_q_heads=1, k_store=32, buffer_cap=4)
+    big.append(k, v)
+    big.set_k(9, 20)
+    assert np.array_equal(big.decode(q), st.decode(q))
+
+
 ALL_PINS = [pin_rotation_orthogonal, pin_rotation_orientation, pin_prune_bruteforce,
             pin_k_equals_d_is_dense, pin_decompression_free, pin_buffer_semantics,
             pin_split_combine, pin_k_prefix, pin_gqa_mapping, pin_formulas, pin_e4m3_rounding,
-            pin_fp8_cache_is_rounded_sparse_cache]
+            pin_fp8_cache_is_rounded_sparse_cache, pin_asymmetric_keep_counts]

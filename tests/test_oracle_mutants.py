@@ -24,13 +24,13 @@ MUTANTS = [
     ("rotate_back_without_transpose",
      "@ np.asarray(R, np.float64).T", "@ np.asarray(R, np.float64)", 1),
     ("prune_smallest",
-     'np.argsort(-mag, axis=-1, kind="stable")[..., :k]',
-     'np.argsort(mag, axis=-1, kind="stable")[..., :k]', 1),
+     'np.argsort(-mag, axis=-1, kind="stable")[..., :k]\n    vals',
+     'np.argsort(mag, axis=-1, kind="stable")[..., :k]\n    vals', 1),
     ("prune_signed_not_magnitude",
      "mag = np.abs(x16.astype(np.float64))", "mag = x16.astype(np.float64)", 1),
     ("prune_ties_to_higher_index",
-     'order = np.argsort(-mag, axis=-1, kind="stable")[..., :k]',
-     'order = (mag.shape[-1] - 1 - np.argsort(-mag[..., ::-1], axis=-1, kind="stable"))[..., :k]', 1),
+     'order = np.argsort(-mag, axis=-1, kind="stable")[..., :k]\n    vals',
+     'order = (mag.shape[-1] - 1 - np.argsort(-mag[..., ::-1], axis=-1, kind="stable"))[..., :k]\n    vals', 1),
     ("scale_sqrt_k",
      "s = np.concatenate([s_sp, s_bf]) / math.sqrt(d)",
      "s = np.concatenate([s_sp, s_bf]) / math.sqrt(ka)", 1),
@@ -40,11 +40,17 @@ MUTANTS = [
      "w = np.asarray(p, np.float64)[:, None] * np.asarray(vals, np.float64)",
      "w = np.asarray(vals, np.float64) + 0 * np.asarray(p)[:, None]", 1),
     ("key_indices_used_for_values",
-     "o = sparse_value_sum(p[:n_sp], sp_idx_v[:, :ka]", "o = sparse_value_sum(p[:n_sp], sp_idx[:, :ka]", 1),
+     "o = sparse_value_sum(p[:n_sp], sp_idx_v[:, :kv]", "o = sparse_value_sum(p[:n_sp], sp_idx[:, :kv]", 1),
     ("combine_wrong_sign",
      "np.exp(ms - m)", "np.exp(m - ms)", 1),
     ("evict_newest",
-     "ik, vk = self._prune(self.buf_k[:, :, :n])", "ik, vk = self._prune(self.buf_k[:, :, -n:])", 1),
+     "ik, vk = self._prune(self.buf_k[:, :, :n], self.k_store)",
+     "ik, vk = self._prune(self.buf_k[:, :, -n:], self.k_store)", 1),
+    ("keys_pruned_with_the_value_count",
+     "ik, vk = self._prune(self.buf_k[:, :, :n], self.k_store)",
+     "ik, vk = self._prune(self.buf_k[:, :, :n], self.k_store_v)", 1),
+    ("values_use_the_key_keep_count",
+     "kv = k_active if k_active_v is None else k_active_v", "kv = k_active", 1),
     ("gqa_modulo_mapping",
      "h = hq // self.G\n                q_hat", "h = hq % self.H_kv\n                q_hat", 1),
     ("no_fp16_storage",

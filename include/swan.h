@@ -80,6 +80,9 @@ typedef struct swan_config {
                        E4M3, round to nearest even, saturating to +-448; the
                        entries are still chosen on the fp16 vector and the
                        dense buffer stays fp16 */
+  int k_store_v;   /* value entries kept per vector, 1..d; 0 = k_store.  Keys
+                      and values may keep different counts (Appendix,
+                      ablation on key and value pruning ratios) */
 } swan_config;
 
 enum { SWAN_VALUES_FP16 = 0, SWAN_VALUES_FP8_E4M3 = 1 };
@@ -108,6 +111,14 @@ swan_status swan_destroy(swan_ctx* ctx);
  * Errors: INVALID_ARG unless 1 <= k_active <= k_store.
  */
 swan_status swan_set_k(swan_ctx* ctx, int k_active);
+
+/*
+ * Separate runtime keep counts for keys (1..k_store) and values
+ * (1..k_store_v) (Appendix, ablation on key and value pruning ratios).
+ * swan_set_k(ctx, k) is swan_set_kv(ctx, k, min(k, k_store_v)).
+ * Errors: INVALID_ARG when a count is out of range.
+ */
+swan_status swan_set_kv(swan_ctx* ctx, int k_active, int k_active_v);
 
 /*
  * Append T tokens to every sequence of one layer (Algorithm 1, generalised
@@ -157,6 +168,9 @@ typedef struct swan_layer_info {
   int64_t page_bytes;   /* bytes of one page (keys and values) */
   int64_t device_bytes; /* device memory owned by the whole context */
   int value_format;     /* SWAN_VALUES_FP16 or SWAN_VALUES_FP8_E4M3 */
+  int k_active_v;       /* value entries used per vector */
+  int k_store_v;        /* value entries stored per vector */
+  int k_slots_v;        /* k_store_v rounded up to a multiple of 8 */
 } swan_layer_info;
 
 swan_status swan_query(const swan_ctx* ctx, int layer, swan_layer_info* info);
@@ -167,7 +181,8 @@ swan_status swan_query(const swan_ctx* ctx, int layer, swan_layer_info* info);
  *   SWAN_EXPORT_BUFFER_K / _V: fp16 [batch][n_kv_heads][buffer_len][d],
  *     oldest first.
  *   SWAN_EXPORT_SPARSE_K / _V: uint8 indices [batch][n_kv_heads]
- *     [sparse_len][k_store], then fp16 values of the same shape, each vector's
+ *     [sparse_len][k_store] (k_store_v for _V), then fp16 values of the same
+ *     shape, each vector's
  *     entries in stored (decreasing magnitude) order (8-bit values are
  *     widened to fp16, exactly).
  * bytes must equal the exact size of the requested view.
@@ -224,13 +239,14 @@ swan_status swan_timing_read(swan_ctx* ctx, swan_timing* out);
  * view: the caller's cache, all pointers device pointers on the current
  *   device, caller-owned:
  *   pages       page pool; page p holds P = page_tokens tokens as P/32
- *               blocks of 32 tokens.  With fp16 values a block is
- *               192 * k_slots bytes: K values [k_slots/8][32][8] fp16 at 0,
- *               K indices [k_slots/8][32][8] uint8 at 64 * k_slots, V values
- *               at 96 * k_slots, V indices at 160 * k_slots.  With E4M3
- *               values a block is 128 * k_slots bytes: K records
- *               [k_slots/8][32][16 bytes] at 0 (8 E4M3 values, then 8
- *               indices), V records at 64 * k_slots.  Page p starts at
+ *               blocks of 32 tokens; keys keep ks = k_slots and values
+ *               vs = k_slots_v entries.  With fp16 values a block is
+ *               96 * (ks + vs) bytes: K values [ks/8][32][8] fp16 at 0,
+ *               K indices [ks/8][32][8] uint8 at 64 * ks, V values
+ *               [vs/8][32][8] at 96 * ks, V indices at 96 * ks + 64 * vs.
+ *               With E4M3 values a block is 64 * (ks + vs) bytes: K records
+ *               [ks/8][32][16 bytes] at 0 (8 E4M3 values, then 8 indices),
+ *               V records [vs/8][32][16 bytes] at 64 * ks.  Page p starts at
  *               pages + p * (P / 32) * block bytes.  Chunk c of token t holds
  *               entries 8c..8c+7 of the token's kept coordinates in
  *               decreasing magnitude order; indices must be < 128.  This is
@@ -280,6 +296,8 @@ typedef struct swan_cache_view {
   const float* R_qk;
   const float* R_vo_t;
   int value_format;      /* SWAN_VALUES_FP16 or SWAN_VALUES_FP8_E4M3 */
+  int k_slots_v;         /* value entries stored per vector; 0 = k_slots */
+  int k_active_v;        /* value entries used; 0 = k_active */
 } swan_cache_view;
 swan_status swan_decode_noalloc(const swan_cache_view* view, const void* q, void* out,
                                 void* stream);

@@ -62,12 +62,14 @@ __device__ __forceinline__ void warp_prune_store(uint2 raw, int lane, int kind, 
   }
   uint8_t* blk = g.pool + (int64_t)phys * g.page_bytes + (int64_t)(slot >> 5) * g.block_bytes();
   const int t = slot & 31;
-  if (lane < (g.k_slots >> 2)) {
+  const int slots = kind ? g.k_slots_v : g.k_slots;
+  const int kept = kind ? g.k_store_v : g.k_store;
+  if (lane < (slots >> 2)) {
     const int c = lane >> 1, half = lane & 1;
     uint32_t vb[4], ib[4];
 #pragma unroll
     for (int s = 0; s < 4; ++s) {
-      const bool keep = (4 * lane + s) < g.k_store;
+      const bool keep = (4 * lane + s) < kept;
       const uint32_t j = 127u - ((key[s] >> 1) & 127u);
       const uint32_t bits = ((key[s] & 1u) << 15) | (key[s] >> 16);
       vb[s] = keep ? bits : 0u;

@@ -285,13 +285,14 @@ __global__ void __launch_bounds__(decode_warps<MAXC>() * 32, 1) decode_kernel(De
   const uint32_t ab = base + (1 + warp) * kRegionBytes + (lane << 2);
 
   const CacheGeom& g = p.geom;
-  const int kfull = p.k_full_chunks, krem = p.k_rem;
+  const int kfull = p.k_full_chunks, krem = p.k_rem;          // keys
   const int nchunks = kfull + (krem ? 1 : 0);
-  const int ks = g.k_slots;
+  const int kfull_v = p.k_full_chunks_v, krem_v = p.k_rem_v;  // values
+  const int nchunks_v = kfull_v + (krem_v ? 1 : 0);
   // this lane's record runs inside a block
   const int o_kv = lane * 16, o_ki = g.kidx_off() + lane * 8;
   const int o_vv = g.vval_off() + lane * 16, o_vi = g.vidx_off() + lane * 8;
-  const bool whole_block = nchunks * 8 == ks;
+  const bool whole_block = nchunks * 8 == g.k_slots && nchunks_v * 8 == g.k_slots_v;
   const int bsh = p.blocks_per_page_log2, bmask = (1 << bsh) - 1;
 
   const int64_t g_begin = (int64_t)blockIdx.x * p.range;
@@ -339,11 +340,11 @@ __global__ void __launch_bounds__(decode_warps<MAXC>() * 32, 1) decode_kernel(De
       } else if constexpr (FMT == kFmtFp16) {
         prefetch_l2(blk, nchunks * 512u);
         prefetch_l2(blk + g.kidx_off(), nchunks * 256u);
-        prefetch_l2(blk + g.vval_off(), nchunks * 512u);
-        prefetch_l2(blk + g.vidx_off(), nchunks * 256u);
+        prefetch_l2(blk + g.vval_off(), nchunks_v * 512u);
+        prefetch_l2(blk + g.vidx_off(), nchunks_v * 256u);
       } else {
         prefetch_l2(blk, nchunks * 512u);
-        prefetch_l2(blk + g.vval_off(), nchunks * 512u);
+        prefetch_l2(blk + g.vval_off(), nchunks_v * 512u);
       }
     };
 
@@ -372,7 +373,7 @@ __global__ void __launch_bounds__(decode_warps<MAXC>() * 32, 1) decode_kernel(De
         Chunk<FMT> vc[MAXC];
 #pragma unroll
         for (int c = 0; c < MAXC; ++c)
-          if (c < nchunks) vc[c] = load_chunk<FMT, false>(src + o_vv, src + o_vi, c);
+          if (c < nchunks_v) vc[c] = load_chunk<FMT, false>(src + o_vv, src + o_vi, c);
         // two blocks ahead: into L2
         const uint8_t* b_n2 = block_of(gi + 2);
         prefetch_block(b_n2);
@@ -414,7 +415,7 @@ __global__ void __launch_bounds__(decode_warps<MAXC>() * 32, 1) decode_kernel(De
 
 #pragma unroll
         for (int c = 0; c < MAXC; ++c)
-          if (c < kfull) {
+          if (c < kfull_v) {
             float f[8];
             chunk_vals<FMT>(vc[c], f);
             uint2 ix = chunk_idx<FMT>(vc[c]);
@@ -424,13 +425,13 @@ __global__ void __launch_bounds__(decode_warps<MAXC>() * 32, 1) decode_kernel(De
             }
             value_chunk(ab, pr, f, ix);
           }
-        if (krem && valid) {
+        if (krem_v && valid) {
 #pragma unroll
           for (int c = 0; c < MAXC; ++c)
-            if (c == kfull) {
+            if (c == kfull_v) {
               float f[8];
               chunk_vals<FMT>(vc[c], f);
-              value_chunk_partial(ab, pr, f, chunk_idx<FMT>(vc[c]), krem);
+              value_chunk_partial(ab, pr, f, chunk_idx<FMT>(vc[c]), krem_v);
             }
         }
       } else {
@@ -633,10 +634,11 @@ __global__ void __launch_bounds__(kGqaWarps * 32, 1) decode_gqa_kernel(DecodePar
   const uint32_t ab = base + (1 + warp) * kPairRegionBytes + (lane << 3);
 
   const CacheGeom& g = p.geom;
-  const int kfull = p.k_full_chunks, krem = p.k_rem;
+  const int kfull = p.k_full_chunks, krem = p.k_rem;          // keys
   const int nchunks = kfull + (krem ? 1 : 0);
-  const int ks = g.k_slots;
-  const bool whole_block = nchunks * 8 == ks;
+  const int kfull_v = p.k_full_chunks_v, krem_v = p.k_rem_v;  // values
+  const int nchunks_v = kfull_v + (krem_v ? 1 : 0);
+  const bool whole_block = nchunks * 8 == g.k_slots && nchunks_v * 8 == g.k_slots_v;
   const int bsh = p.blocks_per_page_log2, bmask = (1 << bsh) - 1;
 
   const int64_t g_begin = (int64_t)blockIdx.x * p.range;
@@ -685,11 +687,11 @@ __global__ void __launch_bounds__(kGqaWarps * 32, 1) decode_gqa_kernel(DecodePar
       } else if constexpr (FMT == kFmtFp16) {
         prefetch_l2(blk, nchunks * 512u);
         prefetch_l2(blk + g.kidx_off(), nchunks * 256u);
-        prefetch_l2(blk + g.vval_off(), nchunks * 512u);
-        prefetch_l2(blk + g.vidx_off(), nchunks * 256u);
+        prefetch_l2(blk + g.vval_off(), nchunks_v * 512u);
+        prefetch_l2(blk + g.vidx_off(), nchunks_v * 256u);
       } else {
         prefetch_l2(blk, nchunks * 512u);
-        prefetch_l2(blk + g.vval_off(), nchunks * 512u);
+        prefetch_l2(blk + g.vval_off(), nchunks_v * 512u);
       }
     };
     // records of item `half` of a block for this lane's token
@@ -724,7 +726,7 @@ __global__ void __launch_bounds__(kGqaWarps * 32, 1) decode_gqa_kernel(DecodePar
         Chunk<FMT> vc[MAXC];
 #pragma unroll
         for (int c = 0; c < MAXC; ++c)
-          if (c < nchunks)
+          if (c < nchunks_v)
             vc[c] = load_chunk<FMT, true>(src + g.vval_off() + tt * 16, src + g.vidx_off() + tt * 8, c);
         const bool last_half = half == HALVES - 1;
         const uint8_t* b_n2 = nullptr;
@@ -783,7 +785,7 @@ __global__ void __launch_bounds__(kGqaWarps * 32, 1) decode_gqa_kernel(DecodePar
 
 #pragma unroll
         for (int c = 0; c < MAXC; ++c)
-          if (c < kfull) {
+          if (c < kfull_v) {
             float f[8];
             chunk_vals<FMT>(vc[c], f);
             uint2 ix = chunk_idx<FMT>(vc[c]);
@@ -793,13 +795,13 @@ __global__ void __launch_bounds__(kGqaWarps * 32, 1) decode_gqa_kernel(DecodePar
             }
             value2_chunk(ab, p0, p1, f, ix);
           }
-        if (krem && valid) {
+        if (krem_v && valid) {
 #pragma unroll
           for (int c = 0; c < MAXC; ++c)
-            if (c == kfull) {
+            if (c == kfull_v) {
               float f[8];
               chunk_vals<FMT>(vc[c], f);
-              value2_chunk_partial(ab, p0, p1, f, chunk_idx<FMT>(vc[c]), krem);
+              value2_chunk_partial(ab, p0, p1, f, chunk_idx<FMT>(vc[c]), krem_v);
             }
         }
       } else {

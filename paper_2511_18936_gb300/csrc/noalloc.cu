@@ -92,6 +92,11 @@ extern "C" swan_status swan_decode_noalloc(const swan_cache_view* v, const void*
   if (v->k_slots < 8 || v->k_slots > kHeadDim || v->k_slots % 8)
     return err(SWAN_ERR_INVALID_ARG, "k_slots must be a multiple of 8 in [8, 128]");
   if (v->k_active < 1 || v->k_active > v->k_slots) return err(SWAN_ERR_INVALID_ARG, "k_active out of range");
+  const int ksv = v->k_slots_v ? v->k_slots_v : v->k_slots;    // 0: as for keys
+  const int kav = v->k_active_v ? v->k_active_v : v->k_active;
+  if (ksv < 8 || ksv > kHeadDim || ksv % 8)
+    return err(SWAN_ERR_INVALID_ARG, "k_slots_v must be a multiple of 8 in [8, 128]");
+  if (kav < 1 || kav > ksv) return err(SWAN_ERR_INVALID_ARG, "k_active_v out of range");
   if (v->page_tokens < 32 || v->page_tokens > 4096 || (v->page_tokens & (v->page_tokens - 1)))
     return err(SWAN_ERR_INVALID_ARG, "page_tokens must be a power of two in [32, 4096]");
   if (v->sparse_len < 0 || v->buf_len < 0 || v->buf_len > v->buffer_cap || v->buffer_cap < 0 ||
@@ -122,7 +127,8 @@ extern "C" swan_status swan_decode_noalloc(const swan_cache_view* v, const void*
   const int64_t total = units * N_g;
   int64_t range = 1, grid = 0;
   if (total > 0) {
-    const int64_t ctas = std::min<int64_t>((int64_t)ds->sms * ds->ctas_per_sm[gi(G)][v->k_active > 64], total);
+    const int64_t ctas =
+        std::min<int64_t>((int64_t)ds->sms * ds->ctas_per_sm[gi(G)][std::max(v->k_active, kav) > 64], total);
     range = (total + ctas - 1) / ctas;
     grid = (total + range - 1) / range;
   }
@@ -158,8 +164,10 @@ extern "C" swan_status swan_decode_noalloc(const swan_cache_view* v, const void*
     p.geom.P = v->page_tokens;
     p.geom.k_slots = v->k_slots;
     p.geom.k_store = v->k_slots;
+    p.geom.k_slots_v = ksv;
+    p.geom.k_store_v = ksv;
     p.geom.fmt = fmt;
-    p.geom.page_bytes = (int64_t)v->page_tokens * v->k_slots * (fmt == kFmtFp8 ? 4 : 6);
+    p.geom.page_bytes = page_bytes_for(v->page_tokens, v->k_slots, ksv, fmt);
     p.ring_k = static_cast<const __half*>(v->buf_k);
     p.ring_v = static_cast<const __half*>(v->buf_v);
     p.cap = v->buffer_cap > 0 ? v->buffer_cap : 1;
@@ -175,13 +183,15 @@ extern "C" swan_status swan_decode_noalloc(const swan_cache_view* v, const void*
     p.blocks_per_page_log2 = __builtin_ctz((unsigned)(v->page_tokens / 32));
     p.k_full_chunks = v->k_active / 8;
     p.k_rem = v->k_active % 8;
+    p.k_full_chunks_v = kav / 8;
+    p.k_rem_v = kav % 8;
     p.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)kHeadDim));
     p.partials = partials;
     p.counters = counters;
     p.R_voT = v->R_vo_t;
     p.out = static_cast<__half*>(out);
     p.status = status;
-    if (launch_decode(p, G, (v->k_active + 7) / 8 * 8, (int)grid, s) != cudaSuccess)
+    if (launch_decode(p, G, (std::max(v->k_active, kav) + 7) / 8 * 8, (int)grid, s) != cudaSuccess)
       return err(SWAN_ERR_CUDA, "decode launch failed");
     return SWAN_OK;
   }

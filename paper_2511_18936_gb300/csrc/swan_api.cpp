@@ -48,8 +48,11 @@ struct EventPair {
 struct swan_ctx {
   swan_config cfg{};
   int G = 1;
-  int k_slots = 0;
+  int k_slots = 0;    // key entries stored per vector, rounded up to 8
   int k_active = 0;
+  int k_store_v = 0;  // value entries kept per vector
+  int k_slots_v = 0;
+  int k_active_v = 0;
   int P = 128;
   int ppu = 0;  // pages per unit
   int64_t page_bytes = 0;
@@ -187,6 +190,8 @@ CacheGeom geom_for(const swan_ctx* c, int layer) {
   g.P = c->P;
   g.k_slots = c->k_slots;
   g.k_store = c->cfg.k_store;
+  g.k_slots_v = c->k_slots_v;
+  g.k_store_v = c->k_store_v;
   g.page_bytes = c->page_bytes;
   g.fmt = c->fmt;
   return g;
@@ -289,6 +294,9 @@ swan_status swan_init(swan_ctx** out, const swan_config* cfg, const float* R_qk,
     return fail(SWAN_ERR_UNSUPPORTED, "group size %d: only 1, 2 and 4 are built", G);
   if (C.k_store < 1 || C.k_store > C.head_dim)
     return fail(SWAN_ERR_INVALID_ARG, "k_store %d out of [1, %d]", C.k_store, C.head_dim);
+  const int k_store_v = C.k_store_v ? C.k_store_v : C.k_store;
+  if (k_store_v < 1 || k_store_v > C.head_dim)
+    return fail(SWAN_ERR_INVALID_ARG, "k_store_v %d out of [1, %d]", C.k_store_v, C.head_dim);
   if (C.buffer_cap < 0 || C.buffer_cap > kMaxBufferCap)
     return fail(SWAN_ERR_INVALID_ARG, "buffer_cap %d out of [0, %d]", C.buffer_cap, kMaxBufferCap);
   if (C.max_seq < 1) return fail(SWAN_ERR_INVALID_ARG, "max_seq must be >= 1");
@@ -311,10 +319,13 @@ swan_status swan_init(swan_ctx** out, const swan_config* cfg, const float* R_qk,
   c->G = G;
   c->k_slots = (C.k_store + 7) / 8 * 8;
   c->k_active = C.k_store;
+  c->k_store_v = k_store_v;
+  c->k_slots_v = (k_store_v + 7) / 8 * 8;
+  c->k_active_v = k_store_v;
   c->P = P;
   c->ppu = (int)((C.max_seq + P - 1) / P);
   c->fmt = C.value_format == SWAN_VALUES_FP8_E4M3 ? kFmtFp8 : kFmtFp16;
-  c->page_bytes = (int64_t)P * c->k_slots * (c->fmt == kFmtFp8 ? 4 : 6);
+  c->page_bytes = page_bytes_for(P, c->k_slots, c->k_slots_v, c->fmt);
   c->units = (int64_t)C.batch * C.n_kv_heads;
   c->num_pages = (int64_t)C.num_layers * c->units * c->ppu;
   c->stream = static_cast<cudaStream_t>(C.stream);
@@ -322,7 +333,7 @@ swan_status swan_init(swan_ctx** out, const swan_config* cfg, const float* R_qk,
   c->num_sms = sms;
   c->layers.assign(C.num_layers, LayerState{});
 
-  const int per_sm = decode_ctas_per_sm(G, c->k_slots);
+  const int per_sm = decode_ctas_per_sm(G, std::max(c->k_slots, c->k_slots_v));
   if (per_sm < 1) {
     delete c;
     return fail(SWAN_ERR_CUDA, "decode kernel does not fit on an SM (%s)",
@@ -397,12 +408,25 @@ swan_status swan_destroy(swan_ctx* c) {
   return SWAN_OK;
 }
 
+swan_status swan_set_kv(swan_ctx* c, int k_active, int k_active_v) {
+  swan_status s = usable(c);
+  if (s != SWAN_OK) return s;
+  if (k_active < 1 || k_active > c->cfg.k_store)
+    return fail(SWAN_ERR_INVALID_ARG, "k_active %d out of [1, %d]", k_active, c->cfg.k_store);
+  if (k_active_v < 1 || k_active_v > c->k_store_v)
+    return fail(SWAN_ERR_INVALID_ARG, "k_active_v %d out of [1, %d]", k_active_v, c->k_store_v);
+  c->k_active = k_active;
+  c->k_active_v = k_active_v;
+  return SWAN_OK;
+}
+
 swan_status swan_set_k(swan_ctx* c, int k_active) {
   swan_status s = usable(c);
   if (s != SWAN_OK) return s;
   if (k_active < 1 || k_active > c->cfg.k_store)
     return fail(SWAN_ERR_INVALID_ARG, "k_active %d out of [1, %d]", k_active, c->cfg.k_store);
   c->k_active = k_active;
+  c->k_active_v = std::min(k_active, c->k_store_v);
   return SWAN_OK;
 }
 
@@ -537,6 +561,8 @@ swan_status swan_decode(swan_ctx* c, int layer, const void* q, void* out) {
     p.blocks_per_page_log2 = __builtin_ctz((unsigned)(c->P / 32));
     p.k_full_chunks = c->k_active / 8;
     p.k_rem = c->k_active % 8;
+    p.k_full_chunks_v = c->k_active_v / 8;
+    p.k_rem_v = c->k_active_v % 8;
     p.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)kHeadDim));
     p.partials = c->partials;
     p.counters = c->counters;
@@ -545,7 +571,10 @@ swan_status swan_decode(swan_ctx* c, int layer, const void* q, void* out) {
     p.status = c->status;
     // the split combine and the rotate-back run inside the decode kernel
     return launch(c, SWAN_KERNEL_DECODE, "decode kernel",
-                  [&] { return launch_decode(p, G, (c->k_active + 7) / 8 * 8, (int)grid, c->stream); });
+                  [&] {
+                    const int k_read = (std::max(c->k_active, c->k_active_v) + 7) / 8 * 8;
+                    return launch_decode(p, G, k_read, (int)grid, c->stream);
+                  });
   }
   // empty cache: the combine kernel writes zeros
 
@@ -573,6 +602,9 @@ swan_status swan_query(const swan_ctx* c, int layer, swan_layer_info* info) {
   info->k_active = c->k_active;
   info->k_store = c->cfg.k_store;
   info->k_slots = c->k_slots;
+  info->k_active_v = c->k_active_v;
+  info->k_store_v = c->k_store_v;
+  info->k_slots_v = c->k_slots_v;
   info->page_tokens = c->P;
   info->page_bytes = c->page_bytes;
   info->device_bytes = c->device_bytes;
@@ -609,7 +641,8 @@ swan_status swan_debug_export(swan_ctx* c, int layer, int what, void* host_dst, 
     return SWAN_OK;
   }
   if (what == SWAN_EXPORT_SPARSE_K || what == SWAN_EXPORT_SPARSE_V) {
-    const int ks = c->cfg.k_store;
+    const bool isv_ = what == SWAN_EXPORT_SPARSE_V;
+    const int ks = isv_ ? c->k_store_v : c->cfg.k_store;
     const size_t n_ent = (size_t)c->units * L.sparse_len * ks;
     const size_t need = n_ent * 3;
     if (bytes != need) return fail(SWAN_ERR_INVALID_ARG, "bytes %zu != %zu", bytes, need);
@@ -617,12 +650,12 @@ swan_status swan_debug_export(swan_ctx* c, int layer, int what, void* host_dst, 
     const bool isv = what == SWAN_EXPORT_SPARSE_V;
     const bool fp8 = c->fmt == kFmtFp8;
     const int64_t P = c->P;
-    const int64_t ks8 = c->k_slots;
-    const int64_t blk = (fp8 ? 128 : 192) * ks8;
+    const int64_t ksk = c->k_slots, ksv = c->k_slots_v;
+    const int64_t blk = (fp8 ? 64 : 96) * (ksk + ksv);
     // fp16: value records of 16 B and index records of 8 B in separate
     // regions; fp8: 16-byte records of 8 values then 8 indices
-    const int64_t voff = fp8 ? (isv ? 64 * ks8 : 0) : (isv ? 96 * ks8 : 0);
-    const int64_t ioff = fp8 ? voff + 8 : (isv ? 160 * ks8 : 64 * ks8);
+    const int64_t voff = fp8 ? (isv ? 64 * ksk : 0) : (isv ? 96 * ksk : 0);
+    const int64_t ioff = fp8 ? voff + 8 : (isv ? 96 * ksk + 64 * ksv : 64 * ksk);
     std::vector<int32_t> pt((size_t)c->units * c->ppu);
     e = cudaMemcpy(pt.data(), c->page_table + (int64_t)layer * c->units * c->ppu, pt.size() * 4,
                    cudaMemcpyDeviceToHost);

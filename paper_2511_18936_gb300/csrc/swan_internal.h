@@ -4,25 +4,25 @@
 // for 128-bit coalesced loads on sm_103a).  A page holds P tokens (P a power
 // of two >= 32) of one (layer, batch, kv-head) unit, as P/32 consecutive
 // blocks of 32 tokens.  Each vector's kept entries are grouped in chunks of
-// 8, in stored (decreasing magnitude) order.  With fp16 values a block
-// (192 * k_slots bytes) is
+// 8, in stored (decreasing magnitude) order; keys keep ks_k entries (k_slots
+// = ks_k rounded up to 8) and values ks_v (the two may differ).  With fp16
+// values a block (96 * (ks_k + ks_v) bytes) is
 //
-//   [K values  : k_slots/8 chunks][32 tokens][8 x fp16]   at 0
-//   [K indices : k_slots/8 chunks][32 tokens][8 x uint8]  at 64 * k_slots
-//   [V values  : same shape as K values]                  at 96 * k_slots
-//   [V indices : same shape as K indices]                 at 160 * k_slots
+//   [K values  : ks_k/8 chunks][32 tokens][8 x fp16]    at 0
+//   [K indices : ks_k/8 chunks][32 tokens][8 x uint8]   at 64 * ks_k
+//   [V values  : ks_v/8 chunks][32 tokens][8 x fp16]    at 96 * ks_k
+//   [V indices : ks_v/8 chunks][32 tokens][8 x uint8]   at 96 * ks_k + 64 * ks_v
 //
 // and with 8-bit (E4M3) values (Section 4.3, Section 5.1) a block
-// (128 * k_slots bytes) is
+// (64 * (ks_k + ks_v) bytes) is
 //
-//   [K records : k_slots/8 chunks][32 tokens][8 x e4m3, 8 x uint8]  at 0
-//   [V records : same shape]                                         at 64 * k_slots
+//   [K records : ks_k/8 chunks][32 tokens][8 x e4m3, 8 x uint8]  at 0
+//   [V records : ks_v/8 chunks][32 tokens][8 x e4m3, 8 x uint8]  at 64 * ks_k
 //
 // A warp that handles the 32 tokens of a block (one per lane) reads chunk c
 // of all of them as one contiguous 512-byte run (values or records), at
-// compile-time offsets from the region base.  A runtime keep count
-// k_active <= k_store reads only the first ceil(k_active / 8) chunks: a
-// contiguous prefix of each region.
+// compile-time offsets from the region base.  A runtime keep count reads only
+// the first ceil(k_active / 8) chunks: a contiguous prefix of each region.
 #pragma once
 
 #include <cuda_fp16.h>
@@ -52,16 +52,24 @@ struct CacheGeom {
   int pages_per_unit;
   int64_t num_pages;         // pages in the pool (bounds check)
   int P;                     // tokens per page
-  int k_slots;               // k_store rounded up to 8
-  int k_store;
+  int k_slots;               // key entries stored per vector, rounded up to 8
+  int k_store;               // key entries kept per vector
+  int k_slots_v;             // the same for values
+  int k_store_v;
   int64_t page_bytes;        // P / 32 * block_bytes()
   int fmt;                   // kFmtFp16 or kFmtFp8
   // offsets inside a 32-token block (index regions: fp16 only)
-  __device__ __host__ int block_bytes() const { return (fmt == kFmtFp8 ? 128 : 192) * k_slots; }
+  __device__ __host__ int block_bytes() const {
+    return (fmt == kFmtFp8 ? 64 : 96) * (k_slots + k_slots_v);
+  }
   __device__ __host__ int kidx_off() const { return 64 * k_slots; }
   __device__ __host__ int vval_off() const { return (fmt == kFmtFp8 ? 64 : 96) * k_slots; }
-  __device__ __host__ int vidx_off() const { return 160 * k_slots; }
+  __device__ __host__ int vidx_off() const { return 96 * k_slots + 64 * k_slots_v; }
 };
+
+inline int64_t page_bytes_for(int P, int k_slots, int k_slots_v, int fmt) {
+  return (int64_t)(P / 32) * (fmt == kFmtFp8 ? 64 : 96) * (k_slots + k_slots_v);
+}
 
 // Rotate T new tokens per unit, then either write them to the ring buffer or
 // prune them straight into the sparse cache (Algorithm 1, generalised to T).
@@ -115,8 +123,10 @@ struct DecodeParams {
   int64_t total_groups, range;
   int H_kv, H_q;
   int blocks_per_page_log2; // log2(P / 32)
-  int k_full_chunks;       // k_active / 8
-  int k_rem;               // k_active % 8
+  int k_full_chunks;       // keys: k_active / 8
+  int k_rem;               // keys: k_active % 8
+  int k_full_chunks_v;     // values: k_active_v / 8
+  int k_rem_v;             // values: k_active_v % 8
   float scale_log2;        // log2(e) / sqrt(d)
   float* partials;         // [pairs][G][d + 2]
   int* counters;           // [units] arrival counters, zero between decodes

@@ -28,7 +28,7 @@ KERNEL_NAMES = {KERNEL_ROTATE_Q: "rotate_q", KERNEL_DECODE: "decode", KERNEL_COM
 EXPORTED = ["swan_init", "swan_destroy", "swan_set_k", "swan_append", "swan_flush_buffer",
             "swan_decode", "swan_query", "swan_debug_export", "swan_check",
             "swan_timing_enable", "swan_timing_read", "swan_launch_count",
-            "swan_status_string", "swan_last_error", "swan_decode_noalloc"]
+            "swan_status_string", "swan_last_error", "swan_decode_noalloc", "swan_set_kv"]
 
 
 class SwanConfig(ctypes.Structure):
@@ -37,14 +37,15 @@ class SwanConfig(ctypes.Structure):
                 ("head_dim", ctypes.c_int), ("k_store", ctypes.c_int),
                 ("buffer_cap", ctypes.c_int), ("max_seq", ctypes.c_int),
                 ("page_tokens", ctypes.c_int), ("stream", ctypes.c_void_p),
-                ("value_format", ctypes.c_int)]
+                ("value_format", ctypes.c_int), ("k_store_v", ctypes.c_int)]
 
 
 class LayerInfo(ctypes.Structure):
     _fields_ = [("sparse_len", ctypes.c_int64), ("buffer_len", ctypes.c_int64),
                 ("k_active", ctypes.c_int), ("k_store", ctypes.c_int), ("k_slots", ctypes.c_int),
                 ("page_tokens", ctypes.c_int), ("page_bytes", ctypes.c_int64),
-                ("device_bytes", ctypes.c_int64), ("value_format", ctypes.c_int)]
+                ("device_bytes", ctypes.c_int64), ("value_format", ctypes.c_int),
+                ("k_active_v", ctypes.c_int), ("k_store_v", ctypes.c_int), ("k_slots_v", ctypes.c_int)]
 
 
 class Timing(ctypes.Structure):
@@ -60,7 +61,7 @@ class CacheView(ctypes.Structure):
                 ("buf_start", ctypes.c_int), ("buf_len", ctypes.c_int), ("sparse_len", ctypes.c_int64),
                 ("batch", ctypes.c_int), ("n_q_heads", ctypes.c_int), ("n_kv_heads", ctypes.c_int),
                 ("head_dim", ctypes.c_int), ("R_qk", ctypes.c_void_p), ("R_vo_t", ctypes.c_void_p),
-                ("value_format", ctypes.c_int)]
+                ("value_format", ctypes.c_int), ("k_slots_v", ctypes.c_int), ("k_active_v", ctypes.c_int)]
 
 
 class SwanError(RuntimeError):
@@ -86,6 +87,7 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "swan_init": (i, [ctypes.POINTER(vp), ctypes.POINTER(SwanConfig), vp, vp]),
         "swan_destroy": (i, [vp]),
         "swan_set_k": (i, [vp, i]),
+        "swan_set_kv": (i, [vp, i, i]),
         "swan_append": (i, [vp, i, vp, vp, i]),
         "swan_flush_buffer": (i, [vp, i]),
         "swan_decode": (i, [vp, i, vp, vp]),
@@ -135,7 +137,7 @@ class Context:
     def __init__(self, R_qk, R_vo=None, *, num_layers: int, batch: int, n_q_heads: int,
                  n_kv_heads: int, k_store: int, buffer_cap: int, max_seq: int,
                  page_tokens: int = 0, head_dim: int = 128, stream=None,
-                 value_format: str = "fp16"):
+                 value_format: str = "fp16", k_store_v: int = 0):
         import torch
         self._lib = load_library()
         if stream is None:
@@ -145,9 +147,10 @@ class Context:
             raise ValueError(f"value_format must be one of {sorted(VALUE_FORMATS)}")
         self.cfg = SwanConfig(num_layers, batch, n_q_heads, n_kv_heads, head_dim, k_store,
                               buffer_cap, max_seq, page_tokens, ctypes.c_void_p(stream.cuda_stream),
-                              VALUE_FORMATS[value_format])
+                              VALUE_FORMATS[value_format], k_store_v)
         self.batch, self.n_q_heads, self.n_kv_heads = batch, n_q_heads, n_kv_heads
         self.num_layers, self.k_store, self.head_dim = num_layers, k_store, head_dim
+        self.k_store_v = k_store_v or k_store
         h = ctypes.c_void_p()
         _check(self._lib.swan_init(ctypes.byref(h), ctypes.byref(self.cfg), _ptr(R_qk),
                                    None if R_vo is None else _ptr(R_vo)), "swan_init")
@@ -172,8 +175,11 @@ class Context:
         self.close()
 
     # -- the hot path ------------------------------------------------------
-    def set_k(self, k_active: int):
-        _check(self._lib.swan_set_k(self._h, int(k_active)), "swan_set_k")
+    def set_k(self, k_active: int, k_active_v: int | None = None):
+        if k_active_v is None:
+            _check(self._lib.swan_set_k(self._h, int(k_active)), "swan_set_k")
+        else:
+            _check(self._lib.swan_set_kv(self._h, int(k_active), int(k_active_v)), "swan_set_kv")
 
     def append(self, layer: int, k_new, v_new, T: int | None = None):
         if T is None:
@@ -212,7 +218,8 @@ class Context:
 
     def export_sparse(self, layer: int, which: str):
         info = self.query(layer)
-        shape = (self.batch, self.n_kv_heads, info.sparse_len, self.k_store)
+        shape = (self.batch, self.n_kv_heads, info.sparse_len,
+                 self.k_store if which == "k" else self.k_store_v)
         n = int(np.prod(shape))
         raw = np.empty(n * 3, np.uint8)
         what = EXPORT_SPARSE_K if which == "k" else EXPORT_SPARSE_V

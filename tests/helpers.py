@@ -10,11 +10,11 @@ TOL_OUT = 2e-3  # max-abs tolerance on attention outputs (fp16 storage, fp32 acc
 
 
 def run_ops(ops, R, Rv, *, B, H_kv, G, k_store, cap, max_seq=None, page_tokens=0,
-            check_each=True, value_format="fp16"):
+            check_each=True, value_format="fp16", k_store_v=None):
     """Replay ``ops`` on the oracle and on a libswan context.
 
-    ops: ("append", k, v) | ("flush",) | ("set_k", k) | ("decode", q); all
-    arrays fp16 NumPy.  Returns (ctx, ref, [(gpu_out, ref_out), ...]).
+    ops: ("append", k, v) | ("flush",) | ("set_k", k) | ("set_kv", k, k_v) |
+    ("decode", q); all arrays fp16 NumPy.  Returns (ctx, ref, [(gpu_out, ref_out), ...]).
     """
     import torch
 
@@ -24,12 +24,12 @@ def run_ops(ops, R, Rv, *, B, H_kv, G, k_store, cap, max_seq=None, page_tokens=0
     if max_seq is None:
         max_seq = sum(op[1].shape[2] for op in ops if op[0] == "append") or 1
     ref = oracle.SwanOracle(R, Rv, batch=B, n_q_heads=H_kv * G, k_store=k_store, buffer_cap=cap,
-                            value_format=value_format)
+                            value_format=value_format, k_store_v=k_store_v)
     Rt = torch.from_numpy(np.asarray(R, np.float32))[None].to(dev).contiguous()
     Rvt = None if Rv is None else torch.from_numpy(np.asarray(Rv, np.float32))[None].to(dev).contiguous()
     ctx = swan.Context(Rt, Rvt, num_layers=1, batch=B, n_q_heads=H_kv * G, n_kv_heads=H_kv,
                        k_store=k_store, buffer_cap=cap, max_seq=max_seq, page_tokens=page_tokens,
-                       value_format=value_format)
+                       value_format=value_format, k_store_v=k_store_v or 0)
     outs = []
     for op in ops:
         if op[0] == "append":
@@ -41,6 +41,9 @@ def run_ops(ops, R, Rv, *, B, H_kv, G, k_store, cap, max_seq=None, page_tokens=0
         elif op[0] == "set_k":
             ref.set_k(op[1])
             ctx.set_k(op[1])
+        elif op[0] == "set_kv":
+            ref.set_k(op[1], op[2])
+            ctx.set_k(op[1], op[2])
         elif op[0] == "decode":
             want = ref.decode(op[1])
             got = ctx.decode(0, torch.from_numpy(op[1]).to(dev))

@@ -410,3 +410,100 @@ def test_fp8_decode_matches_oracle(B, H, G, L, cap, ks, kas, P):
         err = np.abs(got - want).max()
         assert err <= TOL_OUT, err
     ctx.close()
+
+
+# ---------------------------------------------------------------------------
+# Separate keep counts for keys and values (Appendix, ablation on key and
+# value pruning ratios)
+# ---------------------------------------------------------------------------
+
+@pytest.mark.parametrize("fmt", ["fp16", "fp8_e4m3"])
+@pytest.mark.parametrize("k_store,k_store_v,cap,P", [(40, 24, 5, 64), (16, 96, 0, 32), (128, 8, 64, 128),
+                                                     (3, 61, 20, 32)])
+def test_asymmetric_prune_bitexact_on_identical_rotated_inputs(fmt, k_store, k_store_v, cap, P):
+    B, H = 2, 3
+    eye = np.broadcast_to(np.eye(D, dtype=np.float32), (H, D, D)).copy()
+    R = _rot(H, 141)
+    kraw, vraw = _kv(B, H, 301, seed=142)
+    k16 = oracle.to_fp16(np.einsum("bhti,hij->bhtj", kraw.astype(np.float64), R.astype(np.float64)))
+    v16 = oracle.to_fp16(np.einsum("bhti,hij->bhtj", vraw.astype(np.float64), R.astype(np.float64)))
+    k16[0, 0, :40] = _tricky_vectors(40, 143)
+    v16[1, 2, :40] = _tricky_vectors(40, 144)
+    ops = [("append", k16[:, :, :37].copy(), v16[:, :, :37].copy()),
+           ("append", k16[:, :, 37:38].copy(), v16[:, :, 37:38].copy()),
+           ("append", k16[:, :, 38:].copy(), v16[:, :, 38:].copy()), ("flush",)]
+    ctx, ref, _ = run_ops(ops, eye, None, B=B, H_kv=H, G=1, k_store=k_store, cap=cap, page_tokens=P,
+                          value_format=fmt, k_store_v=k_store_v)
+    info = ctx.query(0)
+    assert (info.k_store, info.k_store_v, info.k_active, info.k_active_v) == (k_store, k_store_v,
+                                                                              k_store, k_store_v)
+    for which, ri, rv in (("k", ref.sp_idx_k, ref.sp_val_k), ("v", ref.sp_idx_v, ref.sp_val_v)):
+        gi, gv = ctx.export_sparse(0, which)
+        assert gi.shape[-1] == (k_store if which == "k" else k_store_v)
+        assert np.array_equal(gi, ri), which
+        assert np.array_equal(gv.view(np.uint16), rv.view(np.uint16)), which
+    ctx.close()
+
+
+ASYM_DECODE_CASES = [
+    # B, H_kv, G, L_total, cap, k_store, k_store_v, [(k_active, k_active_v)], page_tokens, fmt
+    (2, 2, 1, 1000, 64, 64, 32, [(64, 32), (32, 32), (17, 9)], 128, "fp16"),
+    (2, 2, 1, 1000, 64, 32, 96, [(32, 96), (8, 64), (32, 1)], 64, "fp16"),
+    (2, 4, 2, 777, 16, 60, 20, [(60, 20), (7, 13)], 32, "fp16"),
+    (2, 2, 4, 1500, 128, 24, 72, [(24, 72), (24, 40)], 64, "fp16"),
+    (2, 2, 1, 1000, 64, 64, 32, [(64, 32), (40, 5)], 128, "fp8_e4m3"),
+    (2, 2, 4, 900, 32, 96, 16, [(96, 16), (65, 16)], 32, "fp8_e4m3"),
+]
+
+
+@pytest.mark.parametrize("B,H,G,L,cap,ks,ksv,kas,P,fmt", ASYM_DECODE_CASES)
+def test_asymmetric_decode_matches_oracle(B, H, G, L, cap, ks, ksv, kas, P, fmt):
+    R, Rv = _rot(H, 150 + L), _rot(H, 150 + L, synth.T_R_VO)
+    k, v = _kv(B, H, L, seed=L + 11)
+    q = _q(B, H * G, seed=L + 12)
+    qp = _q(B, H * G, seed=L + 13, scale=4.0)
+    cut = max(1, L // 3)
+    ops = [("append", k[:, :, :cut].copy(), v[:, :, :cut].copy()), ("decode", q),
+           ("append", k[:, :, cut:].copy(), v[:, :, cut:].copy())]
+    for ka, kav in kas:
+        ops += [("set_kv", ka, kav), ("decode", q), ("decode", qp)]
+    ops += [("set_k", ks), ("decode", q)]   # set_k clamps the value count at k_store_v
+    ctx, ref, outs = run_ops(ops, R, Rv, B=B, H_kv=H, G=G, k_store=ks, cap=cap, page_tokens=P,
+                             value_format=fmt, k_store_v=ksv)
+    assert ctx.query(0).k_active_v == min(ks, ksv)
+    for got, want in outs:
+        err = np.abs(got - want).max()
+        assert err <= TOL_OUT, err
+    ctx.close()
+
+
+def test_runtime_value_prefix_equals_stored_split():
+    """A symmetric k_store = 128 cache decoded at (k, k_v) gives the result of
+    a cache stored with k_store = k, k_store_v = k_v: both keep the same
+    leading entries of each vector."""
+    import torch
+
+    from paper_2511_18936_gb300 import swan
+    dev = torch.device("cuda")
+    B, H, G, L, cap = 2, 2, 2, 900, 64
+    R = _rot(H, 160)
+    k, v = _kv(B, H, L, seed=161)
+    q = torch.from_numpy(_q(B, H * G, seed=162, scale=2.0)).to(dev)
+    Rt = torch.from_numpy(R)[None].to(dev)
+    kt, vt = torch.from_numpy(k).to(dev), torch.from_numpy(v).to(dev)
+    full = swan.Context(Rt, num_layers=1, batch=B, n_q_heads=H * G, n_kv_heads=H, k_store=128,
+                        buffer_cap=cap, max_seq=L)
+    full.append(0, kt, vt)
+    for ka, kav in ((48, 16), (16, 48), (64, 64)):
+        split = swan.Context(Rt, num_layers=1, batch=B, n_q_heads=H * G, n_kv_heads=H, k_store=ka,
+                             k_store_v=kav, buffer_cap=cap, max_seq=L)
+        split.append(0, kt, vt)
+        full.set_k(ka, kav)
+        a = full.decode(0, q).float()
+        b = split.decode(0, q).float()
+        torch.cuda.synchronize()
+        assert (a - b).abs().max().item() <= 1e-3, (ka, kav)
+        split.check()
+        split.close()
+    full.check()
+    full.close()

@@ -44,7 +44,7 @@ def test_status_strings(lib):
 
 def _cfg(**kw):
     base = dict(num_layers=1, batch=1, n_q_heads=1, n_kv_heads=1, head_dim=128, k_store=64,
-                buffer_cap=64, max_seq=1024, page_tokens=0, stream=None, value_format=0)
+                buffer_cap=64, max_seq=1024, page_tokens=0, stream=None, value_format=0, k_store_v=0)
     base.update(kw)
     return swan.SwanConfig(*[base[f] for f, _ in swan.SwanConfig._fields_])
 
@@ -66,6 +66,8 @@ def _cfg(**kw):
     (dict(batch=0), swan.ERR_INVALID_ARG),
     (dict(value_format=2), swan.ERR_INVALID_ARG),
     (dict(value_format=-1), swan.ERR_INVALID_ARG),
+    (dict(k_store_v=129), swan.ERR_INVALID_ARG),
+    (dict(k_store_v=-2), swan.ERR_INVALID_ARG),
 ])
 def test_init_rejects_bad_config_without_cuda(lib, kw, status):
     h = ctypes.c_void_p(123)
@@ -82,6 +84,7 @@ def test_null_arguments(lib):
     cfg = _cfg()
     assert lib.swan_init(ctypes.byref(h), ctypes.byref(cfg), None, None) == swan.ERR_INVALID_ARG
     assert lib.swan_set_k(None, 4) == swan.ERR_INVALID_ARG
+    assert lib.swan_set_kv(None, 4, 4) == swan.ERR_INVALID_ARG
     assert lib.swan_append(None, 0, None, None, 1) == swan.ERR_INVALID_ARG
     assert lib.swan_decode(None, 0, None, None) == swan.ERR_INVALID_ARG
     assert lib.swan_flush_buffer(None, 0) == swan.ERR_INVALID_ARG

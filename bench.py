@@ -68,13 +68,13 @@ def measured_peaks():
         return None
 
 
-def decode_kernel_traffic(workload: str, values: str = "fp16"):
+def decode_kernel_traffic(workload: str, values: str = "fp16", variant: str = ""):
     """DRAM bytes per decode-kernel launch from the committed ncu summary, if
     it was taken on the current kernel source (else None)."""
     src = os.path.join(ROOT, "paper_2511_18936_gb300", "csrc", "decode.cu")
     digest = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
     text = None
-    suffix = "" if values == "fp16" else "-fp8"
+    suffix = ("" if values == "fp16" else "-fp8") + variant
     for name in (f"decode_kernel_{workload}{suffix}.md", f"decode_gqa_kernel_{workload}{suffix}.md"):
         try:
             text = open(os.path.join(ROOT, "profiles", name)).read()
@@ -158,11 +158,12 @@ def oracle_sample(wl, n_units: int, seed: int = 0):
         R = synth.rotations(1, D, seed=seed, workload=7, layer=0, tensor_id=synth.T_R_QK, )
         k = synth.lowrank_kv(1, 1, L + 64, D, seed, 7, u, synth.T_K)
         v = synth.lowrank_kv(1, 1, L + 64, D, seed, 7, u, synth.T_V)
-        st = oracle.SwanOracle(R, batch=1, n_q_heads=G, k_store=wl["k_store"], buffer_cap=wl["n_b"])
+        st = oracle.SwanOracle(R, batch=1, n_q_heads=G, k_store=wl["k_store"], buffer_cap=wl["n_b"],
+                               value_format=wl["values"], k_store_v=wl["k_store_v"])
         st.append(k[:, :, :L_s], v[:, :, :L_s])
         st.flush()
         st.append(k[:, :, L_s:L], v[:, :, L_s:L])
-        st.set_k(wl["k"])
+        st.set_k(wl["k"], wl["k_v"])
         q = synth.gaussian_fp16((1, G, D), seed, 7, u, synth.T_Q)
         states.append((st, k[:, :, L:], v[:, :, L:], q))
     step_no = [0]
@@ -182,7 +183,7 @@ def oracle_sample(wl, n_units: int, seed: int = 0):
 def run_reference(args, wl, rank: int):
     if rank != 0:
         return None
-    n_units = 2
+    n_units = min(2, wl["B"] * wl["H_kv"])
     t0 = time.perf_counter()
     step = oracle_sample(wl, n_units)
     prep = time.perf_counter() - t0
@@ -261,7 +262,7 @@ class LayerRun:
             R = torch.from_numpy(synth.rotations(H_kv, D, seed=seed, workload=1, layer=0))[None].to(dev)
             self.ctx = swan.Context(R, num_layers=1, batch=B, n_q_heads=H_q, n_kv_heads=H_kv,
                                     k_store=wl["k_store"], buffer_cap=n_b, max_seq=self.max_seq,
-                                    stream=stream, value_format=wl["values"])
+                                    stream=stream, value_format=wl["values"], k_store_v=wl["k_store_v"])
             kk = synth.torch_lowrank_kv(B, H_kv, L_s + n_b, D, seed, synth.T_K, dev)
             vv = synth.torch_lowrank_kv(B, H_kv, L_s + n_b, D, seed, synth.T_V, dev)
             self.ctx.append(0, kk, vv)
@@ -273,7 +274,7 @@ class LayerRun:
             del k_new, v_new
             self.qs = synth.torch_gaussian_fp16((steps_total, B, H_q, D), seed, synth.T_Q, dev)
             self.out = torch.empty((B, H_q, D), dtype=torch.float16, device=dev)
-            self.ctx.set_k(wl["k"])
+            self.ctx.set_k(wl["k"], wl["k_v"])
         stream.synchronize()
         self.ctx.check()
 
@@ -316,8 +317,8 @@ class StackRun:
             Rt = torch.from_numpy(R).to(dev)
             self.ctx = swan.Context(Rt, num_layers=Lyr, batch=B, n_q_heads=H, n_kv_heads=H,
                                     k_store=wl["k_store"], buffer_cap=cap, max_seq=self.max_seq,
-                                    stream=stream, value_format=wl["values"])
-            self.ctx.set_k(wl["k"])
+                                    stream=stream, value_format=wl["values"], k_store_v=wl["k_store_v"])
+            self.ctx.set_k(wl["k"], wl["k_v"])
         stream.synchronize()
         # prefix: one append per layer (plain Gaussian K/V), timed on the stream
         ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -481,17 +482,17 @@ def run_swan(args, wl, rank: int, world: int, local_rank: int):
     sp_mean = statistics.mean(sp for sp, _ in kctxs)
     bf_mean = statistics.mean(bf for _, bf in kctxs)
     # algorithmic bytes of one decode-kernel launch (one layer): per (sparse
-    # token, kv head) 2 * (value + index bytes) * k (K and V: 6k with fp16
-    # values, 4k with 8-bit values); per (buffer token, kv head) 2 * 2 * d
-    ent = 4 if wl["values"] == "fp8_e4m3" else 6
-    alg_decode = B * H_kv * (sp_mean * ent * k + bf_mean * 4 * D)
+    # token, kv head) (value + index bytes) * (k + k_v) (6k with fp16 values
+    # and k_v = k, 4k with 8-bit values); per (buffer token, kv head) 2 * 2 * d
+    sp_bytes = (2 if wl["values"] == "fp8_e4m3" else 3) * (k + wl["k_v"])
+    alg_decode = B * H_kv * (sp_mean * sp_bytes + bf_mean * 4 * D)
     achieved = alg_decode / avg_dec_s / 1e9
     peaks = measured_peaks()
     peak = float(peaks["hbm_gbs"]) if peaks else 6800.0
     step_s = t_max / 1e3 / args.steps
     sp_step = statistics.mean(sp for sp, _ in ctxs)
     bf_step = statistics.mean(bf for _, bf in ctxs)
-    alg_decode_step = B * H_kv * (sp_step * ent * k + bf_step * 4 * D)
+    alg_decode_step = B * H_kv * (sp_step * sp_bytes + bf_step * 4 * D)
     # whole-step algorithmic bytes per layer: decode reads + q/out (fp16) + R
     # (fp32, once per kv head, query and value rotations) + the append's new
     # vectors (fp16 in, fp16 to the buffer)
@@ -502,6 +503,7 @@ def run_swan(args, wl, rank: int, world: int, local_rank: int):
     cfg = {"workload": args.workload, "desc": wl["desc"], "batch": B, "n_q_heads": H_q,
            "n_kv_heads": H_kv, "layers": run.layers, "sparse_tokens": wl.get("L_s", wl.get("prefix")),
            "buffer_tokens": wl["n_b"], "k": k, "k_store": wl["k_store"],
+           "k_v": wl["k_v"], "k_store_v": wl["k_store_v"],
            "storage": ("e4m3" if wl["values"] == "fp8_e4m3" else "fp16")
                       + " values + uint8 indices (sparse), fp16 (buffer)", "l2": l2_note,
            "parallelism": f"replicas x{world} (independent batches per GPU)" if world > 1
@@ -521,7 +523,9 @@ def run_swan(args, wl, rank: int, world: int, local_rank: int):
                      else "fallback 6.8 TB/s",
                      "pct_of_8tbs": 100.0 * achieved / NOMINAL_HBM_GBS,
                      "alg_bytes_per_launch": alg_decode, "avg_launch_ms": avg_dec_s * 1e3,
-                     "traffic": decode_kernel_traffic(args.workload, wl["values"])},
+                     "traffic": decode_kernel_traffic(
+                         args.workload, wl["values"],
+                         "" if wl["k_store_v"] == wl["k_store"] else f"-ksv{wl['k_store_v']}")},
         "kernels_ms_per_step": {name: v[0] / args.steps for name, v in kt.items() if v[1]},
         "kernels_timed": "second timed region of the same length, CUDA events around every launch",
         "gpu_launches": launches,
@@ -553,6 +557,10 @@ def main():
                     help="kept sparse values as fp16 (3k bytes per vector) or E4M3 (2k)")
     ap.add_argument("--k-active", type=int, default=0,
                     help="runtime keep count (ksweep-32k: 32, 48, 64, 96 or 128)")
+    ap.add_argument("--k-store-v", type=int, default=0,
+                    help="value entries stored per vector (default: as for keys)")
+    ap.add_argument("--k-active-v", type=int, default=0,
+                    help="runtime value keep count (default: min(k_active, k_store_v))")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
@@ -568,6 +576,17 @@ def main():
             ap.error(f"--k-active must be in [1, {wl['k_store']}]")
         wl["k"] = args.k_active
         wl["desc"] += f" (k_active {args.k_active})"
+    wl["k_store_v"] = args.k_store_v or wl["k_store"]
+    if not 1 <= wl["k_store_v"] <= D:
+        ap.error(f"--k-store-v must be in [1, {D}]")
+    if args.k_store_v:
+        wl["desc"] += f" (k_store_v {wl['k_store_v']})"
+    wl["k_v"] = min(wl["k"], wl["k_store_v"])
+    if args.k_active_v:
+        if not 1 <= args.k_active_v <= wl["k_store_v"]:
+            ap.error(f"--k-active-v must be in [1, {wl['k_store_v']}]")
+        wl["k_v"] = args.k_active_v
+        wl["desc"] += f" (k_active_v {args.k_active_v})"
 
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))

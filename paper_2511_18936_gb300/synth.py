@@ -17,6 +17,14 @@ Section 6; no weights or datasets are used here, these stand in for them):
   the triangular factor is positive, cast to fp32 (the paper's random
   orthogonal projection ablation, Appendix, "Random Projection").
 * Plain Gaussian K/V/q for the 32-layer stack workload.
+* Calibration sets for the offline basis (Section 4.1): per kv head ``j``
+  two random orthogonal bases ``W_qk[j]`` and ``W_vo[j]``; the G query heads
+  of the group and the key head draw ``Z diag(sigma) W_qk[j]^T`` (queries
+  with the flatter spectrum ``sigma_i ∝ i^-1/2``, keys with ``∝ 1/i``), the
+  value head ``Z diag(sigma) W_vo[j]^T``, and the output-projection slice of
+  each query head of the group is ``W_vo[j] diag(tau) Y`` (``tau_i ∝ i^-1/2``,
+  ``Y`` Gaussian ``d x d_model`` scaled by ``d_model^-1/2``), so that the
+  columns of every slice share the value basis of their kv head.
 
 Seeds: ``numpy.random.SeedSequence([seed, workload, layer, tensor_id])``.
 Large workloads are drawn on the GPU with a seeded ``torch.Generator`` (the
@@ -29,6 +37,8 @@ import numpy as np
 
 # tensor ids inside a SeedSequence
 T_R_QK, T_R_VO, T_K, T_V, T_Q, T_KBASIS, T_VBASIS, T_NEWK, T_NEWV = range(9)
+# calibration activations and weights for the offline basis
+T_CAL_Q, T_CAL_K, T_CAL_V, T_CAL_WO, T_QK_BASIS, T_VO_BASIS = range(9, 15)
 
 
 def seed_seq(seed: int, workload: int, layer: int, tensor_id: int, *extra: int):
@@ -135,3 +145,65 @@ def torch_gaussian_fp16(shape, seed: int, tensor_id: int, device, scale: float =
     gen.manual_seed(int(seed_seq(seed, 2000, 0, tensor_id, *extra).generate_state(1)[0]))
     x = torch.randn(shape, generator=gen, device=device, dtype=torch.float32) * scale
     return x.to(torch.float16)
+
+
+def spectrum(d: int, power: float) -> np.ndarray:
+    """sigma_i ∝ i^-power (i = 1..d), normalised so that sum sigma_i^2 = d."""
+    s = np.arange(1, d + 1, dtype=np.float64) ** -power
+    return s * np.sqrt(d / np.sum(s * s))
+
+
+def calibration(n_kv_heads: int, group: int, n_tokens: int, d: int, d_model: int, seed: int,
+                workload: int, layer: int):
+    """Host calibration set: fp16 ``Q [n_kv_heads*group][n_tokens][d]``,
+    ``K, V [n_kv_heads][n_tokens][d]``, ``W_O [n_kv_heads*group*d][d_model]``."""
+    H_q = n_kv_heads * group
+    Q = np.empty((H_q, n_tokens, d), np.float16)
+    K = np.empty((n_kv_heads, n_tokens, d), np.float16)
+    V = np.empty((n_kv_heads, n_tokens, d), np.float16)
+    W_O = np.empty((H_q * d, d_model), np.float16)
+    s_flat, s_steep = spectrum(d, 0.5), spectrum(d, 1.0)
+    for j in range(n_kv_heads):
+        w_qk = random_orthogonal(d, rng(seed, workload, layer, T_QK_BASIS, j))
+        w_vo = random_orthogonal(d, rng(seed, workload, layer, T_VO_BASIS, j))
+        for g in range(group):
+            h = j * group + g
+            z = rng(seed, workload, layer, T_CAL_Q, h).standard_normal((n_tokens, d))
+            Q[h] = ((z * s_flat) @ w_qk.T).astype(np.float16)
+            y = rng(seed, workload, layer, T_CAL_WO, h).standard_normal((d, d_model)) / np.sqrt(d_model)
+            W_O[h * d:(h + 1) * d] = ((w_vo * s_flat[None, :]) @ y).astype(np.float16)
+        z = rng(seed, workload, layer, T_CAL_K, j).standard_normal((n_tokens, d))
+        K[j] = ((z * s_steep) @ w_qk.T).astype(np.float16)
+        z = rng(seed, workload, layer, T_CAL_V, j).standard_normal((n_tokens, d))
+        V[j] = ((z * s_steep) @ w_vo.T).astype(np.float16)
+    return Q, K, V, W_O
+
+
+def torch_calibration(n_kv_heads: int, group: int, n_tokens: int, d: int, d_model: int, seed: int,
+                      device, chunk_tokens: int = 8192):
+    """Same recipe as :func:`calibration`, drawn on ``device`` (large sets)."""
+    import torch
+    H_q = n_kv_heads * group
+    gen = torch.Generator(device=device)
+    gen.manual_seed(int(seed_seq(seed, 3000, 0, T_CAL_Q).generate_state(1)[0]))
+    s_flat = torch.from_numpy(spectrum(d, 0.5).astype(np.float32)).to(device)
+    s_steep = torch.from_numpy(spectrum(d, 1.0).astype(np.float32)).to(device)
+    w_qk = torch.from_numpy(np.stack([random_orthogonal(d, rng(seed, 3000, 0, T_QK_BASIS, j))
+                                      for j in range(n_kv_heads)]).astype(np.float32)).to(device)
+    w_vo = torch.from_numpy(np.stack([random_orthogonal(d, rng(seed, 3000, 0, T_VO_BASIS, j))
+                                      for j in range(n_kv_heads)]).astype(np.float32)).to(device)
+    Q = torch.empty((H_q, n_tokens, d), dtype=torch.float16, device=device)
+    K = torch.empty((n_kv_heads, n_tokens, d), dtype=torch.float16, device=device)
+    V = torch.empty((n_kv_heads, n_tokens, d), dtype=torch.float16, device=device)
+    wq_t = w_qk.repeat_interleave(group, 0).transpose(1, 2).contiguous()
+    for t0 in range(0, n_tokens, chunk_tokens):
+        t1 = min(n_tokens, t0 + chunk_tokens)
+        z = torch.randn((H_q, t1 - t0, d), generator=gen, device=device)
+        Q[:, t0:t1] = torch.bmm(z * s_flat, wq_t).to(torch.float16)
+        z = torch.randn((n_kv_heads, t1 - t0, d), generator=gen, device=device)
+        K[:, t0:t1] = torch.bmm(z * s_steep, w_qk.transpose(1, 2)).to(torch.float16)
+        z = torch.randn((n_kv_heads, t1 - t0, d), generator=gen, device=device)
+        V[:, t0:t1] = torch.bmm(z * s_steep, w_vo.transpose(1, 2)).to(torch.float16)
+    y = torch.randn((H_q, d, d_model), generator=gen, device=device) / float(np.sqrt(d_model))
+    W_O = torch.bmm(w_vo.repeat_interleave(group, 0) * s_flat[None, None, :], y)
+    return Q, K, V, W_O.reshape(H_q * d, d_model).to(torch.float16)

@@ -305,3 +305,117 @@ ALL_PINS = [pin_rotation_orthogonal, pin_rotation_orientation, pin_prune_brutefo
             pin_k_equals_d_is_dense, pin_decompression_free, pin_buffer_semantics,
             pin_split_combine, pin_k_prefix, pin_gqa_mapping, pin_formulas, pin_e4m3_rounding,
             pin_fp8_cache_is_rounded_sparse_cache, pin_asymmetric_keep_counts]
+
+
+# -- Offline basis (Section 4.1); each takes the basis oracle module ---------
+
+def _orthonormal_columns(m, n, gen):
+    q, _ = np.linalg.qr(gen.standard_normal((m, n)))
+    return q
+
+
+def pin_basis_recovers_planted_svd(b):
+    """S = U diag(sigma) W^T with known factors: the basis is W (columns, in
+    order of decreasing sigma, up to the sign rule) and the singular values
+    are sigma."""
+    gen = np.random.default_rng(101)
+    d, m = 16, 60
+    W = synth.random_orthogonal(d, gen)
+    U = _orthonormal_columns(m, d, gen)
+    sigma = 2.0 ** -(np.arange(d) / 2.0)
+    P, s = b.principal_basis(U @ np.diag(sigma) @ W.T)
+    assert P.shape == (d, d)
+    assert np.allclose(s, sigma, atol=1e-12)
+    for j in range(d):
+        assert abs(abs(P[:, j] @ W[:, j]) - 1.0) < 1e-10, j
+        lead = int(np.argmax(np.abs(P[:, j])))
+        assert P[lead, j] > 0, j
+    assert np.allclose(P.T @ P, np.eye(d), atol=1e-12)
+
+
+def pin_basis_ky_fan_maximum(b):
+    """For every k the first k basis vectors keep the most energy of any
+    k-dimensional orthonormal set (Ky Fan): sum_{j<k} |S p_j|^2 equals the sum
+    of the k largest eigenvalues of S^T S and no random basis beats it."""
+    gen = np.random.default_rng(102)
+    S = gen.standard_normal((200, 12)) * np.linspace(3.0, 0.2, 12)[None, :] @ synth.random_orthogonal(12, gen)
+    P, _ = b.principal_basis(S)
+    lam = np.sort(np.linalg.eigvalsh(S.T @ S))[::-1]
+    kept = np.cumsum(np.sum((S @ P) ** 2, axis=0))
+    assert np.allclose(kept, np.cumsum(lam), rtol=1e-10)
+    for _ in range(20):
+        Qr = synth.random_orthogonal(12, gen)
+        other = np.cumsum(np.sum((S @ Qr) ** 2, axis=0))
+        assert (other <= kept * (1 + 1e-12)).all()
+
+
+def _planted_groups(gen, n_kv, G, n, d, d_model, r):
+    """Per kv head j four planted r-dimensional subspaces: the query heads
+    jG..jG+G-1 live in span(Bq[j]), key head j in span(Bk[j]), value head j
+    in span(Bv[j]) and the columns of the W_O slices of those query heads in
+    span(Bw[j])."""
+    Bq, Bk, Bv, Bw = ([_orthonormal_columns(d, r, gen) for _ in range(n_kv)] for _ in range(4))
+    Q = np.stack([gen.standard_normal((n, r)) @ Bq[h // G].T for h in range(n_kv * G)])
+    K = np.stack([gen.standard_normal((n, r)) @ Bk[j].T for j in range(n_kv)])
+    V = np.stack([gen.standard_normal((n, r)) @ Bv[j].T for j in range(n_kv)])
+    W_O = np.concatenate([Bw[h // G] @ gen.standard_normal((r, d_model)) for h in range(n_kv * G)])
+    return Bq, Bk, Bv, Bw, Q, K, V, W_O
+
+
+def pin_joint_matrices_group_heads(b):
+    """Section 4.1.1 grouping and Section 4.1.2 concatenation: with query
+    heads jG..jG+G-1, key head j, value head j and the W_O slices of those
+    query heads each in their own planted r-dimensional subspace, the first
+    2r basis vectors of S_QK[j] span exactly span(Bq[j], Bk[j]) and those of
+    S_VO[j] span(Bv[j], Bw[j]); a wrong grouping or a dropped part leaves a
+    different span."""
+    gen = np.random.default_rng(103)
+    n_kv, G, n, d, d_model, r = 3, 2, 40, 16, 24, 3
+    Bq, Bk, Bv, Bw, Q, K, V, W_O = _planted_groups(gen, n_kv, G, n, d, d_model, r)
+    sqk = b.joint_qk(Q, K, G)
+    svo = b.joint_vo(V, W_O, G)
+    assert len(sqk) == n_kv and len(svo) == n_kv
+    for j in range(n_kv):
+        assert sqk[j].shape == ((G + 1) * n, d)
+        assert svo[j].shape == (n + G * d_model, d)
+        for S, B in ((sqk[j], np.hstack([Bq[j], Bk[j]])), (svo[j], np.hstack([Bv[j], Bw[j]]))):
+            P, sigma = b.principal_basis(S)
+            B, _ = np.linalg.qr(B)
+            assert np.linalg.norm(B.T @ P[:, :2 * r]) ** 2 > 2 * r - 1e-9, j
+            assert sigma[2 * r] < 1e-9 * sigma[0]
+
+
+def pin_energy_curve_bruteforce(b):
+    """E[k] is the sum over vectors of the best k-subset of squared rotated
+    coordinates (brute force over all subsets, d = 8); E[0] = 0 and E[d] is
+    the total energy (P orthogonal)."""
+    gen = np.random.default_rng(104)
+    d = 8
+    X = gen.standard_normal((30, d)) * np.array([3, 1, 0.5, 2, 0.1, 1, 4, 0.3])
+    P = synth.random_orthogonal(d, gen)
+    E = b.energy_curve(X, P)
+    Y = X @ P
+    for k in range(d + 1):
+        best = 0.0
+        for y in Y:
+            best += max((sum(y[list(c)] ** 2) for c in itertools.combinations(range(d), k)), default=0.0)
+        assert abs(E[k] - best) < 1e-9 * max(1.0, best), k
+    assert E[0] == 0.0 and abs(E[d] - np.sum(X * X)) < 1e-9
+
+
+def pin_energy_planted_rank(b):
+    """Vectors in the span of the first r columns of an orthogonal W keep all
+    their energy at k = r with P = W, and with the principal basis of the
+    vectors themselves; a random basis keeps less."""
+    gen = np.random.default_rng(105)
+    d, r = 16, 4
+    W = synth.random_orthogonal(d, gen)
+    X = gen.standard_normal((50, r)) @ W[:, :r].T
+    for P in (W, b.principal_basis(X)[0]):
+        E = b.energy_curve(X, P)
+        assert abs(E[r] - E[d]) < 1e-9 * E[d]
+    assert b.energy_curve(X, synth.random_orthogonal(d, gen))[r] < 0.99 * np.sum(X * X)
+
+
+BASIS_PINS = [pin_basis_recovers_planted_svd, pin_basis_ky_fan_maximum, pin_joint_matrices_group_heads,
+              pin_energy_curve_bruteforce, pin_energy_planted_rank]

@@ -10,10 +10,11 @@ import types
 
 import pytest
 
-from tests.oracle_pins import ALL_PINS
+from tests.oracle_pins import ALL_PINS, BASIS_PINS
 
-SRC = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))),
-                   "oracle", "swan_oracle.py")
+ORACLE_DIR = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "oracle")
+SRC = os.path.join(ORACLE_DIR, "swan_oracle.py")
+BASIS_SRC = os.path.join(ORACLE_DIR, "basis_oracle.py")
 
 # (name, original text, mutated text, count of occurrences to replace)
 MUTANTS = [
@@ -74,14 +75,46 @@ MUTANTS = [
 ]
 
 
-def _load_mutant(name, old, new, count):
-    src = open(SRC).read()
+BASIS_MUTANTS = [
+    ("basis_rows_of_vt", "P = vt.T\n", "P = vt\n", 1),
+    ("basis_ascending", "P = vt.T\n", "P = vt.T[:, ::-1]\n", 1),
+    ("basis_no_sign_rule", "return fix_signs(P), sigma", "return P * np.sign(P[0])[None, :], sigma", 1),
+    ("qk_grouped_by_modulo",
+     "q_rows = Q[j * group:(j + 1) * group]", "q_rows = Q[j::n_kv]", 1),
+    ("vo_slice_rows_not_columns", "parts.append(W_O[h * d:(h + 1) * d, :].T)",
+     "parts.append(W_O[h * d:(h + 1) * d, :d].T)", 1),
+    ("vo_values_dropped", "parts = [V[j]]", "parts = [0 * V[j]]", 1),
+    ("energy_smallest_first", "sq = np.sort(Y * Y, axis=1)[:, ::-1]", "sq = np.sort(Y * Y, axis=1)", 1),
+    ("energy_unsquared", "sq = np.sort(Y * Y, axis=1)[:, ::-1]", "sq = np.sort(np.abs(Y), axis=1)[:, ::-1]", 1),
+    ("energy_unrotated", "Y = np.asarray(X, np.float64) @ np.asarray(P, np.float64)",
+     "Y = np.asarray(X, np.float64) + 0 * np.asarray(P)[0, 0]", 1),
+]
+
+
+def _load_mutant(name, old, new, count, src_path=SRC):
+    src = open(src_path).read()
     assert src.count(old) == count, (name, src.count(old))
     mod = types.ModuleType("oracle_mutant_" + name)
-    mod.__file__ = SRC
+    mod.__file__ = src_path
     sys.modules[mod.__name__] = mod
-    exec(compile(src.replace(old, new), SRC, "exec"), mod.__dict__)
+    exec(compile(src.replace(old, new), src_path, "exec"), mod.__dict__)
     return mod
+
+
+def _caught(mod, pins):
+    failed = []
+    for pin in pins:
+        try:
+            pin(mod)
+        except Exception as e:  # noqa: BLE001 - any failure counts as caught
+            failed.append((pin.__name__, type(e).__name__))
+    return failed
+
+
+@pytest.mark.parametrize("name,old,new,count", BASIS_MUTANTS, ids=[m[0] for m in BASIS_MUTANTS])
+def test_basis_mutant_is_caught(name, old, new, count):
+    mod = _load_mutant(name, old, new, count, BASIS_SRC)
+    assert _caught(mod, BASIS_PINS), f"mutant {name} passed every pin"
 
 
 @pytest.mark.parametrize("name,old,new,count", MUTANTS, ids=[m[0] for m in MUTANTS])

@@ -53,7 +53,7 @@ typedef enum swan_status {
   SWAN_ERR_CAPACITY = 3,       /* would exceed max_seq; nothing was changed */
   SWAN_ERR_CUDA = 4,           /* a CUDA runtime call failed */
   SWAN_ERR_STATE = 5,          /* context poisoned by an earlier CUDA error */
-  SWAN_ERR_DEVICE_TIMEOUT = 6, /* reserved: a bounded device wait ran out */
+  SWAN_ERR_DEVICE_TIMEOUT = 6, /* a bounded device wait ran out */
   SWAN_ERR_NOMEM = 7,          /* device or host allocation failed in init */
   SWAN_ERR_DEVICE_CHECK = 8    /* a device-side consistency check failed */
 } swan_status;

@@ -20,7 +20,7 @@ LIB = os.path.join(PKG, "libswan.so")
 INCLUDE = os.path.join(ROOT, "include")
 
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
-SOURCES = ["swan_api.cpp", "decode.cu", "append.cu", "noalloc.cu"]
+SOURCES = ["swan_api.cpp", "decode.cu", "append.cu", "noalloc.cu", "basis.cu", "basis_api.cpp"]
 
 
 def _nvcc() -> str:

@@ -24,11 +24,13 @@ KERNEL_KINDS = 8
 KERNEL_NAMES = {KERNEL_ROTATE_Q: "rotate_q", KERNEL_DECODE: "decode", KERNEL_COMBINE: "combine",
                 KERNEL_APPEND: "append", KERNEL_PRUNE: "prune_ring"}
 
-# Every symbol include/swan.h declares.
+# Every symbol include/swan.h and include/swan_basis.h declare.
 EXPORTED = ["swan_init", "swan_destroy", "swan_set_k", "swan_append", "swan_flush_buffer",
             "swan_decode", "swan_query", "swan_debug_export", "swan_check",
             "swan_timing_enable", "swan_timing_read", "swan_launch_count",
-            "swan_status_string", "swan_last_error", "swan_decode_noalloc", "swan_set_kv"]
+            "swan_status_string", "swan_last_error", "swan_decode_noalloc", "swan_set_kv",
+            "swan_gram_workspace_bytes", "swan_gram", "swan_basis_eig", "swan_energy",
+            "swan_basis_check"]
 
 
 class SwanConfig(ctypes.Structure):
@@ -62,6 +64,14 @@ class CacheView(ctypes.Structure):
                 ("batch", ctypes.c_int), ("n_q_heads", ctypes.c_int), ("n_kv_heads", ctypes.c_int),
                 ("head_dim", ctypes.c_int), ("R_qk", ctypes.c_void_p), ("R_vo_t", ctypes.c_void_p),
                 ("value_format", ctypes.c_int), ("k_slots_v", ctypes.c_int), ("k_active_v", ctypes.c_int)]
+
+
+class SwanVectors(ctypes.Structure):
+    """A set of fp16 vectors in device memory (see swan_basis.h)."""
+    _fields_ = [("data", ctypes.c_void_p), ("n_mats", ctypes.c_int), ("group", ctypes.c_int),
+                ("count", ctypes.c_int64), ("stride_mat", ctypes.c_int64),
+                ("stride_group", ctypes.c_int64), ("stride_pos", ctypes.c_int64),
+                ("stride_coord", ctypes.c_int64)]
 
 
 class SwanError(RuntimeError):
@@ -100,6 +110,11 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "swan_status_string": (ctypes.c_char_p, [i]),
         "swan_last_error": (ctypes.c_char_p, []),
         "swan_decode_noalloc": (i, [ctypes.POINTER(CacheView), vp, vp, vp]),
+        "swan_gram_workspace_bytes": (ctypes.c_size_t, [i]),
+        "swan_gram": (i, [ctypes.POINTER(SwanVectors), vp, i, vp, ctypes.c_size_t, vp]),
+        "swan_basis_eig": (i, [vp, i, vp, vp, vp, vp]),
+        "swan_energy": (i, [ctypes.POINTER(SwanVectors), vp, vp, i, vp]),
+        "swan_basis_check": (i, [vp, vp]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(lib, name)
@@ -252,4 +267,106 @@ def decode_noalloc(view: CacheView, q, out, stream=None):
         stream = torch.cuda.current_stream()
     _check(lib.swan_decode_noalloc(ctypes.byref(view), _ptr(q), _ptr(out),
                                    ctypes.c_void_p(stream.cuda_stream)), "swan_decode_noalloc")
+    return out
+
+
+# ---------------------------------------------------------------------------
+# Offline basis construction (swan_basis.h)
+# ---------------------------------------------------------------------------
+
+def _stream_handle(stream):
+    import torch
+    return (stream or torch.cuda.current_stream()).cuda_stream
+
+
+def rows_of(t, group: int = 1) -> SwanVectors:
+    """Vectors that are the contiguous last dimension (128) of a CUDA fp16
+    tensor ``[n_mats * group][count][128]`` (e.g. Q ``[N_q][n][d]`` grouped by
+    kv head, or K / V ``[N_kv][n][d]``)."""
+    if t.dim() != 3 or t.shape[-1] != 128:
+        raise ValueError("expected [heads][count][128]")
+    if t.shape[0] % group:
+        raise ValueError("heads not divisible by group")
+    s = t.stride()
+    if s[2] != 1:
+        raise ValueError("the last dimension must be contiguous")
+    v = SwanVectors(_ptr_any(t), t.shape[0] // group, group, t.shape[1], s[0] * group, s[0], s[1], 1)
+    v._tensor = t  # the description holds the tensor's memory alive
+    return v
+
+
+def columns_of(w, group: int = 1) -> SwanVectors:
+    """Vectors that are the columns of the ``[128][d_model]`` row blocks of a
+    CUDA fp16 matrix ``[n_mats * group * 128][d_model]`` (W_O; block h is
+    query head h's slice)."""
+    if w.dim() != 2 or w.shape[0] % (128 * group):
+        raise ValueError("expected [n_mats * group * 128][d_model]")
+    if w.stride(1) != 1:
+        raise ValueError("rows must be contiguous")
+    ld = w.stride(0)
+    v = SwanVectors(_ptr_any(w), w.shape[0] // (128 * group), group, w.shape[1], group * 128 * ld, 128 * ld,
+                    1, ld)
+    v._tensor = w  # the description holds the tensor's memory alive
+    return v
+
+
+def _ptr_any(t) -> int:
+    if not t.is_cuda:
+        raise ValueError("tensor must live on the GPU")
+    return t.data_ptr()
+
+
+class Gram:
+    """Accumulates S^T S of joint matrices on the GPU (swan_gram) into a CUDA
+    fp32 tensor ``[n_mats][128][128]``; owns the workspace."""
+
+    def __init__(self, n_mats: int, device=None, stream=None):
+        import torch
+        self._lib = load_library()
+        self.stream = stream
+        self.n_mats = n_mats
+        self.gram = torch.zeros((n_mats, 128, 128), dtype=torch.float32, device=device or "cuda")
+        nbytes = self._lib.swan_gram_workspace_bytes(n_mats)
+        self._ws = torch.empty(nbytes + 256, dtype=torch.uint8, device=self.gram.device)
+        base = self._ws.data_ptr()
+        self._ws_ptr = (base + 255) // 256 * 256
+        self._ws_bytes = nbytes
+
+    def add(self, vectors: SwanVectors, accumulate: bool = True):
+        if vectors.n_mats != self.n_mats:
+            raise ValueError("n_mats differs from the Gram matrices'")
+        _check(self._lib.swan_gram(ctypes.byref(vectors), ctypes.c_void_p(self.gram.data_ptr()),
+                                   int(accumulate), ctypes.c_void_p(self._ws_ptr), self._ws_bytes,
+                                   ctypes.c_void_p(_stream_handle(self.stream))), "swan_gram")
+        return self
+
+    def check(self):
+        _check(self._lib.swan_basis_check(ctypes.c_void_p(self._ws_ptr),
+                                          ctypes.c_void_p(_stream_handle(self.stream))), "swan_basis_check")
+
+
+def basis_eig(gram, stream=None):
+    """Eigenvectors (R, columns by decreasing eigenvalue), eigenvalues and
+    sweep counts of CUDA fp32 Gram matrices ``[n][128][128]``."""
+    import torch
+    lib = load_library()
+    n = gram.shape[0]
+    R = torch.empty_like(gram)
+    lam = torch.empty((n, 128), dtype=torch.float32, device=gram.device)
+    sweeps = torch.empty((n,), dtype=torch.int32, device=gram.device)
+    _check(lib.swan_basis_eig(ctypes.c_void_p(_ptr(gram)), n, ctypes.c_void_p(R.data_ptr()),
+                              ctypes.c_void_p(lam.data_ptr()), ctypes.c_void_p(sweeps.data_ptr()),
+                              ctypes.c_void_p(_stream_handle(stream))), "swan_basis_eig")
+    return R, lam, sweeps
+
+
+def energy(vectors: SwanVectors, R, out=None, accumulate: bool = False, stream=None):
+    """Energy kept by top-k pruning in the basis R, for k = 0..128: CUDA fp64
+    ``[n_mats][129]``."""
+    import torch
+    lib = load_library()
+    if out is None:
+        out = torch.zeros((vectors.n_mats, 129), dtype=torch.float64, device=R.device)
+    _check(lib.swan_energy(ctypes.byref(vectors), ctypes.c_void_p(_ptr(R)), ctypes.c_void_p(out.data_ptr()),
+                           int(accumulate), ctypes.c_void_p(_stream_handle(stream))), "swan_energy")
     return out

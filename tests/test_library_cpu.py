@@ -10,7 +10,7 @@ import pytest
 from paper_2511_18936_gb300 import swan
 
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
-HEADER = os.path.join(ROOT, "include", "swan.h")
+HEADERS = [os.path.join(ROOT, "include", h) for h in ("swan.h", "swan_basis.h")]
 
 
 @pytest.fixture(scope="module")
@@ -22,9 +22,11 @@ def lib():
 
 
 def declared_functions():
-    text = open(HEADER).read()
-    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
-    return sorted(set(re.findall(r"\b(swan_[a-z_]+)\s*\(", text)))
+    names = set()
+    for h in HEADERS:
+        text = re.sub(r"/\*.*?\*/", "", open(h).read(), flags=re.S)
+        names |= set(re.findall(r"\b(swan_[a-z_]+)\s*\(", text))
+    return sorted(names)
 
 
 def test_header_declares_the_binding_list():
@@ -91,3 +93,55 @@ def test_null_arguments(lib):
     assert lib.swan_check(None) == swan.ERR_INVALID_ARG
     assert lib.swan_destroy(None) == swan.OK
     assert lib.swan_launch_count(None) == 0
+
+
+# ---------------------------------------------------------------------------
+# Offline basis entry points: host-side validation (no launch happens)
+# ---------------------------------------------------------------------------
+
+def _vec(**kw):
+    d = dict(data=4096, n_mats=2, group=1, count=100, stride_mat=12800, stride_group=0, stride_pos=128,
+             stride_coord=1)
+    d.update(kw)
+    return swan.SwanVectors(**d)
+
+
+@pytest.mark.parametrize("kw,needle", [
+    (dict(data=0), "data is NULL"),
+    (dict(data=4100), "16-byte aligned"),
+    (dict(n_mats=0), "n_mats"),
+    (dict(group=0), "group"),
+    (dict(count=0), "count"),
+    (dict(count=1 << 31), "count"),
+    (dict(stride_pos=100), "stride_pos"),
+    (dict(stride_coord=2, stride_pos=128), "either stride_coord or stride_pos"),
+    (dict(stride_coord=100, stride_pos=1), "stride_coord"),
+    (dict(group=2, stride_group=4), "stride_group"),
+    (dict(stride_mat=0), "stride_mat"),
+])
+def test_basis_vectors_validation(lib, kw, needle):
+    v = _vec(**kw)
+    st = lib.swan_gram(ctypes.byref(v), ctypes.c_void_p(4096), 0, ctypes.c_void_p(1 << 20),
+                       lib.swan_gram_workspace_bytes(2), None)
+    assert st == swan.ERR_INVALID_ARG
+    assert needle in lib.swan_last_error().decode()
+    st = lib.swan_energy(ctypes.byref(v), ctypes.c_void_p(4096), ctypes.c_void_p(4096), 0, None)
+    assert st == swan.ERR_INVALID_ARG
+
+
+def test_basis_workspace_and_pointer_checks(lib):
+    v = _vec()
+    assert lib.swan_gram_workspace_bytes(0) == 0
+    assert lib.swan_gram_workspace_bytes(1) == 320 * 65536 + 256
+    assert lib.swan_gram_workspace_bytes(1000) == 1000 * 65536 + 256
+    ws = lib.swan_gram_workspace_bytes(2)
+    assert lib.swan_gram(ctypes.byref(v), None, 0, ctypes.c_void_p(1 << 20), ws, None) == swan.ERR_INVALID_ARG
+    assert lib.swan_gram(ctypes.byref(v), ctypes.c_void_p(4096), 0, ctypes.c_void_p((1 << 20) + 16), ws,
+                         None) == swan.ERR_INVALID_ARG
+    assert lib.swan_gram(ctypes.byref(v), ctypes.c_void_p(4096), 0, ctypes.c_void_p(1 << 20), ws - 1,
+                         None) == swan.ERR_INVALID_ARG
+    assert "smaller" in lib.swan_last_error().decode()
+    assert lib.swan_basis_eig(None, 1, ctypes.c_void_p(4096), None, None, None) == swan.ERR_INVALID_ARG
+    assert lib.swan_basis_eig(ctypes.c_void_p(4096), 0, ctypes.c_void_p(4096), None, None,
+                              None) == swan.ERR_INVALID_ARG
+    assert lib.swan_basis_check(None, None) == swan.ERR_INVALID_ARG

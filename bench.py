@@ -55,8 +55,14 @@ WORKLOADS = {
                         desc="32-layer Llama-2-7B-shaped KV stack, batch 8, 8192-token prefix "
                              "compressed by one append per layer, decode steps appending one token "
                              "per layer, buffers flushed every 128 steps, k 64"),
+    "basis-llama3-8b": dict(kind="basis", n_kv=8, G=4, n=65536, d_model=4096,
+                            desc="offline basis (Section 4.1) for one Llama-3-8B-shaped layer: 32 q / 8 kv "
+                                 "heads, d 128, d_model 4096; one step accumulates S_QK^T S_QK and "
+                                 "S_VO^T S_VO over a calibration batch of 65536 tokens (Q, K, V and the "
+                                 "W_O columns); the eigensolver runs once after the batches"),
 }
 METRIC = "decode-attention KV-tokens/s and achieved HBM GB/s (% of 8 TB/s) at 32k ctx"
+BASIS_METRIC = "offline-basis calibration vectors/s (Gram accumulation on the tensor cores)"
 NOMINAL_HBM_GBS = 8000.0
 
 
@@ -180,9 +186,27 @@ def oracle_sample(wl, n_units: int, seed: int = 0):
     return step
 
 
+def basis_oracle_step(wl, n_tokens: int, seed: int = 0):
+    """One oracle step of the basis workload on a bounded sample: the joint
+    matrices of one kv head over ``n_tokens`` tokens and their SVD basis.
+    Returns (step function, vectors per step)."""
+    import oracle
+    from paper_2511_18936_gb300 import synth
+    G, d_model = wl["G"], wl["d_model"]
+    Q, K, V, W_O = synth.calibration(1, G, n_tokens, D, d_model, seed=seed, workload=8, layer=0)
+    bo = oracle.basis_oracle
+
+    def step():
+        bo.principal_basis(bo.joint_qk(Q, K, G)[0])
+        bo.principal_basis(bo.joint_vo(V, W_O, G)[0])
+    return step, (G + 2) * n_tokens + G * d_model
+
+
 def run_reference(args, wl, rank: int):
     if rank != 0:
         return None
+    if wl.get("kind") == "basis":
+        return run_reference_basis(args, wl)
     n_units = min(2, wl["B"] * wl["H_kv"])
     t0 = time.perf_counter()
     step = oracle_sample(wl, n_units)
@@ -208,6 +232,183 @@ def run_reference(args, wl, rank: int):
                              "sample": sample},
             "e2e": {"value": value, "unit": "KV-tokens/s", "h2d_bytes_per_step": 0,
                     "d2h_bytes_per_step": 0}}
+    return line
+
+
+def run_reference_basis(args, wl):
+    n_tok = 8192
+    step, vecs = basis_oracle_step(wl, n_tok)
+    for _ in range(args.warmup):
+        step()
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        step()
+    total = time.perf_counter() - t0
+    value = vecs * args.steps / total
+    sample = (f"1 of {wl['n_kv']} kv heads, {n_tok} of {wl['n']} calibration tokens: the joint matrices "
+              f"S_QK and S_VO and their SVD bases (NumPy fp64)")
+    return {"impl": "reference", "metric": BASIS_METRIC, "value": value, "unit": "vectors/s",
+            "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": 1e3 * total / args.steps, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": args.workload, "desc": wl["desc"], "parallelism": "none (host CPU)"},
+            "cpu_baseline": {"value": value, "unit": "vectors/s", "cores": 1, "kind": "oracle", "sample": sample},
+            "e2e": {"value": value, "unit": "vectors/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+
+
+def cpu_baseline_basis(wl, budget_s: float = 15.0):
+    n_tok = 16384
+    step, vecs = basis_oracle_step(wl, n_tok)
+    step()
+    t0 = time.perf_counter()
+    n = 0
+    while time.perf_counter() - t0 < budget_s:
+        step()
+        n += 1
+    dt = time.perf_counter() - t0
+    return {"value": vecs * n / dt, "unit": "vectors/s", "cores": 1, "kind": "oracle",
+            "sample": f"1 of {wl['n_kv']} kv heads, {n_tok} calibration tokens, joint matrices + SVD "
+                      f"basis (NumPy fp64, one thread), {n} steps in {dt:.1f} s"}
+
+
+def gram_kernel_traffic(workload: str):
+    """DRAM bytes per Gram launch from the committed ncu summary, if it was
+    taken on the current kernel source (else None)."""
+    src = os.path.join(ROOT, "paper_2511_18936_gb300", "csrc", "basis.cu")
+    digest = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+    try:
+        text = open(os.path.join(ROOT, "profiles", f"gram_kernel_{workload}.md")).read()
+    except OSError:
+        return None
+    m_src = re.search(r"basis\.cu sha256\[:16\]:\s*([0-9a-f]{16})", text)
+    m_tr = re.search(r"dram bytes per launch:\s*([0-9.eE+]+)", text)
+    if not m_src or not m_tr or m_src.group(1) != digest:
+        return None
+    return float(m_tr.group(1))
+
+
+def run_basis(args, wl, rank: int, world: int, local_rank: int):
+    """The offline-basis workload: Gram accumulation of the joint matrices
+    over calibration batches on the tensor cores (the data-parallel part),
+    the eigensolver timed once."""
+    import torch
+
+    from paper_2511_18936_gb300 import swan, synth
+    dev = torch.device("cuda", local_rank)
+    torch.cuda.set_device(dev)
+    n_kv, G, n, d_model = wl["n_kv"], wl["G"], wl["n"], wl["d_model"]
+    stream = torch.cuda.Stream(dev)
+    with torch.cuda.stream(stream):
+        Q, K, V, W_O = synth.torch_calibration(n_kv, G, n, D, d_model, seed=args.seed + rank, device=dev)
+        gq, gv = swan.Gram(n_kv, dev, stream), swan.Gram(n_kv, dev, stream)
+    stream.synchronize()
+    parts = [("Q", gq, swan.rows_of(Q, G)), ("K", gq, swan.rows_of(K)), ("V", gv, swan.rows_of(V)),
+             ("W_O", gv, swan.columns_of(W_O, G))]
+    vecs = n_kv * G * n + 2 * n_kv * n + n_kv * G * d_model
+    part_bytes = {"Q": Q.numel() * 2, "K": K.numel() * 2, "V": V.numel() * 2, "W_O": W_O.numel() * 2}
+
+    def step():
+        for name, g, v in parts:
+            g.add(v, accumulate=True)
+
+    with torch.cuda.stream(stream):
+        for _ in range(args.warmup):
+            step()
+    stream.synchronize()
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize(dev)
+    with ClockSampler(local_rank) as clk:
+        with torch.cuda.stream(stream):
+            ev0.record(stream)
+            for _ in range(args.steps):
+                step()
+            ev1.record(stream)
+        stream.synchronize()
+    ms = ev0.elapsed_time(ev1)
+    if world > 1:
+        torch.distributed.barrier()
+    gq.check()
+    gv.check()
+
+    # per-part times (memset + Gram kernel + split reduction) in a second region
+    part_ms = {}
+    with torch.cuda.stream(stream):
+        for name, g, v in parts:
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            for _ in range(args.steps):
+                g.add(v, accumulate=True)
+            b.record(stream)
+            stream.synchronize()
+            part_ms[name] = a.elapsed_time(b) / args.steps
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        both = torch.cat([gq.gram, gv.gram])  # one launch, one CTA per matrix
+        a.record(stream)
+        R_all, _, sw_all = swan.basis_eig(both, stream)
+        b.record(stream)
+    stream.synchronize()
+    eig_ms = a.elapsed_time(b)
+
+    # end to end: Q, K, V of the batch copied from pinned host memory every
+    # step, the Gram matrices read back
+    host = [t.cpu().pin_memory() for t in (Q, K, V)]
+    dev_in = [torch.empty_like(t) for t in (Q, K, V)]
+    e2e_parts = [(gq, swan.rows_of(dev_in[0], G)), (gq, swan.rows_of(dev_in[1])), (gv, swan.rows_of(dev_in[2])),
+                 (gv, swan.columns_of(W_O, G))]
+    host_out = [torch.empty_like(g.gram, device="cpu").pin_memory() for g in (gq, gv)]
+
+    def e2e_step():
+        with torch.cuda.stream(stream):
+            for d, h in zip(dev_in, host):
+                d.copy_(h, non_blocking=True)
+            for g, v in e2e_parts:
+                g.add(v, accumulate=True)
+            for ho, g in zip(host_out, (gq, gv)):
+                ho.copy_(g.gram, non_blocking=True)
+        stream.synchronize()
+
+    e2e_step()
+    t0 = time.perf_counter()
+    for _ in range(args.e2e_steps):
+        e2e_step()
+    e2e_s = time.perf_counter() - t0
+
+    value, e2e_value, t_max = aggregate_ranks(vecs * args.steps, ms, vecs * args.e2e_steps, e2e_s, world, dev)
+    peaks = measured_peaks()
+    peak = float(peaks["hbm_gbs"]) if peaks else 6800.0
+    q_s = part_ms["Q"] / 1e3
+    achieved = part_bytes["Q"] / q_s / 1e9
+    tflops = part_bytes["Q"] / 256 * 2 * D * D / q_s / 1e12
+    tpeak = float(peaks["bf16_tflops"]) if peaks and "bf16_tflops" in peaks else 1900.0
+    line = {
+        "metric": BASIS_METRIC, "value": value, "unit": "vectors/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": t_max / args.steps, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f16 x f16 -> f32",
+        "data": "synthetic calibration set (seeded per-head principal bases, power-law spectra)",
+        "config": {"workload": args.workload, "desc": wl["desc"], "n_kv_heads": n_kv, "group": G,
+                   "tokens_per_batch": n, "d_model": d_model,
+                   "l2": f"inputs larger than L2: {sum(part_bytes.values()) / 1e9:.2f} GB read per step, no flush",
+                   "parallelism": f"replicas x{world} (independent batches per GPU)" if world > 1
+                   else "single GPU"},
+        "roofline": {"kernel": "gram (Q part: memset + gram_kernel + split reduction)", "bound": "hbm",
+                     "achieved": achieved, "peak": peak, "unit": "GB/s", "frac": achieved / peak,
+                     "peak_source": "MEASURED_PEAKS.json hbm_gbs (measured copy)" if peaks else "fallback 6.8 TB/s",
+                     "alg_bytes_per_launch": part_bytes["Q"], "avg_launch_ms": part_ms["Q"],
+                     "tensor_tflops": tflops, "tensor_frac_of_bf16_peak": tflops / tpeak,
+                     "traffic": gram_kernel_traffic(args.workload)},
+        "parts_ms_per_step": part_ms,
+        "eig_ms_16_matrices": eig_ms,
+        "eig_sweeps": sw_all.tolist(),
+        "gpu_launches": 2 * len(parts) * args.steps,
+        "e2e": {"value": e2e_value, "unit": "vectors/s",
+                "h2d_bytes_per_step": sum(t.numel() * t.element_size() for t in host),
+                "d2h_bytes_per_step": sum(t.numel() * t.element_size() for t in host_out),
+                "steps": args.e2e_steps},
+        "clocks": clk.summary(),
+    }
     return line
 
 
@@ -541,6 +742,21 @@ def run_swan(args, wl, rank: int, world: int, local_rank: int):
     return line
 
 
+def _keep_counts(ap, args, wl):
+    """Value keep counts of the decode workloads from the command line."""
+    wl["k_store_v"] = args.k_store_v or wl["k_store"]
+    if not 1 <= wl["k_store_v"] <= D:
+        ap.error(f"--k-store-v must be in [1, {D}]")
+    if args.k_store_v:
+        wl["desc"] += f" (k_store_v {wl['k_store_v']})"
+    wl["k_v"] = min(wl["k"], wl["k_store_v"])
+    if args.k_active_v:
+        if not 1 <= args.k_active_v <= wl["k_store_v"]:
+            ap.error(f"--k-active-v must be in [1, {wl['k_store_v']}]")
+        wl["k_v"] = args.k_active_v
+        wl["desc"] += f" (k_active_v {args.k_active_v})"
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -557,6 +773,8 @@ def main():
                     help="kept sparse values as fp16 (3k bytes per vector) or E4M3 (2k)")
     ap.add_argument("--k-active", type=int, default=0,
                     help="runtime keep count (ksweep-32k: 32, 48, 64, 96 or 128)")
+    ap.add_argument("--tokens", type=int, default=0,
+                    help="basis workload: calibration tokens per batch (smaller cases for profiling)")
     ap.add_argument("--k-store-v", type=int, default=0,
                     help="value entries stored per vector (default: as for keys)")
     ap.add_argument("--k-active-v", type=int, default=0,
@@ -576,17 +794,13 @@ def main():
             ap.error(f"--k-active must be in [1, {wl['k_store']}]")
         wl["k"] = args.k_active
         wl["desc"] += f" (k_active {args.k_active})"
-    wl["k_store_v"] = args.k_store_v or wl["k_store"]
-    if not 1 <= wl["k_store_v"] <= D:
-        ap.error(f"--k-store-v must be in [1, {D}]")
-    if args.k_store_v:
-        wl["desc"] += f" (k_store_v {wl['k_store_v']})"
-    wl["k_v"] = min(wl["k"], wl["k_store_v"])
-    if args.k_active_v:
-        if not 1 <= args.k_active_v <= wl["k_store_v"]:
-            ap.error(f"--k-active-v must be in [1, {wl['k_store_v']}]")
-        wl["k_v"] = args.k_active_v
-        wl["desc"] += f" (k_active_v {args.k_active_v})"
+    if wl.get("kind") == "basis":
+        wl["k_store_v"] = wl["k_v"] = None
+        if args.tokens:
+            wl["n"] = args.tokens
+            wl["desc"] += f" (tokens per batch overridden to {args.tokens})"
+    else:
+        _keep_counts(ap, args, wl)
 
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
@@ -601,10 +815,11 @@ def main():
     if world > 1:
         import torch
         torch.distributed.init_process_group("nccl")
-    line = run_swan(args, wl, rank, world, local_rank)
+    basis = wl.get("kind") == "basis"
+    line = (run_basis if basis else run_swan)(args, wl, rank, world, local_rank)
     if rank == 0:
         if not args.no_cpu_baseline and world == 1:
-            line["cpu_baseline"] = cpu_baseline_leg(wl)
+            line["cpu_baseline"] = cpu_baseline_basis(wl) if basis else cpu_baseline_leg(wl)
         print(json.dumps(line), flush=True)
     if world > 1:
         import torch

@@ -157,14 +157,30 @@ __global__ void __launch_bounds__(128, 1) gram_kernel(const __grid_constant__ CU
   if (warp == 1) tmem_dealloc(tmem, 128);
 }
 
-// gram[m] = (accumulate ? gram[m] : 0) + sum over splits, in split order,
-// summed in fp64 (the fp32 rounding of the result is the only one added).
-__global__ void gram_reduce_kernel(const float* partials, float* gram, int splits, int accumulate) {
+// gram[m] = (accumulate ? gram[m] : 0) + sum over splits in a fixed order.
+// A block takes 32 consecutive entries; its 8 warps take the splits
+// s = w, w + 8, ... (many independent loads in flight), then warp 0 adds
+// the 8 warp sums in order.  fp32 throughout (fp64 arithmetic is slow on
+// this part); each entry sees at most splits / 8 + 9 additions.
+constexpr int kReduceGroups = 8;
+__global__ void __launch_bounds__(32 * kReduceGroups) gram_reduce_kernel(const float* partials, float* gram,
+                                                                         int splits, int accumulate) {
+  __shared__ float part[kReduceGroups][32];
   const int m = blockIdx.y;
-  const int e = blockIdx.x * blockDim.x + threadIdx.x;  // < 16384
-  double acc = accumulate ? (double)gram[(size_t)m * 16384 + e] : 0.0;
-  for (int s = 0; s < splits; ++s) acc += (double)partials[((size_t)m * splits + s) * 16384 + e];
-  gram[(size_t)m * 16384 + e] = (float)acc;
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  const int e = blockIdx.x * 32 + lane;  // < 16384
+  const float* src = partials + (size_t)m * splits * 16384 + e;
+  float acc = 0.f;
+#pragma unroll 4
+  for (int s = w; s < splits; s += kReduceGroups) acc += __ldg(src + (size_t)s * 16384);
+  part[w][lane] = acc;
+  __syncthreads();
+  if (w == 0) {
+    float tot = accumulate ? gram[(size_t)m * 16384 + e] : 0.f;
+#pragma unroll
+    for (int g = 0; g < kReduceGroups; ++g) tot += part[g][lane];
+    gram[(size_t)m * 16384 + e] = tot;
+  }
 }
 
 // ---------------------------------------------------------------------------
@@ -176,7 +192,7 @@ __global__ void gram_reduce_kernel(const float* partials, float* gram, int split
 // eigenvector, sign-fixed so that its largest-magnitude coordinate is
 // positive.
 // ---------------------------------------------------------------------------
-constexpr int kEigThreads = 512;
+constexpr int kEigThreads = 1024;
 constexpr int kLd = 129;  // padded row length
 
 __device__ __forceinline__ int rr_player(int pos, int round) {
@@ -231,39 +247,42 @@ __global__ void __launch_bounds__(kEigThreads, 1) jacobi_eig_kernel(EigParams p)
         dqq[i] = aqq + t * apq;
       }
       __syncthreads();
-      // columns: A <- A J, V <- V J
-      for (int e = threadIdx.x; e < 64 * 128; e += kEigThreads) {
-        const int i = e >> 7, k = e & 127;
-        const int a = pp[i], b = qq[i];
-        const float c = cs[i], s = sn[i];
-        if (s != 0.f) {
-          const float x = A[k * kLd + a], y = A[k * kLd + b];
-          A[k * kLd + a] = c * x - s * y;
-          A[k * kLd + b] = s * x + c * y;
-          const float u = V[k * kLd + a], w = V[k * kLd + b];
-          V[k * kLd + a] = c * u - s * w;
-          V[k * kLd + b] = s * u + c * w;
+      // A <- J^T A J as 64 x 64 independent 2 x 2 blocks (rows of pair i,
+      // columns of pair j), and V <- V J; one pass, no intermediate barrier.
+      for (int e = threadIdx.x; e < 64 * 64; e += kEigThreads) {
+        const int i = e >> 6, j = e & 63;
+        const float si = sn[i], sj = sn[j];
+        if (si == 0.f && sj == 0.f) continue;
+        const int ai = pp[i], bi = qq[i], aj = pp[j], bj = qq[j];
+        if (i == j) {
+          // the rotated pair's own block becomes diagonal
+          A[ai * kLd + ai] = dpp[i];
+          A[bi * kLd + bi] = dqq[i];
+          A[ai * kLd + bi] = 0.f;
+          A[bi * kLd + ai] = 0.f;
+          continue;
         }
+        const float ci = cs[i], cj = cs[j];
+        const float x00 = A[ai * kLd + aj], x01 = A[ai * kLd + bj];
+        const float x10 = A[bi * kLd + aj], x11 = A[bi * kLd + bj];
+        // rows: J_i^T X
+        const float r00 = ci * x00 - si * x10, r01 = ci * x01 - si * x11;
+        const float r10 = si * x00 + ci * x10, r11 = si * x01 + ci * x11;
+        // columns: (J_i^T X) J_j
+        A[ai * kLd + aj] = cj * r00 - sj * r01;
+        A[ai * kLd + bj] = sj * r00 + cj * r01;
+        A[bi * kLd + aj] = cj * r10 - sj * r11;
+        A[bi * kLd + bj] = sj * r10 + cj * r11;
       }
-      __syncthreads();
-      // rows: A <- J^T A
-      for (int e = threadIdx.x; e < 64 * 128; e += kEigThreads) {
-        const int i = e >> 7, k = e & 127;
-        const int a = pp[i], b = qq[i];
-        const float c = cs[i], s = sn[i];
-        if (s != 0.f) {
-          const float x = A[a * kLd + k], y = A[b * kLd + k];
-          A[a * kLd + k] = c * x - s * y;
-          A[b * kLd + k] = s * x + c * y;
-        }
-      }
-      __syncthreads();
-      if (threadIdx.x < 64 && sn[threadIdx.x] != 0.f) {
-        const int a = pp[threadIdx.x], b = qq[threadIdx.x];
-        A[a * kLd + a] = dpp[threadIdx.x];
-        A[b * kLd + b] = dqq[threadIdx.x];
-        A[a * kLd + b] = 0.f;
-        A[b * kLd + a] = 0.f;
+      for (int e = threadIdx.x; e < 128 * 64; e += kEigThreads) {
+        const int k = e >> 6, j = e & 63;
+        const float sj = sn[j];
+        if (sj == 0.f) continue;
+        const int aj = pp[j], bj = qq[j];
+        const float cj = cs[j];
+        const float u = V[k * kLd + aj], w = V[k * kLd + bj];
+        V[k * kLd + aj] = cj * u - sj * w;
+        V[k * kLd + bj] = sj * u + cj * w;
       }
       __syncthreads();
     }
@@ -483,7 +502,7 @@ cudaError_t launch_gram(const CUtensorMap& tmap, const GramParams& p, bool mn_ma
 
 cudaError_t launch_gram_reduce(const float* partials, float* gram, int n_mats, int splits, int accumulate,
                                cudaStream_t s) {
-  gram_reduce_kernel<<<dim3(16384 / 256, n_mats), 256, 0, s>>>(partials, gram, splits, accumulate);
+  gram_reduce_kernel<<<dim3(16384 / 32, n_mats), 32 * kReduceGroups, 0, s>>>(partials, gram, splits, accumulate);
   return cudaGetLastError();
 }
 

@@ -33,7 +33,9 @@
  *     poisoned and every later call returns SWAN_ERR_STATE.
  *   - No call allocates device memory after swan_init.
  *   - One context per stream; a context is not thread-safe.
- *   - All sequences of a batch have the same length.
+ *   - Rows (sequences) of a batch may differ in length (swan_append_varlen,
+ *     swan_reset_sequence); equal-length batches take the uniform fast path
+ *     of every kernel.
  *   - Nothing throws across the ABI and nothing calls abort().
  */
 #ifndef SWAN_H
@@ -83,6 +85,15 @@ typedef struct swan_config {
   int k_store_v;   /* value entries kept per vector, 1..d; 0 = k_store.  Keys
                       and values may keep different counts (Appendix,
                       ablation on key and value pruning ratios) */
+  int pool_pages;  /* 0: every (layer, row, kv head) owns the pages for
+                      max_seq tokens.  > 0: one pool of this many pages for
+                      all layers and rows; a row takes pages as its sparse
+                      history grows and returns them at swan_reset_sequence,
+                      so rows of different lengths share the memory
+                      (PagedAttention-style paging, Section 2's serving
+                      context).  An append or flush that needs more pages
+                      than are free returns SWAN_ERR_CAPACITY and changes
+                      nothing. */
 } swan_config;
 
 enum { SWAN_VALUES_FP16 = 0, SWAN_VALUES_FP8_E4M3 = 1 };
@@ -145,6 +156,28 @@ swan_status swan_append(swan_ctx* ctx, int layer, const void* k_new,
 swan_status swan_flush_buffer(swan_ctx* ctx, int layer);
 
 /*
+ * Append a different number of tokens to each row (sequence) of the batch:
+ * row b takes the first n_new[b] (0..T) of the T tokens given for it; the
+ * rest of k_new / v_new ([batch][n_kv_heads][T][d] fp16, device) is ignored.
+ * Each row then follows Algorithm 1 on its own: its buffer evicts its oldest
+ * tokens beyond b_cap into its sparse history.  Rows may thus differ in
+ * length; every call works per row from then on (swan_decode attends each
+ * row over its own tokens; a row with no token outputs zeros).
+ * n_new: HOST int32 [batch].  Errors: INVALID_ARG (n_new out of range),
+ * CAPACITY (a row beyond max_seq, or the page pool exhausted); nothing
+ * changes on error.
+ */
+swan_status swan_append_varlen(swan_ctx* ctx, int layer, const void* k_new, const void* v_new, int T,
+                               const int32_t* n_new);
+
+/*
+ * Forget row b in every layer (a finished request): its tokens are dropped
+ * and, with a page pool, its pages return to the pool.  Host-side only; the
+ * next call on the row starts from an empty cache.  Errors: INVALID_ARG.
+ */
+swan_status swan_reset_sequence(swan_ctx* ctx, int b);
+
+/*
  * One decode step of attention for one layer (Algorithm 1, attention part):
  *   q:   device fp16 [batch][n_q_heads][d], post-RoPE, unrotated.
  *   out: device fp16 [batch][n_q_heads][d], written as
@@ -171,7 +204,14 @@ typedef struct swan_layer_info {
   int k_active_v;       /* value entries used per vector */
   int k_store_v;        /* value entries stored per vector */
   int k_slots_v;        /* k_store_v rounded up to a multiple of 8 */
+  int uniform;          /* 1 if every row has the same lengths; sparse_len and
+                           buffer_len above are the largest over the rows */
+  int64_t pool_pages;   /* pages in the pool (all layers) */
+  int64_t free_pages;   /* free pages of a shared pool (pool_pages > 0) */
 } swan_layer_info;
+
+/* Per-row lengths of a layer: sparse_len, buffer_len HOST arrays [batch]. */
+swan_status swan_query_lengths(const swan_ctx* ctx, int layer, int64_t* sparse_len, int32_t* buffer_len);
 
 swan_status swan_query(const swan_ctx* ctx, int layer, swan_layer_info* info);
 
@@ -185,7 +225,8 @@ swan_status swan_query(const swan_ctx* ctx, int layer, swan_layer_info* info);
  *     shape, each vector's
  *     entries in stored (decreasing magnitude) order (8-bit values are
  *     widened to fp16, exactly).
- * bytes must equal the exact size of the requested view.
+ * bytes must equal the exact size of the requested view.  Every row must
+ * have the same lengths (else INVALID_ARG: export the rows one at a time).
  * Errors: INVALID_ARG (what, layer, size), STATE, CUDA.
  */
 enum {
@@ -196,6 +237,9 @@ enum {
 };
 swan_status swan_debug_export(swan_ctx* ctx, int layer, int what,
                               void* host_dst, size_t bytes);
+
+/* The same for row b alone: shapes [n_kv_heads][len_b][...]. */
+swan_status swan_debug_export_seq(swan_ctx* ctx, int layer, int b, int what, void* host_dst, size_t bytes);
 
 /*
  * Synchronise the stream and read the device status word that kernels set

@@ -334,6 +334,53 @@ class SwanOracle:
         return rotate_back(o_hat, self.R_vo[h])
 
 
+class RaggedOracle:
+    """A batch whose sequences (rows) differ in length: one single-row
+    ``SwanOracle`` per row, each following Algorithm 1 on its own tokens.
+    ``append(k, v, n_new)`` gives row b the first ``n_new[b]`` of the ``T``
+    tokens ``k[b, :, :T]``; ``reset(b)`` empties row b.  An empty row decodes
+    to zeros."""
+
+    def __init__(self, R_qk, R_vo=None, *, batch: int, n_q_heads: int, k_store: int, buffer_cap: int,
+                 value_format: str = "fp16", k_store_v: int | None = None):
+        self._args = dict(batch=1, n_q_heads=n_q_heads, k_store=k_store, buffer_cap=buffer_cap,
+                          value_format=value_format, k_store_v=k_store_v)
+        self._R = (R_qk, R_vo)
+        self.rows = [SwanOracle(R_qk, R_vo, **self._args) for _ in range(batch)]
+        self.k_active, self.k_active_v = k_store, k_store if k_store_v is None else k_store_v
+
+    def append(self, k_new, v_new, n_new=None):
+        T = k_new.shape[2]
+        for b, row in enumerate(self.rows):
+            n = T if n_new is None else int(n_new[b])
+            if n:
+                row.append(k_new[b:b + 1, :, :n], v_new[b:b + 1, :, :n])
+
+    def flush(self):
+        for row in self.rows:
+            row.flush()
+
+    def reset(self, b: int):
+        self.rows[b] = SwanOracle(*self._R, **self._args)
+        self.rows[b].set_k(self.k_active, self.k_active_v)
+
+    def set_k(self, k_active: int, k_active_v: int | None = None):
+        for row in self.rows:
+            row.set_k(k_active, k_active_v)
+        self.k_active, self.k_active_v = self.rows[0].k_active, self.rows[0].k_active_v
+
+    def decode(self, q):
+        return np.concatenate([row.decode(q[b:b + 1]) for b, row in enumerate(self.rows)])
+
+    @property
+    def sparse_lens(self):
+        return [row.sparse_len for row in self.rows]
+
+    @property
+    def buffer_lens(self):
+        return [row.buffer_len for row in self.rows]
+
+
 # ---------------------------------------------------------------------------
 # Byte and FLOP accounting (Section 5, Appendix "Derivation of Computational
 # Complexity")

@@ -100,6 +100,17 @@ __device__ __forceinline__ void warp_prune_store(uint2 raw, int lane, int kind, 
   }
 }
 
+// Lengths of row b for an append: the uniform scalars, or its SeqInfo entry.
+struct RowView {
+  int64_t sparse_len, evict;
+  int n_b, buf_start, n_new, prune;
+};
+__device__ __forceinline__ RowView row_view(const AppendParams& p, int64_t b, int evict_old) {
+  if (p.seq == nullptr) return RowView{p.sparse_len, p.evict, p.n_b, p.buf_start, p.T, evict_old};
+  const SeqInfo& q = p.seq[b];
+  return RowView{q.sparse_len, q.evict, q.n_b, q.buf_start, q.n_new, q.prune};
+}
+
 __device__ __forceinline__ float half_at(const uint4 (&xr)[16], int i) {
   const uint4 w = xr[i >> 3];
   const int q = (i >> 1) & 3;
@@ -134,12 +145,11 @@ __global__ void __launch_bounds__(kThreads, 1) append_kernel(AppendParams p) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int64_t nvec = (int64_t)p.B * p.T;
   const int64_t n = (int64_t)blockIdx.x * kThreads + threadIdx.x;
-  const bool valid = n < nvec;
-  int64_t b = 0, j = 0;
+  const int64_t b = n < nvec ? n / p.T : 0, j = n < nvec ? n % p.T : 0;
+  const RowView rv = row_view(p, b, 0);
+  const bool valid = n < nvec && j < rv.n_new;
   uint4 xr[16];
   if (valid) {
-    b = n / p.T;
-    j = n % p.T;
     const uint4* src = reinterpret_cast<const uint4*>(X + (((size_t)b * p.H + h) * p.T + j) * kHeadDim);
 #pragma unroll
     for (int i = 0; i < 16; ++i) xr[i] = __ldg(src + i);
@@ -149,11 +159,11 @@ __global__ void __launch_bounds__(kThreads, 1) append_kernel(AppendParams p) {
   }
   __syncthreads();
 
-  const int64_t pos = (int64_t)p.n_b + j;  // logical position in (buffer, new tokens)
-  const bool to_ring = valid && pos >= p.evict;
+  const int64_t pos = (int64_t)rv.n_b + j;  // logical position in (buffer, new tokens)
+  const bool to_ring = valid && pos >= rv.evict;
   __half* ring_row = nullptr;
   if (to_ring) {
-    const int slot = (int)((p.buf_start + pos) % p.cap);
+    const int slot = (int)((rv.buf_start + pos) % p.cap);
     ring_row = ring + (((size_t)b * p.H + h) * p.cap + slot) * kHeadDim;
   }
   uint32_t* my_stage = stage + threadIdx.x * kStageWords;
@@ -200,11 +210,13 @@ __global__ void __launch_bounds__(kThreads, 1) append_kernel(AppendParams p) {
     const int64_t nv = warp_first + v;
     if (nv >= nvec) break;
     const int64_t bv = nv / p.T, jv = nv % p.T;
-    const int64_t posv = (int64_t)p.n_b + jv;
-    if (posv >= p.evict) continue;
+    const RowView rvv = row_view(p, bv, 0);
+    if (jv >= rvv.n_new) continue;
+    const int64_t posv = (int64_t)rvv.n_b + jv;
+    if (posv >= rvv.evict) continue;
     const uint32_t* row = stage + (warp * 32 + v) * kStageWords;
     const uint2 raw = make_uint2(row[2 * lane], row[2 * lane + 1]);
-    warp_prune_store(raw, lane, kind, bv * p.H + h, p.sparse_len + posv, p.geom, p.status);
+    warp_prune_store(raw, lane, kind, bv * p.H + h, rvv.sparse_len + posv, p.geom, p.status);
   }
 }
 
@@ -233,16 +245,20 @@ __global__ void __launch_bounds__(kThreads) append_small_kernel(AppendParams p, 
   // phase 1: evict the oldest buffered vectors (sparse positions L_s + i)
   for (int item = warp; item < nb * evict_old; item += kWarpsPerCta) {
     const int b = b0 + item / evict_old, i = item % evict_old;
+    const RowView rv = row_view(p, b, evict_old);
+    if (i >= rv.prune) continue;
     const int64_t unit = (int64_t)b * p.H + h;
-    const int slot = (p.buf_start + i) % p.cap;
+    const int slot = (rv.buf_start + i) % p.cap;
     const uint2 raw = __ldg(reinterpret_cast<const uint2*>(ring + (unit * p.cap + slot) * kHeadDim) + lane);
-    warp_prune_store(raw, lane, kind, unit, p.sparse_len + i, p.geom, p.status);
+    warp_prune_store(raw, lane, kind, unit, rv.sparse_len + i, p.geom, p.status);
   }
   __syncthreads();
 
   // phase 2: the new vectors
   for (int item = warp; item < nb * p.T; item += kWarpsPerCta) {
     const int b = b0 + item / p.T, j = item % p.T;
+    const RowView rv = row_view(p, b, evict_old);
+    if (j >= rv.n_new) continue;
     const int64_t unit = (int64_t)b * p.H + h;
     const uint2 xw = __ldg(reinterpret_cast<const uint2*>(X + ((unit * p.T) + j) * kHeadDim) + lane);
     const float2 x01 = __half22float2(*reinterpret_cast<const __half2*>(&xw.x));
@@ -263,11 +279,11 @@ __global__ void __launch_bounds__(kThreads) append_small_kernel(AppendParams p, 
            ((uint32_t)__half_as_ushort(__float2half_rn(acc[1])) << 16);
     yw.y = (uint32_t)__half_as_ushort(__float2half_rn(acc[2])) |
            ((uint32_t)__half_as_ushort(__float2half_rn(acc[3])) << 16);
-    const int64_t pos = (int64_t)p.n_b + j;
-    if (pos < p.evict) {
-      warp_prune_store(yw, lane, kind, unit, p.sparse_len + pos, p.geom, p.status);
+    const int64_t pos = (int64_t)rv.n_b + j;
+    if (pos < rv.evict) {
+      warp_prune_store(yw, lane, kind, unit, rv.sparse_len + pos, p.geom, p.status);
     } else {
-      const int slot = (int)((p.buf_start + pos) % p.cap);
+      const int slot = (int)((rv.buf_start + pos) % p.cap);
       reinterpret_cast<uint2*>(ring + (unit * p.cap + slot) * kHeadDim)[lane] = yw;
     }
   }
@@ -285,10 +301,18 @@ __global__ void __launch_bounds__(kThreads) prune_ring_kernel(PruneRingParams p)
   const int64_t rest = gw >> 1;
   const int64_t unit = rest / p.count;
   const int i = (int)(rest % p.count);
-  const int slot = (p.buf_start + i) % p.cap;
+  int buf_start = p.buf_start;
+  int64_t sparse_len = p.sparse_len;
+  if (p.seq != nullptr) {
+    const SeqInfo& q = p.seq[unit / p.H];
+    if (i >= q.prune) return;
+    buf_start = q.buf_start;
+    sparse_len = q.sparse_len;
+  }
+  const int slot = (buf_start + i) % p.cap;
   const __half* row = (kind ? p.ring_v : p.ring_k) + ((size_t)unit * p.cap + slot) * kHeadDim;
   const uint2 raw = __ldg(reinterpret_cast<const uint2*>(row) + lane);
-  warp_prune_store(raw, lane, kind, unit, p.sparse_len + i, p.geom, p.status);
+  warp_prune_store(raw, lane, kind, unit, sparse_len + i, p.geom, p.status);
 }
 
 __global__ void transpose_r_kernel(const float* src, float* dst, int64_t mats) {
@@ -304,7 +328,21 @@ __global__ void transpose_r_kernel(const float* src, float* dst, int64_t mats) {
     d[(bx + r) * kHeadDim + by + threadIdx.x] = tile[threadIdx.x][r];
 }
 
+__global__ void scatter_pages_kernel(const int2* pairs, int n, int32_t* table) {
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i < n) {
+    const int2 pr = pairs[i];
+    table[pr.x] = pr.y;
+  }
+}
+
 }  // namespace
+
+cudaError_t launch_scatter_pages(const int2* pairs, int n, int32_t* table, cudaStream_t s) {
+  if (n <= 0) return cudaSuccess;
+  scatter_pages_kernel<<<(n + 255) / 256, 256, 0, s>>>(pairs, n, table);
+  return cudaGetLastError();
+}
 
 cudaError_t launch_append(const AppendParams& p, cudaStream_t s) {
   static bool attr_set = false;

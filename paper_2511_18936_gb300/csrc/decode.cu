@@ -202,16 +202,60 @@ __device__ __forceinline__ void value_chunk_partial(uint32_t ab, float p, const 
 
 constexpr uint32_t kRegionBytes = kHeadDim * 32 * sizeof(float);  // 16 KB
 
+// Geometry of unit u's groups in the flat split: its first group `goff`,
+// its group count and lengths; uniform rows read the scalars, ragged rows
+// their SeqInfo entry.
+struct UnitView {
+  int64_t goff, N_g, sparse_len;
+  int n_sg, n_b, buf_start;
+};
+__device__ __forceinline__ UnitView unit_view(const DecodeParams& p, int64_t u) {
+  UnitView v;
+  if (p.seq == nullptr) {
+    v.goff = u * p.N_g;
+    v.N_g = p.N_g;
+    v.sparse_len = p.sparse_len;
+    v.n_sg = (int)p.n_sg;
+    v.n_b = p.n_b;
+    v.buf_start = p.buf_start;
+  } else {
+    const int64_t b = u / p.H_kv, h = u - b * p.H_kv;
+    const SeqInfo& q = p.seq[b];
+    v.sparse_len = q.sparse_len;
+    v.n_sg = (int)((q.sparse_len + 31) >> 5);
+    v.n_b = q.n_b;
+    v.buf_start = q.buf_start;
+    v.N_g = row_groups(q.sparse_len, q.n_b);
+    v.goff = q.group_prefix * p.H_kv + h * v.N_g;
+  }
+  return v;
+}
+// The unit that holds flat group g (0 <= g < total_groups).
+__device__ __forceinline__ int64_t unit_of(const DecodeParams& p, int64_t g) {
+  if (p.seq == nullptr) return g / p.N_g;
+  int lo = 0, hi = p.B - 1;  // the last row whose first group is <= g
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (p.seq[mid].group_prefix * p.H_kv <= g) lo = mid;
+    else hi = mid - 1;
+  }
+  const SeqInfo& q = p.seq[lo];
+  const int64_t ng = row_groups(q.sparse_len, q.n_b);
+  const int64_t h = min((int64_t)p.H_kv - 1, (g - q.group_prefix * p.H_kv) / ng);
+  return (int64_t)lo * p.H_kv + h;
+}
+
 // The last CTA to finish a segment of unit u merges the unit's partials,
 // normalises, rotates back (o = o_hat R_vo^T) and writes the output.  The
 // arrival counter resets itself for the next decode; nothing waits.
 // `scratch` holds G * 128 floats (free at this point); `flag` one float.
 template <int G, int NT>
-__device__ __forceinline__ void finish_unit(const DecodeParams& p, int64_t u, int64_t b, int64_t h,
+__device__ __forceinline__ void finish_unit(const DecodeParams& p, const UnitView& uv, int64_t u, int64_t b,
+                                            int64_t h,
                                             float* scratch, float* flag) {
   __threadfence();
   __syncthreads();
-  const int64_t c0 = (u * p.N_g) / p.range, c1 = ((u + 1) * p.N_g - 1) / p.range;
+  const int64_t c0 = uv.goff / p.range, c1 = (uv.goff + uv.N_g - 1) / p.range;
   if (threadIdx.x == 0) {
     const int old = atomicAdd(p.counters + u, 1);
     const bool last = old == (int)(c1 - c0);
@@ -299,12 +343,13 @@ __global__ void __launch_bounds__(decode_warps<MAXC>() * 32, 1) decode_kernel(De
   const int64_t g_end = min(p.total_groups, g_begin + p.range);
   pdl_wait();
   if (g_begin >= g_end) return;
-  const int64_t u_first = g_begin / p.N_g, u_last = (g_end - 1) / p.N_g;
-  const int n_sg = (int)p.n_sg;
+  const int64_t u_first = unit_of(p, g_begin), u_last = unit_of(p, g_end - 1);
 
   for (int64_t u = u_first; u <= u_last; ++u) {
-    const int s0 = (int)(max(g_begin, u * p.N_g) - u * p.N_g);
-    const int s1 = (int)(min(g_end, (u + 1) * p.N_g) - u * p.N_g);
+    const UnitView uv = unit_view(p, u);
+    const int n_sg = uv.n_sg;
+    const int s0 = (int)(max(g_begin, uv.goff) - uv.goff);
+    const int s1 = (int)(min(g_end, uv.goff + uv.N_g) - uv.goff);
     const int64_t b = u / p.H_kv, h = u % p.H_kv;
     // this warp's contiguous run of groups [t_lo, t_hi)
     const int len = s1 - s0;
@@ -367,8 +412,8 @@ __global__ void __launch_bounds__(decode_warps<MAXC>() * 32, 1) decode_kernel(De
         // ---- sparse group: tokens 32*gi .. 32*gi+31 of the sparse history
         const int64_t t0 = (int64_t)gi * 32;
         const bool ok = b_cur != nullptr;
-        const bool valid = ok && t0 + lane < p.sparse_len;
-        const bool tail = !ok || t0 + 32 > p.sparse_len;  // warp-uniform
+        const bool valid = ok && t0 + lane < uv.sparse_len;
+        const bool tail = !ok || t0 + 32 > uv.sparse_len;  // warp-uniform
         const uint8_t* src = ok ? b_cur : g.pool;
         Chunk<FMT> vc[MAXC];
 #pragma unroll
@@ -437,8 +482,8 @@ __global__ void __launch_bounds__(decode_warps<MAXC>() * 32, 1) decode_kernel(De
       } else {
         // ---- buffer group: dense rotated fp16 vectors of the ring buffer
         const int64_t i = (int64_t)(gi - n_sg) * 32 + lane;
-        const bool valid = i < p.n_b;
-        const int slot = valid ? (int)((p.buf_start + i) % p.cap) : 0;
+        const bool valid = i < uv.n_b;
+        const int slot = valid ? (int)((uv.buf_start + i) % p.cap) : 0;
         const size_t row = ((size_t)u * p.cap + slot) * kHeadDim;
         const uint4* kr = reinterpret_cast<const uint4*>(p.ring_k + row);
         const uint4* vr = reinterpret_cast<const uint4*>(p.ring_v + row);
@@ -522,7 +567,7 @@ __global__ void __launch_bounds__(decode_warps<MAXC>() * 32, 1) decode_kernel(De
         dst[1] = L;
       }
     }
-    finish_unit<1, NT>(p, u, b, h, qrep, red_m);
+    finish_unit<1, NT>(p, uv, u, b, h, qrep, red_m);
   }
 }
 
@@ -645,12 +690,13 @@ __global__ void __launch_bounds__(kGqaWarps * 32, 1) decode_gqa_kernel(DecodePar
   const int64_t g_end = min(p.total_groups, g_begin + p.range);
   pdl_wait();
   if (g_begin >= g_end) return;
-  const int64_t u_first = g_begin / p.N_g, u_last = (g_end - 1) / p.N_g;
-  const int n_sg = (int)p.n_sg;
+  const int64_t u_first = unit_of(p, g_begin), u_last = unit_of(p, g_end - 1);
 
   for (int64_t u = u_first; u <= u_last; ++u) {
-    const int s0 = (int)(max(g_begin, u * p.N_g) - u * p.N_g);
-    const int s1 = (int)(min(g_end, (u + 1) * p.N_g) - u * p.N_g);
+    const UnitView uv = unit_view(p, u);
+    const int n_sg = uv.n_sg;
+    const int s0 = (int)(max(g_begin, uv.goff) - uv.goff);
+    const int s1 = (int)(min(g_end, uv.goff + uv.N_g) - uv.goff);
     const int64_t b = u / p.H_kv, h = u % p.H_kv;
     // this warp's contiguous run of items (half-blocks for G = 4)
     const int items = (s1 - s0) * HALVES;
@@ -719,8 +765,8 @@ __global__ void __launch_bounds__(kGqaWarps * 32, 1) decode_gqa_kernel(DecodePar
         // ---- sparse tokens 32*gi + half*TS + ts
         const int64_t t = (int64_t)gi * 32 + half * TS + ts;
         const bool ok = b_cur != nullptr;
-        valid = ok && t < p.sparse_len;
-        const bool tail = !ok || (int64_t)gi * 32 + (half + 1) * TS > p.sparse_len;  // warp-uniform
+        valid = ok && t < uv.sparse_len;
+        const bool tail = !ok || (int64_t)gi * 32 + (half + 1) * TS > uv.sparse_len;  // warp-uniform
         const uint8_t* src = ok ? b_cur : g.pool;
         const int tt = half * TS + ts;
         Chunk<FMT> vc[MAXC];
@@ -807,8 +853,8 @@ __global__ void __launch_bounds__(kGqaWarps * 32, 1) decode_gqa_kernel(DecodePar
       } else {
         // ---- dense buffer tokens
         const int64_t i = (int64_t)(gi - n_sg) * 32 + half * TS + ts;
-        valid = i < p.n_b;
-        const int slot = valid ? (int)((p.buf_start + i) % p.cap) : 0;
+        valid = i < uv.n_b;
+        const int slot = valid ? (int)((uv.buf_start + i) % p.cap) : 0;
         const size_t row = ((size_t)u * p.cap + slot) * kHeadDim;
         const uint4* kr = reinterpret_cast<const uint4*>(p.ring_k + row);
         const uint4* vr = reinterpret_cast<const uint4*>(p.ring_v + row);
@@ -897,7 +943,7 @@ __global__ void __launch_bounds__(kGqaWarps * 32, 1) decode_gqa_kernel(DecodePar
         dst[1] = L;
       }
     }
-    finish_unit<G, NT>(p, u, b, h, qrep, flag);
+    finish_unit<G, NT>(p, uv, u, b, h, qrep, flag);
   }
 }
 

@@ -32,10 +32,23 @@ swan_status fail(swan_status s, const char* fmt, ...) {
   return s;
 }
 
-struct LayerState {
+// One sequence (batch row) of one layer.
+struct SeqState {
   int64_t sparse_len = 0;
   int buf_start = 0;  // ring slot of the oldest buffered token
   int buf_count = 0;
+  bool operator==(const SeqState& o) const {
+    return sparse_len == o.sparse_len && buf_start == o.buf_start && buf_count == o.buf_count;
+  }
+};
+
+struct LayerState {
+  std::vector<SeqState> seq;  // [batch]
+  bool uniform() const {
+    for (const SeqState& q : seq)
+      if (!(q == seq[0])) return false;
+    return true;
+  }
 };
 
 struct EventPair {
@@ -57,6 +70,9 @@ struct swan_ctx {
   int ppu = 0;  // pages per unit
   int64_t page_bytes = 0;
   int64_t num_pages = 0;
+  bool paged = false;               // pages handed out on demand from a shared pool
+  std::vector<int32_t> free_pages;  // paged: free page ids
+  std::vector<int32_t> pt_host;     // paged: host copy of the page tables, -1 = none
   int fmt = kFmtFp16;
   int64_t units = 0;  // batch * n_kv_heads (per layer)
   cudaStream_t stream = nullptr;
@@ -75,6 +91,8 @@ struct swan_ctx {
   float* partials = nullptr;
   int* counters = nullptr;  // per-unit arrival counters of the fused combine
   unsigned* status = nullptr;
+  SeqInfo* seq_dev = nullptr;  // [layers][batch] per-row lengths for ragged calls
+  int2* pt_pairs = nullptr;    // paged: (entry, page) updates of one call
   int64_t device_bytes = 0;
 
   std::vector<LayerState> layers;
@@ -105,6 +123,8 @@ void free_all(swan_ctx* c) {
   cudaFree(c->partials);
   cudaFree(c->counters);
   cudaFree(c->status);
+  cudaFree(c->seq_dev);
+  cudaFree(c->pt_pairs);
   for (auto& e : c->ev_free) {
     cudaEventDestroy(e.start);
     cudaEventDestroy(e.stop);
@@ -229,27 +249,107 @@ uint16_t e4m3_to_half_bits(uint8_t b) {
   return sign | (uint16_t)(he << 10) | (uint16_t)hm;
 }
 
-// Prune buffered tokens 0..count-1 of a layer into the sparse cache.
-swan_status prune_from_ring(swan_ctx* c, int layer, int count) {
-  if (count <= 0) return SWAN_OK;
+int64_t pages_for(int64_t tokens, int P) { return (tokens + P - 1) / P; }
+
+// Paged pool: give every unit of each row the pages its sparse history needs
+// to reach new_len[b] tokens, and write them into the device page table.
+// Nothing changes when the pool is too small.
+swan_status grow_pages(swan_ctx* c, int layer, const std::vector<int64_t>& new_len) {
+  if (!c->paged) return SWAN_OK;
   LayerState& L = c->layers[layer];
+  const int H = c->cfg.n_kv_heads;
+  int64_t need = 0;
+  for (int b = 0; b < c->cfg.batch; ++b)
+    need += (int64_t)H * std::max<int64_t>(0, pages_for(new_len[b], c->P) - pages_for(L.seq[b].sparse_len, c->P));
+  if (need == 0) return SWAN_OK;
+  if (need > (int64_t)c->free_pages.size())
+    return fail(SWAN_ERR_CAPACITY, "layer %d needs %lld more pages, the pool has %zu free", layer, (long long)need,
+                c->free_pages.size());
+  std::vector<int2> pairs;
+  pairs.reserve((size_t)need);
+  for (int b = 0; b < c->cfg.batch; ++b) {
+    const int64_t p0 = pages_for(L.seq[b].sparse_len, c->P), p1 = pages_for(new_len[b], c->P);
+    for (int h = 0; h < H; ++h) {
+      const int64_t unit = (int64_t)b * H + h;
+      for (int64_t pg = p0; pg < p1; ++pg) {
+        const int32_t id = c->free_pages.back();
+        c->free_pages.pop_back();
+        c->pt_host[((size_t)layer * c->units + unit) * c->ppu + pg] = id;
+        pairs.push_back(make_int2((int)(unit * c->ppu + pg), id));
+      }
+    }
+  }
+  cudaError_t e = cudaMemcpyAsync(c->pt_pairs, pairs.data(), pairs.size() * sizeof(int2), cudaMemcpyHostToDevice,
+                                  c->stream);
+  if (e != cudaSuccess) return cuda_fail(c, e, "uploading page-table entries");
+  int32_t* table = c->page_table + (int64_t)layer * c->units * c->ppu;
+  return launch(c, SWAN_KERNEL_PRUNE, "page-table scatter",
+                [&] { return launch_scatter_pages(c->pt_pairs, (int)pairs.size(), table, c->stream); });
+}
+
+// Upload a layer's per-row table for the next ragged launch (ordered on the
+// stream; the host vector may be reused once this returns).
+swan_status upload_rows(swan_ctx* c, int layer, const std::vector<SeqInfo>& rows) {
+  cudaError_t e = cudaMemcpyAsync(c->seq_dev + (size_t)layer * c->cfg.batch, rows.data(),
+                                  rows.size() * sizeof(SeqInfo), cudaMemcpyHostToDevice, c->stream);
+  if (e != cudaSuccess) return cuda_fail(c, e, "uploading per-row lengths");
+  return SWAN_OK;
+}
+
+// Prune buffered tokens 0..count[b]-1 of every row b of a layer into the
+// sparse cache (eviction before a bulk append, and flush).
+swan_status prune_from_ring(swan_ctx* c, int layer, const std::vector<int>& count) {
+  LayerState& L = c->layers[layer];
+  const int B = c->cfg.batch;
+  int most = 0;
+  bool same = L.uniform();
+  for (int b = 0; b < B; ++b) {
+    most = std::max(most, count[b]);
+    same = same && count[b] == count[0];
+  }
+  if (most <= 0) return SWAN_OK;
+  std::vector<int64_t> new_len(B);
+  for (int b = 0; b < B; ++b) new_len[b] = L.seq[b].sparse_len + count[b];
+  swan_status s = grow_pages(c, layer, new_len);
+  if (s != SWAN_OK) return s;
   PruneRingParams p{};
   p.ring_k = c->ring_k + (size_t)layer * ring_elems_per_layer(c);
   p.ring_v = c->ring_v + (size_t)layer * ring_elems_per_layer(c);
   p.units = (int)c->units;
   p.cap = c->cfg.buffer_cap;
-  p.buf_start = L.buf_start;
-  p.count = count;
-  p.sparse_len = L.sparse_len;
+  p.buf_start = L.seq[0].buf_start;
+  p.count = most;
+  p.sparse_len = L.seq[0].sparse_len;
+  p.H = c->cfg.n_kv_heads;
   p.geom = geom_for(c, layer);
   p.status = c->status;
-  swan_status s = launch(c, SWAN_KERNEL_PRUNE, "prune_ring kernel",
-                         [&] { return launch_prune_ring(p, c->stream); });
+  if (!same) {
+    std::vector<SeqInfo> rows(B);
+    for (int b = 0; b < B; ++b) {
+      rows[b] = SeqInfo{};
+      rows[b].sparse_len = L.seq[b].sparse_len;
+      rows[b].buf_start = L.seq[b].buf_start;
+      rows[b].n_b = L.seq[b].buf_count;
+      rows[b].prune = count[b];
+    }
+    if ((s = upload_rows(c, layer, rows)) != SWAN_OK) return s;
+    p.seq = c->seq_dev + (size_t)layer * B;
+  }
+  s = launch(c, SWAN_KERNEL_PRUNE, "prune_ring kernel", [&] { return launch_prune_ring(p, c->stream); });
   if (s != SWAN_OK) return s;
-  L.sparse_len += count;
-  L.buf_start = c->cfg.buffer_cap ? (L.buf_start + count) % c->cfg.buffer_cap : 0;
-  L.buf_count -= count;
+  for (int b = 0; b < B; ++b) {
+    SeqState& q = L.seq[b];
+    q.sparse_len += count[b];
+    q.buf_start = c->cfg.buffer_cap ? (q.buf_start + count[b]) % c->cfg.buffer_cap : 0;
+    q.buf_count -= count[b];
+  }
   return SWAN_OK;
+}
+
+std::vector<int> buffer_counts(const LayerState& L) {
+  std::vector<int> n(L.seq.size());
+  for (size_t b = 0; b < L.seq.size(); ++b) n[b] = L.seq[b].buf_count;
+  return n;
 }
 
 }  // namespace
@@ -305,6 +405,7 @@ swan_status swan_init(swan_ctx** out, const swan_config* cfg, const float* R_qk,
   const int P = C.page_tokens ? C.page_tokens : 128;
   if (P < 32 || P > 4096 || (P & (P - 1)))
     return fail(SWAN_ERR_INVALID_ARG, "page_tokens %d must be a power of two in [32, 4096]", P);
+  if (C.pool_pages < 0) return fail(SWAN_ERR_INVALID_ARG, "pool_pages %d < 0", C.pool_pages);
 
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
@@ -327,11 +428,14 @@ swan_status swan_init(swan_ctx** out, const swan_config* cfg, const float* R_qk,
   c->fmt = C.value_format == SWAN_VALUES_FP8_E4M3 ? kFmtFp8 : kFmtFp16;
   c->page_bytes = page_bytes_for(P, c->k_slots, c->k_slots_v, c->fmt);
   c->units = (int64_t)C.batch * C.n_kv_heads;
-  c->num_pages = (int64_t)C.num_layers * c->units * c->ppu;
+  const int64_t full_pages = (int64_t)C.num_layers * c->units * c->ppu;
+  c->paged = C.pool_pages > 0;
+  c->num_pages = c->paged ? (int64_t)C.pool_pages : full_pages;
   c->stream = static_cast<cudaStream_t>(C.stream);
   c->device = dev;
   c->num_sms = sms;
   c->layers.assign(C.num_layers, LayerState{});
+  for (LayerState& L : c->layers) L.seq.assign(C.batch, SeqState{});
 
   const int per_sm = decode_ctas_per_sm(G, std::max(c->k_slots, c->k_slots_v));
   if (per_sm < 1) {
@@ -346,9 +450,9 @@ swan_status swan_init(swan_ctx** out, const swan_config* cfg, const float* R_qk,
   const size_t q_elems = (size_t)C.batch * C.n_q_heads * kHeadDim;
   const size_t pairs = (size_t)c->decode_ctas + (size_t)c->units;
   const size_t part_elems = pairs * G * (kHeadDim + 2);
-  const size_t pt_elems = (size_t)c->num_pages;
-  if (c->num_pages > INT32_MAX) {
-    const long long np = (long long)c->num_pages;
+  const size_t pt_elems = (size_t)full_pages;  // page-table entries: [layer][unit][page]
+  if (full_pages > INT32_MAX || c->num_pages > INT32_MAX) {
+    const long long np = (long long)std::max(full_pages, c->num_pages);
     delete c;
     return fail(SWAN_ERR_UNSUPPORTED, "too many pages (%lld)", np);
   }
@@ -366,6 +470,10 @@ swan_status swan_init(swan_ctx** out, const swan_config* cfg, const float* R_qk,
   if (s == SWAN_OK) s = dev_alloc(c, (void**)&c->partials, part_elems * sizeof(float), "split partials");
   if (s == SWAN_OK) s = dev_alloc(c, (void**)&c->counters, (size_t)c->units * sizeof(int), "counters");
   if (s == SWAN_OK) s = dev_alloc(c, (void**)&c->status, sizeof(unsigned), "status word");
+  if (s == SWAN_OK)
+    s = dev_alloc(c, (void**)&c->seq_dev, (size_t)C.num_layers * C.batch * sizeof(SeqInfo), "per-row lengths");
+  if (s == SWAN_OK && c->paged)
+    s = dev_alloc(c, (void**)&c->pt_pairs, (size_t)c->units * c->ppu * sizeof(int2), "page-table updates");
   if (s != SWAN_OK) {
     free_all(c);
     delete c;
@@ -374,8 +482,14 @@ swan_status swan_init(swan_ctx** out, const swan_config* cfg, const float* R_qk,
   if (!R_vo) c->R_vo = c->R_qk;
 
   // Contents: R copies, identity page table, zeroed pool and rings.
+  // every unit owns its pages (identity table), or none until it needs them
   std::vector<int32_t> pt(pt_elems);
-  for (size_t i = 0; i < pt_elems; ++i) pt[i] = (int32_t)i;
+  for (size_t i = 0; i < pt_elems; ++i) pt[i] = c->paged ? -1 : (int32_t)i;
+  if (c->paged) {
+    c->pt_host = pt;
+    c->free_pages.resize((size_t)c->num_pages);
+    for (int64_t i = 0; i < c->num_pages; ++i) c->free_pages[(size_t)i] = (int32_t)(c->num_pages - 1 - i);
+  }
   cudaStream_t st = c->stream;
   e = cudaMemcpyAsync(c->R_qk, R_qk, rmat * sizeof(float), cudaMemcpyDeviceToDevice, st);
   if (e == cudaSuccess && R_vo)
@@ -430,40 +544,93 @@ swan_status swan_set_k(swan_ctx* c, int k_active) {
   return SWAN_OK;
 }
 
-swan_status swan_append(swan_ctx* c, int layer, const void* k_new, const void* v_new, int T) {
+namespace {
+
+// Append T (padded) tokens per row; row b takes n_new[b] of them (all T when
+// n_new is null).  Algorithm 1 generalised to T tokens, per row: logical
+// positions 0..n_b-1 are the buffered tokens (oldest first), n_b..n_b+T_b-1
+// the new ones; everything before evict = max(0, n_b + T_b - b_cap) goes to
+// the sparse history, in order.
+swan_status append_rows(swan_ctx* c, int layer, const void* k_new, const void* v_new, int T,
+                        const int32_t* n_new) {
   swan_status s = usable(c);
   if (s != SWAN_OK) return s;
   if ((s = check_layer(c, layer)) != SWAN_OK) return s;
   if (T < 0) return fail(SWAN_ERR_INVALID_ARG, "T %d < 0", T);
   if (T == 0) return SWAN_OK;
   if (!k_new || !v_new) return fail(SWAN_ERR_INVALID_ARG, "k_new or v_new is NULL");
+  if ((int64_t)c->cfg.batch * T > (int64_t)INT32_MAX * 128) return fail(SWAN_ERR_INVALID_ARG, "T too large");
   LayerState& L = c->layers[layer];
+  const int B = c->cfg.batch;
   const int cap = c->cfg.buffer_cap;
-  const int64_t total = L.sparse_len + L.buf_count + (int64_t)T;
-  if (total > c->cfg.max_seq)
-    return fail(SWAN_ERR_CAPACITY, "layer %d would hold %lld tokens > max_seq %d", layer, (long long)total,
-                c->cfg.max_seq);
-  if ((int64_t)c->cfg.batch * T > (int64_t)INT32_MAX * 128)
-    return fail(SWAN_ERR_INVALID_ARG, "T too large");
+  std::vector<int> Tb(B, T);
+  if (n_new) {
+    for (int b = 0; b < B; ++b) {
+      if (n_new[b] < 0 || n_new[b] > T)
+        return fail(SWAN_ERR_INVALID_ARG, "n_new[%d] = %d out of [0, %d]", b, n_new[b], T);
+      Tb[b] = n_new[b];
+    }
+  }
+  std::vector<int64_t> evict(B), new_len(B);
+  std::vector<int> old_evict(B);
+  int most_tokens = 0, most_old = 0;
+  bool same = L.uniform();
+  for (int b = 0; b < B; ++b) {
+    const SeqState& q = L.seq[b];
+    const int64_t total = q.sparse_len + q.buf_count + (int64_t)Tb[b];
+    if (total > c->cfg.max_seq)
+      return fail(SWAN_ERR_CAPACITY, "layer %d row %d would hold %lld tokens > max_seq %d", layer, b,
+                  (long long)total, c->cfg.max_seq);
+    evict[b] = std::max<int64_t>(0, (int64_t)q.buf_count + Tb[b] - cap);
+    old_evict[b] = (int)std::min<int64_t>(evict[b], q.buf_count);
+    new_len[b] = q.sparse_len + evict[b];
+    most_tokens = std::max(most_tokens, Tb[b]);
+    most_old = std::max(most_old, old_evict[b]);
+    same = same && Tb[b] == T;
+  }
+  if (most_tokens == 0) return SWAN_OK;
+  // pages for the tokens that reach the sparse history (paged pool)
+  if ((s = grow_pages(c, layer, new_len)) != SWAN_OK) return s;
 
-  // Algorithm 1 generalised to T tokens: logical positions 0..n_b-1 are the
-  // buffered tokens (oldest first), n_b..n_b+T-1 the new ones; everything
-  // before `evict` goes to the sparse history, in order.
-  const int64_t evict = std::max<int64_t>(0, (int64_t)L.buf_count + T - cap);
-  const int old_evict = (int)std::min<int64_t>(evict, L.buf_count);
-
-  const int64_t sparse_before = L.sparse_len;
-  const int start_before = L.buf_start;
-  const int count_before = L.buf_count;
   // Decode-step appends (few vectors per head) run as one launch that evicts
   // and inserts; bulk appends as a pruning launch for the evicted buffered
   // tokens followed by the rotation launch.
-  const bool small = (int64_t)c->cfg.batch * T <= kSmallAppendVectors &&
-                     (int64_t)c->cfg.batch * old_evict <= kSmallAppendVectors;
+  const bool small = (int64_t)B * T <= kSmallAppendVectors && (int64_t)B * most_old <= kSmallAppendVectors;
+  const std::vector<SeqState> before = L.seq;
+  const SeqInfo* rows_dev = nullptr;
+  if (!same) {
+    std::vector<SeqInfo> rows(B);
+    for (int b = 0; b < B; ++b) {
+      rows[b] = SeqInfo{};
+      rows[b].sparse_len = before[b].sparse_len;
+      rows[b].buf_start = before[b].buf_start;
+      rows[b].n_b = before[b].buf_count;
+      rows[b].n_new = Tb[b];
+      rows[b].evict = (int32_t)evict[b];
+      rows[b].prune = old_evict[b];
+    }
+    if ((s = upload_rows(c, layer, rows)) != SWAN_OK) return s;
+    rows_dev = c->seq_dev + (size_t)layer * B;
+  }
 
   // 1) prune the evicted buffered tokens (they leave the ring first, so the
-  //    new tokens may reuse their slots)
-  if (!small && (s = prune_from_ring(c, layer, old_evict)) != SWAN_OK) return s;
+  //    new tokens may reuse their slots); the table above carries the counts
+  if (!small && most_old > 0) {
+    PruneRingParams pr{};
+    pr.ring_k = c->ring_k + (size_t)layer * ring_elems_per_layer(c);
+    pr.ring_v = c->ring_v + (size_t)layer * ring_elems_per_layer(c);
+    pr.units = (int)c->units;
+    pr.cap = cap;
+    pr.buf_start = before[0].buf_start;
+    pr.count = most_old;
+    pr.sparse_len = before[0].sparse_len;
+    pr.seq = rows_dev;
+    pr.H = c->cfg.n_kv_heads;
+    pr.geom = geom_for(c, layer);
+    pr.status = c->status;
+    s = launch(c, SWAN_KERNEL_PRUNE, "prune_ring kernel", [&] { return launch_prune_ring(pr, c->stream); });
+    if (s != SWAN_OK) return s;
+  }
 
   // 2) rotate the new tokens; those before `evict` are pruned directly, the
   //    rest land in the ring after the surviving buffered tokens
@@ -474,39 +641,87 @@ swan_status swan_append(swan_ctx* c, int layer, const void* k_new, const void* v
   p.R_vo = c->R_vo + (size_t)layer * c->cfg.n_kv_heads * kHeadDim * kHeadDim;
   p.ring_k = c->ring_k + (size_t)layer * ring_elems_per_layer(c);
   p.ring_v = c->ring_v + (size_t)layer * ring_elems_per_layer(c);
-  p.B = c->cfg.batch;
+  p.B = B;
   p.H = c->cfg.n_kv_heads;
   p.T = T;
   p.cap = cap > 0 ? cap : 1;
-  p.buf_start = start_before;
-  p.n_b = count_before;
-  p.evict = evict;
-  p.sparse_len = sparse_before;
+  p.buf_start = before[0].buf_start;
+  p.n_b = before[0].buf_count;
+  p.evict = evict[0];
+  p.sparse_len = before[0].sparse_len;
+  p.seq = rows_dev;
   p.geom = geom_for(c, layer);
   p.status = c->status;
   if (small)
     s = launch(c, SWAN_KERNEL_APPEND, "append_small kernel",
-               [&] { return launch_append_small(p, old_evict, c->stream); });
+               [&] { return launch_append_small(p, most_old, c->stream); });
   else
     s = launch(c, SWAN_KERNEL_APPEND, "append kernel", [&] { return launch_append(p, c->stream); });
   if (s != SWAN_OK) return s;
 
-  L.sparse_len = sparse_before + evict;
-  L.buf_count = (int)((int64_t)count_before + T - evict);
-  L.buf_start = cap > 0 ? (int)((start_before + evict) % cap) : 0;
+  for (int b = 0; b < B; ++b) {
+    SeqState& q = L.seq[b];
+    q.sparse_len = before[b].sparse_len + evict[b];
+    q.buf_count = (int)((int64_t)before[b].buf_count + Tb[b] - evict[b]);
+    q.buf_start = cap > 0 ? (int)((before[b].buf_start + evict[b]) % cap) : 0;
+  }
   return SWAN_OK;
+}
+
+}  // namespace
+
+swan_status swan_append(swan_ctx* c, int layer, const void* k_new, const void* v_new, int T) {
+  return append_rows(c, layer, k_new, v_new, T, nullptr);
+}
+
+swan_status swan_append_varlen(swan_ctx* c, int layer, const void* k_new, const void* v_new, int T,
+                               const int32_t* n_new) {
+  if (!n_new) return fail(SWAN_ERR_INVALID_ARG, "n_new is NULL");
+  return append_rows(c, layer, k_new, v_new, T, n_new);
 }
 
 swan_status swan_flush_buffer(swan_ctx* c, int layer) {
   swan_status s = usable(c);
   if (s != SWAN_OK) return s;
   if (layer == -1) {
+    if (c->paged) {  // all layers or none: check the pool first
+      int64_t need = 0;
+      for (int l = 0; l < c->cfg.num_layers; ++l)
+        for (const SeqState& q : c->layers[l].seq)
+          need += (int64_t)c->cfg.n_kv_heads *
+                  (pages_for(q.sparse_len + q.buf_count, c->P) - pages_for(q.sparse_len, c->P));
+      if (need > (int64_t)c->free_pages.size())
+        return fail(SWAN_ERR_CAPACITY, "flushing every layer needs %lld more pages, the pool has %zu free",
+                    (long long)need, c->free_pages.size());
+    }
     for (int l = 0; l < c->cfg.num_layers; ++l)
-      if ((s = prune_from_ring(c, l, c->layers[l].buf_count)) != SWAN_OK) return s;
+      if ((s = prune_from_ring(c, l, buffer_counts(c->layers[l]))) != SWAN_OK) return s;
     return SWAN_OK;
   }
   if ((s = check_layer(c, layer)) != SWAN_OK) return s;
-  return prune_from_ring(c, layer, c->layers[layer].buf_count);
+  return prune_from_ring(c, layer, buffer_counts(c->layers[layer]));
+}
+
+swan_status swan_reset_sequence(swan_ctx* c, int b) {
+  swan_status s = usable(c);
+  if (s != SWAN_OK) return s;
+  if (b < 0 || b >= c->cfg.batch) return fail(SWAN_ERR_INVALID_ARG, "row %d out of [0, %d)", b, c->cfg.batch);
+  for (int l = 0; l < c->cfg.num_layers; ++l) {
+    SeqState& q = c->layers[l].seq[b];
+    if (c->paged) {
+      const int64_t used = pages_for(q.sparse_len, c->P);
+      for (int h = 0; h < c->cfg.n_kv_heads; ++h) {
+        const int64_t unit = (int64_t)b * c->cfg.n_kv_heads + h;
+        for (int64_t pg = 0; pg < used; ++pg) {
+          int32_t& id = c->pt_host[((size_t)l * c->units + unit) * c->ppu + pg];
+          c->free_pages.push_back(id);
+          id = -1;
+        }
+      }
+    }
+    q = SeqState{};
+  }
+  return SWAN_OK;
 }
 
 swan_status swan_decode(swan_ctx* c, int layer, const void* q, void* out) {
@@ -532,10 +747,31 @@ swan_status swan_decode(swan_ctx* c, int layer, const void* q, void* out) {
              [&] { return launch_rotate_q(rq, c->cfg.batch, c->stream); });
   if (s != SWAN_OK) return s;
 
-  const int64_t n_sg = (L.sparse_len + 31) / 32;
-  const int64_t n_bg = (L.buf_count + 31) / 32;
+  // Uniform rows: every unit has the same groups.  Ragged rows: each row's
+  // groups (at least one, so an empty row still writes its zero output),
+  // offsets in a per-row table.
+  const bool same = L.uniform();
+  const SeqState& q0 = L.seq[0];
+  const int64_t n_sg = (q0.sparse_len + 31) / 32;
+  const int64_t n_bg = (q0.buf_count + 31) / 32;
   const int64_t N_g = n_sg + n_bg;
-  const int64_t total = c->units * N_g;
+  int64_t total = c->units * N_g;
+  const SeqInfo* rows_dev = nullptr;
+  if (!same) {
+    std::vector<SeqInfo> rows(c->cfg.batch);
+    int64_t prefix = 0;
+    for (int b = 0; b < c->cfg.batch; ++b) {
+      rows[b] = SeqInfo{};
+      rows[b].sparse_len = L.seq[b].sparse_len;
+      rows[b].buf_start = L.seq[b].buf_start;
+      rows[b].n_b = L.seq[b].buf_count;
+      rows[b].group_prefix = prefix;
+      prefix += row_groups(L.seq[b].sparse_len, L.seq[b].buf_count);
+    }
+    total = prefix * c->cfg.n_kv_heads;
+    if ((s = upload_rows(c, layer, rows)) != SWAN_OK) return s;
+    rows_dev = c->seq_dev + (size_t)layer * c->cfg.batch;
+  }
   int64_t range = 1, grid = 0;
   if (total > 0) {
     const int64_t ctas = std::min<int64_t>(c->decode_ctas, total);
@@ -549,13 +785,15 @@ swan_status swan_decode(swan_ctx* c, int layer, const void* q, void* out) {
     p.ring_k = c->ring_k + (size_t)layer * ring_elems_per_layer(c);
     p.ring_v = c->ring_v + (size_t)layer * ring_elems_per_layer(c);
     p.cap = c->cfg.buffer_cap > 0 ? c->cfg.buffer_cap : 1;
-    p.buf_start = L.buf_start;
-    p.n_b = L.buf_count;
-    p.sparse_len = L.sparse_len;
+    p.buf_start = q0.buf_start;
+    p.n_b = q0.buf_count;
+    p.sparse_len = q0.sparse_len;
     p.n_sg = n_sg;
     p.N_g = N_g;
     p.total_groups = total;
     p.range = range;
+    p.seq = rows_dev;
+    p.B = c->cfg.batch;
     p.H_kv = c->cfg.n_kv_heads;
     p.H_q = c->cfg.n_q_heads;
     p.blocks_per_page_log2 = __builtin_ctz((unsigned)(c->P / 32));
@@ -597,8 +835,16 @@ swan_status swan_query(const swan_ctx* c, int layer, swan_layer_info* info) {
   if (s != SWAN_OK) return s;
   if ((s = check_layer(c, layer)) != SWAN_OK) return s;
   if (!info) return fail(SWAN_ERR_INVALID_ARG, "info is NULL");
-  info->sparse_len = c->layers[layer].sparse_len;
-  info->buffer_len = c->layers[layer].buf_count;
+  const LayerState& L = c->layers[layer];
+  info->sparse_len = 0;
+  info->buffer_len = 0;
+  for (const SeqState& q : L.seq) {
+    info->sparse_len = std::max<int64_t>(info->sparse_len, q.sparse_len);
+    info->buffer_len = std::max<int64_t>(info->buffer_len, q.buf_count);
+  }
+  info->uniform = L.uniform() ? 1 : 0;
+  info->pool_pages = c->num_pages;
+  info->free_pages = c->paged ? (int64_t)c->free_pages.size() : 0;
   info->k_active = c->k_active;
   info->k_store = c->cfg.k_store;
   info->k_slots = c->k_slots;
@@ -612,42 +858,49 @@ swan_status swan_query(const swan_ctx* c, int layer, swan_layer_info* info) {
   return SWAN_OK;
 }
 
-swan_status swan_debug_export(swan_ctx* c, int layer, int what, void* host_dst, size_t bytes) {
-  swan_status s = usable(c);
-  if (s != SWAN_OK) return s;
-  if ((s = check_layer(c, layer)) != SWAN_OK) return s;
-  if (!host_dst) return fail(SWAN_ERR_INVALID_ARG, "host_dst is NULL");
+namespace {
+
+// Export the buffer or the sparse history of rows [b0, b1) of a layer (they
+// must have equal lengths), in the layouts swan_debug_export documents.
+swan_status export_rows(swan_ctx* c, int layer, int b0, int b1, int what, void* host_dst, size_t bytes) {
+  if (!host_dst && bytes) return fail(SWAN_ERR_INVALID_ARG, "host_dst is NULL");
   const LayerState& L = c->layers[layer];
+  for (int b = b0 + 1; b < b1; ++b)
+    if (!(L.seq[b] == L.seq[b0]))
+      return fail(SWAN_ERR_INVALID_ARG, "rows differ in length: export them one at a time (swan_debug_export_seq)");
+  const SeqState& q = L.seq[b0];
+  const int H = c->cfg.n_kv_heads;
+  const int64_t u0 = (int64_t)b0 * H, u1 = (int64_t)b1 * H, nu = u1 - u0;
   const int cap = c->cfg.buffer_cap;
   cudaError_t e = cudaStreamSynchronize(c->stream);
   if (e != cudaSuccess) return cuda_fail(c, e, "cudaStreamSynchronize");
 
   if (what == SWAN_EXPORT_BUFFER_K || what == SWAN_EXPORT_BUFFER_V) {
-    const size_t need = (size_t)c->units * L.buf_count * kHeadDim * 2;
+    const size_t need = (size_t)nu * q.buf_count * kHeadDim * 2;
     if (bytes != need) return fail(SWAN_ERR_INVALID_ARG, "bytes %zu != %zu", bytes, need);
     if (need == 0) return SWAN_OK;
     const __half* ring = (what == SWAN_EXPORT_BUFFER_K ? c->ring_k : c->ring_v) +
-                         (size_t)layer * ring_elems_per_layer(c);
-    std::vector<uint16_t> all((size_t)c->units * cap * kHeadDim);
+                         (size_t)layer * ring_elems_per_layer(c) + (size_t)u0 * cap * kHeadDim;
+    std::vector<uint16_t> all((size_t)nu * cap * kHeadDim);
     e = cudaMemcpy(all.data(), ring, all.size() * 2, cudaMemcpyDeviceToHost);
     if (e != cudaSuccess) return cuda_fail(c, e, "cudaMemcpy");
     uint16_t* dst = static_cast<uint16_t*>(host_dst);
-    for (int64_t u = 0; u < c->units; ++u)
-      for (int i = 0; i < L.buf_count; ++i) {
-        const int slot = (L.buf_start + i) % cap;
-        std::memcpy(dst + ((size_t)u * L.buf_count + i) * kHeadDim,
+    for (int64_t u = 0; u < nu; ++u)
+      for (int i = 0; i < q.buf_count; ++i) {
+        const int slot = (q.buf_start + i) % cap;
+        std::memcpy(dst + ((size_t)u * q.buf_count + i) * kHeadDim,
                     all.data() + ((size_t)u * cap + slot) * kHeadDim, kHeadDim * 2);
       }
     return SWAN_OK;
   }
   if (what == SWAN_EXPORT_SPARSE_K || what == SWAN_EXPORT_SPARSE_V) {
-    const bool isv_ = what == SWAN_EXPORT_SPARSE_V;
-    const int ks = isv_ ? c->k_store_v : c->cfg.k_store;
-    const size_t n_ent = (size_t)c->units * L.sparse_len * ks;
+    const bool isv = what == SWAN_EXPORT_SPARSE_V;
+    const int ks = isv ? c->k_store_v : c->cfg.k_store;
+    const int64_t Ls = q.sparse_len;
+    const size_t n_ent = (size_t)nu * Ls * ks;
     const size_t need = n_ent * 3;
     if (bytes != need) return fail(SWAN_ERR_INVALID_ARG, "bytes %zu != %zu", bytes, need);
     if (need == 0) return SWAN_OK;
-    const bool isv = what == SWAN_EXPORT_SPARSE_V;
     const bool fp8 = c->fmt == kFmtFp8;
     const int64_t P = c->P;
     const int64_t ksk = c->k_slots, ksv = c->k_slots_v;
@@ -656,15 +909,15 @@ swan_status swan_debug_export(swan_ctx* c, int layer, int what, void* host_dst, 
     // regions; fp8: 16-byte records of 8 values then 8 indices
     const int64_t voff = fp8 ? (isv ? 64 * ksk : 0) : (isv ? 96 * ksk : 0);
     const int64_t ioff = fp8 ? voff + 8 : (isv ? 96 * ksk + 64 * ksv : 64 * ksk);
-    std::vector<int32_t> pt((size_t)c->units * c->ppu);
-    e = cudaMemcpy(pt.data(), c->page_table + (int64_t)layer * c->units * c->ppu, pt.size() * 4,
+    std::vector<int32_t> pt((size_t)nu * c->ppu);
+    e = cudaMemcpy(pt.data(), c->page_table + ((int64_t)layer * c->units + u0) * c->ppu, pt.size() * 4,
                    cudaMemcpyDeviceToHost);
     if (e != cudaSuccess) return cuda_fail(c, e, "cudaMemcpy");
     uint8_t* idx_dst = static_cast<uint8_t*>(host_dst);
     uint16_t* val_dst = reinterpret_cast<uint16_t*>(idx_dst + n_ent);
     std::vector<uint8_t> page(c->page_bytes);
-    const int64_t pages_used = (L.sparse_len + P - 1) / P;
-    for (int64_t u = 0; u < c->units; ++u)
+    const int64_t pages_used = pages_for(Ls, (int)P);
+    for (int64_t u = 0; u < nu; ++u)
       for (int64_t pg = 0; pg < pages_used; ++pg) {
         const int32_t phys = pt[(size_t)u * c->ppu + pg];
         if (phys < 0 || phys >= c->num_pages) return fail(SWAN_ERR_DEVICE_CHECK, "page table corrupt");
@@ -673,18 +926,18 @@ swan_status swan_debug_export(swan_ctx* c, int layer, int what, void* host_dst, 
         if (e != cudaSuccess) return cuda_fail(c, e, "cudaMemcpy");
         for (int64_t sl = 0; sl < P; ++sl) {
           const int64_t t = pg * P + sl;
-          if (t >= L.sparse_len) break;
-          const int64_t b0 = (sl / 32) * blk;
+          if (t >= Ls) break;
+          const int64_t bo = (sl / 32) * blk;
           for (int r = 0; r < ks; ++r) {
             const int64_t rec = (int64_t)(r / 8) * 32 + (sl % 32);
-            const size_t o = ((size_t)u * L.sparse_len + t) * ks + r;
+            const size_t o = ((size_t)u * Ls + t) * ks + r;
             if (fp8) {
-              idx_dst[o] = page[b0 + ioff + rec * 16 + (r % 8)];
-              val_dst[o] = e4m3_to_half_bits(page[b0 + voff + rec * 16 + (r % 8)]);
+              idx_dst[o] = page[bo + ioff + rec * 16 + (r % 8)];
+              val_dst[o] = e4m3_to_half_bits(page[bo + voff + rec * 16 + (r % 8)]);
             } else {
-              idx_dst[o] = page[b0 + ioff + rec * 8 + (r % 8)];
+              idx_dst[o] = page[bo + ioff + rec * 8 + (r % 8)];
               uint16_t v;
-              std::memcpy(&v, page.data() + b0 + voff + rec * 16 + (r % 8) * 2, 2);
+              std::memcpy(&v, page.data() + bo + voff + rec * 16 + (r % 8) * 2, 2);
               val_dst[o] = v;
             }
           }
@@ -693,6 +946,37 @@ swan_status swan_debug_export(swan_ctx* c, int layer, int what, void* host_dst, 
     return SWAN_OK;
   }
   return fail(SWAN_ERR_INVALID_ARG, "unknown export kind %d", what);
+}
+
+}  // namespace
+
+swan_status swan_debug_export(swan_ctx* c, int layer, int what, void* host_dst, size_t bytes) {
+  swan_status s = usable(c);
+  if (s != SWAN_OK) return s;
+  if ((s = check_layer(c, layer)) != SWAN_OK) return s;
+  if (!host_dst) return fail(SWAN_ERR_INVALID_ARG, "host_dst is NULL");
+  return export_rows(c, layer, 0, c->cfg.batch, what, host_dst, bytes);
+}
+
+swan_status swan_debug_export_seq(swan_ctx* c, int layer, int b, int what, void* host_dst, size_t bytes) {
+  swan_status s = usable(c);
+  if (s != SWAN_OK) return s;
+  if ((s = check_layer(c, layer)) != SWAN_OK) return s;
+  if (b < 0 || b >= c->cfg.batch) return fail(SWAN_ERR_INVALID_ARG, "row %d out of [0, %d)", b, c->cfg.batch);
+  return export_rows(c, layer, b, b + 1, what, host_dst, bytes);
+}
+
+swan_status swan_query_lengths(const swan_ctx* c, int layer, int64_t* sparse_len, int32_t* buffer_len) {
+  swan_status s = usable(c);
+  if (s != SWAN_OK) return s;
+  if ((s = check_layer(c, layer)) != SWAN_OK) return s;
+  if (!sparse_len || !buffer_len) return fail(SWAN_ERR_INVALID_ARG, "output arrays must not be NULL");
+  const LayerState& L = c->layers[layer];
+  for (int b = 0; b < c->cfg.batch; ++b) {
+    sparse_len[b] = L.seq[b].sparse_len;
+    buffer_len[b] = L.seq[b].buf_count;
+  }
+  return SWAN_OK;
 }
 
 swan_status swan_check(swan_ctx* c) {

@@ -71,6 +71,27 @@ inline int64_t page_bytes_for(int P, int k_slots, int k_slots_v, int fmt) {
   return (int64_t)(P / 32) * (fmt == kFmtFp8 ? 64 : 96) * (k_slots + k_slots_v);
 }
 
+// Per-sequence state for batches whose sequences differ in length (one entry
+// per batch row, shared by the row's kv heads).  A kernel reads it instead of
+// the uniform scalars of its parameter block when the block's `seq` is set.
+struct SeqInfo {
+  int64_t sparse_len;    // sparse tokens (before the call; decode: current)
+  int64_t group_prefix;  // decode: 32-token groups of rows 0..b-1, per kv head
+  int32_t buf_start;     // ring slot of the oldest buffered token
+  int32_t n_b;           // buffered tokens (before the call; decode: current)
+  int32_t n_new;         // append: new tokens of this row (<= T)
+  int32_t evict;         // append: logical positions < evict go to the sparse cache
+  int32_t prune;         // prune_ring: buffered tokens 0..prune-1 are pruned
+  int32_t pad;
+};
+
+// Groups a decode walks for a row: sparse groups, then buffer groups; at
+// least one, so that an empty row still gets its (zero) output written.
+__host__ __device__ inline int64_t row_groups(int64_t sparse_len, int n_b) {
+  const int64_t g = (sparse_len + 31) / 32 + (n_b + 31) / 32;
+  return g > 0 ? g : 1;
+}
+
 // Rotate T new tokens per unit, then either write them to the ring buffer or
 // prune them straight into the sparse cache (Algorithm 1, generalised to T).
 struct AppendParams {
@@ -85,6 +106,7 @@ struct AppendParams {
   int n_b;              // buffered tokens before the append
   int64_t evict;        // logical positions < evict go to the sparse cache
   int64_t sparse_len;   // sparse tokens before the append
+  const SeqInfo* seq;   // per-row state instead of the four scalars above, or null
   CacheGeom geom;
   unsigned* status;
 };
@@ -94,8 +116,10 @@ struct AppendParams {
 struct PruneRingParams {
   const __half* ring_k;
   const __half* ring_v;
-  int units, cap, buf_start, count;
+  int units, cap, buf_start, count;  // count: the most tokens of any row
   int64_t sparse_len;
+  const SeqInfo* seq;   // per-row start, count (prune) and length, or null
+  int H;                // kv heads (row of a unit = unit / H)
   CacheGeom geom;
   unsigned* status;
 };
@@ -121,6 +145,8 @@ struct DecodeParams {
   int64_t sparse_len;
   int64_t n_sg, N_g;       // sparse groups per unit; groups per unit
   int64_t total_groups, range;
+  const SeqInfo* seq;      // per-row lengths (then the five scalars above are unused), or null
+  int B;                   // rows
   int H_kv, H_q;
   int blocks_per_page_log2; // log2(P / 32)
   int k_full_chunks;       // keys: k_active / 8
@@ -196,6 +222,8 @@ cudaError_t launch_rotate_q(const RotateQParams& p, int B, cudaStream_t s);
 cudaError_t launch_decode(const DecodeParams& p, int G, int k_read, int grid, cudaStream_t s);
 cudaError_t launch_combine(const CombineParams& p, int B, cudaStream_t s);
 cudaError_t launch_transpose_r(const float* src, float* dst, int64_t mats, cudaStream_t s);
+// table[pairs[i].x] = pairs[i].y for i < n (page-table entries of a shared pool).
+cudaError_t launch_scatter_pages(const int2* pairs, int n, int32_t* table, cudaStream_t s);
 // Decode CTAs that fit on one SM together (for the grid size).
 int decode_ctas_per_sm(int G, int k_slots);
 // Record the detail string that swan_last_error() returns on this thread.

@@ -30,7 +30,8 @@ EXPORTED = ["swan_init", "swan_destroy", "swan_set_k", "swan_append", "swan_flus
             "swan_timing_enable", "swan_timing_read", "swan_launch_count",
             "swan_status_string", "swan_last_error", "swan_decode_noalloc", "swan_set_kv",
             "swan_gram_workspace_bytes", "swan_gram", "swan_basis_eig", "swan_energy",
-            "swan_basis_check"]
+            "swan_basis_check", "swan_append_varlen", "swan_reset_sequence", "swan_query_lengths",
+            "swan_debug_export_seq"]
 
 
 class SwanConfig(ctypes.Structure):
@@ -39,7 +40,7 @@ class SwanConfig(ctypes.Structure):
                 ("head_dim", ctypes.c_int), ("k_store", ctypes.c_int),
                 ("buffer_cap", ctypes.c_int), ("max_seq", ctypes.c_int),
                 ("page_tokens", ctypes.c_int), ("stream", ctypes.c_void_p),
-                ("value_format", ctypes.c_int), ("k_store_v", ctypes.c_int)]
+                ("value_format", ctypes.c_int), ("k_store_v", ctypes.c_int), ("pool_pages", ctypes.c_int)]
 
 
 class LayerInfo(ctypes.Structure):
@@ -47,7 +48,8 @@ class LayerInfo(ctypes.Structure):
                 ("k_active", ctypes.c_int), ("k_store", ctypes.c_int), ("k_slots", ctypes.c_int),
                 ("page_tokens", ctypes.c_int), ("page_bytes", ctypes.c_int64),
                 ("device_bytes", ctypes.c_int64), ("value_format", ctypes.c_int),
-                ("k_active_v", ctypes.c_int), ("k_store_v", ctypes.c_int), ("k_slots_v", ctypes.c_int)]
+                ("k_active_v", ctypes.c_int), ("k_store_v", ctypes.c_int), ("k_slots_v", ctypes.c_int),
+                ("uniform", ctypes.c_int), ("pool_pages", ctypes.c_int64), ("free_pages", ctypes.c_int64)]
 
 
 class Timing(ctypes.Structure):
@@ -99,6 +101,10 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "swan_set_k": (i, [vp, i]),
         "swan_set_kv": (i, [vp, i, i]),
         "swan_append": (i, [vp, i, vp, vp, i]),
+        "swan_append_varlen": (i, [vp, i, vp, vp, i, ctypes.POINTER(ctypes.c_int32)]),
+        "swan_reset_sequence": (i, [vp, i]),
+        "swan_query_lengths": (i, [vp, i, ctypes.POINTER(ctypes.c_int64), ctypes.POINTER(ctypes.c_int32)]),
+        "swan_debug_export_seq": (i, [vp, i, i, i, vp, ctypes.c_size_t]),
         "swan_flush_buffer": (i, [vp, i]),
         "swan_decode": (i, [vp, i, vp, vp]),
         "swan_query": (i, [vp, i, ctypes.POINTER(LayerInfo)]),
@@ -152,7 +158,7 @@ class Context:
     def __init__(self, R_qk, R_vo=None, *, num_layers: int, batch: int, n_q_heads: int,
                  n_kv_heads: int, k_store: int, buffer_cap: int, max_seq: int,
                  page_tokens: int = 0, head_dim: int = 128, stream=None,
-                 value_format: str = "fp16", k_store_v: int = 0):
+                 value_format: str = "fp16", k_store_v: int = 0, pool_pages: int = 0):
         import torch
         self._lib = load_library()
         if stream is None:
@@ -162,7 +168,7 @@ class Context:
             raise ValueError(f"value_format must be one of {sorted(VALUE_FORMATS)}")
         self.cfg = SwanConfig(num_layers, batch, n_q_heads, n_kv_heads, head_dim, k_store,
                               buffer_cap, max_seq, page_tokens, ctypes.c_void_p(stream.cuda_stream),
-                              VALUE_FORMATS[value_format], k_store_v)
+                              VALUE_FORMATS[value_format], k_store_v, pool_pages)
         self.batch, self.n_q_heads, self.n_kv_heads = batch, n_q_heads, n_kv_heads
         self.num_layers, self.k_store, self.head_dim = num_layers, k_store, head_dim
         self.k_store_v = k_store_v or k_store
@@ -196,11 +202,28 @@ class Context:
         else:
             _check(self._lib.swan_set_kv(self._h, int(k_active), int(k_active_v)), "swan_set_kv")
 
-    def append(self, layer: int, k_new, v_new, T: int | None = None):
+    def append(self, layer: int, k_new, v_new, T: int | None = None, n_new=None):
+        """Append ``T`` tokens per row (``k_new``/``v_new`` ``[B][H][T][d]``), or
+        ``n_new[b]`` of them to row b (a host sequence of ``batch`` ints)."""
         if T is None:
             T = k_new.shape[2]
-        _check(self._lib.swan_append(self._h, int(layer), _ptr(k_new), _ptr(v_new), int(T)),
-               "swan_append")
+        if n_new is None:
+            _check(self._lib.swan_append(self._h, int(layer), _ptr(k_new), _ptr(v_new), int(T)),
+                   "swan_append")
+            return
+        counts = (ctypes.c_int32 * self.batch)(*[int(x) for x in n_new])
+        _check(self._lib.swan_append_varlen(self._h, int(layer), _ptr(k_new), _ptr(v_new), int(T), counts),
+               "swan_append_varlen")
+
+    def reset_sequence(self, b: int):
+        _check(self._lib.swan_reset_sequence(self._h, int(b)), "swan_reset_sequence")
+
+    def lengths(self, layer: int = 0):
+        """Per-row (sparse, buffered) token counts of a layer."""
+        sp = (ctypes.c_int64 * self.batch)()
+        bf = (ctypes.c_int32 * self.batch)()
+        _check(self._lib.swan_query_lengths(self._h, int(layer), sp, bf), "swan_query_lengths")
+        return list(sp), list(bf)
 
     def flush(self, layer: int = -1):
         _check(self._lib.swan_flush_buffer(self._h, int(layer)), "swan_flush_buffer")
@@ -244,6 +267,26 @@ class Context:
         idx = raw[:n].reshape(shape)
         vals = raw[n:].view(np.float16).reshape(shape)
         return idx, vals
+
+    def export_buffer_seq(self, layer: int, b: int, which: str) -> np.ndarray:
+        sp, bf = self.lengths(layer)
+        out = np.empty((self.n_kv_heads, bf[b], self.head_dim), np.float16)
+        what = EXPORT_BUFFER_K if which == "k" else EXPORT_BUFFER_V
+        _check(self._lib.swan_debug_export_seq(self._h, int(layer), int(b), what,
+                                               out.ctypes.data_as(ctypes.c_void_p), out.nbytes),
+               "swan_debug_export_seq")
+        return out
+
+    def export_sparse_seq(self, layer: int, b: int, which: str):
+        sp, bf = self.lengths(layer)
+        shape = (self.n_kv_heads, sp[b], self.k_store if which == "k" else self.k_store_v)
+        n = int(np.prod(shape))
+        raw = np.empty(max(1, n * 3), np.uint8)
+        what = EXPORT_SPARSE_K if which == "k" else EXPORT_SPARSE_V
+        _check(self._lib.swan_debug_export_seq(self._h, int(layer), int(b), what,
+                                               raw.ctypes.data_as(ctypes.c_void_p), n * 3),
+               "swan_debug_export_seq")
+        return raw[:n].reshape(shape), raw[n:n * 3].view(np.float16).reshape(shape)
 
     def timing_enable(self, on: bool = True):
         _check(self._lib.swan_timing_enable(self._h, 1 if on else 0), "swan_timing_enable")

@@ -419,3 +419,30 @@ def pin_energy_planted_rank(b):
 
 BASIS_PINS = [pin_basis_recovers_planted_svd, pin_basis_ky_fan_maximum, pin_joint_matrices_group_heads,
               pin_energy_curve_bruteforce, pin_energy_planted_rank]
+
+
+def pin_ragged_rows_are_independent(o):
+    """A batch of rows of different lengths: with equal appends the ragged
+    state machine equals the batched one bitwise, row b's outputs depend only
+    on row b's own tokens, and a reset row equals a fresh cache fed only what
+    came after the reset."""
+    R, Rv, k, v, q = _small_problem(61, B=3, H_kv=2, G=2, d=16, L=30)
+    bat = o.SwanOracle(R, Rv, batch=3, n_q_heads=4, k_store=5, buffer_cap=4)
+    rag = o.RaggedOracle(R, Rv, batch=3, n_q_heads=4, k_store=5, buffer_cap=4)
+    bat.append(k[:, :, :20], v[:, :, :20])
+    rag.append(k[:, :, :20], v[:, :, :20])
+    assert np.array_equal(bat.decode(q), rag.decode(q))
+    rag.append(k[:, :, 20:30], v[:, :, 20:30], n_new=[10, 0, 3])
+    assert rag.sparse_lens == [26, 16, 19] and rag.buffer_lens == [4, 4, 4]
+    solo = o.SwanOracle(R, Rv, batch=1, n_q_heads=4, k_store=5, buffer_cap=4)
+    solo.append(k[2:3, :, :23], v[2:3, :, :23])
+    assert np.array_equal(rag.decode(q)[2], solo.decode(q[2:3])[0])
+    rag.reset(1)
+    assert np.array_equal(rag.decode(q)[1], np.zeros((4, 16)))
+    rag.append(k[:, :, 25:30], v[:, :, 25:30], n_new=[0, 5, 0])
+    fresh = o.SwanOracle(R, Rv, batch=1, n_q_heads=4, k_store=5, buffer_cap=4)
+    fresh.append(k[1:2, :, 25:30], v[1:2, :, 25:30])
+    assert np.array_equal(rag.decode(q)[1], fresh.decode(q[1:2])[0])
+
+
+ALL_PINS.append(pin_ragged_rows_are_independent)

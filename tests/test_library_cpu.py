@@ -46,7 +46,7 @@ def test_status_strings(lib):
 
 def _cfg(**kw):
     base = dict(num_layers=1, batch=1, n_q_heads=1, n_kv_heads=1, head_dim=128, k_store=64,
-                buffer_cap=64, max_seq=1024, page_tokens=0, stream=None, value_format=0, k_store_v=0)
+                buffer_cap=64, max_seq=1024, page_tokens=0, stream=None, value_format=0, k_store_v=0, pool_pages=0)
     base.update(kw)
     return swan.SwanConfig(*[base[f] for f, _ in swan.SwanConfig._fields_])
 
@@ -70,6 +70,7 @@ def _cfg(**kw):
     (dict(value_format=-1), swan.ERR_INVALID_ARG),
     (dict(k_store_v=129), swan.ERR_INVALID_ARG),
     (dict(k_store_v=-2), swan.ERR_INVALID_ARG),
+    (dict(pool_pages=-1), swan.ERR_INVALID_ARG),
 ])
 def test_init_rejects_bad_config_without_cuda(lib, kw, status):
     h = ctypes.c_void_p(123)
@@ -87,6 +88,10 @@ def test_null_arguments(lib):
     assert lib.swan_init(ctypes.byref(h), ctypes.byref(cfg), None, None) == swan.ERR_INVALID_ARG
     assert lib.swan_set_k(None, 4) == swan.ERR_INVALID_ARG
     assert lib.swan_set_kv(None, 4, 4) == swan.ERR_INVALID_ARG
+    assert lib.swan_reset_sequence(None, 0) == swan.ERR_INVALID_ARG
+    assert lib.swan_append_varlen(None, 0, None, None, 1, None) == swan.ERR_INVALID_ARG
+    assert lib.swan_query_lengths(None, 0, None, None) == swan.ERR_INVALID_ARG
+    assert lib.swan_debug_export_seq(None, 0, 0, 1, None, 0) == swan.ERR_INVALID_ARG
     assert lib.swan_append(None, 0, None, None, 1) == swan.ERR_INVALID_ARG
     assert lib.swan_decode(None, 0, None, None) == swan.ERR_INVALID_ARG
     assert lib.swan_flush_buffer(None, 0) == swan.ERR_INVALID_ARG

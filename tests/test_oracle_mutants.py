@@ -69,6 +69,8 @@ MUTANTS = [
      "e = np.maximum(e, -6.0)", "e = np.maximum(e, -30.0)", 1),
     ("fp8_values_not_rounded",
      "vals = to_e4m3(vals.astype(np.float64)).astype(np.float16)", "vals = vals", 1),
+    ("ragged_append_ignores_counts",
+     "n = T if n_new is None else int(n_new[b])", "n = T", 1),
     ("runtime_k_ignored",
      "s_sp = sparse_scores(q_hat, sp_idx[:, :ka], sp_vals_k[:, :ka])",
      "s_sp = sparse_scores(q_hat, sp_idx, sp_vals_k)", 1),

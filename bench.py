@@ -55,6 +55,12 @@ WORKLOADS = {
                         desc="32-layer Llama-2-7B-shaped KV stack, batch 8, 8192-token prefix "
                              "compressed by one append per layer, decode steps appending one token "
                              "per layer, buffers flushed every 128 steps, k 64"),
+    "ragged-serve-32": dict(kind="ragged", B=32, H_q=32, H_kv=32, n_b=128, k=64, k_store=64,
+                            len_lo=1024, len_hi=65536, P=128, L_s=8192,
+                            desc="serving batch of 32 Llama-2-7B-shaped sequences (32 MHA heads, d 128) "
+                                 "whose contexts are drawn log-uniformly from 1024 to 65536 tokens (seeded), "
+                                 "k 64, 128-token buffers; the pages come from one shared pool sized to "
+                                 "the contexts (not to 32 x the longest)"),
     "basis-llama3-8b": dict(kind="basis", n_kv=8, G=4, n=65536, d_model=4096,
                             desc="offline basis (Section 4.1) for one Llama-3-8B-shaped layer: 32 q / 8 kv "
                                  "heads, d 128, d_model 4096; one step accumulates S_QK^T S_QK and "
@@ -498,6 +504,64 @@ class LayerRun:
         return [self.out]
 
 
+class RaggedRun(LayerRun):
+    """A batch of sequences of different lengths sharing one page pool:
+    prefilled in 2048-token chunks with per-row counts, then per step one
+    token appended to every row and one decode."""
+
+    def __init__(self, wl, dev, stream, seed, steps_total):
+        import torch
+
+        from paper_2511_18936_gb300 import swan, synth
+        self.wl = wl
+        B, H_q, H_kv, n_b, P = wl["B"], wl["H_q"], wl["H_kv"], wl["n_b"], wl["P"]
+        gen = np.random.default_rng(synth.seed_seq(seed, 6, 0, 0))
+        lo, hi = np.log(wl["len_lo"]), np.log(wl["len_hi"])
+        self.lens = [int(x) for x in np.exp(gen.uniform(lo, hi, size=B)).round()]
+        self.layers = 1
+        self.max_seq = max(self.lens) + steps_total + 8
+        sparse_max = [max(0, L + steps_total - n_b) for L in self.lens]
+        pool = H_kv * sum((s + P - 1) // P for s in sparse_max) + B * H_kv
+        self.pool_pages = pool
+        with torch.cuda.stream(stream):
+            R = torch.from_numpy(synth.rotations(H_kv, D, seed=seed, workload=1, layer=0))[None].to(dev)
+            self.ctx = swan.Context(R, num_layers=1, batch=B, n_q_heads=H_q, n_kv_heads=H_kv,
+                                    k_store=wl["k_store"], buffer_cap=n_b, max_seq=self.max_seq, page_tokens=P,
+                                    stream=stream, value_format=wl["values"], k_store_v=wl["k_store_v"],
+                                    pool_pages=pool)
+            chunk = 2048
+            for ci, t0 in enumerate(range(0, max(self.lens), chunk)):
+                n_new = [max(0, min(chunk, L - t0)) for L in self.lens]
+                kk = synth.torch_lowrank_kv(B, H_kv, chunk, D, seed * 1000 + ci, synth.T_K, dev)
+                vv = synth.torch_lowrank_kv(B, H_kv, chunk, D, seed * 1000 + ci, synth.T_V, dev)
+                self.ctx.append(0, kk, vv, chunk, n_new=n_new)
+                del kk, vv
+            k_new = synth.torch_lowrank_kv(B, H_kv, steps_total, D, seed, synth.T_NEWK, dev)
+            v_new = synth.torch_lowrank_kv(B, H_kv, steps_total, D, seed, synth.T_NEWV, dev)
+            self.k_steps = [k_new[:, :, i:i + 1].contiguous() for i in range(steps_total)]
+            self.v_steps = [v_new[:, :, i:i + 1].contiguous() for i in range(steps_total)]
+            del k_new, v_new
+            self.qs = synth.torch_gaussian_fp16((steps_total, B, H_q, D), seed, synth.T_Q, dev)
+            self.out = torch.empty((B, H_q, D), dtype=torch.float16, device=dev)
+            self.ctx.set_k(wl["k"], wl["k_v"])
+        stream.synchronize()
+        self.ctx.check()
+        self.page_bytes = self.ctx.query(0).page_bytes
+
+    def rows_after(self, i):
+        """Per-row (sparse, buffer) tokens attended by the decode of step i."""
+        n_b = self.wl["n_b"]
+        out = []
+        for L in self.lens:
+            tot = L + i + 1
+            out.append((max(0, tot - n_b), min(tot, n_b)))
+        return out
+
+    def context_after(self, i):
+        rows = self.rows_after(i)
+        return (sum(sp for sp, _ in rows) / len(rows), sum(bf for _, bf in rows) / len(rows))
+
+
 class StackRun:
     """A 32-layer KV stack: the prefix of every layer compressed by one
     append (timed separately), flushed, then decode steps that append one
@@ -585,7 +649,7 @@ def run_swan(args, wl, rank: int, world: int, local_rank: int):
     kind = wl.get("kind", "layer")
     if kind == "stack" and steps_total > wl["max_steps"]:
         raise SystemExit(f"the stack workload runs at most {wl['max_steps']} decode steps")
-    run = (StackRun if kind == "stack" else LayerRun)(wl, dev, stream, seed, steps_total)
+    run = {"stack": StackRun, "ragged": RaggedRun}.get(kind, LayerRun)(wl, dev, stream, seed, steps_total)
     ctx = run.ctx
     flush_l2 = wl.get("l2_flush", False)
     l2_buf = torch.empty(512 * 1024 * 1024 // 4, dtype=torch.float32, device=dev) if flush_l2 else None
@@ -709,6 +773,12 @@ def run_swan(args, wl, rank: int, world: int, local_rank: int):
                       + " values + uint8 indices (sparse), fp16 (buffer)", "l2": l2_note,
            "parallelism": f"replicas x{world} (independent batches per GPU)" if world > 1
            else "single GPU"}
+    if kind == "ragged":
+        pb = run.page_bytes
+        cfg["sparse_tokens"] = None
+        cfg["context_lengths"] = {"min": min(run.lens), "mean": statistics.mean(run.lens), "max": max(run.lens)}
+        cfg["pool_gb"] = run.pool_pages * pb / 1e9
+        cfg["full_reservation_gb"] = B * H_kv * ((run.max_seq + wl["P"] - 1) // wl["P"]) * pb / 1e9
     line = {
         "metric": METRIC, "value": value, "unit": "KV-tokens/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": t_max / args.steps,

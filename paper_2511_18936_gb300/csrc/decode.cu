@@ -244,18 +244,70 @@ __device__ __forceinline__ int64_t unit_of(const DecodeParams& p, int64_t g) {
   const int64_t h = min((int64_t)p.H_kv - 1, (g - q.group_prefix * p.H_kv) / ng);
   return (int64_t)lo * p.H_kv + h;
 }
+// Split of a segment [s0, s1) of a unit's groups (the first n_sg sparse,
+// the rest dense-buffer groups, which cost about kBufferGroupCost sparse
+// groups) into `parts` contiguous runs of equal cost; returns where run
+// `part` starts (part == parts gives s1).
+constexpr int kBufferGroupCost = 2;
+__device__ __forceinline__ int split_at(int s0, int s1, int n_sg, int part, int parts) {
+  const int sp_in = max(0, min(s1, n_sg) - s0);
+  const int bf_in = (s1 - s0) - sp_in;
+  const int cost = sp_in + kBufferGroupCost * bf_in;
+  const int c = (int)(((int64_t)cost * part) / parts);
+  return c <= sp_in ? s0 + c : s0 + sp_in + (c - sp_in + kBufferGroupCost - 1) / kBufferGroupCost;
+}
+
+// First group of CTA c (c <= gridDim.x) and the CTA that holds group g.
+__device__ __forceinline__ int64_t cta_begin(const DecodeParams& p, int64_t c) {
+  if (p.cta_start == nullptr) return min(p.total_groups, c * p.range);
+  return p.cta_start[c];
+}
+__device__ __forceinline__ int64_t cta_of(const DecodeParams& p, int64_t g) {
+  if (p.cta_start == nullptr) return g / p.range;
+  int lo = 0, hi = (int)gridDim.x - 1;  // the last CTA whose first group is <= g
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (p.cta_start[mid] <= g) lo = mid;
+    else hi = mid - 1;
+  }
+  return lo;
+}
 
 // The last CTA to finish a segment of unit u merges the unit's partials,
 // normalises, rotates back (o = o_hat R_vo^T) and writes the output.  The
 // arrival counter resets itself for the next decode; nothing waits.
 // `scratch` holds G * 128 floats (free at this point); `flag` one float.
+// out = o_hat R_vo^T for the G query heads of unit (b, h); o_hat in shared
+// memory [G][128].
 template <int G, int NT>
-__device__ __forceinline__ void finish_unit(const DecodeParams& p, const UnitView& uv, int64_t u, int64_t b,
-                                            int64_t h,
-                                            float* scratch, float* flag) {
+__device__ __forceinline__ void rotate_back_out(const DecodeParams& p, int64_t b, int64_t h, const float* o_hat) {
+  const float* RT = p.R_voT + (size_t)h * kHeadDim * kHeadDim;
+  for (int o = threadIdx.x; o < G * kHeadDim; o += NT) {
+    const int gh = o / kHeadDim, i = o % kHeadDim;
+    const float* oh = o_hat + gh * kHeadDim;
+    float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
+#pragma unroll 8
+    for (int j = 0; j < kHeadDim; j += 4) {
+      a0 = fmaf(oh[j + 0], __ldg(RT + (j + 0) * kHeadDim + i), a0);
+      a1 = fmaf(oh[j + 1], __ldg(RT + (j + 1) * kHeadDim + i), a1);
+      a2 = fmaf(oh[j + 2], __ldg(RT + (j + 2) * kHeadDim + i), a2);
+      a3 = fmaf(oh[j + 3], __ldg(RT + (j + 3) * kHeadDim + i), a3);
+    }
+    p.out[((b * p.H_q) + h * G + gh) * kHeadDim + i] = __float2half_rn((a0 + a1) + (a2 + a3));
+  }
+}
+
+// The last CTA to finish a segment of unit u merges the unit's partials,
+// normalises, rotates back (o = o_hat R_vo^T) and writes the output.  The
+// arrival counter resets itself for the next decode; nothing waits.
+// `scratch` holds G * 128 floats (free at this point); `flag` one float.
+// (A unit that one CTA holds entirely never comes here: it is finished from
+// shared memory by that CTA.)
+template <int G, int NT>
+__device__ __forceinline__ void finish_unit(const DecodeParams& p, int64_t c0, int64_t c1, int64_t u, int64_t b,
+                                            int64_t h, float* scratch, float* flag) {
   __threadfence();
   __syncthreads();
-  const int64_t c0 = uv.goff / p.range, c1 = (uv.goff + uv.N_g - 1) / p.range;
   if (threadIdx.x == 0) {
     const int old = atomicAdd(p.counters + u, 1);
     const bool last = old == (int)(c1 - c0);
@@ -282,20 +334,7 @@ __device__ __forceinline__ void finish_unit(const DecodeParams& p, const UnitVie
     o_hat[o] = (L > 0.f) ? A / L : 0.f;
   }
   __syncthreads();
-  const float* RT = p.R_voT + (size_t)h * kHeadDim * kHeadDim;
-  for (int o = threadIdx.x; o < G * kHeadDim; o += NT) {
-    const int gh = o / kHeadDim, i = o % kHeadDim;
-    const float* oh = o_hat + gh * kHeadDim;
-    float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
-#pragma unroll 8
-    for (int j = 0; j < kHeadDim; j += 4) {
-      a0 = fmaf(oh[j + 0], __ldg(RT + (j + 0) * kHeadDim + i), a0);
-      a1 = fmaf(oh[j + 1], __ldg(RT + (j + 1) * kHeadDim + i), a1);
-      a2 = fmaf(oh[j + 2], __ldg(RT + (j + 2) * kHeadDim + i), a2);
-      a3 = fmaf(oh[j + 3], __ldg(RT + (j + 3) * kHeadDim + i), a3);
-    }
-    p.out[((b * p.H_q) + h * G + gh) * kHeadDim + i] = __float2half_rn((a0 + a1) + (a2 + a3));
-  }
+  rotate_back_out<G, NT>(p, b, h, o_hat);
 }
 
 // Warps per CTA of the one-head kernel: as many lane-private accumulators as
@@ -339,8 +378,8 @@ __global__ void __launch_bounds__(decode_warps<MAXC>() * 32, 1) decode_kernel(De
   const bool whole_block = nchunks * 8 == g.k_slots && nchunks_v * 8 == g.k_slots_v;
   const int bsh = p.blocks_per_page_log2, bmask = (1 << bsh) - 1;
 
-  const int64_t g_begin = (int64_t)blockIdx.x * p.range;
-  const int64_t g_end = min(p.total_groups, g_begin + p.range);
+  const int64_t g_begin = cta_begin(p, blockIdx.x);
+  const int64_t g_end = min(p.total_groups, cta_begin(p, blockIdx.x + 1));
   pdl_wait();
   if (g_begin >= g_end) return;
   const int64_t u_first = unit_of(p, g_begin), u_last = unit_of(p, g_end - 1);
@@ -352,9 +391,8 @@ __global__ void __launch_bounds__(decode_warps<MAXC>() * 32, 1) decode_kernel(De
     const int s1 = (int)(min(g_end, uv.goff + uv.N_g) - uv.goff);
     const int64_t b = u / p.H_kv, h = u % p.H_kv;
     // this warp's contiguous run of groups [t_lo, t_hi)
-    const int len = s1 - s0;
-    const int t_lo = s0 + (len * warp) / NW;
-    const int t_hi = s0 + (len * (warp + 1)) / NW;
+    const int t_lo = split_at(s0, s1, n_sg, warp, NW);
+    const int t_hi = split_at(s0, s1, n_sg, warp + 1, NW);
     const int sp_hi = min(t_hi, n_sg);  // sparse groups of the run: [t_lo, sp_hi)
     const int32_t* ptab = g.page_table + u * g.pages_per_unit;
 
@@ -544,6 +582,8 @@ __global__ void __launch_bounds__(decode_warps<MAXC>() * 32, 1) decode_kernel(De
       red_l[warp] = l_sum;
     }
     __syncthreads();
+    const int64_t c0 = cta_of(p, uv.goff), c1 = cta_of(p, uv.goff + uv.N_g - 1);
+    const bool solo = c0 == c1;  // this CTA holds the whole unit
     for (int dd = threadIdx.x; dd < kHeadDim; dd += NT) {
       float M = -INFINITY;
 #pragma unroll
@@ -560,6 +600,10 @@ __global__ void __launch_bounds__(decode_warps<MAXC>() * 32, 1) decode_kernel(De
         tot = fmaf(f, sum, tot);
         L = fmaf(f, red_l[w], L);
       }
+      if (solo) {
+        qrep[dd] = (L > 0.f) ? tot / L : 0.f;  // q' is no longer needed
+        continue;
+      }
       float* dst = p.partials + ((size_t)(blockIdx.x + u)) * (kHeadDim + 2);
       dst[2 + dd] = tot;
       if (dd == 0) {
@@ -567,7 +611,12 @@ __global__ void __launch_bounds__(decode_warps<MAXC>() * 32, 1) decode_kernel(De
         dst[1] = L;
       }
     }
-    finish_unit<1, NT>(p, uv, u, b, h, qrep, red_m);
+    if (solo) {
+      __syncthreads();
+      rotate_back_out<1, NT>(p, b, h, qrep);
+    } else {
+      finish_unit<1, NT>(p, c0, c1, u, b, h, qrep, red_m);
+    }
   }
 }
 
@@ -686,8 +735,8 @@ __global__ void __launch_bounds__(kGqaWarps * 32, 1) decode_gqa_kernel(DecodePar
   const bool whole_block = nchunks * 8 == g.k_slots && nchunks_v * 8 == g.k_slots_v;
   const int bsh = p.blocks_per_page_log2, bmask = (1 << bsh) - 1;
 
-  const int64_t g_begin = (int64_t)blockIdx.x * p.range;
-  const int64_t g_end = min(p.total_groups, g_begin + p.range);
+  const int64_t g_begin = cta_begin(p, blockIdx.x);
+  const int64_t g_end = min(p.total_groups, cta_begin(p, blockIdx.x + 1));
   pdl_wait();
   if (g_begin >= g_end) return;
   const int64_t u_first = unit_of(p, g_begin), u_last = unit_of(p, g_end - 1);
@@ -699,9 +748,9 @@ __global__ void __launch_bounds__(kGqaWarps * 32, 1) decode_gqa_kernel(DecodePar
     const int s1 = (int)(min(g_end, uv.goff + uv.N_g) - uv.goff);
     const int64_t b = u / p.H_kv, h = u % p.H_kv;
     // this warp's contiguous run of items (half-blocks for G = 4)
-    const int items = (s1 - s0) * HALVES;
-    const int i_lo = s0 * HALVES + (items * warp) / NW;
-    const int i_hi = s0 * HALVES + (items * (warp + 1)) / NW;
+    // items are half-blocks (G = 4) or blocks (G = 2): split like groups
+    const int i_lo = split_at(s0 * HALVES, s1 * HALVES, n_sg * HALVES, warp, NW);
+    const int i_hi = split_at(s0 * HALVES, s1 * HALVES, n_sg * HALVES, warp + 1, NW);
     const int32_t* ptab = g.page_table + u * g.pages_per_unit;
 
     __syncthreads();  // the previous segment is done with shared memory
@@ -918,6 +967,8 @@ __global__ void __launch_bounds__(kGqaWarps * 32, 1) decode_gqa_kernel(DecodePar
       red_l[warp * G + 2 * hg + 1] = l1;
     }
     __syncthreads();
+    const int64_t c0 = cta_of(p, uv.goff), c1 = cta_of(p, uv.goff + uv.N_g - 1);
+    const bool solo = c0 == c1;  // this CTA holds the whole unit
     for (int o = threadIdx.x; o < G * kHeadDim; o += NT) {
       const int hd = o / kHeadDim, dd = o % kHeadDim;
       const int grp = hd >> 1, j = hd & 1;
@@ -936,6 +987,10 @@ __global__ void __launch_bounds__(kGqaWarps * 32, 1) decode_gqa_kernel(DecodePar
         tot = fmaf(f, sum, tot);
         L = fmaf(f, red_l[w * G + hd], L);
       }
+      if (solo) {
+        qrep[o] = (L > 0.f) ? tot / L : 0.f;  // q' is no longer needed
+        continue;
+      }
       float* dst = p.partials + ((size_t)(blockIdx.x + u) * G + hd) * (kHeadDim + 2);
       dst[2 + dd] = tot;
       if (dd == 0) {
@@ -943,7 +998,12 @@ __global__ void __launch_bounds__(kGqaWarps * 32, 1) decode_gqa_kernel(DecodePar
         dst[1] = L;
       }
     }
-    finish_unit<G, NT>(p, uv, u, b, h, qrep, flag);
+    if (solo) {
+      __syncthreads();
+      rotate_back_out<G, NT>(p, b, h, qrep);
+    } else {
+      finish_unit<G, NT>(p, c0, c1, u, b, h, qrep, flag);
+    }
   }
 }
 

@@ -91,7 +91,8 @@ struct swan_ctx {
   float* partials = nullptr;
   int* counters = nullptr;  // per-unit arrival counters of the fused combine
   unsigned* status = nullptr;
-  SeqInfo* seq_dev = nullptr;  // [layers][batch] per-row lengths for ragged calls
+  uint8_t* seq_dev = nullptr;  // per layer: [batch] SeqInfo, then [decode_ctas + 1] CTA starts
+  size_t seq_stride = 0;       // bytes per layer of seq_dev
   int2* pt_pairs = nullptr;    // paged: (entry, page) updates of one call
   int64_t device_bytes = 0;
 
@@ -287,13 +288,55 @@ swan_status grow_pages(swan_ctx* c, int layer, const std::vector<int64_t>& new_l
                 [&] { return launch_scatter_pages(c->pt_pairs, (int)pairs.size(), table, c->stream); });
 }
 
-// Upload a layer's per-row table for the next ragged launch (ordered on the
-// stream; the host vector may be reused once this returns).
-swan_status upload_rows(swan_ctx* c, int layer, const std::vector<SeqInfo>& rows) {
-  cudaError_t e = cudaMemcpyAsync(c->seq_dev + (size_t)layer * c->cfg.batch, rows.data(),
-                                  rows.size() * sizeof(SeqInfo), cudaMemcpyHostToDevice, c->stream);
+SeqInfo* rows_of(swan_ctx* c, int layer) {
+  return reinterpret_cast<SeqInfo*>(c->seq_dev + (size_t)layer * c->seq_stride);
+}
+int64_t* cta_starts_of(swan_ctx* c, int layer) {
+  return reinterpret_cast<int64_t*>(c->seq_dev + (size_t)layer * c->seq_stride + (size_t)c->cfg.batch * sizeof(SeqInfo));
+}
+
+// Upload a layer's per-row table (and, for a decode, the CTA starts right
+// after it) for the next ragged launch: one copy, ordered on the stream; the
+// host vectors may be reused once this returns.
+swan_status upload_rows(swan_ctx* c, int layer, const std::vector<SeqInfo>& rows,
+                        const std::vector<int64_t>* starts = nullptr) {
+  std::vector<uint8_t> buf(rows.size() * sizeof(SeqInfo) + (starts ? starts->size() * sizeof(int64_t) : 0));
+  std::memcpy(buf.data(), rows.data(), rows.size() * sizeof(SeqInfo));
+  if (starts) std::memcpy(buf.data() + rows.size() * sizeof(SeqInfo), starts->data(), starts->size() * sizeof(int64_t));
+  cudaError_t e = cudaMemcpyAsync(rows_of(c, layer), buf.data(), buf.size(), cudaMemcpyHostToDevice, c->stream);
   if (e != cudaSuccess) return cuda_fail(c, e, "uploading per-row lengths");
   return SWAN_OK;
+}
+
+// Work of one unit segment of a decode CTA beyond its groups (staging q',
+// the merge, the rotate-back), in 32-token groups.
+constexpr int64_t kSegmentCostGroups = 12;
+
+// First group of each decode CTA for ragged rows: contiguous ranges of equal
+// cost, a unit costing its groups plus kSegmentCostGroups for every CTA it
+// is processed by, so that CTAs covering many short rows take fewer groups.
+std::vector<int64_t> balanced_starts(const std::vector<int64_t>& row_groups, int H, int64_t max_ctas) {
+  int64_t total = 0;
+  for (int64_t g : row_groups) total += g * H;
+  const int64_t units = (int64_t)row_groups.size() * H;
+  const int64_t ctas = std::max<int64_t>(1, std::min<int64_t>(max_ctas, total));
+  const double target = ((double)total + (double)kSegmentCostGroups * units) / (double)ctas;
+  std::vector<int64_t> starts{0};
+  int64_t next = 1, goff = 0, u = 0;
+  for (int64_t ng : row_groups)
+    for (int h = 0; h < H; ++h, ++u) {
+      // group goff + j costs base + j so far (this unit's overhead included)
+      const double base = (double)goff + (double)kSegmentCostGroups * (double)(u + 1);
+      while (next < ctas && (double)next * target <= base + (double)(ng - 1)) {
+        const int64_t j = std::max<int64_t>(0, (int64_t)std::ceil((double)next * target - base));
+        const int64_t g = goff + j;
+        if (g > starts.back() && g < total) starts.push_back(g);
+        ++next;
+      }
+      goff += ng;
+    }
+  starts.push_back(total);
+  return starts;
 }
 
 // Prune buffered tokens 0..count[b]-1 of every row b of a layer into the
@@ -333,7 +376,7 @@ swan_status prune_from_ring(swan_ctx* c, int layer, const std::vector<int>& coun
       rows[b].prune = count[b];
     }
     if ((s = upload_rows(c, layer, rows)) != SWAN_OK) return s;
-    p.seq = c->seq_dev + (size_t)layer * B;
+    p.seq = rows_of(c, layer);
   }
   s = launch(c, SWAN_KERNEL_PRUNE, "prune_ring kernel", [&] { return launch_prune_ring(p, c->stream); });
   if (s != SWAN_OK) return s;
@@ -470,8 +513,9 @@ swan_status swan_init(swan_ctx** out, const swan_config* cfg, const float* R_qk,
   if (s == SWAN_OK) s = dev_alloc(c, (void**)&c->partials, part_elems * sizeof(float), "split partials");
   if (s == SWAN_OK) s = dev_alloc(c, (void**)&c->counters, (size_t)c->units * sizeof(int), "counters");
   if (s == SWAN_OK) s = dev_alloc(c, (void**)&c->status, sizeof(unsigned), "status word");
+  c->seq_stride = ((size_t)C.batch * sizeof(SeqInfo) + ((size_t)c->decode_ctas + 1) * sizeof(int64_t) + 255) / 256 * 256;
   if (s == SWAN_OK)
-    s = dev_alloc(c, (void**)&c->seq_dev, (size_t)C.num_layers * C.batch * sizeof(SeqInfo), "per-row lengths");
+    s = dev_alloc(c, (void**)&c->seq_dev, (size_t)C.num_layers * c->seq_stride, "per-row lengths");
   if (s == SWAN_OK && c->paged)
     s = dev_alloc(c, (void**)&c->pt_pairs, (size_t)c->units * c->ppu * sizeof(int2), "page-table updates");
   if (s != SWAN_OK) {
@@ -610,7 +654,7 @@ swan_status append_rows(swan_ctx* c, int layer, const void* k_new, const void* v
       rows[b].prune = old_evict[b];
     }
     if ((s = upload_rows(c, layer, rows)) != SWAN_OK) return s;
-    rows_dev = c->seq_dev + (size_t)layer * B;
+    rows_dev = rows_of(c, layer);
   }
 
   // 1) prune the evicted buffered tokens (they leave the ring first, so the
@@ -757,8 +801,11 @@ swan_status swan_decode(swan_ctx* c, int layer, const void* q, void* out) {
   const int64_t N_g = n_sg + n_bg;
   int64_t total = c->units * N_g;
   const SeqInfo* rows_dev = nullptr;
+  const int64_t* starts_dev = nullptr;
+  int64_t ragged_grid = 0;
   if (!same) {
     std::vector<SeqInfo> rows(c->cfg.batch);
+    std::vector<int64_t> groups(c->cfg.batch);
     int64_t prefix = 0;
     for (int b = 0; b < c->cfg.batch; ++b) {
       rows[b] = SeqInfo{};
@@ -766,17 +813,21 @@ swan_status swan_decode(swan_ctx* c, int layer, const void* q, void* out) {
       rows[b].buf_start = L.seq[b].buf_start;
       rows[b].n_b = L.seq[b].buf_count;
       rows[b].group_prefix = prefix;
-      prefix += row_groups(L.seq[b].sparse_len, L.seq[b].buf_count);
+      groups[b] = row_groups(L.seq[b].sparse_len, L.seq[b].buf_count);
+      prefix += groups[b];
     }
     total = prefix * c->cfg.n_kv_heads;
-    if ((s = upload_rows(c, layer, rows)) != SWAN_OK) return s;
-    rows_dev = c->seq_dev + (size_t)layer * c->cfg.batch;
+    const std::vector<int64_t> starts = balanced_starts(groups, c->cfg.n_kv_heads, c->decode_ctas);
+    ragged_grid = (int64_t)starts.size() - 1;
+    if ((s = upload_rows(c, layer, rows, &starts)) != SWAN_OK) return s;
+    rows_dev = rows_of(c, layer);
+    starts_dev = cta_starts_of(c, layer);
   }
   int64_t range = 1, grid = 0;
   if (total > 0) {
     const int64_t ctas = std::min<int64_t>(c->decode_ctas, total);
     range = (total + ctas - 1) / ctas;
-    grid = (total + range - 1) / range;
+    grid = starts_dev ? ragged_grid : (total + range - 1) / range;
   }
   if (grid > 0) {
     DecodeParams p{};
@@ -793,6 +844,7 @@ swan_status swan_decode(swan_ctx* c, int layer, const void* q, void* out) {
     p.total_groups = total;
     p.range = range;
     p.seq = rows_dev;
+    p.cta_start = starts_dev;
     p.B = c->cfg.batch;
     p.H_kv = c->cfg.n_kv_heads;
     p.H_q = c->cfg.n_q_heads;

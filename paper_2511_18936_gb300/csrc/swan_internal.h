@@ -146,6 +146,7 @@ struct DecodeParams {
   int64_t n_sg, N_g;       // sparse groups per unit; groups per unit
   int64_t total_groups, range;
   const SeqInfo* seq;      // per-row lengths (then the five scalars above are unused), or null
+  const int64_t* cta_start;  // [grid + 1] first group of each CTA (cost-balanced), or null: c * range
   int B;                   // rows
   int H_kv, H_q;
   int blocks_per_page_log2; // log2(P / 32)

@@ -246,9 +246,11 @@ __device__ __forceinline__ int64_t unit_of(const DecodeParams& p, int64_t g) {
 }
 // Split of a segment [s0, s1) of a unit's groups (the first n_sg sparse,
 // the rest dense-buffer groups, which cost about kBufferGroupCost sparse
-// groups) into `parts` contiguous runs of equal cost; returns where run
+// groups: 512 instead of 384 bytes and twice the shared-memory work per
+// token, set by measurement) into `parts` contiguous runs of equal cost;
+// returns where run
 // `part` starts (part == parts gives s1).
-constexpr int kBufferGroupCost = 2;
+constexpr int kBufferGroupCost = 3;
 __device__ __forceinline__ int split_at(int s0, int s1, int n_sg, int part, int parts) {
   const int sp_in = max(0, min(s1, n_sg) - s0);
   const int bf_in = (s1 - s0) - sp_in;

@@ -1009,6 +1009,397 @@ __global__ void __launch_bounds__(kGqaWarps * 32, 1) decode_gqa_kernel(DecodePar
   }
 }
 
+// ---------------------------------------------------------------------------
+// Grouped-query heads with the value product on the tensor cores (G = 2, 4).
+//   Lane = token, as in the one-head kernel; each lane scores its token for
+//   all G query heads of the kv head from q' replicated per lane
+//   ([128][32][G] fp32: one 8- or 16-byte conflict-free gather per entry).
+//   The value product o_h += sum_t p_h(t) v_t is dense once the kept
+//   entries are scattered into a zero-filled [32 tokens][128] fp16 tile per
+//   warp, so it runs as mma.sync.m16n8k16 (rows = the G heads, k = the 32
+//   tokens, n = the 128 coordinates) with the fp32 accumulators in
+//   registers; p is split into fp16 hi + lo parts (two products), so the
+//   result keeps fp32 accuracy.  No per-warp shared accumulator: the tile
+//   and a [G][32] p table are all a warp holds in shared memory.
+// ---------------------------------------------------------------------------
+constexpr int kMmaWarps = 8;
+constexpr int kVRowBytes = 272;                      // 128 fp16 + 16 B pad: conflict-free ldmatrix rows
+constexpr uint32_t kVTileBytes = 32 * kVRowBytes;    // 8704
+constexpr uint32_t kPTileBytes = 4 * 32 * 4;         // p [<= 4 heads][32 tokens] fp32
+constexpr uint32_t kMmaWarpBytes = kVTileBytes + kPTileBytes;
+template <int G>
+__host__ __device__ constexpr size_t mma_smem() {
+  return (size_t)kHeadDim * 32 * G * 4 + (size_t)kMmaWarps * kMmaWarpBytes + 16;
+}
+
+__device__ __forceinline__ float4 lds4(uint32_t a) {
+  float4 v;
+  asm volatile("ld.shared.v4.f32 {%0,%1,%2,%3}, [%4];" : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w) : "r"(a));
+  return v;
+}
+// Tile accesses carry a memory clobber: they alias the C++ accesses to the
+// same tile (the p table, the o rows of the merge).
+__device__ __forceinline__ void sts_u16(uint32_t a, uint32_t v) {
+  asm volatile("st.shared.u16 [%0], %1;" ::"r"(a), "h"((unsigned short)v) : "memory");
+}
+__device__ __forceinline__ void sts_v4(uint32_t a, uint4 v) {
+  asm volatile("st.shared.v4.u32 [%0], {%1,%2,%3,%4};" ::"r"(a), "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w)
+               : "memory");
+}
+__device__ __forceinline__ void ldsm_x4_trans(uint32_t a, uint32_t (&r)[4]) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+               : "r"(a)
+               : "memory");
+}
+// d[0..1] += A (16 x 16, rows g and g + 8) * B (16 x 8); the rows g + 8 of A
+// are zero, so their accumulators are dropped.
+__device__ __forceinline__ void mma_16816(float (&d)[2], uint32_t a0, uint32_t a2, uint32_t b0, uint32_t b1) {
+  float x2, x3;
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+      "{%10,%11,%12,%13};"
+      : "=f"(d[0]), "=f"(d[1]), "=f"(x2), "=f"(x3)
+      : "r"(a0), "r"(0u), "r"(a2), "r"(0u), "r"(b0), "r"(b1), "f"(d[0]), "f"(d[1]), "f"(0.f), "f"(0.f));
+}
+// Two fp32 values as (hi, lo) fp16 pairs: x = hi + lo to ~2^-22 relative.
+__device__ __forceinline__ void split_pair(float x0, float x1, uint32_t& hi, uint32_t& lo) {
+  const __half h0 = __float2half_rn(x0), h1 = __float2half_rn(x1);
+  const __half l0 = __float2half_rn(x0 - __half2float(h0)), l1 = __float2half_rn(x1 - __half2float(h1));
+  hi = (uint32_t)__half_as_ushort(h0) | ((uint32_t)__half_as_ushort(h1) << 16);
+  lo = (uint32_t)__half_as_ushort(l0) | ((uint32_t)__half_as_ushort(l1) << 16);
+}
+// The 8 values of a chunk as fp16 bits, two per word.
+template <int FMT>
+__device__ __forceinline__ void chunk_half_words(const Chunk<FMT>& ch, uint32_t (&w)[4]) {
+  if constexpr (FMT == kFmtFp16) {
+    w[0] = ch.v.x, w[1] = ch.v.y, w[2] = ch.v.z, w[3] = ch.v.w;
+  } else {
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const uint32_t src = q < 2 ? ch.r.x : ch.r.y;
+      const __half2_raw h = __nv_cvt_fp8x2_to_halfraw2(
+          (__nv_fp8x2_storage_t)((q & 1) ? (src >> 16) : (src & 0xffffu)), __NV_E4M3);
+      w[q] = (uint32_t)h.x | ((uint32_t)h.y << 16);
+    }
+  }
+}
+// Scores of G heads for one chunk: q' row idx of this lane is G floats.
+template <int G>
+__device__ __forceinline__ void score_g_chunk(uint32_t qb, const float (&f)[8], uint2 ix, float (&s)[G]) {
+#pragma unroll
+  for (int e = 0; e < 8; ++e) {
+    const uint32_t w = e < 4 ? ix.x : ix.y;
+    const uint32_t a = qb + ((w >> (8 * (e & 3))) & 0x7fu) * (uint32_t)(128 * G);
+    if constexpr (G == 4) {
+      const float4 q = lds4(a);
+      s[0] = fmaf(q.x, f[e], s[0]);
+      s[1] = fmaf(q.y, f[e], s[1]);
+      s[2] = fmaf(q.z, f[e], s[2]);
+      s[3] = fmaf(q.w, f[e], s[3]);
+    } else {
+      const float2 q = lds2(a);
+      s[0] = fmaf(q.x, f[e], s[0]);
+      s[1] = fmaf(q.y, f[e], s[1]);
+    }
+  }
+}
+// Scatter the first n (<= 8) entries of a chunk into this lane's tile row.
+__device__ __forceinline__ void scatter_chunk(uint32_t vrow, const uint32_t (&w)[4], uint2 ix, int n) {
+#pragma unroll
+  for (int e = 0; e < 8; ++e) {
+    if (e < n) {
+      const uint32_t iw = e < 4 ? ix.x : ix.y;
+      const uint32_t idx = (iw >> (8 * (e & 3))) & 0x7fu;
+      const uint32_t hw = w[e >> 1];
+      sts_u16(vrow + idx * 2, (e & 1) ? (hw >> 16) : (hw & 0xffffu));
+    }
+  }
+}
+
+template <int G, int MAXC, int FMT>
+__global__ void __launch_bounds__(kMmaWarps * 32, 1) decode_mma_kernel(DecodeParams p) {
+  constexpr int NW = kMmaWarps, NT = NW * 32;
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  __shared__ float red_m[NW * G], red_l[NW * G];
+  __shared__ float flag[1];
+  pdl_trigger();
+
+  const uint32_t raw = (uint32_t)__cvta_generic_to_shared(smem_raw);
+  const uint32_t base = (raw + 15u) & ~15u;
+  unsigned char* base_ptr = smem_raw + (base - raw);
+  float* qrep = reinterpret_cast<float*>(base_ptr);                         // [128][32][G]
+  const uint32_t wbase = base + kHeadDim * 32 * G * 4;                      // per-warp regions
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t vtile = wbase + warp * kMmaWarpBytes;                      // [32][272 B] fp16
+  float* ptile_f = reinterpret_cast<float*>(base_ptr + (vtile + kVTileBytes - base));  // [G][32] fp32
+  const uint32_t qb = base + lane * (G * 4);
+  const uint32_t vrow = vtile + lane * kVRowBytes;
+  const int gq = lane >> 2, cq = lane & 3;  // mma fragment coordinates
+
+  const CacheGeom& g = p.geom;
+  const int kfull = p.k_full_chunks, krem = p.k_rem;
+  const int nchunks = kfull + (krem ? 1 : 0);
+  const int kfull_v = p.k_full_chunks_v, krem_v = p.k_rem_v;
+  const int nchunks_v = kfull_v + (krem_v ? 1 : 0);
+  const int o_kv = lane * 16, o_ki = g.kidx_off() + lane * 8;
+  const int o_vv = g.vval_off() + lane * 16, o_vi = g.vidx_off() + lane * 8;
+  const bool whole_block = nchunks * 8 == g.k_slots && nchunks_v * 8 == g.k_slots_v;
+  const int bsh = p.blocks_per_page_log2, bmask = (1 << bsh) - 1;
+
+  const int64_t g_begin = cta_begin(p, blockIdx.x);
+  const int64_t g_end = min(p.total_groups, cta_begin(p, blockIdx.x + 1));
+  pdl_wait();
+  if (g_begin >= g_end) return;
+  const int64_t u_first = unit_of(p, g_begin), u_last = unit_of(p, g_end - 1);
+
+  // the tiles start zeroed; every use restores the zeros it disturbed
+  for (int c = 0; c < 16; ++c) sts_v4(vrow + c * 16, make_uint4(0, 0, 0, 0));
+
+  for (int64_t u = u_first; u <= u_last; ++u) {
+    const UnitView uv = unit_view(p, u);
+    const int n_sg = uv.n_sg;
+    const int s0 = (int)(max(g_begin, uv.goff) - uv.goff);
+    const int s1 = (int)(min(g_end, uv.goff + uv.N_g) - uv.goff);
+    const int64_t b = u / p.H_kv, h = u % p.H_kv;
+    const int t_lo = split_at(s0, s1, n_sg, warp, NW);
+    const int t_hi = split_at(s0, s1, n_sg, warp + 1, NW);
+    const int sp_hi = min(t_hi, n_sg);
+    const int32_t* ptab = g.page_table + u * g.pages_per_unit;
+
+    __syncthreads();  // the previous segment is done with q'
+    for (int i = threadIdx.x; i < kHeadDim * 32 * G; i += NT) {
+      const int c = i / (32 * G), j = i % G;
+      qrep[i] = __ldg(p.qprime + ((b * p.H_q + h * G + j) * kHeadDim + c));
+    }
+    __syncthreads();
+
+    float m[G], l[G];
+#pragma unroll
+    for (int j = 0; j < G; ++j) m[j] = -INFINITY, l[j] = 0.f;
+    float acc[16][2];
+#pragma unroll
+    for (int nt = 0; nt < 16; ++nt) acc[nt][0] = acc[nt][1] = 0.f;
+
+    auto block_of = [&](int gi) -> const uint8_t* {
+      if (gi >= sp_hi) return nullptr;
+      const int32_t ph = __ldg(ptab + (gi >> bsh));
+      if (ph < 0 || ph >= g.num_pages) {
+        atomicOr(p.status, kStatusPageRange);
+        return nullptr;
+      }
+      return g.pool + (int64_t)ph * g.page_bytes + (int64_t)(gi & bmask) * g.block_bytes();
+    };
+    auto prefetch_block = [&](const uint8_t* blk) {
+      if (blk == nullptr || lane != 0) return;
+      if (whole_block) {
+        prefetch_l2(blk, (uint32_t)g.block_bytes());
+      } else if constexpr (FMT == kFmtFp16) {
+        prefetch_l2(blk, nchunks * 512u);
+        prefetch_l2(blk + g.kidx_off(), nchunks * 256u);
+        prefetch_l2(blk + g.vval_off(), nchunks_v * 512u);
+        prefetch_l2(blk + g.vidx_off(), nchunks_v * 256u);
+      } else {
+        prefetch_l2(blk, nchunks * 512u);
+        prefetch_l2(blk + g.vval_off(), nchunks_v * 512u);
+      }
+    };
+    Chunk<FMT> kc[MAXC];
+    auto load_k = [&](const uint8_t* blk) {
+      const uint8_t* src = blk ? blk : g.pool;
+#pragma unroll
+      for (int c = 0; c < MAXC; ++c)
+        if (c < nchunks) kc[c] = load_chunk<FMT, false>(src + o_kv, src + o_ki, c);
+    };
+
+    const uint8_t* b_cur = block_of(t_lo);
+    const uint8_t* b_n1 = block_of(t_lo + 1);
+    prefetch_block(b_n1);
+    if (t_lo < sp_hi) load_k(b_cur);
+
+    for (int gi = t_lo; gi < t_hi; ++gi) {
+      float s[G];
+#pragma unroll
+      for (int j = 0; j < G; ++j) s[j] = 0.f;
+      bool valid;
+      if (gi < n_sg) {
+        // ---- sparse tokens 32 gi .. 32 gi + 31
+        const int64_t t0 = (int64_t)gi * 32;
+        const bool ok = b_cur != nullptr;
+        valid = ok && t0 + lane < uv.sparse_len;
+        const uint8_t* src = ok ? b_cur : g.pool;
+        const uint8_t* b_n2 = block_of(gi + 2);
+        prefetch_block(b_n2);
+        if (valid) {
+#pragma unroll
+          for (int c = 0; c < MAXC; ++c)
+            if (c < nchunks) {
+              float f[8];
+              chunk_vals<FMT>(kc[c], f);
+              if (krem && c == nchunks - 1) keep_first(f, krem);
+              score_g_chunk<G>(qb, f, chunk_idx<FMT>(kc[c]), s);
+            }
+          // this token's kept values into its tile row (loaded now, when
+          // the key records are dead, to keep the registers down; the block
+          // is already in L2)
+#pragma unroll
+          for (int c = 0; c < MAXC; ++c)
+            if (c < nchunks_v) {
+              const Chunk<FMT> vc = load_chunk<FMT, false>(src + o_vv, src + o_vi, c);
+              uint32_t w[4];
+              chunk_half_words<FMT>(vc, w);
+              scatter_chunk(vrow, w, chunk_idx<FMT>(vc), (krem_v && c == nchunks_v - 1) ? krem_v : 8);
+            }
+        }
+        if (gi + 1 < sp_hi) load_k(b_n1);
+        b_cur = b_n1;
+        b_n1 = b_n2;
+      } else {
+        // ---- dense buffer tokens: scores over all 128 coordinates, the
+        // value row copied into the tile
+        const int64_t i = (int64_t)(gi - n_sg) * 32 + lane;
+        valid = i < uv.n_b;
+        if (valid) {
+          const int slot = (int)((uv.buf_start + i) % p.cap);
+          const size_t row = ((size_t)u * p.cap + slot) * kHeadDim;
+          const uint4* kr = reinterpret_cast<const uint4*>(p.ring_k + row);
+          const uint4* vr = reinterpret_cast<const uint4*>(p.ring_v + row);
+#pragma unroll 2
+          for (int c = 0; c < 16; ++c) {
+            const uint4 w = __ldg(kr + c);
+            const float2 a = h2f(w.x), bb = h2f(w.y), cc = h2f(w.z), d = h2f(w.w);
+            const float f[8] = {a.x, a.y, bb.x, bb.y, cc.x, cc.y, d.x, d.y};
+#pragma unroll
+            for (int e = 0; e < 8; ++e) {
+              const uint32_t qa = qb + (uint32_t)(c * 8 + e) * (128 * G);
+              if constexpr (G == 4) {
+                const float4 q = lds4(qa);
+                s[0] = fmaf(q.x, f[e], s[0]);
+                s[1] = fmaf(q.y, f[e], s[1]);
+                s[2] = fmaf(q.z, f[e], s[2]);
+                s[3] = fmaf(q.w, f[e], s[3]);
+              } else {
+                const float2 q = lds2(qa);
+                s[0] = fmaf(q.x, f[e], s[0]);
+                s[1] = fmaf(q.y, f[e], s[1]);
+              }
+            }
+          }
+#pragma unroll 4
+          for (int c = 0; c < 16; ++c) sts_v4(vrow + c * 16, __ldg(vr + c));
+        }
+      }
+
+      // ---- online softmax per head (lazy rescale of the register accumulators)
+      float pj[G];
+#pragma unroll
+      for (int j = 0; j < G; ++j) {
+        const float sj = valid ? s[j] * p.scale_log2 : -INFINITY;
+        const float gmax = warp_max(sj);
+        if (gmax > m[j] + kLazyRescale) {
+          if (m[j] != -INFINITY) {
+            const float fs = exp2f(m[j] - gmax);
+            l[j] *= fs;
+            if (gq == j) {
+#pragma unroll
+              for (int nt = 0; nt < 16; ++nt) acc[nt][0] *= fs, acc[nt][1] *= fs;
+            }
+          }
+          m[j] = gmax;
+        }
+        pj[j] = valid ? exp2f(sj - m[j]) : 0.f;
+        l[j] += pj[j];
+        ptile_f[j * 32 + lane] = pj[j];
+      }
+      __syncwarp();
+
+      // ---- o[head][:] += p[head][tokens] * tile[tokens][:] on the tensor cores
+#pragma unroll
+      for (int ks = 0; ks < 2; ++ks) {
+        uint32_t ahi0 = 0, alo0 = 0, ahi2 = 0, alo2 = 0;
+        if (gq < G) {
+          const float* pr = ptile_f + gq * 32 + ks * 16 + 2 * cq;
+          split_pair(pr[0], pr[1], ahi0, alo0);
+          split_pair(pr[8], pr[9], ahi2, alo2);
+        }
+#pragma unroll
+        for (int np = 0; np < 8; ++np) {
+          const int mi = lane >> 3;
+          const uint32_t addr = vtile + (uint32_t)(ks * 16 + (mi & 1) * 8 + (lane & 7)) * kVRowBytes +
+                                (uint32_t)(16 * np + 8 * (mi >> 1)) * 2;
+          uint32_t bf[4];
+          ldsm_x4_trans(addr, bf);
+          mma_16816(acc[2 * np], ahi0, ahi2, bf[0], bf[1]);
+          mma_16816(acc[2 * np], alo0, alo2, bf[0], bf[1]);
+          mma_16816(acc[2 * np + 1], ahi0, ahi2, bf[2], bf[3]);
+          mma_16816(acc[2 * np + 1], alo0, alo2, bf[2], bf[3]);
+        }
+      }
+      __syncwarp();
+      // restore the zeros of this lane's tile row
+      if (valid)
+        for (int c = 0; c < 16; ++c) sts_v4(vrow + c * 16, make_uint4(0, 0, 0, 0));
+    }
+
+    // ---- merge lanes and warps per query head into one partial
+#pragma unroll
+    for (int j = 0; j < G; ++j) l[j] = warp_sum(l[j]);
+    if (lane == 0) {
+#pragma unroll
+      for (int j = 0; j < G; ++j) {
+        red_m[warp * G + j] = m[j];
+        red_l[warp * G + j] = l[j];
+      }
+    }
+    // this warp's o rows into its tile region ([G][128] fp32)
+    __syncwarp();
+    float* obuf = reinterpret_cast<float*>(base_ptr + (vtile - base));
+    if (gq < G) {
+#pragma unroll
+      for (int nt = 0; nt < 16; ++nt) {
+        obuf[gq * kHeadDim + nt * 8 + 2 * cq] = acc[nt][0];
+        obuf[gq * kHeadDim + nt * 8 + 2 * cq + 1] = acc[nt][1];
+      }
+    }
+    __syncthreads();
+    const int64_t c0 = cta_of(p, uv.goff), c1 = cta_of(p, uv.goff + uv.N_g - 1);
+    const bool solo = c0 == c1;
+    for (int o = threadIdx.x; o < G * kHeadDim; o += NT) {
+      const int hd = o / kHeadDim, dd = o % kHeadDim;
+      float M = -INFINITY;
+#pragma unroll
+      for (int w = 0; w < NW; ++w) M = fmaxf(M, red_m[w * G + hd]);
+      float tot = 0.f, L = 0.f;
+#pragma unroll
+      for (int w = 0; w < NW; ++w) {
+        const float mw = red_m[w * G + hd];
+        const float f = (mw == -INFINITY) ? 0.f : exp2f(mw - M);
+        const float* ob = reinterpret_cast<const float*>(base_ptr + (wbase - base) + w * kMmaWarpBytes);
+        tot = fmaf(f, ob[hd * kHeadDim + dd], tot);
+        L = fmaf(f, red_l[w * G + hd], L);
+      }
+      if (solo) {
+        qrep[o] = (L > 0.f) ? tot / L : 0.f;  // q' is no longer needed
+        continue;
+      }
+      float* dst = p.partials + ((size_t)(blockIdx.x + u) * G + hd) * (kHeadDim + 2);
+      dst[2 + dd] = tot;
+      if (dd == 0) {
+        dst[0] = M;
+        dst[1] = L;
+      }
+    }
+    __syncthreads();
+    // the o rows overwrote part of the tiles: zero them again
+    for (int c = 0; c < 16; ++c) sts_v4(vrow + c * 16, make_uint4(0, 0, 0, 0));
+    if (solo) {
+      rotate_back_out<G, NT>(p, b, h, qrep);
+    } else {
+      finish_unit<G, NT>(p, c0, c1, u, b, h, qrep, flag);
+    }
+  }
+}
+
 // q' = q R_qk: one CTA per (kv head, up to 8 query vectors of that head),
 // R in shared memory, one warp per query vector; lane l computes coordinates
 // 4l..4l+3 in a sequential fp32 FMA chain.
@@ -1111,13 +1502,14 @@ cudaError_t launch_t(const DecodeParams& p, int grid, cudaStream_t s) {
     }
     return launch_pdl(decode_kernel<MAXC, FMT>, dim3(grid), dim3(decode_warps<MAXC>() * 32), smem, s, p);
   } else {
+    constexpr size_t smem = mma_smem<G>();
     if (!attr_set) {
-      cudaError_t e = cudaFuncSetAttribute(decode_gqa_kernel<G, MAXC, FMT>,
-                                           cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kGqaSmem);
+      cudaError_t e = cudaFuncSetAttribute(decode_mma_kernel<G, MAXC, FMT>,
+                                           cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
       if (e != cudaSuccess) return e;
       attr_set = true;
     }
-    return launch_pdl(decode_gqa_kernel<G, MAXC, FMT>, dim3(grid), dim3(kGqaWarps * 32), kGqaSmem, s, p);
+    return launch_pdl(decode_mma_kernel<G, MAXC, FMT>, dim3(grid), dim3(kMmaWarps * 32), smem, s, p);
   }
 }
 
@@ -1135,11 +1527,11 @@ int decode_ctas_per_sm(int G, int k_slots) {
     return big ? occupancy(decode_kernel<16, kFmtFp16>, decode_warps<16>() * 32, one_head_smem(16))
                : occupancy(decode_kernel<8, kFmtFp16>, decode_warps<8>() * 32, one_head_smem(8));
   if (G == 2)
-    return big ? occupancy(decode_gqa_kernel<2, 16, kFmtFp16>, kGqaWarps * 32, kGqaSmem)
-               : occupancy(decode_gqa_kernel<2, 8, kFmtFp16>, kGqaWarps * 32, kGqaSmem);
+    return big ? occupancy(decode_mma_kernel<2, 16, kFmtFp16>, kMmaWarps * 32, mma_smem<2>())
+               : occupancy(decode_mma_kernel<2, 8, kFmtFp16>, kMmaWarps * 32, mma_smem<2>());
   if (G == 4)
-    return big ? occupancy(decode_gqa_kernel<4, 16, kFmtFp16>, kGqaWarps * 32, kGqaSmem)
-               : occupancy(decode_gqa_kernel<4, 8, kFmtFp16>, kGqaWarps * 32, kGqaSmem);
+    return big ? occupancy(decode_mma_kernel<4, 16, kFmtFp16>, kMmaWarps * 32, mma_smem<4>())
+               : occupancy(decode_mma_kernel<4, 8, kFmtFp16>, kMmaWarps * 32, mma_smem<4>());
   return 0;
 }
 

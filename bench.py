@@ -87,7 +87,7 @@ def decode_kernel_traffic(workload: str, values: str = "fp16", variant: str = ""
     digest = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
     text = None
     suffix = ("" if values == "fp16" else "-fp8") + variant
-    for name in (f"decode_kernel_{workload}{suffix}.md", f"decode_gqa_kernel_{workload}{suffix}.md"):
+    for name in (f"decode_kernel_{workload}{suffix}.md", f"decode_mma_kernel_{workload}{suffix}.md"):
         try:
             text = open(os.path.join(ROOT, "profiles", name)).read()
             break

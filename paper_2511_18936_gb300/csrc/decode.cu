@@ -123,9 +123,6 @@ __device__ __forceinline__ float2 lds2(uint32_t a) {
   asm volatile("ld.shared.v2.f32 {%0,%1}, [%2];" : "=f"(v.x), "=f"(v.y) : "r"(a));
   return v;
 }
-__device__ __forceinline__ void sts2(uint32_t a, float2 v) {
-  asm volatile("st.shared.v2.f32 [%0], {%1,%2};" ::"r"(a), "f"(v.x), "f"(v.y));
-}
 
 // Ask the memory system to bring `bytes` (a multiple of 16, 16-byte aligned)
 // into L2 ahead of the loads that will read them.
@@ -623,393 +620,6 @@ __global__ void __launch_bounds__(decode_warps<MAXC>() * 32, 1) decode_kernel(De
 }
 
 // ---------------------------------------------------------------------------
-// Grouped-query heads (G = 2 or 4): each lane carries a pair of query heads
-// of one token, so the index decoding, the value conversion and the record
-// loads are shared by two heads, and one accumulator array serves the whole
-// group: lanes 16..31 take heads 2..3 of the tokens that lanes 0..15 take
-// heads 0..1 of (G = 4).  q' and the accumulators are [128][32 lanes][2]
-// fp32 (32 KB), so 32 lanes reading or updating arbitrary coordinates with
-// 8-byte accesses never share a bank within a half-warp.
-// ---------------------------------------------------------------------------
-
-constexpr uint32_t kPairRegionBytes = kHeadDim * 32 * 2 * sizeof(float);  // 32 KB
-constexpr int kGqaWarps = 5;  // q' + 5 accumulators at 32 KB-aligned offsets fit in 227 KB
-
-// base | (idx & 127) << 8 | lane << 3 for byte e of an index word (base 32 KB aligned)
-template <int E>
-__device__ __forceinline__ uint32_t addr2_of(uint32_t w, uint32_t base) {
-  if (E == 0) return ((w << 8) & 0x7f00u) | base;
-  if (E == 1) return (w & 0x7f00u) | base;
-  if (E == 2) return ((w >> 8) & 0x7f00u) | base;
-  return ((w >> 16) & 0x7f00u) | base;
-}
-
-// Scores of two heads for one chunk: s[0..1] head 0, s[2..3] head 1.
-__device__ __forceinline__ void score2_chunk(uint32_t qb, const float (&f)[8], uint2 ix, float (&s)[4]) {
-  const float2 q0 = lds2(addr2_of<0>(ix.x, qb)), q1 = lds2(addr2_of<1>(ix.x, qb));
-  const float2 q2 = lds2(addr2_of<2>(ix.x, qb)), q3 = lds2(addr2_of<3>(ix.x, qb));
-  const float2 q4 = lds2(addr2_of<0>(ix.y, qb)), q5 = lds2(addr2_of<1>(ix.y, qb));
-  const float2 q6 = lds2(addr2_of<2>(ix.y, qb)), q7 = lds2(addr2_of<3>(ix.y, qb));
-  s[0] = fmaf(q0.x, f[0], s[0]); s[2] = fmaf(q0.y, f[0], s[2]);
-  s[1] = fmaf(q1.x, f[1], s[1]); s[3] = fmaf(q1.y, f[1], s[3]);
-  s[0] = fmaf(q2.x, f[2], s[0]); s[2] = fmaf(q2.y, f[2], s[2]);
-  s[1] = fmaf(q3.x, f[3], s[1]); s[3] = fmaf(q3.y, f[3], s[3]);
-  s[0] = fmaf(q4.x, f[4], s[0]); s[2] = fmaf(q4.y, f[4], s[2]);
-  s[1] = fmaf(q5.x, f[5], s[1]); s[3] = fmaf(q5.y, f[5], s[3]);
-  s[0] = fmaf(q6.x, f[6], s[0]); s[2] = fmaf(q6.y, f[6], s[2]);
-  s[1] = fmaf(q7.x, f[7], s[1]); s[3] = fmaf(q7.y, f[7], s[3]);
-}
-
-__device__ __forceinline__ float2 fma2(float p0, float p1, float v, float2 o) {
-  return make_float2(fmaf(p0, v, o.x), fmaf(p1, v, o.y));
-}
-
-// acc[idx_e] += (p0, p1) * val_e for one full chunk (distinct indices).
-__device__ __forceinline__ void value2_chunk(uint32_t ab, float p0, float p1, const float (&f)[8], uint2 ix) {
-  const uint32_t a0 = addr2_of<0>(ix.x, ab), a1 = addr2_of<1>(ix.x, ab);
-  const uint32_t a2 = addr2_of<2>(ix.x, ab), a3 = addr2_of<3>(ix.x, ab);
-  const uint32_t a4 = addr2_of<0>(ix.y, ab), a5 = addr2_of<1>(ix.y, ab);
-  const uint32_t a6 = addr2_of<2>(ix.y, ab), a7 = addr2_of<3>(ix.y, ab);
-  const float2 o0 = lds2(a0), o1 = lds2(a1), o2 = lds2(a2), o3 = lds2(a3);
-  const float2 o4 = lds2(a4), o5 = lds2(a5), o6 = lds2(a6), o7 = lds2(a7);
-  sts2(a0, fma2(p0, p1, f[0], o0));
-  sts2(a1, fma2(p0, p1, f[1], o1));
-  sts2(a2, fma2(p0, p1, f[2], o2));
-  sts2(a3, fma2(p0, p1, f[3], o3));
-  sts2(a4, fma2(p0, p1, f[4], o4));
-  sts2(a5, fma2(p0, p1, f[5], o5));
-  sts2(a6, fma2(p0, p1, f[6], o6));
-  sts2(a7, fma2(p0, p1, f[7], o7));
-}
-
-__device__ __forceinline__ void value2_chunk_partial(uint32_t ab, float p0, float p1, const float (&f)[8],
-                                                     uint2 ix, int n) {
-#pragma unroll
-  for (int e = 0; e < 7; ++e) {
-    if (e < n) {
-      const uint32_t w = e < 4 ? ix.x : ix.y;
-      const uint32_t a = ((w >> (8u * (e & 3))) & 0x7fu) << 8 | ab;
-      sts2(a, fma2(p0, p1, f[e], lds2(a)));
-    }
-  }
-}
-
-// Reduce over the lanes of one head group (TS lanes: the whole warp for
-// G = 2, a half-warp for G = 4).
-template <int TS>
-__device__ __forceinline__ float group_max(float v) {
-#pragma unroll
-  for (int o = TS / 2; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
-  return v;
-}
-template <int TS>
-__device__ __forceinline__ float group_sum(float v) {
-#pragma unroll
-  for (int o = TS / 2; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-  return v;
-}
-
-template <int G, int MAXC, int FMT>
-__global__ void __launch_bounds__(kGqaWarps * 32, 1) decode_gqa_kernel(DecodeParams p) {
-  constexpr int NW = kGqaWarps, NT = NW * 32;
-  constexpr int LPT = G / 2;          // lanes per token
-  constexpr int TS = 32 / LPT;        // tokens per warp iteration
-  constexpr int HALVES = 32 / TS;     // iterations per 32-token block
-  extern __shared__ __align__(16) unsigned char smem_raw[];
-  __shared__ float red_m[NW * G], red_l[NW * G], flag[1];
-  pdl_trigger();
-
-  const uint32_t raw = (uint32_t)__cvta_generic_to_shared(smem_raw);
-  const uint32_t base = (raw + kPairRegionBytes - 1) & ~(kPairRegionBytes - 1);
-  float* qrep = reinterpret_cast<float*>(smem_raw + (base - raw));  // [128][32][2]
-  float* accs = qrep + kHeadDim * 32 * 2;                            // [NW][128][32][2]
-
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int ts = lane % TS, hg = lane / TS;  // token slot, head pair
-  const uint32_t qb = base + (lane << 3);
-  const uint32_t ab = base + (1 + warp) * kPairRegionBytes + (lane << 3);
-
-  const CacheGeom& g = p.geom;
-  const int kfull = p.k_full_chunks, krem = p.k_rem;          // keys
-  const int nchunks = kfull + (krem ? 1 : 0);
-  const int kfull_v = p.k_full_chunks_v, krem_v = p.k_rem_v;  // values
-  const int nchunks_v = kfull_v + (krem_v ? 1 : 0);
-  const bool whole_block = nchunks * 8 == g.k_slots && nchunks_v * 8 == g.k_slots_v;
-  const int bsh = p.blocks_per_page_log2, bmask = (1 << bsh) - 1;
-
-  const int64_t g_begin = cta_begin(p, blockIdx.x);
-  const int64_t g_end = min(p.total_groups, cta_begin(p, blockIdx.x + 1));
-  pdl_wait();
-  if (g_begin >= g_end) return;
-  const int64_t u_first = unit_of(p, g_begin), u_last = unit_of(p, g_end - 1);
-
-  for (int64_t u = u_first; u <= u_last; ++u) {
-    const UnitView uv = unit_view(p, u);
-    const int n_sg = uv.n_sg;
-    const int s0 = (int)(max(g_begin, uv.goff) - uv.goff);
-    const int s1 = (int)(min(g_end, uv.goff + uv.N_g) - uv.goff);
-    const int64_t b = u / p.H_kv, h = u % p.H_kv;
-    // this warp's contiguous run of items (half-blocks for G = 4)
-    // items are half-blocks (G = 4) or blocks (G = 2): split like groups
-    const int i_lo = split_at(s0 * HALVES, s1 * HALVES, n_sg * HALVES, warp, NW);
-    const int i_hi = split_at(s0 * HALVES, s1 * HALVES, n_sg * HALVES, warp + 1, NW);
-    const int32_t* ptab = g.page_table + u * g.pages_per_unit;
-
-    __syncthreads();  // the previous segment is done with shared memory
-    for (int i = threadIdx.x; i < kHeadDim * 32 * 2; i += NT) {
-      const int dd = i >> 6, l = (i >> 1) & 31, j = i & 1;
-      const int head = 2 * (l / TS) + j;
-      qrep[i] = __ldg(p.qprime + ((b * p.H_q + h * G + head) * kHeadDim + dd));
-    }
-#pragma unroll 8
-    for (int dd = 0; dd < kHeadDim; ++dd) sts2(ab + dd * 256, make_float2(0.f, 0.f));
-    __syncthreads();
-
-    float m0 = -INFINITY, m1 = -INFINITY;  // running maxima (log2), uniform in the head group
-    float l0 = 0.f, l1 = 0.f;
-
-    auto block_of = [&](int gi) -> const uint8_t* {
-      if (gi >= n_sg || gi * HALVES >= i_hi) return nullptr;
-      const int32_t ph = __ldg(ptab + (gi >> bsh));
-      if (ph < 0 || ph >= g.num_pages) {
-        atomicOr(p.status, kStatusPageRange);
-        return nullptr;
-      }
-      return g.pool + (int64_t)ph * g.page_bytes + (int64_t)(gi & bmask) * g.block_bytes();
-    };
-    auto prefetch_block = [&](const uint8_t* blk) {
-      if (blk == nullptr || lane != 0) return;
-      if (whole_block) {
-        prefetch_l2(blk, (uint32_t)g.block_bytes());
-      } else if constexpr (FMT == kFmtFp16) {
-        prefetch_l2(blk, nchunks * 512u);
-        prefetch_l2(blk + g.kidx_off(), nchunks * 256u);
-        prefetch_l2(blk + g.vval_off(), nchunks_v * 512u);
-        prefetch_l2(blk + g.vidx_off(), nchunks_v * 256u);
-      } else {
-        prefetch_l2(blk, nchunks * 512u);
-        prefetch_l2(blk + g.vval_off(), nchunks_v * 512u);
-      }
-    };
-    // records of item `half` of a block for this lane's token
-    Chunk<FMT> kc[MAXC];
-    auto load_k = [&](const uint8_t* blk, int half) {
-      const uint8_t* src = blk ? blk : g.pool;
-      const int t = half * TS + ts;
-#pragma unroll
-      for (int c = 0; c < MAXC; ++c)
-        if (c < nchunks) kc[c] = load_chunk<FMT, true>(src + t * 16, src + g.kidx_off() + t * 8, c);
-    };
-
-    int gi0 = i_lo / HALVES;
-    const uint8_t* b_cur = block_of(gi0);
-    const uint8_t* b_n1 = block_of(gi0 + 1);
-    prefetch_block(b_n1);
-    if (i_lo < i_hi && gi0 < n_sg) load_k(b_cur, i_lo % HALVES);
-
-    for (int it = i_lo; it < i_hi; ++it) {
-      const int gi = it / HALVES, half = it % HALVES;
-      float s[4] = {0.f, 0.f, 0.f, 0.f};
-      float p0, p1;
-      bool valid;
-      if (gi < n_sg) {
-        // ---- sparse tokens 32*gi + half*TS + ts
-        const int64_t t = (int64_t)gi * 32 + half * TS + ts;
-        const bool ok = b_cur != nullptr;
-        valid = ok && t < uv.sparse_len;
-        const bool tail = !ok || (int64_t)gi * 32 + (half + 1) * TS > uv.sparse_len;  // warp-uniform
-        const uint8_t* src = ok ? b_cur : g.pool;
-        const int tt = half * TS + ts;
-        Chunk<FMT> vc[MAXC];
-#pragma unroll
-        for (int c = 0; c < MAXC; ++c)
-          if (c < nchunks_v)
-            vc[c] = load_chunk<FMT, true>(src + g.vval_off() + tt * 16, src + g.vidx_off() + tt * 8, c);
-        const bool last_half = half == HALVES - 1;
-        const uint8_t* b_n2 = nullptr;
-        if (last_half) {
-          b_n2 = block_of(gi + 2);
-          prefetch_block(b_n2);
-        }
-
-#pragma unroll
-        for (int c = 0; c < MAXC; ++c)
-          if (c < nchunks) {
-            float f[8];
-            chunk_vals<FMT>(kc[c], f);
-            uint2 ix = chunk_idx<FMT>(kc[c]);
-            if (krem && c == nchunks - 1) keep_first(f, krem);
-            if (tail && !valid) {
-              keep_first(f, 0);
-              ix = make_uint2(0, 0);
-            }
-            score2_chunk(qb, f, ix, s);
-          }
-
-        // next item's key records (same block's next half, or the next block)
-        const int nit = it + 1;
-        if (nit < i_hi) {
-          const int ngi = nit / HALVES;
-          if (ngi < n_sg) load_k(last_half ? b_n1 : b_cur, nit % HALVES);
-        }
-        if (last_half) {
-          b_cur = b_n1;
-          b_n1 = b_n2;
-        }
-
-        const float s0v = valid ? (s[0] + s[1]) * p.scale_log2 : -INFINITY;
-        const float s1v = valid ? (s[2] + s[3]) * p.scale_log2 : -INFINITY;
-        const float g0 = group_max<TS>(s0v), g1 = group_max<TS>(s1v);
-        if (g0 > m0 + kLazyRescale || g1 > m1 + kLazyRescale) {
-          const float n0 = (g0 > m0 + kLazyRescale) ? g0 : m0;
-          const float n1 = (g1 > m1 + kLazyRescale) ? g1 : m1;
-          const float f0 = (m0 == -INFINITY) ? 1.f : exp2f(m0 - n0);
-          const float f1 = (m1 == -INFINITY) ? 1.f : exp2f(m1 - n1);
-          l0 *= f0;
-          l1 *= f1;
-#pragma unroll 8
-          for (int dd = 0; dd < kHeadDim; ++dd) {
-            const float2 o = lds2(ab + dd * 256);
-            sts2(ab + dd * 256, make_float2(o.x * f0, o.y * f1));
-          }
-          m0 = n0;
-          m1 = n1;
-        }
-        p0 = valid ? exp2f(s0v - m0) : 0.f;
-        p1 = valid ? exp2f(s1v - m1) : 0.f;
-        l0 += p0;
-        l1 += p1;
-
-#pragma unroll
-        for (int c = 0; c < MAXC; ++c)
-          if (c < kfull_v) {
-            float f[8];
-            chunk_vals<FMT>(vc[c], f);
-            uint2 ix = chunk_idx<FMT>(vc[c]);
-            if (tail && !valid) {
-              keep_first(f, 0);
-              ix = make_uint2(0, 0);
-            }
-            value2_chunk(ab, p0, p1, f, ix);
-          }
-        if (krem_v && valid) {
-#pragma unroll
-          for (int c = 0; c < MAXC; ++c)
-            if (c == kfull_v) {
-              float f[8];
-              chunk_vals<FMT>(vc[c], f);
-              value2_chunk_partial(ab, p0, p1, f, chunk_idx<FMT>(vc[c]), krem_v);
-            }
-        }
-      } else {
-        // ---- dense buffer tokens
-        const int64_t i = (int64_t)(gi - n_sg) * 32 + half * TS + ts;
-        valid = i < uv.n_b;
-        const int slot = valid ? (int)((uv.buf_start + i) % p.cap) : 0;
-        const size_t row = ((size_t)u * p.cap + slot) * kHeadDim;
-        const uint4* kr = reinterpret_cast<const uint4*>(p.ring_k + row);
-        const uint4* vr = reinterpret_cast<const uint4*>(p.ring_v + row);
-#pragma unroll 2
-        for (int c = 0; c < 16; ++c) {
-          const uint4 w = __ldg(kr + c);
-          const float2 a = h2f(w.x), bb = h2f(w.y), cc = h2f(w.z), d = h2f(w.w);
-          const float vals[8] = {a.x, a.y, bb.x, bb.y, cc.x, cc.y, d.x, d.y};
-#pragma unroll
-          for (int e = 0; e < 8; ++e) {
-            const float2 q = lds2(qb + (c * 8 + e) * 256);
-            s[(e & 1)] = fmaf(q.x, vals[e], s[(e & 1)]);
-            s[2 + (e & 1)] = fmaf(q.y, vals[e], s[2 + (e & 1)]);
-          }
-        }
-        const float s0v = valid ? (s[0] + s[1]) * p.scale_log2 : -INFINITY;
-        const float s1v = valid ? (s[2] + s[3]) * p.scale_log2 : -INFINITY;
-        const float g0 = group_max<TS>(s0v), g1 = group_max<TS>(s1v);
-        if (g0 > m0 + kLazyRescale || g1 > m1 + kLazyRescale) {
-          const float n0 = (g0 > m0 + kLazyRescale) ? g0 : m0;
-          const float n1 = (g1 > m1 + kLazyRescale) ? g1 : m1;
-          const float f0 = (m0 == -INFINITY) ? 1.f : exp2f(m0 - n0);
-          const float f1 = (m1 == -INFINITY) ? 1.f : exp2f(m1 - n1);
-          l0 *= f0;
-          l1 *= f1;
-#pragma unroll 8
-          for (int dd = 0; dd < kHeadDim; ++dd) {
-            const float2 o = lds2(ab + dd * 256);
-            sts2(ab + dd * 256, make_float2(o.x * f0, o.y * f1));
-          }
-          m0 = n0;
-          m1 = n1;
-        }
-        p0 = valid ? exp2f(s0v - m0) : 0.f;
-        p1 = valid ? exp2f(s1v - m1) : 0.f;
-        l0 += p0;
-        l1 += p1;
-        if (valid) {
-#pragma unroll 2
-          for (int c = 0; c < 16; ++c) {
-            const uint4 w = __ldg(vr + c);
-            const float2 a = h2f(w.x), bb = h2f(w.y), cc = h2f(w.z), d = h2f(w.w);
-            const float vals[8] = {a.x, a.y, bb.x, bb.y, cc.x, cc.y, d.x, d.y};
-            float2 o[8];
-#pragma unroll
-            for (int e = 0; e < 8; ++e) o[e] = lds2(ab + (c * 8 + e) * 256);
-#pragma unroll
-            for (int e = 0; e < 8; ++e) sts2(ab + (c * 8 + e) * 256, fma2(p0, p1, vals[e], o[e]));
-          }
-        }
-      }
-    }
-
-    // ---- merge lanes and warps per query head into one partial
-    l0 = group_sum<TS>(l0);
-    l1 = group_sum<TS>(l1);
-    if (ts == 0) {
-      red_m[warp * G + 2 * hg] = m0;
-      red_m[warp * G + 2 * hg + 1] = m1;
-      red_l[warp * G + 2 * hg] = l0;
-      red_l[warp * G + 2 * hg + 1] = l1;
-    }
-    __syncthreads();
-    const int64_t c0 = cta_of(p, uv.goff), c1 = cta_of(p, uv.goff + uv.N_g - 1);
-    const bool solo = c0 == c1;  // this CTA holds the whole unit
-    for (int o = threadIdx.x; o < G * kHeadDim; o += NT) {
-      const int hd = o / kHeadDim, dd = o % kHeadDim;
-      const int grp = hd >> 1, j = hd & 1;
-      float M = -INFINITY;
-#pragma unroll
-      for (int w = 0; w < NW; ++w) M = fmaxf(M, red_m[w * G + hd]);
-      float tot = 0.f, L = 0.f;
-#pragma unroll
-      for (int w = 0; w < NW; ++w) {
-        const float mw = red_m[w * G + hd];
-        const float f = (mw == -INFINITY) ? 0.f : exp2f(mw - M);
-        const float* a = accs + (size_t)w * kHeadDim * 64 + dd * 64 + j;
-        float sum = 0.f;
-#pragma unroll 4
-        for (int jj = 0; jj < TS; ++jj) sum += a[2 * (grp * TS + ((jj + dd) % TS))];
-        tot = fmaf(f, sum, tot);
-        L = fmaf(f, red_l[w * G + hd], L);
-      }
-      if (solo) {
-        qrep[o] = (L > 0.f) ? tot / L : 0.f;  // q' is no longer needed
-        continue;
-      }
-      float* dst = p.partials + ((size_t)(blockIdx.x + u) * G + hd) * (kHeadDim + 2);
-      dst[2 + dd] = tot;
-      if (dd == 0) {
-        dst[0] = M;
-        dst[1] = L;
-      }
-    }
-    if (solo) {
-      __syncthreads();
-      rotate_back_out<G, NT>(p, b, h, qrep);
-    } else {
-      finish_unit<G, NT>(p, c0, c1, u, b, h, qrep, flag);
-    }
-  }
-}
-
-// ---------------------------------------------------------------------------
 // Grouped-query heads with the value product on the tensor cores (G = 2, 4).
 //   Lane = token, as in the one-head kernel; each lane scores its token for
 //   all G query heads of the kv head from q' replicated per lane
@@ -1022,14 +632,37 @@ __global__ void __launch_bounds__(kGqaWarps * 32, 1) decode_gqa_kernel(DecodePar
 //   result keeps fp32 accuracy.  No per-warp shared accumulator: the tile
 //   and a [G][32] p table are all a warp holds in shared memory.
 // ---------------------------------------------------------------------------
-constexpr int kMmaWarps = 8;
 constexpr int kVRowBytes = 272;                      // 128 fp16 + 16 B pad: conflict-free ldmatrix rows
 constexpr uint32_t kVTileBytes = 32 * kVRowBytes;    // 8704
 constexpr uint32_t kPTileBytes = 4 * 32 * 4;         // p [<= 4 heads][32 tokens] fp32
-constexpr uint32_t kMmaWarpBytes = kVTileBytes + kPTileBytes;
-template <int G>
+// Per warp: the tile, the p table and a staging area for the value records
+// of the next block (cp.async: MAXC chunks of 512 B values + 256 B indices).
+template <int MAXC>
+__host__ __device__ constexpr uint32_t mma_warp_bytes() {
+  return kVTileBytes + kPTileBytes + (uint32_t)MAXC * 768;
+}
+template <int MAXC>
+__host__ __device__ constexpr int mma_warps() { return MAXC <= 8 ? 8 : 6; }
+template <int G, int MAXC>
 __host__ __device__ constexpr size_t mma_smem() {
-  return (size_t)kHeadDim * 32 * G * 4 + (size_t)kMmaWarps * kMmaWarpBytes + 16;
+  return (size_t)kHeadDim * 32 * G * 4 + (size_t)mma_warps<MAXC>() * mma_warp_bytes<MAXC>() + 16;
+}
+
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_group 0;" ::: "memory"); }
+__device__ __forceinline__ uint4 lds_v4u(uint32_t a) {
+  uint4 v;
+  asm volatile("ld.shared.v4.u32 {%0,%1,%2,%3}, [%4];" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(a)
+               : "memory");
+  return v;
+}
+__device__ __forceinline__ uint2 lds_v2u(uint32_t a) {
+  uint2 v;
+  asm volatile("ld.shared.v2.u32 {%0,%1}, [%2];" : "=r"(v.x), "=r"(v.y) : "r"(a) : "memory");
+  return v;
 }
 
 __device__ __forceinline__ float4 lds4(uint32_t a) {
@@ -1055,11 +688,11 @@ __device__ __forceinline__ void ldsm_x4_trans(uint32_t a, uint32_t (&r)[4]) {
 // d[0..1] += A (16 x 16, rows g and g + 8) * B (16 x 8); the rows g + 8 of A
 // are zero, so their accumulators are dropped.
 __device__ __forceinline__ void mma_16816(float (&d)[2], uint32_t a0, uint32_t a2, uint32_t b0, uint32_t b1) {
-  float x2, x3;
   asm volatile(
-      "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
-      "{%10,%11,%12,%13};"
-      : "=f"(d[0]), "=f"(d[1]), "=f"(x2), "=f"(x3)
+      "{\n\t.reg .f32 x2, x3;\n\t"
+      "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0,%1,x2,x3}, {%2,%3,%4,%5}, {%6,%7}, "
+      "{%8,%9,%10,%11};\n\t}"
+      : "=f"(d[0]), "=f"(d[1])
       : "r"(a0), "r"(0u), "r"(a2), "r"(0u), "r"(b0), "r"(b1), "f"(d[0]), "f"(d[1]), "f"(0.f), "f"(0.f));
 }
 // Two fp32 values as (hi, lo) fp16 pairs: x = hi + lo to ~2^-22 relative.
@@ -1118,8 +751,9 @@ __device__ __forceinline__ void scatter_chunk(uint32_t vrow, const uint32_t (&w)
 }
 
 template <int G, int MAXC, int FMT>
-__global__ void __launch_bounds__(kMmaWarps * 32, 1) decode_mma_kernel(DecodeParams p) {
-  constexpr int NW = kMmaWarps, NT = NW * 32;
+__global__ void __launch_bounds__(mma_warps<MAXC>() * 32, 1) decode_mma_kernel(DecodeParams p) {
+  constexpr int NW = mma_warps<MAXC>(), NT = NW * 32;
+  constexpr uint32_t kWarpBytes = mma_warp_bytes<MAXC>();
   extern __shared__ __align__(16) unsigned char smem_raw[];
   __shared__ float red_m[NW * G], red_l[NW * G];
   __shared__ float flag[1];
@@ -1131,8 +765,9 @@ __global__ void __launch_bounds__(kMmaWarps * 32, 1) decode_mma_kernel(DecodePar
   float* qrep = reinterpret_cast<float*>(base_ptr);                         // [128][32][G]
   const uint32_t wbase = base + kHeadDim * 32 * G * 4;                      // per-warp regions
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const uint32_t vtile = wbase + warp * kMmaWarpBytes;                      // [32][272 B] fp16
+  const uint32_t vtile = wbase + warp * kWarpBytes;                         // [32][272 B] fp16
   float* ptile_f = reinterpret_cast<float*>(base_ptr + (vtile + kVTileBytes - base));  // [G][32] fp32
+  const uint32_t vstage = vtile + kVTileBytes + kPTileBytes;                  // value records, next block
   const uint32_t qb = base + lane * (G * 4);
   const uint32_t vrow = vtile + lane * kVRowBytes;
   const int gq = lane >> 2, cq = lane & 3;  // mma fragment coordinates
@@ -1211,11 +846,28 @@ __global__ void __launch_bounds__(kMmaWarps * 32, 1) decode_mma_kernel(DecodePar
       for (int c = 0; c < MAXC; ++c)
         if (c < nchunks) kc[c] = load_chunk<FMT, false>(src + o_kv, src + o_ki, c);
     };
+    // the value records of a block into this warp's staging area, in flight
+    // while the warp works on the block before it
+    auto stage_v = [&](const uint8_t* blk) {
+      if (blk != nullptr) {
+        const int n_val = nchunks_v * 32;  // 16-byte pieces
+        for (int i = lane; i < n_val; i += 32) cp_async16(vstage + i * 16, blk + g.vval_off() + i * 16);
+        if constexpr (FMT == kFmtFp16) {
+          const int n_idx = nchunks_v * 16;
+          for (int i = lane; i < n_idx; i += 32)
+            cp_async16(vstage + nchunks_v * 512 + i * 16, blk + g.vidx_off() + i * 16);
+        }
+      }
+      cp_async_commit();
+    };
 
     const uint8_t* b_cur = block_of(t_lo);
     const uint8_t* b_n1 = block_of(t_lo + 1);
     prefetch_block(b_n1);
-    if (t_lo < sp_hi) load_k(b_cur);
+    if (t_lo < sp_hi) {
+      load_k(b_cur);
+      stage_v(b_cur);
+    }
 
     for (int gi = t_lo; gi < t_hi; ++gi) {
       float s[G];
@@ -1227,7 +879,6 @@ __global__ void __launch_bounds__(kMmaWarps * 32, 1) decode_mma_kernel(DecodePar
         const int64_t t0 = (int64_t)gi * 32;
         const bool ok = b_cur != nullptr;
         valid = ok && t0 + lane < uv.sparse_len;
-        const uint8_t* src = ok ? b_cur : g.pool;
         const uint8_t* b_n2 = block_of(gi + 2);
         prefetch_block(b_n2);
         if (valid) {
@@ -1239,19 +890,31 @@ __global__ void __launch_bounds__(kMmaWarps * 32, 1) decode_mma_kernel(DecodePar
               if (krem && c == nchunks - 1) keep_first(f, krem);
               score_g_chunk<G>(qb, f, chunk_idx<FMT>(kc[c]), s);
             }
-          // this token's kept values into its tile row (loaded now, when
-          // the key records are dead, to keep the registers down; the block
-          // is already in L2)
+        }
+        // this token's kept values (staged by cp.async) into its tile row
+        cp_async_wait_all();
+        __syncwarp();
+        if (valid) {
 #pragma unroll
           for (int c = 0; c < MAXC; ++c)
             if (c < nchunks_v) {
-              const Chunk<FMT> vc = load_chunk<FMT, false>(src + o_vv, src + o_vi, c);
+              Chunk<FMT> vc;
+              if constexpr (FMT == kFmtFp16) {
+                vc.v = lds_v4u(vstage + c * 512 + lane * 16);
+                vc.i = lds_v2u(vstage + nchunks_v * 512 + c * 256 + lane * 8);
+              } else {
+                vc.r = lds_v4u(vstage + c * 512 + lane * 16);
+              }
               uint32_t w[4];
               chunk_half_words<FMT>(vc, w);
               scatter_chunk(vrow, w, chunk_idx<FMT>(vc), (krem_v && c == nchunks_v - 1) ? krem_v : 8);
             }
         }
-        if (gi + 1 < sp_hi) load_k(b_n1);
+        __syncwarp();
+        if (gi + 1 < sp_hi) {
+          load_k(b_n1);
+          stage_v(b_n1);
+        }
         b_cur = b_n1;
         b_n1 = b_n2;
       } else {
@@ -1374,7 +1037,7 @@ __global__ void __launch_bounds__(kMmaWarps * 32, 1) decode_mma_kernel(DecodePar
       for (int w = 0; w < NW; ++w) {
         const float mw = red_m[w * G + hd];
         const float f = (mw == -INFINITY) ? 0.f : exp2f(mw - M);
-        const float* ob = reinterpret_cast<const float*>(base_ptr + (wbase - base) + w * kMmaWarpBytes);
+        const float* ob = reinterpret_cast<const float*>(base_ptr + (wbase - base) + w * kWarpBytes);
         tot = fmaf(f, ob[hd * kHeadDim + dd], tot);
         L = fmaf(f, red_l[w * G + hd], L);
       }
@@ -1478,7 +1141,6 @@ size_t one_head_smem(int maxc) {
   const int nw = maxc <= 8 ? decode_warps<8>() : decode_warps<16>();
   return (size_t)(1 + nw + 1) * kRegionBytes;
 }
-constexpr size_t kGqaSmem = 7 * kPairRegionBytes;
 
 template <typename K>
 int occupancy(K kernel, int threads, size_t smem) {
@@ -1502,14 +1164,14 @@ cudaError_t launch_t(const DecodeParams& p, int grid, cudaStream_t s) {
     }
     return launch_pdl(decode_kernel<MAXC, FMT>, dim3(grid), dim3(decode_warps<MAXC>() * 32), smem, s, p);
   } else {
-    constexpr size_t smem = mma_smem<G>();
+    constexpr size_t smem = mma_smem<G, MAXC>();
     if (!attr_set) {
       cudaError_t e = cudaFuncSetAttribute(decode_mma_kernel<G, MAXC, FMT>,
                                            cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
       if (e != cudaSuccess) return e;
       attr_set = true;
     }
-    return launch_pdl(decode_mma_kernel<G, MAXC, FMT>, dim3(grid), dim3(kMmaWarps * 32), smem, s, p);
+    return launch_pdl(decode_mma_kernel<G, MAXC, FMT>, dim3(grid), dim3(mma_warps<MAXC>() * 32), smem, s, p);
   }
 }
 
@@ -1527,11 +1189,11 @@ int decode_ctas_per_sm(int G, int k_slots) {
     return big ? occupancy(decode_kernel<16, kFmtFp16>, decode_warps<16>() * 32, one_head_smem(16))
                : occupancy(decode_kernel<8, kFmtFp16>, decode_warps<8>() * 32, one_head_smem(8));
   if (G == 2)
-    return big ? occupancy(decode_mma_kernel<2, 16, kFmtFp16>, kMmaWarps * 32, mma_smem<2>())
-               : occupancy(decode_mma_kernel<2, 8, kFmtFp16>, kMmaWarps * 32, mma_smem<2>());
+    return big ? occupancy(decode_mma_kernel<2, 16, kFmtFp16>, mma_warps<16>() * 32, mma_smem<2, 16>())
+               : occupancy(decode_mma_kernel<2, 8, kFmtFp16>, mma_warps<8>() * 32, mma_smem<2, 8>());
   if (G == 4)
-    return big ? occupancy(decode_mma_kernel<4, 16, kFmtFp16>, kMmaWarps * 32, mma_smem<4>())
-               : occupancy(decode_mma_kernel<4, 8, kFmtFp16>, kMmaWarps * 32, mma_smem<4>());
+    return big ? occupancy(decode_mma_kernel<4, 16, kFmtFp16>, mma_warps<16>() * 32, mma_smem<4, 16>())
+               : occupancy(decode_mma_kernel<4, 8, kFmtFp16>, mma_warps<8>() * 32, mma_smem<4, 8>());
   return 0;
 }
 

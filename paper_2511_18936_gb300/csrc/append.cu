@@ -3,6 +3,7 @@
 // Section 4.3; Section 5.1).
 #include <cuda_fp8.h>
 
+#include "sm100.h"
 #include "swan_internal.h"
 
 namespace swan {
@@ -111,114 +112,6 @@ __device__ __forceinline__ RowView row_view(const AppendParams& p, int64_t b, in
   return RowView{q.sparse_len, q.evict, q.n_b, q.buf_start, q.n_new, q.prune};
 }
 
-__device__ __forceinline__ float half_at(const uint4 (&xr)[16], int i) {
-  const uint4 w = xr[i >> 3];
-  const int q = (i >> 1) & 3;
-  const uint32_t word = q == 0 ? w.x : q == 1 ? w.y : q == 2 ? w.z : w.w;
-  const unsigned short bits = (i & 1) ? (unsigned short)(word >> 16) : (unsigned short)(word & 0xffffu);
-  return __half2float(__ushort_as_half(bits));
-}
-
-constexpr int kStageWords = 65;  // 64 words of fp16 pairs + 1 pad (bank skew)
-constexpr size_t kAppendSmem = 128 * 128 * sizeof(float) + kThreads * kStageWords * 4;
-
-// One CTA: one kv head (blockIdx.y), keys or values (blockIdx.z), 256 of the
-// B*T new vectors (one per thread).  R is staged in shared memory; each lane
-// computes its vector's 128 rotated coordinates in fp32 (32 at a time) and
-// rounds them to fp16.  Vectors that stay dense go to their ring slot;
-// vectors past the eviction point are pruned by their warp.
-__global__ void __launch_bounds__(kThreads, 1) append_kernel(AppendParams p) {
-  extern __shared__ __align__(16) unsigned char smem_raw[];
-  float* Rs = reinterpret_cast<float*>(smem_raw);
-  uint32_t* stage = reinterpret_cast<uint32_t*>(smem_raw + 128 * 128 * sizeof(float));
-
-  const int kind = blockIdx.z;
-  const int h = blockIdx.y;
-  const float* R = (kind ? p.R_vo : p.R_qk) + (size_t)h * kHeadDim * kHeadDim;
-  const __half* X = kind ? p.v_new : p.k_new;
-  __half* ring = kind ? p.ring_v : p.ring_k;
-
-  pdl_trigger();
-  stage_matrix(Rs, R);
-  pdl_wait();
-
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int64_t nvec = (int64_t)p.B * p.T;
-  const int64_t n = (int64_t)blockIdx.x * kThreads + threadIdx.x;
-  const int64_t b = n < nvec ? n / p.T : 0, j = n < nvec ? n % p.T : 0;
-  const RowView rv = row_view(p, b, 0);
-  const bool valid = n < nvec && j < rv.n_new;
-  uint4 xr[16];
-  if (valid) {
-    const uint4* src = reinterpret_cast<const uint4*>(X + (((size_t)b * p.H + h) * p.T + j) * kHeadDim);
-#pragma unroll
-    for (int i = 0; i < 16; ++i) xr[i] = __ldg(src + i);
-  } else {
-#pragma unroll
-    for (int i = 0; i < 16; ++i) xr[i] = make_uint4(0, 0, 0, 0);
-  }
-  __syncthreads();
-
-  const int64_t pos = (int64_t)rv.n_b + j;  // logical position in (buffer, new tokens)
-  const bool to_ring = valid && pos >= rv.evict;
-  __half* ring_row = nullptr;
-  if (to_ring) {
-    const int slot = (int)((rv.buf_start + pos) % p.cap);
-    ring_row = ring + (((size_t)b * p.H + h) * p.cap + slot) * kHeadDim;
-  }
-  uint32_t* my_stage = stage + threadIdx.x * kStageWords;
-
-#pragma unroll 1
-  for (int cb = 0; cb < 4; ++cb) {
-    float acc[32];
-#pragma unroll
-    for (int m = 0; m < 32; ++m) acc[m] = 0.f;
-#pragma unroll
-    for (int i = 0; i < kHeadDim; ++i) {
-      const float xi = half_at(xr, i);
-      const float4* Rrow = reinterpret_cast<const float4*>(Rs + i * kHeadDim + cb * 32);
-#pragma unroll
-      for (int q = 0; q < 8; ++q) {
-        const float4 r = Rrow[q];
-        acc[4 * q + 0] = fmaf(xi, r.x, acc[4 * q + 0]);
-        acc[4 * q + 1] = fmaf(xi, r.y, acc[4 * q + 1]);
-        acc[4 * q + 2] = fmaf(xi, r.z, acc[4 * q + 2]);
-        acc[4 * q + 3] = fmaf(xi, r.w, acc[4 * q + 3]);
-      }
-    }
-    uint32_t packed[16];
-#pragma unroll
-    for (int m = 0; m < 16; ++m) {
-      const unsigned short lo = __half_as_ushort(__float2half_rn(acc[2 * m]));
-      const unsigned short hi = __half_as_ushort(__float2half_rn(acc[2 * m + 1]));
-      packed[m] = (uint32_t)lo | ((uint32_t)hi << 16);
-      my_stage[cb * 16 + m] = packed[m];
-    }
-    if (to_ring) {
-      uint4* dst = reinterpret_cast<uint4*>(ring_row + cb * 32);
-#pragma unroll
-      for (int q = 0; q < 4; ++q)
-        dst[q] = make_uint4(packed[4 * q], packed[4 * q + 1], packed[4 * q + 2], packed[4 * q + 3]);
-    }
-  }
-  __syncwarp();
-
-  // Prune this warp's vectors that land past the eviction point.
-  const int64_t warp_first = (int64_t)blockIdx.x * kThreads + warp * 32;
-#pragma unroll 1
-  for (int v = 0; v < 32; ++v) {
-    const int64_t nv = warp_first + v;
-    if (nv >= nvec) break;
-    const int64_t bv = nv / p.T, jv = nv % p.T;
-    const RowView rvv = row_view(p, bv, 0);
-    if (jv >= rvv.n_new) continue;
-    const int64_t posv = (int64_t)rvv.n_b + jv;
-    if (posv >= rvv.evict) continue;
-    const uint32_t* row = stage + (warp * 32 + v) * kStageWords;
-    const uint2 raw = make_uint2(row[2 * lane], row[2 * lane + 1]);
-    warp_prune_store(raw, lane, kind, bv * p.H + h, rvv.sparse_len + posv, p.geom, p.status);
-  }
-}
 
 // Small appends (decode steps): one CTA per (kv head, K or V).  Phase 1
 // prunes the `evict_old` oldest buffered vectors of every sequence out of the
@@ -328,6 +221,162 @@ __global__ void transpose_r_kernel(const float* src, float* dst, int64_t mats) {
     d[(bx + r) * kHeadDim + by + threadIdx.x] = tile[threadIdx.x][r];
 }
 
+// ---------------------------------------------------------------------------
+// Bulk append with the rotation on the tensor cores.
+//   One CTA: 128 new vectors of one (row, kv head, K or V).  TMA brings the
+//   fp16 vectors (A: 128 x 128, K-major, 128-byte swizzle) and the split
+//   rotation R^T = R_hi^T + 2^-12 R_lo^T (B: two fp16 128 x 128 tiles); two
+//   tcgen05.mma chains (K = 16 each step) accumulate x R_hi and x R_lo in two
+//   128-column TMEM accumulators; warps 0-3 read them back (row = vector),
+//   form y = hi + 2^-12 lo in fp32, round to fp16 and stage the rows in
+//   shared memory (16-byte chunks XOR-swizzled by row); then all 8 warps
+//   write each vector to its ring slot or prune it (warp_prune_store).  The
+//   products are exact (fp16 x fp16) and summed in fp32; the split leaves
+//   2^-22 |R| per term, inside the fp32-dot bound of the CUDA-core path.
+// ---------------------------------------------------------------------------
+constexpr uint32_t kTcTile = 128 * 128 * 2;  // 32 KB: one fp16 128 x 128 tile
+constexpr size_t kTcSmem = 3 * kTcTile + 1024;
+constexpr uint64_t kTcWaitNs = 2000000000ull;
+
+// byte offset of (row v, coordinate c) in the staged fp16 rows
+__device__ __forceinline__ uint32_t staged_off(int v, int c) {
+  return (uint32_t)v * 256u + ((uint32_t)((c >> 3) ^ (v & 15)) << 4) + (uint32_t)(c & 7) * 2u;
+}
+
+__global__ void __launch_bounds__(kThreads, 1) append_tc_kernel(const __grid_constant__ CUtensorMap xk,
+                                                                 const __grid_constant__ CUtensorMap xv,
+                                                                 const __grid_constant__ CUtensorMap rhi,
+                                                                 const __grid_constant__ CUtensorMap rlo,
+                                                                 AppendParams p, int r_slice0) {
+  using namespace sm100;
+  extern __shared__ __align__(1024) unsigned char smem_raw[];
+  __shared__ __align__(8) uint64_t bars[2];
+  __shared__ uint32_t tmem_slot;
+  __shared__ int failed;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int kind = blockIdx.z, h = blockIdx.y;
+  const int tiles_per_row = (p.T + 127) / 128;
+  const int b = blockIdx.x / tiles_per_row, j0 = (blockIdx.x % tiles_per_row) * 128;
+  const RowView rv = row_view(p, b, 0);
+  pdl_trigger();
+  if (j0 >= rv.n_new) return;  // no new token of this row in the tile (uniform in the CTA)
+
+  const uint32_t raw = smem_u32(smem_raw);
+  const uint32_t ta = (raw + 1023u) & ~1023u;  // A, then the staged rows
+  const uint32_t tb_hi = ta + kTcTile, tb_lo = tb_hi + kTcTile;
+  unsigned char* stage = smem_raw + (ta - raw);
+  const uint32_t full = smem_u32(&bars[0]), done = smem_u32(&bars[1]);
+  if (threadIdx.x == 0) {
+    mbar_init(full, 1);
+    mbar_init(done, 1);
+    failed = 0;
+    fence_barrier_init();
+  }
+  if (warp == 1) tmem_alloc(smem_u32(&tmem_slot), 256);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = tmem_slot;
+  pdl_wait();
+
+  if (threadIdx.x == 0) {
+    const CUtensorMap* xm = kind ? &xv : &xk;
+    const int slice = r_slice0 + kind * p.H + h;
+    mbar_arrive_expect_tx(full, 3 * kTcTile);
+    tma_load_4d(ta, xm, full, 0, j0, h, b);
+    tma_load_4d(ta + kTcTile / 2, xm, full, 64, j0, h, b);
+    tma_load_3d(tb_hi, &rhi, full, 0, 0, slice);
+    tma_load_3d(tb_hi + kTcTile / 2, &rhi, full, 64, 0, slice);
+    tma_load_3d(tb_lo, &rlo, full, 0, 0, slice);
+    tma_load_3d(tb_lo + kTcTile / 2, &rlo, full, 64, 0, slice);
+    if (!mbar_wait(full, 0, kTcWaitNs)) {
+      atomicOr(p.status, kStatusTimeout);
+      failed = 1;
+    } else {
+      tc_fence_after();
+      constexpr uint32_t idesc = idesc_f16_f32(128, 128, 0, 0);
+#pragma unroll
+      for (int kk = 0; kk < 8; ++kk) {
+        const uint32_t off = (uint32_t)(kk >> 2) * (kTcTile / 2) + (uint32_t)(kk & 3) * 32;
+        const uint64_t da = sdesc_sw128(ta + off, 16, 1024);
+        mma_f16(tmem, da, sdesc_sw128(tb_hi + off, 16, 1024), idesc, kk > 0);
+        mma_f16(tmem + 128, da, sdesc_sw128(tb_lo + off, 16, 1024), idesc, kk > 0);
+      }
+    }
+    mma_commit(done);
+  }
+  __syncwarp();
+
+  // ---- TMEM -> fp16 rows in shared memory (A's tile, free once the MMAs are done)
+  if (warp < 4) {
+    if (!mbar_wait(done, 0, kTcWaitNs)) {
+      atomicOr(p.status, kStatusTimeout);
+      failed = 1;
+    }
+    tc_fence_after();
+  }
+  __syncthreads();
+  const bool ok = failed == 0;  // uniform in the CTA
+  if (warp < 4 && ok) {
+    const int v = 32 * warp + lane;
+    const uint32_t taddr = tmem + ((uint32_t)(32 * warp) << 16);
+#pragma unroll 1
+    for (int c = 0; c < 4; ++c) {
+      uint32_t hi[32], lo[32];
+      tmem_ld32(taddr + c * 32, hi);
+      tmem_ld32(taddr + 128 + c * 32, lo);
+      tmem_wait_ld();
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        uint32_t w[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const int m = 8 * q + 2 * e;
+          const float y0 = fmaf(__uint_as_float(lo[m]), 1.f / 4096.f, __uint_as_float(hi[m]));
+          const float y1 = fmaf(__uint_as_float(lo[m + 1]), 1.f / 4096.f, __uint_as_float(hi[m + 1]));
+          w[e] = (uint32_t)__half_as_ushort(__float2half_rn(y0)) |
+                 ((uint32_t)__half_as_ushort(__float2half_rn(y1)) << 16);
+        }
+        *reinterpret_cast<uint4*>(stage + staged_off(v, c * 32 + q * 8)) = make_uint4(w[0], w[1], w[2], w[3]);
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) tmem_dealloc(tmem, 256);
+  if (!ok) return;
+
+  // ---- ring insert or prune, one vector per warp at a time
+  __half* ring = kind ? p.ring_v : p.ring_k;
+  const int64_t unit = (int64_t)b * p.H + h;
+  for (int v = warp; v < 128; v += kWarpsPerCta) {
+    const int j = j0 + v;
+    if (j >= rv.n_new) break;
+    const uint2 raw2 = *reinterpret_cast<const uint2*>(stage + staged_off(v, 4 * lane));
+    const int64_t pos = (int64_t)rv.n_b + j;
+    if (pos < rv.evict) {
+      warp_prune_store(raw2, lane, kind, unit, rv.sparse_len + pos, p.geom, p.status);
+    } else {
+      const int slot = (int)((rv.buf_start + pos) % p.cap);
+      reinterpret_cast<uint2*>(ring + (unit * p.cap + slot) * kHeadDim)[lane] = raw2;
+    }
+  }
+}
+
+__global__ void split_r_kernel(const float* R_qk, const float* R_vo, __half* hi, __half* lo, int H) {
+  // blockIdx.y: layer * 2 + kind; blockIdx.x: head; threads over (n, k)
+  const int lk = blockIdx.y, kind = lk & 1, layer = lk >> 1, h = blockIdx.x;
+  const float* R = (kind ? R_vo : R_qk) + ((size_t)layer * H + h) * kHeadDim * kHeadDim;
+  const size_t dst = ((size_t)lk * H + h) * kHeadDim * kHeadDim;
+  for (int e = threadIdx.x; e < kHeadDim * kHeadDim; e += blockDim.x) {
+    const int n = e >> 7, k = e & 127;
+    const float r = R[k * kHeadDim + n];
+    const __half rh = __float2half_rn(r);
+    hi[dst + e] = rh;
+    lo[dst + e] = __float2half_rn((r - __half2float(rh)) * 4096.f);
+  }
+}
+
 __global__ void scatter_pages_kernel(const int2* pairs, int n, int32_t* table) {
   const int i = blockIdx.x * blockDim.x + threadIdx.x;
   if (i < n) {
@@ -338,23 +387,29 @@ __global__ void scatter_pages_kernel(const int2* pairs, int n, int32_t* table) {
 
 }  // namespace
 
+cudaError_t launch_append_tc(const AppendParams& p, const CUtensorMap* maps, int r_slice0, cudaStream_t s) {
+  static bool attr_set = false;
+  if (!attr_set) {
+    cudaError_t e = cudaFuncSetAttribute(append_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)kTcSmem);
+    if (e != cudaSuccess) return e;
+    attr_set = true;
+  }
+  const int tiles = p.B * ((p.T + 127) / 128);
+  return launch_pdl(append_tc_kernel, dim3((unsigned)tiles, (unsigned)p.H, 2), dim3(kThreads), kTcSmem, s,
+                    maps[0], maps[1], maps[2], maps[3], p, r_slice0);
+}
+
+cudaError_t launch_split_r(const float* R_qk, const float* R_vo, __half* hi, __half* lo, int layers, int H,
+                           cudaStream_t s) {
+  split_r_kernel<<<dim3((unsigned)H, (unsigned)(2 * layers)), 256, 0, s>>>(R_qk, R_vo, hi, lo, H);
+  return cudaGetLastError();
+}
+
 cudaError_t launch_scatter_pages(const int2* pairs, int n, int32_t* table, cudaStream_t s) {
   if (n <= 0) return cudaSuccess;
   scatter_pages_kernel<<<(n + 255) / 256, 256, 0, s>>>(pairs, n, table);
   return cudaGetLastError();
-}
-
-cudaError_t launch_append(const AppendParams& p, cudaStream_t s) {
-  static bool attr_set = false;
-  if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(append_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)kAppendSmem);
-    if (e != cudaSuccess) return e;
-    attr_set = true;
-  }
-  const int64_t nvec = (int64_t)p.B * p.T;
-  dim3 grid((unsigned)((nvec + kThreads - 1) / kThreads), (unsigned)p.H, 2);
-  return launch_pdl(append_kernel, grid, dim3(kThreads), kAppendSmem, s, p);
 }
 
 cudaError_t launch_append_small(const AppendParams& p, int evict_old, cudaStream_t s) {

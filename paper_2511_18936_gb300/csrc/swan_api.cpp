@@ -83,6 +83,9 @@ struct swan_ctx {
   float* R_qk = nullptr;
   float* R_vo = nullptr;   // == R_qk when the caller passed NULL
   float* R_voT = nullptr;  // transposed copy for the rotate-back
+  __half* R_hi = nullptr;  // split rotations for the tensor-core append: [layer][2][H][n][k] fp16
+  __half* R_lo = nullptr;
+  CUtensorMap r_maps[2];   // TMA maps over R_hi, R_lo
   uint8_t* pool = nullptr;
   int32_t* page_table = nullptr;
   __half* ring_k = nullptr;
@@ -116,6 +119,8 @@ void free_all(swan_ctx* c) {
   if (c->R_vo && c->R_vo != c->R_qk) cudaFree(c->R_vo);
   cudaFree(c->R_qk);
   cudaFree(c->R_voT);
+  cudaFree(c->R_hi);
+  cudaFree(c->R_lo);
   cudaFree(c->pool);
   cudaFree(c->page_table);
   cudaFree(c->ring_k);
@@ -506,6 +511,8 @@ swan_status swan_init(swan_ctx** out, const swan_config* cfg, const float* R_qk,
   if (s == SWAN_OK) s = dev_alloc(c, (void**)&c->R_qk, rmat * sizeof(float), "R_qk");
   if (s == SWAN_OK && R_vo) s = dev_alloc(c, (void**)&c->R_vo, rmat * sizeof(float), "R_vo");
   if (s == SWAN_OK) s = dev_alloc(c, (void**)&c->R_voT, rmat * sizeof(float), "R_vo^T");
+  if (s == SWAN_OK) s = dev_alloc(c, (void**)&c->R_hi, 2 * rmat * sizeof(__half), "split R (hi)");
+  if (s == SWAN_OK) s = dev_alloc(c, (void**)&c->R_lo, 2 * rmat * sizeof(__half), "split R (lo)");
   if (s == SWAN_OK)
     s = dev_alloc(c, (void**)&c->pool, (size_t)c->num_pages * (size_t)c->page_bytes, "page pool");
   if (s == SWAN_OK) s = dev_alloc(c, (void**)&c->page_table, pt_elems * sizeof(int32_t), "page table");
@@ -541,6 +548,7 @@ swan_status swan_init(swan_ctx** out, const swan_config* cfg, const float* R_qk,
   if (e == cudaSuccess && R_vo)
     e = cudaMemcpyAsync(c->R_vo, R_vo, rmat * sizeof(float), cudaMemcpyDeviceToDevice, st);
   if (e == cudaSuccess) e = launch_transpose_r(c->R_vo, c->R_voT, (int64_t)C.num_layers * C.n_kv_heads, st);
+  if (e == cudaSuccess) e = launch_split_r(c->R_qk, c->R_vo, c->R_hi, c->R_lo, C.num_layers, C.n_kv_heads, st);
   if (e == cudaSuccess)
     e = cudaMemcpyAsync(c->page_table, pt.data(), pt_elems * sizeof(int32_t), cudaMemcpyHostToDevice, st);
   if (e == cudaSuccess) e = cudaMemsetAsync(c->pool, 0, (size_t)c->num_pages * (size_t)c->page_bytes, st);
@@ -554,6 +562,28 @@ swan_status swan_init(swan_ctx** out, const swan_config* cfg, const float* R_qk,
     free_all(c);
     delete c;
     return r;
+  }
+  {
+    EncodeTiledFn enc = tensor_map_encoder();
+    CUresult r = CUDA_ERROR_NOT_FOUND;
+    if (enc) {
+      const cuuint64_t dims[3] = {128, 128, (cuuint64_t)2 * C.num_layers * C.n_kv_heads};
+      const cuuint64_t strides[2] = {256, 128 * 256};
+      const cuuint32_t box[3] = {64, 128, 1}, estr[3] = {1, 1, 1};
+      r = enc(&c->r_maps[0], CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 3, c->R_hi, dims, strides, box, estr,
+              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+      if (r == CUDA_SUCCESS)
+        r = enc(&c->r_maps[1], CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 3, c->R_lo, dims, strides, box, estr,
+                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    }
+    if (r != CUDA_SUCCESS) {
+      swan_status rs = fail(SWAN_ERR_CUDA, "encoding the rotation tensor maps failed (%d)", (int)r);
+      free_all(c);
+      delete c;
+      return rs;
+    }
   }
   *out = c;
   return SWAN_OK;
@@ -605,6 +635,8 @@ swan_status append_rows(swan_ctx* c, int layer, const void* k_new, const void* v
   if (T < 0) return fail(SWAN_ERR_INVALID_ARG, "T %d < 0", T);
   if (T == 0) return SWAN_OK;
   if (!k_new || !v_new) return fail(SWAN_ERR_INVALID_ARG, "k_new or v_new is NULL");
+  if ((uintptr_t)k_new % 16 || (uintptr_t)v_new % 16)
+    return fail(SWAN_ERR_INVALID_ARG, "k_new and v_new must be 16-byte aligned");
   if ((int64_t)c->cfg.batch * T > (int64_t)INT32_MAX * 128) return fail(SWAN_ERR_INVALID_ARG, "T too large");
   LayerState& L = c->layers[layer];
   const int B = c->cfg.batch;
@@ -635,13 +667,29 @@ swan_status append_rows(swan_ctx* c, int layer, const void* k_new, const void* v
     same = same && Tb[b] == T;
   }
   if (most_tokens == 0) return SWAN_OK;
-  // pages for the tokens that reach the sparse history (paged pool)
-  if ((s = grow_pages(c, layer, new_len)) != SWAN_OK) return s;
 
   // Decode-step appends (few vectors per head) run as one launch that evicts
   // and inserts; bulk appends as a pruning launch for the evicted buffered
-  // tokens followed by the rotation launch.
+  // tokens followed by the rotation launch (tensor cores; TMA maps of this
+  // call's keys and values, encoded before anything changes).
   const bool small = (int64_t)B * T <= kSmallAppendVectors && (int64_t)B * most_old <= kSmallAppendVectors;
+  CUtensorMap maps[4];
+  if (!small) {
+    EncodeTiledFn enc = tensor_map_encoder();
+    const cuuint64_t dims[4] = {128, (cuuint64_t)T, (cuuint64_t)c->cfg.n_kv_heads, (cuuint64_t)B};
+    const cuuint64_t strides[3] = {256, (cuuint64_t)T * 256, (cuuint64_t)T * 256 * c->cfg.n_kv_heads};
+    const cuuint32_t box[4] = {64, 128, 1, 1}, estr[4] = {1, 1, 1, 1};
+    CUresult r = enc ? CUDA_SUCCESS : CUDA_ERROR_NOT_FOUND;
+    for (int kk = 0; kk < 2 && r == CUDA_SUCCESS; ++kk)
+      r = enc(&maps[kk], CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 4, const_cast<void*>(kk ? v_new : k_new), dims,
+              strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) return fail(SWAN_ERR_INVALID_ARG, "k_new / v_new: tensor-map encoding failed (%d)", (int)r);
+    maps[2] = c->r_maps[0];
+    maps[3] = c->r_maps[1];
+  }
+  // pages for the tokens that reach the sparse history (paged pool)
+  if ((s = grow_pages(c, layer, new_len)) != SWAN_OK) return s;
   const std::vector<SeqState> before = L.seq;
   const SeqInfo* rows_dev = nullptr;
   if (!same) {
@@ -702,7 +750,8 @@ swan_status append_rows(swan_ctx* c, int layer, const void* k_new, const void* v
     s = launch(c, SWAN_KERNEL_APPEND, "append_small kernel",
                [&] { return launch_append_small(p, most_old, c->stream); });
   else
-    s = launch(c, SWAN_KERNEL_APPEND, "append kernel", [&] { return launch_append(p, c->stream); });
+    s = launch(c, SWAN_KERNEL_APPEND, "append kernel",
+               [&] { return launch_append_tc(p, maps, layer * 2 * c->cfg.n_kv_heads, c->stream); });
   if (s != SWAN_OK) return s;
 
   for (int b = 0; b < B; ++b) {

@@ -25,6 +25,7 @@
 // the first ceil(k_active / 8) chunks: a contiguous prefix of each region.
 #pragma once
 
+#include <cuda.h>
 #include <cuda_fp16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
@@ -42,6 +43,7 @@ constexpr float kLazyRescale = 8.0f;
 // Device status word bits (set instead of faulting on inconsistent state).
 constexpr unsigned kStatusPageRange = 1u;
 constexpr unsigned kStatusRingRange = 2u;
+constexpr unsigned kStatusTimeout = 4u;  // a bounded barrier wait gave up
 
 constexpr int kFmtFp16 = 0;  // fp16 values
 constexpr int kFmtFp8 = 1;   // E4M3 values
@@ -213,7 +215,19 @@ __device__ __forceinline__ void stage_matrix(float* dst, const float* src) {
 #endif
 
 // Launchers (return the launch error, if any).
-cudaError_t launch_append(const AppendParams& p, cudaStream_t s);
+// Bulk append with the rotation on the tensor cores: maps[0..1] the new keys
+// and values ([B][H][T][128] fp16, 64 x 128-vector boxes), maps[2..3] the
+// split rotations (see launch_split_r), r_slice0 = layer * 2 * H.
+cudaError_t launch_append_tc(const AppendParams& p, const CUtensorMap* maps, int r_slice0, cudaStream_t s);
+// R_hi^T and R_lo^T (fp16, [layer][2 kinds][H][n][k]) from fp32 R: hi = fp16(R),
+// lo = fp16((R - hi) * 2^12); kind 0 from R_qk, 1 from R_vo.
+cudaError_t launch_split_r(const float* R_qk, const float* R_vo, __half* hi, __half* lo, int layers, int H,
+                           cudaStream_t s);
+// cuTensorMapEncodeTiled from the driver (null if unavailable).
+using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                   const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                   CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+EncodeTiledFn tensor_map_encoder();
 // Eviction of `evict_old` buffered tokens and insertion of T new ones in one
 // launch; for small batch * T (decode steps).
 cudaError_t launch_append_small(const AppendParams& p, int evict_old, cudaStream_t s);

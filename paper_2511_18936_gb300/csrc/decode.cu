@@ -641,11 +641,19 @@ template <int MAXC>
 __host__ __device__ constexpr uint32_t mma_warp_bytes() {
   return kVTileBytes + kPTileBytes + (uint32_t)MAXC * 768;
 }
+// 8 warps: the registers (~240 a thread) allow no more without spills, and a
+// sweep on the GB300 measured 8 < 10 < 12 warps in time (0.480, 0.491,
+// 0.565 ms on the GQA 131k layer).
 template <int MAXC>
-__host__ __device__ constexpr int mma_warps() { return MAXC <= 8 ? 8 : 6; }
+__host__ __device__ constexpr int mma_warps() { return 8; }
+// q' replicated in 32 / G copies per coordinate: [128][32 / G][G] fp32, 16 KB.
+// A G-float gather is served in phases of 32 / G lanes (16-byte loads: 8
+// lanes, 8-byte loads: 16), and the lanes of a phase read distinct copies,
+// so they never share a bank.
+constexpr uint32_t kQrepBytes = kHeadDim * 32 * 4;
 template <int G, int MAXC>
 __host__ __device__ constexpr size_t mma_smem() {
-  return (size_t)kHeadDim * 32 * G * 4 + (size_t)mma_warps<MAXC>() * mma_warp_bytes<MAXC>() + 16;
+  return (size_t)kQrepBytes + (size_t)mma_warps<MAXC>() * mma_warp_bytes<MAXC>() + 16;
 }
 
 __device__ __forceinline__ void cp_async16(uint32_t dst, const void* src) {
@@ -723,7 +731,7 @@ __device__ __forceinline__ void score_g_chunk(uint32_t qb, const float (&f)[8], 
 #pragma unroll
   for (int e = 0; e < 8; ++e) {
     const uint32_t w = e < 4 ? ix.x : ix.y;
-    const uint32_t a = qb + ((w >> (8 * (e & 3))) & 0x7fu) * (uint32_t)(128 * G);
+    const uint32_t a = qb + ((w >> (8 * (e & 3))) & 0x7fu) * 128u;
     if constexpr (G == 4) {
       const float4 q = lds4(a);
       s[0] = fmaf(q.x, f[e], s[0]);
@@ -762,13 +770,13 @@ __global__ void __launch_bounds__(mma_warps<MAXC>() * 32, 1) decode_mma_kernel(D
   const uint32_t raw = (uint32_t)__cvta_generic_to_shared(smem_raw);
   const uint32_t base = (raw + 15u) & ~15u;
   unsigned char* base_ptr = smem_raw + (base - raw);
-  float* qrep = reinterpret_cast<float*>(base_ptr);                         // [128][32][G]
-  const uint32_t wbase = base + kHeadDim * 32 * G * 4;                      // per-warp regions
+  float* qrep = reinterpret_cast<float*>(base_ptr);                         // [128][32/G][G]
+  const uint32_t wbase = base + kQrepBytes;                                 // per-warp regions
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t vtile = wbase + warp * kWarpBytes;                         // [32][272 B] fp16
   float* ptile_f = reinterpret_cast<float*>(base_ptr + (vtile + kVTileBytes - base));  // [G][32] fp32
   const uint32_t vstage = vtile + kVTileBytes + kPTileBytes;                  // value records, next block
-  const uint32_t qb = base + lane * (G * 4);
+  const uint32_t qb = base + (lane & (32 / G - 1)) * (G * 4);  // this lane's copy
   const uint32_t vrow = vtile + lane * kVRowBytes;
   const int gq = lane >> 2, cq = lane & 3;  // mma fragment coordinates
 
@@ -803,8 +811,8 @@ __global__ void __launch_bounds__(mma_warps<MAXC>() * 32, 1) decode_mma_kernel(D
     const int32_t* ptab = g.page_table + u * g.pages_per_unit;
 
     __syncthreads();  // the previous segment is done with q'
-    for (int i = threadIdx.x; i < kHeadDim * 32 * G; i += NT) {
-      const int c = i / (32 * G), j = i % G;
+    for (int i = threadIdx.x; i < kHeadDim * 32; i += NT) {
+      const int c = i / 32, j = i % G;  // 32 floats per coordinate: 32 / G copies of G heads
       qrep[i] = __ldg(p.qprime + ((b * p.H_q + h * G + j) * kHeadDim + c));
     }
     __syncthreads();
@@ -934,7 +942,7 @@ __global__ void __launch_bounds__(mma_warps<MAXC>() * 32, 1) decode_mma_kernel(D
             const float f[8] = {a.x, a.y, bb.x, bb.y, cc.x, cc.y, d.x, d.y};
 #pragma unroll
             for (int e = 0; e < 8; ++e) {
-              const uint32_t qa = qb + (uint32_t)(c * 8 + e) * (128 * G);
+              const uint32_t qa = qb + (uint32_t)(c * 8 + e) * 128u;
               if constexpr (G == 4) {
                 const float4 q = lds4(qa);
                 s[0] = fmaf(q.x, f[e], s[0]);

@@ -134,16 +134,18 @@ swan_status swan_set_kv(swan_ctx* ctx, int k_active, int k_active_v);
 /*
  * Append T tokens to every sequence of one layer (Algorithm 1, generalised
  * to T tokens at once).
- *   k_new, v_new: device fp16 [batch][n_kv_heads][T][d], post-RoPE keys and
- *   unrotated values.  The library rotates them: k_hat = k R_qk,
- *   v_hat = v R_vo (fp32 arithmetic, rounded to fp16 round-to-nearest-even).
+ *   k_new, v_new: device fp16 [batch][n_kv_heads][T][d], 16-byte aligned,
+ *   post-RoPE keys and unrotated values.  The library rotates them:
+ *   k_hat = k R_qk, v_hat = v R_vo, to fp32 accuracy (decode-step appends on
+ *   the CUDA cores; bulk appends on the tensor cores with R split into fp16
+ *   hi + 2^-12 lo parts), rounded to fp16 round-to-nearest-even.
  * If buffer_count + T > buffer_cap, the oldest (buffer_count + T - buffer_cap)
  * vectors of (buffer, then new tokens) are pruned to their k_store
  * largest-magnitude coordinates (ties to the lower index; keys and values
  * separately) and appended to the sparse history, in order; the rest stay
  * dense in the buffer.  T == 0 is a no-op.
- * Errors: INVALID_ARG (layer, T < 0, NULL), CAPACITY (sparse + buffer would
- * exceed max_seq), STATE, CUDA.
+ * Errors: INVALID_ARG (layer, T < 0, NULL, misaligned), CAPACITY (sparse +
+ * buffer would exceed max_seq, or the page pool is exhausted), STATE, CUDA.
  */
 swan_status swan_append(swan_ctx* ctx, int layer, const void* k_new,
                         const void* v_new, int T);
@@ -244,8 +246,10 @@ swan_status swan_debug_export_seq(swan_ctx* ctx, int layer, int b, int what, voi
 /*
  * Synchronise the stream and read the device status word that kernels set
  * when a device-side consistency check fails (for instance a page-table
- * entry out of range); such a kernel skips the access instead of faulting.
- * Returns OK, DEVICE_CHECK (and clears the word), STATE or CUDA.
+ * entry out of range; such a kernel skips the access instead of faulting) or
+ * a bounded wait of a tensor-core pipeline gave up (2 s; the launch's
+ * results are then invalid).  Returns OK, DEVICE_TIMEOUT or DEVICE_CHECK
+ * (and clears the word), STATE or CUDA.
  */
 swan_status swan_check(swan_ctx* ctx);
 

@@ -1093,6 +1093,8 @@ swan_status swan_check(swan_ctx* c) {
   if (word) {
     e = cudaMemset(c->status, 0, sizeof(unsigned));
     if (e != cudaSuccess) return cuda_fail(c, e, "cudaMemset");
+    if (word & kStatusTimeout)
+      return fail(SWAN_ERR_DEVICE_TIMEOUT, "a tensor-core pipeline wait gave up (status word 0x%x)", word);
     return fail(SWAN_ERR_DEVICE_CHECK, "device status word 0x%x", word);
   }
   return SWAN_OK;

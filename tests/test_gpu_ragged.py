@@ -197,3 +197,46 @@ def test_page_pool_shared_by_rows():
     assert ctx.lengths(0) == (ref.sparse_lens, ref.buffer_lens)
     ctx.check()
     ctx.close()
+
+
+def test_bulk_append_tiles_and_alignment():
+    """Bulk appends whose token count leaves a partial 128-vector tile (T = 129
+    and T = 255 per row, rows taking different counts), then a decode; and a
+    misaligned input is refused before anything changes."""
+    import torch
+
+    from paper_2511_18936_gb300 import swan
+    B, H, G = 3, 2, 2
+    R, Rv = _rot(H, 70), _rot(H, 70, synth.T_R_VO)
+    k, v = _kv(B, H, 400, seed=71)
+    q = _q(B, H * G, seed=72)
+    ops = [("append", k[:, :, :129].copy(), v[:, :, :129].copy(), [129, 128, 1]), ("decode", q),
+           ("append", k[:, :, 129:384].copy(), v[:, :, 129:384].copy(), [255, 0, 200]), ("decode", q)]
+    ctx, ref, _ = run_ragged(ops, R, Rv, B=B, H_kv=H, G=G, k_store=48, cap=16, max_seq=400, page_tokens=64)
+    before = ctx.lengths(0)
+    buf = torch.from_numpy(np.concatenate([k[:, :, 384:], k[:, :, 384:]], axis=2)).cuda()
+    mis = buf.view(-1)[1:1 + B * H * 8 * D].view(B, H, 8, D)  # 2-byte offset
+    with pytest.raises(swan.SwanError) as e:
+        ctx.append(0, mis, mis)
+    assert e.value.status == swan.ERR_INVALID_ARG and "aligned" in str(e.value)
+    assert ctx.lengths(0) == before
+    ctx.check()
+    ctx.close()
+
+
+def test_ragged_fp8_separate_counts_and_pool():
+    """Everything at once: rows of different lengths, E4M3 values, keys and
+    values keeping different counts, a shared page pool, grouped-query heads."""
+    B, H, G, P = 4, 2, 4, 32
+    R, Rv = _rot(H, 80), _rot(H, 80, synth.T_R_VO)
+    k, v = _kv(B, H, 900, seed=81)
+    q = _q(B, H * G, seed=82, scale=2.0)
+    pool = H * (900 // P + 2) * 3
+    ops = [("append", k[:, :, :600].copy(), v[:, :, :600].copy(), [600, 17, 0, 333]), ("decode", q),
+           ("set_k", 40, 12), ("decode", q),
+           ("append", k[:, :, 600:601].copy(), v[:, :, 600:601].copy(), [1, 1, 0, 1]), ("decode", q),
+           ("reset", 0), ("append", k[:, :, 601:900].copy(), v[:, :, 601:900].copy(), [299, 0, 299, 0]),
+           ("decode", q), ("flush",), ("decode", q)]
+    ctx, ref, _ = run_ragged(ops, R, Rv, B=B, H_kv=H, G=G, k_store=40, cap=24, max_seq=900, page_tokens=P,
+                             value_format="fp8_e4m3", k_store_v=24, pool_pages=pool)
+    ctx.close()

@@ -313,6 +313,13 @@ swan_status upload_rows(swan_ctx* c, int layer, const std::vector<SeqInfo>& rows
   return SWAN_OK;
 }
 
+// Fewest 32-token groups a decode CTA takes: a small cache is split over
+// fewer CTAs so that each one's fixed cost (staging q', the merge) and the
+// final combine over the CTAs' partials stay small next to its groups
+// (swept on the GB300 over 1..16 for one head at 1088 tokens: decode 39.7 us
+// at 1, 23.8 us at 8).
+constexpr int64_t kMinGroupsPerCta = 8;
+
 // Work of one unit segment of a decode CTA beyond its groups (staging q',
 // the merge, the rotate-back, and the pipeline start of every warp's short
 // run), in 32-token groups; measured on the ragged serving batch (a sweep of
@@ -868,7 +875,8 @@ swan_status swan_decode(swan_ctx* c, int layer, const void* q, void* out) {
       prefix += groups[b];
     }
     total = prefix * c->cfg.n_kv_heads;
-    const std::vector<int64_t> starts = balanced_starts(groups, c->cfg.n_kv_heads, c->decode_ctas);
+    const std::vector<int64_t> starts = balanced_starts(
+        groups, c->cfg.n_kv_heads, std::min<int64_t>(c->decode_ctas, std::max<int64_t>(1, total / kMinGroupsPerCta)));
     ragged_grid = (int64_t)starts.size() - 1;
     if ((s = upload_rows(c, layer, rows, &starts)) != SWAN_OK) return s;
     rows_dev = rows_of(c, layer);
@@ -876,7 +884,7 @@ swan_status swan_decode(swan_ctx* c, int layer, const void* q, void* out) {
   }
   int64_t range = 1, grid = 0;
   if (total > 0) {
-    const int64_t ctas = std::min<int64_t>(c->decode_ctas, total);
+    const int64_t ctas = std::min<int64_t>(c->decode_ctas, std::max<int64_t>(1, total / kMinGroupsPerCta));
     range = (total + ctas - 1) / ctas;
     grid = starts_dev ? ragged_grid : (total + range - 1) / range;
   }

@@ -83,7 +83,7 @@ def measured_peaks():
 def decode_kernel_traffic(workload: str, values: str = "fp16", variant: str = ""):
     """DRAM bytes per decode-kernel launch from the committed ncu summary, if
     it was taken on the current kernel source (else None)."""
-    src = os.path.join(ROOT, "paper_2511_18936_gb300", "csrc", "decode.cu")
+    src = os.path.join(ROOT, "paper_2511_18936_gb300", "csrc", "decode_kernels.cuh")
     digest = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
     text = None
     suffix = ("" if values == "fp16" else "-fp8") + variant
@@ -95,7 +95,7 @@ def decode_kernel_traffic(workload: str, values: str = "fp16", variant: str = ""
             continue
     if text is None:
         return None
-    m_src = re.search(r"decode\.cu sha256\[:16\]:\s*([0-9a-f]{16})", text)
+    m_src = re.search(r"decode_kernels\.cuh sha256\[:16\]:\s*([0-9a-f]{16})", text)
     m_tr = re.search(r"dram bytes per launch:\s*([0-9.eE+]+)", text)
     if not m_src or not m_tr or m_src.group(1) != digest:
         return None

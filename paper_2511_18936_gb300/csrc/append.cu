@@ -388,13 +388,8 @@ __global__ void scatter_pages_kernel(const int2* pairs, int n, int32_t* table) {
 }  // namespace
 
 cudaError_t launch_append_tc(const AppendParams& p, const CUtensorMap* maps, int r_slice0, cudaStream_t s) {
-  static bool attr_set = false;
-  if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(append_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)kTcSmem);
-    if (e != cudaSuccess) return e;
-    attr_set = true;
-  }
+  cudaError_t e = ensure_smem<append_tc_kernel>(kTcSmem);
+  if (e != cudaSuccess) return e;
   const int tiles = p.B * ((p.T + 127) / 128);
   return launch_pdl(append_tc_kernel, dim3((unsigned)tiles, (unsigned)p.H, 2), dim3(kThreads), kTcSmem, s,
                     maps[0], maps[1], maps[2], maps[3], p, r_slice0);
@@ -413,14 +408,9 @@ cudaError_t launch_scatter_pages(const int2* pairs, int n, int32_t* table, cudaS
 }
 
 cudaError_t launch_append_small(const AppendParams& p, int evict_old, cudaStream_t s) {
-  static bool attr_set = false;
   constexpr size_t smem = 128 * 128 * sizeof(float);
-  if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(append_small_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)smem);
-    if (e != cudaSuccess) return e;
-    attr_set = true;
-  }
+  cudaError_t e = ensure_smem<append_small_kernel>(smem);
+  if (e != cudaSuccess) return e;
   // enough sequences per CTA for one vector per warp and phase
   const int per = max(p.T, evict_old);
   const int bpc = max(1, kWarpsPerCta / max(per, 1));

@@ -1,0 +1,1153 @@
+// Device code of the decode path (Algorithm 1, attention part; Section 4.3):
+// the split decode kernels with the fused combine and rotate-back (Appendix
+// A.1, Lemma 2), the query rotation and the empty-cache combine.  Included
+// by decode.cu, which holds the host launchers; this file is what the
+// committed profiles' source hash covers.
+#pragma once
+
+#include <cuda_fp8.h>
+
+#include "swan_internal.h"
+
+namespace swan {
+namespace {
+
+// Streaming loads of cache records.  With one query head per kv head nothing
+// is re-read, so the records bypass L1; with head pairs split over two lanes
+// the two lanes of a token read the same record in one instruction.
+template <bool kL1>
+__device__ __forceinline__ uint4 ld_rec16(const void* ptr) {
+  uint4 r;
+  if (kL1)
+    asm("ld.global.nc.v4.u32 {%0,%1,%2,%3}, [%4];"
+        : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w) : "l"(ptr));
+  else
+    asm("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
+        : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w) : "l"(ptr));
+  return r;
+}
+template <bool kL1>
+__device__ __forceinline__ uint2 ld_rec8(const void* ptr) {
+  uint2 r;
+  if (kL1)
+    asm("ld.global.nc.v2.u32 {%0,%1}, [%2];" : "=r"(r.x), "=r"(r.y) : "l"(ptr));
+  else
+    asm("ld.global.nc.L1::no_allocate.v2.u32 {%0,%1}, [%2];" : "=r"(r.x), "=r"(r.y) : "l"(ptr));
+  return r;
+}
+
+__device__ __forceinline__ float2 h2f(uint32_t w) {
+  return __half22float2(*reinterpret_cast<const __half2*>(&w));
+}
+
+// Two E4M3 values (low 16 bits of w, or the high 16 bits) to fp32.
+__device__ __forceinline__ float2 e4m3x2_to_f2(uint32_t w, bool hi) {
+  const __nv_fp8x2_storage_t pair = (__nv_fp8x2_storage_t)(hi ? (w >> 16) : (w & 0xffffu));
+  const __half2_raw h = __nv_cvt_fp8x2_to_halfraw2(pair, __NV_E4M3);
+  return __half22float2(*reinterpret_cast<const __half2*>(&h));
+}
+
+// ---------------------------------------------------------------------------
+// One 8-entry chunk of a cached vector, per value format:
+//   fp16: a 16-byte record of 8 fp16 values and an 8-byte record of indices;
+//   fp8:  one 16-byte record: 8 E4M3 values, then 8 indices.
+// ---------------------------------------------------------------------------
+template <int FMT>
+struct Chunk;
+template <>
+struct Chunk<kFmtFp16> {
+  uint4 v;
+  uint2 i;
+};
+template <>
+struct Chunk<kFmtFp8> {
+  uint4 r;
+};
+
+// vb: this lane's 16-byte record run, ib: its 8-byte index run (fp16 only)
+template <int FMT, bool kL1>
+__device__ __forceinline__ Chunk<FMT> load_chunk(const uint8_t* vb, const uint8_t* ib, int c) {
+  Chunk<FMT> ch;
+  if constexpr (FMT == kFmtFp16) {
+    ch.v = ld_rec16<kL1>(vb + c * 512);
+    ch.i = ld_rec8<kL1>(ib + c * 256);
+  } else {
+    ch.r = ld_rec16<kL1>(vb + c * 512);
+  }
+  return ch;
+}
+template <int FMT>
+__device__ __forceinline__ uint2 chunk_idx(const Chunk<FMT>& ch) {
+  if constexpr (FMT == kFmtFp16)
+    return ch.i;
+  else
+    return make_uint2(ch.r.z, ch.r.w);
+}
+template <int FMT>
+__device__ __forceinline__ void chunk_vals(const Chunk<FMT>& ch, float (&f)[8]) {
+  float2 a, b, c, d;
+  if constexpr (FMT == kFmtFp16) {
+    a = h2f(ch.v.x), b = h2f(ch.v.y), c = h2f(ch.v.z), d = h2f(ch.v.w);
+  } else {
+    a = e4m3x2_to_f2(ch.r.x, false), b = e4m3x2_to_f2(ch.r.x, true);
+    c = e4m3x2_to_f2(ch.r.y, false), d = e4m3x2_to_f2(ch.r.y, true);
+  }
+  f[0] = a.x, f[1] = a.y, f[2] = b.x, f[3] = b.y, f[4] = c.x, f[5] = c.y, f[6] = d.x, f[7] = d.y;
+}
+__device__ __forceinline__ void keep_first(float (&f)[8], int n) {
+#pragma unroll
+  for (int e = 0; e < 8; ++e) f[e] = (e < n) ? f[e] : 0.f;
+}
+
+__device__ __forceinline__ float warp_max(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+  return v;
+}
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+// Shared-memory accesses by 32-bit shared-window address.  They are volatile
+// so that they keep their program order among themselves: each chunk's eight
+// loads are issued back to back, then its eight stores (the indices of one
+// vector are distinct, so the batch never aliases).
+__device__ __forceinline__ float lds(uint32_t a) {
+  float v;
+  asm volatile("ld.shared.f32 %0, [%1];" : "=f"(v) : "r"(a));
+  return v;
+}
+__device__ __forceinline__ void sts(uint32_t a, float v) {
+  asm volatile("st.shared.f32 [%0], %1;" ::"r"(a), "f"(v));
+}
+__device__ __forceinline__ float2 lds2(uint32_t a) {
+  float2 v;
+  asm volatile("ld.shared.v2.f32 {%0,%1}, [%2];" : "=f"(v.x), "=f"(v.y) : "r"(a));
+  return v;
+}
+
+// Ask the memory system to bring `bytes` (a multiple of 16, 16-byte aligned)
+// into L2 ahead of the loads that will read them.
+__device__ __forceinline__ void prefetch_l2(const void* ptr, uint32_t bytes) {
+  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(ptr), "r"(bytes) : "memory");
+}
+
+// ---------------------------------------------------------------------------
+// One query head per kv head: lane = token, lane-private accumulators.
+// ---------------------------------------------------------------------------
+
+// Address of coordinate idx (byte e of the index word w) in a [128][32]
+// lane-interleaved fp32 array whose base is 16 KB aligned:
+// base | (idx & 127) << 7 | lane << 2.  One shift and one LOP3; element
+// (idx, lane) sits at idx*32 + lane, so 32 lanes gathering arbitrary
+// coordinates hit 32 distinct banks, and any index byte stays inside the
+// array.
+template <int E>
+__device__ __forceinline__ uint32_t addr_of(uint32_t w, uint32_t base) {
+  if (E == 0) return ((w << 7) & 0x3f80u) | base;
+  if (E == 1) return ((w >> 1) & 0x3f80u) | base;
+  if (E == 2) return ((w >> 9) & 0x3f80u) | base;
+  return ((w >> 17) & 0x3f80u) | base;
+}
+
+// Score contribution of one chunk into four partial sums.
+__device__ __forceinline__ void score_chunk(uint32_t qb, const float (&f)[8], uint2 ix, float (&s)[4]) {
+  const float q0 = lds(addr_of<0>(ix.x, qb)), q1 = lds(addr_of<1>(ix.x, qb));
+  const float q2 = lds(addr_of<2>(ix.x, qb)), q3 = lds(addr_of<3>(ix.x, qb));
+  const float q4 = lds(addr_of<0>(ix.y, qb)), q5 = lds(addr_of<1>(ix.y, qb));
+  const float q6 = lds(addr_of<2>(ix.y, qb)), q7 = lds(addr_of<3>(ix.y, qb));
+  s[0] = fmaf(q0, f[0], s[0]);
+  s[1] = fmaf(q1, f[1], s[1]);
+  s[2] = fmaf(q2, f[2], s[2]);
+  s[3] = fmaf(q3, f[3], s[3]);
+  s[0] = fmaf(q4, f[4], s[0]);
+  s[1] = fmaf(q5, f[5], s[1]);
+  s[2] = fmaf(q6, f[6], s[2]);
+  s[3] = fmaf(q7, f[7], s[3]);
+}
+
+// acc[idx_e] += p * val_e for one full chunk (distinct indices): eight loads,
+// eight FMAs, eight stores.
+__device__ __forceinline__ void value_chunk(uint32_t ab, float p, const float (&f)[8], uint2 ix) {
+  const uint32_t a0 = addr_of<0>(ix.x, ab), a1 = addr_of<1>(ix.x, ab);
+  const uint32_t a2 = addr_of<2>(ix.x, ab), a3 = addr_of<3>(ix.x, ab);
+  const uint32_t a4 = addr_of<0>(ix.y, ab), a5 = addr_of<1>(ix.y, ab);
+  const uint32_t a6 = addr_of<2>(ix.y, ab), a7 = addr_of<3>(ix.y, ab);
+  const float o0 = lds(a0), o1 = lds(a1), o2 = lds(a2), o3 = lds(a3);
+  const float o4 = lds(a4), o5 = lds(a5), o6 = lds(a6), o7 = lds(a7);
+  sts(a0, fmaf(p, f[0], o0));
+  sts(a1, fmaf(p, f[1], o1));
+  sts(a2, fmaf(p, f[2], o2));
+  sts(a3, fmaf(p, f[3], o3));
+  sts(a4, fmaf(p, f[4], o4));
+  sts(a5, fmaf(p, f[5], o5));
+  sts(a6, fmaf(p, f[6], o6));
+  sts(a7, fmaf(p, f[7], o7));
+}
+
+// The first `n` (< 8) entries of a chunk, one read-modify-write at a time
+// (the tail of a runtime keep count that is not a multiple of 8).
+__device__ __forceinline__ void value_chunk_partial(uint32_t ab, float p, const float (&f)[8], uint2 ix,
+                                                    int n) {
+#pragma unroll
+  for (int e = 0; e < 7; ++e) {
+    if (e < n) {
+      const uint32_t w = e < 4 ? ix.x : ix.y;
+      const uint32_t a = ((w >> (8u * (e & 3))) & 0x7fu) << 7 | ab;
+      sts(a, fmaf(p, f[e], lds(a)));
+    }
+  }
+}
+
+constexpr uint32_t kRegionBytes = kHeadDim * 32 * sizeof(float);  // 16 KB
+
+// Geometry of unit u's groups in the flat split: its first group `goff`,
+// its group count and lengths; uniform rows read the scalars, ragged rows
+// their SeqInfo entry.
+struct UnitView {
+  int64_t goff, N_g, sparse_len;
+  int n_sg, n_b, buf_start;
+};
+__device__ __forceinline__ UnitView unit_view(const DecodeParams& p, int64_t u) {
+  UnitView v;
+  if (p.seq == nullptr) {
+    v.goff = u * p.N_g;
+    v.N_g = p.N_g;
+    v.sparse_len = p.sparse_len;
+    v.n_sg = (int)p.n_sg;
+    v.n_b = p.n_b;
+    v.buf_start = p.buf_start;
+  } else {
+    const int64_t b = u / p.H_kv, h = u - b * p.H_kv;
+    const SeqInfo& q = p.seq[b];
+    v.sparse_len = q.sparse_len;
+    v.n_sg = (int)((q.sparse_len + 31) >> 5);
+    v.n_b = q.n_b;
+    v.buf_start = q.buf_start;
+    v.N_g = row_groups(q.sparse_len, q.n_b);
+    v.goff = q.group_prefix * p.H_kv + h * v.N_g;
+  }
+  return v;
+}
+// The unit that holds flat group g (0 <= g < total_groups).
+__device__ __forceinline__ int64_t unit_of(const DecodeParams& p, int64_t g) {
+  if (p.seq == nullptr) return g / p.N_g;
+  int lo = 0, hi = p.B - 1;  // the last row whose first group is <= g
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (p.seq[mid].group_prefix * p.H_kv <= g) lo = mid;
+    else hi = mid - 1;
+  }
+  const SeqInfo& q = p.seq[lo];
+  const int64_t ng = row_groups(q.sparse_len, q.n_b);
+  const int64_t h = min((int64_t)p.H_kv - 1, (g - q.group_prefix * p.H_kv) / ng);
+  return (int64_t)lo * p.H_kv + h;
+}
+// Split of a segment [s0, s1) of a unit's groups (the first n_sg sparse,
+// the rest dense-buffer groups, which cost about kBufferGroupCost sparse
+// groups: 512 instead of 384 bytes and twice the shared-memory work per
+// token, set by measurement) into `parts` contiguous runs of equal cost;
+// returns where run
+// `part` starts (part == parts gives s1).
+constexpr int kBufferGroupCost = 3;
+__device__ __forceinline__ int split_at(int s0, int s1, int n_sg, int part, int parts) {
+  const int sp_in = max(0, min(s1, n_sg) - s0);
+  const int bf_in = (s1 - s0) - sp_in;
+  const int cost = sp_in + kBufferGroupCost * bf_in;
+  const int c = (int)(((int64_t)cost * part) / parts);
+  return c <= sp_in ? s0 + c : s0 + sp_in + (c - sp_in + kBufferGroupCost - 1) / kBufferGroupCost;
+}
+
+// First group of CTA c (c <= gridDim.x) and the CTA that holds group g.
+__device__ __forceinline__ int64_t cta_begin(const DecodeParams& p, int64_t c) {
+  if (p.cta_start == nullptr) return min(p.total_groups, c * p.range);
+  return p.cta_start[c];
+}
+__device__ __forceinline__ int64_t cta_of(const DecodeParams& p, int64_t g) {
+  if (p.cta_start == nullptr) return g / p.range;
+  int lo = 0, hi = (int)gridDim.x - 1;  // the last CTA whose first group is <= g
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (p.cta_start[mid] <= g) lo = mid;
+    else hi = mid - 1;
+  }
+  return lo;
+}
+
+// The last CTA to finish a segment of unit u merges the unit's partials,
+// normalises, rotates back (o = o_hat R_vo^T) and writes the output.  The
+// arrival counter resets itself for the next decode; nothing waits.
+// `scratch` holds G * 128 floats (free at this point); `flag` one float.
+// out = o_hat R_vo^T for the G query heads of unit (b, h); o_hat in shared
+// memory [G][128].
+template <int G, int NT>
+__device__ __forceinline__ void rotate_back_out(const DecodeParams& p, int64_t b, int64_t h, const float* o_hat) {
+  const float* RT = p.R_voT + (size_t)h * kHeadDim * kHeadDim;
+  for (int o = threadIdx.x; o < G * kHeadDim; o += NT) {
+    const int gh = o / kHeadDim, i = o % kHeadDim;
+    const float* oh = o_hat + gh * kHeadDim;
+    float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
+#pragma unroll 8
+    for (int j = 0; j < kHeadDim; j += 4) {
+      a0 = fmaf(oh[j + 0], __ldg(RT + (j + 0) * kHeadDim + i), a0);
+      a1 = fmaf(oh[j + 1], __ldg(RT + (j + 1) * kHeadDim + i), a1);
+      a2 = fmaf(oh[j + 2], __ldg(RT + (j + 2) * kHeadDim + i), a2);
+      a3 = fmaf(oh[j + 3], __ldg(RT + (j + 3) * kHeadDim + i), a3);
+    }
+    p.out[((b * p.H_q) + h * G + gh) * kHeadDim + i] = __float2half_rn((a0 + a1) + (a2 + a3));
+  }
+}
+
+// The last CTA to finish a segment of unit u merges the unit's partials,
+// normalises, rotates back (o = o_hat R_vo^T) and writes the output.  The
+// arrival counter resets itself for the next decode; nothing waits.
+// `scratch` holds G * 128 floats (free at this point); `flag` one float.
+// (A unit that one CTA holds entirely never comes here: it is finished from
+// shared memory by that CTA.)
+template <int G, int NT>
+__device__ __forceinline__ void finish_unit(const DecodeParams& p, int64_t c0, int64_t c1, int64_t u, int64_t b,
+                                            int64_t h, float* scratch, float* flag) {
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    const int old = atomicAdd(p.counters + u, 1);
+    const bool last = old == (int)(c1 - c0);
+    if (last) p.counters[u] = 0;
+    flag[0] = last ? 1.f : 0.f;
+  }
+  __syncthreads();
+  if (flag[0] == 0.f) return;
+  __threadfence();
+  float* o_hat = scratch;  // [G][128]
+  for (int o = threadIdx.x; o < G * kHeadDim; o += NT) {
+    const int gh = o / kHeadDim, dd = o % kHeadDim;
+    float M = -INFINITY;
+    for (int64_t c = c0; c <= c1; ++c)
+      M = fmaxf(M, __ldcg(p.partials + ((size_t)(c + u) * G + gh) * (kHeadDim + 2)));
+    float L = 0.f, A = 0.f;
+    for (int64_t c = c0; c <= c1; ++c) {
+      const float* part = p.partials + ((size_t)(c + u) * G + gh) * (kHeadDim + 2);
+      const float mc = __ldcg(part);
+      const float w = (mc == -INFINITY) ? 0.f : exp2f(mc - M);
+      L = fmaf(w, __ldcg(part + 1), L);
+      A = fmaf(w, __ldcg(part + 2 + dd), A);
+    }
+    o_hat[o] = (L > 0.f) ? A / L : 0.f;
+  }
+  __syncthreads();
+  rotate_back_out<G, NT>(p, b, h, o_hat);
+}
+
+// Warps per CTA of the one-head kernel: as many lane-private accumulators as
+// fit next to q' (16 KB each, 227 KB of shared memory per CTA) and, for 16
+// chunks, as many as the registers allow.
+template <int MAXC>
+__host__ __device__ constexpr int decode_warps() { return MAXC <= 8 ? 12 : 8; }
+
+// Split decode kernel, one query head per kv head.
+//   The flat list of 32-token blocks of all units is cut into equal ranges,
+//   one per CTA.  Shared memory (16 KB-aligned regions): q' replicated per
+//   lane ([128][32] fp32) and one lane-private rotated-space accumulator per
+//   warp ([128][32] fp32).  Lane = token; each warp walks a contiguous run of
+//   blocks.  While block g is processed, the key records of block g+1 are in
+//   flight to registers and block g+2 is being prefetched into L2.
+template <int MAXC, int FMT>
+__global__ void __launch_bounds__(decode_warps<MAXC>() * 32, 1) decode_kernel(DecodeParams p) {
+  constexpr int NW = decode_warps<MAXC>();
+  constexpr int NT = NW * 32;
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  __shared__ float red_m[NW], red_l[NW];
+  pdl_trigger();
+
+  const uint32_t raw = (uint32_t)__cvta_generic_to_shared(smem_raw);
+  const uint32_t base = (raw + kRegionBytes - 1) & ~(kRegionBytes - 1);
+  float* qrep = reinterpret_cast<float*>(smem_raw + (base - raw));  // [128][32]
+  float* accs = qrep + kHeadDim * 32;                                // [NW][128][32]
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t qb = base + (lane << 2);
+  const uint32_t ab = base + (1 + warp) * kRegionBytes + (lane << 2);
+
+  const CacheGeom& g = p.geom;
+  const int kfull = p.k_full_chunks, krem = p.k_rem;          // keys
+  const int nchunks = kfull + (krem ? 1 : 0);
+  const int kfull_v = p.k_full_chunks_v, krem_v = p.k_rem_v;  // values
+  const int nchunks_v = kfull_v + (krem_v ? 1 : 0);
+  // this lane's record runs inside a block
+  const int o_kv = lane * 16, o_ki = g.kidx_off() + lane * 8;
+  const int o_vv = g.vval_off() + lane * 16, o_vi = g.vidx_off() + lane * 8;
+  const bool whole_block = nchunks * 8 == g.k_slots && nchunks_v * 8 == g.k_slots_v;
+  const int bsh = p.blocks_per_page_log2, bmask = (1 << bsh) - 1;
+
+  const int64_t g_begin = cta_begin(p, blockIdx.x);
+  const int64_t g_end = min(p.total_groups, cta_begin(p, blockIdx.x + 1));
+  pdl_wait();
+  if (g_begin >= g_end) return;
+  const int64_t u_first = unit_of(p, g_begin), u_last = unit_of(p, g_end - 1);
+
+  for (int64_t u = u_first; u <= u_last; ++u) {
+    const UnitView uv = unit_view(p, u);
+    const int n_sg = uv.n_sg;
+    const int s0 = (int)(max(g_begin, uv.goff) - uv.goff);
+    const int s1 = (int)(min(g_end, uv.goff + uv.N_g) - uv.goff);
+    const int64_t b = u / p.H_kv, h = u % p.H_kv;
+    // this warp's contiguous run of groups [t_lo, t_hi)
+    const int t_lo = split_at(s0, s1, n_sg, warp, NW);
+    const int t_hi = split_at(s0, s1, n_sg, warp + 1, NW);
+    const int sp_hi = min(t_hi, n_sg);  // sparse groups of the run: [t_lo, sp_hi)
+    const int32_t* ptab = g.page_table + u * g.pages_per_unit;
+
+    __syncthreads();  // the previous segment is done with shared memory
+    for (int i = threadIdx.x; i < kHeadDim * 32; i += NT)
+      qrep[i] = __ldg(p.qprime + ((b * p.H_q + h) * kHeadDim + (i >> 5)));
+#pragma unroll 8
+    for (int dd = 0; dd < kHeadDim; ++dd) sts(ab + dd * 128, 0.f);
+    __syncthreads();
+
+    float m_w = -INFINITY;  // running max (log2 domain), uniform in the warp
+    float l_sum = 0.f;      // this lane's sum of exp2(s - m_w)
+
+    // block of sparse group gi (nullptr past the run or on a bad page)
+    auto block_of = [&](int gi) -> const uint8_t* {
+      if (gi >= sp_hi) return nullptr;
+      const int32_t ph = __ldg(ptab + (gi >> bsh));
+      if (ph < 0 || ph >= g.num_pages) {
+        atomicOr(p.status, kStatusPageRange);
+        return nullptr;
+      }
+      return g.pool + (int64_t)ph * g.page_bytes + (int64_t)(gi & bmask) * g.block_bytes();
+    };
+    auto prefetch_block = [&](const uint8_t* blk) {
+      if (blk == nullptr || lane != 0) return;
+      if (whole_block) {
+        prefetch_l2(blk, (uint32_t)g.block_bytes());
+      } else if constexpr (FMT == kFmtFp16) {
+        prefetch_l2(blk, nchunks * 512u);
+        prefetch_l2(blk + g.kidx_off(), nchunks * 256u);
+        prefetch_l2(blk + g.vval_off(), nchunks_v * 512u);
+        prefetch_l2(blk + g.vidx_off(), nchunks_v * 256u);
+      } else {
+        prefetch_l2(blk, nchunks * 512u);
+        prefetch_l2(blk + g.vval_off(), nchunks_v * 512u);
+      }
+    };
+
+    Chunk<FMT> kc[MAXC];
+    auto load_k = [&](const uint8_t* blk) {
+      const uint8_t* src = blk ? blk : g.pool;
+#pragma unroll
+      for (int c = 0; c < MAXC; ++c)
+        if (c < nchunks) kc[c] = load_chunk<FMT, false>(src + o_kv, src + o_ki, c);
+    };
+
+    const uint8_t* b_cur = block_of(t_lo);
+    const uint8_t* b_n1 = block_of(t_lo + 1);
+    prefetch_block(b_n1);
+    if (t_lo < sp_hi) load_k(b_cur);
+
+    for (int gi = t_lo; gi < t_hi; ++gi) {
+      float s2, pr;
+      if (gi < n_sg) {
+        // ---- sparse group: tokens 32*gi .. 32*gi+31 of the sparse history
+        const int64_t t0 = (int64_t)gi * 32;
+        const bool ok = b_cur != nullptr;
+        const bool valid = ok && t0 + lane < uv.sparse_len;
+        const bool tail = !ok || t0 + 32 > uv.sparse_len;  // warp-uniform
+        const uint8_t* src = ok ? b_cur : g.pool;
+        Chunk<FMT> vc[MAXC];
+#pragma unroll
+        for (int c = 0; c < MAXC; ++c)
+          if (c < nchunks_v) vc[c] = load_chunk<FMT, false>(src + o_vv, src + o_vi, c);
+        // two blocks ahead: into L2
+        const uint8_t* b_n2 = block_of(gi + 2);
+        prefetch_block(b_n2);
+
+        float s[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+        for (int c = 0; c < MAXC; ++c)
+          if (c < nchunks) {
+            float f[8];
+            chunk_vals<FMT>(kc[c], f);
+            uint2 ix = chunk_idx<FMT>(kc[c]);
+            if (krem && c == nchunks - 1) keep_first(f, krem);
+            if (tail && !valid) {
+              keep_first(f, 0);
+              ix = make_uint2(0, 0);
+            }
+            score_chunk(qb, f, ix, s);
+          }
+        s2 = valid ? ((s[0] + s[1]) + (s[2] + s[3])) * p.scale_log2 : -INFINITY;
+
+        // the next block's key records into registers while this block's
+        // values are accumulated
+        if (gi + 1 < sp_hi) load_k(b_n1);
+        b_cur = b_n1;
+        b_n1 = b_n2;
+
+        const float gmax = warp_max(s2);
+        if (gmax > m_w + kLazyRescale) {
+          if (m_w != -INFINITY) {
+            const float fs = exp2f(m_w - gmax);
+            l_sum *= fs;
+#pragma unroll 8
+            for (int dd = 0; dd < kHeadDim; ++dd) sts(ab + dd * 128, lds(ab + dd * 128) * fs);
+          }
+          m_w = gmax;
+        }
+        pr = valid ? exp2f(s2 - m_w) : 0.f;
+        l_sum += pr;
+
+#pragma unroll
+        for (int c = 0; c < MAXC; ++c)
+          if (c < kfull_v) {
+            float f[8];
+            chunk_vals<FMT>(vc[c], f);
+            uint2 ix = chunk_idx<FMT>(vc[c]);
+            if (tail && !valid) {
+              keep_first(f, 0);
+              ix = make_uint2(0, 0);
+            }
+            value_chunk(ab, pr, f, ix);
+          }
+        if (krem_v && valid) {
+#pragma unroll
+          for (int c = 0; c < MAXC; ++c)
+            if (c == kfull_v) {
+              float f[8];
+              chunk_vals<FMT>(vc[c], f);
+              value_chunk_partial(ab, pr, f, chunk_idx<FMT>(vc[c]), krem_v);
+            }
+        }
+      } else {
+        // ---- buffer group: dense rotated fp16 vectors of the ring buffer
+        const int64_t i = (int64_t)(gi - n_sg) * 32 + lane;
+        const bool valid = i < uv.n_b;
+        const int slot = valid ? (int)((uv.buf_start + i) % p.cap) : 0;
+        const size_t row = ((size_t)u * p.cap + slot) * kHeadDim;
+        const uint4* kr = reinterpret_cast<const uint4*>(p.ring_k + row);
+        const uint4* vr = reinterpret_cast<const uint4*>(p.ring_v + row);
+        float s[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll 4
+        for (int c = 0; c < 16; ++c) {
+          const uint4 w = __ldg(kr + c);
+          const float2 a = h2f(w.x), bb = h2f(w.y), cc = h2f(w.z), d = h2f(w.w);
+          const uint32_t q = qb + c * 8 * 128;
+          s[0] = fmaf(lds(q + 0 * 128), a.x, s[0]);
+          s[1] = fmaf(lds(q + 1 * 128), a.y, s[1]);
+          s[2] = fmaf(lds(q + 2 * 128), bb.x, s[2]);
+          s[3] = fmaf(lds(q + 3 * 128), bb.y, s[3]);
+          s[0] = fmaf(lds(q + 4 * 128), cc.x, s[0]);
+          s[1] = fmaf(lds(q + 5 * 128), cc.y, s[1]);
+          s[2] = fmaf(lds(q + 6 * 128), d.x, s[2]);
+          s[3] = fmaf(lds(q + 7 * 128), d.y, s[3]);
+        }
+        s2 = valid ? ((s[0] + s[1]) + (s[2] + s[3])) * p.scale_log2 : -INFINITY;
+        const float gmax = warp_max(s2);
+        if (gmax > m_w + kLazyRescale) {
+          if (m_w != -INFINITY) {
+            const float fs = exp2f(m_w - gmax);
+            l_sum *= fs;
+#pragma unroll 8
+            for (int dd = 0; dd < kHeadDim; ++dd) sts(ab + dd * 128, lds(ab + dd * 128) * fs);
+          }
+          m_w = gmax;
+        }
+        pr = valid ? exp2f(s2 - m_w) : 0.f;
+        l_sum += pr;
+        if (valid) {
+#pragma unroll 2
+          for (int c = 0; c < 16; ++c) {
+            const uint4 w = __ldg(vr + c);
+            const float2 a = h2f(w.x), bb = h2f(w.y), cc = h2f(w.z), d = h2f(w.w);
+            const uint32_t t = ab + c * 8 * 128;
+            const float o0 = lds(t + 0 * 128), o1 = lds(t + 1 * 128), o2 = lds(t + 2 * 128),
+                        o3 = lds(t + 3 * 128), o4 = lds(t + 4 * 128), o5 = lds(t + 5 * 128),
+                        o6 = lds(t + 6 * 128), o7 = lds(t + 7 * 128);
+            sts(t + 0 * 128, fmaf(pr, a.x, o0));
+            sts(t + 1 * 128, fmaf(pr, a.y, o1));
+            sts(t + 2 * 128, fmaf(pr, bb.x, o2));
+            sts(t + 3 * 128, fmaf(pr, bb.y, o3));
+            sts(t + 4 * 128, fmaf(pr, cc.x, o4));
+            sts(t + 5 * 128, fmaf(pr, cc.y, o5));
+            sts(t + 6 * 128, fmaf(pr, d.x, o6));
+            sts(t + 7 * 128, fmaf(pr, d.y, o7));
+          }
+        }
+      }
+    }
+
+    // ---- merge the lanes and warps into one partial
+    l_sum = warp_sum(l_sum);
+    if (lane == 0) {
+      red_m[warp] = m_w;
+      red_l[warp] = l_sum;
+    }
+    __syncthreads();
+    const int64_t c0 = cta_of(p, uv.goff), c1 = cta_of(p, uv.goff + uv.N_g - 1);
+    const bool solo = c0 == c1;  // this CTA holds the whole unit
+    for (int dd = threadIdx.x; dd < kHeadDim; dd += NT) {
+      float M = -INFINITY;
+#pragma unroll
+      for (int w = 0; w < NW; ++w) M = fmaxf(M, red_m[w]);
+      float tot = 0.f, L = 0.f;
+#pragma unroll
+      for (int w = 0; w < NW; ++w) {
+        const float mw = red_m[w];
+        const float f = (mw == -INFINITY) ? 0.f : exp2f(mw - M);
+        const float* a = accs + w * kHeadDim * 32 + dd * 32;
+        float sum = 0.f;
+#pragma unroll 8
+        for (int jj = 0; jj < 32; ++jj) sum += a[(jj + dd) & 31];
+        tot = fmaf(f, sum, tot);
+        L = fmaf(f, red_l[w], L);
+      }
+      if (solo) {
+        qrep[dd] = (L > 0.f) ? tot / L : 0.f;  // q' is no longer needed
+        continue;
+      }
+      float* dst = p.partials + ((size_t)(blockIdx.x + u)) * (kHeadDim + 2);
+      dst[2 + dd] = tot;
+      if (dd == 0) {
+        dst[0] = M;
+        dst[1] = L;
+      }
+    }
+    if (solo) {
+      __syncthreads();
+      rotate_back_out<1, NT>(p, b, h, qrep);
+    } else {
+      finish_unit<1, NT>(p, c0, c1, u, b, h, qrep, red_m);
+    }
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Grouped-query heads with the value product on the tensor cores (G = 2, 4).
+//   Lane = token, as in the one-head kernel; each lane scores its token for
+//   all G query heads of the kv head from q' replicated per lane
+//   ([128][32][G] fp32: one 8- or 16-byte conflict-free gather per entry).
+//   The value product o_h += sum_t p_h(t) v_t is dense once the kept
+//   entries are scattered into a zero-filled [32 tokens][128] fp16 tile per
+//   warp, so it runs as mma.sync.m16n8k16 (rows = the G heads, k = the 32
+//   tokens, n = the 128 coordinates) with the fp32 accumulators in
+//   registers; p is split into fp16 hi + lo parts (two products), so the
+//   result keeps fp32 accuracy.  No per-warp shared accumulator: the tile
+//   and a [G][32] p table are all a warp holds in shared memory.
+// ---------------------------------------------------------------------------
+constexpr int kVRowBytes = 272;                      // 128 fp16 + 16 B pad: conflict-free ldmatrix rows
+constexpr uint32_t kVTileBytes = 32 * kVRowBytes;    // 8704
+constexpr uint32_t kPTileBytes = 4 * 32 * 4;         // p [<= 4 heads][32 tokens] fp32
+// Per warp: the tile, the p table and a staging area for the value records
+// of the next block (cp.async: MAXC chunks of 512 B values + 256 B indices).
+template <int MAXC>
+__host__ __device__ constexpr uint32_t mma_warp_bytes() {
+  return kVTileBytes + kPTileBytes + (uint32_t)MAXC * 768;
+}
+// 8 warps: the registers (~240 a thread) allow no more without spills, and a
+// sweep on the GB300 measured 8 < 10 < 12 warps in time (0.480, 0.491,
+// 0.565 ms on the GQA 131k layer).
+template <int MAXC>
+__host__ __device__ constexpr int mma_warps() { return 8; }
+// q' replicated in 32 / G copies per coordinate: [128][32 / G][G] fp32, 16 KB.
+// A G-float gather is served in phases of 32 / G lanes (16-byte loads: 8
+// lanes, 8-byte loads: 16), and the lanes of a phase read distinct copies,
+// so they never share a bank.
+constexpr uint32_t kQrepBytes = kHeadDim * 32 * 4;
+template <int G, int MAXC>
+__host__ __device__ constexpr size_t mma_smem() {
+  return (size_t)kQrepBytes + (size_t)mma_warps<MAXC>() * mma_warp_bytes<MAXC>() + 16;
+}
+
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_group 0;" ::: "memory"); }
+__device__ __forceinline__ uint4 lds_v4u(uint32_t a) {
+  uint4 v;
+  asm volatile("ld.shared.v4.u32 {%0,%1,%2,%3}, [%4];" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(a)
+               : "memory");
+  return v;
+}
+__device__ __forceinline__ uint2 lds_v2u(uint32_t a) {
+  uint2 v;
+  asm volatile("ld.shared.v2.u32 {%0,%1}, [%2];" : "=r"(v.x), "=r"(v.y) : "r"(a) : "memory");
+  return v;
+}
+
+__device__ __forceinline__ float4 lds4(uint32_t a) {
+  float4 v;
+  asm volatile("ld.shared.v4.f32 {%0,%1,%2,%3}, [%4];" : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w) : "r"(a));
+  return v;
+}
+// Tile accesses carry a memory clobber: they alias the C++ accesses to the
+// same tile (the p table, the o rows of the merge).
+__device__ __forceinline__ void sts_u16(uint32_t a, uint32_t v) {
+  asm volatile("st.shared.u16 [%0], %1;" ::"r"(a), "h"((unsigned short)v) : "memory");
+}
+__device__ __forceinline__ void sts_v4(uint32_t a, uint4 v) {
+  asm volatile("st.shared.v4.u32 [%0], {%1,%2,%3,%4};" ::"r"(a), "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w)
+               : "memory");
+}
+__device__ __forceinline__ void ldsm_x4_trans(uint32_t a, uint32_t (&r)[4]) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+               : "r"(a)
+               : "memory");
+}
+// d[0..1] += A (16 x 16, rows g and g + 8) * B (16 x 8); the rows g + 8 of A
+// are zero, so their accumulators are dropped.
+__device__ __forceinline__ void mma_16816(float (&d)[2], uint32_t a0, uint32_t a2, uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "{\n\t.reg .f32 x2, x3;\n\t"
+      "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0,%1,x2,x3}, {%2,%3,%4,%5}, {%6,%7}, "
+      "{%8,%9,%10,%11};\n\t}"
+      : "=f"(d[0]), "=f"(d[1])
+      : "r"(a0), "r"(0u), "r"(a2), "r"(0u), "r"(b0), "r"(b1), "f"(d[0]), "f"(d[1]), "f"(0.f), "f"(0.f));
+}
+// Two fp32 values as (hi, lo) fp16 pairs: x = hi + lo to ~2^-22 relative.
+__device__ __forceinline__ void split_pair(float x0, float x1, uint32_t& hi, uint32_t& lo) {
+  const __half h0 = __float2half_rn(x0), h1 = __float2half_rn(x1);
+  const __half l0 = __float2half_rn(x0 - __half2float(h0)), l1 = __float2half_rn(x1 - __half2float(h1));
+  hi = (uint32_t)__half_as_ushort(h0) | ((uint32_t)__half_as_ushort(h1) << 16);
+  lo = (uint32_t)__half_as_ushort(l0) | ((uint32_t)__half_as_ushort(l1) << 16);
+}
+// The 8 values of a chunk as fp16 bits, two per word.
+template <int FMT>
+__device__ __forceinline__ void chunk_half_words(const Chunk<FMT>& ch, uint32_t (&w)[4]) {
+  if constexpr (FMT == kFmtFp16) {
+    w[0] = ch.v.x, w[1] = ch.v.y, w[2] = ch.v.z, w[3] = ch.v.w;
+  } else {
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const uint32_t src = q < 2 ? ch.r.x : ch.r.y;
+      const __half2_raw h = __nv_cvt_fp8x2_to_halfraw2(
+          (__nv_fp8x2_storage_t)((q & 1) ? (src >> 16) : (src & 0xffffu)), __NV_E4M3);
+      w[q] = (uint32_t)h.x | ((uint32_t)h.y << 16);
+    }
+  }
+}
+// Scores of G heads for one chunk: q' row idx of this lane is G floats.
+template <int G>
+__device__ __forceinline__ void score_g_chunk(uint32_t qb, const float (&f)[8], uint2 ix, float (&s)[G]) {
+#pragma unroll
+  for (int e = 0; e < 8; ++e) {
+    const uint32_t w = e < 4 ? ix.x : ix.y;
+    const uint32_t a = qb + ((w >> (8 * (e & 3))) & 0x7fu) * 128u;
+    if constexpr (G == 4) {
+      const float4 q = lds4(a);
+      s[0] = fmaf(q.x, f[e], s[0]);
+      s[1] = fmaf(q.y, f[e], s[1]);
+      s[2] = fmaf(q.z, f[e], s[2]);
+      s[3] = fmaf(q.w, f[e], s[3]);
+    } else {
+      const float2 q = lds2(a);
+      s[0] = fmaf(q.x, f[e], s[0]);
+      s[1] = fmaf(q.y, f[e], s[1]);
+    }
+  }
+}
+// Scatter the first n (<= 8) entries of a chunk into this lane's tile row.
+__device__ __forceinline__ void scatter_chunk(uint32_t vrow, const uint32_t (&w)[4], uint2 ix, int n) {
+#pragma unroll
+  for (int e = 0; e < 8; ++e) {
+    if (e < n) {
+      const uint32_t iw = e < 4 ? ix.x : ix.y;
+      const uint32_t idx = (iw >> (8 * (e & 3))) & 0x7fu;
+      const uint32_t hw = w[e >> 1];
+      sts_u16(vrow + idx * 2, (e & 1) ? (hw >> 16) : (hw & 0xffffu));
+    }
+  }
+}
+
+template <int G, int MAXC, int FMT>
+__global__ void __launch_bounds__(mma_warps<MAXC>() * 32, 1) decode_mma_kernel(DecodeParams p) {
+  constexpr int NW = mma_warps<MAXC>(), NT = NW * 32;
+  constexpr uint32_t kWarpBytes = mma_warp_bytes<MAXC>();
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  __shared__ float red_m[NW * G], red_l[NW * G];
+  __shared__ float flag[1];
+  pdl_trigger();
+
+  const uint32_t raw = (uint32_t)__cvta_generic_to_shared(smem_raw);
+  const uint32_t base = (raw + 15u) & ~15u;
+  unsigned char* base_ptr = smem_raw + (base - raw);
+  float* qrep = reinterpret_cast<float*>(base_ptr);                         // [128][32/G][G]
+  const uint32_t wbase = base + kQrepBytes;                                 // per-warp regions
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t vtile = wbase + warp * kWarpBytes;                         // [32][272 B] fp16
+  float* ptile_f = reinterpret_cast<float*>(base_ptr + (vtile + kVTileBytes - base));  // [G][32] fp32
+  const uint32_t vstage = vtile + kVTileBytes + kPTileBytes;                  // value records, next block
+  const uint32_t qb = base + (lane & (32 / G - 1)) * (G * 4);  // this lane's copy
+  const uint32_t vrow = vtile + lane * kVRowBytes;
+  const int gq = lane >> 2, cq = lane & 3;  // mma fragment coordinates
+
+  const CacheGeom& g = p.geom;
+  const int kfull = p.k_full_chunks, krem = p.k_rem;
+  const int nchunks = kfull + (krem ? 1 : 0);
+  const int kfull_v = p.k_full_chunks_v, krem_v = p.k_rem_v;
+  const int nchunks_v = kfull_v + (krem_v ? 1 : 0);
+  const int o_kv = lane * 16, o_ki = g.kidx_off() + lane * 8;
+  const int o_vv = g.vval_off() + lane * 16, o_vi = g.vidx_off() + lane * 8;
+  const bool whole_block = nchunks * 8 == g.k_slots && nchunks_v * 8 == g.k_slots_v;
+  const int bsh = p.blocks_per_page_log2, bmask = (1 << bsh) - 1;
+
+  const int64_t g_begin = cta_begin(p, blockIdx.x);
+  const int64_t g_end = min(p.total_groups, cta_begin(p, blockIdx.x + 1));
+  pdl_wait();
+  if (g_begin >= g_end) return;
+  const int64_t u_first = unit_of(p, g_begin), u_last = unit_of(p, g_end - 1);
+
+  // the tiles start zeroed; every use restores the zeros it disturbed
+  for (int c = 0; c < 16; ++c) sts_v4(vrow + c * 16, make_uint4(0, 0, 0, 0));
+
+  for (int64_t u = u_first; u <= u_last; ++u) {
+    const UnitView uv = unit_view(p, u);
+    const int n_sg = uv.n_sg;
+    const int s0 = (int)(max(g_begin, uv.goff) - uv.goff);
+    const int s1 = (int)(min(g_end, uv.goff + uv.N_g) - uv.goff);
+    const int64_t b = u / p.H_kv, h = u % p.H_kv;
+    const int t_lo = split_at(s0, s1, n_sg, warp, NW);
+    const int t_hi = split_at(s0, s1, n_sg, warp + 1, NW);
+    const int sp_hi = min(t_hi, n_sg);
+    const int32_t* ptab = g.page_table + u * g.pages_per_unit;
+
+    __syncthreads();  // the previous segment is done with q'
+    for (int i = threadIdx.x; i < kHeadDim * 32; i += NT) {
+      const int c = i / 32, j = i % G;  // 32 floats per coordinate: 32 / G copies of G heads
+      qrep[i] = __ldg(p.qprime + ((b * p.H_q + h * G + j) * kHeadDim + c));
+    }
+    __syncthreads();
+
+    float m[G], l[G];
+#pragma unroll
+    for (int j = 0; j < G; ++j) m[j] = -INFINITY, l[j] = 0.f;
+    float acc[16][2];
+#pragma unroll
+    for (int nt = 0; nt < 16; ++nt) acc[nt][0] = acc[nt][1] = 0.f;
+
+    auto block_of = [&](int gi) -> const uint8_t* {
+      if (gi >= sp_hi) return nullptr;
+      const int32_t ph = __ldg(ptab + (gi >> bsh));
+      if (ph < 0 || ph >= g.num_pages) {
+        atomicOr(p.status, kStatusPageRange);
+        return nullptr;
+      }
+      return g.pool + (int64_t)ph * g.page_bytes + (int64_t)(gi & bmask) * g.block_bytes();
+    };
+    auto prefetch_block = [&](const uint8_t* blk) {
+      if (blk == nullptr || lane != 0) return;
+      if (whole_block) {
+        prefetch_l2(blk, (uint32_t)g.block_bytes());
+      } else if constexpr (FMT == kFmtFp16) {
+        prefetch_l2(blk, nchunks * 512u);
+        prefetch_l2(blk + g.kidx_off(), nchunks * 256u);
+        prefetch_l2(blk + g.vval_off(), nchunks_v * 512u);
+        prefetch_l2(blk + g.vidx_off(), nchunks_v * 256u);
+      } else {
+        prefetch_l2(blk, nchunks * 512u);
+        prefetch_l2(blk + g.vval_off(), nchunks_v * 512u);
+      }
+    };
+    Chunk<FMT> kc[MAXC];
+    auto load_k = [&](const uint8_t* blk) {
+      const uint8_t* src = blk ? blk : g.pool;
+#pragma unroll
+      for (int c = 0; c < MAXC; ++c)
+        if (c < nchunks) kc[c] = load_chunk<FMT, false>(src + o_kv, src + o_ki, c);
+    };
+    // the value records of a block into this warp's staging area, in flight
+    // while the warp works on the block before it
+    auto stage_v = [&](const uint8_t* blk) {
+      if (blk != nullptr) {
+        const int n_val = nchunks_v * 32;  // 16-byte pieces
+        for (int i = lane; i < n_val; i += 32) cp_async16(vstage + i * 16, blk + g.vval_off() + i * 16);
+        if constexpr (FMT == kFmtFp16) {
+          const int n_idx = nchunks_v * 16;
+          for (int i = lane; i < n_idx; i += 32)
+            cp_async16(vstage + nchunks_v * 512 + i * 16, blk + g.vidx_off() + i * 16);
+        }
+      }
+      cp_async_commit();
+    };
+
+    const uint8_t* b_cur = block_of(t_lo);
+    const uint8_t* b_n1 = block_of(t_lo + 1);
+    prefetch_block(b_n1);
+    if (t_lo < sp_hi) {
+      load_k(b_cur);
+      stage_v(b_cur);
+    }
+
+    for (int gi = t_lo; gi < t_hi; ++gi) {
+      float s[G];
+#pragma unroll
+      for (int j = 0; j < G; ++j) s[j] = 0.f;
+      bool valid;
+      if (gi < n_sg) {
+        // ---- sparse tokens 32 gi .. 32 gi + 31
+        const int64_t t0 = (int64_t)gi * 32;
+        const bool ok = b_cur != nullptr;
+        valid = ok && t0 + lane < uv.sparse_len;
+        const uint8_t* b_n2 = block_of(gi + 2);
+        prefetch_block(b_n2);
+        if (valid) {
+#pragma unroll
+          for (int c = 0; c < MAXC; ++c)
+            if (c < nchunks) {
+              float f[8];
+              chunk_vals<FMT>(kc[c], f);
+              if (krem && c == nchunks - 1) keep_first(f, krem);
+              score_g_chunk<G>(qb, f, chunk_idx<FMT>(kc[c]), s);
+            }
+        }
+        // this token's kept values (staged by cp.async) into its tile row
+        cp_async_wait_all();
+        __syncwarp();
+        if (valid) {
+#pragma unroll
+          for (int c = 0; c < MAXC; ++c)
+            if (c < nchunks_v) {
+              Chunk<FMT> vc;
+              if constexpr (FMT == kFmtFp16) {
+                vc.v = lds_v4u(vstage + c * 512 + lane * 16);
+                vc.i = lds_v2u(vstage + nchunks_v * 512 + c * 256 + lane * 8);
+              } else {
+                vc.r = lds_v4u(vstage + c * 512 + lane * 16);
+              }
+              uint32_t w[4];
+              chunk_half_words<FMT>(vc, w);
+              scatter_chunk(vrow, w, chunk_idx<FMT>(vc), (krem_v && c == nchunks_v - 1) ? krem_v : 8);
+            }
+        }
+        __syncwarp();
+        if (gi + 1 < sp_hi) {
+          load_k(b_n1);
+          stage_v(b_n1);
+        }
+        b_cur = b_n1;
+        b_n1 = b_n2;
+      } else {
+        // ---- dense buffer tokens: scores over all 128 coordinates, the
+        // value row copied into the tile
+        const int64_t i = (int64_t)(gi - n_sg) * 32 + lane;
+        valid = i < uv.n_b;
+        if (valid) {
+          const int slot = (int)((uv.buf_start + i) % p.cap);
+          const size_t row = ((size_t)u * p.cap + slot) * kHeadDim;
+          const uint4* kr = reinterpret_cast<const uint4*>(p.ring_k + row);
+          const uint4* vr = reinterpret_cast<const uint4*>(p.ring_v + row);
+#pragma unroll 2
+          for (int c = 0; c < 16; ++c) {
+            const uint4 w = __ldg(kr + c);
+            const float2 a = h2f(w.x), bb = h2f(w.y), cc = h2f(w.z), d = h2f(w.w);
+            const float f[8] = {a.x, a.y, bb.x, bb.y, cc.x, cc.y, d.x, d.y};
+#pragma unroll
+            for (int e = 0; e < 8; ++e) {
+              const uint32_t qa = qb + (uint32_t)(c * 8 + e) * 128u;
+              if constexpr (G == 4) {
+                const float4 q = lds4(qa);
+                s[0] = fmaf(q.x, f[e], s[0]);
+                s[1] = fmaf(q.y, f[e], s[1]);
+                s[2] = fmaf(q.z, f[e], s[2]);
+                s[3] = fmaf(q.w, f[e], s[3]);
+              } else {
+                const float2 q = lds2(qa);
+                s[0] = fmaf(q.x, f[e], s[0]);
+                s[1] = fmaf(q.y, f[e], s[1]);
+              }
+            }
+          }
+#pragma unroll 4
+          for (int c = 0; c < 16; ++c) sts_v4(vrow + c * 16, __ldg(vr + c));
+        }
+      }
+
+      // ---- online softmax per head (lazy rescale of the register accumulators)
+      float pj[G];
+#pragma unroll
+      for (int j = 0; j < G; ++j) {
+        const float sj = valid ? s[j] * p.scale_log2 : -INFINITY;
+        const float gmax = warp_max(sj);
+        if (gmax > m[j] + kLazyRescale) {
+          if (m[j] != -INFINITY) {
+            const float fs = exp2f(m[j] - gmax);
+            l[j] *= fs;
+            if (gq == j) {
+#pragma unroll
+              for (int nt = 0; nt < 16; ++nt) acc[nt][0] *= fs, acc[nt][1] *= fs;
+            }
+          }
+          m[j] = gmax;
+        }
+        pj[j] = valid ? exp2f(sj - m[j]) : 0.f;
+        l[j] += pj[j];
+        ptile_f[j * 32 + lane] = pj[j];
+      }
+      __syncwarp();
+
+      // ---- o[head][:] += p[head][tokens] * tile[tokens][:] on the tensor cores
+#pragma unroll
+      for (int ks = 0; ks < 2; ++ks) {
+        uint32_t ahi0 = 0, alo0 = 0, ahi2 = 0, alo2 = 0;
+        if (gq < G) {
+          const float* pr = ptile_f + gq * 32 + ks * 16 + 2 * cq;
+          split_pair(pr[0], pr[1], ahi0, alo0);
+          split_pair(pr[8], pr[9], ahi2, alo2);
+        }
+#pragma unroll
+        for (int np = 0; np < 8; ++np) {
+          const int mi = lane >> 3;
+          const uint32_t addr = vtile + (uint32_t)(ks * 16 + (mi & 1) * 8 + (lane & 7)) * kVRowBytes +
+                                (uint32_t)(16 * np + 8 * (mi >> 1)) * 2;
+          uint32_t bf[4];
+          ldsm_x4_trans(addr, bf);
+          mma_16816(acc[2 * np], ahi0, ahi2, bf[0], bf[1]);
+          mma_16816(acc[2 * np], alo0, alo2, bf[0], bf[1]);
+          mma_16816(acc[2 * np + 1], ahi0, ahi2, bf[2], bf[3]);
+          mma_16816(acc[2 * np + 1], alo0, alo2, bf[2], bf[3]);
+        }
+      }
+      __syncwarp();
+      // restore the zeros of this lane's tile row
+      if (valid)
+        for (int c = 0; c < 16; ++c) sts_v4(vrow + c * 16, make_uint4(0, 0, 0, 0));
+    }
+
+    // ---- merge lanes and warps per query head into one partial
+#pragma unroll
+    for (int j = 0; j < G; ++j) l[j] = warp_sum(l[j]);
+    if (lane == 0) {
+#pragma unroll
+      for (int j = 0; j < G; ++j) {
+        red_m[warp * G + j] = m[j];
+        red_l[warp * G + j] = l[j];
+      }
+    }
+    // this warp's o rows into its tile region ([G][128] fp32)
+    __syncwarp();
+    float* obuf = reinterpret_cast<float*>(base_ptr + (vtile - base));
+    if (gq < G) {
+#pragma unroll
+      for (int nt = 0; nt < 16; ++nt) {
+        obuf[gq * kHeadDim + nt * 8 + 2 * cq] = acc[nt][0];
+        obuf[gq * kHeadDim + nt * 8 + 2 * cq + 1] = acc[nt][1];
+      }
+    }
+    __syncthreads();
+    const int64_t c0 = cta_of(p, uv.goff), c1 = cta_of(p, uv.goff + uv.N_g - 1);
+    const bool solo = c0 == c1;
+    for (int o = threadIdx.x; o < G * kHeadDim; o += NT) {
+      const int hd = o / kHeadDim, dd = o % kHeadDim;
+      float M = -INFINITY;
+#pragma unroll
+      for (int w = 0; w < NW; ++w) M = fmaxf(M, red_m[w * G + hd]);
+      float tot = 0.f, L = 0.f;
+#pragma unroll
+      for (int w = 0; w < NW; ++w) {
+        const float mw = red_m[w * G + hd];
+        const float f = (mw == -INFINITY) ? 0.f : exp2f(mw - M);
+        const float* ob = reinterpret_cast<const float*>(base_ptr + (wbase - base) + w * kWarpBytes);
+        tot = fmaf(f, ob[hd * kHeadDim + dd], tot);
+        L = fmaf(f, red_l[w * G + hd], L);
+      }
+      if (solo) {
+        qrep[o] = (L > 0.f) ? tot / L : 0.f;  // q' is no longer needed
+        continue;
+      }
+      float* dst = p.partials + ((size_t)(blockIdx.x + u) * G + hd) * (kHeadDim + 2);
+      dst[2 + dd] = tot;
+      if (dd == 0) {
+        dst[0] = M;
+        dst[1] = L;
+      }
+    }
+    __syncthreads();
+    // the o rows overwrote part of the tiles: zero them again
+    for (int c = 0; c < 16; ++c) sts_v4(vrow + c * 16, make_uint4(0, 0, 0, 0));
+    if (solo) {
+      rotate_back_out<G, NT>(p, b, h, qrep);
+    } else {
+      finish_unit<G, NT>(p, c0, c1, u, b, h, qrep, flag);
+    }
+  }
+}
+
+// q' = q R_qk: one CTA per (kv head, up to 8 query vectors of that head),
+// R in shared memory, one warp per query vector; lane l computes coordinates
+// 4l..4l+3 in a sequential fp32 FMA chain.
+__global__ void __launch_bounds__(kThreads) rotate_q_kernel(RotateQParams p, int B) {
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  float* Rs = reinterpret_cast<float*>(smem_raw);
+  const int h = blockIdx.x;
+  const float* R = p.R_qk + (size_t)h * kHeadDim * kHeadDim;
+  pdl_trigger();
+  stage_matrix(Rs, R);
+  __syncthreads();
+  pdl_wait();
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  for (int item = blockIdx.y * kWarpsPerCta + warp; item < min(B * p.G, (int)(blockIdx.y + 1) * kWarpsPerCta);
+       item += kWarpsPerCta) {
+    const int b = item / p.G, gh = item % p.G;
+    const int64_t bq = (int64_t)b * p.H_q + h * p.G + gh;
+    const uint2 xw = __ldg(reinterpret_cast<const uint2*>(p.q + bq * kHeadDim) + lane);
+    const float2 x01 = __half22float2(*reinterpret_cast<const __half2*>(&xw.x));
+    const float2 x23 = __half22float2(*reinterpret_cast<const __half2*>(&xw.y));
+    const float xs[4] = {x01.x, x01.y, x23.x, x23.y};
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll 8
+    for (int i = 0; i < kHeadDim; ++i) {
+      const float xi = __shfl_sync(0xffffffffu, xs[i & 3], i >> 2);
+      const float4 r = reinterpret_cast<const float4*>(Rs + i * kHeadDim)[lane];
+      acc.x = fmaf(xi, r.x, acc.x);
+      acc.y = fmaf(xi, r.y, acc.y);
+      acc.z = fmaf(xi, r.z, acc.z);
+      acc.w = fmaf(xi, r.w, acc.w);
+    }
+    reinterpret_cast<float4*>(p.qprime + bq * kHeadDim)[lane] = acc;
+  }
+}
+
+// Empty cache: writes zeros (the rotate-back of an empty attention).
+__global__ void __launch_bounds__(kHeadDim) combine_kernel(CombineParams p) {
+  __shared__ float o_hat[kHeadDim];
+  pdl_trigger();
+  pdl_wait();
+  const int64_t bq = blockIdx.x;
+  const int64_t b = bq / p.H_q;
+  const int hq = (int)(bq % p.H_q);
+  const int h = hq / p.G, gh = hq % p.G;
+  const int64_t u = b * p.H_kv + h;
+  const int dd = threadIdx.x;
+  float val = 0.f;
+  if (p.total_groups > 0) {
+    const int64_t c0 = (u * p.N_g) / p.range;
+    const int64_t c1 = ((u + 1) * p.N_g - 1) / p.range;
+    float M = -INFINITY;
+    for (int64_t c = c0; c <= c1; ++c)
+      M = fmaxf(M, p.partials[((size_t)(c + u) * p.G + gh) * (kHeadDim + 2)]);
+    float L = 0.f, A = 0.f;
+    for (int64_t c = c0; c <= c1; ++c) {
+      const float* part = p.partials + ((size_t)(c + u) * p.G + gh) * (kHeadDim + 2);
+      const float w = (part[0] == -INFINITY) ? 0.f : exp2f(part[0] - M);
+      L = fmaf(w, part[1], L);
+      A = fmaf(w, part[2 + dd], A);
+    }
+    val = (L > 0.f) ? A / L : 0.f;
+  }
+  o_hat[dd] = val;
+  __syncthreads();
+  const float* RT = p.R_voT + (size_t)h * kHeadDim * kHeadDim;
+  float a0 = 0.f, a1 = 0.f;
+#pragma unroll 8
+  for (int j = 0; j < kHeadDim; j += 2) {
+    a0 = fmaf(o_hat[j], __ldg(RT + j * kHeadDim + dd), a0);
+    a1 = fmaf(o_hat[j + 1], __ldg(RT + (j + 1) * kHeadDim + dd), a1);
+  }
+  p.out[bq * kHeadDim + dd] = __float2half_rn(a0 + a1);
+}
+
+}  // namespace
+}  // namespace swan

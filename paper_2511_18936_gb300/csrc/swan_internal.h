@@ -30,6 +30,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <atomic>
+
 namespace swan {
 
 constexpr int kHeadDim = 128;
@@ -213,6 +215,21 @@ __device__ __forceinline__ void stage_matrix(float* dst, const float* src) {
   for (int k = 0; k < 16; ++k) reinterpret_cast<float4*>(dst)[threadIdx.x + k * kThreads] = r[k];
 }
 #endif
+
+// Raise a kernel's dynamic shared-memory limit once per device (the limit
+// is a per-device function attribute; thread-safe).
+template <auto Kernel>
+cudaError_t ensure_smem(size_t bytes) {
+  static std::atomic<uint64_t> done{0};
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  const uint64_t bit = dev < 64 ? (uint64_t)1 << dev : 0;
+  if (bit && (done.load(std::memory_order_acquire) & bit)) return cudaSuccess;
+  e = cudaFuncSetAttribute(Kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
+  if (e == cudaSuccess && bit) done.fetch_or(bit, std::memory_order_release);
+  return e;
+}
 
 // Launchers (return the launch error, if any).
 // Bulk append with the rotation on the tensor cores: maps[0..1] the new keys

@@ -67,13 +67,10 @@ cudaError_t launch_decode(const DecodeParams& p, int G, int k_read, int grid, cu
 }
 
 cudaError_t launch_rotate_q(const RotateQParams& p, int B, cudaStream_t s) {
-  constexpr size_t smem = kHeadDim * kHeadDim * sizeof(float);
-  const cudaError_t e = ensure_smem<rotate_q_kernel>(smem);
-  if (e != cudaSuccess) return e;
   const int vecs = B * p.G;  // query vectors per kv head
   return launch_pdl(rotate_q_kernel,
-                    dim3((unsigned)(p.H_q / p.G), (unsigned)((vecs + kWarpsPerCta - 1) / kWarpsPerCta)),
-                    dim3(kThreads), smem, s, p, B);
+                    dim3((unsigned)(p.H_q / p.G), (unsigned)((vecs + kWarpsPerCta - 1) / kWarpsPerCta), 4),
+                    dim3(kThreads), 0, s, p, B);
 }
 
 cudaError_t launch_combine(const CombineParams& p, int B, cudaStream_t s) {

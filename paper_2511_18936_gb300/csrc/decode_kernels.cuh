@@ -1075,16 +1075,19 @@ __global__ void __launch_bounds__(mma_warps<MAXC>() * 32, 1) decode_mma_kernel(D
   }
 }
 
-// q' = q R_qk: one CTA per (kv head, up to 8 query vectors of that head),
-// R in shared memory, one warp per query vector; lane l computes coordinates
-// 4l..4l+3 in a sequential fp32 FMA chain.
+// q' = q R_qk: one CTA per (kv head, up to 8 query vectors of that head,
+// 32 of the 128 output coordinates), the 128 x 32 slice of R in shared
+// memory, one warp per query vector; lane l computes coordinate
+// 32 z + l in a sequential fp32 FMA chain over the 128 inputs.
 __global__ void __launch_bounds__(kThreads) rotate_q_kernel(RotateQParams p, int B) {
-  extern __shared__ __align__(16) unsigned char smem_raw[];
-  float* Rs = reinterpret_cast<float*>(smem_raw);
-  const int h = blockIdx.x;
-  const float* R = p.R_qk + (size_t)h * kHeadDim * kHeadDim;
+  __shared__ float Rs[kHeadDim * 32];
+  const int h = blockIdx.x, z = blockIdx.z;
+  const float* R = p.R_qk + (size_t)h * kHeadDim * kHeadDim + z * 32;
   pdl_trigger();
-  stage_matrix(Rs, R);
+  for (int e = threadIdx.x; e < kHeadDim * 8; e += kThreads) {  // 128 rows x 8 float4
+    const int i = e >> 3, c = e & 7;
+    reinterpret_cast<float4*>(Rs)[e] = __ldg(reinterpret_cast<const float4*>(R + i * kHeadDim) + c);
+  }
   __syncthreads();
   pdl_wait();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -1096,17 +1099,13 @@ __global__ void __launch_bounds__(kThreads) rotate_q_kernel(RotateQParams p, int
     const float2 x01 = __half22float2(*reinterpret_cast<const __half2*>(&xw.x));
     const float2 x23 = __half22float2(*reinterpret_cast<const __half2*>(&xw.y));
     const float xs[4] = {x01.x, x01.y, x23.x, x23.y};
-    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll 8
+    float acc = 0.f;
+#pragma unroll 16
     for (int i = 0; i < kHeadDim; ++i) {
       const float xi = __shfl_sync(0xffffffffu, xs[i & 3], i >> 2);
-      const float4 r = reinterpret_cast<const float4*>(Rs + i * kHeadDim)[lane];
-      acc.x = fmaf(xi, r.x, acc.x);
-      acc.y = fmaf(xi, r.y, acc.y);
-      acc.z = fmaf(xi, r.z, acc.z);
-      acc.w = fmaf(xi, r.w, acc.w);
+      acc = fmaf(xi, Rs[i * 32 + lane], acc);
     }
-    reinterpret_cast<float4*>(p.qprime + bq * kHeadDim)[lane] = acc;
+    p.qprime[bq * kHeadDim + z * 32 + lane] = acc;
   }
 }
 

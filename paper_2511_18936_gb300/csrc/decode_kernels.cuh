@@ -1,8 +1,9 @@
-// Device code of the decode path (Algorithm 1, attention part; Section 4.3):
-// the split decode kernels with the fused combine and rotate-back (Appendix
-// A.1, Lemma 2), the query rotation and the empty-cache combine.  Included
-// by decode.cu, which holds the host launchers; this file is what the
-// committed profiles' source hash covers.
+// Device code of the decode kernels (Algorithm 1, attention part; Section
+// 4.3): the split decode with the fused combine and rotate-back (Appendix
+// A.1, Lemma 2), one query head per kv head and grouped-query heads.
+// Included by decode.cu, which holds the query rotation, the empty-cache
+// combine and the host launchers; this file is what the committed profiles'
+// source hash covers.
 #pragma once
 
 #include <cuda_fp8.h>
@@ -1073,79 +1074,6 @@ __global__ void __launch_bounds__(mma_warps<MAXC>() * 32, 1) decode_mma_kernel(D
       finish_unit<G, NT>(p, c0, c1, u, b, h, qrep, flag);
     }
   }
-}
-
-// q' = q R_qk: one CTA per (kv head, up to 8 query vectors of that head,
-// 32 of the 128 output coordinates), the 128 x 32 slice of R in shared
-// memory, one warp per query vector; lane l computes coordinate
-// 32 z + l in a sequential fp32 FMA chain over the 128 inputs.
-__global__ void __launch_bounds__(kThreads) rotate_q_kernel(RotateQParams p, int B) {
-  __shared__ float Rs[kHeadDim * 32];
-  const int h = blockIdx.x, z = blockIdx.z;
-  const float* R = p.R_qk + (size_t)h * kHeadDim * kHeadDim + z * 32;
-  pdl_trigger();
-  for (int e = threadIdx.x; e < kHeadDim * 8; e += kThreads) {  // 128 rows x 8 float4
-    const int i = e >> 3, c = e & 7;
-    reinterpret_cast<float4*>(Rs)[e] = __ldg(reinterpret_cast<const float4*>(R + i * kHeadDim) + c);
-  }
-  __syncthreads();
-  pdl_wait();
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  for (int item = blockIdx.y * kWarpsPerCta + warp; item < min(B * p.G, (int)(blockIdx.y + 1) * kWarpsPerCta);
-       item += kWarpsPerCta) {
-    const int b = item / p.G, gh = item % p.G;
-    const int64_t bq = (int64_t)b * p.H_q + h * p.G + gh;
-    const uint2 xw = __ldg(reinterpret_cast<const uint2*>(p.q + bq * kHeadDim) + lane);
-    const float2 x01 = __half22float2(*reinterpret_cast<const __half2*>(&xw.x));
-    const float2 x23 = __half22float2(*reinterpret_cast<const __half2*>(&xw.y));
-    const float xs[4] = {x01.x, x01.y, x23.x, x23.y};
-    float acc = 0.f;
-#pragma unroll 16
-    for (int i = 0; i < kHeadDim; ++i) {
-      const float xi = __shfl_sync(0xffffffffu, xs[i & 3], i >> 2);
-      acc = fmaf(xi, Rs[i * 32 + lane], acc);
-    }
-    p.qprime[bq * kHeadDim + z * 32 + lane] = acc;
-  }
-}
-
-// Empty cache: writes zeros (the rotate-back of an empty attention).
-__global__ void __launch_bounds__(kHeadDim) combine_kernel(CombineParams p) {
-  __shared__ float o_hat[kHeadDim];
-  pdl_trigger();
-  pdl_wait();
-  const int64_t bq = blockIdx.x;
-  const int64_t b = bq / p.H_q;
-  const int hq = (int)(bq % p.H_q);
-  const int h = hq / p.G, gh = hq % p.G;
-  const int64_t u = b * p.H_kv + h;
-  const int dd = threadIdx.x;
-  float val = 0.f;
-  if (p.total_groups > 0) {
-    const int64_t c0 = (u * p.N_g) / p.range;
-    const int64_t c1 = ((u + 1) * p.N_g - 1) / p.range;
-    float M = -INFINITY;
-    for (int64_t c = c0; c <= c1; ++c)
-      M = fmaxf(M, p.partials[((size_t)(c + u) * p.G + gh) * (kHeadDim + 2)]);
-    float L = 0.f, A = 0.f;
-    for (int64_t c = c0; c <= c1; ++c) {
-      const float* part = p.partials + ((size_t)(c + u) * p.G + gh) * (kHeadDim + 2);
-      const float w = (part[0] == -INFINITY) ? 0.f : exp2f(part[0] - M);
-      L = fmaf(w, part[1], L);
-      A = fmaf(w, part[2 + dd], A);
-    }
-    val = (L > 0.f) ? A / L : 0.f;
-  }
-  o_hat[dd] = val;
-  __syncthreads();
-  const float* RT = p.R_voT + (size_t)h * kHeadDim * kHeadDim;
-  float a0 = 0.f, a1 = 0.f;
-#pragma unroll 8
-  for (int j = 0; j < kHeadDim; j += 2) {
-    a0 = fmaf(o_hat[j], __ldg(RT + j * kHeadDim + dd), a0);
-    a1 = fmaf(o_hat[j + 1], __ldg(RT + (j + 1) * kHeadDim + dd), a1);
-  }
-  p.out[bq * kHeadDim + dd] = __float2half_rn(a0 + a1);
 }
 
 }  // namespace

@@ -486,8 +486,7 @@ class LayerRun:
         self.ctx.check()
 
     def step(self, i):
-        self.ctx.append(0, self.k_steps[i], self.v_steps[i], 1)
-        self.ctx.decode(0, self.qs[i], self.out)
+        self.ctx.append_decode(0, self.k_steps[i], self.v_steps[i], self.qs[i], self.out, 1)
 
     def context_after(self, i):
         """(sparse, buffer) tokens attended by the decode of step i."""
@@ -499,8 +498,7 @@ class LayerRun:
 
     def step_with(self, dev_inputs):
         dk, dv, dq = dev_inputs
-        self.ctx.append(0, dk, dv, 1)
-        self.ctx.decode(0, dq, self.out)
+        self.ctx.append_decode(0, dk, dv, dq, self.out, 1)
         return [self.out]
 
 
@@ -613,8 +611,7 @@ class StackRun:
 
     def step(self, i):
         for l in range(self.layers):
-            self.ctx.append(l, self.kn[l, i], self.vn[l, i], 1)
-            self.ctx.decode(l, self.qs[l, i], self.out[l])
+            self.ctx.append_decode(l, self.kn[l, i], self.vn[l, i], self.qs[l, i], self.out[l], 1)
         if self._flush_due(i):
             self.ctx.flush(-1)
 
@@ -630,8 +627,7 @@ class StackRun:
         dk, dv, dq = dev_inputs
         i = self._e2e_i
         for l in range(self.layers):
-            self.ctx.append(l, dk[l], dv[l], 1)
-            self.ctx.decode(l, dq[l], self.out[l])
+            self.ctx.append_decode(l, dk[l], dv[l], dq[l], self.out[l], 1)
         if self._flush_due(i):
             self.ctx.flush(-1)
         return [self.out]

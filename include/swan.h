@@ -17,6 +17,8 @@
  *                      dense-dense score products, softmax, value product),
  *                      followed by the rotate-back o = o_hat R_vo^T
  *                      (Appendix A.1, Lemma 2)
+ *   swan_append_decode a decode step's append and decode in one call (the
+ *                      query rotation runs inside the append's launch)
  *   swan_set_k         runtime keep count (Section 1 contributions, Section
  *                      4.3: the pruning threshold is tunable at inference)
  *
@@ -192,6 +194,20 @@ swan_status swan_reset_sequence(swan_ctx* ctx, int b);
  */
 swan_status swan_decode(swan_ctx* ctx, int layer, const void* q, void* out);
 
+/*
+ * One serving step of a layer (Algorithm 1 in full: compress the step's new
+ * tokens, then attend): exactly swan_append_varlen(ctx, layer, k_new, v_new,
+ * T, n_new) followed by swan_decode(ctx, layer, q, out), with the same
+ * arguments, results and errors (n_new may be NULL: every row takes T
+ * tokens).  A decode-step append (few vectors) computes the query rotation
+ * q' = q R_qk in its own launch, so the step takes two launches instead of
+ * three; q' has the same bits as swan_decode's.  With timing enabled, that
+ * launch counts as SWAN_KERNEL_APPEND.  q and out are checked before
+ * anything runs: on any error nothing is appended and nothing is decoded.
+ */
+swan_status swan_append_decode(swan_ctx* ctx, int layer, const void* k_new, const void* v_new, int T,
+                               const int32_t* n_new, const void* q, void* out);
+
 /* Host-side view of a layer's cache (no synchronisation). */
 typedef struct swan_layer_info {
   int64_t sparse_len;   /* tokens per sequence in the sparse history */
@@ -246,7 +262,8 @@ swan_status swan_debug_export_seq(swan_ctx* ctx, int layer, int b, int what, voi
 /*
  * Synchronise the stream and read the device status word that kernels set
  * when a device-side consistency check fails (for instance a page-table
- * entry out of range; such a kernel skips the access instead of faulting) or
+ * entry out of range, or too little shared memory for a kernel's aligned
+ * layout; such a kernel skips the access or the launch instead of faulting) or
  * a bounded wait of a tensor-core pipeline gave up (2 s; the launch's
  * results are then invalid).  Returns OK, DEVICE_TIMEOUT or DEVICE_CHECK
  * (and clears the word), STATE or CUDA.

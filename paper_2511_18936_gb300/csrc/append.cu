@@ -113,25 +113,22 @@ __device__ __forceinline__ RowView row_view(const AppendParams& p, int64_t b, in
 }
 
 
-// Small appends (decode steps): one CTA per (kv head, K or V).  Phase 1
-// prunes the `evict_old` oldest buffered vectors of every sequence out of the
-// ring; after a barrier, phase 2 rotates the new vectors one per warp (lane l
-// computes coordinates 4l..4l+3 from R in shared memory, in the same fp32
-// order as append_kernel) and either prunes them or writes them to the ring.
-// Ring slots freed in phase 1 are reused in phase 2 only after the barrier.
-__global__ void __launch_bounds__(kThreads) append_small_kernel(AppendParams p, int evict_old, int bpc) {
-  extern __shared__ __align__(16) unsigned char smem_raw[];
-  float* Rs = reinterpret_cast<float*>(smem_raw);
-  const int kind = blockIdx.y;
-  const int h = blockIdx.x;
-  const int b0 = blockIdx.z * bpc;                 // this CTA's sequences: [b0, b0 + nb)
+// Small appends (decode steps): one CTA per (kv head h, K or V, bpc
+// sequences from bz * bpc).  Phase 1 prunes the `evict_old` oldest buffered
+// vectors of every sequence out of the ring; after a barrier, phase 2 rotates
+// the new vectors one per warp (lane l computes coordinates 4l..4l+3 from R
+// in shared memory, Rs: 64 KB, as a sequential fp32 FMA chain over the 128
+// inputs) and either prunes them or writes them to the ring.  Ring slots
+// freed in phase 1 are reused in phase 2 only after the barrier.
+__device__ __forceinline__ void append_small_cta(const AppendParams& p, int evict_old, int bpc, int kind,
+                                                 int h, int bz, float* Rs) {
+  const int b0 = bz * bpc;                         // this CTA's sequences: [b0, b0 + nb)
   const int nb = min(bpc, p.B - b0);
   const float* R = (kind ? p.R_vo : p.R_qk) + (size_t)h * kHeadDim * kHeadDim;
   const __half* X = kind ? p.v_new : p.k_new;
   __half* ring = kind ? p.ring_v : p.ring_k;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
-  pdl_trigger();
   stage_matrix(Rs, R);
   pdl_wait();
 
@@ -179,6 +176,29 @@ __global__ void __launch_bounds__(kThreads) append_small_kernel(AppendParams p, 
       const int slot = (int)((rv.buf_start + pos) % p.cap);
       reinterpret_cast<uint2*>(ring + (unit * p.cap + slot) * kHeadDim)[lane] = yw;
     }
+  }
+}
+
+__global__ void __launch_bounds__(kThreads) append_small_kernel(AppendParams p, int evict_old, int bpc) {
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  pdl_trigger();
+  append_small_cta(p, evict_old, bpc, blockIdx.y, blockIdx.x, blockIdx.z, reinterpret_cast<float*>(smem_raw));
+}
+
+// A decode step's append and query rotation in one launch (they touch
+// disjoint data): blockIdx.y 0 and 1 are the append's key and value CTAs
+// (blockIdx.z < append_z), 2..5 the four coordinate slices of the query
+// rotation (blockIdx.z < rotate_z query chunks).  CTAs beyond either range
+// exit at once.
+__global__ void __launch_bounds__(kThreads) append_rotate_kernel(AppendParams p, int evict_old, int bpc,
+                                                                 int append_z, RotateQParams rq, int rotate_z) {
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  float* Rs = reinterpret_cast<float*>(smem_raw);
+  pdl_trigger();
+  if (blockIdx.y < 2) {
+    if ((int)blockIdx.z < append_z) append_small_cta(p, evict_old, bpc, blockIdx.y, blockIdx.x, blockIdx.z, Rs);
+  } else if ((int)blockIdx.z < rotate_z) {
+    rotate_q_slice(rq, p.B, blockIdx.x, blockIdx.z, blockIdx.y - 2, Rs);
   }
 }
 
@@ -407,15 +427,23 @@ cudaError_t launch_scatter_pages(const int2* pairs, int n, int32_t* table, cudaS
   return cudaGetLastError();
 }
 
-cudaError_t launch_append_small(const AppendParams& p, int evict_old, cudaStream_t s) {
+cudaError_t launch_append_small(const AppendParams& p, int evict_old, const RotateQParams* rq, cudaStream_t s) {
   constexpr size_t smem = 128 * 128 * sizeof(float);
-  cudaError_t e = ensure_smem<append_small_kernel>(smem);
-  if (e != cudaSuccess) return e;
   // enough sequences per CTA for one vector per warp and phase
   const int per = max(p.T, evict_old);
   const int bpc = max(1, kWarpsPerCta / max(per, 1));
-  return launch_pdl(append_small_kernel, dim3((unsigned)p.H, 2, (unsigned)((p.B + bpc - 1) / bpc)),
-                    dim3(kThreads), smem, s, p, evict_old, bpc);
+  const int append_z = (p.B + bpc - 1) / bpc;
+  if (rq == nullptr) {
+    const cudaError_t e = ensure_smem<append_small_kernel>(smem);
+    if (e != cudaSuccess) return e;
+    return launch_pdl(append_small_kernel, dim3((unsigned)p.H, 2, (unsigned)append_z), dim3(kThreads), smem, s,
+                      p, evict_old, bpc);
+  }
+  const cudaError_t e = ensure_smem<append_rotate_kernel>(smem);
+  if (e != cudaSuccess) return e;
+  const int rotate_z = (p.B * rq->G + kWarpsPerCta - 1) / kWarpsPerCta;
+  return launch_pdl(append_rotate_kernel, dim3((unsigned)p.H, 6, (unsigned)max(append_z, rotate_z)),
+                    dim3(kThreads), smem, s, p, evict_old, bpc, append_z, *rq, rotate_z);
 }
 
 cudaError_t launch_prune_ring(const PruneRingParams& p, cudaStream_t s) {

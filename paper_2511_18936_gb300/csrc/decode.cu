@@ -7,37 +7,11 @@ namespace swan {
 namespace {
 
 // q' = q R_qk: one CTA per (kv head, up to 8 query vectors of that head,
-// 32 of the 128 output coordinates), the 128 x 32 slice of R in shared
-// memory, one warp per query vector; lane l computes coordinate
-// 32 z + l in a sequential fp32 FMA chain over the 128 inputs.
+// 32 of the 128 output coordinates); see rotate_q_slice.
 __global__ void __launch_bounds__(kThreads) rotate_q_kernel(RotateQParams p, int B) {
-  __shared__ float Rs[kHeadDim * 32];
-  const int h = blockIdx.x, z = blockIdx.z;
-  const float* R = p.R_qk + (size_t)h * kHeadDim * kHeadDim + z * 32;
+  __shared__ __align__(16) float Rs[kHeadDim * 32];
   pdl_trigger();
-  for (int e = threadIdx.x; e < kHeadDim * 8; e += kThreads) {  // 128 rows x 8 float4
-    const int i = e >> 3, c = e & 7;
-    reinterpret_cast<float4*>(Rs)[e] = __ldg(reinterpret_cast<const float4*>(R + i * kHeadDim) + c);
-  }
-  __syncthreads();
-  pdl_wait();
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  for (int item = blockIdx.y * kWarpsPerCta + warp; item < min(B * p.G, (int)(blockIdx.y + 1) * kWarpsPerCta);
-       item += kWarpsPerCta) {
-    const int b = item / p.G, gh = item % p.G;
-    const int64_t bq = (int64_t)b * p.H_q + h * p.G + gh;
-    const uint2 xw = __ldg(reinterpret_cast<const uint2*>(p.q + bq * kHeadDim) + lane);
-    const float2 x01 = __half22float2(*reinterpret_cast<const __half2*>(&xw.x));
-    const float2 x23 = __half22float2(*reinterpret_cast<const __half2*>(&xw.y));
-    const float xs[4] = {x01.x, x01.y, x23.x, x23.y};
-    float acc = 0.f;
-#pragma unroll 16
-    for (int i = 0; i < kHeadDim; ++i) {
-      const float xi = __shfl_sync(0xffffffffu, xs[i & 3], i >> 2);
-      acc = fmaf(xi, Rs[i * 32 + lane], acc);
-    }
-    p.qprime[bq * kHeadDim + z * 32 + lane] = acc;
-  }
+  rotate_q_slice(p, B, blockIdx.x, blockIdx.y, blockIdx.z, Rs);
 }
 
 // Empty cache: writes zeros (the rotate-back of an empty attention).
@@ -79,9 +53,12 @@ __global__ void __launch_bounds__(kHeadDim) combine_kernel(CombineParams p) {
   p.out[bq * kHeadDim + dd] = __float2half_rn(a0 + a1);
 }
 
+// Dynamic shared memory of the one-head kernel: the warps' accumulators and
+// one more 16 KB region for the alignment gap, which holds q' (8 KB) unless
+// the allocation starts within 8 KB below a 16 KB boundary.
 size_t one_head_smem(int maxc) {
   const int nw = maxc <= 8 ? decode_warps<8>() : decode_warps<16>();
-  return (size_t)(1 + nw + 1) * kRegionBytes;
+  return (size_t)(nw + 1) * kRegionBytes;
 }
 
 template <typename K>

@@ -139,26 +139,34 @@ __device__ __forceinline__ void prefetch_l2(const void* ptr, uint32_t bytes) {
 // One query head per kv head: lane = token, lane-private accumulators.
 // ---------------------------------------------------------------------------
 
-// Address of coordinate idx (byte e of the index word w) in a [128][32]
-// lane-interleaved fp32 array whose base is 16 KB aligned:
-// base | (idx & 127) << 7 | lane << 2.  One shift and one LOP3; element
-// (idx, lane) sits at idx*32 + lane, so 32 lanes gathering arbitrary
-// coordinates hit 32 distinct banks, and any index byte stays inside the
-// array.
-template <int E>
+// Address of coordinate idx (byte e of the index word w) in a [128][R]
+// lane-interleaved fp32 array (R = 32 for the accumulators, 16 for q'), row
+// 2^SH = 4R bytes, base aligned to 128 rows: base | (idx & 127) << SH |
+// (lane % R) << 2.  One shift and one LOP3.  With R = 32 the 32 lanes
+// gathering arbitrary coordinates hit 32 distinct banks; with R = 16 lanes
+// l and l + 16 share a copy (two wavefronts when their coordinates differ
+// but have the same parity).  Any index byte stays inside the array.
+template <int E, int SH = 7>
 __device__ __forceinline__ uint32_t addr_of(uint32_t w, uint32_t base) {
-  if (E == 0) return ((w << 7) & 0x3f80u) | base;
-  if (E == 1) return ((w >> 1) & 0x3f80u) | base;
-  if (E == 2) return ((w >> 9) & 0x3f80u) | base;
-  return ((w >> 17) & 0x3f80u) | base;
+  constexpr uint32_t mask = 0x7fu << SH;
+  constexpr int sh = SH - 8 * E;  // where byte e's low bit goes
+  if constexpr (sh >= 0) return ((w << sh) & mask) | base;
+  else return ((w >> -sh) & mask) | base;
 }
+
+// q' of the one-head kernel: 16 copies of each coordinate ([128][16] fp32,
+// 64-byte rows, 8 KB aligned).
+constexpr int kQRep = 16;
+constexpr int kQRowShift = 6;
+constexpr uint32_t kQBytes = kHeadDim * kQRep * sizeof(float);  // 8 KB
 
 // Score contribution of one chunk into four partial sums.
 __device__ __forceinline__ void score_chunk(uint32_t qb, const float (&f)[8], uint2 ix, float (&s)[4]) {
-  const float q0 = lds(addr_of<0>(ix.x, qb)), q1 = lds(addr_of<1>(ix.x, qb));
-  const float q2 = lds(addr_of<2>(ix.x, qb)), q3 = lds(addr_of<3>(ix.x, qb));
-  const float q4 = lds(addr_of<0>(ix.y, qb)), q5 = lds(addr_of<1>(ix.y, qb));
-  const float q6 = lds(addr_of<2>(ix.y, qb)), q7 = lds(addr_of<3>(ix.y, qb));
+  constexpr int Q = kQRowShift;
+  const float q0 = lds(addr_of<0, Q>(ix.x, qb)), q1 = lds(addr_of<1, Q>(ix.x, qb));
+  const float q2 = lds(addr_of<2, Q>(ix.x, qb)), q3 = lds(addr_of<3, Q>(ix.x, qb));
+  const float q4 = lds(addr_of<0, Q>(ix.y, qb)), q5 = lds(addr_of<1, Q>(ix.y, qb));
+  const float q6 = lds(addr_of<2, Q>(ix.y, qb)), q7 = lds(addr_of<3, Q>(ix.y, qb));
   s[0] = fmaf(q0, f[0], s[0]);
   s[1] = fmaf(q1, f[1], s[1]);
   s[2] = fmaf(q2, f[2], s[2]);
@@ -277,50 +285,84 @@ __device__ __forceinline__ int64_t cta_of(const DecodeParams& p, int64_t g) {
   return lo;
 }
 
-// The last CTA to finish a segment of unit u merges the unit's partials,
-// normalises, rotates back (o = o_hat R_vo^T) and writes the output.  The
-// arrival counter resets itself for the next decode; nothing waits.
-// `scratch` holds G * 128 floats (free at this point); `flag` one float.
 // out = o_hat R_vo^T for the G query heads of unit (b, h); o_hat in shared
-// memory [G][128].
+// memory [G][128].  With at least twice as many threads as outputs, each
+// output's 128-term sum is cut into S = NT / (128 G) slices computed by
+// different threads (partial sums in `part`, S * G * 128 floats of shared
+// memory apart from o_hat), so more loads of R_vo^T are in flight at once.
 template <int G, int NT>
-__device__ __forceinline__ void rotate_back_out(const DecodeParams& p, int64_t b, int64_t h, const float* o_hat) {
+__device__ __forceinline__ void rotate_back_out(const DecodeParams& p, int64_t b, int64_t h, const float* o_hat,
+                                                float* part) {
+  constexpr int OUT = G * kHeadDim;
+  constexpr int S = NT >= 2 * OUT ? NT / OUT : 1;
   const float* RT = p.R_voT + (size_t)h * kHeadDim * kHeadDim;
-  for (int o = threadIdx.x; o < G * kHeadDim; o += NT) {
-    const int gh = o / kHeadDim, i = o % kHeadDim;
-    const float* oh = o_hat + gh * kHeadDim;
-    float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
+  if constexpr (S == 1) {
+    for (int o = threadIdx.x; o < OUT; o += NT) {
+      const int gh = o / kHeadDim, i = o % kHeadDim;
+      const float* oh = o_hat + gh * kHeadDim;
+      float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
 #pragma unroll 8
-    for (int j = 0; j < kHeadDim; j += 4) {
-      a0 = fmaf(oh[j + 0], __ldg(RT + (j + 0) * kHeadDim + i), a0);
-      a1 = fmaf(oh[j + 1], __ldg(RT + (j + 1) * kHeadDim + i), a1);
-      a2 = fmaf(oh[j + 2], __ldg(RT + (j + 2) * kHeadDim + i), a2);
-      a3 = fmaf(oh[j + 3], __ldg(RT + (j + 3) * kHeadDim + i), a3);
+      for (int j = 0; j < kHeadDim; j += 4) {
+        a0 = fmaf(oh[j + 0], __ldg(RT + (j + 0) * kHeadDim + i), a0);
+        a1 = fmaf(oh[j + 1], __ldg(RT + (j + 1) * kHeadDim + i), a1);
+        a2 = fmaf(oh[j + 2], __ldg(RT + (j + 2) * kHeadDim + i), a2);
+        a3 = fmaf(oh[j + 3], __ldg(RT + (j + 3) * kHeadDim + i), a3);
+      }
+      p.out[((b * p.H_q) + h * G + gh) * kHeadDim + i] = __float2half_rn((a0 + a1) + (a2 + a3));
     }
-    p.out[((b * p.H_q) + h * G + gh) * kHeadDim + i] = __float2half_rn((a0 + a1) + (a2 + a3));
+  } else {
+    const int t = threadIdx.x;
+    if (t < S * OUT) {
+      const int o = t % OUT, sl = t / OUT;
+      const int gh = o / kHeadDim, i = o % kHeadDim;
+      const float* oh = o_hat + gh * kHeadDim;
+      const int j0 = sl * kHeadDim / S, j1 = (sl + 1) * kHeadDim / S;
+      float a0 = 0.f, a1 = 0.f;
+      int j = j0;
+#pragma unroll 4
+      for (; j + 1 < j1; j += 2) {
+        a0 = fmaf(oh[j + 0], __ldg(RT + (j + 0) * kHeadDim + i), a0);
+        a1 = fmaf(oh[j + 1], __ldg(RT + (j + 1) * kHeadDim + i), a1);
+      }
+      if (j < j1) a0 = fmaf(oh[j], __ldg(RT + j * kHeadDim + i), a0);
+      part[sl * OUT + o] = a0 + a1;
+    }
+    __syncthreads();
+    for (int o = t; o < OUT; o += NT) {
+      const int gh = o / kHeadDim, i = o % kHeadDim;
+      float a = 0.f;
+#pragma unroll
+      for (int k = 0; k < S; ++k) a += part[k * OUT + o];
+      p.out[((b * p.H_q) + h * G + gh) * kHeadDim + i] = __float2half_rn(a);
+    }
   }
 }
 
 // The last CTA to finish a segment of unit u merges the unit's partials,
 // normalises, rotates back (o = o_hat R_vo^T) and writes the output.  The
 // arrival counter resets itself for the next decode; nothing waits.
-// `scratch` holds G * 128 floats (free at this point); `flag` one float.
+// `scratch` holds (S + 1) * G * 128 floats (free at this point; S as in
+// rotate_back_out); `flag` one float.  Every thread's partial writes are
+// ordered before thread 0's fence by the barrier, and the fence before the
+// arrival (the release pattern of a grid-wide barrier).
 // (A unit that one CTA holds entirely never comes here: it is finished from
 // shared memory by that CTA.)
 template <int G, int NT>
 __device__ __forceinline__ void finish_unit(const DecodeParams& p, int64_t c0, int64_t c1, int64_t u, int64_t b,
                                             int64_t h, float* scratch, float* flag) {
-  __threadfence();
   __syncthreads();
   if (threadIdx.x == 0) {
+    __threadfence();
     const int old = atomicAdd(p.counters + u, 1);
     const bool last = old == (int)(c1 - c0);
-    if (last) p.counters[u] = 0;
+    if (last) {
+      p.counters[u] = 0;
+      __threadfence();
+    }
     flag[0] = last ? 1.f : 0.f;
   }
   __syncthreads();
   if (flag[0] == 0.f) return;
-  __threadfence();
   float* o_hat = scratch;  // [G][128]
   for (int o = threadIdx.x; o < G * kHeadDim; o += NT) {
     const int gh = o / kHeadDim, dd = o % kHeadDim;
@@ -338,38 +380,57 @@ __device__ __forceinline__ void finish_unit(const DecodeParams& p, int64_t c0, i
     o_hat[o] = (L > 0.f) ? A / L : 0.f;
   }
   __syncthreads();
-  rotate_back_out<G, NT>(p, b, h, o_hat);
+  rotate_back_out<G, NT>(p, b, h, o_hat, scratch + G * kHeadDim);
 }
 
-// Warps per CTA of the one-head kernel: as many lane-private accumulators as
-// fit next to q' (16 KB each, 227 KB of shared memory per CTA) and, for 16
-// chunks, as many as the registers allow.
+// Warps per CTA of the one-head kernel: one lane-private accumulator each
+// (16 KB); for 16 chunks as many as the registers allow.
 template <int MAXC>
-__host__ __device__ constexpr int decode_warps() { return MAXC <= 8 ? 12 : 8; }
+__host__ __device__ constexpr int decode_warps() { return MAXC <= 8 ? 6 : 8; }
+// CTAs of the one-head kernel per SM (registers and shared memory allow two
+// of 6 warps; one CTA's barriers, merges and finishes then overlap the
+// other's streaming)
+template <int MAXC>
+__host__ __device__ constexpr int decode_min_ctas() { return MAXC <= 8 ? 2 : 1; }
 
 // Split decode kernel, one query head per kv head.
 //   The flat list of 32-token blocks of all units is cut into equal ranges,
-//   one per CTA.  Shared memory (16 KB-aligned regions): q' replicated per
-//   lane ([128][32] fp32) and one lane-private rotated-space accumulator per
-//   warp ([128][32] fp32).  Lane = token; each warp walks a contiguous run of
-//   blocks.  While block g is processed, the key records of block g+1 are in
-//   flight to registers and block g+2 is being prefetched into L2.
+//   one per CTA.  Shared memory (dynamic, laid out from its actual start):
+//   one lane-private rotated-space accumulator per warp ([128][32] fp32,
+//   16 KB-aligned regions) and q' with 16 copies per coordinate ([128][16]
+//   fp32, 8 KB aligned), in the gap before the first aligned region when it
+//   fits there, else after the accumulators.
+//   Lane = token; each warp walks a contiguous run of blocks.  While block g
+//   is processed, the key records of block g+1 are in flight to registers
+//   and block g+2 is being prefetched into L2.
 template <int MAXC, int FMT>
-__global__ void __launch_bounds__(decode_warps<MAXC>() * 32, 1) decode_kernel(DecodeParams p) {
+__global__ void __launch_bounds__(decode_warps<MAXC>() * 32, decode_min_ctas<MAXC>())
+    decode_kernel(DecodeParams p) {
   constexpr int NW = decode_warps<MAXC>();
   constexpr int NT = NW * 32;
-  extern __shared__ __align__(16) unsigned char smem_raw[];
+  extern __shared__ __align__(16) unsigned char smem_dyn[];
   __shared__ float red_m[NW], red_l[NW];
+  __shared__ float q_stage[kHeadDim];  // q' of the next unit, before replication
   pdl_trigger();
 
-  const uint32_t raw = (uint32_t)__cvta_generic_to_shared(smem_raw);
+  const uint32_t raw = (uint32_t)__cvta_generic_to_shared(smem_dyn);
   const uint32_t base = (raw + kRegionBytes - 1) & ~(kRegionBytes - 1);
-  float* qrep = reinterpret_cast<float*>(smem_raw + (base - raw));  // [128][32]
-  float* accs = qrep + kHeadDim * 32;                                // [NW][128][32]
+  uint32_t qbase = (raw + kQBytes - 1) & ~(kQBytes - 1);
+  if (qbase + kQBytes > base) qbase = base + NW * kRegionBytes;
+  {
+    uint32_t dyn_bytes;
+    asm("mov.u32 %0, %%dynamic_smem_size;" : "=r"(dyn_bytes));
+    if (max(base + NW * kRegionBytes, qbase + kQBytes) > raw + dyn_bytes) {
+      if (threadIdx.x == 0) atomicOr(p.status, kStatusLayout);
+      return;  // the launch gave too little shared memory for this layout
+    }
+  }
+  float* accs = reinterpret_cast<float*>(smem_dyn + (base - raw));  // [NW][128][32]
+  float* qrep = reinterpret_cast<float*>(smem_dyn + (qbase - raw)); // [128][16]
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const uint32_t qb = base + (lane << 2);
-  const uint32_t ab = base + (1 + warp) * kRegionBytes + (lane << 2);
+  const uint32_t qb = qbase + ((lane & (kQRep - 1)) << 2);
+  const uint32_t ab = base + warp * kRegionBytes + (lane << 2);
 
   const CacheGeom& g = p.geom;
   const int kfull = p.k_full_chunks, krem = p.k_rem;          // keys
@@ -387,6 +448,13 @@ __global__ void __launch_bounds__(decode_warps<MAXC>() * 32, 1) decode_kernel(De
   pdl_wait();
   if (g_begin >= g_end) return;
   const int64_t u_first = unit_of(p, g_begin), u_last = unit_of(p, g_end - 1);
+  // q' of the unit the next segment starts: one coalesced load, issued a
+  // segment ahead (the first one here)
+  auto q_of = [&](int64_t un) {
+    const int64_t bn = un / p.H_kv, hn = un - bn * p.H_kv;
+    return __ldg(p.qprime + (bn * p.H_q + hn) * kHeadDim + threadIdx.x);
+  };
+  float q_next = threadIdx.x < kHeadDim ? q_of(u_first) : 0.f;
 
   for (int64_t u = u_first; u <= u_last; ++u) {
     const UnitView uv = unit_view(p, u);
@@ -400,12 +468,20 @@ __global__ void __launch_bounds__(decode_warps<MAXC>() * 32, 1) decode_kernel(De
     const int sp_hi = min(t_hi, n_sg);  // sparse groups of the run: [t_lo, sp_hi)
     const int32_t* ptab = g.page_table + u * g.pages_per_unit;
 
+    if (threadIdx.x < kHeadDim) q_stage[threadIdx.x] = q_next;
     __syncthreads();  // the previous segment is done with shared memory
-    for (int i = threadIdx.x; i < kHeadDim * 32; i += NT)
-      qrep[i] = __ldg(p.qprime + ((b * p.H_q + h) * kHeadDim + (i >> 5)));
+    // q' copies (float4 f of the [128][16] layout holds row f / 4)
+    for (int f = threadIdx.x; f < kHeadDim * kQRep / 4; f += NT) {
+      const float v = q_stage[f >> 2];
+      reinterpret_cast<float4*>(qrep)[f] = make_float4(v, v, v, v);
+    }
+    {
+      float4* az = reinterpret_cast<float4*>(accs + warp * kHeadDim * 32);
 #pragma unroll 8
-    for (int dd = 0; dd < kHeadDim; ++dd) sts(ab + dd * 128, 0.f);
+      for (int f = lane; f < kHeadDim * 8; f += 32) az[f] = make_float4(0.f, 0.f, 0.f, 0.f);
+    }
     __syncthreads();
+    if (u < u_last && threadIdx.x < kHeadDim) q_next = q_of(u + 1);
 
     float m_w = -INFINITY;  // running max (log2 domain), uniform in the warp
     float l_sum = 0.f;      // this lane's sum of exp2(s - m_w)
@@ -534,15 +610,16 @@ __global__ void __launch_bounds__(decode_warps<MAXC>() * 32, 1) decode_kernel(De
         for (int c = 0; c < 16; ++c) {
           const uint4 w = __ldg(kr + c);
           const float2 a = h2f(w.x), bb = h2f(w.y), cc = h2f(w.z), d = h2f(w.w);
-          const uint32_t q = qb + c * 8 * 128;
-          s[0] = fmaf(lds(q + 0 * 128), a.x, s[0]);
-          s[1] = fmaf(lds(q + 1 * 128), a.y, s[1]);
-          s[2] = fmaf(lds(q + 2 * 128), bb.x, s[2]);
-          s[3] = fmaf(lds(q + 3 * 128), bb.y, s[3]);
-          s[0] = fmaf(lds(q + 4 * 128), cc.x, s[0]);
-          s[1] = fmaf(lds(q + 5 * 128), cc.y, s[1]);
-          s[2] = fmaf(lds(q + 6 * 128), d.x, s[2]);
-          s[3] = fmaf(lds(q + 7 * 128), d.y, s[3]);
+          constexpr uint32_t QR = 1u << kQRowShift;
+          const uint32_t q = qb + c * 8 * QR;
+          s[0] = fmaf(lds(q + 0 * QR), a.x, s[0]);
+          s[1] = fmaf(lds(q + 1 * QR), a.y, s[1]);
+          s[2] = fmaf(lds(q + 2 * QR), bb.x, s[2]);
+          s[3] = fmaf(lds(q + 3 * QR), bb.y, s[3]);
+          s[0] = fmaf(lds(q + 4 * QR), cc.x, s[0]);
+          s[1] = fmaf(lds(q + 5 * QR), cc.y, s[1]);
+          s[2] = fmaf(lds(q + 6 * QR), d.x, s[2]);
+          s[3] = fmaf(lds(q + 7 * QR), d.y, s[3]);
         }
         s2 = valid ? ((s[0] + s[1]) + (s[2] + s[3])) * p.scale_log2 : -INFINITY;
         const float gmax = warp_max(s2);
@@ -579,8 +656,24 @@ __global__ void __launch_bounds__(decode_warps<MAXC>() * 32, 1) decode_kernel(De
       }
     }
 
-    // ---- merge the lanes and warps into one partial
+    // ---- merge the lanes and warps into one partial: each warp sums its
+    // lanes' accumulators (lane l coordinates l, l+32, l+64, l+96, reading
+    // the columns in rotated order: conflict-free) into the first 128 floats
+    // of its region, then one thread per coordinate combines the warps
     l_sum = warp_sum(l_sum);
+    {
+      float* a = accs + warp * kHeadDim * 32;
+      float sum[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll 8
+      for (int jj = 0; jj < 32; ++jj) {
+        const int col = (jj + lane) & 31;
+#pragma unroll
+        for (int k = 0; k < 4; ++k) sum[k] += a[(lane + 32 * k) * 32 + col];
+      }
+      __syncwarp();
+#pragma unroll
+      for (int k = 0; k < 4; ++k) a[lane + 32 * k] = sum[k];
+    }
     if (lane == 0) {
       red_m[warp] = m_w;
       red_l[warp] = l_sum;
@@ -597,11 +690,7 @@ __global__ void __launch_bounds__(decode_warps<MAXC>() * 32, 1) decode_kernel(De
       for (int w = 0; w < NW; ++w) {
         const float mw = red_m[w];
         const float f = (mw == -INFINITY) ? 0.f : exp2f(mw - M);
-        const float* a = accs + w * kHeadDim * 32 + dd * 32;
-        float sum = 0.f;
-#pragma unroll 8
-        for (int jj = 0; jj < 32; ++jj) sum += a[(jj + dd) & 31];
-        tot = fmaf(f, sum, tot);
+        tot = fmaf(f, accs[w * kHeadDim * 32 + dd], tot);
         L = fmaf(f, red_l[w], L);
       }
       if (solo) {
@@ -617,7 +706,7 @@ __global__ void __launch_bounds__(decode_warps<MAXC>() * 32, 1) decode_kernel(De
     }
     if (solo) {
       __syncthreads();
-      rotate_back_out<1, NT>(p, b, h, qrep);
+      rotate_back_out<1, NT>(p, b, h, qrep, qrep + kHeadDim);
     } else {
       finish_unit<1, NT>(p, c0, c1, u, b, h, qrep, red_m);
     }
@@ -1069,7 +1158,7 @@ __global__ void __launch_bounds__(mma_warps<MAXC>() * 32, 1) decode_mma_kernel(D
     // the o rows overwrote part of the tiles: zero them again
     for (int c = 0; c < 16; ++c) sts_v4(vrow + c * 16, make_uint4(0, 0, 0, 0));
     if (solo) {
-      rotate_back_out<G, NT>(p, b, h, qrep);
+      rotate_back_out<G, NT>(p, b, h, qrep, qrep + G * kHeadDim);
     } else {
       finish_unit<G, NT>(p, c0, c1, u, b, h, qrep, flag);
     }

@@ -634,8 +634,12 @@ namespace {
 // positions 0..n_b-1 are the buffered tokens (oldest first), n_b..n_b+T_b-1
 // the new ones; everything before evict = max(0, n_b + T_b - b_cap) goes to
 // the sparse history, in order.
+// Append (Algorithm 1, compression part).  rq non-null: a decode step's query
+// rotation that may run in the append's own launch; *rotated says whether it
+// did (only a small append takes it).
 swan_status append_rows(swan_ctx* c, int layer, const void* k_new, const void* v_new, int T,
-                        const int32_t* n_new) {
+                        const int32_t* n_new, const RotateQParams* rq = nullptr, bool* rotated = nullptr) {
+  if (rotated) *rotated = false;
   swan_status s = usable(c);
   if (s != SWAN_OK) return s;
   if ((s = check_layer(c, layer)) != SWAN_OK) return s;
@@ -754,12 +758,13 @@ swan_status append_rows(swan_ctx* c, int layer, const void* k_new, const void* v
   p.geom = geom_for(c, layer);
   p.status = c->status;
   if (small)
-    s = launch(c, SWAN_KERNEL_APPEND, "append_small kernel",
-               [&] { return launch_append_small(p, most_old, c->stream); });
+    s = launch(c, SWAN_KERNEL_APPEND, rq ? "append_rotate kernel" : "append_small kernel",
+               [&] { return launch_append_small(p, most_old, rq, c->stream); });
   else
     s = launch(c, SWAN_KERNEL_APPEND, "append kernel",
                [&] { return launch_append_tc(p, maps, layer * 2 * c->cfg.n_kv_heads, c->stream); });
   if (s != SWAN_OK) return s;
+  if (rotated) *rotated = small && rq != nullptr;
 
   for (int b = 0; b < B; ++b) {
     SeqState& q = L.seq[b];
@@ -826,28 +831,39 @@ swan_status swan_reset_sequence(swan_ctx* c, int b) {
   return SWAN_OK;
 }
 
-swan_status swan_decode(swan_ctx* c, int layer, const void* q, void* out) {
-  swan_status s = usable(c);
-  if (s != SWAN_OK) return s;
-  if ((s = check_layer(c, layer)) != SWAN_OK) return s;
+namespace {
+
+swan_status check_decode_args(const swan_ctx* c, const void* q, const void* out) {
   if (!q || !out) return fail(SWAN_ERR_INVALID_ARG, "q or out is NULL");
   const size_t qbytes = (size_t)c->cfg.batch * c->cfg.n_q_heads * kHeadDim * 2;
   const char* qa = static_cast<const char*>(q);
   const char* oa = static_cast<const char*>(out);
   if (qa < oa + qbytes && oa < qa + qbytes) return fail(SWAN_ERR_INVALID_ARG, "q and out overlap");
-  const LayerState& L = c->layers[layer];
-  const int G = c->G;
-  const float* R_qk = c->R_qk + (size_t)layer * c->cfg.n_kv_heads * kHeadDim * kHeadDim;
+  return SWAN_OK;
+}
 
+// q' = q R_qk of one layer into the context's q' buffer (Section 4.3).
+RotateQParams rotation_of(const swan_ctx* c, int layer, const void* q) {
   RotateQParams rq{};
   rq.q = static_cast<const __half*>(q);
-  rq.R_qk = R_qk;
+  rq.R_qk = c->R_qk + (size_t)layer * c->cfg.n_kv_heads * kHeadDim * kHeadDim;
   rq.qprime = c->qprime;
   rq.H_q = c->cfg.n_q_heads;
-  rq.G = G;
-  s = launch(c, SWAN_KERNEL_ROTATE_Q, "rotate_q kernel",
-             [&] { return launch_rotate_q(rq, c->cfg.batch, c->stream); });
-  if (s != SWAN_OK) return s;
+  rq.G = c->G;
+  return rq;
+}
+
+swan_status launch_rotation(swan_ctx* c, const RotateQParams& rq) {
+  return launch(c, SWAN_KERNEL_ROTATE_Q, "rotate_q kernel",
+                [&] { return launch_rotate_q(rq, c->cfg.batch, c->stream); });
+}
+
+// Attention of the rotated queries (already in the q' buffer) over the
+// layer's cache, split-K combine and rotate-back into `out`.
+swan_status decode_rotated(swan_ctx* c, int layer, void* out) {
+  swan_status s = SWAN_OK;
+  const LayerState& L = c->layers[layer];
+  const int G = c->G;
 
   // Uniform rows: every unit has the same groups.  Ragged rows: each row's
   // groups (at least one, so an empty row still writes its zero output),
@@ -939,6 +955,30 @@ swan_status swan_decode(swan_ctx* c, int layer, const void* q, void* out) {
   cp.total_groups = total;
   return launch(c, SWAN_KERNEL_COMBINE, "combine kernel",
                 [&] { return launch_combine(cp, c->cfg.batch, c->stream); });
+}
+
+}  // namespace
+
+swan_status swan_decode(swan_ctx* c, int layer, const void* q, void* out) {
+  swan_status s = usable(c);
+  if (s != SWAN_OK) return s;
+  if ((s = check_layer(c, layer)) != SWAN_OK) return s;
+  if ((s = check_decode_args(c, q, out)) != SWAN_OK) return s;
+  if ((s = launch_rotation(c, rotation_of(c, layer, q))) != SWAN_OK) return s;
+  return decode_rotated(c, layer, out);
+}
+
+swan_status swan_append_decode(swan_ctx* c, int layer, const void* k_new, const void* v_new, int T,
+                               const int32_t* n_new, const void* q, void* out) {
+  swan_status s = usable(c);
+  if (s != SWAN_OK) return s;
+  if ((s = check_layer(c, layer)) != SWAN_OK) return s;
+  if ((s = check_decode_args(c, q, out)) != SWAN_OK) return s;
+  const RotateQParams rq = rotation_of(c, layer, q);
+  bool rotated = false;
+  if ((s = append_rows(c, layer, k_new, v_new, T, n_new, &rq, &rotated)) != SWAN_OK) return s;
+  if (!rotated && (s = launch_rotation(c, rq)) != SWAN_OK) return s;
+  return decode_rotated(c, layer, out);
 }
 
 swan_status swan_query(const swan_ctx* c, int layer, swan_layer_info* info) {

@@ -46,6 +46,7 @@ constexpr float kLazyRescale = 8.0f;
 constexpr unsigned kStatusPageRange = 1u;
 constexpr unsigned kStatusRingRange = 2u;
 constexpr unsigned kStatusTimeout = 4u;  // a bounded barrier wait gave up
+constexpr unsigned kStatusLayout = 8u;   // too little shared memory for a kernel's layout (kernel skipped)
 
 constexpr int kFmtFp16 = 0;  // fp16 values
 constexpr int kFmtFp8 = 1;   // E4M3 values
@@ -214,6 +215,42 @@ __device__ __forceinline__ void stage_matrix(float* dst, const float* src) {
 #pragma unroll
   for (int k = 0; k < 16; ++k) reinterpret_cast<float4*>(dst)[threadIdx.x + k * kThreads] = r[k];
 }
+
+// One slice of q' = q R_qk (Section 4.3: the query is rotated once, the cache
+// never is): query vectors [8 chunk, 8 chunk + 8) of kv head h (row-major
+// over (b, group member)), output coordinates [32 z, 32 z + 32).  Stages the
+// 128 x 32 slice of R in Rs (16 KB of shared memory), waits for the previous
+// kernel, then one warp per query vector: lane l computes coordinate 32 z + l
+// as a sequential fp32 FMA chain over the 128 inputs.  The query-rotation
+// kernel and the fused append + rotation kernel both run this, so q' has the
+// same bits either way.
+__device__ __forceinline__ void rotate_q_slice(const RotateQParams& p, int B, int h, int chunk, int z,
+                                               float* Rs) {
+  const float* R = p.R_qk + (size_t)h * kHeadDim * kHeadDim + z * 32;
+  for (int e = threadIdx.x; e < kHeadDim * 8; e += kThreads) {  // 128 rows x 8 float4
+    const int i = e >> 3, c = e & 7;
+    reinterpret_cast<float4*>(Rs)[e] = __ldg(reinterpret_cast<const float4*>(R + i * kHeadDim) + c);
+  }
+  __syncthreads();
+  pdl_wait();
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  for (int item = chunk * kWarpsPerCta + warp; item < min(B * p.G, (chunk + 1) * kWarpsPerCta);
+       item += kWarpsPerCta) {
+    const int b = item / p.G, gh = item % p.G;
+    const int64_t bq = (int64_t)b * p.H_q + h * p.G + gh;
+    const uint2 xw = __ldg(reinterpret_cast<const uint2*>(p.q + bq * kHeadDim) + lane);
+    const float2 x01 = __half22float2(*reinterpret_cast<const __half2*>(&xw.x));
+    const float2 x23 = __half22float2(*reinterpret_cast<const __half2*>(&xw.y));
+    const float xs[4] = {x01.x, x01.y, x23.x, x23.y};
+    float acc = 0.f;
+#pragma unroll 16
+    for (int i = 0; i < kHeadDim; ++i) {
+      const float xi = __shfl_sync(0xffffffffu, xs[i & 3], i >> 2);
+      acc = fmaf(xi, Rs[i * 32 + lane], acc);
+    }
+    p.qprime[bq * kHeadDim + z * 32 + lane] = acc;
+  }
+}
 #endif
 
 // Raise a kernel's dynamic shared-memory limit once per device (the limit
@@ -246,8 +283,9 @@ using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t
                                    CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
 EncodeTiledFn tensor_map_encoder();
 // Eviction of `evict_old` buffered tokens and insertion of T new ones in one
-// launch; for small batch * T (decode steps).
-cudaError_t launch_append_small(const AppendParams& p, int evict_old, cudaStream_t s);
+// launch; for small batch * T (decode steps).  With rq non-null the same
+// launch also computes the query rotation q' = q R_qk of rq.
+cudaError_t launch_append_small(const AppendParams& p, int evict_old, const RotateQParams* rq, cudaStream_t s);
 cudaError_t launch_prune_ring(const PruneRingParams& p, cudaStream_t s);
 cudaError_t launch_rotate_q(const RotateQParams& p, int B, cudaStream_t s);
 // k_read: entries read per vector rounded up to 8 (selects the kernel variant)

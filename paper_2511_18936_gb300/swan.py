@@ -31,7 +31,7 @@ EXPORTED = ["swan_init", "swan_destroy", "swan_set_k", "swan_append", "swan_flus
             "swan_status_string", "swan_last_error", "swan_decode_noalloc", "swan_set_kv",
             "swan_gram_workspace_bytes", "swan_gram", "swan_basis_eig", "swan_energy",
             "swan_basis_check", "swan_append_varlen", "swan_reset_sequence", "swan_query_lengths",
-            "swan_debug_export_seq"]
+            "swan_debug_export_seq", "swan_append_decode"]
 
 
 class SwanConfig(ctypes.Structure):
@@ -107,6 +107,7 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "swan_debug_export_seq": (i, [vp, i, i, i, vp, ctypes.c_size_t]),
         "swan_flush_buffer": (i, [vp, i]),
         "swan_decode": (i, [vp, i, vp, vp]),
+        "swan_append_decode": (i, [vp, i, vp, vp, i, ctypes.POINTER(ctypes.c_int32), vp, vp]),
         "swan_query": (i, [vp, i, ctypes.POINTER(LayerInfo)]),
         "swan_debug_export": (i, [vp, i, i, vp, ctypes.c_size_t]),
         "swan_check": (i, [vp]),
@@ -233,6 +234,20 @@ class Context:
             import torch
             out = torch.empty_like(q)
         _check(self._lib.swan_decode(self._h, int(layer), _ptr(q), _ptr(out)), "swan_decode")
+        return out
+
+    def append_decode(self, layer: int, k_new, v_new, q, out=None, T: int | None = None, n_new=None):
+        """One serving step: ``append(layer, k_new, v_new, T, n_new)`` then
+        ``decode(layer, q, out)`` (the query rotation runs inside the append's
+        launch for a decode-step append)."""
+        if T is None:
+            T = k_new.shape[2]
+        if out is None:
+            import torch
+            out = torch.empty_like(q)
+        counts = None if n_new is None else (ctypes.c_int32 * self.batch)(*[int(x) for x in n_new])
+        _check(self._lib.swan_append_decode(self._h, int(layer), _ptr(k_new), _ptr(v_new), int(T), counts,
+                                            _ptr(q), _ptr(out)), "swan_append_decode")
         return out
 
     # -- inspection --------------------------------------------------------

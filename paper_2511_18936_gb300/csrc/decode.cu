@@ -14,43 +14,11 @@ __global__ void __launch_bounds__(kThreads) rotate_q_kernel(RotateQParams p, int
   rotate_q_slice(p, B, blockIdx.x, blockIdx.y, blockIdx.z, Rs);
 }
 
-// Empty cache: writes zeros (the rotate-back of an empty attention).
+// Empty cache: the output is zero (one CTA per query vector).
 __global__ void __launch_bounds__(kHeadDim) combine_kernel(CombineParams p) {
-  __shared__ float o_hat[kHeadDim];
   pdl_trigger();
   pdl_wait();
-  const int64_t bq = blockIdx.x;
-  const int64_t b = bq / p.H_q;
-  const int hq = (int)(bq % p.H_q);
-  const int h = hq / p.G, gh = hq % p.G;
-  const int64_t u = b * p.H_kv + h;
-  const int dd = threadIdx.x;
-  float val = 0.f;
-  if (p.total_groups > 0) {
-    const int64_t c0 = (u * p.N_g) / p.range;
-    const int64_t c1 = ((u + 1) * p.N_g - 1) / p.range;
-    float M = -INFINITY;
-    for (int64_t c = c0; c <= c1; ++c)
-      M = fmaxf(M, p.partials[((size_t)(c + u) * p.G + gh) * (kHeadDim + 2)]);
-    float L = 0.f, A = 0.f;
-    for (int64_t c = c0; c <= c1; ++c) {
-      const float* part = p.partials + ((size_t)(c + u) * p.G + gh) * (kHeadDim + 2);
-      const float w = (part[0] == -INFINITY) ? 0.f : exp2f(part[0] - M);
-      L = fmaf(w, part[1], L);
-      A = fmaf(w, part[2 + dd], A);
-    }
-    val = (L > 0.f) ? A / L : 0.f;
-  }
-  o_hat[dd] = val;
-  __syncthreads();
-  const float* RT = p.R_voT + (size_t)h * kHeadDim * kHeadDim;
-  float a0 = 0.f, a1 = 0.f;
-#pragma unroll 8
-  for (int j = 0; j < kHeadDim; j += 2) {
-    a0 = fmaf(o_hat[j], __ldg(RT + j * kHeadDim + dd), a0);
-    a1 = fmaf(o_hat[j + 1], __ldg(RT + (j + 1) * kHeadDim + dd), a1);
-  }
-  p.out[bq * kHeadDim + dd] = __float2half_rn(a0 + a1);
+  p.out[(int64_t)blockIdx.x * kHeadDim + threadIdx.x] = __float2half_rn(0.f);
 }
 
 // Dynamic shared memory of the one-head kernel: the warps' accumulators and

@@ -270,12 +270,29 @@ __device__ __forceinline__ int split_at(int s0, int s1, int n_sg, int part, int 
 }
 
 // First group of CTA c (c <= gridDim.x) and the CTA that holds group g.
+// Ragged rows: the host's table.  Uniform rows: unit u's groups take cost
+// positions [u U, u U + N_g) with U = N_g + V, and V positions follow each
+// unit but the last (the extra visit a CTA crossing into the next unit
+// pays); CTA c starts at cost x_c = floor(c T / grid), T = units U - V, at
+// the first group at or after x_c.  Group g (unit u, offset o) sits at
+// y = u U + o, and cta_begin(c) <= g exactly when x_c <= y, so the CTA
+// holding g is the last c with x_c <= y: floor(((y + 1) grid - 1) / T).
 __device__ __forceinline__ int64_t cta_begin(const DecodeParams& p, int64_t c) {
-  if (p.cta_start == nullptr) return min(p.total_groups, c * p.range);
-  return p.cta_start[c];
+  if (p.cta_start != nullptr) return p.cta_start[c];
+  const int64_t U = p.N_g + p.visit_cost;
+  const int64_t T = (p.total_groups / p.N_g) * U - p.visit_cost;
+  const int64_t x = c * T / (int64_t)gridDim.x;
+  const int64_t u = x / U;
+  return u * p.N_g + min(x - u * U, p.N_g);
 }
 __device__ __forceinline__ int64_t cta_of(const DecodeParams& p, int64_t g) {
-  if (p.cta_start == nullptr) return g / p.range;
+  if (p.cta_start == nullptr) {
+    const int64_t U = p.N_g + p.visit_cost;
+    const int64_t u = g / p.N_g;
+    const int64_t y = u * U + (g - u * p.N_g);
+    const int64_t T = (p.total_groups / p.N_g) * U - p.visit_cost;
+    return min((int64_t)gridDim.x - 1, ((y + 1) * (int64_t)gridDim.x - 1) / T);
+  }
   int lo = 0, hi = (int)gridDim.x - 1;  // the last CTA whose first group is <= g
   while (lo < hi) {
     const int mid = (lo + hi + 1) >> 1;
@@ -286,65 +303,59 @@ __device__ __forceinline__ int64_t cta_of(const DecodeParams& p, int64_t g) {
 }
 
 // out = o_hat R_vo^T for the G query heads of unit (b, h); o_hat in shared
-// memory [G][128].  With at least twice as many threads as outputs, each
-// output's 128-term sum is cut into S = NT / (128 G) slices computed by
-// different threads (partial sums in `part`, S * G * 128 floats of shared
-// memory apart from o_hat), so more loads of R_vo^T are in flight at once.
+// memory [G][128].  Thread t takes outputs 4q..4q+3 (q = t % 32) of every
+// head over rows j of slice t / 32 (S = NT / 32 slices of the 128 rows): its
+// float4 loads of R_vo^T are independent, so they are in flight together,
+// and each element serves all G heads.  The slices' partial sums meet in
+// `part` (S * G * 128 floats of shared memory, which may overlap o_hat) and
+// are added in slice order.
 template <int G, int NT>
 __device__ __forceinline__ void rotate_back_out(const DecodeParams& p, int64_t b, int64_t h, const float* o_hat,
                                                 float* part) {
-  constexpr int OUT = G * kHeadDim;
-  constexpr int S = NT >= 2 * OUT ? NT / OUT : 1;
-  const float* RT = p.R_voT + (size_t)h * kHeadDim * kHeadDim;
-  if constexpr (S == 1) {
-    for (int o = threadIdx.x; o < OUT; o += NT) {
-      const int gh = o / kHeadDim, i = o % kHeadDim;
-      const float* oh = o_hat + gh * kHeadDim;
-      float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
-#pragma unroll 8
-      for (int j = 0; j < kHeadDim; j += 4) {
-        a0 = fmaf(oh[j + 0], __ldg(RT + (j + 0) * kHeadDim + i), a0);
-        a1 = fmaf(oh[j + 1], __ldg(RT + (j + 1) * kHeadDim + i), a1);
-        a2 = fmaf(oh[j + 2], __ldg(RT + (j + 2) * kHeadDim + i), a2);
-        a3 = fmaf(oh[j + 3], __ldg(RT + (j + 3) * kHeadDim + i), a3);
-      }
-      p.out[((b * p.H_q) + h * G + gh) * kHeadDim + i] = __float2half_rn((a0 + a1) + (a2 + a3));
-    }
-  } else {
-    const int t = threadIdx.x;
-    if (t < S * OUT) {
-      const int o = t % OUT, sl = t / OUT;
-      const int gh = o / kHeadDim, i = o % kHeadDim;
-      const float* oh = o_hat + gh * kHeadDim;
-      const int j0 = sl * kHeadDim / S, j1 = (sl + 1) * kHeadDim / S;
-      float a0 = 0.f, a1 = 0.f;
-      int j = j0;
-#pragma unroll 4
-      for (; j + 1 < j1; j += 2) {
-        a0 = fmaf(oh[j + 0], __ldg(RT + (j + 0) * kHeadDim + i), a0);
-        a1 = fmaf(oh[j + 1], __ldg(RT + (j + 1) * kHeadDim + i), a1);
-      }
-      if (j < j1) a0 = fmaf(oh[j], __ldg(RT + j * kHeadDim + i), a0);
-      part[sl * OUT + o] = a0 + a1;
-    }
-    __syncthreads();
-    for (int o = t; o < OUT; o += NT) {
-      const int gh = o / kHeadDim, i = o % kHeadDim;
-      float a = 0.f;
+  constexpr int S = NT / 32;
+  static_assert(NT % 32 == 0 && S >= 1, "whole warps");
+  const int q = threadIdx.x & 31, sl = threadIdx.x >> 5;
+  const int j0 = sl * kHeadDim / S, j1 = (sl + 1) * kHeadDim / S;
+  const float4* RT4 = reinterpret_cast<const float4*>(p.R_voT + (size_t)h * kHeadDim * kHeadDim);
+  float acc[G][4];
 #pragma unroll
-      for (int k = 0; k < S; ++k) a += part[k * OUT + o];
-      p.out[((b * p.H_q) + h * G + gh) * kHeadDim + i] = __float2half_rn(a);
+  for (int gh = 0; gh < G; ++gh) acc[gh][0] = acc[gh][1] = acc[gh][2] = acc[gh][3] = 0.f;
+#pragma unroll 8
+  for (int j = j0; j < j1; ++j) {
+    const float4 r = __ldg(RT4 + j * (kHeadDim / 4) + q);
+#pragma unroll
+    for (int gh = 0; gh < G; ++gh) {
+      const float o = o_hat[gh * kHeadDim + j];
+      acc[gh][0] = fmaf(o, r.x, acc[gh][0]);
+      acc[gh][1] = fmaf(o, r.y, acc[gh][1]);
+      acc[gh][2] = fmaf(o, r.z, acc[gh][2]);
+      acc[gh][3] = fmaf(o, r.w, acc[gh][3]);
     }
+  }
+  __syncthreads();  // o_hat is read; part may reuse it
+#pragma unroll
+  for (int gh = 0; gh < G; ++gh)
+    reinterpret_cast<float4*>(part + (sl * G + gh) * kHeadDim)[q] =
+        make_float4(acc[gh][0], acc[gh][1], acc[gh][2], acc[gh][3]);
+  __syncthreads();
+  for (int o = threadIdx.x; o < G * kHeadDim; o += NT) {
+    const int gh = o / kHeadDim, i = o % kHeadDim;
+    float a = 0.f;
+#pragma unroll
+    for (int k = 0; k < S; ++k) a += part[(k * G + gh) * kHeadDim + i];
+    p.out[((b * p.H_q) + h * G + gh) * kHeadDim + i] = __float2half_rn(a);
   }
 }
 
 // The last CTA to finish a segment of unit u merges the unit's partials,
 // normalises, rotates back (o = o_hat R_vo^T) and writes the output.  The
 // arrival counter resets itself for the next decode; nothing waits.
-// `scratch` holds (S + 1) * G * 128 floats (free at this point; S as in
-// rotate_back_out); `flag` one float.  Every thread's partial writes are
-// ordered before thread 0's fence by the barrier, and the fence before the
-// arrival (the release pattern of a grid-wide barrier).
+// `scratch` holds NT / 32 * G * 128 floats (free at this point); `flag` one
+// float.  Every thread's partial writes are ordered before thread 0's fence
+// by the barrier, and the fence before the arrival (the release pattern of a
+// grid-wide barrier).  Each thread merges its outputs' n = c1 - c0 + 1
+// partials eight at a time with all their loads issued together (an online
+// max over the batches), so a merge costs one round trip per batch.
 // (A unit that one CTA holds entirely never comes here: it is finished from
 // shared memory by that CTA.)
 template <int G, int NT>
@@ -363,24 +374,42 @@ __device__ __forceinline__ void finish_unit(const DecodeParams& p, int64_t c0, i
   }
   __syncthreads();
   if (flag[0] == 0.f) return;
+  const int n = (int)(c1 - c0 + 1);
   float* o_hat = scratch;  // [G][128]
   for (int o = threadIdx.x; o < G * kHeadDim; o += NT) {
     const int gh = o / kHeadDim, dd = o % kHeadDim;
-    float M = -INFINITY;
-    for (int64_t c = c0; c <= c1; ++c)
-      M = fmaxf(M, __ldcg(p.partials + ((size_t)(c + u) * G + gh) * (kHeadDim + 2)));
-    float L = 0.f, A = 0.f;
-    for (int64_t c = c0; c <= c1; ++c) {
-      const float* part = p.partials + ((size_t)(c + u) * G + gh) * (kHeadDim + 2);
-      const float mc = __ldcg(part);
-      const float w = (mc == -INFINITY) ? 0.f : exp2f(mc - M);
-      L = fmaf(w, __ldcg(part + 1), L);
-      A = fmaf(w, __ldcg(part + 2 + dd), A);
+    float M = -INFINITY, L = 0.f, A = 0.f;
+    for (int cb = 0; cb < n; cb += 8) {
+      float mc[8], lc[8], ac[8];
+#pragma unroll
+      for (int k = 0; k < 8; ++k) {
+        mc[k] = -INFINITY, lc[k] = 0.f, ac[k] = 0.f;
+        if (cb + k < n) {
+          const float* part = p.partials + ((size_t)(c0 + cb + k + u) * G + gh) * (kHeadDim + 2);
+          mc[k] = __ldcg(part);
+          lc[k] = __ldcg(part + 1);
+          ac[k] = __ldcg(part + 2 + dd);
+        }
+      }
+      float Mn = M;
+#pragma unroll
+      for (int k = 0; k < 8; ++k) Mn = fmaxf(Mn, mc[k]);
+      if (Mn == -INFINITY) continue;  // nothing attended so far
+      const float f = (M == -INFINITY) ? 0.f : exp2f(M - Mn);
+      L *= f;
+      A *= f;
+#pragma unroll
+      for (int k = 0; k < 8; ++k) {
+        const float w = (mc[k] == -INFINITY) ? 0.f : exp2f(mc[k] - Mn);
+        L = fmaf(w, lc[k], L);
+        A = fmaf(w, ac[k], A);
+      }
+      M = Mn;
     }
     o_hat[o] = (L > 0.f) ? A / L : 0.f;
   }
   __syncthreads();
-  rotate_back_out<G, NT>(p, b, h, o_hat, scratch + G * kHeadDim);
+  rotate_back_out<G, NT>(p, b, h, o_hat, scratch);
 }
 
 // Warps per CTA of the one-head kernel: one lane-private accumulator each
@@ -706,7 +735,7 @@ __global__ void __launch_bounds__(decode_warps<MAXC>() * 32, decode_min_ctas<MAX
     }
     if (solo) {
       __syncthreads();
-      rotate_back_out<1, NT>(p, b, h, qrep, qrep + kHeadDim);
+      rotate_back_out<1, NT>(p, b, h, qrep, qrep);
     } else {
       finish_unit<1, NT>(p, c0, c1, u, b, h, qrep, red_m);
     }
@@ -720,10 +749,10 @@ __global__ void __launch_bounds__(decode_warps<MAXC>() * 32, decode_min_ctas<MAX
 //   ([128][32][G] fp32: one 8- or 16-byte conflict-free gather per entry).
 //   The value product o_h += sum_t p_h(t) v_t is dense once the kept
 //   entries are scattered into a zero-filled [32 tokens][128] fp16 tile per
-//   warp, so it runs as mma.sync.m16n8k16 (rows = the G heads, k = the 32
-//   tokens, n = the 128 coordinates) with the fp32 accumulators in
-//   registers; p is split into fp16 hi + lo parts (two products), so the
-//   result keeps fp32 accuracy.  No per-warp shared accumulator: the tile
+//   warp, so it runs as mma.sync.m16n8k16 (k = the 32 tokens, n = the 128
+//   coordinates) with the fp32 accumulators in registers; p is split into
+//   fp16 hi + lo parts, rows 0..G-1 and G..2G-1 of the same product, so the
+//   result keeps fp32 accuracy at one product per tile.  No per-warp shared accumulator: the tile
 //   and a [G][32] p table are all a warp holds in shared memory.
 // ---------------------------------------------------------------------------
 constexpr int kVRowBytes = 272;                      // 128 fp16 + 16 B pad: conflict-free ldmatrix rows
@@ -820,22 +849,25 @@ __device__ __forceinline__ void chunk_half_words(const Chunk<FMT>& ch, uint32_t 
   }
 }
 // Scores of G heads for one chunk: q' row idx of this lane is G floats.
+// Even and odd entries go to two partial sums per head (half-length FMA
+// chains).
 template <int G>
-__device__ __forceinline__ void score_g_chunk(uint32_t qb, const float (&f)[8], uint2 ix, float (&s)[G]) {
+__device__ __forceinline__ void score_g_chunk(uint32_t qb, const float (&f)[8], uint2 ix, float (&s)[2][G]) {
 #pragma unroll
   for (int e = 0; e < 8; ++e) {
     const uint32_t w = e < 4 ? ix.x : ix.y;
     const uint32_t a = qb + ((w >> (8 * (e & 3))) & 0x7fu) * 128u;
+    float* t = s[e & 1];
     if constexpr (G == 4) {
       const float4 q = lds4(a);
-      s[0] = fmaf(q.x, f[e], s[0]);
-      s[1] = fmaf(q.y, f[e], s[1]);
-      s[2] = fmaf(q.z, f[e], s[2]);
-      s[3] = fmaf(q.w, f[e], s[3]);
+      t[0] = fmaf(q.x, f[e], t[0]);
+      t[1] = fmaf(q.y, f[e], t[1]);
+      t[2] = fmaf(q.z, f[e], t[2]);
+      t[3] = fmaf(q.w, f[e], t[3]);
     } else {
       const float2 q = lds2(a);
-      s[0] = fmaf(q.x, f[e], s[0]);
-      s[1] = fmaf(q.y, f[e], s[1]);
+      t[0] = fmaf(q.x, f[e], t[0]);
+      t[1] = fmaf(q.y, f[e], t[1]);
     }
   }
 }
@@ -859,6 +891,9 @@ __global__ void __launch_bounds__(mma_warps<MAXC>() * 32, 1) decode_mma_kernel(D
   extern __shared__ __align__(16) unsigned char smem_raw[];
   __shared__ float red_m[NW * G], red_l[NW * G];
   __shared__ float flag[1];
+  __shared__ __align__(16) float q_stage[G * kHeadDim];  // q' of the next unit's G heads
+  static_assert(G * kHeadDim % NT == 0, "whole q' loads per thread");
+  constexpr int QL = G * kHeadDim / NT;  // q' floats each thread loads
   pdl_trigger();
 
   const uint32_t raw = (uint32_t)__cvta_generic_to_shared(smem_raw);
@@ -889,6 +924,16 @@ __global__ void __launch_bounds__(mma_warps<MAXC>() * 32, 1) decode_mma_kernel(D
   pdl_wait();
   if (g_begin >= g_end) return;
   const int64_t u_first = unit_of(p, g_begin), u_last = unit_of(p, g_end - 1);
+  // q' of the G heads of the unit the next segment starts (G * 128
+  // consecutive floats): coalesced loads issued a segment ahead
+  float q_next[QL];
+  auto load_q = [&](int64_t un) {
+    const int64_t bn = un / p.H_kv, hn = un - bn * p.H_kv;
+    const float* src = p.qprime + (bn * p.H_q + hn * G) * kHeadDim;
+#pragma unroll
+    for (int k = 0; k < QL; ++k) q_next[k] = __ldg(src + threadIdx.x + k * NT);
+  };
+  load_q(u_first);
 
   // the tiles start zeroed; every use restores the zeros it disturbed
   for (int c = 0; c < 16; ++c) sts_v4(vrow + c * 16, make_uint4(0, 0, 0, 0));
@@ -904,12 +949,22 @@ __global__ void __launch_bounds__(mma_warps<MAXC>() * 32, 1) decode_mma_kernel(D
     const int sp_hi = min(t_hi, n_sg);
     const int32_t* ptab = g.page_table + u * g.pages_per_unit;
 
-    __syncthreads();  // the previous segment is done with q'
-    for (int i = threadIdx.x; i < kHeadDim * 32; i += NT) {
-      const int c = i / 32, j = i % G;  // 32 floats per coordinate: 32 / G copies of G heads
-      qrep[i] = __ldg(p.qprime + ((b * p.H_q + h * G + j) * kHeadDim + c));
+#pragma unroll
+    for (int k = 0; k < QL; ++k) q_stage[threadIdx.x + k * NT] = q_next[k];
+    __syncthreads();  // the previous segment is done with q'; q_stage is set
+    // 32 floats per coordinate c: 32 / G copies of its G heads (float4 f
+    // holds coordinate f / 8, heads 0..3 or 0, 1, 0, 1)
+    for (int f = threadIdx.x; f < kHeadDim * 8; f += NT) {
+      const int c = f >> 3;
+      float4 v;
+      if constexpr (G == 4)
+        v = make_float4(q_stage[c], q_stage[kHeadDim + c], q_stage[2 * kHeadDim + c], q_stage[3 * kHeadDim + c]);
+      else
+        v = make_float4(q_stage[c], q_stage[kHeadDim + c], q_stage[c], q_stage[kHeadDim + c]);
+      reinterpret_cast<float4*>(qrep)[f] = v;
     }
     __syncthreads();
+    if (u < u_last) load_q(u + 1);
 
     float m[G], l[G];
 #pragma unroll
@@ -973,8 +1028,9 @@ __global__ void __launch_bounds__(mma_warps<MAXC>() * 32, 1) decode_mma_kernel(D
 
     for (int gi = t_lo; gi < t_hi; ++gi) {
       float s[G];
+      float s2[2][G];
 #pragma unroll
-      for (int j = 0; j < G; ++j) s[j] = 0.f;
+      for (int j = 0; j < G; ++j) s2[0][j] = s2[1][j] = 0.f;
       bool valid;
       if (gi < n_sg) {
         // ---- sparse tokens 32 gi .. 32 gi + 31
@@ -990,26 +1046,36 @@ __global__ void __launch_bounds__(mma_warps<MAXC>() * 32, 1) decode_mma_kernel(D
               float f[8];
               chunk_vals<FMT>(kc[c], f);
               if (krem && c == nchunks - 1) keep_first(f, krem);
-              score_g_chunk<G>(qb, f, chunk_idx<FMT>(kc[c]), s);
+              score_g_chunk<G>(qb, f, chunk_idx<FMT>(kc[c]), s2);
             }
         }
-        // this token's kept values (staged by cp.async) into its tile row
+#pragma unroll
+        for (int j = 0; j < G; ++j) s[j] = s2[0][j] + s2[1][j];
+        // this token's kept values (staged by cp.async) into its tile row;
+        // each staged chunk is read before the previous one is stored
         cp_async_wait_all();
         __syncwarp();
         if (valid) {
+          auto staged = [&](int c) {
+            Chunk<FMT> vc;
+            if constexpr (FMT == kFmtFp16) {
+              vc.v = lds_v4u(vstage + c * 512 + lane * 16);
+              vc.i = lds_v2u(vstage + nchunks_v * 512 + c * 256 + lane * 8);
+            } else {
+              vc.r = lds_v4u(vstage + c * 512 + lane * 16);
+            }
+            return vc;
+          };
+          Chunk<FMT> vc = staged(0);
 #pragma unroll
           for (int c = 0; c < MAXC; ++c)
             if (c < nchunks_v) {
-              Chunk<FMT> vc;
-              if constexpr (FMT == kFmtFp16) {
-                vc.v = lds_v4u(vstage + c * 512 + lane * 16);
-                vc.i = lds_v2u(vstage + nchunks_v * 512 + c * 256 + lane * 8);
-              } else {
-                vc.r = lds_v4u(vstage + c * 512 + lane * 16);
-              }
+              Chunk<FMT> vn = vc;
+              if (c + 1 < nchunks_v) vn = staged(c + 1);
               uint32_t w[4];
               chunk_half_words<FMT>(vc, w);
               scatter_chunk(vrow, w, chunk_idx<FMT>(vc), (krem_v && c == nchunks_v - 1) ? krem_v : 8);
+              vc = vn;
             }
         }
         __syncwarp();
@@ -1024,6 +1090,8 @@ __global__ void __launch_bounds__(mma_warps<MAXC>() * 32, 1) decode_mma_kernel(D
         // value row copied into the tile
         const int64_t i = (int64_t)(gi - n_sg) * 32 + lane;
         valid = i < uv.n_b;
+#pragma unroll
+        for (int j = 0; j < G; ++j) s[j] = 0.f;
         if (valid) {
           const int slot = (int)((uv.buf_start + i) % p.cap);
           const size_t row = ((size_t)u * p.cap + slot) * kHeadDim;
@@ -1037,19 +1105,22 @@ __global__ void __launch_bounds__(mma_warps<MAXC>() * 32, 1) decode_mma_kernel(D
 #pragma unroll
             for (int e = 0; e < 8; ++e) {
               const uint32_t qa = qb + (uint32_t)(c * 8 + e) * 128u;
+              float* t = s2[e & 1];
               if constexpr (G == 4) {
                 const float4 q = lds4(qa);
-                s[0] = fmaf(q.x, f[e], s[0]);
-                s[1] = fmaf(q.y, f[e], s[1]);
-                s[2] = fmaf(q.z, f[e], s[2]);
-                s[3] = fmaf(q.w, f[e], s[3]);
+                t[0] = fmaf(q.x, f[e], t[0]);
+                t[1] = fmaf(q.y, f[e], t[1]);
+                t[2] = fmaf(q.z, f[e], t[2]);
+                t[3] = fmaf(q.w, f[e], t[3]);
               } else {
                 const float2 q = lds2(qa);
-                s[0] = fmaf(q.x, f[e], s[0]);
-                s[1] = fmaf(q.y, f[e], s[1]);
+                t[0] = fmaf(q.x, f[e], t[0]);
+                t[1] = fmaf(q.y, f[e], t[1]);
               }
             }
           }
+#pragma unroll
+          for (int j = 0; j < G; ++j) s[j] = s2[0][j] + s2[1][j];
 #pragma unroll 4
           for (int c = 0; c < 16; ++c) sts_v4(vrow + c * 16, __ldg(vr + c));
         }
@@ -1065,7 +1136,7 @@ __global__ void __launch_bounds__(mma_warps<MAXC>() * 32, 1) decode_mma_kernel(D
           if (m[j] != -INFINITY) {
             const float fs = exp2f(m[j] - gmax);
             l[j] *= fs;
-            if (gq == j) {
+            if (gq == j || gq == j + G) {  // the head's hi and lo rows
 #pragma unroll
               for (int nt = 0; nt < 16; ++nt) acc[nt][0] *= fs, acc[nt][1] *= fs;
             }
@@ -1078,14 +1149,21 @@ __global__ void __launch_bounds__(mma_warps<MAXC>() * 32, 1) decode_mma_kernel(D
       }
       __syncwarp();
 
-      // ---- o[head][:] += p[head][tokens] * tile[tokens][:] on the tensor cores
+      // ---- o[head][:] += p[head][tokens] * tile[tokens][:] on the tensor cores:
+      // A rows 0..G-1 hold the fp16 hi parts of p, rows G..2G-1 the lo
+      // parts, so one product covers both (the two row sets are added at
+      // the merge)
 #pragma unroll
       for (int ks = 0; ks < 2; ++ks) {
-        uint32_t ahi0 = 0, alo0 = 0, ahi2 = 0, alo2 = 0;
-        if (gq < G) {
-          const float* pr = ptile_f + gq * 32 + ks * 16 + 2 * cq;
-          split_pair(pr[0], pr[1], ahi0, alo0);
-          split_pair(pr[8], pr[9], ahi2, alo2);
+        uint32_t a0 = 0, a2 = 0;
+        if (gq < 2 * G) {
+          const bool hi_row = gq < G;
+          const float* pr = ptile_f + (hi_row ? gq : gq - G) * 32 + ks * 16 + 2 * cq;
+          uint32_t hi0, lo0, hi2, lo2;
+          split_pair(pr[0], pr[1], hi0, lo0);
+          split_pair(pr[8], pr[9], hi2, lo2);
+          a0 = hi_row ? hi0 : lo0;
+          a2 = hi_row ? hi2 : lo2;
         }
 #pragma unroll
         for (int np = 0; np < 8; ++np) {
@@ -1094,10 +1172,8 @@ __global__ void __launch_bounds__(mma_warps<MAXC>() * 32, 1) decode_mma_kernel(D
                                 (uint32_t)(16 * np + 8 * (mi >> 1)) * 2;
           uint32_t bf[4];
           ldsm_x4_trans(addr, bf);
-          mma_16816(acc[2 * np], ahi0, ahi2, bf[0], bf[1]);
-          mma_16816(acc[2 * np], alo0, alo2, bf[0], bf[1]);
-          mma_16816(acc[2 * np + 1], ahi0, ahi2, bf[2], bf[3]);
-          mma_16816(acc[2 * np + 1], alo0, alo2, bf[2], bf[3]);
+          mma_16816(acc[2 * np], a0, a2, bf[0], bf[1]);
+          mma_16816(acc[2 * np + 1], a0, a2, bf[2], bf[3]);
         }
       }
       __syncwarp();
@@ -1116,7 +1192,13 @@ __global__ void __launch_bounds__(mma_warps<MAXC>() * 32, 1) decode_mma_kernel(D
         red_l[warp * G + j] = l[j];
       }
     }
-    // this warp's o rows into its tile region ([G][128] fp32)
+    // the lo rows (G..2G-1, lanes 4G above) onto the hi rows, then this
+    // warp's o rows into its tile region ([G][128] fp32)
+#pragma unroll
+    for (int nt = 0; nt < 16; ++nt) {
+      acc[nt][0] += __shfl_down_sync(0xffffffffu, acc[nt][0], 4 * G);
+      acc[nt][1] += __shfl_down_sync(0xffffffffu, acc[nt][1], 4 * G);
+    }
     __syncwarp();
     float* obuf = reinterpret_cast<float*>(base_ptr + (vtile - base));
     if (gq < G) {
@@ -1158,7 +1240,7 @@ __global__ void __launch_bounds__(mma_warps<MAXC>() * 32, 1) decode_mma_kernel(D
     // the o rows overwrote part of the tiles: zero them again
     for (int c = 0; c < 16; ++c) sts_v4(vrow + c * 16, make_uint4(0, 0, 0, 0));
     if (solo) {
-      rotate_back_out<G, NT>(p, b, h, qrep, qrep + G * kHeadDim);
+      rotate_back_out<G, NT>(p, b, h, qrep, qrep);
     } else {
       finish_unit<G, NT>(p, c0, c1, u, b, h, qrep, flag);
     }

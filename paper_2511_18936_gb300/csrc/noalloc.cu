@@ -125,13 +125,9 @@ extern "C" swan_status swan_decode_noalloc(const swan_cache_view* v, const void*
   const int64_t n_bg = ((int64_t)v->buf_len + 31) / 32;
   const int64_t N_g = n_sg + n_bg;
   const int64_t total = units * N_g;
-  int64_t range = 1, grid = 0;
-  if (total > 0) {
-    const int64_t ctas =
-        std::min<int64_t>((int64_t)ds->sms * ds->ctas_per_sm[gi(G)][std::max(v->k_active, kav) > 64], total);
-    range = (total + ctas - 1) / ctas;
-    grid = (total + range - 1) / range;
-  }
+  int64_t grid = 0;
+  if (total > 0)
+    grid = std::min<int64_t>((int64_t)ds->sms * ds->ctas_per_sm[gi(G)][std::max(v->k_active, kav) > 64], total);
   if ((grid + units) * G > kNoallocMaxSlots)
     return err(SWAN_ERR_INVALID_ARG, "(decode CTAs + batch * n_kv_heads) * G exceeds 2048 (static scratch)");
 
@@ -177,7 +173,7 @@ extern "C" swan_status swan_decode_noalloc(const swan_cache_view* v, const void*
     p.n_sg = n_sg;
     p.N_g = N_g;
     p.total_groups = total;
-    p.range = range;
+    p.visit_cost = decode_visit_cost(G, false);
     p.H_kv = v->n_kv_heads;
     p.H_q = v->n_q_heads;
     p.blocks_per_page_log2 = __builtin_ctz((unsigned)(v->page_tokens / 32));
@@ -197,15 +193,8 @@ extern "C" swan_status swan_decode_noalloc(const swan_cache_view* v, const void*
   }
 
   CombineParams cp{};
-  cp.partials = partials;
-  cp.R_voT = v->R_vo_t;
   cp.out = static_cast<__half*>(out);
-  cp.H_kv = v->n_kv_heads;
   cp.H_q = v->n_q_heads;
-  cp.G = G;
-  cp.N_g = N_g > 0 ? N_g : 1;
-  cp.range = range;
-  cp.total_groups = total;
   if (launch_combine(cp, v->batch, s) != cudaSuccess) return err(SWAN_ERR_CUDA, "combine launch failed");
   return SWAN_OK;
 }

@@ -324,23 +324,22 @@ constexpr int64_t kMinGroupsPerCta = 8;
 // the merge, the rotate-back, and the pipeline start of every warp's short
 // run), in 32-token groups; measured on the ragged serving batch (a sweep of
 // 12 to 96 took its decode from 1.89 to 1.12 ms, level with equal rows).
-constexpr int64_t kSegmentCostGroups = 96;
-
 // First group of each decode CTA for ragged rows: contiguous ranges of equal
-// cost, a unit costing its groups plus kSegmentCostGroups for every CTA it
-// is processed by, so that CTAs covering many short rows take fewer groups.
-std::vector<int64_t> balanced_starts(const std::vector<int64_t>& row_groups, int H, int64_t max_ctas) {
+// cost, a unit costing its groups plus `visit` groups for every CTA it is
+// processed by, so that CTAs covering many short rows take fewer groups.
+std::vector<int64_t> balanced_starts(const std::vector<int64_t>& row_groups, int H, int64_t max_ctas,
+                                     int64_t visit) {
   int64_t total = 0;
   for (int64_t g : row_groups) total += g * H;
   const int64_t units = (int64_t)row_groups.size() * H;
   const int64_t ctas = std::max<int64_t>(1, std::min<int64_t>(max_ctas, total));
-  const double target = ((double)total + (double)kSegmentCostGroups * units) / (double)ctas;
+  const double target = ((double)total + (double)visit * units) / (double)ctas;
   std::vector<int64_t> starts{0};
   int64_t next = 1, goff = 0, u = 0;
   for (int64_t ng : row_groups)
     for (int h = 0; h < H; ++h, ++u) {
       // group goff + j costs base + j so far (this unit's overhead included)
-      const double base = (double)goff + (double)kSegmentCostGroups * (double)(u + 1);
+      const double base = (double)goff + (double)visit * (double)(u + 1);
       while (next < ctas && (double)next * target <= base + (double)(ng - 1)) {
         const int64_t j = std::max<int64_t>(0, (int64_t)std::ceil((double)next * target - base));
         const int64_t g = goff + j;
@@ -892,18 +891,17 @@ swan_status decode_rotated(swan_ctx* c, int layer, void* out) {
     }
     total = prefix * c->cfg.n_kv_heads;
     const std::vector<int64_t> starts = balanced_starts(
-        groups, c->cfg.n_kv_heads, std::min<int64_t>(c->decode_ctas, std::max<int64_t>(1, total / kMinGroupsPerCta)));
+        groups, c->cfg.n_kv_heads, std::min<int64_t>(c->decode_ctas, std::max<int64_t>(1, total / kMinGroupsPerCta)),
+        decode_visit_cost(G, true));
     ragged_grid = (int64_t)starts.size() - 1;
     if ((s = upload_rows(c, layer, rows, &starts)) != SWAN_OK) return s;
     rows_dev = rows_of(c, layer);
     starts_dev = cta_starts_of(c, layer);
   }
-  int64_t range = 1, grid = 0;
-  if (total > 0) {
-    const int64_t ctas = std::min<int64_t>(c->decode_ctas, std::max<int64_t>(1, total / kMinGroupsPerCta));
-    range = (total + ctas - 1) / ctas;
-    grid = starts_dev ? ragged_grid : (total + range - 1) / range;
-  }
+  int64_t grid = 0;
+  if (total > 0)
+    grid = starts_dev ? ragged_grid
+                      : std::min<int64_t>(c->decode_ctas, std::max<int64_t>(1, total / kMinGroupsPerCta));
   if (grid > 0) {
     DecodeParams p{};
     p.qprime = c->qprime;
@@ -917,7 +915,7 @@ swan_status decode_rotated(swan_ctx* c, int layer, void* out) {
     p.n_sg = n_sg;
     p.N_g = N_g;
     p.total_groups = total;
-    p.range = range;
+    p.visit_cost = decode_visit_cost(G, false);
     p.seq = rows_dev;
     p.cta_start = starts_dev;
     p.B = c->cfg.batch;
@@ -944,15 +942,8 @@ swan_status decode_rotated(swan_ctx* c, int layer, void* out) {
   // empty cache: the combine kernel writes zeros
 
   CombineParams cp{};
-  cp.partials = c->partials;
-  cp.R_voT = c->R_voT + (size_t)layer * c->cfg.n_kv_heads * kHeadDim * kHeadDim;
   cp.out = static_cast<__half*>(out);
-  cp.H_kv = c->cfg.n_kv_heads;
   cp.H_q = c->cfg.n_q_heads;
-  cp.G = G;
-  cp.N_g = N_g > 0 ? N_g : 1;
-  cp.range = range;
-  cp.total_groups = total;
   return launch(c, SWAN_KERNEL_COMBINE, "combine kernel",
                 [&] { return launch_combine(cp, c->cfg.batch, c->stream); });
 }

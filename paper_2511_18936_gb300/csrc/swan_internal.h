@@ -137,10 +137,11 @@ struct RotateQParams {
 };
 
 // Split decode: the flat list of 32-token groups of all units is cut into
-// equal contiguous ranges, one per CTA.  Group g of unit u is a sparse group
-// for g < n_sg (tokens 32g..32g+31 of the sparse history) and a buffer group
-// after that.  A CTA writes one partial (m, l, acc[d]) per (unit, head) it
-// touches, at pair index (cta + unit).
+// contiguous ranges of equal cost, one per CTA, a unit costing its groups
+// plus `visit_cost` groups for each CTA that works on it.  Group g of unit u
+// is a sparse group for g < n_sg (tokens 32g..32g+31 of the sparse history)
+// and a buffer group after that.  A CTA writes one partial (m, l, acc[d])
+// per (unit, head) it touches, at pair index (cta + unit).
 struct DecodeParams {
   const float* qprime;     // [B][H_q][d]
   CacheGeom geom;
@@ -149,9 +150,10 @@ struct DecodeParams {
   int cap, buf_start, n_b;
   int64_t sparse_len;
   int64_t n_sg, N_g;       // sparse groups per unit; groups per unit
-  int64_t total_groups, range;
+  int64_t total_groups;
+  int64_t visit_cost;      // groups a CTA's visit to a unit costs (uniform split)
   const SeqInfo* seq;      // per-row lengths (then the five scalars above are unused), or null
-  const int64_t* cta_start;  // [grid + 1] first group of each CTA (cost-balanced), or null: c * range
+  const int64_t* cta_start;  // [grid + 1] first group of each CTA (ragged rows), or null: computed
   int B;                   // rows
   int H_kv, H_q;
   int blocks_per_page_log2; // log2(P / 32)
@@ -167,12 +169,11 @@ struct DecodeParams {
   unsigned* status;
 };
 
+// A decode over an empty cache: the output is the rotate-back of an empty
+// attention, zero.
 struct CombineParams {
-  const float* partials;
-  const float* R_voT;      // this layer: [H_kv][d][d], transposed
   __half* out;             // [B][H_q][d]
-  int H_kv, H_q, G;
-  int64_t N_g, range, total_groups;
+  int H_q;
 };
 
 #ifdef __CUDACC__
@@ -296,6 +297,14 @@ cudaError_t launch_transpose_r(const float* src, float* dst, int64_t mats, cudaS
 cudaError_t launch_scatter_pages(const int2* pairs, int n, int32_t* table, cudaStream_t s);
 // Decode CTAs that fit on one SM together (for the grid size).
 int decode_ctas_per_sm(int G, int k_slots);
+// What a CTA's extra visit to a unit (prologue, merge, arrival) costs in
+// 32-token groups of streaming, for the cost-balanced split of the decode
+// kernels: equal-length rows (computed in the kernel) and ragged rows (the
+// host's table).  Set by measurement on the GB300.
+inline int64_t decode_visit_cost(int G, bool ragged) {
+  if (ragged) return 48;
+  return G == 1 ? 12 : 40;
+}
 // Record the detail string that swan_last_error() returns on this thread.
 void set_last_error(const char* msg);
 

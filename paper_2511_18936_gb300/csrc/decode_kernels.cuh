@@ -305,31 +305,43 @@ __device__ __forceinline__ int64_t cta_of(const DecodeParams& p, int64_t g) {
 // out = o_hat R_vo^T for the G query heads of unit (b, h); o_hat in shared
 // memory [G][128].  Thread t takes outputs 4q..4q+3 (q = t % 32) of every
 // head over rows j of slice t / 32 (S = NT / 32 slices of the 128 rows): its
-// float4 loads of R_vo^T are independent, so they are in flight together,
-// and each element serves all G heads.  The slices' partial sums meet in
+// float4 loads of R_vo^T are independent, eight in flight at a time, and
+// each element serves all G heads.  The slices' partial sums meet in
 // `part` (S * G * 128 floats of shared memory, which may overlap o_hat) and
 // are added in slice order.
 template <int G, int NT>
 __device__ __forceinline__ void rotate_back_out(const DecodeParams& p, int64_t b, int64_t h, const float* o_hat,
                                                 float* part) {
   constexpr int S = NT / 32;
+  constexpr int RS = (kHeadDim + S - 1) / S;  // rows per slice (the last may have fewer)
   static_assert(NT % 32 == 0 && S >= 1, "whole warps");
   const int q = threadIdx.x & 31, sl = threadIdx.x >> 5;
-  const int j0 = sl * kHeadDim / S, j1 = (sl + 1) * kHeadDim / S;
   const float4* RT4 = reinterpret_cast<const float4*>(p.R_voT + (size_t)h * kHeadDim * kHeadDim);
   float acc[G][4];
 #pragma unroll
   for (int gh = 0; gh < G; ++gh) acc[gh][0] = acc[gh][1] = acc[gh][2] = acc[gh][3] = 0.f;
-#pragma unroll 8
-  for (int j = j0; j < j1; ++j) {
-    const float4 r = __ldg(RT4 + j * (kHeadDim / 4) + q);
+  // eight rows in flight at a time
+#pragma unroll 1
+  for (int kb = 0; kb < RS; kb += 8) {
+    float4 r[8];
 #pragma unroll
-    for (int gh = 0; gh < G; ++gh) {
-      const float o = o_hat[gh * kHeadDim + j];
-      acc[gh][0] = fmaf(o, r.x, acc[gh][0]);
-      acc[gh][1] = fmaf(o, r.y, acc[gh][1]);
-      acc[gh][2] = fmaf(o, r.z, acc[gh][2]);
-      acc[gh][3] = fmaf(o, r.w, acc[gh][3]);
+    for (int k = 0; k < 8; ++k) {
+      const int j = sl * RS + kb + k;
+      r[k] = (kb + k < RS && j < kHeadDim) ? __ldg(RT4 + j * (kHeadDim / 4) + q) : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+      const int j = sl * RS + kb + k;
+      if (kb + k < RS && j < kHeadDim) {
+#pragma unroll
+        for (int gh = 0; gh < G; ++gh) {
+          const float o = o_hat[gh * kHeadDim + j];
+          acc[gh][0] = fmaf(o, r[k].x, acc[gh][0]);
+          acc[gh][1] = fmaf(o, r[k].y, acc[gh][1]);
+          acc[gh][2] = fmaf(o, r[k].z, acc[gh][2]);
+          acc[gh][3] = fmaf(o, r[k].w, acc[gh][3]);
+        }
+      }
     }
   }
   __syncthreads();  // o_hat is read; part may reuse it
@@ -511,6 +523,17 @@ __global__ void __launch_bounds__(decode_warps<MAXC>() * 32, decode_min_ctas<MAX
     }
     __syncthreads();
     if (u < u_last && threadIdx.x < kHeadDim) q_next = q_of(u + 1);
+    // into L2 ahead of use: R_vo^T of this head (64 KB, for the rotate-back)
+    // and the dense-buffer rows of this warp's run (read without a pipeline)
+    if (threadIdx.x == 0) prefetch_l2(p.R_voT + (size_t)h * kHeadDim * kHeadDim, kHeadDim * kHeadDim * 4);
+    for (int gi = max(t_lo, n_sg); gi < t_hi; ++gi) {
+      const int64_t i = (int64_t)(gi - n_sg) * 32 + lane;
+      if (i < uv.n_b) {
+        const size_t row = ((size_t)u * p.cap + (int)((uv.buf_start + i) % p.cap)) * kHeadDim;
+        prefetch_l2(p.ring_k + row, kHeadDim * 2);
+        prefetch_l2(p.ring_v + row, kHeadDim * 2);
+      }
+    }
 
     float m_w = -INFINITY;  // running max (log2 domain), uniform in the warp
     float l_sum = 0.f;      // this lane's sum of exp2(s - m_w)
@@ -1097,9 +1120,15 @@ __global__ void __launch_bounds__(mma_warps<MAXC>() * 32, 1) decode_mma_kernel(D
           const size_t row = ((size_t)u * p.cap + slot) * kHeadDim;
           const uint4* kr = reinterpret_cast<const uint4*>(p.ring_k + row);
           const uint4* vr = reinterpret_cast<const uint4*>(p.ring_v + row);
-#pragma unroll 2
-          for (int c = 0; c < 16; ++c) {
-            const uint4 w = __ldg(kr + c);
+#pragma unroll 1
+          for (int cb = 0; cb < 16; cb += 8) {
+          uint4 wk[8];
+#pragma unroll
+          for (int k = 0; k < 8; ++k) wk[k] = __ldg(kr + cb + k);
+#pragma unroll
+          for (int k = 0; k < 8; ++k) {
+            const int c = cb + k;
+            const uint4 w = wk[k];
             const float2 a = h2f(w.x), bb = h2f(w.y), cc = h2f(w.z), d = h2f(w.w);
             const float f[8] = {a.x, a.y, bb.x, bb.y, cc.x, cc.y, d.x, d.y};
 #pragma unroll
@@ -1119,10 +1148,17 @@ __global__ void __launch_bounds__(mma_warps<MAXC>() * 32, 1) decode_mma_kernel(D
               }
             }
           }
+          }
 #pragma unroll
           for (int j = 0; j < G; ++j) s[j] = s2[0][j] + s2[1][j];
-#pragma unroll 4
-          for (int c = 0; c < 16; ++c) sts_v4(vrow + c * 16, __ldg(vr + c));
+#pragma unroll 1
+          for (int cb = 0; cb < 16; cb += 8) {
+            uint4 wv[8];
+#pragma unroll
+            for (int k = 0; k < 8; ++k) wv[k] = __ldg(vr + cb + k);
+#pragma unroll
+            for (int k = 0; k < 8; ++k) sts_v4(vrow + (cb + k) * 16, wv[k]);
+          }
         }
       }
 

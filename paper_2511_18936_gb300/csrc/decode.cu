@@ -22,11 +22,13 @@ __global__ void __launch_bounds__(kHeadDim) combine_kernel(CombineParams p) {
 }
 
 // Dynamic shared memory of the one-head kernel: the warps' accumulators and
-// one more 16 KB region for the alignment gap, which holds q' (8 KB) unless
-// the allocation starts within 8 KB below a 16 KB boundary.
+// one more 16 KB region for the alignment gap, which holds an 8 KB q' unless
+// the allocation starts within 8 KB below a 16 KB boundary; a 16 KB q' goes
+// after the accumulators.
 size_t one_head_smem(int maxc) {
   const int nw = maxc <= 8 ? decode_warps<8>() : decode_warps<16>();
-  return (size_t)(nw + 1) * kRegionBytes;
+  const int q_regions = (maxc <= 8 ? decode_q_shift<8>() : decode_q_shift<16>()) == 7 ? 1 : 0;
+  return (size_t)(nw + 1 + q_regions) * kRegionBytes;
 }
 
 template <typename K>

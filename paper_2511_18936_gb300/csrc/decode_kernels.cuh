@@ -129,6 +129,12 @@ __device__ __forceinline__ float2 lds2(uint32_t a) {
   return v;
 }
 
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_group 0;" ::: "memory"); }
+
 // Ask the memory system to bring `bytes` (a multiple of 16, 16-byte aligned)
 // into L2 ahead of the loads that will read them.
 __device__ __forceinline__ void prefetch_l2(const void* ptr, uint32_t bytes) {
@@ -154,15 +160,14 @@ __device__ __forceinline__ uint32_t addr_of(uint32_t w, uint32_t base) {
   else return ((w >> -sh) & mask) | base;
 }
 
-// q' of the one-head kernel: 16 copies of each coordinate ([128][16] fp32,
-// 64-byte rows, 8 KB aligned).
-constexpr int kQRep = 16;
-constexpr int kQRowShift = 6;
-constexpr uint32_t kQBytes = kHeadDim * kQRep * sizeof(float);  // 8 KB
+// q' of the one-head kernel: 2^QS / 4 copies of each coordinate, rows of
+// 2^QS bytes, aligned to their 128-row size: 16 copies (8 KB) where two CTAs
+// share an SM, 32 (16 KB, conflict-free) where one CTA has the SM.
 
 // Score contribution of one chunk into four partial sums.
+template <int QS>
 __device__ __forceinline__ void score_chunk(uint32_t qb, const float (&f)[8], uint2 ix, float (&s)[4]) {
-  constexpr int Q = kQRowShift;
+  constexpr int Q = QS;
   const float q0 = lds(addr_of<0, Q>(ix.x, qb)), q1 = lds(addr_of<1, Q>(ix.x, qb));
   const float q2 = lds(addr_of<2, Q>(ix.x, qb)), q3 = lds(addr_of<3, Q>(ix.x, qb));
   const float q4 = lds(addr_of<0, Q>(ix.y, qb)), q5 = lds(addr_of<1, Q>(ix.y, qb));
@@ -433,14 +438,17 @@ __host__ __device__ constexpr int decode_warps() { return MAXC <= 8 ? 6 : 8; }
 // other's streaming)
 template <int MAXC>
 __host__ __device__ constexpr int decode_min_ctas() { return MAXC <= 8 ? 2 : 1; }
+// q' row shift of the one-head kernel (16 or 32 copies per coordinate)
+template <int MAXC>
+__host__ __device__ constexpr int decode_q_shift() { return MAXC <= 8 ? 6 : 7; }
 
 // Split decode kernel, one query head per kv head.
 //   The flat list of 32-token blocks of all units is cut into equal ranges,
 //   one per CTA.  Shared memory (dynamic, laid out from its actual start):
 //   one lane-private rotated-space accumulator per warp ([128][32] fp32,
-//   16 KB-aligned regions) and q' with 16 copies per coordinate ([128][16]
-//   fp32, 8 KB aligned), in the gap before the first aligned region when it
-//   fits there, else after the accumulators.
+//   16 KB-aligned regions) and q' with 16 or 32 copies per coordinate
+//   ([128][16 | 32] fp32, aligned to its size), in the gap before the first
+//   aligned region when it fits there, else after the accumulators.
 //   Lane = token; each warp walks a contiguous run of blocks.  While block g
 //   is processed, the key records of block g+1 are in flight to registers
 //   and block g+2 is being prefetched into L2.
@@ -449,9 +457,12 @@ __global__ void __launch_bounds__(decode_warps<MAXC>() * 32, decode_min_ctas<MAX
     decode_kernel(DecodeParams p) {
   constexpr int NW = decode_warps<MAXC>();
   constexpr int NT = NW * 32;
+  constexpr int QS = decode_q_shift<MAXC>();
+  constexpr int QREP = (1 << QS) / 4;                       // copies per coordinate
+  constexpr uint32_t kQBytes = kHeadDim << QS;              // 8 or 16 KB
   extern __shared__ __align__(16) unsigned char smem_dyn[];
   __shared__ float red_m[NW], red_l[NW];
-  __shared__ float q_stage[kHeadDim];  // q' of the next unit, before replication
+  __shared__ __align__(16) float q_stage[kHeadDim];  // q' of the next unit, before replication
   pdl_trigger();
 
   const uint32_t raw = (uint32_t)__cvta_generic_to_shared(smem_dyn);
@@ -470,7 +481,7 @@ __global__ void __launch_bounds__(decode_warps<MAXC>() * 32, decode_min_ctas<MAX
   float* qrep = reinterpret_cast<float*>(smem_dyn + (qbase - raw)); // [128][16]
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const uint32_t qb = qbase + ((lane & (kQRep - 1)) << 2);
+  const uint32_t qb = qbase + ((lane & (QREP - 1)) << 2);
   const uint32_t ab = base + warp * kRegionBytes + (lane << 2);
 
   const CacheGeom& g = p.geom;
@@ -489,13 +500,17 @@ __global__ void __launch_bounds__(decode_warps<MAXC>() * 32, decode_min_ctas<MAX
   pdl_wait();
   if (g_begin >= g_end) return;
   const int64_t u_first = unit_of(p, g_begin), u_last = unit_of(p, g_end - 1);
-  // q' of the unit the next segment starts: one coalesced load, issued a
-  // segment ahead (the first one here)
-  auto q_of = [&](int64_t un) {
-    const int64_t bn = un / p.H_kv, hn = un - bn * p.H_kv;
-    return __ldg(p.qprime + (bn * p.H_q + hn) * kHeadDim + threadIdx.x);
+  // q' of the unit the next segment starts, copied into q_stage by
+  // cp.async a segment ahead (the first one here): no registers held
+  const uint32_t q_stage_s = (uint32_t)__cvta_generic_to_shared(q_stage);
+  auto stage_q = [&](int64_t un) {
+    if (threadIdx.x < kHeadDim / 4) {
+      const int64_t bn = un / p.H_kv, hn = un - bn * p.H_kv;
+      cp_async16(q_stage_s + threadIdx.x * 16, p.qprime + (bn * p.H_q + hn) * kHeadDim + threadIdx.x * 4);
+    }
+    cp_async_commit();
   };
-  float q_next = threadIdx.x < kHeadDim ? q_of(u_first) : 0.f;
+  stage_q(u_first);
 
   for (int64_t u = u_first; u <= u_last; ++u) {
     const UnitView uv = unit_view(p, u);
@@ -509,11 +524,11 @@ __global__ void __launch_bounds__(decode_warps<MAXC>() * 32, decode_min_ctas<MAX
     const int sp_hi = min(t_hi, n_sg);  // sparse groups of the run: [t_lo, sp_hi)
     const int32_t* ptab = g.page_table + u * g.pages_per_unit;
 
-    if (threadIdx.x < kHeadDim) q_stage[threadIdx.x] = q_next;
-    __syncthreads();  // the previous segment is done with shared memory
-    // q' copies (float4 f of the [128][16] layout holds row f / 4)
-    for (int f = threadIdx.x; f < kHeadDim * kQRep / 4; f += NT) {
-      const float v = q_stage[f >> 2];
+    cp_async_wait_all();
+    __syncthreads();  // the previous segment is done with shared memory; q_stage has landed
+    // q' copies (float4 f of the [128][QREP] layout holds row f / (QREP / 4))
+    for (int f = threadIdx.x; f < kHeadDim * QREP / 4; f += NT) {
+      const float v = q_stage[f / (QREP / 4)];
       reinterpret_cast<float4*>(qrep)[f] = make_float4(v, v, v, v);
     }
     {
@@ -522,7 +537,7 @@ __global__ void __launch_bounds__(decode_warps<MAXC>() * 32, decode_min_ctas<MAX
       for (int f = lane; f < kHeadDim * 8; f += 32) az[f] = make_float4(0.f, 0.f, 0.f, 0.f);
     }
     __syncthreads();
-    if (u < u_last && threadIdx.x < kHeadDim) q_next = q_of(u + 1);
+    if (u < u_last) stage_q(u + 1);
     // into L2 ahead of use: R_vo^T of this head (64 KB, for the rotate-back)
     // and the dense-buffer rows of this warp's run (read without a pipeline)
     if (threadIdx.x == 0) prefetch_l2(p.R_voT + (size_t)h * kHeadDim * kHeadDim, kHeadDim * kHeadDim * 4);
@@ -605,7 +620,7 @@ __global__ void __launch_bounds__(decode_warps<MAXC>() * 32, decode_min_ctas<MAX
               keep_first(f, 0);
               ix = make_uint2(0, 0);
             }
-            score_chunk(qb, f, ix, s);
+            score_chunk<QS>(qb, f, ix, s);
           }
         s2 = valid ? ((s[0] + s[1]) + (s[2] + s[3])) * p.scale_log2 : -INFINITY;
 
@@ -662,7 +677,7 @@ __global__ void __launch_bounds__(decode_warps<MAXC>() * 32, decode_min_ctas<MAX
         for (int c = 0; c < 16; ++c) {
           const uint4 w = __ldg(kr + c);
           const float2 a = h2f(w.x), bb = h2f(w.y), cc = h2f(w.z), d = h2f(w.w);
-          constexpr uint32_t QR = 1u << kQRowShift;
+          constexpr uint32_t QR = 1u << QS;
           const uint32_t q = qb + c * 8 * QR;
           s[0] = fmaf(lds(q + 0 * QR), a.x, s[0]);
           s[1] = fmaf(lds(q + 1 * QR), a.y, s[1]);
@@ -802,11 +817,6 @@ __host__ __device__ constexpr size_t mma_smem() {
   return (size_t)kQrepBytes + (size_t)mma_warps<MAXC>() * mma_warp_bytes<MAXC>() + 16;
 }
 
-__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src) {
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
-}
-__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
-__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_group 0;" ::: "memory"); }
 __device__ __forceinline__ uint4 lds_v4u(uint32_t a) {
   uint4 v;
   asm volatile("ld.shared.v4.u32 {%0,%1,%2,%3}, [%4];" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(a)
@@ -915,8 +925,7 @@ __global__ void __launch_bounds__(mma_warps<MAXC>() * 32, 1) decode_mma_kernel(D
   __shared__ float red_m[NW * G], red_l[NW * G];
   __shared__ float flag[1];
   __shared__ __align__(16) float q_stage[G * kHeadDim];  // q' of the next unit's G heads
-  static_assert(G * kHeadDim % NT == 0, "whole q' loads per thread");
-  constexpr int QL = G * kHeadDim / NT;  // q' floats each thread loads
+  static_assert(G * kHeadDim / 4 <= NT, "one 16-byte piece of q' per thread");
   pdl_trigger();
 
   const uint32_t raw = (uint32_t)__cvta_generic_to_shared(smem_raw);
@@ -948,15 +957,16 @@ __global__ void __launch_bounds__(mma_warps<MAXC>() * 32, 1) decode_mma_kernel(D
   if (g_begin >= g_end) return;
   const int64_t u_first = unit_of(p, g_begin), u_last = unit_of(p, g_end - 1);
   // q' of the G heads of the unit the next segment starts (G * 128
-  // consecutive floats): coalesced loads issued a segment ahead
-  float q_next[QL];
-  auto load_q = [&](int64_t un) {
-    const int64_t bn = un / p.H_kv, hn = un - bn * p.H_kv;
-    const float* src = p.qprime + (bn * p.H_q + hn * G) * kHeadDim;
-#pragma unroll
-    for (int k = 0; k < QL; ++k) q_next[k] = __ldg(src + threadIdx.x + k * NT);
+  // consecutive floats), copied into q_stage by cp.async a segment ahead
+  const uint32_t q_stage_s = (uint32_t)__cvta_generic_to_shared(q_stage);
+  auto stage_q = [&](int64_t un) {
+    if (threadIdx.x < G * kHeadDim / 4) {
+      const int64_t bn = un / p.H_kv, hn = un - bn * p.H_kv;
+      cp_async16(q_stage_s + threadIdx.x * 16, p.qprime + (bn * p.H_q + hn * G) * kHeadDim + threadIdx.x * 4);
+    }
+    cp_async_commit();
   };
-  load_q(u_first);
+  stage_q(u_first);
 
   // the tiles start zeroed; every use restores the zeros it disturbed
   for (int c = 0; c < 16; ++c) sts_v4(vrow + c * 16, make_uint4(0, 0, 0, 0));
@@ -972,9 +982,8 @@ __global__ void __launch_bounds__(mma_warps<MAXC>() * 32, 1) decode_mma_kernel(D
     const int sp_hi = min(t_hi, n_sg);
     const int32_t* ptab = g.page_table + u * g.pages_per_unit;
 
-#pragma unroll
-    for (int k = 0; k < QL; ++k) q_stage[threadIdx.x + k * NT] = q_next[k];
-    __syncthreads();  // the previous segment is done with q'; q_stage is set
+    cp_async_wait_all();
+    __syncthreads();  // the previous segment is done with q'; q_stage has landed
     // 32 floats per coordinate c: 32 / G copies of its G heads (float4 f
     // holds coordinate f / 8, heads 0..3 or 0, 1, 0, 1)
     for (int f = threadIdx.x; f < kHeadDim * 8; f += NT) {
@@ -987,7 +996,7 @@ __global__ void __launch_bounds__(mma_warps<MAXC>() * 32, 1) decode_mma_kernel(D
       reinterpret_cast<float4*>(qrep)[f] = v;
     }
     __syncthreads();
-    if (u < u_last) load_q(u + 1);
+    if (u < u_last) stage_q(u + 1);
 
     float m[G], l[G];
 #pragma unroll

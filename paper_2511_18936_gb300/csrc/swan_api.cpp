@@ -78,7 +78,8 @@ struct swan_ctx {
   cudaStream_t stream = nullptr;
   int device = 0;
   int num_sms = 0;
-  int decode_ctas = 0;  // max decode CTAs resident at once
+  int decode_ctas = 0;  // max decode CTAs resident at once (either kernel variant)
+  int decode_ctas_small = 0, decode_ctas_big = 0;  // for <= 64 and > 64 entries read
 
   float* R_qk = nullptr;
   float* R_vo = nullptr;   // == R_qk when the caller passed NULL
@@ -493,13 +494,18 @@ swan_status swan_init(swan_ctx** out, const swan_config* cfg, const float* R_qk,
   c->layers.assign(C.num_layers, LayerState{});
   for (LayerState& L : c->layers) L.seq.assign(C.batch, SeqState{});
 
-  const int per_sm = decode_ctas_per_sm(G, std::max(c->k_slots, c->k_slots_v));
-  if (per_sm < 1) {
+  // resident decode CTAs of the kernel variant each runtime keep count uses
+  const bool big_slots = std::max(c->k_slots, c->k_slots_v) > 64;
+  const int per_sm_small = decode_ctas_per_sm(G, 64);
+  const int per_sm_big = big_slots ? decode_ctas_per_sm(G, 128) : per_sm_small;
+  if (per_sm_small < 1 || per_sm_big < 1) {
     delete c;
     return fail(SWAN_ERR_CUDA, "decode kernel does not fit on an SM (%s)",
                 cudaGetErrorString(cudaGetLastError()));
   }
-  c->decode_ctas = per_sm * sms;
+  c->decode_ctas_small = per_sm_small * sms;
+  c->decode_ctas_big = per_sm_big * sms;
+  c->decode_ctas = std::max(c->decode_ctas_small, c->decode_ctas_big);
 
   const size_t rmat = (size_t)C.num_layers * C.n_kv_heads * kHeadDim * kHeadDim;
   const size_t ring_elems = (size_t)C.num_layers * ring_elems_per_layer(c);
@@ -869,6 +875,10 @@ swan_status decode_rotated(swan_ctx* c, int layer, void* out) {
   // offsets in a per-row table.
   const bool same = L.uniform();
   const SeqState& q0 = L.seq[0];
+  // entries read per vector, rounded up to 8: selects the kernel variant
+  // and so how many of its CTAs fit at once
+  const int k_read = (std::max(c->k_active, c->k_active_v) + 7) / 8 * 8;
+  const int64_t max_ctas = k_read > 64 ? c->decode_ctas_big : c->decode_ctas_small;
   const int64_t n_sg = (q0.sparse_len + 31) / 32;
   const int64_t n_bg = (q0.buf_count + 31) / 32;
   const int64_t N_g = n_sg + n_bg;
@@ -891,7 +901,7 @@ swan_status decode_rotated(swan_ctx* c, int layer, void* out) {
     }
     total = prefix * c->cfg.n_kv_heads;
     const std::vector<int64_t> starts = balanced_starts(
-        groups, c->cfg.n_kv_heads, std::min<int64_t>(c->decode_ctas, std::max<int64_t>(1, total / kMinGroupsPerCta)),
+        groups, c->cfg.n_kv_heads, std::min<int64_t>(max_ctas, std::max<int64_t>(1, total / kMinGroupsPerCta)),
         decode_visit_cost(G, true));
     ragged_grid = (int64_t)starts.size() - 1;
     if ((s = upload_rows(c, layer, rows, &starts)) != SWAN_OK) return s;
@@ -901,7 +911,7 @@ swan_status decode_rotated(swan_ctx* c, int layer, void* out) {
   int64_t grid = 0;
   if (total > 0)
     grid = starts_dev ? ragged_grid
-                      : std::min<int64_t>(c->decode_ctas, std::max<int64_t>(1, total / kMinGroupsPerCta));
+                      : std::min<int64_t>(max_ctas, std::max<int64_t>(1, total / kMinGroupsPerCta));
   if (grid > 0) {
     DecodeParams p{};
     p.qprime = c->qprime;
@@ -934,10 +944,7 @@ swan_status decode_rotated(swan_ctx* c, int layer, void* out) {
     p.status = c->status;
     // the split combine and the rotate-back run inside the decode kernel
     return launch(c, SWAN_KERNEL_DECODE, "decode kernel",
-                  [&] {
-                    const int k_read = (std::max(c->k_active, c->k_active_v) + 7) / 8 * 8;
-                    return launch_decode(p, G, k_read, (int)grid, c->stream);
-                  });
+                  [&] { return launch_decode(p, G, k_read, (int)grid, c->stream); });
   }
   // empty cache: the combine kernel writes zeros
 

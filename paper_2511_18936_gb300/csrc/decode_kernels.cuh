@@ -443,8 +443,9 @@ template <int MAXC>
 __host__ __device__ constexpr int decode_q_shift() { return MAXC <= 8 ? 6 : 7; }
 
 // Split decode kernel, one query head per kv head.
-//   The flat list of 32-token blocks of all units is cut into equal ranges,
-//   one per CTA.  Shared memory (dynamic, laid out from its actual start):
+//   The flat list of 32-token blocks of all units is cut into ranges of
+//   equal cost (cta_begin), one per CTA.  Shared memory (dynamic, laid out
+//   from its actual start):
 //   one lane-private rotated-space accumulator per warp ([128][32] fp32,
 //   16 KB-aligned regions) and q' with 16 or 32 copies per coordinate
 //   ([128][16 | 32] fp32, aligned to its size), in the gap before the first
@@ -802,8 +803,9 @@ template <int MAXC>
 __host__ __device__ constexpr uint32_t mma_warp_bytes() {
   return kVTileBytes + kPTileBytes + (uint32_t)MAXC * 768;
 }
-// 8 warps: the registers (~240 a thread) allow no more without spills, and a
-// sweep on the GB300 measured 8 < 10 < 12 warps in time (0.480, 0.491,
+// 8 warps: the kernel needs ~230-255 registers a thread; registers are
+// allocated per scheduler, so 9 to 12 warps all get 168 a thread and spill
+// (a sweep on the GB300 measured 8 < 10 < 12 warps in time: 0.480, 0.491,
 // 0.565 ms on the GQA 131k layer).
 template <int MAXC>
 __host__ __device__ constexpr int mma_warps() { return 8; }

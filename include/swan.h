@@ -370,6 +370,24 @@ swan_status swan_decode_noalloc(const swan_cache_view* view, const void* q, void
 /* Number of kernels this context has launched since swan_init. */
 int64_t swan_launch_count(const swan_ctx* ctx);
 
+/*
+ * Test hooks.  Every device buffer of a context sits between two 256-byte
+ * guard regions filled with 0xA5 at swan_init; swan_debug_check_guards
+ * synchronises the stream and returns SWAN_ERR_DEVICE_CHECK (naming the
+ * buffer) if a kernel wrote into one, else SWAN_OK (STATE, CUDA as usual).
+ *
+ * swan_debug_fail_after makes the library fail on the host, without calling
+ * CUDA, at the (n+1)-th next device allocation (SWAN_FAULT_ALLOC: the call
+ * returns SWAN_ERR_NOMEM, and swan_init frees what it had allocated) or
+ * kernel launch (SWAN_FAULT_LAUNCH: nothing is launched, the call returns
+ * SWAN_ERR_CUDA and the context is poisoned), counted over all contexts of
+ * the process; it fires once.  n = -1 turns it off.  Not for concurrent
+ * use.  Errors: INVALID_ARG (kind, n < -1).
+ */
+enum { SWAN_FAULT_ALLOC = 1, SWAN_FAULT_LAUNCH = 2 };
+swan_status swan_debug_fail_after(int kind, int64_t n);
+swan_status swan_debug_check_guards(swan_ctx* ctx);
+
 /* Static string for a status code. */
 const char* swan_status_string(swan_status s);
 

@@ -100,6 +100,14 @@ struct swan_ctx {
   int2* pt_pairs = nullptr;    // paged: (entry, page) updates of one call
   int64_t device_bytes = 0;
 
+  // every device allocation, with guard regions before and after it
+  struct DevBuf {
+    void* base;
+    size_t bytes;  // without the guards
+    const char* what;
+  };
+  std::vector<DevBuf> bufs;
+
   std::vector<LayerState> layers;
   bool poisoned = false;
   int64_t launches = 0;
@@ -116,22 +124,26 @@ constexpr int kMaxBufferCap = 4096;
 constexpr int64_t kSmallAppendVectors = 256;  // batch * T per kv head
 constexpr size_t kMaxEventPairs = 4096;
 
+// Guard regions: kGuardBytes of kGuardByte before and after every device
+// buffer (256 bytes keep the buffers' alignment); swan_debug_check_guards
+// reports any that a kernel overwrote.
+constexpr size_t kGuardBytes = 256;
+constexpr unsigned char kGuardByte = 0xA5;
+
+// Test hooks: the n-th next device allocation / kernel launch fails (n = 0:
+// the next one); -1 = off.  Process-wide.
+std::atomic<int64_t> g_fail_alloc{-1};
+std::atomic<int64_t> g_fail_launch{-1};
+bool injected(std::atomic<int64_t>& n) {
+  int64_t v = n.load();
+  while (v >= 0)
+    if (n.compare_exchange_weak(v, v - 1)) return v == 0;
+  return false;
+}
+
 void free_all(swan_ctx* c) {
-  if (c->R_vo && c->R_vo != c->R_qk) cudaFree(c->R_vo);
-  cudaFree(c->R_qk);
-  cudaFree(c->R_voT);
-  cudaFree(c->R_hi);
-  cudaFree(c->R_lo);
-  cudaFree(c->pool);
-  cudaFree(c->page_table);
-  cudaFree(c->ring_k);
-  cudaFree(c->ring_v);
-  cudaFree(c->qprime);
-  cudaFree(c->partials);
-  cudaFree(c->counters);
-  cudaFree(c->status);
-  cudaFree(c->seq_dev);
-  cudaFree(c->pt_pairs);
+  for (const auto& b : c->bufs) cudaFree(b.base);
+  c->bufs.clear();
   for (auto& e : c->ev_free) {
     cudaEventDestroy(e.start);
     cudaEventDestroy(e.stop);
@@ -144,14 +156,18 @@ void free_all(swan_ctx* c) {
 
 swan_status dev_alloc(swan_ctx* c, void** p, size_t bytes, const char* what) {
   if (bytes == 0) bytes = 256;
-  cudaError_t e = cudaMalloc(p, bytes);
+  *p = nullptr;
+  if (injected(g_fail_alloc)) return fail(SWAN_ERR_NOMEM, "allocation for %s failed (injected)", what);
+  void* base = nullptr;
+  cudaError_t e = cudaMalloc(&base, bytes + 2 * kGuardBytes);
   if (e != cudaSuccess) {
     cudaGetLastError();
-    *p = nullptr;
     return fail(SWAN_ERR_NOMEM, "cudaMalloc of %zu bytes for %s failed: %s", bytes, what,
                 cudaGetErrorString(e));
   }
-  c->device_bytes += (int64_t)bytes;
+  c->bufs.push_back({base, bytes, what});
+  *p = static_cast<char*>(base) + kGuardBytes;
+  c->device_bytes += (int64_t)(bytes + 2 * kGuardBytes);
   return SWAN_OK;
 }
 
@@ -181,6 +197,7 @@ swan_status drain_events(swan_ctx* c) {
 // with an event pair on the context's stream.
 template <typename F>
 swan_status launch(swan_ctx* c, int kind, const char* name, F&& f) {
+  if (injected(g_fail_launch)) return cuda_fail(c, cudaErrorLaunchFailure, name);  // nothing launched
   EventPair ev{};
   if (c->timing) {
     if (c->ev_used.size() >= kMaxEventPairs) {
@@ -568,6 +585,11 @@ swan_status swan_init(swan_ctx** out, const swan_config* cfg, const float* R_qk,
   if (e == cudaSuccess) e = cudaMemsetAsync(c->ring_v, 0, ring_elems * sizeof(__half), st);
   if (e == cudaSuccess) e = cudaMemsetAsync(c->counters, 0, (size_t)c->units * sizeof(int), st);
   if (e == cudaSuccess) e = cudaMemsetAsync(c->status, 0, sizeof(unsigned), st);
+  for (const auto& b : c->bufs) {
+    if (e == cudaSuccess) e = cudaMemsetAsync(b.base, kGuardByte, kGuardBytes, st);
+    if (e == cudaSuccess)
+      e = cudaMemsetAsync(static_cast<char*>(b.base) + kGuardBytes + b.bytes, kGuardByte, kGuardBytes, st);
+  }
   if (e == cudaSuccess) e = cudaStreamSynchronize(st);  // pt is a pageable host vector
   if (e != cudaSuccess) {
     swan_status r = fail(SWAN_ERR_CUDA, "initialising the cache: %s", cudaGetErrorString(e));
@@ -1173,5 +1195,32 @@ swan_status swan_timing_read(swan_ctx* c, swan_timing* out) {
 }
 
 int64_t swan_launch_count(const swan_ctx* c) { return c ? c->launches : 0; }
+
+swan_status swan_debug_fail_after(int kind, int64_t n) {
+  if (n < -1) return fail(SWAN_ERR_INVALID_ARG, "n = %lld < -1", (long long)n);
+  if (kind == SWAN_FAULT_ALLOC) g_fail_alloc.store(n);
+  else if (kind == SWAN_FAULT_LAUNCH) g_fail_launch.store(n);
+  else return fail(SWAN_ERR_INVALID_ARG, "unknown fault kind %d", kind);
+  return SWAN_OK;
+}
+
+swan_status swan_debug_check_guards(swan_ctx* c) {
+  swan_status s = usable(c);
+  if (s != SWAN_OK) return s;
+  cudaError_t e = cudaStreamSynchronize(c->stream);
+  if (e != cudaSuccess) return cuda_fail(c, e, "cudaStreamSynchronize");
+  std::vector<unsigned char> g(kGuardBytes);
+  for (const auto& b : c->bufs)
+    for (int side = 0; side < 2; ++side) {
+      const char* at = static_cast<const char*>(b.base) + (side ? kGuardBytes + b.bytes : 0);
+      e = cudaMemcpy(g.data(), at, kGuardBytes, cudaMemcpyDeviceToHost);
+      if (e != cudaSuccess) return cuda_fail(c, e, "cudaMemcpy");
+      for (size_t i = 0; i < kGuardBytes; ++i)
+        if (g[i] != kGuardByte)
+          return fail(SWAN_ERR_DEVICE_CHECK, "the guard region %s %s was overwritten (byte %zu)",
+                      side ? "after" : "before", b.what, i);
+    }
+  return SWAN_OK;
+}
 
 }  // extern "C"

@@ -21,6 +21,7 @@ EXPORT_BUFFER_K, EXPORT_BUFFER_V, EXPORT_SPARSE_K, EXPORT_SPARSE_V = 1, 2, 3, 4
 VALUE_FORMATS = {"fp16": 0, "fp8_e4m3": 1}
 KERNEL_ROTATE_Q, KERNEL_DECODE, KERNEL_COMBINE, KERNEL_APPEND, KERNEL_PRUNE = range(5)
 KERNEL_KINDS = 8
+FAULT_ALLOC, FAULT_LAUNCH = 1, 2
 KERNEL_NAMES = {KERNEL_ROTATE_Q: "rotate_q", KERNEL_DECODE: "decode", KERNEL_COMBINE: "combine",
                 KERNEL_APPEND: "append", KERNEL_PRUNE: "prune_ring"}
 
@@ -31,7 +32,8 @@ EXPORTED = ["swan_init", "swan_destroy", "swan_set_k", "swan_append", "swan_flus
             "swan_status_string", "swan_last_error", "swan_decode_noalloc", "swan_set_kv",
             "swan_gram_workspace_bytes", "swan_gram", "swan_basis_eig", "swan_energy",
             "swan_basis_check", "swan_append_varlen", "swan_reset_sequence", "swan_query_lengths",
-            "swan_debug_export_seq", "swan_append_decode"]
+            "swan_debug_export_seq", "swan_append_decode", "swan_debug_fail_after",
+            "swan_debug_check_guards"]
 
 
 class SwanConfig(ctypes.Structure):
@@ -122,6 +124,8 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "swan_basis_eig": (i, [vp, i, vp, vp, vp, vp]),
         "swan_energy": (i, [ctypes.POINTER(SwanVectors), vp, vp, i, vp]),
         "swan_basis_check": (i, [vp, vp]),
+        "swan_debug_fail_after": (i, [i, i64]),
+        "swan_debug_check_guards": (i, [vp]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(lib, name)
@@ -259,6 +263,10 @@ class Context:
     def check(self):
         _check(self._lib.swan_check(self._h), "swan_check")
 
+    def check_guards(self):
+        """Raise if a kernel wrote into the guard regions around any device buffer."""
+        _check(self._lib.swan_debug_check_guards(self._h), "swan_debug_check_guards")
+
     def export_buffer(self, layer: int, which: str) -> np.ndarray:
         info = self.query(layer)
         shape = (self.batch, self.n_kv_heads, info.buffer_len, self.head_dim)
@@ -313,6 +321,12 @@ class Context:
 
     def launch_count(self) -> int:
         return int(self._lib.swan_launch_count(self._h))
+
+
+def debug_fail_after(kind: int, n: int):
+    """Test hook: the (n+1)-th next device allocation (FAULT_ALLOC) or kernel
+    launch (FAULT_LAUNCH) fails on the host; n = -1 turns it off."""
+    _check(load_library().swan_debug_fail_after(int(kind), int(n)), "swan_debug_fail_after")
 
 
 def decode_noalloc(view: CacheView, q, out, stream=None):

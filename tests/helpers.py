@@ -56,6 +56,7 @@ def run_ops(ops, R, Rv, *, B, H_kv, G, k_store, cap, max_seq=None, page_tokens=0
             assert info.sparse_len == ref.sparse_len, (info.sparse_len, ref.sparse_len)
             assert info.buffer_len == ref.buffer_len, (info.buffer_len, ref.buffer_len)
     ctx.check()
+    ctx.check_guards()
     return ctx, ref, outs
 
 

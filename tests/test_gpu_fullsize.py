@@ -61,6 +61,7 @@ def _layer_case(B, H_q, H_kv, L_s, n_b, k_store, k_actives, samples, seed=0, ste
     info = ctx.query(0)
     assert info.sparse_len == L_s + steps and info.buffer_len == n_b
     ctx.check()
+    ctx.check_guards()
     ctx.close()
     return worst
 
@@ -162,4 +163,5 @@ def test_stack_32_layers_prefix_and_flush_schedule_sampled():
         info = ctx.query(l)
         assert info.sparse_len == pre + steps and info.buffer_len == 0
     ctx.check()
+    ctx.check_guards()
     ctx.close()

@@ -343,6 +343,7 @@ def test_capacity_error_leaves_state_unchanged():
     with pytest.raises(swan.SwanError):
         ctx.decode(1, torch.zeros(1, 1, D, dtype=torch.float16, device="cuda"))
     ctx.check()
+    ctx.check_guards()
     ctx.close()
 
 
@@ -367,6 +368,7 @@ def test_multi_layer_state_is_independent():
         got = ctx.decode(l, torch.from_numpy(q).cuda()).float().cpu().numpy()
         assert np.abs(got - ref.decode(q)).max() <= TOL_OUT
     ctx.check()
+    ctx.check_guards()
     ctx.close()
 
 

@@ -69,6 +69,7 @@ def run_ragged(ops, R, Rv, *, B, H_kv, G, k_store, cap, max_seq, page_tokens=0, 
         sp, bf = ctx.lengths(0)
         assert sp == ref.sparse_lens and bf == ref.buffer_lens, (op[0], sp, ref.sparse_lens, bf, ref.buffer_lens)
     ctx.check()
+    ctx.check_guards()
     return ctx, ref, worst
 
 
@@ -196,6 +197,7 @@ def test_page_pool_shared_by_rows():
     assert np.abs(got - ref.decode(q)).max() <= TOL_OUT
     assert ctx.lengths(0) == (ref.sparse_lens, ref.buffer_lens)
     ctx.check()
+    ctx.check_guards()
     ctx.close()
 
 
@@ -221,6 +223,7 @@ def test_bulk_append_tiles_and_alignment():
     assert e.value.status == swan.ERR_INVALID_ARG and "aligned" in str(e.value)
     assert ctx.lengths(0) == before
     ctx.check()
+    ctx.check_guards()
     ctx.close()
 
 

@@ -86,6 +86,8 @@ def test_append_decode_equals_append_then_decode(G, fmt, ragged, cap):
             assert np.array_equal(fi, si) and np.array_equal(fv, sv)
     fused.check()
     split.check()
+    fused.check_guards()
+    split.check_guards()
     fused.close()
     split.close()
 

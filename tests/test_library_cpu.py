@@ -98,6 +98,25 @@ def test_null_arguments(lib):
     assert lib.swan_check(None) == swan.ERR_INVALID_ARG
     assert lib.swan_destroy(None) == swan.OK
     assert lib.swan_launch_count(None) == 0
+    assert lib.swan_append_decode(None, 0, None, None, 1, None, None, None) == swan.ERR_INVALID_ARG
+    assert lib.swan_debug_check_guards(None) == swan.ERR_INVALID_ARG
+
+
+def test_fault_hook_arguments(lib):
+    """The test hook validates its arguments; arming and disarming it needs no GPU."""
+    assert lib.swan_debug_fail_after(0, 0) == swan.ERR_INVALID_ARG
+    assert lib.swan_debug_fail_after(3, 0) == swan.ERR_INVALID_ARG
+    assert lib.swan_debug_fail_after(swan.FAULT_ALLOC, -2) == swan.ERR_INVALID_ARG
+    for kind in (swan.FAULT_ALLOC, swan.FAULT_LAUNCH):
+        assert lib.swan_debug_fail_after(kind, 5) == swan.OK
+        assert lib.swan_debug_fail_after(kind, -1) == swan.OK
+    # a bad configuration is rejected before any allocation, so an armed
+    # allocation fault stays armed and is then turned off
+    assert lib.swan_debug_fail_after(swan.FAULT_ALLOC, 0) == swan.OK
+    h = ctypes.c_void_p()
+    cfg = _cfg(k_store=0)
+    assert lib.swan_init(ctypes.byref(h), ctypes.byref(cfg), ctypes.c_void_p(4096), None) == swan.ERR_INVALID_ARG
+    assert lib.swan_debug_fail_after(swan.FAULT_ALLOC, -1) == swan.OK
 
 
 # ---------------------------------------------------------------------------

@@ -114,6 +114,7 @@ def test_decode_noalloc_matches_decode_twice():
         err = (got.float() - want.float()).abs().max().item()
         assert err <= TOL_OUT, err
     ctx.check()
+    ctx.check_guards()
     ctx.close()
 
     # sizes beyond the static scratch are rejected with a clear error

@@ -371,8 +371,9 @@ swan_status swan_decode_noalloc(const swan_cache_view* view, const void* q, void
 int64_t swan_launch_count(const swan_ctx* ctx);
 
 /*
- * Test hooks.  Every device buffer of a context sits between two 256-byte
- * guard regions filled with 0xA5 at swan_init; swan_debug_check_guards
+ * Test hooks.  Every device buffer of a context sits between guard regions
+ * (64 KB before, 256 bytes after) filled with 0xA5 at swan_init;
+ * swan_debug_check_guards
  * synchronises the stream and returns SWAN_ERR_DEVICE_CHECK (naming the
  * buffer) if a kernel wrote into one, else SWAN_OK (STATE, CUDA as usual).
  *

@@ -124,10 +124,12 @@ constexpr int kMaxBufferCap = 4096;
 constexpr int64_t kSmallAppendVectors = 256;  // batch * T per kv head
 constexpr size_t kMaxEventPairs = 4096;
 
-// Guard regions: kGuardBytes of kGuardByte before and after every device
-// buffer (256 bytes keep the buffers' alignment); swan_debug_check_guards
-// reports any that a kernel overwrote.
-constexpr size_t kGuardBytes = 256;
+// Guard regions of kGuardByte before (64 KB: the buffer keeps the 64 KB
+// alignment of a large allocation, which the decode stream measurably
+// prefers over a 256-byte offset) and after (256 bytes) every device buffer;
+// swan_debug_check_guards reports any that a kernel overwrote.
+constexpr size_t kFrontGuard = 65536;
+constexpr size_t kBackGuard = 256;
 constexpr unsigned char kGuardByte = 0xA5;
 
 // Test hooks: the n-th next device allocation / kernel launch fails (n = 0:
@@ -159,15 +161,15 @@ swan_status dev_alloc(swan_ctx* c, void** p, size_t bytes, const char* what) {
   *p = nullptr;
   if (injected(g_fail_alloc)) return fail(SWAN_ERR_NOMEM, "allocation for %s failed (injected)", what);
   void* base = nullptr;
-  cudaError_t e = cudaMalloc(&base, bytes + 2 * kGuardBytes);
+  cudaError_t e = cudaMalloc(&base, kFrontGuard + bytes + kBackGuard);
   if (e != cudaSuccess) {
     cudaGetLastError();
     return fail(SWAN_ERR_NOMEM, "cudaMalloc of %zu bytes for %s failed: %s", bytes, what,
                 cudaGetErrorString(e));
   }
   c->bufs.push_back({base, bytes, what});
-  *p = static_cast<char*>(base) + kGuardBytes;
-  c->device_bytes += (int64_t)(bytes + 2 * kGuardBytes);
+  *p = static_cast<char*>(base) + kFrontGuard;
+  c->device_bytes += (int64_t)(kFrontGuard + bytes + kBackGuard);
   return SWAN_OK;
 }
 
@@ -586,9 +588,9 @@ swan_status swan_init(swan_ctx** out, const swan_config* cfg, const float* R_qk,
   if (e == cudaSuccess) e = cudaMemsetAsync(c->counters, 0, (size_t)c->units * sizeof(int), st);
   if (e == cudaSuccess) e = cudaMemsetAsync(c->status, 0, sizeof(unsigned), st);
   for (const auto& b : c->bufs) {
-    if (e == cudaSuccess) e = cudaMemsetAsync(b.base, kGuardByte, kGuardBytes, st);
+    if (e == cudaSuccess) e = cudaMemsetAsync(b.base, kGuardByte, kFrontGuard, st);
     if (e == cudaSuccess)
-      e = cudaMemsetAsync(static_cast<char*>(b.base) + kGuardBytes + b.bytes, kGuardByte, kGuardBytes, st);
+      e = cudaMemsetAsync(static_cast<char*>(b.base) + kFrontGuard + b.bytes, kGuardByte, kBackGuard, st);
   }
   if (e == cudaSuccess) e = cudaStreamSynchronize(st);  // pt is a pageable host vector
   if (e != cudaSuccess) {
@@ -1209,13 +1211,14 @@ swan_status swan_debug_check_guards(swan_ctx* c) {
   if (s != SWAN_OK) return s;
   cudaError_t e = cudaStreamSynchronize(c->stream);
   if (e != cudaSuccess) return cuda_fail(c, e, "cudaStreamSynchronize");
-  std::vector<unsigned char> g(kGuardBytes);
+  std::vector<unsigned char> g(kFrontGuard);
   for (const auto& b : c->bufs)
     for (int side = 0; side < 2; ++side) {
-      const char* at = static_cast<const char*>(b.base) + (side ? kGuardBytes + b.bytes : 0);
-      e = cudaMemcpy(g.data(), at, kGuardBytes, cudaMemcpyDeviceToHost);
+      const char* at = static_cast<const char*>(b.base) + (side ? kFrontGuard + b.bytes : 0);
+      const size_t n = side ? kBackGuard : kFrontGuard;
+      e = cudaMemcpy(g.data(), at, n, cudaMemcpyDeviceToHost);
       if (e != cudaSuccess) return cuda_fail(c, e, "cudaMemcpy");
-      for (size_t i = 0; i < kGuardBytes; ++i)
+      for (size_t i = 0; i < n; ++i)
         if (g[i] != kGuardByte)
           return fail(SWAN_ERR_DEVICE_CHECK, "the guard region %s %s was overwritten (byte %zu)",
                       side ? "after" : "before", b.what, i);

@@ -794,8 +794,12 @@ __global__ void __launch_bounds__(decode_warps<MAXC>() * 32, decode_min_ctas<MAX
 //   result keeps fp32 accuracy at one product per tile.  No per-warp shared accumulator: the tile
 //   and a [G][32] p table are all a warp holds in shared memory.
 // ---------------------------------------------------------------------------
-constexpr int kVRowBytes = 272;                      // 128 fp16 + 16 B pad: conflict-free ldmatrix rows
-constexpr uint32_t kVTileBytes = 32 * kVRowBytes;    // 8704
+// Value tile rows: 128 fp16 (256 bytes, 256-byte aligned), the 16-byte
+// chunk j of token t's row stored at chunk j ^ (t & 7), so an ldmatrix of 8
+// token rows at one chunk hits 8 distinct bank groups, and the scatter
+// address is (2 idx) ^ (row | (t & 7) << 4): one shift and one LOP3.
+constexpr int kVRowBytes = 256;
+constexpr uint32_t kVTileBytes = 32 * kVRowBytes;    // 8192
 constexpr uint32_t kPTileBytes = 4 * 32 * 4;         // p [<= 4 heads][32 tokens] fp32
 // Per warp: the tile, the p table and a staging area for the value records
 // of the next block (cp.async: MAXC chunks of 512 B values + 256 B indices).
@@ -815,8 +819,8 @@ __host__ __device__ constexpr int mma_warps() { return 8; }
 // so they never share a bank.
 constexpr uint32_t kQrepBytes = kHeadDim * 32 * 4;
 template <int G, int MAXC>
-__host__ __device__ constexpr size_t mma_smem() {
-  return (size_t)kQrepBytes + (size_t)mma_warps<MAXC>() * mma_warp_bytes<MAXC>() + 16;
+__host__ __device__ constexpr size_t mma_smem() {  // + the 16 KB alignment slack
+  return (size_t)kQrepBytes + (size_t)mma_warps<MAXC>() * mma_warp_bytes<MAXC>() + 16384;
 }
 
 __device__ __forceinline__ uint4 lds_v4u(uint32_t a) {
@@ -883,15 +887,17 @@ __device__ __forceinline__ void chunk_half_words(const Chunk<FMT>& ch, uint32_t 
     }
   }
 }
-// Scores of G heads for one chunk: q' row idx of this lane is G floats.
-// Even and odd entries go to two partial sums per head (half-length FMA
-// chains).
+// Scores of G heads for one chunk: q' row idx of this lane is G floats
+// (128-byte rows, 16 KB-aligned base: the address is one shift and one
+// LOP3).  Even and odd entries go to two partial sums per head
+// (half-length FMA chains).
 template <int G>
 __device__ __forceinline__ void score_g_chunk(uint32_t qb, const float (&f)[8], uint2 ix, float (&s)[2][G]) {
 #pragma unroll
   for (int e = 0; e < 8; ++e) {
     const uint32_t w = e < 4 ? ix.x : ix.y;
-    const uint32_t a = qb + ((w >> (8 * (e & 3))) & 0x7fu) * 128u;
+    const int sh = 7 - 8 * (e & 3);  // byte e & 3 of w to bits 7..13
+    const uint32_t a = ((sh >= 0 ? (w << sh) : (w >> -sh)) & 0x3f80u) | qb;
     float* t = s[e & 1];
     if constexpr (G == 4) {
       const float4 q = lds4(a);
@@ -906,15 +912,17 @@ __device__ __forceinline__ void score_g_chunk(uint32_t qb, const float (&f)[8], 
     }
   }
 }
-// Scatter the first n (<= 8) entries of a chunk into this lane's tile row.
-__device__ __forceinline__ void scatter_chunk(uint32_t vrow, const uint32_t (&w)[4], uint2 ix, int n) {
+// Scatter the first n (<= 8) entries of a chunk into this lane's tile row
+// (vsw = the row's address | (lane & 7) << 4, the chunk swizzle).
+__device__ __forceinline__ void scatter_chunk(uint32_t vsw, const uint32_t (&w)[4], uint2 ix, int n) {
 #pragma unroll
   for (int e = 0; e < 8; ++e) {
     if (e < n) {
       const uint32_t iw = e < 4 ? ix.x : ix.y;
-      const uint32_t idx = (iw >> (8 * (e & 3))) & 0x7fu;
+      const int sh = 1 - 8 * (e & 3);  // byte e & 3 of iw, times 2
+      const uint32_t off = (sh >= 0 ? (iw << sh) : (iw >> -sh)) & 0xfeu;
       const uint32_t hw = w[e >> 1];
-      sts_u16(vrow + idx * 2, (e & 1) ? (hw >> 16) : (hw & 0xffffu));
+      sts_u16(off ^ vsw, (e & 1) ? (hw >> 16) : (hw & 0xffffu));
     }
   }
 }
@@ -931,16 +939,17 @@ __global__ void __launch_bounds__(mma_warps<MAXC>() * 32, 1) decode_mma_kernel(D
   pdl_trigger();
 
   const uint32_t raw = (uint32_t)__cvta_generic_to_shared(smem_raw);
-  const uint32_t base = (raw + 15u) & ~15u;
+  const uint32_t base = (raw + 16383u) & ~16383u;  // 16 KB aligned: q' and 256-byte tile rows
   unsigned char* base_ptr = smem_raw + (base - raw);
   float* qrep = reinterpret_cast<float*>(base_ptr);                         // [128][32/G][G]
   const uint32_t wbase = base + kQrepBytes;                                 // per-warp regions
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const uint32_t vtile = wbase + warp * kWarpBytes;                         // [32][272 B] fp16
+  const uint32_t vtile = wbase + warp * kWarpBytes;                         // [32][256 B] fp16, swizzled
   float* ptile_f = reinterpret_cast<float*>(base_ptr + (vtile + kVTileBytes - base));  // [G][32] fp32
   const uint32_t vstage = vtile + kVTileBytes + kPTileBytes;                  // value records, next block
   const uint32_t qb = base + (lane & (32 / G - 1)) * (G * 4);  // this lane's copy
   const uint32_t vrow = vtile + lane * kVRowBytes;
+  const uint32_t vsw = vrow | ((uint32_t)(lane & 7) << 4);  // this row with its chunk swizzle
   const int gq = lane >> 2, cq = lane & 3;  // mma fragment coordinates
 
   const CacheGeom& g = p.geom;
@@ -971,7 +980,7 @@ __global__ void __launch_bounds__(mma_warps<MAXC>() * 32, 1) decode_mma_kernel(D
   stage_q(u_first);
 
   // the tiles start zeroed; every use restores the zeros it disturbed
-  for (int c = 0; c < 16; ++c) sts_v4(vrow + c * 16, make_uint4(0, 0, 0, 0));
+  for (int c = 0; c < 16; ++c) sts_v4(vsw ^ (uint32_t)(c << 4), make_uint4(0, 0, 0, 0));
 
   for (int64_t u = u_first; u <= u_last; ++u) {
     const UnitView uv = unit_view(p, u);
@@ -1108,7 +1117,7 @@ __global__ void __launch_bounds__(mma_warps<MAXC>() * 32, 1) decode_mma_kernel(D
               if (c + 1 < nchunks_v) vn = staged(c + 1);
               uint32_t w[4];
               chunk_half_words<FMT>(vc, w);
-              scatter_chunk(vrow, w, chunk_idx<FMT>(vc), (krem_v && c == nchunks_v - 1) ? krem_v : 8);
+              scatter_chunk(vsw, w, chunk_idx<FMT>(vc), (krem_v && c == nchunks_v - 1) ? krem_v : 8);
               vc = vn;
             }
         }
@@ -1168,7 +1177,7 @@ __global__ void __launch_bounds__(mma_warps<MAXC>() * 32, 1) decode_mma_kernel(D
 #pragma unroll
             for (int k = 0; k < 8; ++k) wv[k] = __ldg(vr + cb + k);
 #pragma unroll
-            for (int k = 0; k < 8; ++k) sts_v4(vrow + (cb + k) * 16, wv[k]);
+            for (int k = 0; k < 8; ++k) sts_v4(vsw ^ (uint32_t)((cb + k) << 4), wv[k]);
           }
         }
       }
@@ -1215,8 +1224,9 @@ __global__ void __launch_bounds__(mma_warps<MAXC>() * 32, 1) decode_mma_kernel(D
 #pragma unroll
         for (int np = 0; np < 8; ++np) {
           const int mi = lane >> 3;
+          const uint32_t chunk = 2 * np + (mi >> 1);  // of 8 coordinates; rows of tokens, row & 7 = lane & 7
           const uint32_t addr = vtile + (uint32_t)(ks * 16 + (mi & 1) * 8 + (lane & 7)) * kVRowBytes +
-                                (uint32_t)(16 * np + 8 * (mi >> 1)) * 2;
+                                ((chunk ^ (uint32_t)(lane & 7)) << 4);
           uint32_t bf[4];
           ldsm_x4_trans(addr, bf);
           mma_16816(acc[2 * np], a0, a2, bf[0], bf[1]);
@@ -1226,7 +1236,7 @@ __global__ void __launch_bounds__(mma_warps<MAXC>() * 32, 1) decode_mma_kernel(D
       __syncwarp();
       // restore the zeros of this lane's tile row
       if (valid)
-        for (int c = 0; c < 16; ++c) sts_v4(vrow + c * 16, make_uint4(0, 0, 0, 0));
+        for (int c = 0; c < 16; ++c) sts_v4(vsw ^ (uint32_t)(c << 4), make_uint4(0, 0, 0, 0));
     }
 
     // ---- merge lanes and warps per query head into one partial
@@ -1285,7 +1295,7 @@ __global__ void __launch_bounds__(mma_warps<MAXC>() * 32, 1) decode_mma_kernel(D
     }
     __syncthreads();
     // the o rows overwrote part of the tiles: zero them again
-    for (int c = 0; c < 16; ++c) sts_v4(vrow + c * 16, make_uint4(0, 0, 0, 0));
+    for (int c = 0; c < 16; ++c) sts_v4(vsw ^ (uint32_t)(c << 4), make_uint4(0, 0, 0, 0));
     if (solo) {
       rotate_back_out<G, NT>(p, b, h, qrep, qrep);
     } else {

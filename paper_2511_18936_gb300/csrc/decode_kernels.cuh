@@ -100,10 +100,13 @@ __device__ __forceinline__ void keep_first(float (&f)[8], int n) {
   for (int e = 0; e < 8; ++e) f[e] = (e < n) ? f[e] : 0.f;
 }
 
+// Exact maximum over the warp in one reduction: floats compare as their
+// bits for v >= 0 and as bits ^ 0x7fffffff below zero (an order-preserving
+// map to int32 that is its own inverse).
 __device__ __forceinline__ float warp_max(float v) {
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
-  return v;
+  const int i = __float_as_int(v);
+  const int m = __reduce_max_sync(0xffffffffu, i >= 0 ? i : (i ^ 0x7fffffff));
+  return __int_as_float(m >= 0 ? m : (m ^ 0x7fffffff));
 }
 __device__ __forceinline__ float warp_sum(float v) {
 #pragma unroll
@@ -867,10 +870,11 @@ __device__ __forceinline__ void mma_16816(float (&d)[2], uint32_t a0, uint32_t a
 }
 // Two fp32 values as (hi, lo) fp16 pairs: x = hi + lo to ~2^-22 relative.
 __device__ __forceinline__ void split_pair(float x0, float x1, uint32_t& hi, uint32_t& lo) {
-  const __half h0 = __float2half_rn(x0), h1 = __float2half_rn(x1);
-  const __half l0 = __float2half_rn(x0 - __half2float(h0)), l1 = __float2half_rn(x1 - __half2float(h1));
-  hi = (uint32_t)__half_as_ushort(h0) | ((uint32_t)__half_as_ushort(h1) << 16);
-  lo = (uint32_t)__half_as_ushort(l0) | ((uint32_t)__half_as_ushort(l1) << 16);
+  const __half2 h = __floats2half2_rn(x0, x1);  // x0 in the low half
+  const float2 hf = __half22float2(h);
+  const __half2 l = __floats2half2_rn(x0 - hf.x, x1 - hf.y);
+  hi = *reinterpret_cast<const uint32_t*>(&h);
+  lo = *reinterpret_cast<const uint32_t*>(&l);
 }
 // The 8 values of a chunk as fp16 bits, two per word.
 template <int FMT>

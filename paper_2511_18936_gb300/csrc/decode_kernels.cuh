@@ -108,6 +108,13 @@ __device__ __forceinline__ float warp_max(float v) {
   const int m = __reduce_max_sync(0xffffffffu, i >= 0 ? i : (i ^ 0x7fffffff));
   return __int_as_float(m >= 0 ? m : (m ^ 0x7fffffff));
 }
+// 2^x by the hardware approximation (relative error ~2^-22; results below
+// 2^-126 flush to zero, negligible next to the running maximum's 1).
+__device__ __forceinline__ float ex2(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
 __device__ __forceinline__ float warp_sum(float v) {
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
@@ -1194,7 +1201,7 @@ __global__ void __launch_bounds__(mma_warps<MAXC>() * 32, 1) decode_mma_kernel(D
         const float gmax = warp_max(sj);
         if (gmax > m[j] + kLazyRescale) {
           if (m[j] != -INFINITY) {
-            const float fs = exp2f(m[j] - gmax);
+            const float fs = ex2(m[j] - gmax);
             l[j] *= fs;
             if (gq == j || gq == j + G) {  // the head's hi and lo rows
 #pragma unroll
@@ -1203,7 +1210,7 @@ __global__ void __launch_bounds__(mma_warps<MAXC>() * 32, 1) decode_mma_kernel(D
           }
           m[j] = gmax;
         }
-        pj[j] = valid ? exp2f(sj - m[j]) : 0.f;
+        pj[j] = valid ? ex2(sj - m[j]) : 0.f;
         l[j] += pj[j];
         ptile_f[j * 32 + lane] = pj[j];
       }

@@ -269,7 +269,7 @@ __global__ void __launch_bounds__(kThreads, 1) append_tc_kernel(const __grid_con
                                                                  const __grid_constant__ CUtensorMap rlo,
                                                                  AppendParams p, int r_slice0) {
   using namespace sm100;
-  extern __shared__ __align__(1024) unsigned char smem_raw[];
+  extern __shared__ __align__(1024) unsigned char smem_tc[];
   __shared__ __align__(8) uint64_t bars[2];
   __shared__ uint32_t tmem_slot;
   __shared__ int failed;
@@ -281,10 +281,10 @@ __global__ void __launch_bounds__(kThreads, 1) append_tc_kernel(const __grid_con
   pdl_trigger();
   if (j0 >= rv.n_new) return;  // no new token of this row in the tile (uniform in the CTA)
 
-  const uint32_t raw = smem_u32(smem_raw);
+  const uint32_t raw = smem_u32(smem_tc);
   const uint32_t ta = (raw + 1023u) & ~1023u;  // A, then the staged rows
   const uint32_t tb_hi = ta + kTcTile, tb_lo = tb_hi + kTcTile;
-  unsigned char* stage = smem_raw + (ta - raw);
+  unsigned char* stage = smem_tc + (ta - raw);
   const uint32_t full = smem_u32(&bars[0]), done = smem_u32(&bars[1]);
   if (threadIdx.x == 0) {
     mbar_init(full, 1);

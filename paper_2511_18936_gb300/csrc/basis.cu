@@ -33,13 +33,13 @@ constexpr uint64_t kWaitLimitNs = 2000000000ull;  // 2 s per barrier wait
 // ---------------------------------------------------------------------------
 template <bool kMnMajor>
 __global__ void __launch_bounds__(128, 1) gram_kernel(const __grid_constant__ CUtensorMap tmap, GramParams p) {
-  extern __shared__ __align__(1024) unsigned char smem_raw[];
+  extern __shared__ __align__(1024) unsigned char smem_tc[];
   __shared__ __align__(8) uint64_t bars[2 * kGramStages + 1];
   __shared__ uint32_t tmem_base_slot;
   __shared__ int abort_flag;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const uint32_t raw = smem_u32(smem_raw);
+  const uint32_t raw = smem_u32(smem_tc);
   const uint32_t tiles = (raw + 1023u) & ~1023u;
   const uint32_t full0 = smem_u32(&bars[0]), empty0 = smem_u32(&bars[kGramStages]);
   const uint32_t done = smem_u32(&bars[2 * kGramStages]);

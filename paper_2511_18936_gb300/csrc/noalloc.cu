@@ -127,7 +127,8 @@ extern "C" swan_status swan_decode_noalloc(const swan_cache_view* v, const void*
   const int64_t total = units * N_g;
   int64_t grid = 0;
   if (total > 0)
-    grid = std::min<int64_t>((int64_t)ds->sms * ds->ctas_per_sm[gi(G)][std::max(v->k_active, kav) > 64], total);
+    grid = std::min<int64_t>((int64_t)ds->sms * ds->ctas_per_sm[gi(G)][std::max(v->k_active, kav) > 64],
+                             std::max<int64_t>(1, total / kMinGroupsPerCta));
   if ((grid + units) * G > kNoallocMaxSlots)
     return err(SWAN_ERR_INVALID_ARG, "(decode CTAs + batch * n_kv_heads) * G exceeds 2048 (static scratch)");
 

@@ -333,12 +333,6 @@ swan_status upload_rows(swan_ctx* c, int layer, const std::vector<SeqInfo>& rows
   return SWAN_OK;
 }
 
-// Fewest 32-token groups a decode CTA takes: a small cache is split over
-// fewer CTAs so that each one's fixed cost (staging q', the merge) and the
-// final combine over the CTAs' partials stay small next to its groups
-// (swept on the GB300 for one head at 1088 tokens, L2 flushed: decode 20.4 us
-// at 2 and 4, 22.4 us at 8, 24.8 us at 16).
-constexpr int64_t kMinGroupsPerCta = 4;
 
 // Work of one unit segment of a decode CTA beyond its groups (staging q',
 // the merge, the rotate-back, and the pipeline start of every warp's short

@@ -297,6 +297,12 @@ cudaError_t launch_transpose_r(const float* src, float* dst, int64_t mats, cudaS
 cudaError_t launch_scatter_pages(const int2* pairs, int n, int32_t* table, cudaStream_t s);
 // Decode CTAs that fit on one SM together (for the grid size).
 int decode_ctas_per_sm(int G, int k_slots);
+// Fewest 32-token groups a decode CTA takes: a small cache is split over
+// fewer CTAs so that each one's fixed cost (staging q', the merge) and the
+// final combine over the CTAs' partials stay small next to its groups
+// (swept on the GB300 for one head at 1088 tokens, L2 flushed: decode 20.4 us
+// at 2 and 4, 22.4 us at 8, 24.8 us at 16).
+constexpr int64_t kMinGroupsPerCta = 4;
 // What a CTA's extra visit to a unit (prologue, merge, arrival) costs in
 // 32-token groups of streaming, for the cost-balanced split of the decode
 // kernels: equal-length rows (computed in the kernel) and ragged rows (the

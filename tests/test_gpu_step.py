@@ -132,3 +132,39 @@ def test_append_decode_launches_and_errors():
     assert torch.equal(out, snap)
     fused.check()
     fused.close()
+
+
+def test_documented_usage_matches_the_oracle():
+    """The flow the README shows (prefill, decode, a fused serving step, a
+    smaller runtime k), on layer 1 of a two-layer GQA context, against the
+    oracle fed the same operations."""
+    import torch
+
+    from paper_2511_18936_gb300 import swan
+    B, Hq, Hkv, cap = 2, 4, 2, 16
+    R = np.stack([synth.rotations(Hkv, D, seed=9, workload=98, layer=l) for l in range(2)])
+    dev = torch.device("cuda")
+    ctx = swan.Context(torch.from_numpy(R).to(dev), num_layers=2, batch=B, n_q_heads=Hq, n_kv_heads=Hkv,
+                       k_store=64, buffer_cap=cap, max_seq=512)
+    ref = oracle.SwanOracle(R[1], None, batch=B, n_q_heads=Hq, k_store=64, buffer_cap=cap)
+    k = synth.lowrank_kv(B, Hkv, 300, D, 9, 98, 1, synth.T_K)
+    v = synth.lowrank_kv(B, Hkv, 300, D, 9, 98, 1, synth.T_V)
+    q = synth.gaussian_fp16((B, Hq, D), 9, 98, 1, synth.T_Q)
+    tq = torch.from_numpy(q).to(dev)
+    ctx.append(1, torch.from_numpy(k).to(dev), torch.from_numpy(v).to(dev))
+    ref.append(k, v)
+    outs = [(ctx.decode(1, tq), ref.decode(q))]
+    k1 = synth.lowrank_kv(B, Hkv, 1, D, 9, 98, 2, synth.T_K)
+    v1 = synth.lowrank_kv(B, Hkv, 1, D, 9, 98, 2, synth.T_V)
+    outs.append((ctx.append_decode(1, torch.from_numpy(k1).to(dev), torch.from_numpy(v1).to(dev), tq), None))
+    ref.append(k1, v1)
+    outs[-1] = (outs[-1][0], ref.decode(q))
+    ctx.set_k(48)
+    ref.set_k(48)
+    outs.append((ctx.decode(1, tq), ref.decode(q)))
+    ctx.check()
+    ctx.check_guards()
+    for got, want in outs:
+        assert np.abs(got.float().cpu().numpy() - want).max() <= TOL_OUT
+    assert ctx.lengths(0) == ([0] * B, [0] * B)  # the other layer is untouched
+    ctx.close()

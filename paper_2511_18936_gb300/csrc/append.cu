@@ -4,6 +4,7 @@
 #include <cuda_fp8.h>
 
 #include "sm100.h"
+#include "sortnet.cuh"
 #include "swan_internal.h"
 
 namespace swan {
@@ -243,37 +244,88 @@ __global__ void transpose_r_kernel(const float* src, float* dst, int64_t mats) {
 
 // ---------------------------------------------------------------------------
 // Bulk append with the rotation on the tensor cores.
-//   One CTA: 128 new vectors of one (row, kv head, K or V).  TMA brings the
-//   fp16 vectors (A: 128 x 128, K-major, 128-byte swizzle) and the split
-//   rotation R^T = R_hi^T + 2^-12 R_lo^T (B: two fp16 128 x 128 tiles); two
-//   tcgen05.mma chains (K = 16 each step) accumulate x R_hi and x R_lo in two
-//   128-column TMEM accumulators; warps 0-3 read them back (row = vector),
-//   form y = hi + 2^-12 lo in fp32, round to fp16 and stage the rows in
-//   shared memory (16-byte chunks XOR-swizzled by row); then all 8 warps
-//   write each vector to its ring slot or prune it (warp_prune_store).  The
-//   products are exact (fp16 x fp16) and summed in fp32; the split leaves
-//   2^-22 |R| per term, inside the fp32-dot bound of the CUDA-core path.
+//   One CTA of 128 threads: 128 new vectors of one (row, kv head, K or V).
+//   TMA brings the fp16 vectors (A: 128 x 128, K-major, 128-byte swizzle) and
+//   the split rotation R^T = R_hi^T + 2^-12 R_lo^T (B: two fp16 128 x 128
+//   tiles); two tcgen05.mma chains (K = 16 each step) accumulate x R_hi and
+//   x R_lo in two 128-column TMEM accumulators.  Thread v then reads row v
+//   (vector v) back, forms y = hi + 2^-12 lo in fp32 and rounds it to fp16,
+//   and handles the vector alone: the 128 sort keys stay in its registers,
+//   a sorting network (sortnet.cuh) orders them, and it writes its ring row
+//   or its sparse records (consecutive threads hold consecutive tokens, so
+//   each chunk of 32 records is one coalesced 512-byte run).  The products
+//   are exact (fp16 x fp16) and summed in fp32; the split leaves 2^-22 |R|
+//   per term, inside the fp32-dot bound of the CUDA-core path.
 // ---------------------------------------------------------------------------
+constexpr int kTcThreads = 128;              // one thread per vector of the tile
 constexpr uint32_t kTcTile = 128 * 128 * 2;  // 32 KB: one fp16 128 x 128 tile
 constexpr size_t kTcSmem = 3 * kTcTile + 1024;
 constexpr uint64_t kTcWaitNs = 2000000000ull;
+// a key that decodes to value +0 at index 0 (the padding entries of a chunk)
+constexpr uint32_t kPadKey = 127u << 1;
 
-// byte offset of (row v, coordinate c) in the staged fp16 rows
-__device__ __forceinline__ uint32_t staged_off(int v, int c) {
-  return (uint32_t)v * 256u + ((uint32_t)((c >> 3) ^ (v & 15)) << 4) + (uint32_t)(c & 7) * 2u;
+// fp16 bits of two keys, packed (first key in the low half)
+__device__ __forceinline__ uint32_t key_bits2(uint32_t ka, uint32_t kb) {
+  return __byte_perm(ka, kb, 0x7632) | ((ka & 1u) << 15) | (kb << 31);
+}
+// coordinate indices of four keys, one per byte
+__device__ __forceinline__ uint32_t key_idx4(uint32_t k0, uint32_t k1, uint32_t k2, uint32_t k3) {
+  const uint32_t lo = __byte_perm(~k0 >> 1, ~k1 >> 1, 0x0040);
+  const uint32_t hi = __byte_perm(~k2 >> 1, ~k3 >> 1, 0x0040);
+  return __byte_perm(lo, hi, 0x5410) & 0x7f7f7f7fu;
 }
 
-__global__ void __launch_bounds__(kThreads, 1) append_tc_kernel(const __grid_constant__ CUtensorMap xk,
-                                                                 const __grid_constant__ CUtensorMap xv,
-                                                                 const __grid_constant__ CUtensorMap rhi,
-                                                                 const __grid_constant__ CUtensorMap rlo,
-                                                                 AppendParams p, int r_slice0) {
+// Write the first `slots` sorted keys of one vector (those at or beyond
+// `kept` as padding) to its records: chunk c of 8 entries at record
+// c * 32 + t of the block.
+template <int NCH>
+__device__ __forceinline__ void store_sorted(const uint32_t (&key)[128], int slots, int kept, uint8_t* vals,
+                                             uint8_t* idx, int t, bool fp8) {
+#pragma unroll
+  for (int c = 0; c < NCH; ++c) {
+    if (8 * c >= slots) break;
+    uint32_t k[8];
+#pragma unroll
+    for (int e = 0; e < 8; ++e) k[e] = (8 * c + e < kept) ? key[8 * c + e] : kPadKey;
+    const int rec = c * 32 + t;
+    const uint32_t i0 = key_idx4(k[0], k[1], k[2], k[3]), i1 = key_idx4(k[4], k[5], k[6], k[7]);
+    if (fp8) {
+      // one 16-byte record: 8 E4M3 values (round to nearest even, saturating
+      // to +-448), then the 8 indices
+      uint32_t v8[2];
+#pragma unroll
+      for (int w = 0; w < 2; ++w) {
+        uint32_t pair[2];
+#pragma unroll
+        for (int q = 0; q < 2; ++q) {
+          const uint32_t b2 = key_bits2(k[4 * w + 2 * q], k[4 * w + 2 * q + 1]);
+          __half2_raw hr;
+          hr.x = (unsigned short)(b2 & 0xffffu);
+          hr.y = (unsigned short)(b2 >> 16);
+          pair[q] = __nv_cvt_halfraw2_to_fp8x2(hr, __NV_SATFINITE, __NV_E4M3);
+        }
+        v8[w] = pair[0] | (pair[1] << 16);
+      }
+      *reinterpret_cast<uint4*>(vals + rec * 16) = make_uint4(v8[0], v8[1], i0, i1);
+    } else {
+      *reinterpret_cast<uint4*>(vals + rec * 16) =
+          make_uint4(key_bits2(k[0], k[1]), key_bits2(k[2], k[3]), key_bits2(k[4], k[5]), key_bits2(k[6], k[7]));
+      *reinterpret_cast<uint2*>(idx + rec * 8) = make_uint2(i0, i1);
+    }
+  }
+}
+
+__global__ void __launch_bounds__(kTcThreads, 1) append_tc_kernel(const __grid_constant__ CUtensorMap xk,
+                                                                   const __grid_constant__ CUtensorMap xv,
+                                                                   const __grid_constant__ CUtensorMap rhi,
+                                                                   const __grid_constant__ CUtensorMap rlo,
+                                                                   AppendParams p, int r_slice0) {
   using namespace sm100;
   extern __shared__ __align__(1024) unsigned char smem_tc[];
   __shared__ __align__(8) uint64_t bars[2];
   __shared__ uint32_t tmem_slot;
   __shared__ int failed;
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int warp = threadIdx.x >> 5;
   const int kind = blockIdx.z, h = blockIdx.y;
   const int tiles_per_row = (p.T + 127) / 128;
   const int b = blockIdx.x / tiles_per_row, j0 = (blockIdx.x % tiles_per_row) * 128;
@@ -282,9 +334,8 @@ __global__ void __launch_bounds__(kThreads, 1) append_tc_kernel(const __grid_con
   if (j0 >= rv.n_new) return;  // no new token of this row in the tile (uniform in the CTA)
 
   const uint32_t raw = smem_u32(smem_tc);
-  const uint32_t ta = (raw + 1023u) & ~1023u;  // A, then the staged rows
+  const uint32_t ta = (raw + 1023u) & ~1023u;
   const uint32_t tb_hi = ta + kTcTile, tb_lo = tb_hi + kTcTile;
-  unsigned char* stage = smem_tc + (ta - raw);
   const uint32_t full = smem_u32(&bars[0]), done = smem_u32(&bars[1]);
   if (threadIdx.x == 0) {
     mbar_init(full, 1);
@@ -327,18 +378,19 @@ __global__ void __launch_bounds__(kThreads, 1) append_tc_kernel(const __grid_con
   }
   __syncwarp();
 
-  // ---- TMEM -> fp16 rows in shared memory (A's tile, free once the MMAs are done)
-  if (warp < 4) {
-    if (!mbar_wait(done, 0, kTcWaitNs)) {
-      atomicOr(p.status, kStatusTimeout);
-      failed = 1;
-    }
-    tc_fence_after();
+  // ---- TMEM -> this thread's vector as 128 sort keys, through shared memory
+  // (the operand tiles are free once the MMAs are done): key c of vector v at
+  // 16 * (128 * (c / 4) + v) + 4 * (c % 4), so that the 32 vectors of a warp
+  // move 4 keys each as one conflict-free 512-byte run.  The key of
+  // coordinate c is (|y_c| as fp16 bits, 127 - c, sign): unique, ordered by
+  // magnitude first, then lower index first.
+  if (!mbar_wait(done, 0, kTcWaitNs)) {
+    atomicOr(p.status, kStatusTimeout);
+    failed = 1;
   }
-  __syncthreads();
-  const bool ok = failed == 0;  // uniform in the CTA
-  if (warp < 4 && ok) {
-    const int v = 32 * warp + lane;
+  tc_fence_after();
+  uint4* keys_s = reinterpret_cast<uint4*>(smem_tc + (ta - raw)) + threadIdx.x;
+  {
     const uint32_t taddr = tmem + ((uint32_t)(32 * warp) << 16);
 #pragma unroll 1
     for (int c = 0; c < 4; ++c) {
@@ -346,40 +398,79 @@ __global__ void __launch_bounds__(kThreads, 1) append_tc_kernel(const __grid_con
       tmem_ld32(taddr + c * 32, hi);
       tmem_ld32(taddr + 128 + c * 32, lo);
       tmem_wait_ld();
+      tmem_regs_ready(hi);
+      tmem_regs_ready(lo);
 #pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        uint32_t w[4];
+      for (int q = 0; q < 8; ++q) {
+        uint32_t k[4];
 #pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          const int m = 8 * q + 2 * e;
+        for (int e = 0; e < 4; e += 2) {
+          const int m = 4 * q + e;
           const float y0 = fmaf(__uint_as_float(lo[m]), 1.f / 4096.f, __uint_as_float(hi[m]));
           const float y1 = fmaf(__uint_as_float(lo[m + 1]), 1.f / 4096.f, __uint_as_float(hi[m + 1]));
-          w[e] = (uint32_t)__half_as_ushort(__float2half_rn(y0)) |
-                 ((uint32_t)__half_as_ushort(__float2half_rn(y1)) << 16);
+          const __half2 y2 = __floats2half2_rn(y0, y1);
+          const uint32_t h2 = *reinterpret_cast<const uint32_t*>(&y2);
+          const uint32_t j = (uint32_t)(32 * c + m);
+          k[e] = ((h2 & 0x7fffu) << 16) | ((127u - j) << 1) | ((h2 >> 15) & 1u);
+          k[e + 1] = (h2 & 0x7fff0000u) | ((126u - j) << 1) | (h2 >> 31);
         }
-        *reinterpret_cast<uint4*>(stage + staged_off(v, c * 32 + q * 8)) = make_uint4(w[0], w[1], w[2], w[3]);
+        keys_s[128 * (8 * c + q)] = make_uint4(k[0], k[1], k[2], k[3]);
       }
     }
   }
   tc_fence_before();
   __syncthreads();
   if (warp == 1) tmem_dealloc(tmem, 256);
-  if (!ok) return;
+  if (failed != 0) return;  // uniform in the CTA
 
-  // ---- ring insert or prune, one vector per warp at a time
-  __half* ring = kind ? p.ring_v : p.ring_k;
+  // ---- ring insert or prune of vector v
+  const int v = threadIdx.x, j = j0 + v;
+  if (j >= rv.n_new) return;
+  uint32_t key[128];
+#pragma unroll
+  for (int q = 0; q < 32; ++q) {
+    const uint4 k4 = keys_s[128 * q];
+    key[4 * q] = k4.x;
+    key[4 * q + 1] = k4.y;
+    key[4 * q + 2] = k4.z;
+    key[4 * q + 3] = k4.w;
+  }
   const int64_t unit = (int64_t)b * p.H + h;
-  for (int v = warp; v < 128; v += kWarpsPerCta) {
-    const int j = j0 + v;
-    if (j >= rv.n_new) break;
-    const uint2 raw2 = *reinterpret_cast<const uint2*>(stage + staged_off(v, 4 * lane));
-    const int64_t pos = (int64_t)rv.n_b + j;
-    if (pos < rv.evict) {
-      warp_prune_store(raw2, lane, kind, unit, rv.sparse_len + pos, p.geom, p.status);
-    } else {
-      const int slot = (int)((rv.buf_start + pos) % p.cap);
-      reinterpret_cast<uint2*>(ring + (unit * p.cap + slot) * kHeadDim)[lane] = raw2;
-    }
+  const int64_t pos = (int64_t)rv.n_b + j;
+  if (pos >= rv.evict) {
+    const int slot = (int)((rv.buf_start + pos) % p.cap);
+    uint4* row = reinterpret_cast<uint4*>((kind ? p.ring_v : p.ring_k) + (unit * p.cap + slot) * kHeadDim);
+#pragma unroll
+    for (int q = 0; q < 16; ++q)
+      row[q] = make_uint4(key_bits2(key[8 * q], key[8 * q + 1]), key_bits2(key[8 * q + 2], key[8 * q + 3]),
+                          key_bits2(key[8 * q + 4], key[8 * q + 5]), key_bits2(key[8 * q + 6], key[8 * q + 7]));
+    return;
+  }
+  const CacheGeom& g = p.geom;
+  const int64_t sp = rv.sparse_len + pos;
+  const int64_t page = sp / g.P;
+  const int slot = (int)(sp % g.P);
+  if (page >= g.pages_per_unit) {
+    atomicOr(p.status, kStatusPageRange);
+    return;
+  }
+  const int32_t phys = g.page_table[unit * g.pages_per_unit + page];
+  if (phys < 0 || phys >= g.num_pages) {
+    atomicOr(p.status, kStatusPageRange);
+    return;
+  }
+  uint8_t* blk = g.pool + (int64_t)phys * g.page_bytes + (int64_t)(slot >> 5) * g.block_bytes();
+  const bool fp8 = g.fmt == kFmtFp8;
+  const int slots = kind ? g.k_slots_v : g.k_slots;
+  const int kept = kind ? g.k_store_v : g.k_store;
+  uint8_t* vals = blk + (kind ? g.vval_off() : 0);
+  uint8_t* idx = blk + (kind ? g.vidx_off() : g.kidx_off());
+  if (slots <= 64) {
+    sortnet::top64_of128_desc(key);
+    store_sorted<8>(key, slots, kept, vals, idx, slot & 31, fp8);
+  } else {
+    sortnet::sort128_desc_full(key);
+    store_sorted<16>(key, slots, kept, vals, idx, slot & 31, fp8);
   }
 }
 
@@ -411,7 +502,7 @@ cudaError_t launch_append_tc(const AppendParams& p, const CUtensorMap* maps, int
   cudaError_t e = ensure_smem<append_tc_kernel>(kTcSmem);
   if (e != cudaSuccess) return e;
   const int tiles = p.B * ((p.T + 127) / 128);
-  return launch_pdl(append_tc_kernel, dim3((unsigned)tiles, (unsigned)p.H, 2), dim3(kThreads), kTcSmem, s,
+  return launch_pdl(append_tc_kernel, dim3((unsigned)tiles, (unsigned)p.H, 2), dim3(kTcThreads), kTcSmem, s,
                     maps[0], maps[1], maps[2], maps[3], p, r_slice0);
 }
 

@@ -244,20 +244,22 @@ __global__ void transpose_r_kernel(const float* src, float* dst, int64_t mats) {
 
 // ---------------------------------------------------------------------------
 // Bulk append with the rotation on the tensor cores.
-//   One CTA of 128 threads: 128 new vectors of one (row, kv head, K or V).
+//   One CTA of 256 threads: 128 new vectors of one (row, kv head, K or V).
 //   TMA brings the fp16 vectors (A: 128 x 128, K-major, 128-byte swizzle) and
 //   the split rotation R^T = R_hi^T + 2^-12 R_lo^T (B: two fp16 128 x 128
 //   tiles); two tcgen05.mma chains (K = 16 each step) accumulate x R_hi and
-//   x R_lo in two 128-column TMEM accumulators.  Thread v then reads row v
-//   (vector v) back, forms y = hi + 2^-12 lo in fp32 and rounds it to fp16,
-//   and handles the vector alone: the 128 sort keys stay in its registers,
-//   a sorting network (sortnet.cuh) orders them, and it writes its ring row
-//   or its sparse records (consecutive threads hold consecutive tokens, so
-//   each chunk of 32 records is one coalesced 512-byte run).  The products
-//   are exact (fp16 x fp16) and summed in fp32; the split leaves 2^-22 |R|
-//   per term, inside the fp32-dot bound of the CUDA-core path.
+//   x R_lo in two 128-column TMEM accumulators.  The rows are read back as
+//   y = hi + 2^-12 lo in fp32, rounded to fp16 and turned into sort keys,
+//   which pass through shared memory to their owners: lanes 2v and 2v+1 hold
+//   coordinates 0..63 and 64..127 of vector v.  Each lane sorts its 64 keys
+//   in registers (sortnet.cuh); the pair then merges the two sorted halves
+//   with shuffles and writes its ring row or its sparse records (consecutive
+//   pairs hold consecutive tokens, so the records of a chunk are contiguous).
+//   The products are exact (fp16 x fp16) and summed in fp32; the split
+//   leaves 2^-22 |R| per term, inside the fp32-dot bound of the CUDA-core
+//   path.
 // ---------------------------------------------------------------------------
-constexpr int kTcThreads = 128;              // one thread per vector of the tile
+constexpr int kTcThreads = 256;              // two threads per vector of the tile
 constexpr uint32_t kTcTile = 128 * 128 * 2;  // 32 KB: one fp16 128 x 128 tile
 constexpr size_t kTcSmem = 3 * kTcTile + 1024;
 constexpr uint64_t kTcWaitNs = 2000000000ull;
@@ -268,25 +270,74 @@ constexpr uint32_t kPadKey = 127u << 1;
 __device__ __forceinline__ uint32_t key_bits2(uint32_t ka, uint32_t kb) {
   return __byte_perm(ka, kb, 0x7632) | ((ka & 1u) << 15) | (kb << 31);
 }
-// coordinate indices of four keys, one per byte
+// coordinate indices of four keys, one per byte: the low key byte is
+// (127 - c) << 1 | sign, and (~byte >> 1) & 127 = c
 __device__ __forceinline__ uint32_t key_idx4(uint32_t k0, uint32_t k1, uint32_t k2, uint32_t k3) {
-  const uint32_t lo = __byte_perm(~k0 >> 1, ~k1 >> 1, 0x0040);
-  const uint32_t hi = __byte_perm(~k2 >> 1, ~k3 >> 1, 0x0040);
-  return __byte_perm(lo, hi, 0x5410) & 0x7f7f7f7fu;
+  const uint32_t w = __byte_perm(__byte_perm(k0, k1, 0x0040), __byte_perm(k2, k3, 0x0040), 0x5410);
+  return (~w >> 1) & 0x7f7f7f7fu;
 }
 
-// Write the first `slots` sorted keys of one vector (those at or beyond
-// `kept` as padding) to its records: chunk c of 8 entries at record
-// c * 32 + t of the block.
-template <int NCH>
-__device__ __forceinline__ void store_sorted(const uint32_t (&key)[128], int slots, int kept, uint8_t* vals,
-                                             uint8_t* idx, int t, bool fp8) {
+// r ? x : y for r in {0, 1}, as multiply-adds (off the integer min/max pipe)
+__device__ __forceinline__ uint32_t pick(uint32_t r, uint32_t x, uint32_t y, uint32_t one) {
+  return r * (x - y * one) + y;
+}
+
+// The 64 largest keys of a vector whose halves A (lane r = 0) and B (r = 1)
+// are each sorted decreasing in a[]: A followed by B reversed is a bitonic
+// run whose first half-cleaner keeps C[i] = max(A[i], B[63 - i]), the 64
+// largest, again bitonic; its merge starts with a half-cleaner across the
+// pair.  Afterwards lane r holds ranks 32 r .. 32 r + 31 in c[].
+__device__ __forceinline__ void pair_top64(const uint32_t (&a)[64], uint32_t (&c)[32], uint32_t r,
+                                           uint32_t one) {
 #pragma unroll
-  for (int c = 0; c < NCH; ++c) {
+  for (int m = 0; m < 32; ++m) {  // lane r computes C[32 r + m]
+    const uint32_t send = pick(r, a[63 - m], a[32 + m], one);
+    const uint32_t own = pick(r, a[31 - m], a[m], one);
+    c[m] = sortnet::umax(own, __shfl_xor_sync(0xffffffffu, send, 1));
+  }
+#pragma unroll
+  for (int m = 0; m < 32; ++m) {  // larger to lane 0, smaller to lane 1
+    const uint32_t o = __shfl_xor_sync(0xffffffffu, c[m], 1);
+    const uint32_t hi = sortnet::umax(c[m], o);
+    c[m] = pick(r, (c[m] * one + o) - hi * one, hi, one);
+  }
+  sortnet::merge_desc<0, 32>(c, one);
+}
+
+// All 128 keys: the first half-cleaner of the same bitonic run crosses the
+// pair (A[i] against B[63 - i]); afterwards lane r holds ranks 64 r ..
+// 64 r + 63 in a[].
+__device__ __forceinline__ void pair_sort128(uint32_t (&a)[64], uint32_t r, uint32_t one) {
+  uint32_t s[64];
+#pragma unroll
+  for (int i = 0; i < 64; ++i) {
+    const uint32_t own = pick(r, a[63 - i], a[i], one);
+    const uint32_t o = __shfl_xor_sync(0xffffffffu, own, 1);
+    const uint32_t hi = sortnet::umax(own, o);
+    s[i] = pick(r, (own * one + o) - hi * one, hi, one);
+  }
+#pragma unroll
+  for (int i = 0; i < 64; ++i) a[i] = s[i];
+  sortnet::merge_desc<0, 64>(a, one);
+}
+
+// Write sorted keys of ranks rank0 .. rank0 + N - 1 of one vector (ranks at
+// or beyond `kept` as padding, none at or beyond `slots`) to its records:
+// the chunk of ranks 8c .. 8c + 7 at record c * 32 + t of the block.
+template <int N>
+__device__ __forceinline__ void store_sorted(const uint32_t (&key)[N], int rank0, int slots, int kept,
+                                             uint8_t* vals, uint8_t* idx, int t, bool fp8) {
+#pragma unroll
+  for (int cc = 0; cc < N / 8; ++cc) {
+    const int c = rank0 / 8 + cc;
     if (8 * c >= slots) break;
     uint32_t k[8];
 #pragma unroll
-    for (int e = 0; e < 8; ++e) k[e] = (8 * c + e < kept) ? key[8 * c + e] : kPadKey;
+    for (int e = 0; e < 8; ++e) k[e] = key[8 * cc + e];
+    if (8 * c + 8 > kept) {  // the last kept chunk (uniform in the CTA)
+#pragma unroll
+      for (int e = 0; e < 8; ++e) k[e] = (8 * c + e < kept) ? k[e] : kPadKey;
+    }
     const int rec = c * 32 + t;
     const uint32_t i0 = key_idx4(k[0], k[1], k[2], k[3]), i1 = key_idx4(k[4], k[5], k[6], k[7]);
     if (fp8) {
@@ -315,17 +366,17 @@ __device__ __forceinline__ void store_sorted(const uint32_t (&key)[128], int slo
   }
 }
 
-__global__ void __launch_bounds__(kTcThreads, 1) append_tc_kernel(const __grid_constant__ CUtensorMap xk,
+__global__ void __launch_bounds__(kTcThreads, 2) append_tc_kernel(const __grid_constant__ CUtensorMap xk,
                                                                    const __grid_constant__ CUtensorMap xv,
                                                                    const __grid_constant__ CUtensorMap rhi,
                                                                    const __grid_constant__ CUtensorMap rlo,
-                                                                   AppendParams p, int r_slice0) {
+                                                                   AppendParams p, int r_slice0, uint32_t one) {
   using namespace sm100;
   extern __shared__ __align__(1024) unsigned char smem_tc[];
   __shared__ __align__(8) uint64_t bars[2];
   __shared__ uint32_t tmem_slot;
   __shared__ int failed;
-  const int warp = threadIdx.x >> 5;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int kind = blockIdx.z, h = blockIdx.y;
   const int tiles_per_row = (p.T + 127) / 128;
   const int b = blockIdx.x / tiles_per_row, j0 = (blockIdx.x % tiles_per_row) * 128;
@@ -378,22 +429,24 @@ __global__ void __launch_bounds__(kTcThreads, 1) append_tc_kernel(const __grid_c
   }
   __syncwarp();
 
-  // ---- TMEM -> this thread's vector as 128 sort keys, through shared memory
-  // (the operand tiles are free once the MMAs are done): key c of vector v at
-  // 16 * (128 * (c / 4) + v) + 4 * (c % 4), so that the 32 vectors of a warp
-  // move 4 keys each as one conflict-free 512-byte run.  The key of
-  // coordinate c is (|y_c| as fp16 bits, 127 - c, sign): unique, ordered by
-  // magnitude first, then lower index first.
+  // ---- TMEM -> sort keys in shared memory (the operand tiles are free once
+  // the MMAs are done).  Warp w reads rows 32 (w % 4) .. + 31 (its TMEM lane
+  // quarter), coordinates 64 (w / 4) .. + 63.  The key of coordinate c is
+  // (|y_c| as fp16 bits, 127 - c, sign): unique, ordered by magnitude first,
+  // then lower index first.  Keys 4q .. 4q + 3 of half r of vector v sit at
+  // 16-byte slot 256 q + 2 v + r: each lane's later reload of its 64 keys is
+  // a conflict-free 512-byte run per warp.
   if (!mbar_wait(done, 0, kTcWaitNs)) {
     atomicOr(p.status, kStatusTimeout);
     failed = 1;
   }
   tc_fence_after();
-  uint4* keys_s = reinterpret_cast<uint4*>(smem_tc + (ta - raw)) + threadIdx.x;
+  uint4* keys_s = reinterpret_cast<uint4*>(smem_tc + (ta - raw));
   {
-    const uint32_t taddr = tmem + ((uint32_t)(32 * warp) << 16);
+    const int row = 32 * (warp & 3) + lane, half = warp >> 2;
+    const uint32_t taddr = tmem + ((uint32_t)(32 * (warp & 3)) << 16) + 64 * half;
 #pragma unroll 1
-    for (int c = 0; c < 4; ++c) {
+    for (int c = 0; c < 2; ++c) {
       uint32_t hi[32], lo[32];
       tmem_ld32(taddr + c * 32, hi);
       tmem_ld32(taddr + 128 + c * 32, lo);
@@ -410,11 +463,11 @@ __global__ void __launch_bounds__(kTcThreads, 1) append_tc_kernel(const __grid_c
           const float y1 = fmaf(__uint_as_float(lo[m + 1]), 1.f / 4096.f, __uint_as_float(hi[m + 1]));
           const __half2 y2 = __floats2half2_rn(y0, y1);
           const uint32_t h2 = *reinterpret_cast<const uint32_t*>(&y2);
-          const uint32_t j = (uint32_t)(32 * c + m);
+          const uint32_t j = (uint32_t)(64 * half + 32 * c + m);
           k[e] = ((h2 & 0x7fffu) << 16) | ((127u - j) << 1) | ((h2 >> 15) & 1u);
           k[e + 1] = (h2 & 0x7fff0000u) | ((126u - j) << 1) | (h2 >> 31);
         }
-        keys_s[128 * (8 * c + q)] = make_uint4(k[0], k[1], k[2], k[3]);
+        keys_s[256 * (8 * c + q) + 2 * row + half] = make_uint4(k[0], k[1], k[2], k[3]);
       }
     }
   }
@@ -423,54 +476,58 @@ __global__ void __launch_bounds__(kTcThreads, 1) append_tc_kernel(const __grid_c
   if (warp == 1) tmem_dealloc(tmem, 256);
   if (failed != 0) return;  // uniform in the CTA
 
-  // ---- ring insert or prune of vector v
-  const int v = threadIdx.x, j = j0 + v;
-  if (j >= rv.n_new) return;
-  uint32_t key[128];
+  // ---- lanes 2v, 2v+1: vector v (coordinates 64 r .. 64 r + 63 in a[])
+  const int v = threadIdx.x >> 1, j = j0 + v;
+  const uint32_t r = threadIdx.x & 1u;
+  uint32_t a[64];
 #pragma unroll
-  for (int q = 0; q < 32; ++q) {
-    const uint4 k4 = keys_s[128 * q];
-    key[4 * q] = k4.x;
-    key[4 * q + 1] = k4.y;
-    key[4 * q + 2] = k4.z;
-    key[4 * q + 3] = k4.w;
+  for (int q = 0; q < 16; ++q) {
+    const uint4 k4 = keys_s[256 * q + threadIdx.x];
+    a[4 * q] = k4.x;
+    a[4 * q + 1] = k4.y;
+    a[4 * q + 2] = k4.z;
+    a[4 * q + 3] = k4.w;
   }
   const int64_t unit = (int64_t)b * p.H + h;
   const int64_t pos = (int64_t)rv.n_b + j;
-  if (pos >= rv.evict) {
+  const bool live = j < rv.n_new;  // the same for both lanes of a pair
+  if (live && pos >= rv.evict) {
     const int slot = (int)((rv.buf_start + pos) % p.cap);
-    uint4* row = reinterpret_cast<uint4*>((kind ? p.ring_v : p.ring_k) + (unit * p.cap + slot) * kHeadDim);
+    uint4* row = reinterpret_cast<uint4*>((kind ? p.ring_v : p.ring_k) + (unit * p.cap + slot) * kHeadDim) + 8 * (int)r;
 #pragma unroll
-    for (int q = 0; q < 16; ++q)
-      row[q] = make_uint4(key_bits2(key[8 * q], key[8 * q + 1]), key_bits2(key[8 * q + 2], key[8 * q + 3]),
-                          key_bits2(key[8 * q + 4], key[8 * q + 5]), key_bits2(key[8 * q + 6], key[8 * q + 7]));
-    return;
+    for (int q = 0; q < 8; ++q)
+      row[q] = make_uint4(key_bits2(a[8 * q], a[8 * q + 1]), key_bits2(a[8 * q + 2], a[8 * q + 3]),
+                          key_bits2(a[8 * q + 4], a[8 * q + 5]), key_bits2(a[8 * q + 6], a[8 * q + 7]));
   }
+  const bool prune = live && pos < rv.evict;
+  if (!__any_sync(0xffffffffu, prune)) return;  // the pair exchanges below need the whole warp
+
   const CacheGeom& g = p.geom;
   const int64_t sp = rv.sparse_len + pos;
   const int64_t page = sp / g.P;
   const int slot = (int)(sp % g.P);
-  if (page >= g.pages_per_unit) {
-    atomicOr(p.status, kStatusPageRange);
-    return;
+  int32_t phys = -1;
+  if (prune) {
+    if (page < g.pages_per_unit) phys = g.page_table[unit * g.pages_per_unit + page];
+    if (phys < 0 || phys >= g.num_pages) {
+      if (r == 0) atomicOr(p.status, kStatusPageRange);
+      phys = -1;
+    }
   }
-  const int32_t phys = g.page_table[unit * g.pages_per_unit + page];
-  if (phys < 0 || phys >= g.num_pages) {
-    atomicOr(p.status, kStatusPageRange);
-    return;
-  }
-  uint8_t* blk = g.pool + (int64_t)phys * g.page_bytes + (int64_t)(slot >> 5) * g.block_bytes();
+  uint8_t* blk = g.pool + (int64_t)max(phys, 0) * g.page_bytes + (int64_t)(slot >> 5) * g.block_bytes();
   const bool fp8 = g.fmt == kFmtFp8;
   const int slots = kind ? g.k_slots_v : g.k_slots;
   const int kept = kind ? g.k_store_v : g.k_store;
   uint8_t* vals = blk + (kind ? g.vval_off() : 0);
   uint8_t* idx = blk + (kind ? g.vidx_off() : g.kidx_off());
-  if (slots <= 64) {
-    sortnet::top64_of128_desc(key);
-    store_sorted<8>(key, slots, kept, vals, idx, slot & 31, fp8);
+  sortnet::sort_oe<0, 64, true>(a, one);
+  if (slots <= 64) {  // uniform in the CTA
+    uint32_t c[32];
+    pair_top64(a, c, r, one);
+    if (phys >= 0) store_sorted<32>(c, 32 * (int)r, slots, kept, vals, idx, slot & 31, fp8);
   } else {
-    sortnet::sort128_desc_full(key);
-    store_sorted<16>(key, slots, kept, vals, idx, slot & 31, fp8);
+    pair_sort128(a, r, one);
+    if (phys >= 0) store_sorted<64>(a, 64 * (int)r, slots, kept, vals, idx, slot & 31, fp8);
   }
 }
 
@@ -502,8 +559,9 @@ cudaError_t launch_append_tc(const AppendParams& p, const CUtensorMap* maps, int
   cudaError_t e = ensure_smem<append_tc_kernel>(kTcSmem);
   if (e != cudaSuccess) return e;
   const int tiles = p.B * ((p.T + 127) / 128);
+  // the sorting networks' multiply-adds take their factor 1 at run time
   return launch_pdl(append_tc_kernel, dim3((unsigned)tiles, (unsigned)p.H, 2), dim3(kTcThreads), kTcSmem, s,
-                    maps[0], maps[1], maps[2], maps[3], p, r_slice0);
+                    maps[0], maps[1], maps[2], maps[3], p, r_slice0, 1u);
 }
 
 cudaError_t launch_split_r(const float* R_qk, const float* R_vo, __half* hi, __half* lo, int layers, int H,

@@ -11,11 +11,13 @@
 
 #include "sortnet.cuh"
 
+static uint32_t g_one = 1;
+
 static int check(const std::vector<uint32_t>& keys, const char* what) {
   uint32_t full[128], top[128];
   for (int i = 0; i < 128; ++i) full[i] = top[i] = keys[i];
-  swan::sortnet::sort128_desc_full(full);
-  swan::sortnet::top64_of128_desc(top);
+  swan::sortnet::sort128_desc_full(full, g_one);
+  swan::sortnet::top64_of128_desc(top, g_one);
   std::vector<uint32_t> want(keys);
   std::sort(want.begin(), want.end(), std::greater<uint32_t>());
   for (int i = 0; i < 128; ++i) {
@@ -33,6 +35,7 @@ static int check(const std::vector<uint32_t>& keys, const char* what) {
 
 int main(int argc, char** argv) {
   const int trials = argc > 1 ? std::atoi(argv[1]) : 20000;
+  if (argc > 2) g_one = (uint32_t)std::atoi(argv[2]);  // the run-time 1 of the multiply-adds
   std::mt19937_64 gen(20251124);
   std::vector<uint32_t> keys(128);
   // structured cases: sorted, reversed, one large key at each position

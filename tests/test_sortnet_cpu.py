@@ -1,6 +1,9 @@
 """The register sorting networks of the bulk append (csrc/sortnet.cuh),
 compiled as host C++ and run on random and structured sets of 128 distinct
-keys: the full sort and the top-64 selection must equal std::sort's order."""
+keys: the full sort and the top-64 selection must equal std::sort's order.
+The networks take the smaller key of some compare-exchanges as (a + b) - max
+by multiply-adds with a factor 1 given at run time; a factor of 3 must make the
+check fail."""
 from __future__ import annotations
 
 import os
@@ -20,6 +23,10 @@ def test_sorting_networks_match_std_sort(tmp_path):
     exe = str(tmp_path / "sortnet_check")
     subprocess.run([cxx, "-O1", "-std=c++17", "-I", CSRC, os.path.join(HERE, "native", "sortnet_check.cpp"),
                     "-o", exe], check=True)
-    r = subprocess.run([exe, "5000"], stdout=subprocess.PIPE, stderr=subprocess.STDOUT, text=True)
+    r = subprocess.run([exe, "5000", "1"], stdout=subprocess.PIPE, stderr=subprocess.STDOUT, text=True)
     assert r.returncode == 0, r.stdout
     assert r.stdout.strip() == "ok 5000"
+    # the multiply-add form of the smaller key is exercised: a factor other
+    # than 1 breaks the order, and the check must see it
+    bad = subprocess.run([exe, "50", "3"], stdout=subprocess.PIPE, stderr=subprocess.STDOUT, text=True)
+    assert bad.returncode == 1, bad.stdout

@@ -12,7 +12,7 @@ import pytest
 
 import oracle
 from paper_2511_18936_gb300 import synth
-from tests.helpers import TOL_OUT
+from tests.helpers import TOL_OUT, check_topk_near_ties
 
 pytestmark = pytest.mark.gpu
 
@@ -114,7 +114,8 @@ def test_stack_32_layers_prefix_and_flush_schedule_sampled():
     """32 layers, batch 8, 8192-token prefix compressed by one append per
     layer, then 256 decode steps appending one token per layer with every
     buffer flushed after each 128 steps; sampled (layer, step, unit) outputs
-    against an oracle replay of the same op log."""
+    against an oracle replay of the same op log, and the sampled units'
+    packed caches after the prefix against the fp64 rotation."""
     import torch
 
     from paper_2511_18936_gb300 import swan
@@ -140,6 +141,12 @@ def test_stack_32_layers_prefix_and_flush_schedule_sampled():
                 st.append(kk[b:b + 1, h:h + 1].cpu().numpy(), vv[b:b + 1, h:h + 1].cpu().numpy())
                 st.flush()
                 refs[(l, b, h)] = st
+                # the packed cache the bulk append left, against the fp64
+                # rotation of the same vectors (near-ties allowed)
+                for which, x in (("k", kk), ("v", vv)):
+                    gi, gv = ctx.export_sparse_seq(l, b, which)
+                    y64 = x[b, h].cpu().numpy().astype(np.float64) @ R[l, h].astype(np.float64)
+                    check_topk_near_ties(y64, gi[h], gv[h], k)
         del kk, vv
     knh, vnh, qsh = kn.cpu().numpy(), vn.cpu().numpy(), qs.cpu().numpy()
     outs = torch.empty((Lyr, B, H, D), dtype=torch.float16, device=dev)

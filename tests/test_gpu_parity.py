@@ -67,6 +67,37 @@ def test_prune_bitexact_on_identical_rotated_inputs(k_store, cap, P):
     ctx.close()
 
 
+@pytest.mark.parametrize("k_store,k_store_v,fmt,cap", [(64, 64, "fp16", 5), (128, 40, "fp16", 0),
+                                                      (40, 128, "fp8_e4m3", 16), (8, 64, "fp8_e4m3", 3),
+                                                      (65, 63, "fp16", 7)])
+def test_bulk_prune_bitexact_on_tricky_vectors(k_store, k_store_v, fmt, cap):
+    """The bulk append (batch x T > 256 vectors: tensor-core rotation, register
+    sorting networks, two lanes per vector) on vectors with many exact
+    magnitude ties, +-0, all-equal magnitudes and values beyond the E4M3
+    range, in every tile of the append including the ragged last one; keep
+    counts on both sides of 64 (the top-half and the full-sort paths) and not
+    multiples of 8 (padded chunks)."""
+    B, H, T = 2, 3, 300
+    eye = np.broadcast_to(np.eye(D, dtype=np.float32), (H, D, D)).copy()
+    R = _rot(H, 7)
+    kraw, vraw = _kv(B, H, T, seed=8)
+    k16 = oracle.to_fp16(np.einsum("bhti,hij->bhtj", kraw.astype(np.float64), R.astype(np.float64)))
+    v16 = oracle.to_fp16(np.einsum("bhti,hij->bhtj", vraw.astype(np.float64), R.astype(np.float64)))
+    for i, (b, h, t0) in enumerate([(0, 0, 0), (1, 2, 130), (0, 1, 260), (1, 0, 90)]):
+        k16[b, h, t0:t0 + 40] = _tricky_vectors(40, 20 + i)
+        v16[b, (h + 1) % H, t0:t0 + 40] = _tricky_vectors(40, 30 + i) * np.float16(20)
+    ops = [("append", k16, v16), ("flush",)]
+    ctx, ref, _ = run_ops(ops, eye, None, B=B, H_kv=H, G=1, k_store=k_store, cap=cap, value_format=fmt,
+                          k_store_v=k_store_v)
+    for which, ri, rv in (("k", ref.sp_idx_k, ref.sp_val_k), ("v", ref.sp_idx_v, ref.sp_val_v)):
+        gi, gv = ctx.export_sparse(0, which)
+        assert np.array_equal(gi, ri), which
+        assert np.array_equal(gv.view(np.uint16), rv.view(np.uint16)), which
+    ctx.check()
+    ctx.check_guards()
+    ctx.close()
+
+
 def test_buffer_contents_bitexact_on_identical_inputs():
     B, H = 1, 2
     eye = np.broadcast_to(np.eye(D, dtype=np.float32), (H, D, D)).copy()

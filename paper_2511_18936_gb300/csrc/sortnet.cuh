@@ -8,6 +8,11 @@
 //                         given v[0..64) decreasing and v[64..128) increasing
 //   merge_desc<LO, N>     bitonic merge of the bitonic run v[LO .. LO+N) into
 //                         decreasing order
+//   top64_of128_desc,     the same top-64 and full sort of 128 keys in one
+//   sort128_desc_full     thread.  The bulk append splits a vector over a lane
+//                         pair instead (append.cu), built from sort_oe and
+//                         merge_desc; the host test checks these one-thread
+//                         forms, and with them those building blocks.
 //
 // A compare-exchange takes the larger key with one max.  The smaller is
 // either one min or, for three comparators in five, (a + b) - max: exact in

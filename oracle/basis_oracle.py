@@ -31,7 +31,8 @@ Readings where the paper is silent (each listed in the design notes):
   set that the pruned vectors keep), not a mean of per-vector shares.
 
 Parity status: every function below is pinned in ``tests/oracle_pins.py``
-(planted singular vectors, the Ky Fan maximum property, planted per-group
+(planted singular vectors, the Ky Fan maximum property, the Gram matrix of
+planted factors and by brute force over rows, planted per-group
 subspaces for both joint matrices, brute-force top-k energy on d = 8).
 """
 from __future__ import annotations

@@ -340,13 +340,38 @@ def pin_basis_ky_fan_maximum(b):
     gen = np.random.default_rng(102)
     S = gen.standard_normal((200, 12)) * np.linspace(3.0, 0.2, 12)[None, :] @ synth.random_orthogonal(12, gen)
     P, _ = b.principal_basis(S)
-    lam = np.sort(np.linalg.eigvalsh(S.T @ S))[::-1]
+    lam = np.sort(np.linalg.eigvalsh(b.gram(S)))[::-1]
     kept = np.cumsum(np.sum((S @ P) ** 2, axis=0))
     assert np.allclose(kept, np.cumsum(lam), rtol=1e-10)
     for _ in range(20):
         Qr = synth.random_orthogonal(12, gen)
         other = np.cumsum(np.sum((S @ Qr) ** 2, axis=0))
         assert (other <= kept * (1 + 1e-12)).all()
+
+
+def pin_gram_planted_factors(b):
+    """gram(S) is S^T S, whose eigenvectors are SVD(S)_V (Section 4.1.2):
+    for S = U diag(sigma) W^T with orthonormal U, W it equals
+    W diag(sigma^2) W^T, and for any S it is the sum over the rows s_r of the
+    outer products s_r^T s_r (brute force, every row counted once)."""
+    gen = np.random.default_rng(106)
+    d, m = 12, 40
+    W = synth.random_orthogonal(d, gen)
+    U = _orthonormal_columns(m, d, gen)
+    sigma = np.linspace(3.0, 0.25, d)
+    G = b.gram(U @ np.diag(sigma) @ W.T)
+    assert G.shape == (d, d)
+    assert np.allclose(G, W @ np.diag(sigma ** 2) @ W.T, atol=1e-12)
+    S = gen.standard_normal((7, 5)) * np.array([1.0, 2.0, 0.5, 4.0, 1.5])
+    S[0] *= 9.0                       # a dropped first or last row shows
+    S[-1] *= 7.0
+    brute = np.zeros((5, 5))
+    for r in range(S.shape[0]):
+        for i in range(5):
+            for j in range(5):
+                brute[i, j] += S[r, i] * S[r, j]
+    assert np.allclose(b.gram(S), brute, atol=1e-12)
+    assert b.gram(S).dtype == np.float64
 
 
 def _planted_groups(gen, n_kv, G, n, d, d_model, r):
@@ -417,8 +442,8 @@ def pin_energy_planted_rank(b):
     assert b.energy_curve(X, synth.random_orthogonal(d, gen))[r] < 0.99 * np.sum(X * X)
 
 
-BASIS_PINS = [pin_basis_recovers_planted_svd, pin_basis_ky_fan_maximum, pin_joint_matrices_group_heads,
-              pin_energy_curve_bruteforce, pin_energy_planted_rank]
+BASIS_PINS = [pin_basis_recovers_planted_svd, pin_basis_ky_fan_maximum, pin_gram_planted_factors,
+              pin_joint_matrices_group_heads, pin_energy_curve_bruteforce, pin_energy_planted_rank]
 
 
 def pin_ragged_rows_are_independent(o):

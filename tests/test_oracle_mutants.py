@@ -86,6 +86,10 @@ BASIS_MUTANTS = [
     ("vo_slice_rows_not_columns", "parts.append(W_O[h * d:(h + 1) * d, :].T)",
      "parts.append(W_O[h * d:(h + 1) * d, :d].T)", 1),
     ("vo_values_dropped", "parts = [V[j]]", "parts = [0 * V[j]]", 1),
+    ("gram_transposed", "return S.T @ S", "return S @ S.T", 1),
+    ("gram_drops_first_row", "return S.T @ S", "return S[1:].T @ S[1:]", 1),
+    ("gram_drops_last_row", "return S.T @ S", "return S[:-1].T @ S[:-1]", 1),
+    ("gram_diagonal_only", "return S.T @ S", "return np.diag(np.sum(S * S, axis=0))", 1),
     ("energy_smallest_first", "sq = np.sort(Y * Y, axis=1)[:, ::-1]", "sq = np.sort(Y * Y, axis=1)", 1),
     ("energy_unsquared", "sq = np.sort(Y * Y, axis=1)[:, ::-1]", "sq = np.sort(np.abs(Y), axis=1)[:, ::-1]", 1),
     ("energy_unrotated", "Y = np.asarray(X, np.float64) @ np.asarray(P, np.float64)",

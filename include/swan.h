@@ -332,13 +332,19 @@ swan_status swan_timing_read(swan_ctx* ctx, swan_timing* out);
  * batch * n_q_heads <= 1024 and (decode CTAs + batch * n_kv_heads) * G <=
  * 2048, where decode CTAs is at most (SM count x resident CTAs per SM; 152 on
  * a GB300).  Larger sizes return SWAN_ERR_INVALID_ARG with a message.
+ * Alignment: pages, buf_k, buf_v, R_qk and R_vo_t 16 bytes, q 8 bytes,
+ * page_table 4 bytes, out 2 bytes (the kernels' widest accesses); a
+ * misaligned pointer returns SWAN_ERR_INVALID_ARG before anything is enqueued.
  * The first call on a device resolves the scratch address and the grid limits
  * (cudaGetSymbolAddress, occupancy queries); make that first call before any
- * stream capture.  Every call on a device shares the one scratch array, which
- * keeps the last call's contents: calls that overlap on the GPU (different
- * streams, or different host threads) race and give wrong results; serialise
- * them.  Device-side consistency checks are recorded in the scratch and not
- * reported.  Errors: INVALID_ARG, UNSUPPORTED, CUDA.
+ * stream capture.  The address is resolved again if the device's context is
+ * re-created (cudaDeviceReset).  Every call on a device shares the one scratch
+ * array, which keeps the last call's contents: calls that overlap on the GPU
+ * (different streams, or different host threads) race and give wrong
+ * results; serialise them.  Device-side consistency checks (a page-table
+ * entry out of range, a kernel skipped for too little shared memory) are
+ * recorded in a status word of the scratch that each call clears first;
+ * swan_noalloc_check reads it.  Errors: INVALID_ARG, UNSUPPORTED, CUDA.
  */
 typedef struct swan_cache_view {
   const void* pages;
@@ -367,6 +373,15 @@ typedef struct swan_cache_view {
 swan_status swan_decode_noalloc(const swan_cache_view* view, const void* q, void* out,
                                 void* stream);
 
+/*
+ * Status of the last swan_decode_noalloc on the current device: synchronises
+ * `stream` (the one that call used), reads the scratch's status word and
+ * clears it.  Allocates nothing.  Returns OK, DEVICE_CHECK (the last call's
+ * output is not valid: a page-table entry out of range or a kernel skipped),
+ * DEVICE_TIMEOUT, or CUDA.
+ */
+swan_status swan_noalloc_check(void* stream);
+
 /* Number of kernels this context has launched since swan_init. */
 int64_t swan_launch_count(const swan_ctx* ctx);
 
@@ -388,6 +403,22 @@ int64_t swan_launch_count(const swan_ctx* ctx);
 enum { SWAN_FAULT_ALLOC = 1, SWAN_FAULT_LAUNCH = 2 };
 swan_status swan_debug_fail_after(int kind, int64_t n);
 swan_status swan_debug_check_guards(swan_ctx* ctx);
+
+/*
+ * Test hook for the bounded device waits of the tensor-core kernels (the
+ * bulk append of swan_append, and swan_gram of swan_basis.h): the next such
+ * launch in the process issues none of its TMA copies, so the barrier its
+ * MMA thread waits on is never completed; that wait, and every other barrier
+ * wait of the launch, gives up after limit_ns nanoseconds (instead of 2 s),
+ * sets the timeout bit of the status word and the kernel returns, with no
+ * copy or MMA left in flight and its tensor memory freed.  swan_check (or
+ * swan_basis_check) then returns SWAN_ERR_DEVICE_TIMEOUT.  The starved
+ * launch's results are invalid: for an append, the context's cache no longer
+ * matches its host-side lengths and the context should be destroyed.  Fires
+ * once; limit_ns = 0 disarms it.  Not for concurrent use.
+ * Errors: INVALID_ARG unless limit_ns == 0 or 1e3 <= limit_ns <= 2e9.
+ */
+swan_status swan_debug_starve_tc(int64_t limit_ns);
 
 /* Static string for a status code. */
 const char* swan_status_string(swan_status s);

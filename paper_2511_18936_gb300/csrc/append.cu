@@ -399,19 +399,22 @@ __global__ void __launch_bounds__(kTcThreads, 2) append_tc_kernel(const __grid_c
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = tmem_slot;
+  const uint64_t wait_ns = p.tc_wait_ns ? p.tc_wait_ns : kTcWaitNs;
   pdl_wait();
 
   if (threadIdx.x == 0) {
     const CUtensorMap* xm = kind ? &xv : &xk;
     const int slice = r_slice0 + kind * p.H + h;
-    mbar_arrive_expect_tx(full, 3 * kTcTile);
-    tma_load_4d(ta, xm, full, 0, j0, h, b);
-    tma_load_4d(ta + kTcTile / 2, xm, full, 64, j0, h, b);
-    tma_load_3d(tb_hi, &rhi, full, 0, 0, slice);
-    tma_load_3d(tb_hi + kTcTile / 2, &rhi, full, 64, 0, slice);
-    tma_load_3d(tb_lo, &rlo, full, 0, 0, slice);
-    tma_load_3d(tb_lo + kTcTile / 2, &rlo, full, 64, 0, slice);
-    if (!mbar_wait(full, 0, kTcWaitNs)) {
+    if (!p.tc_starve) {  // starved (test hook): nothing arrives on `full`
+      mbar_arrive_expect_tx(full, 3 * kTcTile);
+      tma_load_4d(ta, xm, full, 0, j0, h, b);
+      tma_load_4d(ta + kTcTile / 2, xm, full, 64, j0, h, b);
+      tma_load_3d(tb_hi, &rhi, full, 0, 0, slice);
+      tma_load_3d(tb_hi + kTcTile / 2, &rhi, full, 64, 0, slice);
+      tma_load_3d(tb_lo, &rlo, full, 0, 0, slice);
+      tma_load_3d(tb_lo + kTcTile / 2, &rlo, full, 64, 0, slice);
+    }
+    if (!mbar_wait(full, 0, wait_ns)) {
       atomicOr(p.status, kStatusTimeout);
       failed = 1;
     } else {
@@ -436,7 +439,7 @@ __global__ void __launch_bounds__(kTcThreads, 2) append_tc_kernel(const __grid_c
   // then lower index first.  Keys 4q .. 4q + 3 of half r of vector v sit at
   // 16-byte slot 256 q + 2 v + r: each lane's later reload of its 64 keys is
   // a conflict-free 512-byte run per warp.
-  if (!mbar_wait(done, 0, kTcWaitNs)) {
+  if (!mbar_wait(done, 0, wait_ns)) {
     atomicOr(p.status, kStatusTimeout);
     failed = 1;
   }

@@ -64,13 +64,14 @@ __global__ void __launch_bounds__(128, 1) gram_kernel(const __grid_constant__ CU
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = tmem_base_slot;
+  const uint64_t wait_ns = p.wait_ns ? p.wait_ns : kWaitLimitNs;
 
-  if (warp == 0 && lane == 0 && n > 0) {
+  if (warp == 0 && lane == 0 && n > 0 && !p.starve) {
     // ---- producer
     int issued = 0;
     for (int i = 0; i < n; ++i) {
       const int s = i % kGramStages, round = i / kGramStages;
-      if (round > 0 && !mbar_wait(empty0 + 8 * s, (round - 1) & 1, kWaitLimitNs)) {
+      if (round > 0 && !mbar_wait(empty0 + 8 * s, (round - 1) & 1, wait_ns)) {
         atomicOr(p.status, kBasisStatusTimeout);
         abort_flag = 1;
         break;
@@ -99,14 +100,14 @@ __global__ void __launch_bounds__(128, 1) gram_kernel(const __grid_constant__ CU
     }
     // copies still in flight must land before the CTA can exit
     for (int i = max(0, issued - kGramStages); i < issued; ++i)
-      mbar_wait(full0 + 8 * (i % kGramStages), (i / kGramStages) & 1, kWaitLimitNs);
+      mbar_wait(full0 + 8 * (i % kGramStages), (i / kGramStages) & 1, wait_ns);
   } else if (warp == 1 && lane == 0 && n > 0) {
     // ---- MMA issuer
     constexpr uint32_t idesc = idesc_f16_f32(128, 128, kMnMajor ? 1 : 0, kMnMajor ? 1 : 0);
     bool ok = true;
     for (int i = 0; i < n && ok; ++i) {
       const int s = i % kGramStages, round = i / kGramStages;
-      if (!mbar_wait(full0 + 8 * s, round & 1, kWaitLimitNs)) {
+      if (!mbar_wait(full0 + 8 * s, round & 1, wait_ns)) {
         atomicOr(p.status, kBasisStatusTimeout);
         abort_flag = 1;
         ok = false;
@@ -130,7 +131,7 @@ __global__ void __launch_bounds__(128, 1) gram_kernel(const __grid_constant__ CU
   // ---- epilogue: TMEM row (32 warp + lane) -> partial row
   const int row = 32 * warp + lane;
   float* dst = p.partials + (((size_t)m * p.splits + split) * 128 + row) * 128;
-  if (n > 0 && !mbar_wait(done, 0, kWaitLimitNs)) {
+  if (n > 0 && !mbar_wait(done, 0, wait_ns)) {
     atomicOr(p.status, kBasisStatusTimeout);
     abort_flag = 1;
   }

@@ -165,6 +165,10 @@ swan_status swan_gram(const swan_vectors* x, float* gram, int accumulate, void* 
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   cudaError_t e = cudaMemsetAsync(p.status, 0, sizeof(uint32_t), s);
   if (e != cudaSuccess) return cuda_err(e, "cudaMemsetAsync");
+  if (const int64_t starve_ns = take_tc_starve()) {
+    p.starve = 1;
+    p.wait_ns = (uint64_t)starve_ns;
+  }
   e = launch_gram(map, p, rows, s);
   if (e != cudaSuccess) return cuda_err(e, "gram kernel launch");
   e = launch_gram_reduce(p.partials, gram, p.n_mats, p.splits, accumulate, s);

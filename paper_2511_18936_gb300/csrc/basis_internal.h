@@ -20,6 +20,10 @@ struct GramParams {
   uint32_t* status;
   int n_mats, splits, group;
   int64_t chunks;    // 64-position chunks per (matrix, group member)
+  // test hook (swan_debug_starve_tc): no copies are issued, so the MMA
+  // warp's barrier wait runs out after wait_ns (0: the default 2 s)
+  int starve;
+  uint64_t wait_ns;
 };
 
 struct EigParams {

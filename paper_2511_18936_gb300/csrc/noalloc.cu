@@ -33,12 +33,45 @@ __device__ __align__(256) float
 constexpr int kMaxDevices = 64;
 struct DeviceSetup {
   bool ready = false;
-  float* scratch = nullptr;  // device address of g_noalloc_scratch
+  unsigned long long ctx_id = 0;  // driver context the address belongs to
+  float* scratch = nullptr;       // device address of g_noalloc_scratch
   int sms = 0;
   int ctas_per_sm[3][2] = {};  // [G = 1, 2, 4][k_slots <= 64, > 64]
 };
 DeviceSetup g_setup[kMaxDevices];
 std::mutex g_setup_mutex;
+
+// The current driver context's unique id (cuCtxGetId; 0 if the driver
+// cannot say).  The static array's device address belongs to the module
+// loaded in one context: after cudaDeviceReset the primary context, and
+// with it the module and the array, are created anew, so the address is
+// resolved again whenever the id changes.
+using CtxGetCurrentFn = CUresult (*)(CUcontext*);
+using CtxGetIdFn = CUresult (*)(CUcontext, unsigned long long*);
+unsigned long long current_ctx_id() {
+  static CtxGetCurrentFn get_current = nullptr;
+  static CtxGetIdFn get_id = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess && q == cudaDriverEntryPointSuccess)
+      get_current = reinterpret_cast<CtxGetCurrentFn>(p);
+    p = nullptr;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetId", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      get_id = reinterpret_cast<CtxGetIdFn>(p);
+  });
+  if (!get_current || !get_id) return 0;
+  CUcontext c = nullptr;
+  unsigned long long id = 0;
+  if (get_current(&c) != CUDA_SUCCESS || !c || get_id(c, &id) != CUDA_SUCCESS) return 0;
+  return id;
+}
+
+// Byte alignment the kernels' widest access to a pointer needs.
+bool aligned(const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) & (a - 1)) == 0; }
 
 thread_local char g_err[256];
 
@@ -50,15 +83,20 @@ swan_status err(swan_status s, const char* msg) {
 
 int gi(int G) { return G == 1 ? 0 : G == 2 ? 1 : 2; }
 
-// Once per device, with that device current: resolve the device address of
-// the static scratch array and the decode grid limits.
+// Once per device (and again if the device's context was re-created), with
+// that device current: resolve the device address of the static scratch
+// array and the decode grid limits.
 swan_status setup_device(int dev, DeviceSetup** out) {
   if (dev < 0 || dev >= kMaxDevices) return err(SWAN_ERR_UNSUPPORTED, "device index out of range");
   std::lock_guard<std::mutex> lock(g_setup_mutex);
   DeviceSetup& s = g_setup[dev];
-  if (!s.ready) {
+  // id 0: no context is current yet, or the driver cannot name it; resolve
+  // again (cheap host calls) rather than trust a cached address
+  const unsigned long long id = current_ctx_id();
+  if (!s.ready || id == 0 || s.ctx_id != id) {
+    s.ready = false;
     void* p = nullptr;
-    cudaError_t e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+    cudaError_t e = cudaGetSymbolAddress(&p, g_noalloc_scratch);  // also makes the context current
     if (e != cudaSuccess || p == nullptr) return err(SWAN_ERR_CUDA, "cudaGetSymbolAddress failed");
     e = cudaDeviceGetAttribute(&s.sms, cudaDevAttrMultiProcessorCount, dev);
     if (e != cudaSuccess) return err(SWAN_ERR_CUDA, "cudaDeviceGetAttribute failed");
@@ -69,6 +107,7 @@ swan_status setup_device(int dev, DeviceSetup** out) {
         if (s.ctas_per_sm[g][big] < 1) return err(SWAN_ERR_CUDA, "decode kernel occupancy query failed");
       }
     s.scratch = static_cast<float*>(p);
+    s.ctx_id = current_ctx_id();
     s.ready = true;
   }
   *out = &s;
@@ -110,6 +149,13 @@ extern "C" swan_status swan_decode_noalloc(const swan_cache_view* v, const void*
   if (!v->R_qk || !v->R_vo_t) return err(SWAN_ERR_INVALID_ARG, "NULL rotation matrix");
   if (v->value_format != SWAN_VALUES_FP16 && v->value_format != SWAN_VALUES_FP8_E4M3)
     return err(SWAN_ERR_INVALID_ARG, "value_format must be fp16 (0) or fp8 e4m3 (1)");
+  // the kernels read pages, buffers and R with 16-byte loads, q with 8-byte
+  // loads, and write out as fp16: a misaligned address would fault the context
+  if ((v->sparse_len > 0 && (!aligned(v->pages, 16) || !aligned(v->page_table, 4))) ||
+      (v->buf_len > 0 && (!aligned(v->buf_k, 16) || !aligned(v->buf_v, 16))) || !aligned(v->R_qk, 16) ||
+      !aligned(v->R_vo_t, 16) || !aligned(q, 8) || !aligned(out, 2))
+    return err(SWAN_ERR_INVALID_ARG,
+               "misaligned pointer (pages, buf_k, buf_v, R_qk, R_vo_t: 16 bytes; q: 8; page_table: 4; out: 2)");
   const int fmt = v->value_format == SWAN_VALUES_FP8_E4M3 ? kFmtFp8 : kFmtFp16;
   const int64_t nq = (int64_t)v->batch * v->n_q_heads;
   if (nq > kNoallocMaxQ) return err(SWAN_ERR_INVALID_ARG, "batch * n_q_heads exceeds 1024 (static scratch)");
@@ -175,6 +221,7 @@ extern "C" swan_status swan_decode_noalloc(const swan_cache_view* v, const void*
     p.N_g = N_g;
     p.total_groups = total;
     p.visit_cost = decode_visit_cost(G, false);
+    p.B = v->batch;
     p.H_kv = v->n_kv_heads;
     p.H_q = v->n_q_heads;
     p.blocks_per_page_log2 = __builtin_ctz((unsigned)(v->page_tokens / 32));
@@ -198,4 +245,27 @@ extern "C" swan_status swan_decode_noalloc(const swan_cache_view* v, const void*
   cp.H_q = v->n_q_heads;
   if (launch_combine(cp, v->batch, s) != cudaSuccess) return err(SWAN_ERR_CUDA, "combine launch failed");
   return SWAN_OK;
+}
+
+extern "C" swan_status swan_noalloc_check(void* stream) {
+  set_last_error("");
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return err(SWAN_ERR_CUDA, "cudaGetDevice failed");
+  DeviceSetup* ds = nullptr;
+  swan_status st = setup_device(dev, &ds);
+  if (st != SWAN_OK) return st;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  unsigned* status = reinterpret_cast<unsigned*>(ds->scratch + kQFloats + kPartFloats + kCounterFloats);
+  unsigned word = 0;
+  if (cudaStreamSynchronize(s) != cudaSuccess) return err(SWAN_ERR_CUDA, "cudaStreamSynchronize failed");
+  if (cudaMemcpyAsync(&word, status, sizeof(word), cudaMemcpyDeviceToHost, s) != cudaSuccess ||
+      cudaStreamSynchronize(s) != cudaSuccess)
+    return err(SWAN_ERR_CUDA, "reading the status word failed");
+  if (!word) return SWAN_OK;
+  if (cudaMemsetAsync(status, 0, sizeof(unsigned), s) != cudaSuccess ||
+      cudaStreamSynchronize(s) != cudaSuccess)
+    return err(SWAN_ERR_CUDA, "clearing the status word failed");
+  char msg[96];
+  snprintf(msg, sizeof(msg), "device status word 0x%x of the last call", word);
+  return err(word & kStatusTimeout ? SWAN_ERR_DEVICE_TIMEOUT : SWAN_ERR_DEVICE_CHECK, msg);
 }

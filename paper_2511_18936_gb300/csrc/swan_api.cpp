@@ -426,6 +426,15 @@ std::vector<int> buffer_counts(const LayerState& L) {
 
 void swan::set_last_error(const char* msg) { g_last_error = msg ? msg : ""; }
 
+namespace swan {
+namespace {
+std::atomic<int64_t> g_tc_starve{0};
+}  // namespace
+int64_t take_tc_starve() {
+  return g_tc_starve.load(std::memory_order_relaxed) ? g_tc_starve.exchange(0) : 0;
+}
+}  // namespace swan
+
 extern "C" {
 
 const char* swan_status_string(swan_status s) {
@@ -783,9 +792,14 @@ swan_status append_rows(swan_ctx* c, int layer, const void* k_new, const void* v
   if (small)
     s = launch(c, SWAN_KERNEL_APPEND, rq ? "append_rotate kernel" : "append_small kernel",
                [&] { return launch_append_small(p, most_old, rq, c->stream); });
-  else
+  else {
+    if (const int64_t starve_ns = take_tc_starve()) {
+      p.tc_starve = 1;
+      p.tc_wait_ns = (uint64_t)starve_ns;
+    }
     s = launch(c, SWAN_KERNEL_APPEND, "append kernel",
                [&] { return launch_append_tc(p, maps, layer * 2 * c->cfg.n_kv_heads, c->stream); });
+  }
   if (s != SWAN_OK) return s;
   if (rotated) *rotated = small && rq != nullptr;
 
@@ -1197,6 +1211,13 @@ swan_status swan_debug_fail_after(int kind, int64_t n) {
   if (kind == SWAN_FAULT_ALLOC) g_fail_alloc.store(n);
   else if (kind == SWAN_FAULT_LAUNCH) g_fail_launch.store(n);
   else return fail(SWAN_ERR_INVALID_ARG, "unknown fault kind %d", kind);
+  return SWAN_OK;
+}
+
+swan_status swan_debug_starve_tc(int64_t limit_ns) {
+  if (limit_ns != 0 && (limit_ns < 1000 || limit_ns > 2000000000))
+    return fail(SWAN_ERR_INVALID_ARG, "limit_ns = %lld outside [1e3, 2e9]", (long long)limit_ns);
+  g_tc_starve.store(limit_ns);
   return SWAN_OK;
 }
 

@@ -114,6 +114,10 @@ struct AppendParams {
   const SeqInfo* seq;   // per-row state instead of the four scalars above, or null
   CacheGeom geom;
   unsigned* status;
+  // test hook (swan_debug_starve_tc): the bulk-append kernel issues no
+  // copies, so its barrier wait runs out after tc_wait_ns (0: the default 2 s)
+  int tc_starve;
+  uint64_t tc_wait_ns;
 };
 
 // Prune `count` buffered tokens (logical positions 0..count-1) per unit from
@@ -313,5 +317,9 @@ inline int64_t decode_visit_cost(int G, bool ragged) {
 }
 // Record the detail string that swan_last_error() returns on this thread.
 void set_last_error(const char* msg);
+// Test hook armed by swan_debug_starve_tc: the wait limit in nanoseconds for
+// the next tensor-core launch, which then issues no copies (0: not armed).
+// Disarms it.
+int64_t take_tc_starve();
 
 }  // namespace swan

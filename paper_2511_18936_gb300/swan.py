@@ -33,7 +33,7 @@ EXPORTED = ["swan_init", "swan_destroy", "swan_set_k", "swan_append", "swan_flus
             "swan_gram_workspace_bytes", "swan_gram", "swan_basis_eig", "swan_energy",
             "swan_basis_check", "swan_append_varlen", "swan_reset_sequence", "swan_query_lengths",
             "swan_debug_export_seq", "swan_append_decode", "swan_debug_fail_after",
-            "swan_debug_check_guards"]
+            "swan_debug_check_guards", "swan_noalloc_check", "swan_debug_starve_tc"]
 
 
 class SwanConfig(ctypes.Structure):
@@ -119,6 +119,8 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "swan_status_string": (ctypes.c_char_p, [i]),
         "swan_last_error": (ctypes.c_char_p, []),
         "swan_decode_noalloc": (i, [ctypes.POINTER(CacheView), vp, vp, vp]),
+        "swan_noalloc_check": (i, [vp]),
+        "swan_debug_starve_tc": (i, [i64]),
         "swan_gram_workspace_bytes": (ctypes.c_size_t, [i]),
         "swan_gram": (i, [ctypes.POINTER(SwanVectors), vp, i, vp, ctypes.c_size_t, vp]),
         "swan_basis_eig": (i, [vp, i, vp, vp, vp, vp]),
@@ -329,6 +331,12 @@ def debug_fail_after(kind: int, n: int):
     _check(load_library().swan_debug_fail_after(int(kind), int(n)), "swan_debug_fail_after")
 
 
+def debug_starve_tc(limit_ns: int):
+    """Test hook: the next tensor-core launch issues no copies and its
+    barrier waits give up after ``limit_ns`` (``swan_debug_starve_tc``)."""
+    _check(load_library().swan_debug_starve_tc(int(limit_ns)), "swan_debug_starve_tc")
+
+
 def decode_noalloc(view: CacheView, q, out, stream=None):
     """One decode step over a caller-owned cache with no device allocation
     (``swan_decode_noalloc``); ``stream``: a ``torch.cuda.Stream`` or None for
@@ -340,6 +348,15 @@ def decode_noalloc(view: CacheView, q, out, stream=None):
     _check(lib.swan_decode_noalloc(ctypes.byref(view), _ptr(q), _ptr(out),
                                    ctypes.c_void_p(stream.cuda_stream)), "swan_decode_noalloc")
     return out
+
+
+def noalloc_check(stream=None):
+    """Raise SwanError if the last ``decode_noalloc`` on this device set its
+    device status word (``swan_noalloc_check``; synchronises ``stream``)."""
+    import torch
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    _check(load_library().swan_noalloc_check(ctypes.c_void_p(stream.cuda_stream)), "swan_noalloc_check")
 
 
 # ---------------------------------------------------------------------------

@@ -131,3 +131,72 @@ def test_guards_hold_across_paths():
         ctx.check()
         ctx.check_guards()
         ctx.close()
+
+
+def test_bulk_append_wait_runs_out_and_reports_timeout():
+    """A bounded barrier wait of the tensor-core bulk append runs out: with
+    swan_debug_starve_tc the next such launch issues no copies, so its MMA
+    thread's wait on the tile barrier (armed, but with no producer) gives up
+    after 1 ms.  Nothing is left in flight; swan_check reports
+    DEVICE_TIMEOUT, and a fresh context on the same device then appends and
+    decodes correctly."""
+    import time
+
+    import torch
+
+    from paper_2511_18936_gb300 import swan
+    dev = torch.device("cuda")
+    ctx = _ctx(H=2)
+    k = torch.from_numpy(synth.lowrank_kv(2, 2, 300, D, 6, 97, 3, synth.T_K)).to(dev)
+    v = torch.from_numpy(synth.lowrank_kv(2, 2, 300, D, 6, 97, 3, synth.T_V)).to(dev)
+    torch.cuda.synchronize()
+    swan.debug_starve_tc(1_000_000)
+    try:
+        t0 = time.perf_counter()
+        ctx.append(0, k, v)              # 600 vectors: the tensor-core path
+        with pytest.raises(swan.SwanError) as e:
+            ctx.check()
+        elapsed = time.perf_counter() - t0
+    finally:
+        swan.debug_starve_tc(0)
+    assert e.value.status == swan.ERR_DEVICE_TIMEOUT, e.value
+    assert elapsed < 1.5, elapsed        # the 1 ms limit, not the default 2 s
+    ctx.check()                          # the word was cleared; nothing else fired
+    ctx.close()
+    kk = synth.lowrank_kv(2, 2, 300, D, 6, 97, 4, synth.T_K)
+    vv = synth.lowrank_kv(2, 2, 300, D, 6, 97, 4, synth.T_V)
+    qq = synth.gaussian_fp16((2, 2, D), 6, 97, 4, synth.T_Q)
+    R = synth.rotations(2, D, seed=6, workload=97, layer=4)
+    ctx2, _, outs = run_ops([("append", kk, vv), ("decode", qq)], R, None, B=2, H_kv=2, G=1, k_store=48, cap=16)
+    for got, want in outs:
+        assert np.abs(got - want).max() <= TOL_OUT
+    ctx2.close()
+
+
+def test_gram_wait_runs_out_and_reports_timeout():
+    """The same for the Gram kernel of the offline basis: starved, every CTA's
+    MMA thread gives up after 1 ms, swan_basis_check reports DEVICE_TIMEOUT
+    (and clears it), and the next accumulation is correct again."""
+    import torch
+
+    from paper_2511_18936_gb300 import swan
+    n_kv, G, n = 2, 2, 700
+    Q, K, _, _ = synth.calibration(n_kv, G, n, D, 64, seed=9, workload=60, layer=0)
+    dev = torch.device("cuda")
+    tq, tk = torch.from_numpy(Q).to(dev), torch.from_numpy(K).to(dev)
+    g = swan.Gram(n_kv)
+    swan.debug_starve_tc(1_000_000)
+    try:
+        g.add(swan.rows_of(tq, G), accumulate=False)
+        with pytest.raises(swan.SwanError) as e:
+            g.check()
+    finally:
+        swan.debug_starve_tc(0)
+    assert e.value.status == swan.ERR_DEVICE_TIMEOUT, e.value
+    g.check()
+    g.add(swan.rows_of(tq, G), accumulate=False).add(swan.rows_of(tk))
+    g.check()
+    got = g.gram.double().cpu().numpy()
+    for j, S in enumerate(oracle.basis_oracle.joint_qk(Q, K, G)):
+        A = np.abs(S)
+        assert (np.abs(got[j] - oracle.basis_oracle.gram(S)) <= 2.0 ** -14 * (A.T @ A) + 1e-30).all(), j

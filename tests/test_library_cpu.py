@@ -169,3 +169,43 @@ def test_basis_workspace_and_pointer_checks(lib):
     assert lib.swan_basis_eig(ctypes.c_void_p(4096), 0, ctypes.c_void_p(4096), None, None,
                               None) == swan.ERR_INVALID_ARG
     assert lib.swan_basis_check(None, None) == swan.ERR_INVALID_ARG
+
+
+def _noalloc_view(**over):
+    """A well-formed no-allocation view over fake, aligned addresses (never
+    dereferenced: every case below fails host validation first)."""
+    base = dict(pages=0x10000, page_table=0x20000, num_pages=4, pages_per_unit=2, page_tokens=64,
+                k_slots=64, k_active=64, buf_k=0x30000, buf_v=0x40000, buffer_cap=16, buf_start=0,
+                buf_len=8, sparse_len=100, batch=1, n_q_heads=2, n_kv_heads=1, head_dim=128,
+                R_qk=0x50000, R_vo_t=0x60000, value_format=0, k_slots_v=0, k_active_v=0)
+    base.update(over)
+    return swan.CacheView(**base)
+
+
+@pytest.mark.parametrize("field,offset", [("pages", 8), ("page_table", 2), ("buf_k", 4), ("buf_v", 8),
+                                          ("R_qk", 4), ("R_vo_t", 8)])
+def test_noalloc_rejects_misaligned_view_pointers(lib, field, offset):
+    v = _noalloc_view()
+    setattr(v, field, getattr(v, field) + offset)
+    assert lib.swan_decode_noalloc(ctypes.byref(v), 0x70000, 0x80000, None) == swan.ERR_INVALID_ARG
+    assert b"misaligned" in lib.swan_last_error()
+
+
+def test_noalloc_rejects_misaligned_q_and_out_and_oversize(lib):
+    v = _noalloc_view()
+    assert lib.swan_decode_noalloc(ctypes.byref(v), 0x70002, 0x80000, None) == swan.ERR_INVALID_ARG
+    assert b"misaligned" in lib.swan_last_error()
+    assert lib.swan_decode_noalloc(ctypes.byref(v), 0x70000, 0x80001, None) == swan.ERR_INVALID_ARG
+    assert b"misaligned" in lib.swan_last_error()
+    big = _noalloc_view(batch=600)
+    assert lib.swan_decode_noalloc(ctypes.byref(big), 0x70000, 0x80000, None) == swan.ERR_INVALID_ARG
+    assert b"static scratch" in lib.swan_last_error()
+    assert lib.swan_decode_noalloc(None, 0x70000, 0x80000, None) == swan.ERR_INVALID_ARG
+
+
+def test_starve_hook_arguments(lib):
+    assert lib.swan_debug_starve_tc(-1) == swan.ERR_INVALID_ARG
+    assert lib.swan_debug_starve_tc(999) == swan.ERR_INVALID_ARG
+    assert lib.swan_debug_starve_tc(2_000_000_001) == swan.ERR_INVALID_ARG
+    assert lib.swan_debug_starve_tc(1_000_000) == swan.OK
+    assert lib.swan_debug_starve_tc(0) == swan.OK          # disarmed again

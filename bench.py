@@ -156,7 +156,7 @@ class ClockSampler:
 # CPU baseline: the oracle as it stands, on a bounded sample of the workload
 # ---------------------------------------------------------------------------
 
-def oracle_sample(wl, n_units: int, seed: int = 0):
+def oracle_sample(wl, n_units: int, seed: int = 0, first_unit: int = 0):
     """Prepare the compressed state of ``n_units`` (batch, kv-head) units of
     the workload on the host (untimed) and return a step function that runs
     one oracle step (append one token, decode every query head of the unit)."""
@@ -167,7 +167,7 @@ def oracle_sample(wl, n_units: int, seed: int = 0):
     L = L_s + wl["n_b"]
     states = []
     compress_s = 0.0
-    for u in range(n_units):
+    for u in range(first_unit, first_unit + n_units):
         R = synth.rotations(1, D, seed=seed, workload=7, layer=0, tensor_id=synth.T_R_QK, )
         k = synth.lowrank_kv(1, 1, L + 64, D, seed, 7, u, synth.T_K)
         v = synth.lowrank_kv(1, 1, L + 64, D, seed, 7, u, synth.T_V)
@@ -200,6 +200,65 @@ def oracle_sample(wl, n_units: int, seed: int = 0):
     return step
 
 
+def host_cores() -> int:
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count() or 1
+
+
+def _oracle_worker(wl, unit, warmup, steps, budget_s, barrier, results):
+    """One host core: one (batch, kv-head) unit of the workload in the oracle
+    (single-threaded NumPy), prepared untimed; then, between two barriers
+    shared with every other core, `steps` oracle steps (or steps until
+    `budget_s` has passed)."""
+    step = oracle_sample(wl, 1, first_unit=unit)
+    for _ in range(warmup):
+        step()
+    tokens, n = 0, 0
+    barrier.wait()
+    t0 = time.perf_counter()
+    while (n < steps) if steps else (time.perf_counter() - t0 < budget_s):
+        tokens += step()
+        n += 1
+    barrier.wait()
+    results.put((tokens, n, step.compress["value"]))
+
+
+def oracle_all_cores(wl, warmup: int = 1, steps: int = 0, budget_s: float = 15.0):
+    """The oracle as it stands on every host core: one single-threaded oracle
+    process per core, each on its own (batch, kv-head) unit of the workload
+    (the units are independent), all timed together between two barriers.
+    Processes are started with `spawn` (safe after CUDA has been used)."""
+    import multiprocessing as mp
+    n = host_cores()
+    ctx = mp.get_context("spawn")
+    barrier = ctx.Barrier(n + 1)
+    results = ctx.Queue()
+    procs = [ctx.Process(target=_oracle_worker, args=(wl, u, warmup, steps, budget_s, barrier, results),
+                         daemon=True) for u in range(n)]
+    for p in procs:
+        p.start()
+    try:
+        barrier.wait(timeout=600)
+        t0 = time.perf_counter()
+        barrier.wait(timeout=600)
+        wall = time.perf_counter() - t0
+        got = [results.get(timeout=60) for _ in procs]
+    finally:
+        for p in procs:
+            p.join(timeout=30)
+            if p.is_alive():
+                p.terminate()
+    tokens = sum(g[0] for g in got)
+    return {"value": tokens / wall, "unit": "KV-tokens/s", "cores": n, "kind": "oracle",
+            "seconds": wall, "steps_per_core": [g[1] for g in got],
+            "compress_per_core": statistics.mean(g[2] for g in got),
+            "sample": f"{n} of {wl['B'] * wl['H_kv']} (batch, kv-head) units of the same workload "
+                      f"({wl['H_q'] // wl['H_kv']} query heads each), one single-threaded NumPy fp64 oracle "
+                      f"process per host core, each step append 1 token + decode, {wall:.1f} s"}
+
+
 def basis_oracle_step(wl, n_tokens: int, seed: int = 0):
     """One oracle step of the basis workload on a bounded sample: the joint
     matrices of one kv head over ``n_tokens`` tokens and their SVD basis.
@@ -221,6 +280,7 @@ def run_reference(args, wl, rank: int):
         return None
     if wl.get("kind") == "basis":
         return run_reference_basis(args, wl)
+    # one thread: two units stepped in turn
     n_units = min(2, wl["B"] * wl["H_kv"])
     t0 = time.perf_counter()
     step = oracle_sample(wl, n_units)
@@ -232,18 +292,25 @@ def run_reference(args, wl, rank: int):
         t = time.perf_counter()
         toks += step()
         times.append(time.perf_counter() - t)
-    total = sum(times)
-    value = toks / total
-    sample = (f"{n_units} of {wl['B'] * wl['H_kv']} (batch, kv-head) units of the workload, "
-              f"{wl['H_q'] // wl['H_kv']} query heads each; one step = append 1 token + decode; "
-              f"state preparation {prep:.1f} s outside the steps (its compress step: 'compress')")
+    total1 = sum(times)
+    single = {"value": toks / total1, "unit": "KV-tokens/s", "cores": 1, "kind": "oracle",
+              "ms_per_step": 1e3 * total1 / args.steps,
+              "sample": f"{n_units} of {wl['B'] * wl['H_kv']} (batch, kv-head) units of the workload, "
+                        f"{wl['H_q'] // wl['H_kv']} query heads each, one thread; one step = append 1 token + "
+                        f"decode; state preparation {prep:.1f} s outside the steps"}
+    # every host core: one unit per core, all stepped at once (the line's value)
+    allc = oracle_all_cores(wl, warmup=args.warmup, steps=args.steps)
+    value = allc["value"]
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "KV-tokens/s",
             "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
-            "ms_per_step": 1e3 * total / args.steps, "higher_is_better": True,
+            "ms_per_step": 1e3 * allc["seconds"] / args.steps, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": {"workload": args.workload, "desc": wl["desc"], "parallelism": "none (host CPU)"},
-            "cpu_baseline": {"value": value, "unit": "KV-tokens/s", "cores": 1, "kind": "oracle",
-                             "sample": sample},
+            "config": {"workload": args.workload, "desc": wl["desc"],
+                       "parallelism": f"host CPU, {allc['cores']} cores (one oracle process per core)"},
+            "cpu_baseline": {"value": value, "unit": "KV-tokens/s", "cores": allc["cores"], "kind": "oracle",
+                             "sample": allc["sample"] + f"; {args.steps} steps per core after {args.warmup} "
+                                                        "untimed"},
+            "single_thread": single,
             "e2e": {"value": value, "unit": "KV-tokens/s", "h2d_bytes_per_step": 0,
                     "d2h_bytes_per_step": 0},
             "compress": step.compress}
@@ -428,6 +495,7 @@ def run_basis(args, wl, rank: int, world: int, local_rank: int):
 
 
 def cpu_baseline_leg(wl, budget_s: float = 15.0):
+    """The oracle on every host core (the reported figure) and on one thread."""
     step = oracle_sample(wl, 1)
     step()
     t0 = time.perf_counter()
@@ -436,11 +504,15 @@ def cpu_baseline_leg(wl, budget_s: float = 15.0):
         toks += step()
         n += 1
     dt = time.perf_counter() - t0
-    return {"value": toks / dt, "unit": "KV-tokens/s", "cores": 1, "kind": "oracle",
-            "sample": f"1 of {wl['B'] * wl['H_kv']} (batch, kv-head) units of the same workload "
-                      f"({wl['H_q'] // wl['H_kv']} query heads), {n} steps of append 1 token + decode, "
-                      f"{dt:.1f} s, NumPy fp64 single thread",
-            "compress": step.compress}
+    single = {"value": toks / dt, "unit": "KV-tokens/s", "cores": 1, "kind": "oracle",
+              "sample": f"1 of {wl['B'] * wl['H_kv']} (batch, kv-head) units of the same workload "
+                        f"({wl['H_q'] // wl['H_kv']} query heads), {n} steps of append 1 token + decode, "
+                        f"{dt:.1f} s, NumPy fp64 single thread",
+              "compress": step.compress}
+    line = oracle_all_cores(wl, budget_s=budget_s)
+    line["single_thread"] = single
+    line["compress"] = step.compress
+    return line
 
 
 # ---------------------------------------------------------------------------
@@ -829,19 +901,102 @@ def run_swan(args, wl, rank: int, world: int, local_rank: int):
     return line
 
 
-def _keep_counts(ap, args, wl):
-    """Value keep counts of the decode workloads from the command line."""
-    wl["k_store_v"] = args.k_store_v or wl["k_store"]
+# Every other configuration of the benchmark, run after the headline line in
+# the default invocation (one GPU) with bounded steps: (label, workload,
+# make_workload overrides).  The k sweep re-prunes one k_store 128 cache at
+# each runtime keep count.
+SUB_WORKLOADS = [
+    ("latency-1k", "latency-1k", {}),
+    ("gqa-131k", "gqa-131k", {}),
+    ("gqa-131k-e4m3", "gqa-131k", {"values": "fp8_e4m3"}),
+    ("llama2-7b-layer-32k-e4m3", "llama2-7b-layer-32k", {"values": "fp8_e4m3"}),
+    ("llama2-7b-layer-32k-kv64-32", "llama2-7b-layer-32k", {"k_store_v": 32}),
+    *[(f"ksweep-32k-k{k}", "ksweep-32k", {"k_active": k}) for k in (32, 48, 64, 96, 128)],
+    ("ragged-serve-32", "ragged-serve-32", {}),
+    ("stack-32x8k", "stack-32x8k", {}),
+    ("basis-llama3-8b", "basis-llama3-8b", {}),
+]
+
+
+def summarize(line):
+    """The per-workload figures of a bench line (for the workloads object)."""
+    rf = line["roofline"]
+    out = {"desc": line["config"]["desc"], "value": line["value"], "unit": line["unit"],
+           "ms_per_step": line["ms_per_step"], "steps": line["steps"], "warmup": line["warmup"],
+           "gpu_launches": line["gpu_launches"], "e2e": line["e2e"], "clocks": line["clocks"],
+           "l2": line["config"].get("l2"),
+           "roofline": {k: rf.get(k) for k in ("kernel", "bound", "achieved", "peak", "unit", "frac", "pct_of_8tbs",
+                                               "alg_bytes_per_launch", "avg_launch_ms", "traffic",
+                                               "tensor_tflops") if k in rf}}
+    if "alg_bytes_per_launch" in rf and rf.get("pct_of_8tbs") is not None and "L2 flushed" not in out["l2"]:
+        # the time the decode launch would take at 70 % of the nominal 8 TB/s
+        out["launch_ms_at_70pct_of_8tbs"] = rf["alg_bytes_per_launch"] / (0.7 * NOMINAL_HBM_GBS * 1e9) * 1e3
+    for key in ("prefill_ms", "prefill_tokens_per_s", "prefix_ms", "prefix_tokens_per_s", "eig_ms_16_matrices"):
+        if key in line:
+            out[key] = line[key]
+    return out
+
+
+def run_workloads(args, rank: int, world: int, local_rank: int):
+    """Run every configuration of SUB_WORKLOADS with bounded steps; a failure
+    is recorded (and the others still run)."""
+    import argparse as _ap
+    import gc
+
+    import torch
+    res = {}
+    for label, name, over in SUB_WORKLOADS:
+        sub = _ap.Namespace(**vars(args))
+        sub.workload = name
+        sub.warmup = 3
+        sub.steps = 20 if name == "latency-1k" else 10
+        sub.e2e_steps = 5
+        try:
+            wl = make_workload(name, **over)
+            line = (run_basis if wl.get("kind") == "basis" else run_swan)(sub, wl, rank, world, local_rank)
+            res[label] = summarize(line)
+        except Exception as e:  # noqa: BLE001 - recorded in the line, the rest still runs
+            res[label] = {"error": f"{type(e).__name__}: {e}"[:300]}
+        gc.collect()
+        torch.cuda.empty_cache()
+    return res
+
+
+def make_workload(name: str, values: str = "fp16", batch: int = 0, k_active: int = 0, tokens: int = 0,
+                  k_store_v: int = 0, k_active_v: int = 0):
+    """The workload dict of ``name`` with the command line's overrides
+    applied (ValueError on an out-of-range keep count)."""
+    wl = dict(WORKLOADS[name])
+    wl["values"] = values
+    if values != "fp16":
+        wl["desc"] += f" ({values} values)"
+    if batch:
+        wl["B"] = batch
+        wl["desc"] += f" (batch overridden to {batch})"
+    if k_active:
+        if not 1 <= k_active <= wl["k_store"]:
+            raise ValueError(f"--k-active must be in [1, {wl['k_store']}]")
+        wl["k"] = k_active
+        wl["desc"] += f" (k_active {k_active})"
+    if wl.get("kind") == "basis":
+        wl["k_store_v"] = wl["k_v"] = None
+        if tokens:
+            wl["n"] = tokens
+            wl["desc"] += f" (tokens per batch overridden to {tokens})"
+        return wl
+    # value keep counts of the decode workloads
+    wl["k_store_v"] = k_store_v or wl["k_store"]
     if not 1 <= wl["k_store_v"] <= D:
-        ap.error(f"--k-store-v must be in [1, {D}]")
-    if args.k_store_v:
+        raise ValueError(f"--k-store-v must be in [1, {D}]")
+    if k_store_v:
         wl["desc"] += f" (k_store_v {wl['k_store_v']})"
     wl["k_v"] = min(wl["k"], wl["k_store_v"])
-    if args.k_active_v:
-        if not 1 <= args.k_active_v <= wl["k_store_v"]:
-            ap.error(f"--k-active-v must be in [1, {wl['k_store_v']}]")
-        wl["k_v"] = args.k_active_v
-        wl["desc"] += f" (k_active_v {args.k_active_v})"
+    if k_active_v:
+        if not 1 <= k_active_v <= wl["k_store_v"]:
+            raise ValueError(f"--k-active-v must be in [1, {wl['k_store_v']}]")
+        wl["k_v"] = k_active_v
+        wl["desc"] += f" (k_active_v {k_active_v})"
+    return wl
 
 
 def main():
@@ -854,6 +1009,8 @@ def main():
     ap.add_argument("--e2e-steps", type=int, default=20)
     ap.add_argument("--seed", type=int, default=0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-workloads", action="store_true",
+                    help="skip the other configurations the default run adds as 'workloads'")
     ap.add_argument("--batch", type=int, default=0,
                     help="override the workload's batch (smaller cases for profiling)")
     ap.add_argument("--values", default="fp16", choices=["fp16", "fp8_e4m3"],
@@ -869,25 +1026,11 @@ def main():
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
-    wl = dict(WORKLOADS[args.workload])
-    wl["values"] = args.values
-    if args.values != "fp16":
-        wl["desc"] += f" ({args.values} values)"
-    if args.batch:
-        wl["B"] = args.batch
-        wl["desc"] += f" (batch overridden to {args.batch})"
-    if args.k_active:
-        if not 1 <= args.k_active <= wl["k_store"]:
-            ap.error(f"--k-active must be in [1, {wl['k_store']}]")
-        wl["k"] = args.k_active
-        wl["desc"] += f" (k_active {args.k_active})"
-    if wl.get("kind") == "basis":
-        wl["k_store_v"] = wl["k_v"] = None
-        if args.tokens:
-            wl["n"] = args.tokens
-            wl["desc"] += f" (tokens per batch overridden to {args.tokens})"
-    else:
-        _keep_counts(ap, args, wl)
+    try:
+        wl = make_workload(args.workload, args.values, args.batch, args.k_active, args.tokens, args.k_store_v,
+                           args.k_active_v)
+    except ValueError as e:
+        ap.error(str(e))
 
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
@@ -904,6 +1047,9 @@ def main():
         torch.distributed.init_process_group("nccl")
     basis = wl.get("kind") == "basis"
     line = (run_basis if basis else run_swan)(args, wl, rank, world, local_rank)
+    if world == 1 and not args.no_workloads and args.workload == "llama2-7b-layer-32k" and \
+            wl["desc"] == WORKLOADS[args.workload]["desc"]:
+        line["workloads"] = run_workloads(args, rank, world, local_rank)
     if rank == 0:
         if not args.no_cpu_baseline and world == 1:
             line["cpu_baseline"] = cpu_baseline_basis(wl) if basis else cpu_baseline_leg(wl)

@@ -26,3 +26,6 @@ def test_reference_arm_line():
                         "d2h_bytes_per_step": 0}
     assert d["compress"]["unit"] == "token-heads/s" and d["compress"]["value"] > 0
     assert "1088 tokens" in d["compress"]["sample"]
+    # the value is the oracle on every host core; the one-thread figure beside it
+    assert d["cpu_baseline"]["cores"] == len(os.sched_getaffinity(0))
+    assert d["single_thread"]["cores"] == 1 and d["single_thread"]["value"] > 0

@@ -25,10 +25,10 @@ __global__ void __launch_bounds__(kHeadDim) combine_kernel(CombineParams p) {
 // one more 16 KB region for the alignment gap, which holds an 8 KB q' unless
 // the allocation starts within 8 KB below a 16 KB boundary; a 16 KB q' goes
 // after the accumulators.
-size_t one_head_smem(int maxc) {
-  const int nw = maxc <= 8 ? decode_warps<8>() : decode_warps<16>();
-  const int q_regions = (maxc <= 8 ? decode_q_shift<8>() : decode_q_shift<16>()) == 7 ? 1 : 0;
-  return (size_t)(nw + 1 + q_regions) * kRegionBytes;
+template <int MAXC>
+size_t one_head_smem() {
+  const int q_regions = decode_q_shift<MAXC>() == 7 ? 1 : 0;
+  return (size_t)(decode_warps<MAXC>() + 1 + q_regions) * kRegionBytes;
 }
 
 template <typename K>
@@ -43,7 +43,7 @@ int occupancy(K kernel, int threads, size_t smem) {
 template <int G, int MAXC, int FMT>
 cudaError_t launch_t(const DecodeParams& p, int grid, cudaStream_t s) {
   if constexpr (G == 1) {
-    const size_t smem = one_head_smem(MAXC);
+    const size_t smem = one_head_smem<MAXC>();
     const cudaError_t e = ensure_smem<decode_kernel<MAXC, FMT>>(smem);
     if (e != cudaSuccess) return e;
     return launch_pdl(decode_kernel<MAXC, FMT>, dim3(grid), dim3(decode_warps<MAXC>() * 32), smem, s, p);
@@ -63,11 +63,14 @@ cudaError_t launch_fmt(const DecodeParams& p, int grid, cudaStream_t s) {
 
 }  // namespace
 
-int decode_ctas_per_sm(int G, int k_slots) {
-  const bool big = k_slots > 64;
-  if (G == 1)
-    return big ? occupancy(decode_kernel<16, kFmtFp16>, decode_warps<16>() * 32, one_head_smem(16))
-               : occupancy(decode_kernel<8, kFmtFp16>, decode_warps<8>() * 32, one_head_smem(8));
+int decode_ctas_per_sm(int G, int k_read) {
+  const bool big = k_read > 64;
+  if (G == 1) {
+    if (k_read <= 64) return occupancy(decode_kernel<8, kFmtFp16>, decode_warps<8>() * 32, one_head_smem<8>());
+    if (k_read <= 96)
+      return occupancy(decode_kernel<12, kFmtFp16>, decode_warps<12>() * 32, one_head_smem<12>());
+    return occupancy(decode_kernel<16, kFmtFp16>, decode_warps<16>() * 32, one_head_smem<16>());
+  }
   if (G == 2)
     return big ? occupancy(decode_mma_kernel<2, 16, kFmtFp16>, mma_warps<16>() * 32, mma_smem<2, 16>())
                : occupancy(decode_mma_kernel<2, 8, kFmtFp16>, mma_warps<8>() * 32, mma_smem<2, 8>());
@@ -80,7 +83,9 @@ int decode_ctas_per_sm(int G, int k_slots) {
 cudaError_t launch_decode(const DecodeParams& p, int G, int k_read, int grid, cudaStream_t s) {
   const bool big = k_read > 64;
   switch (G) {
-    case 1: return big ? launch_fmt<1, 16>(p, grid, s) : launch_fmt<1, 8>(p, grid, s);
+    case 1:
+      return k_read <= 64 ? launch_fmt<1, 8>(p, grid, s)
+                          : k_read <= 96 ? launch_fmt<1, 12>(p, grid, s) : launch_fmt<1, 16>(p, grid, s);
     case 2: return big ? launch_fmt<2, 16>(p, grid, s) : launch_fmt<2, 8>(p, grid, s);
     case 4: return big ? launch_fmt<4, 16>(p, grid, s) : launch_fmt<4, 8>(p, grid, s);
     default: return cudaErrorInvalidValue;

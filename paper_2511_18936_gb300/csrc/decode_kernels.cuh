@@ -8,6 +8,8 @@
 
 #include <cuda_fp8.h>
 
+#include <type_traits>
+
 #include "swan_internal.h"
 
 namespace swan {
@@ -439,18 +441,27 @@ __device__ __forceinline__ void finish_unit(const DecodeParams& p, int64_t c0, i
   rotate_back_out<G, NT>(p, b, h, o_hat, scratch);
 }
 
+// Variants of the one-head kernel by the chunks read per vector (MAXC):
+//   8:  one slot of 8 chunks for keys and one for values;
+//   12: two slots, X (8 chunks) and Y (4), each loaded one phase ahead;
+//   16: one slot of 16 chunks each (the registers allow 8 warps).
+// The two-slot form keeps the 12-warp layout for up to 96 entries; at 128
+// it was slower than the 16-chunk slots (2.65 against 2.31 ms on the 32k
+// layer, while at 96 it took 1.72 against 1.99 ms).
+template <int MAXC>
+__host__ __device__ constexpr bool decode_two_slot() { return MAXC == 12; }
 // Warps per CTA of the one-head kernel: one lane-private accumulator each
 // (16 KB); for 16 chunks as many as the registers allow.
 template <int MAXC>
-__host__ __device__ constexpr int decode_warps() { return MAXC <= 8 ? 6 : 8; }
+__host__ __device__ constexpr int decode_warps() { return MAXC <= 12 ? 6 : 8; }
 // CTAs of the one-head kernel per SM (registers and shared memory allow two
 // of 6 warps; one CTA's barriers, merges and finishes then overlap the
 // other's streaming)
 template <int MAXC>
-__host__ __device__ constexpr int decode_min_ctas() { return MAXC <= 8 ? 2 : 1; }
+__host__ __device__ constexpr int decode_min_ctas() { return MAXC <= 12 ? 2 : 1; }
 // q' row shift of the one-head kernel (16 or 32 copies per coordinate)
 template <int MAXC>
-__host__ __device__ constexpr int decode_q_shift() { return MAXC <= 8 ? 6 : 7; }
+__host__ __device__ constexpr int decode_q_shift() { return MAXC <= 12 ? 6 : 7; }
 
 // Split decode kernel, one query head per kv head.
 //   The flat list of 32-token blocks of all units is cut into ranges of
@@ -469,6 +480,9 @@ __global__ void __launch_bounds__(decode_warps<MAXC>() * 32, decode_min_ctas<MAX
   constexpr int NW = decode_warps<MAXC>();
   constexpr int NT = NW * 32;
   constexpr int QS = decode_q_shift<MAXC>();
+  constexpr bool kTwoSlot = decode_two_slot<MAXC>();
+  constexpr int KS = kTwoSlot ? 8 : MAXC;  // chunks of slot X (kc: keys, then values)
+  constexpr int KY = MAXC - 8;             // chunks of slot Y (two-slot form)
   constexpr int QREP = (1 << QS) / 4;                       // copies per coordinate
   constexpr uint32_t kQBytes = kHeadDim << QS;              // 8 or 16 KB
   extern __shared__ __align__(16) unsigned char smem_dyn[];
@@ -589,11 +603,13 @@ __global__ void __launch_bounds__(decode_warps<MAXC>() * 32, decode_min_ctas<MAX
       }
     };
 
-    Chunk<FMT> kc[MAXC];
+    // key chunks 0 .. KS - 1 of the next block (two-slot form: the rest
+    // are loaded while these are scored)
+    Chunk<FMT> kc[KS];
     auto load_k = [&](const uint8_t* blk) {
       const uint8_t* src = blk ? blk : g.pool;
 #pragma unroll
-      for (int c = 0; c < MAXC; ++c)
+      for (int c = 0; c < KS; ++c)
         if (c < nchunks) kc[c] = load_chunk<FMT, false>(src + o_kv, src + o_ki, c);
     };
 
@@ -611,69 +627,111 @@ __global__ void __launch_bounds__(decode_warps<MAXC>() * 32, decode_min_ctas<MAX
         const bool valid = ok && t0 + lane < uv.sparse_len;
         const bool tail = !ok || t0 + 32 > uv.sparse_len;  // warp-uniform
         const uint8_t* src = ok ? b_cur : g.pool;
-        Chunk<FMT> vc[MAXC];
-#pragma unroll
-        for (int c = 0; c < MAXC; ++c)
-          if (c < nchunks_v) vc[c] = load_chunk<FMT, false>(src + o_vv, src + o_vi, c);
-        // two blocks ahead: into L2
-        const uint8_t* b_n2 = block_of(gi + 2);
-        prefetch_block(b_n2);
-
         float s[4] = {0.f, 0.f, 0.f, 0.f};
+        // scores of the key chunks c0 .. c0 + N - 1 held in cs[N]
+        auto score_slot = [&](const auto& cs, int c0) {
+          constexpr int N = std::extent<std::remove_reference_t<decltype(cs)>>::value;
 #pragma unroll
-        for (int c = 0; c < MAXC; ++c)
-          if (c < nchunks) {
-            float f[8];
-            chunk_vals<FMT>(kc[c], f);
-            uint2 ix = chunk_idx<FMT>(kc[c]);
-            if (krem && c == nchunks - 1) keep_first(f, krem);
-            if (tail && !valid) {
-              keep_first(f, 0);
-              ix = make_uint2(0, 0);
-            }
-            score_chunk<QS>(qb, f, ix, s);
-          }
-        s2 = valid ? ((s[0] + s[1]) + (s[2] + s[3])) * p.scale_log2 : -INFINITY;
-
-        // the next block's key records into registers while this block's
-        // values are accumulated
-        if (gi + 1 < sp_hi) load_k(b_n1);
-        b_cur = b_n1;
-        b_n1 = b_n2;
-
-        const float gmax = warp_max(s2);
-        if (gmax > m_w + kLazyRescale) {
-          if (m_w != -INFINITY) {
-            const float fs = exp2f(m_w - gmax);
-            l_sum *= fs;
-#pragma unroll 8
-            for (int dd = 0; dd < kHeadDim; ++dd) sts(ab + dd * 128, lds(ab + dd * 128) * fs);
-          }
-          m_w = gmax;
-        }
-        pr = valid ? exp2f(s2 - m_w) : 0.f;
-        l_sum += pr;
-
-#pragma unroll
-        for (int c = 0; c < MAXC; ++c)
-          if (c < kfull_v) {
-            float f[8];
-            chunk_vals<FMT>(vc[c], f);
-            uint2 ix = chunk_idx<FMT>(vc[c]);
-            if (tail && !valid) {
-              keep_first(f, 0);
-              ix = make_uint2(0, 0);
-            }
-            value_chunk(ab, pr, f, ix);
-          }
-        if (krem_v && valid) {
-#pragma unroll
-          for (int c = 0; c < MAXC; ++c)
-            if (c == kfull_v) {
+          for (int c = 0; c < N; ++c)
+            if (c0 + c < nchunks) {
               float f[8];
-              chunk_vals<FMT>(vc[c], f);
-              value_chunk_partial(ab, pr, f, chunk_idx<FMT>(vc[c]), krem_v);
+              chunk_vals<FMT>(cs[c], f);
+              uint2 ix = chunk_idx<FMT>(cs[c]);
+              if (krem && c0 + c == nchunks - 1) keep_first(f, krem);
+              if (tail && !valid) {
+                keep_first(f, 0);
+                ix = make_uint2(0, 0);
+              }
+              score_chunk<QS>(qb, f, ix, s);
             }
+        };
+        // key or value chunks c0 .. c0 + N - 1 of this block into cs[N]
+        auto load_slot = [&](auto& cs, int c0, int n, int o_val, int o_idx) {
+          constexpr int N = std::extent<std::remove_reference_t<decltype(cs)>>::value;
+#pragma unroll
+          for (int c = 0; c < N; ++c)
+            if (c0 + c < n) cs[c] = load_chunk<FMT, false>(src + o_val, src + o_idx, c0 + c);
+        };
+        // the online softmax step of this lane's token: returns its weight
+        auto softmax_step = [&]() -> float {
+          const float gmax = warp_max(s2);
+          if (gmax > m_w + kLazyRescale) {
+            if (m_w != -INFINITY) {
+              const float fs = exp2f(m_w - gmax);
+              l_sum *= fs;
+#pragma unroll 8
+              for (int dd = 0; dd < kHeadDim; ++dd) sts(ab + dd * 128, lds(ab + dd * 128) * fs);
+            }
+            m_w = gmax;
+          }
+          const float w = valid ? exp2f(s2 - m_w) : 0.f;
+          l_sum += w;
+          return w;
+        };
+        // acc[idx] += pr * val for the value chunks c0 .. c0 + N - 1 in cs[N]
+        auto value_slot = [&](const auto& cs, int c0) {
+          constexpr int N = std::extent<std::remove_reference_t<decltype(cs)>>::value;
+#pragma unroll
+          for (int c = 0; c < N; ++c)
+            if (c0 + c < kfull_v) {
+              float f[8];
+              chunk_vals<FMT>(cs[c], f);
+              uint2 ix = chunk_idx<FMT>(cs[c]);
+              if (tail && !valid) {
+                keep_first(f, 0);
+                ix = make_uint2(0, 0);
+              }
+              value_chunk(ab, pr, f, ix);
+            }
+          if (krem_v && valid) {
+#pragma unroll
+            for (int c = 0; c < N; ++c)
+              if (c0 + c == kfull_v) {
+                float f[8];
+                chunk_vals<FMT>(cs[c], f);
+                value_chunk_partial(ab, pr, f, chunk_idx<FMT>(cs[c]), krem_v);
+              }
+          }
+        };
+        if constexpr (!kTwoSlot) {
+          // the value records in flight while the keys (loaded during the
+          // previous block) are scored
+          Chunk<FMT> vc[KS];
+          load_slot(vc, 0, nchunks_v, o_vv, o_vi);
+          // two blocks ahead: into L2
+          const uint8_t* b_n2 = block_of(gi + 2);
+          prefetch_block(b_n2);
+          score_slot(kc, 0);
+          s2 = valid ? ((s[0] + s[1]) + (s[2] + s[3])) * p.scale_log2 : -INFINITY;
+          // the next block's key records into registers while this block's
+          // values are accumulated
+          if (gi + 1 < sp_hi) load_k(b_n1);
+          b_cur = b_n1;
+          b_n1 = b_n2;
+          pr = softmax_step();
+          value_slot(vc, 0);
+        } else {
+          // two register slots, X (kc, 8 chunks) and Y (KY chunks), each
+          // loaded one phase ahead of its use: key chunks 8.. into Y while
+          // keys 0..7 are scored, values 0..7 into X while keys 8.. are
+          // scored, values 8.. into Y during the softmax and values 0..7,
+          // the next block's keys 0..7 into X during values 8..
+          Chunk<FMT> cy[KY];
+          load_slot(cy, KS, nchunks, o_kv, o_ki);
+          const uint8_t* b_n2 = block_of(gi + 2);
+          prefetch_block(b_n2);
+          score_slot(kc, 0);
+          load_slot(kc, 0, nchunks_v, o_vv, o_vi);
+          score_slot(cy, KS);
+          load_slot(cy, KS, nchunks_v, o_vv, o_vi);
+          s2 = valid ? ((s[0] + s[1]) + (s[2] + s[3])) * p.scale_log2 : -INFINITY;
+          const uint8_t* b_next = b_n1;
+          b_cur = b_n1;
+          b_n1 = b_n2;
+          pr = softmax_step();
+          value_slot(kc, 0);
+          if (gi + 1 < sp_hi) load_k(b_next);
+          value_slot(cy, KS);
         }
       } else {
         // ---- buffer group: dense rotated fp16 vectors of the ring buffer

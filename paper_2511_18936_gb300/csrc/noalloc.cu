@@ -36,7 +36,7 @@ struct DeviceSetup {
   unsigned long long ctx_id = 0;  // driver context the address belongs to
   float* scratch = nullptr;       // device address of g_noalloc_scratch
   int sms = 0;
-  int ctas_per_sm[3][2] = {};  // [G = 1, 2, 4][k_slots <= 64, > 64]
+  int ctas_per_sm[3][3] = {};  // [G = 1, 2, 4][kernel variant: <= 64, <= 96, <= 128 entries read]
 };
 DeviceSetup g_setup[kMaxDevices];
 std::mutex g_setup_mutex;
@@ -102,9 +102,9 @@ swan_status setup_device(int dev, DeviceSetup** out) {
     if (e != cudaSuccess) return err(SWAN_ERR_CUDA, "cudaDeviceGetAttribute failed");
     const int gs[3] = {1, 2, 4};
     for (int g = 0; g < 3; ++g)
-      for (int big = 0; big < 2; ++big) {
-        s.ctas_per_sm[g][big] = decode_ctas_per_sm(gs[g], big ? 128 : 64);
-        if (s.ctas_per_sm[g][big] < 1) return err(SWAN_ERR_CUDA, "decode kernel occupancy query failed");
+      for (int v = 0; v < 3; ++v) {
+        s.ctas_per_sm[g][v] = decode_ctas_per_sm(gs[g], 64 + 32 * v);
+        if (s.ctas_per_sm[g][v] < 1) return err(SWAN_ERR_CUDA, "decode kernel occupancy query failed");
       }
     s.scratch = static_cast<float*>(p);
     s.ctx_id = current_ctx_id();
@@ -173,8 +173,9 @@ extern "C" swan_status swan_decode_noalloc(const swan_cache_view* v, const void*
   const int64_t total = units * N_g;
   int64_t grid = 0;
   if (total > 0)
-    grid = std::min<int64_t>((int64_t)ds->sms * ds->ctas_per_sm[gi(G)][std::max(v->k_active, kav) > 64],
-                             std::max<int64_t>(1, total / kMinGroupsPerCta));
+    grid = std::min<int64_t>(
+        (int64_t)ds->sms * ds->ctas_per_sm[gi(G)][decode_variant((std::max(v->k_active, kav) + 7) / 8 * 8)],
+        std::max<int64_t>(1, total / kMinGroupsPerCta));
   if ((grid + units) * G > kNoallocMaxSlots)
     return err(SWAN_ERR_INVALID_ARG, "(decode CTAs + batch * n_kv_heads) * G exceeds 2048 (static scratch)");
 

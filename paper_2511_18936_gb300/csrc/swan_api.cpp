@@ -79,7 +79,7 @@ struct swan_ctx {
   int device = 0;
   int num_sms = 0;
   int decode_ctas = 0;  // max decode CTAs resident at once (either kernel variant)
-  int decode_ctas_small = 0, decode_ctas_big = 0;  // for <= 64 and > 64 entries read
+  int decode_ctas_v[3] = {0, 0, 0};  // per kernel variant: <= 64, <= 96, <= 128 entries read
 
   float* R_qk = nullptr;
   float* R_vo = nullptr;   // == R_qk when the caller passed NULL
@@ -517,17 +517,22 @@ swan_status swan_init(swan_ctx** out, const swan_config* cfg, const float* R_qk,
   for (LayerState& L : c->layers) L.seq.assign(C.batch, SeqState{});
 
   // resident decode CTAs of the kernel variant each runtime keep count uses
-  const bool big_slots = std::max(c->k_slots, c->k_slots_v) > 64;
-  const int per_sm_small = decode_ctas_per_sm(G, 64);
-  const int per_sm_big = big_slots ? decode_ctas_per_sm(G, 128) : per_sm_small;
-  if (per_sm_small < 1 || per_sm_big < 1) {
-    delete c;
-    return fail(SWAN_ERR_CUDA, "decode kernel does not fit on an SM (%s)",
-                cudaGetErrorString(cudaGetLastError()));
+  const int slots = std::max(c->k_slots, c->k_slots_v);
+  for (int v = 0; v < 3; ++v) {
+    const int k_read = 64 + 32 * v;  // the largest keep count of the variant
+    if (v > 0 && slots <= k_read - 32) {
+      c->decode_ctas_v[v] = c->decode_ctas_v[v - 1];  // never launched: no larger count is stored
+      continue;
+    }
+    const int per_sm = decode_ctas_per_sm(G, k_read);
+    if (per_sm < 1) {
+      delete c;
+      return fail(SWAN_ERR_CUDA, "decode kernel does not fit on an SM (%s)",
+                  cudaGetErrorString(cudaGetLastError()));
+    }
+    c->decode_ctas_v[v] = per_sm * sms;
+    c->decode_ctas = std::max(c->decode_ctas, c->decode_ctas_v[v]);
   }
-  c->decode_ctas_small = per_sm_small * sms;
-  c->decode_ctas_big = per_sm_big * sms;
-  c->decode_ctas = std::max(c->decode_ctas_small, c->decode_ctas_big);
 
   const size_t rmat = (size_t)C.num_layers * C.n_kv_heads * kHeadDim * kHeadDim;
   const size_t ring_elems = (size_t)C.num_layers * ring_elems_per_layer(c);
@@ -910,7 +915,7 @@ swan_status decode_rotated(swan_ctx* c, int layer, void* out) {
   // entries read per vector, rounded up to 8: selects the kernel variant
   // and so how many of its CTAs fit at once
   const int k_read = (std::max(c->k_active, c->k_active_v) + 7) / 8 * 8;
-  const int64_t max_ctas = k_read > 64 ? c->decode_ctas_big : c->decode_ctas_small;
+  const int64_t max_ctas = c->decode_ctas_v[decode_variant(k_read)];
   const int64_t n_sg = (q0.sparse_len + 31) / 32;
   const int64_t n_bg = (q0.buf_count + 31) / 32;
   const int64_t N_g = n_sg + n_bg;

@@ -20,7 +20,7 @@ D = 128
 
 
 def _layer_case(B, H_q, H_kv, L_s, n_b, k_store, k_actives, samples, seed=0, steps=2,
-                value_format="fp16"):
+                value_format="fp16", q_scale=1.0):
     """Prefill L_s + n_b tokens, then `steps` decode steps (append one token +
     decode at every k in k_actives); compare sampled units with the oracle."""
     import torch
@@ -35,7 +35,7 @@ def _layer_case(B, H_q, H_kv, L_s, n_b, k_store, k_actives, samples, seed=0, ste
     kk = synth.torch_lowrank_kv(B, H_kv, L_s + n_b + steps, D, seed, synth.T_K, dev)
     vv = synth.torch_lowrank_kv(B, H_kv, L_s + n_b + steps, D, seed, synth.T_V, dev)
     ctx.append(0, kk[:, :, :L_s + n_b].contiguous(), vv[:, :, :L_s + n_b].contiguous())
-    qs = synth.torch_gaussian_fp16((steps, B, H_q, D), seed, synth.T_Q, dev)
+    qs = synth.torch_gaussian_fp16((steps, B, H_q, D), seed, synth.T_Q, dev, q_scale)
     refs = {}
     for b, h in samples:
         st = oracle.SwanOracle(R[h:h + 1], batch=1, n_q_heads=G, k_store=k_store, buffer_cap=n_b,
@@ -79,6 +79,14 @@ def test_llama2_layer_32k_fp8_values_sampled():
 def test_gqa_131k_sampled():
     _layer_case(B=4, H_q=32, H_kv=8, L_s=130944, n_b=128, k_store=56, k_actives=(56,),
                 samples=[(0, 0), (3, 7)])
+
+
+@pytest.mark.parametrize("fmt", ["fp16", "fp8_e4m3"])
+def test_gqa_131k_peaked_queries_sampled(fmt):
+    """Queries scaled by 4 (peaked softmax) on the 131k GQA layer: the
+    regime where the score precision (q' gathers) shows most."""
+    _layer_case(B=4, H_q=32, H_kv=8, L_s=130944, n_b=128, k_store=56, k_actives=(56,),
+                samples=[(1, 3)], seed=1, q_scale=4.0, value_format=fmt)
 
 
 def test_ksweep_32k_sampled_and_dense_at_k128():

@@ -176,6 +176,18 @@ __device__ __forceinline__ uint32_t addr_of(uint32_t w, uint32_t base) {
 // 2^QS bytes, aligned to their 128-row size: 16 copies (8 KB) where two CTAs
 // share an SM, 32 (16 KB, conflict-free) where one CTA has the SM.
 
+// Two fp32 fused multiply-adds in one instruction (d = a * b + c per half).
+__device__ __forceinline__ float2 ffma2(float2 a, float2 b, float2 c) {
+  unsigned long long ra, rb, rc, rd;
+  asm("mov.b64 %0, {%1,%2};" : "=l"(ra) : "f"(a.x), "f"(a.y));
+  asm("mov.b64 %0, {%1,%2};" : "=l"(rb) : "f"(b.x), "f"(b.y));
+  asm("mov.b64 %0, {%1,%2};" : "=l"(rc) : "f"(c.x), "f"(c.y));
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(rd) : "l"(ra), "l"(rb), "l"(rc));
+  float2 d;
+  asm("mov.b64 {%0,%1}, %2;" : "=f"(d.x), "=f"(d.y) : "l"(rd));
+  return d;
+}
+
 // Score contribution of one chunk into four partial sums.
 template <int QS>
 __device__ __forceinline__ void score_chunk(uint32_t qb, const float (&f)[8], uint2 ix, float (&s)[4]) {
@@ -184,14 +196,12 @@ __device__ __forceinline__ void score_chunk(uint32_t qb, const float (&f)[8], ui
   const float q2 = lds(addr_of<2, Q>(ix.x, qb)), q3 = lds(addr_of<3, Q>(ix.x, qb));
   const float q4 = lds(addr_of<0, Q>(ix.y, qb)), q5 = lds(addr_of<1, Q>(ix.y, qb));
   const float q6 = lds(addr_of<2, Q>(ix.y, qb)), q7 = lds(addr_of<3, Q>(ix.y, qb));
-  s[0] = fmaf(q0, f[0], s[0]);
-  s[1] = fmaf(q1, f[1], s[1]);
-  s[2] = fmaf(q2, f[2], s[2]);
-  s[3] = fmaf(q3, f[3], s[3]);
-  s[0] = fmaf(q4, f[4], s[0]);
-  s[1] = fmaf(q5, f[5], s[1]);
-  s[2] = fmaf(q6, f[6], s[2]);
-  s[3] = fmaf(q7, f[7], s[3]);
+  float2 s01 = make_float2(s[0], s[1]), s23 = make_float2(s[2], s[3]);
+  s01 = ffma2(make_float2(q0, q1), make_float2(f[0], f[1]), s01);
+  s23 = ffma2(make_float2(q2, q3), make_float2(f[2], f[3]), s23);
+  s01 = ffma2(make_float2(q4, q5), make_float2(f[4], f[5]), s01);
+  s23 = ffma2(make_float2(q6, q7), make_float2(f[6], f[7]), s23);
+  s[0] = s01.x, s[1] = s01.y, s[2] = s23.x, s[3] = s23.y;
 }
 
 // acc[idx_e] += p * val_e for one full chunk (distinct indices): eight loads,
@@ -203,14 +213,19 @@ __device__ __forceinline__ void value_chunk(uint32_t ab, float p, const float (&
   const uint32_t a6 = addr_of<2>(ix.y, ab), a7 = addr_of<3>(ix.y, ab);
   const float o0 = lds(a0), o1 = lds(a1), o2 = lds(a2), o3 = lds(a3);
   const float o4 = lds(a4), o5 = lds(a5), o6 = lds(a6), o7 = lds(a7);
-  sts(a0, fmaf(p, f[0], o0));
-  sts(a1, fmaf(p, f[1], o1));
-  sts(a2, fmaf(p, f[2], o2));
-  sts(a3, fmaf(p, f[3], o3));
-  sts(a4, fmaf(p, f[4], o4));
-  sts(a5, fmaf(p, f[5], o5));
-  sts(a6, fmaf(p, f[6], o6));
-  sts(a7, fmaf(p, f[7], o7));
+  const float2 pp = make_float2(p, p);
+  const float2 r01 = ffma2(pp, make_float2(f[0], f[1]), make_float2(o0, o1));
+  const float2 r23 = ffma2(pp, make_float2(f[2], f[3]), make_float2(o2, o3));
+  const float2 r45 = ffma2(pp, make_float2(f[4], f[5]), make_float2(o4, o5));
+  const float2 r67 = ffma2(pp, make_float2(f[6], f[7]), make_float2(o6, o7));
+  sts(a0, r01.x);
+  sts(a1, r01.y);
+  sts(a2, r23.x);
+  sts(a3, r23.y);
+  sts(a4, r45.x);
+  sts(a5, r45.y);
+  sts(a6, r67.x);
+  sts(a7, r67.y);
 }
 
 // The first `n` (< 8) entries of a chunk, one read-modify-write at a time
@@ -625,10 +640,12 @@ __global__ void __launch_bounds__(decode_warps<MAXC>() * 32, decode_min_ctas<MAX
         const int64_t t0 = (int64_t)gi * 32;
         const bool ok = b_cur != nullptr;
         const bool valid = ok && t0 + lane < uv.sparse_len;
-        const bool tail = !ok || t0 + 32 > uv.sparse_len;  // warp-uniform
         const uint8_t* src = ok ? b_cur : g.pool;
         float s[4] = {0.f, 0.f, 0.f, 0.f};
-        // scores of the key chunks c0 .. c0 + N - 1 held in cs[N]
+        // scores of the key chunks c0 .. c0 + N - 1 held in cs[N] (a lane
+        // past the end of the history scores its unwritten records: any
+        // index byte addresses inside q', and the score is replaced by
+        // -inf below)
         auto score_slot = [&](const auto& cs, int c0) {
           constexpr int N = std::extent<std::remove_reference_t<decltype(cs)>>::value;
 #pragma unroll
@@ -636,13 +653,8 @@ __global__ void __launch_bounds__(decode_warps<MAXC>() * 32, decode_min_ctas<MAX
             if (c0 + c < nchunks) {
               float f[8];
               chunk_vals<FMT>(cs[c], f);
-              uint2 ix = chunk_idx<FMT>(cs[c]);
               if (krem && c0 + c == nchunks - 1) keep_first(f, krem);
-              if (tail && !valid) {
-                keep_first(f, 0);
-                ix = make_uint2(0, 0);
-              }
-              score_chunk<QS>(qb, f, ix, s);
+              score_chunk<QS>(qb, f, chunk_idx<FMT>(cs[c]), s);
             }
         };
         // key or value chunks c0 .. c0 + N - 1 of this block into cs[N]
@@ -669,21 +681,19 @@ __global__ void __launch_bounds__(decode_warps<MAXC>() * 32, decode_min_ctas<MAX
           return w;
         };
         // acc[idx] += pr * val for the value chunks c0 .. c0 + N - 1 in cs[N]
+        // (lanes past the end of the history skip: their records are
+        // unwritten, and 0 * inf would not be 0)
         auto value_slot = [&](const auto& cs, int c0) {
           constexpr int N = std::extent<std::remove_reference_t<decltype(cs)>>::value;
+          if (!valid) return;
 #pragma unroll
           for (int c = 0; c < N; ++c)
             if (c0 + c < kfull_v) {
               float f[8];
               chunk_vals<FMT>(cs[c], f);
-              uint2 ix = chunk_idx<FMT>(cs[c]);
-              if (tail && !valid) {
-                keep_first(f, 0);
-                ix = make_uint2(0, 0);
-              }
-              value_chunk(ab, pr, f, ix);
+              value_chunk(ab, pr, f, chunk_idx<FMT>(cs[c]));
             }
-          if (krem_v && valid) {
+          if (krem_v) {
 #pragma unroll
             for (int c = 0; c < N; ++c)
               if (c0 + c == kfull_v) {

@@ -82,12 +82,12 @@ def measured_peaks():
 
 def decode_kernel_traffic(workload: str, values: str = "fp16", variant: str = ""):
     """DRAM bytes per decode-kernel launch from the committed ncu summary, if
-    it was taken on the current kernel source (else None)."""
-    src = os.path.join(ROOT, "paper_2511_18936_gb300", "csrc", "decode_kernels.cuh")
-    digest = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+    it was taken on the current kernel sources (every `<file> sha256[:16]`
+    line of the summary must match that file now; else None)."""
     text = None
     suffix = ("" if values == "fp16" else "-fp8") + variant
-    for name in (f"decode_kernel_{workload}{suffix}.md", f"decode_mma_kernel_{workload}{suffix}.md"):
+    for name in (f"decode_kernel_{workload}{suffix}.md", f"decode_ws_kernel_{workload}{suffix}.md",
+                 f"decode_mma_kernel_{workload}{suffix}.md"):
         try:
             text = open(os.path.join(ROOT, "profiles", name)).read()
             break
@@ -95,10 +95,18 @@ def decode_kernel_traffic(workload: str, values: str = "fp16", variant: str = ""
             continue
     if text is None:
         return None
-    m_src = re.search(r"decode_kernels\.cuh sha256\[:16\]:\s*([0-9a-f]{16})", text)
+    hashes = re.findall(r"([\w.]+\.cuh) sha256\[:16\]:\s*([0-9a-f]{16})", text)
     m_tr = re.search(r"dram bytes per launch:\s*([0-9.eE+]+)", text)
-    if not m_src or not m_tr or m_src.group(1) != digest:
+    if not hashes or not m_tr:
         return None
+    for fname, want in hashes:
+        src = os.path.join(ROOT, "paper_2511_18936_gb300", "csrc", fname)
+        try:
+            digest = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+        except OSError:
+            return None
+        if digest != want:
+            return None
     return float(m_tr.group(1))
 
 
@@ -880,7 +888,8 @@ def run_swan(args, wl, rank: int, world: int, local_rank: int):
                      "alg_bytes_per_launch": alg_decode, "avg_launch_ms": avg_dec_s * 1e3,
                      "traffic": decode_kernel_traffic(
                          args.workload, wl["values"],
-                         "" if wl["k_store_v"] == wl["k_store"] else f"-ksv{wl['k_store_v']}")},
+                         ("" if wl["k_store_v"] == wl["k_store"] else f"-ksv{wl['k_store_v']}")
+                         + (f"-k{k}" if args.workload == "ksweep-32k" else ""))},
         "kernels_ms_per_step": {name: v[0] / args.steps for name, v in kt.items() if v[1]},
         "kernels_timed": "second timed region of the same length, CUDA events around every launch",
         "gpu_launches": launches,

@@ -66,6 +66,7 @@ cudaError_t launch_fmt(const DecodeParams& p, int grid, cudaStream_t s) {
 int decode_ctas_per_sm(int G, int k_read) {
   const bool big = k_read > 64;
   if (G == 1) {
+    if (k_read <= 32) return occupancy(decode_kernel<4, kFmtFp16>, decode_warps<4>() * 32, one_head_smem<4>());
     if (k_read <= 64) return occupancy(decode_kernel<8, kFmtFp16>, decode_warps<8>() * 32, one_head_smem<8>());
     if (k_read <= 96)
       return occupancy(decode_kernel<12, kFmtFp16>, decode_warps<12>() * 32, one_head_smem<12>());
@@ -84,6 +85,7 @@ cudaError_t launch_decode(const DecodeParams& p, int G, int k_read, int grid, cu
   const bool big = k_read > 64;
   switch (G) {
     case 1:
+      if (k_read <= 32) return launch_fmt<1, 4>(p, grid, s);
       return k_read <= 64 ? launch_fmt<1, 8>(p, grid, s)
                           : k_read <= 96 ? launch_fmt<1, 12>(p, grid, s) : launch_fmt<1, 16>(p, grid, s);
     case 2: return big ? launch_fmt<2, 16>(p, grid, s) : launch_fmt<2, 8>(p, grid, s);

@@ -36,7 +36,7 @@ struct DeviceSetup {
   unsigned long long ctx_id = 0;  // driver context the address belongs to
   float* scratch = nullptr;       // device address of g_noalloc_scratch
   int sms = 0;
-  int ctas_per_sm[3][3] = {};  // [G = 1, 2, 4][kernel variant: <= 64, <= 96, <= 128 entries read]
+  int ctas_per_sm[3][kDecodeVariants] = {};  // [G = 1, 2, 4][kernel variant: <= 32, 64, 96, 128 entries read]
 };
 DeviceSetup g_setup[kMaxDevices];
 std::mutex g_setup_mutex;
@@ -102,8 +102,8 @@ swan_status setup_device(int dev, DeviceSetup** out) {
     if (e != cudaSuccess) return err(SWAN_ERR_CUDA, "cudaDeviceGetAttribute failed");
     const int gs[3] = {1, 2, 4};
     for (int g = 0; g < 3; ++g)
-      for (int v = 0; v < 3; ++v) {
-        s.ctas_per_sm[g][v] = decode_ctas_per_sm(gs[g], 64 + 32 * v);
+      for (int v = 0; v < kDecodeVariants; ++v) {
+        s.ctas_per_sm[g][v] = decode_ctas_per_sm(gs[g], 32 + 32 * v);
         if (s.ctas_per_sm[g][v] < 1) return err(SWAN_ERR_CUDA, "decode kernel occupancy query failed");
       }
     s.scratch = static_cast<float*>(p);

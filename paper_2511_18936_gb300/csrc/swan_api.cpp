@@ -79,7 +79,7 @@ struct swan_ctx {
   int device = 0;
   int num_sms = 0;
   int decode_ctas = 0;  // max decode CTAs resident at once (either kernel variant)
-  int decode_ctas_v[3] = {0, 0, 0};  // per kernel variant: <= 64, <= 96, <= 128 entries read
+  int decode_ctas_v[kDecodeVariants] = {};  // per kernel variant: <= 32, 64, 96, 128 entries read
 
   float* R_qk = nullptr;
   float* R_vo = nullptr;   // == R_qk when the caller passed NULL
@@ -518,8 +518,8 @@ swan_status swan_init(swan_ctx** out, const swan_config* cfg, const float* R_qk,
 
   // resident decode CTAs of the kernel variant each runtime keep count uses
   const int slots = std::max(c->k_slots, c->k_slots_v);
-  for (int v = 0; v < 3; ++v) {
-    const int k_read = 64 + 32 * v;  // the largest keep count of the variant
+  for (int v = 0; v < kDecodeVariants; ++v) {
+    const int k_read = 32 + 32 * v;  // the largest keep count of the variant
     if (v > 0 && slots <= k_read - 32) {
       c->decode_ctas_v[v] = c->decode_ctas_v[v - 1];  // never launched: no larger count is stored
       continue;

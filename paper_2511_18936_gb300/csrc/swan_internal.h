@@ -294,7 +294,8 @@ cudaError_t launch_append_small(const AppendParams& p, int evict_old, const Rota
 cudaError_t launch_prune_ring(const PruneRingParams& p, cudaStream_t s);
 cudaError_t launch_rotate_q(const RotateQParams& p, int B, cudaStream_t s);
 // k_read: entries read per vector rounded up to 8 (selects the kernel variant:
-// up to 64, up to 96 (one query head per kv head) and up to 128)
+// up to 32 and up to 96 (one query head per kv head only), up to 64, up to
+// 128)
 cudaError_t launch_decode(const DecodeParams& p, int G, int k_read, int grid, cudaStream_t s);
 cudaError_t launch_combine(const CombineParams& p, int B, cudaStream_t s);
 cudaError_t launch_transpose_r(const float* src, float* dst, int64_t mats, cudaStream_t s);
@@ -303,8 +304,9 @@ cudaError_t launch_scatter_pages(const int2* pairs, int n, int32_t* table, cudaS
 // Decode CTAs of the variant launch_decode takes for k_read that fit on one
 // SM together (for the grid size).
 int decode_ctas_per_sm(int G, int k_read);
-// The variant class of k_read: 0 (<= 64), 1 (<= 96), 2 (<= 128).
-inline int decode_variant(int k_read) { return k_read <= 64 ? 0 : k_read <= 96 ? 1 : 2; }
+// The variant class of k_read: 0 (<= 32), 1 (<= 64), 2 (<= 96), 3 (<= 128).
+constexpr int kDecodeVariants = 4;
+inline int decode_variant(int k_read) { return k_read <= 32 ? 0 : k_read <= 64 ? 1 : k_read <= 96 ? 2 : 3; }
 // Fewest 32-token groups a decode CTA takes: a small cache is split over
 // fewer CTAs so that each one's fixed cost (staging q', the merge) and the
 // final combine over the CTAs' partials stay small next to its groups

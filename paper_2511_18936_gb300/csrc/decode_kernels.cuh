@@ -599,7 +599,8 @@ __global__ void __launch_bounds__(decode_warps<MAXC>() * 32, decode_min_ctas<MAX
     // block of sparse group gi (nullptr past the run or on a bad page)
     auto block_of = [&](int gi) -> const uint8_t* {
       if (gi >= sp_hi) return nullptr;
-      const int32_t ph = __ldg(ptab + (gi >> bsh));
+      const int64_t ph = g.identity ? g.identity_base + u * g.pages_per_unit + (gi >> bsh)
+                                    : (int64_t)__ldg(ptab + (gi >> bsh));
       if (ph < 0 || ph >= g.num_pages) {
         atomicOr(p.status, kStatusPageRange);
         return nullptr;
@@ -1100,7 +1101,8 @@ __global__ void __launch_bounds__(mma_warps<MAXC>() * 32, 1) decode_mma_kernel(D
 
     auto block_of = [&](int gi) -> const uint8_t* {
       if (gi >= sp_hi) return nullptr;
-      const int32_t ph = __ldg(ptab + (gi >> bsh));
+      const int64_t ph = g.identity ? g.identity_base + u * g.pages_per_unit + (gi >> bsh)
+                                    : (int64_t)__ldg(ptab + (gi >> bsh));
       if (ph < 0 || ph >= g.num_pages) {
         atomicOr(p.status, kStatusPageRange);
         return nullptr;

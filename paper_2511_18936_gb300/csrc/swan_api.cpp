@@ -240,6 +240,8 @@ CacheGeom geom_for(const swan_ctx* c, int layer) {
   g.k_store_v = c->k_store_v;
   g.page_bytes = c->page_bytes;
   g.fmt = c->fmt;
+  g.identity = c->paged ? 0 : 1;
+  g.identity_base = (int64_t)layer * c->units * c->ppu;
   return g;
 }
 

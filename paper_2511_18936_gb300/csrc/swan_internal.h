@@ -63,6 +63,11 @@ struct CacheGeom {
   int k_store_v;
   int64_t page_bytes;        // P / 32 * block_bytes()
   int fmt;                   // kFmtFp16 or kFmtFp8
+  // 1: the table is the identity (every unit owns its pages; never written
+  // after init), so page g of unit u is identity_base + u * pages_per_unit
+  // + g and the decode kernels skip the table read; 0: read the table
+  int identity;
+  int64_t identity_base;
   // offsets inside a 32-token block (index regions: fp16 only)
   __device__ __host__ int block_bytes() const {
     return (fmt == kFmtFp8 ? 64 : 96) * (k_slots + k_slots_v);

@@ -47,6 +47,10 @@ WORKLOADS = {
     "gqa-131k": dict(B=4, H_q=32, H_kv=8, L_s=130944, n_b=128, k=56, k_store=56,
                      desc="Llama-3-8B-shaped GQA layer: batch 4, 32 q / 8 kv heads, d 128, "
                           "130944 sparse + 128 dense-buffer tokens (131072 ctx), k 56"),
+    "gqa8-32k": dict(B=4, H_q=64, H_kv=8, L_s=32640, n_b=128, k=56, k_store=56,
+                     desc="GQA layer with 8 query heads per kv head (64 q / 8 kv heads, d 128, the "
+                          "attention shape of a Llama-3-70B layer): batch 4, 32640 sparse + 128 "
+                          "dense-buffer tokens (32768 ctx), k 56"),
     "ksweep-32k": dict(B=16, H_q=32, H_kv=32, L_s=32768, n_b=128, k=64, k_store=128,
                        desc="Llama-2-7B-shaped layer at 32k with k_store 128, decoded at a runtime "
                             "keep count k (--k-active)"),
@@ -442,6 +446,27 @@ def run_basis(args, wl, rank: int, world: int, local_rank: int):
     stream.synchronize()
     eig_ms = a.elapsed_time(b)
 
+    # the energy that top-k pruning keeps (Section 4.1.2's purpose, without a
+    # model): bases from the first half of the batch, measured on the held-out
+    # second half, against a random orthogonal basis
+    half = n // 2
+    with torch.cuda.stream(stream):
+        h_qk, h_vo = swan.Gram(n_kv, dev, stream), swan.Gram(n_kv, dev, stream)
+        h_qk.add(swan.rows_of(Q[:, :half].contiguous(), G), False).add(swan.rows_of(K[:, :half].contiguous()))
+        h_vo.add(swan.rows_of(V[:, :half].contiguous()), False).add(swan.columns_of(W_O, G))
+        R_h, _, _ = swan.basis_eig(torch.cat([h_qk.gram, h_vo.gram]), stream)
+        gen = np.random.default_rng(args.seed + 7)
+        R_rand = torch.from_numpy(np.stack([synth.random_orthogonal(D, gen) for _ in range(n_kv)])
+                                  .astype(np.float32)).to(dev)
+        energy_kept = {}
+        for name, held, R_data in (("K", K, R_h[:n_kv]), ("V", V, R_h[n_kv:])):
+            rows = swan.rows_of(held[:, half:].contiguous())
+            e_d = swan.energy(rows, R_data.contiguous(), stream=stream).sum(0)
+            e_r = swan.energy(rows, R_rand, stream=stream).sum(0)
+            energy_kept[name] = {f"k{k}": {"data_basis": float(e_d[k] / e_d[D]), "random_basis": float(e_r[k] / e_r[D])}
+                                 for k in (16, 32, 56, 64, 96)}
+    stream.synchronize()
+
     # end to end: Q, K, V of the batch copied from pinned host memory every
     # step, the Gram matrices read back
     host = [t.cpu().pin_memory() for t in (Q, K, V)]
@@ -492,6 +517,8 @@ def run_basis(args, wl, rank: int, world: int, local_rank: int):
         "parts_ms_per_step": part_ms,
         "eig_ms_16_matrices": eig_ms,
         "eig_sweeps": sw_all.tolist(),
+        "energy_kept": {"held_out": f"{n - half} tokens per kv head (bases from the other {half})",
+                        **energy_kept},
         "gpu_launches": 2 * len(parts) * args.steps,
         "e2e": {"value": e2e_value, "unit": "vectors/s",
                 "h2d_bytes_per_step": sum(t.numel() * t.element_size() for t in host),
@@ -918,6 +945,7 @@ SUB_WORKLOADS = [
     ("latency-1k", "latency-1k", {}),
     ("gqa-131k", "gqa-131k", {}),
     ("gqa-131k-e4m3", "gqa-131k", {"values": "fp8_e4m3"}),
+    ("gqa8-32k", "gqa8-32k", {}),
     ("llama2-7b-layer-32k-e4m3", "llama2-7b-layer-32k", {"values": "fp8_e4m3"}),
     ("llama2-7b-layer-32k-kv64-32", "llama2-7b-layer-32k", {"k_store_v": 32}),
     *[(f"ksweep-32k-k{k}", "ksweep-32k", {"k_active": k}) for k in (32, 48, 64, 96, 128)],

@@ -69,7 +69,7 @@ typedef struct swan_config {
   int batch;       /* B >= 1 */
   int n_q_heads;   /* H_q, a multiple of n_kv_heads */
   int n_kv_heads;  /* H_kv; G = H_q / H_kv query heads share a kv head
-                      (Section 4.1.1); G must be 1, 2 or 4 */
+                      (Section 4.1.1); G must be 1, 2, 4 or 8 */
   int head_dim;    /* d, must be 128 */
   int k_store;     /* kept entries stored per vector, 1..d; the runtime keep
                       count k_active may be any value 1..k_store */

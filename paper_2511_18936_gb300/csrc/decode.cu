@@ -78,6 +78,9 @@ int decode_ctas_per_sm(int G, int k_read) {
   if (G == 4)
     return big ? occupancy(decode_mma_kernel<4, 16, kFmtFp16>, mma_warps<16>() * 32, mma_smem<4, 16>())
                : occupancy(decode_mma_kernel<4, 8, kFmtFp16>, mma_warps<8>() * 32, mma_smem<4, 8>());
+  if (G == 8)
+    return big ? occupancy(decode_mma_kernel<8, 16, kFmtFp16>, mma_warps<16>() * 32, mma_smem<8, 16>())
+               : occupancy(decode_mma_kernel<8, 8, kFmtFp16>, mma_warps<8>() * 32, mma_smem<8, 8>());
   return 0;
 }
 
@@ -90,6 +93,7 @@ cudaError_t launch_decode(const DecodeParams& p, int G, int k_read, int grid, cu
                           : k_read <= 96 ? launch_fmt<1, 12>(p, grid, s) : launch_fmt<1, 16>(p, grid, s);
     case 2: return big ? launch_fmt<2, 16>(p, grid, s) : launch_fmt<2, 8>(p, grid, s);
     case 4: return big ? launch_fmt<4, 16>(p, grid, s) : launch_fmt<4, 8>(p, grid, s);
+    case 8: return big ? launch_fmt<8, 16>(p, grid, s) : launch_fmt<8, 8>(p, grid, s);
     default: return cudaErrorInvalidValue;
   }
 }

@@ -864,16 +864,18 @@ __global__ void __launch_bounds__(decode_warps<MAXC>() * 32, decode_min_ctas<MAX
 }
 
 // ---------------------------------------------------------------------------
-// Grouped-query heads with the value product on the tensor cores (G = 2, 4).
+// Grouped-query heads with the value product on the tensor cores (G = 2, 4, 8).
 //   Lane = token, as in the one-head kernel; each lane scores its token for
 //   all G query heads of the kv head from q' replicated per lane
-//   ([128][32][G] fp32: one 8- or 16-byte conflict-free gather per entry).
+//   ([128][32 / G][G] fp32: one 8- or 16-byte conflict-free gather per entry,
+//   two 16-byte gathers at G = 8).
 //   The value product o_h += sum_t p_h(t) v_t is dense once the kept
 //   entries are scattered into a zero-filled [32 tokens][128] fp16 tile per
 //   warp, so it runs as mma.sync.m16n8k16 (k = the 32 tokens, n = the 128
 //   coordinates) with the fp32 accumulators in registers; p is split into
-//   fp16 hi + lo parts, rows 0..G-1 and G..2G-1 of the same product, so the
-//   result keeps fp32 accuracy at one product per tile.  No per-warp shared accumulator: the tile
+//   fp16 hi + lo parts, rows 0..G-1 and G..2G-1 of the same product (at
+//   G = 8 the eight rows take the hi parts, then the lo parts, in two
+//   products into the same accumulators), so the result keeps fp32 accuracy.  No per-warp shared accumulator: the tile
 //   and a [G][32] p table are all a warp holds in shared memory.
 // ---------------------------------------------------------------------------
 // Value tile rows: 128 fp16 (256 bytes, 256-byte aligned), the 16-byte
@@ -882,12 +884,15 @@ __global__ void __launch_bounds__(decode_warps<MAXC>() * 32, decode_min_ctas<MAX
 // address is (2 idx) ^ (row | (t & 7) << 4): one shift and one LOP3.
 constexpr int kVRowBytes = 256;
 constexpr uint32_t kVTileBytes = 32 * kVRowBytes;    // 8192
-constexpr uint32_t kPTileBytes = 4 * 32 * 4;         // p [<= 4 heads][32 tokens] fp32
+// p [max(G, 4) heads][32 tokens] fp32
+template <int G>
+__host__ __device__ constexpr uint32_t mma_ptile_bytes() { return (G > 4 ? G : 4) * 32 * 4; }
 // Per warp: the tile, the p table and a staging area for the value records
 // of the next block (cp.async: MAXC chunks of 512 B values + 256 B indices).
-template <int MAXC>
+// A multiple of 128 bytes, so every warp's tile rows keep their swizzle.
+template <int G, int MAXC>
 __host__ __device__ constexpr uint32_t mma_warp_bytes() {
-  return kVTileBytes + kPTileBytes + (uint32_t)MAXC * 768;
+  return kVTileBytes + mma_ptile_bytes<G>() + (uint32_t)MAXC * 768;
 }
 // 8 warps: the kernel needs ~230-255 registers a thread; registers are
 // allocated per scheduler, so 9 to 12 warps all get 168 a thread and spill
@@ -902,7 +907,8 @@ __host__ __device__ constexpr int mma_warps() { return 8; }
 constexpr uint32_t kQrepBytes = kHeadDim * 32 * 4;
 template <int G, int MAXC>
 __host__ __device__ constexpr size_t mma_smem() {  // + the 16 KB alignment slack
-  return (size_t)kQrepBytes + (size_t)mma_warps<MAXC>() * mma_warp_bytes<MAXC>() + 16384;
+  static_assert(mma_warp_bytes<G, MAXC>() % 128 == 0, "tile rows 128-byte aligned");
+  return (size_t)kQrepBytes + (size_t)mma_warps<MAXC>() * mma_warp_bytes<G, MAXC>() + 16384;
 }
 
 __device__ __forceinline__ uint4 lds_v4u(uint32_t a) {
@@ -972,17 +978,31 @@ __device__ __forceinline__ void chunk_half_words(const Chunk<FMT>& ch, uint32_t 
 }
 // Scores of G heads for one chunk: q' row idx of this lane is G floats
 // (128-byte rows, 16 KB-aligned base: the address is one shift and one
-// LOP3).  Even and odd entries go to two partial sums per head
-// (half-length FMA chains).
-template <int G>
-__device__ __forceinline__ void score_g_chunk(uint32_t qb, const float (&f)[8], uint2 ix, float (&s)[2][G]) {
+// LOP3).  With two partial-sum sets (NS = 2) even and odd entries go to
+// separate sums (half-length FMA chains).  At G = 8 the lane reads its copy's
+// two 16-byte halves in the order its qb gives (bit 4: upper half first), so
+// the 8 lanes of a phase hit 8 distinct bank groups; s[.][0..3] then hold the
+// heads of the first half read and s[.][4..7] the other (g8_heads_in_order
+// puts them back).
+template <int G, int NS>
+__device__ __forceinline__ void score_g_chunk(uint32_t qb, const float (&f)[8], uint2 ix, float (&s)[NS][G]) {
 #pragma unroll
   for (int e = 0; e < 8; ++e) {
     const uint32_t w = e < 4 ? ix.x : ix.y;
     const int sh = 7 - 8 * (e & 3);  // byte e & 3 of w to bits 7..13
     const uint32_t a = ((sh >= 0 ? (w << sh) : (w >> -sh)) & 0x3f80u) | qb;
-    float* t = s[e & 1];
-    if constexpr (G == 4) {
+    float* t = s[e % NS];
+    if constexpr (G == 8) {
+      const float4 q0 = lds4(a), q1 = lds4(a ^ 16u);
+      t[0] = fmaf(q0.x, f[e], t[0]);
+      t[1] = fmaf(q0.y, f[e], t[1]);
+      t[2] = fmaf(q0.z, f[e], t[2]);
+      t[3] = fmaf(q0.w, f[e], t[3]);
+      t[4] = fmaf(q1.x, f[e], t[4]);
+      t[5] = fmaf(q1.y, f[e], t[5]);
+      t[6] = fmaf(q1.z, f[e], t[6]);
+      t[7] = fmaf(q1.w, f[e], t[7]);
+    } else if constexpr (G == 4) {
       const float4 q = lds4(a);
       t[0] = fmaf(q.x, f[e], t[0]);
       t[1] = fmaf(q.y, f[e], t[1]);
@@ -992,6 +1012,19 @@ __device__ __forceinline__ void score_g_chunk(uint32_t qb, const float (&f)[8], 
       const float2 q = lds2(a);
       t[0] = fmaf(q.x, f[e], t[0]);
       t[1] = fmaf(q.y, f[e], t[1]);
+    }
+  }
+}
+// G = 8: a lane that read its copy's upper half first (hi) holds heads 4..7
+// in s[0..3] and heads 0..3 in s[4..7]; swap them into head order.
+template <int G>
+__device__ __forceinline__ void g8_heads_in_order(float (&s)[G], bool hi) {
+  if constexpr (G == 8) {
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const float a = s[j], b = s[j + 4];
+      s[j] = hi ? b : a;
+      s[j + 4] = hi ? a : b;
     }
   }
 }
@@ -1013,7 +1046,8 @@ __device__ __forceinline__ void scatter_chunk(uint32_t vsw, const uint32_t (&w)[
 template <int G, int MAXC, int FMT>
 __global__ void __launch_bounds__(mma_warps<MAXC>() * 32, 1) decode_mma_kernel(DecodeParams p) {
   constexpr int NW = mma_warps<MAXC>(), NT = NW * 32;
-  constexpr uint32_t kWarpBytes = mma_warp_bytes<MAXC>();
+  constexpr uint32_t kWarpBytes = mma_warp_bytes<G, MAXC>();
+  constexpr int NS = G == 8 ? 1 : 2;  // partial-sum sets of the scores
   extern __shared__ __align__(16) unsigned char smem_raw[];
   __shared__ float red_m[NW * G], red_l[NW * G];
   __shared__ float flag[1];
@@ -1029,8 +1063,10 @@ __global__ void __launch_bounds__(mma_warps<MAXC>() * 32, 1) decode_mma_kernel(D
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t vtile = wbase + warp * kWarpBytes;                         // [32][256 B] fp16, swizzled
   float* ptile_f = reinterpret_cast<float*>(base_ptr + (vtile + kVTileBytes - base));  // [G][32] fp32
-  const uint32_t vstage = vtile + kVTileBytes + kPTileBytes;                  // value records, next block
-  const uint32_t qb = base + (lane & (32 / G - 1)) * (G * 4);  // this lane's copy
+  const uint32_t vstage = vtile + kVTileBytes + mma_ptile_bytes<G>();         // value records, next block
+  // this lane's copy (at G = 8 with the half it reads first in bit 4)
+  const bool q_hi_first = G == 8 && ((lane >> 2) & 1);
+  const uint32_t qb = base + (lane & (32 / G - 1)) * (G * 4) + (q_hi_first ? 16u : 0u);
   const uint32_t vrow = vtile + lane * kVRowBytes;
   const uint32_t vsw = vrow | ((uint32_t)(lane & 7) << 4);  // this row with its chunk swizzle
   const int gq = lane >> 2, cq = lane & 3;  // mma fragment coordinates
@@ -1079,14 +1115,12 @@ __global__ void __launch_bounds__(mma_warps<MAXC>() * 32, 1) decode_mma_kernel(D
     cp_async_wait_all();
     __syncthreads();  // the previous segment is done with q'; q_stage has landed
     // 32 floats per coordinate c: 32 / G copies of its G heads (float4 f
-    // holds coordinate f / 8, heads 0..3 or 0, 1, 0, 1)
+    // holds coordinate f / 8, heads (4 (f % 8) + e) % G, e = 0..3: 0..3 at
+    // G = 4, 0, 1, 0, 1 at G = 2, the lower or upper four at G = 8)
     for (int f = threadIdx.x; f < kHeadDim * 8; f += NT) {
-      const int c = f >> 3;
-      float4 v;
-      if constexpr (G == 4)
-        v = make_float4(q_stage[c], q_stage[kHeadDim + c], q_stage[2 * kHeadDim + c], q_stage[3 * kHeadDim + c]);
-      else
-        v = make_float4(q_stage[c], q_stage[kHeadDim + c], q_stage[c], q_stage[kHeadDim + c]);
+      const int c = f >> 3, h0 = (4 * (f & 7)) % G;
+      const float4 v = make_float4(q_stage[(h0 % G) * kHeadDim + c], q_stage[((h0 + 1) % G) * kHeadDim + c],
+                                   q_stage[((h0 + 2) % G) * kHeadDim + c], q_stage[((h0 + 3) % G) * kHeadDim + c]);
       reinterpret_cast<float4*>(qrep)[f] = v;
     }
     __syncthreads();
@@ -1155,9 +1189,11 @@ __global__ void __launch_bounds__(mma_warps<MAXC>() * 32, 1) decode_mma_kernel(D
 
     for (int gi = t_lo; gi < t_hi; ++gi) {
       float s[G];
-      float s2[2][G];
+      float s2[NS][G];
 #pragma unroll
-      for (int j = 0; j < G; ++j) s2[0][j] = s2[1][j] = 0.f;
+      for (int i = 0; i < NS; ++i)
+#pragma unroll
+        for (int j = 0; j < G; ++j) s2[i][j] = 0.f;
       bool valid;
       if (gi < n_sg) {
         // ---- sparse tokens 32 gi .. 32 gi + 31
@@ -1173,11 +1209,12 @@ __global__ void __launch_bounds__(mma_warps<MAXC>() * 32, 1) decode_mma_kernel(D
               float f[8];
               chunk_vals<FMT>(kc[c], f);
               if (krem && c == nchunks - 1) keep_first(f, krem);
-              score_g_chunk<G>(qb, f, chunk_idx<FMT>(kc[c]), s2);
+              score_g_chunk<G, NS>(qb, f, chunk_idx<FMT>(kc[c]), s2);
             }
         }
 #pragma unroll
-        for (int j = 0; j < G; ++j) s[j] = s2[0][j] + s2[1][j];
+        for (int j = 0; j < G; ++j) s[j] = NS == 2 ? s2[0][j] + s2[NS - 1][j] : s2[0][j];
+        g8_heads_in_order<G>(s, q_hi_first);
         // this token's kept values (staged by cp.async) into its tile row;
         // each staged chunk is read before the previous one is stored
         cp_async_wait_all();
@@ -1238,8 +1275,18 @@ __global__ void __launch_bounds__(mma_warps<MAXC>() * 32, 1) decode_mma_kernel(D
 #pragma unroll
             for (int e = 0; e < 8; ++e) {
               const uint32_t qa = qb + (uint32_t)(c * 8 + e) * 128u;
-              float* t = s2[e & 1];
-              if constexpr (G == 4) {
+              float* t = s2[e % NS];
+              if constexpr (G == 8) {
+                const float4 q0 = lds4(qa), q1 = lds4(qa ^ 16u);
+                t[0] = fmaf(q0.x, f[e], t[0]);
+                t[1] = fmaf(q0.y, f[e], t[1]);
+                t[2] = fmaf(q0.z, f[e], t[2]);
+                t[3] = fmaf(q0.w, f[e], t[3]);
+                t[4] = fmaf(q1.x, f[e], t[4]);
+                t[5] = fmaf(q1.y, f[e], t[5]);
+                t[6] = fmaf(q1.z, f[e], t[6]);
+                t[7] = fmaf(q1.w, f[e], t[7]);
+              } else if constexpr (G == 4) {
                 const float4 q = lds4(qa);
                 t[0] = fmaf(q.x, f[e], t[0]);
                 t[1] = fmaf(q.y, f[e], t[1]);
@@ -1254,7 +1301,8 @@ __global__ void __launch_bounds__(mma_warps<MAXC>() * 32, 1) decode_mma_kernel(D
           }
           }
 #pragma unroll
-          for (int j = 0; j < G; ++j) s[j] = s2[0][j] + s2[1][j];
+          for (int j = 0; j < G; ++j) s[j] = NS == 2 ? s2[0][j] + s2[NS - 1][j] : s2[0][j];
+          g8_heads_in_order<G>(s, q_hi_first);
 #pragma unroll 1
           for (int cb = 0; cb < 16; cb += 8) {
             uint4 wv[8];
@@ -1295,6 +1343,28 @@ __global__ void __launch_bounds__(mma_warps<MAXC>() * 32, 1) decode_mma_kernel(D
       // the merge)
 #pragma unroll
       for (int ks = 0; ks < 2; ++ks) {
+        if constexpr (G == 8) {
+          // rows 0..7: the heads' hi parts, then their lo parts, into the
+          // same accumulators
+          const float* pr = ptile_f + gq * 32 + ks * 16 + 2 * cq;
+          uint32_t hi0, lo0, hi2, lo2;
+          split_pair(pr[0], pr[1], hi0, lo0);
+          split_pair(pr[8], pr[9], hi2, lo2);
+#pragma unroll
+          for (int np = 0; np < 8; ++np) {
+            const int mi = lane >> 3;
+            const uint32_t chunk = 2 * np + (mi >> 1);
+            const uint32_t addr = vtile + (uint32_t)(ks * 16 + (mi & 1) * 8 + (lane & 7)) * kVRowBytes +
+                                  ((chunk ^ (uint32_t)(lane & 7)) << 4);
+            uint32_t bf[4];
+            ldsm_x4_trans(addr, bf);
+            mma_16816(acc[2 * np], hi0, hi2, bf[0], bf[1]);
+            mma_16816(acc[2 * np], lo0, lo2, bf[0], bf[1]);
+            mma_16816(acc[2 * np + 1], hi0, hi2, bf[2], bf[3]);
+            mma_16816(acc[2 * np + 1], lo0, lo2, bf[2], bf[3]);
+          }
+          continue;
+        }
         uint32_t a0 = 0, a2 = 0;
         if (gq < 2 * G) {
           const bool hi_row = gq < G;
@@ -1333,12 +1403,15 @@ __global__ void __launch_bounds__(mma_warps<MAXC>() * 32, 1) decode_mma_kernel(D
         red_l[warp * G + j] = l[j];
       }
     }
-    // the lo rows (G..2G-1, lanes 4G above) onto the hi rows, then this
-    // warp's o rows into its tile region ([G][128] fp32)
+    // the lo rows (G..2G-1, lanes 4G above) onto the hi rows (at G = 8 the
+    // products already summed them), then this warp's o rows into its tile
+    // region ([G][128] fp32)
+    if constexpr (G < 8) {
 #pragma unroll
-    for (int nt = 0; nt < 16; ++nt) {
-      acc[nt][0] += __shfl_down_sync(0xffffffffu, acc[nt][0], 4 * G);
-      acc[nt][1] += __shfl_down_sync(0xffffffffu, acc[nt][1], 4 * G);
+      for (int nt = 0; nt < 16; ++nt) {
+        acc[nt][0] += __shfl_down_sync(0xffffffffu, acc[nt][0], 4 * G);
+        acc[nt][1] += __shfl_down_sync(0xffffffffu, acc[nt][1], 4 * G);
+      }
     }
     __syncwarp();
     float* obuf = reinterpret_cast<float*>(base_ptr + (vtile - base));
@@ -1378,13 +1451,16 @@ __global__ void __launch_bounds__(mma_warps<MAXC>() * 32, 1) decode_mma_kernel(D
       }
     }
     __syncthreads();
-    // the o rows overwrote part of the tiles: zero them again
-    for (int c = 0; c < 16; ++c) sts_v4(vsw ^ (uint32_t)(c << 4), make_uint4(0, 0, 0, 0));
     if (solo) {
       rotate_back_out<G, NT>(p, b, h, qrep, qrep);
     } else {
       finish_unit<G, NT>(p, c0, c1, u, b, h, qrep, flag);
     }
+    // the o rows overwrote part of the tiles, and the rotate-back's slices
+    // (NT / 32 * G * 128 floats: past q' into the first warps' regions at
+    // G = 8) more: zero them again once every thread is done with them
+    __syncthreads();
+    for (int c = 0; c < 16; ++c) sts_v4(vsw ^ (uint32_t)(c << 4), make_uint4(0, 0, 0, 0));
   }
 }
 

@@ -36,7 +36,7 @@ struct DeviceSetup {
   unsigned long long ctx_id = 0;  // driver context the address belongs to
   float* scratch = nullptr;       // device address of g_noalloc_scratch
   int sms = 0;
-  int ctas_per_sm[3][kDecodeVariants] = {};  // [G = 1, 2, 4][kernel variant: <= 32, 64, 96, 128 entries read]
+  int ctas_per_sm[4][kDecodeVariants] = {};  // [G = 1, 2, 4, 8][kernel variant: <= 32, 64, 96, 128 entries read]
 };
 DeviceSetup g_setup[kMaxDevices];
 std::mutex g_setup_mutex;
@@ -81,7 +81,7 @@ swan_status err(swan_status s, const char* msg) {
   return s;
 }
 
-int gi(int G) { return G == 1 ? 0 : G == 2 ? 1 : 2; }
+int gi(int G) { return G == 1 ? 0 : G == 2 ? 1 : G == 4 ? 2 : 3; }
 
 // Once per device (and again if the device's context was re-created), with
 // that device current: resolve the device address of the static scratch
@@ -100,8 +100,8 @@ swan_status setup_device(int dev, DeviceSetup** out) {
     if (e != cudaSuccess || p == nullptr) return err(SWAN_ERR_CUDA, "cudaGetSymbolAddress failed");
     e = cudaDeviceGetAttribute(&s.sms, cudaDevAttrMultiProcessorCount, dev);
     if (e != cudaSuccess) return err(SWAN_ERR_CUDA, "cudaDeviceGetAttribute failed");
-    const int gs[3] = {1, 2, 4};
-    for (int g = 0; g < 3; ++g)
+    const int gs[4] = {1, 2, 4, 8};
+    for (int g = 0; g < 4; ++g)
       for (int v = 0; v < kDecodeVariants; ++v) {
         s.ctas_per_sm[g][v] = decode_ctas_per_sm(gs[g], 32 + 32 * v);
         if (s.ctas_per_sm[g][v] < 1) return err(SWAN_ERR_CUDA, "decode kernel occupancy query failed");
@@ -127,7 +127,7 @@ extern "C" swan_status swan_decode_noalloc(const swan_cache_view* v, const void*
   if (v->batch < 1 || v->n_kv_heads < 1 || v->n_q_heads < 1 || v->n_q_heads % v->n_kv_heads)
     return err(SWAN_ERR_INVALID_ARG, "bad batch or head counts");
   const int G = v->n_q_heads / v->n_kv_heads;
-  if (G != 1 && G != 2 && G != 4) return err(SWAN_ERR_UNSUPPORTED, "group size must be 1, 2 or 4");
+  if (G != 1 && G != 2 && G != 4 && G != 8) return err(SWAN_ERR_UNSUPPORTED, "group size must be 1, 2, 4 or 8");
   if (v->k_slots < 8 || v->k_slots > kHeadDim || v->k_slots % 8)
     return err(SWAN_ERR_INVALID_ARG, "k_slots must be a multiple of 8 in [8, 128]");
   if (v->k_active < 1 || v->k_active > v->k_slots) return err(SWAN_ERR_INVALID_ARG, "k_active out of range");

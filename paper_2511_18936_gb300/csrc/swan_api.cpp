@@ -471,8 +471,8 @@ swan_status swan_init(swan_ctx** out, const swan_config* cfg, const float* R_qk,
     return fail(SWAN_ERR_INVALID_ARG, "n_q_heads %d is not a multiple of n_kv_heads %d", C.n_q_heads,
                 C.n_kv_heads);
   const int G = C.n_q_heads / C.n_kv_heads;
-  if (G != 1 && G != 2 && G != 4)
-    return fail(SWAN_ERR_UNSUPPORTED, "group size %d: only 1, 2 and 4 are built", G);
+  if (G != 1 && G != 2 && G != 4 && G != 8)
+    return fail(SWAN_ERR_UNSUPPORTED, "group size %d: only 1, 2, 4 and 8 are built", G);
   if (C.k_store < 1 || C.k_store > C.head_dim)
     return fail(SWAN_ERR_INVALID_ARG, "k_store %d out of [1, %d]", C.k_store, C.head_dim);
   const int k_store_v = C.k_store_v ? C.k_store_v : C.k_store;

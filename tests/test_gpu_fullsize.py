@@ -89,6 +89,15 @@ def test_gqa_131k_peaked_queries_sampled(fmt):
                 samples=[(1, 3)], seed=1, q_scale=4.0, value_format=fmt)
 
 
+@pytest.mark.parametrize("seed,q_scale", [(0, 1.0), (1, 4.0)])
+def test_gqa_g8_32k_sampled(seed, q_scale):
+    """Eight query heads per kv head (a 64-query, 8-kv-head layer) at 32k
+    context: the two-gather q' path and the two-product value path, split
+    over many CTAs, with ordinary and peaked (x4) queries."""
+    _layer_case(B=2, H_q=64, H_kv=8, L_s=32640, n_b=128, k_store=56, k_actives=(56, 24),
+                samples=[(0, 0), (1, 7)], seed=seed, q_scale=q_scale)
+
+
 def test_ksweep_32k_sampled_and_dense_at_k128():
     _layer_case(B=16, H_q=32, H_kv=32, L_s=32768, n_b=128, k_store=128,
                 k_actives=(32, 48, 64, 96, 128), samples=[(2, 5), (11, 30)], steps=1)

@@ -238,6 +238,8 @@ DECODE_CASES = [
     (2, 4, 2, 777, 16, 60, (60, 7), 32),            # G = 2, ragged everything
     (1, 2, 1, 700, 128, 128, (128, 96, 64, 48, 32), 128),  # runtime k sweep
     (3, 2, 4, 300, 0, 24, (24, 5), 32),             # no buffer at all
+    (2, 2, 8, 1300, 64, 56, (56, 40, 3), 64),       # GQA G = 8 (two 16-byte q' gathers)
+    (1, 2, 8, 600, 32, 128, (128, 80), 32),         # G = 8, more than 64 entries read
 ]
 
 
@@ -437,6 +439,7 @@ FP8_DECODE_CASES = [
     (2, 2, 4, 1500, 128, 56, (56, 13), 64),
     (2, 4, 2, 777, 16, 60, (60, 7), 32),
     (1, 2, 1, 700, 128, 128, (128, 96, 32), 128),
+    (2, 2, 8, 1300, 64, 56, (56, 11), 64),
 ]
 
 
@@ -500,6 +503,7 @@ ASYM_DECODE_CASES = [
     (2, 2, 4, 1500, 128, 24, 72, [(24, 72), (24, 40)], 64, "fp16"),
     (2, 2, 1, 1000, 64, 64, 32, [(64, 32), (40, 5)], 128, "fp8_e4m3"),
     (2, 2, 4, 900, 32, 96, 16, [(96, 16), (65, 16)], 32, "fp8_e4m3"),
+    (2, 2, 8, 1100, 32, 40, 80, [(40, 80), (33, 71)], 64, "fp16"),
 ]
 
 

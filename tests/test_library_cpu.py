@@ -54,7 +54,8 @@ def _cfg(**kw):
 @pytest.mark.parametrize("kw,status", [
     (dict(head_dim=64), swan.ERR_UNSUPPORTED),
     (dict(n_q_heads=3, n_kv_heads=1), swan.ERR_UNSUPPORTED),
-    (dict(n_q_heads=8, n_kv_heads=1), swan.ERR_UNSUPPORTED),
+    (dict(n_q_heads=16, n_kv_heads=1), swan.ERR_UNSUPPORTED),
+    (dict(n_q_heads=12, n_kv_heads=2), swan.ERR_UNSUPPORTED),
     (dict(n_q_heads=3, n_kv_heads=2), swan.ERR_INVALID_ARG),
     (dict(k_store=0), swan.ERR_INVALID_ARG),
     (dict(k_store=129), swan.ERR_INVALID_ARG),

@@ -12,7 +12,7 @@ call's contents, so the second call shows that nothing stale leaks in):
 * the caller's cache is built here from the oracle's own state (its pruned
   indices and values, its dense buffer) in the page layout the header
   documents, and the output must match the oracle's decode within the
-  attention tolerance: for G = 1, 2, 4, fp16 and E4M3 values, equal and
+  attention tolerance: for G = 1, 2, 4, 8, fp16 and E4M3 values, equal and
   separate key/value keep counts, the >64-entry kernel variant, a
   buffer-only and an empty cache;
 * the caller's cache is a copy of what a libswan context built, and the
@@ -164,6 +164,8 @@ ORACLE_CASES = [
     (1, "fp8_e4m3", 48, 24, (48, 9)),
     (1, "fp16", 128, 128, (96, 96)),
     (4, "fp16", 128, 100, (72, 100)),
+    (8, "fp16", 56, 56, (56, 21)),
+    (8, "fp8_e4m3", 64, 40, (48, 40)),
 ]
 
 
@@ -215,6 +217,7 @@ CONTEXT_CASES = [
     (2, "fp16", 60, 60, ((60, 60), (29, 29))),
     (1, "fp8_e4m3", 64, 32, ((64, 32), (40, 12))),
     (4, "fp16", 56, 56, ((56, 56), (30, 56))),
+    (8, "fp16", 56, 48, ((56, 48), (17, 48))),
 ]
 
 

@@ -321,9 +321,13 @@ constexpr int64_t kMinGroupsPerCta = 4;
 // What a CTA's extra visit to a unit (prologue, merge, arrival) costs in
 // 32-token groups of streaming, for the cost-balanced split of the decode
 // kernels: equal-length rows (computed in the kernel) and ragged rows (the
-// host's table).  Set by measurement on the GB300.
+// host's table).  Set by sweeps on the GB300: ragged serving batch (32 rows,
+// 1k-56k tokens) 0.914 ms at 48, 0.898 at 56, 0.883 at 64, 0.865 at 72,
+// 0.864 at 80, 0.870 at 88; equal rows flat within 0.5 % from 12 to 64 for
+// one head (32k layer, 32-layer stack: 48 and up 2 % slower there, k 32),
+// GQA best at 40 (0.360 ms; 0.362 at 20 and 60).
 inline int64_t decode_visit_cost(int G, bool ragged) {
-  if (ragged) return 48;
+  if (ragged) return 80;
   return G == 1 ? 12 : 40;
 }
 // Record the detail string that swan_last_error() returns on this thread.

@@ -182,6 +182,22 @@ swan_status swan_append_varlen(swan_ctx* ctx, int layer, const void* k_new, cons
 swan_status swan_reset_sequence(swan_ctx* ctx, int b);
 
 /*
+ * Make row dst a copy of row src in every layer (parallel sampling, beam
+ * search: several continuations of one prompt).  Afterwards dst attends over
+ * the same history and dense buffer as src, and the two rows go on
+ * independently.  Requires a page pool (pool_pages > 0).  dst's own tokens
+ * are dropped first, as by swan_reset_sequence.  The sparse pages are
+ * shared, not copied: appends only ever write into a row's last, partly
+ * filled page, so a row that is about to write into a page other rows still
+ * hold gets its own copy first (copy on write, counted against the pool);
+ * a page returns to the pool when no row holds it.  The dense buffer is
+ * per row and is copied (device to device, on the context's stream).
+ * Errors: INVALID_ARG (rows out of range or equal), UNSUPPORTED (no page
+ * pool), CUDA.
+ */
+swan_status swan_fork_sequence(swan_ctx* ctx, int src, int dst);
+
+/*
  * One decode step of attention for one layer (Algorithm 1, attention part):
  *   q:   device fp16 [batch][n_q_heads][d], post-RoPE, unrotated.
  *   out: device fp16 [batch][n_q_heads][d], written as

@@ -10,6 +10,7 @@
 #include <cstring>
 #include <new>
 #include <string>
+#include <unordered_map>
 #include <vector>
 
 #include "swan.h"
@@ -72,6 +73,7 @@ struct swan_ctx {
   int64_t num_pages = 0;
   bool paged = false;               // pages handed out on demand from a shared pool
   std::vector<int32_t> free_pages;  // paged: free page ids
+  std::vector<int32_t> page_refs;   // paged: rows holding each page (> 1 after swan_fork_sequence)
   std::vector<int32_t> pt_host;     // paged: host copy of the page tables, -1 = none
   int fmt = kFmtFp16;
   int64_t units = 0;  // batch * n_kv_heads (per layer)
@@ -279,16 +281,43 @@ uint16_t e4m3_to_half_bits(uint8_t b) {
 
 int64_t pages_for(int64_t tokens, int P) { return (tokens + P - 1) / P; }
 
+int32_t& pt_entry(swan_ctx* c, int layer, int64_t unit, int64_t pg) {
+  return c->pt_host[((size_t)layer * c->units + unit) * c->ppu + pg];
+}
+
+// Pages a layer's rows need to reach new_len[b] sparse tokens: fresh pages
+// past each row's last one, plus copies of the last, partly filled pages
+// that a row will write into while other rows (forks) still hold them. A
+// page that every holder writes into is copied for all but one of them.
+int64_t pages_needed(swan_ctx* c, int layer, const std::vector<int64_t>& new_len) {
+  const LayerState& L = c->layers[layer];
+  const int H = c->cfg.n_kv_heads;
+  int64_t need = 0;
+  std::unordered_map<int32_t, int> writers;
+  for (int b = 0; b < c->cfg.batch; ++b) {
+    const int64_t len = L.seq[b].sparse_len;
+    need += (int64_t)H * std::max<int64_t>(0, pages_for(new_len[b], c->P) - pages_for(len, c->P));
+    if (new_len[b] > len && len % c->P != 0)
+      for (int h = 0; h < H; ++h) {
+        const int32_t id = pt_entry(c, layer, (int64_t)b * H + h, len / c->P);
+        if (c->page_refs[(size_t)id] > 1) ++writers[id];
+      }
+  }
+  for (const auto& w : writers) need += w.second < c->page_refs[(size_t)w.first] ? w.second : w.second - 1;
+  return need;
+}
+
 // Paged pool: give every unit of each row the pages its sparse history needs
 // to reach new_len[b] tokens, and write them into the device page table.
-// Nothing changes when the pool is too small.
+// A row about to write into a last page it shares with a fork gets its own
+// copy first (copy on write: only a row's last, partly filled page is ever
+// written, so full pages stay shared).  Nothing changes when the pool is too
+// small.
 swan_status grow_pages(swan_ctx* c, int layer, const std::vector<int64_t>& new_len) {
   if (!c->paged) return SWAN_OK;
   LayerState& L = c->layers[layer];
   const int H = c->cfg.n_kv_heads;
-  int64_t need = 0;
-  for (int b = 0; b < c->cfg.batch; ++b)
-    need += (int64_t)H * std::max<int64_t>(0, pages_for(new_len[b], c->P) - pages_for(L.seq[b].sparse_len, c->P));
+  const int64_t need = pages_needed(c, layer, new_len);
   if (need == 0) return SWAN_OK;
   if (need > (int64_t)c->free_pages.size())
     return fail(SWAN_ERR_CAPACITY, "layer %d needs %lld more pages, the pool has %zu free", layer, (long long)need,
@@ -296,13 +325,31 @@ swan_status grow_pages(swan_ctx* c, int layer, const std::vector<int64_t>& new_l
   std::vector<int2> pairs;
   pairs.reserve((size_t)need);
   for (int b = 0; b < c->cfg.batch; ++b) {
-    const int64_t p0 = pages_for(L.seq[b].sparse_len, c->P), p1 = pages_for(new_len[b], c->P);
+    const int64_t len = L.seq[b].sparse_len;
+    const int64_t p0 = pages_for(len, c->P), p1 = pages_for(new_len[b], c->P);
     for (int h = 0; h < H; ++h) {
       const int64_t unit = (int64_t)b * H + h;
+      if (new_len[b] > len && len % c->P != 0) {
+        int32_t& slot = pt_entry(c, layer, unit, len / c->P);
+        const int32_t old = slot;
+        if (c->page_refs[(size_t)old] > 1) {
+          const int32_t id = c->free_pages.back();
+          c->free_pages.pop_back();
+          const cudaError_t e = cudaMemcpyAsync(c->pool + (int64_t)id * c->page_bytes,
+                                                c->pool + (int64_t)old * c->page_bytes, (size_t)c->page_bytes,
+                                                cudaMemcpyDeviceToDevice, c->stream);
+          if (e != cudaSuccess) return cuda_fail(c, e, "copying a shared page");
+          --c->page_refs[(size_t)old];
+          c->page_refs[(size_t)id] = 1;
+          slot = id;
+          pairs.push_back(make_int2((int)(unit * c->ppu + len / c->P), id));
+        }
+      }
       for (int64_t pg = p0; pg < p1; ++pg) {
         const int32_t id = c->free_pages.back();
         c->free_pages.pop_back();
-        c->pt_host[((size_t)layer * c->units + unit) * c->ppu + pg] = id;
+        c->page_refs[(size_t)id] = 1;
+        pt_entry(c, layer, unit, pg) = id;
         pairs.push_back(make_int2((int)(unit * c->ppu + pg), id));
       }
     }
@@ -581,6 +628,7 @@ swan_status swan_init(swan_ctx** out, const swan_config* cfg, const float* R_qk,
   for (size_t i = 0; i < pt_elems; ++i) pt[i] = c->paged ? -1 : (int32_t)i;
   if (c->paged) {
     c->pt_host = pt;
+    c->page_refs.assign((size_t)c->num_pages, 0);
     c->free_pages.resize((size_t)c->num_pages);
     for (int64_t i = 0; i < c->num_pages; ++i) c->free_pages[(size_t)i] = (int32_t)(c->num_pages - 1 - i);
   }
@@ -837,10 +885,11 @@ swan_status swan_flush_buffer(swan_ctx* c, int layer) {
   if (layer == -1) {
     if (c->paged) {  // all layers or none: check the pool first
       int64_t need = 0;
-      for (int l = 0; l < c->cfg.num_layers; ++l)
-        for (const SeqState& q : c->layers[l].seq)
-          need += (int64_t)c->cfg.n_kv_heads *
-                  (pages_for(q.sparse_len + q.buf_count, c->P) - pages_for(q.sparse_len, c->P));
+      for (int l = 0; l < c->cfg.num_layers; ++l) {
+        std::vector<int64_t> new_len;
+        for (const SeqState& q : c->layers[l].seq) new_len.push_back(q.sparse_len + q.buf_count);
+        need += pages_needed(c, l, new_len);
+      }
       if (need > (int64_t)c->free_pages.size())
         return fail(SWAN_ERR_CAPACITY, "flushing every layer needs %lld more pages, the pool has %zu free",
                     (long long)need, c->free_pages.size());
@@ -853,10 +902,11 @@ swan_status swan_flush_buffer(swan_ctx* c, int layer) {
   return prune_from_ring(c, layer, buffer_counts(c->layers[layer]));
 }
 
-swan_status swan_reset_sequence(swan_ctx* c, int b) {
-  swan_status s = usable(c);
-  if (s != SWAN_OK) return s;
-  if (b < 0 || b >= c->cfg.batch) return fail(SWAN_ERR_INVALID_ARG, "row %d out of [0, %d)", b, c->cfg.batch);
+namespace {
+
+// Drop row b's tokens in every layer; its pages go back to the pool once no
+// fork holds them.
+void reset_row(swan_ctx* c, int b) {
   for (int l = 0; l < c->cfg.num_layers; ++l) {
     SeqState& q = c->layers[l].seq[b];
     if (c->paged) {
@@ -864,13 +914,68 @@ swan_status swan_reset_sequence(swan_ctx* c, int b) {
       for (int h = 0; h < c->cfg.n_kv_heads; ++h) {
         const int64_t unit = (int64_t)b * c->cfg.n_kv_heads + h;
         for (int64_t pg = 0; pg < used; ++pg) {
-          int32_t& id = c->pt_host[((size_t)l * c->units + unit) * c->ppu + pg];
-          c->free_pages.push_back(id);
+          int32_t& id = pt_entry(c, l, unit, pg);
+          if (--c->page_refs[(size_t)id] == 0) c->free_pages.push_back(id);
           id = -1;
         }
       }
     }
     q = SeqState{};
+  }
+}
+
+}  // namespace
+
+swan_status swan_reset_sequence(swan_ctx* c, int b) {
+  swan_status s = usable(c);
+  if (s != SWAN_OK) return s;
+  if (b < 0 || b >= c->cfg.batch) return fail(SWAN_ERR_INVALID_ARG, "row %d out of [0, %d)", b, c->cfg.batch);
+  reset_row(c, b);
+  return SWAN_OK;
+}
+
+swan_status swan_fork_sequence(swan_ctx* c, int src, int dst) {
+  swan_status s = usable(c);
+  if (s != SWAN_OK) return s;
+  if (!c->paged) return fail(SWAN_ERR_UNSUPPORTED, "forking a row needs a page pool (pool_pages > 0)");
+  if (src < 0 || src >= c->cfg.batch || dst < 0 || dst >= c->cfg.batch || src == dst)
+    return fail(SWAN_ERR_INVALID_ARG, "rows %d -> %d: two different rows of [0, %d)", src, dst, c->cfg.batch);
+  reset_row(c, dst);
+  const int H = c->cfg.n_kv_heads, cap = c->cfg.buffer_cap;
+  for (int l = 0; l < c->cfg.num_layers; ++l) {
+    LayerState& L = c->layers[l];
+    const int64_t used = pages_for(L.seq[src].sparse_len, c->P);
+    std::vector<int2> pairs;
+    for (int h = 0; h < H; ++h) {
+      const int64_t us = (int64_t)src * H + h, ud = (int64_t)dst * H + h;
+      for (int64_t pg = 0; pg < used; ++pg) {
+        const int32_t id = pt_entry(c, l, us, pg);
+        ++c->page_refs[(size_t)id];
+        pt_entry(c, l, ud, pg) = id;
+        pairs.push_back(make_int2((int)(ud * c->ppu + pg), id));
+      }
+    }
+    cudaError_t e = cudaSuccess;
+    if (!pairs.empty()) {
+      e = cudaMemcpyAsync(c->pt_pairs, pairs.data(), pairs.size() * sizeof(int2), cudaMemcpyHostToDevice,
+                          c->stream);
+      if (e != cudaSuccess) return cuda_fail(c, e, "uploading page-table entries");
+      int32_t* table = c->page_table + (int64_t)l * c->units * c->ppu;
+      s = launch(c, SWAN_KERNEL_PRUNE, "page-table scatter",
+                 [&] { return launch_scatter_pages(c->pt_pairs, (int)pairs.size(), table, c->stream); });
+      if (s != SWAN_OK) return s;
+    }
+    // the dense buffer is per row: copy its ring slots (all H heads of a
+    // row are contiguous)
+    if (cap > 0) {
+      const size_t row = (size_t)H * cap * kHeadDim, off = (size_t)l * ring_elems_per_layer(c);
+      for (__half* ring : {c->ring_k, c->ring_v}) {
+        e = cudaMemcpyAsync(ring + off + (size_t)dst * row, ring + off + (size_t)src * row, row * sizeof(__half),
+                            cudaMemcpyDeviceToDevice, c->stream);
+        if (e != cudaSuccess) return cuda_fail(c, e, "copying a row's dense buffer");
+      }
+    }
+    L.seq[dst] = L.seq[src];
   }
   return SWAN_OK;
 }

@@ -31,8 +31,8 @@ EXPORTED = ["swan_init", "swan_destroy", "swan_set_k", "swan_append", "swan_flus
             "swan_timing_enable", "swan_timing_read", "swan_launch_count",
             "swan_status_string", "swan_last_error", "swan_decode_noalloc", "swan_set_kv",
             "swan_gram_workspace_bytes", "swan_gram", "swan_basis_eig", "swan_energy",
-            "swan_basis_check", "swan_append_varlen", "swan_reset_sequence", "swan_query_lengths",
-            "swan_debug_export_seq", "swan_append_decode", "swan_debug_fail_after",
+            "swan_basis_check", "swan_append_varlen", "swan_reset_sequence", "swan_fork_sequence",
+            "swan_query_lengths", "swan_debug_export_seq", "swan_append_decode", "swan_debug_fail_after",
             "swan_debug_check_guards", "swan_noalloc_check", "swan_debug_starve_tc"]
 
 
@@ -105,6 +105,7 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "swan_append": (i, [vp, i, vp, vp, i]),
         "swan_append_varlen": (i, [vp, i, vp, vp, i, ctypes.POINTER(ctypes.c_int32)]),
         "swan_reset_sequence": (i, [vp, i]),
+        "swan_fork_sequence": (i, [vp, i, i]),
         "swan_query_lengths": (i, [vp, i, ctypes.POINTER(ctypes.c_int64), ctypes.POINTER(ctypes.c_int32)]),
         "swan_debug_export_seq": (i, [vp, i, i, i, vp, ctypes.c_size_t]),
         "swan_flush_buffer": (i, [vp, i]),
@@ -224,6 +225,10 @@ class Context:
 
     def reset_sequence(self, b: int):
         _check(self._lib.swan_reset_sequence(self._h, int(b)), "swan_reset_sequence")
+
+    def fork_sequence(self, src: int, dst: int):
+        """Row dst becomes a copy of row src (shared pages, copied buffer)."""
+        _check(self._lib.swan_fork_sequence(self._h, int(src), int(dst)), "swan_fork_sequence")
 
     def lengths(self, layer: int = 0):
         """Per-row (sparse, buffered) token counts of a layer."""

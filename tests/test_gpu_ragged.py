@@ -2,6 +2,8 @@
 swan_reset_sequence, pool_pages) against the ragged oracle (needs a GB300)."""
 from __future__ import annotations
 
+import copy
+
 import numpy as np
 import pytest
 
@@ -31,7 +33,7 @@ def run_ragged(ops, R, Rv, *, B, H_kv, G, k_store, cap, max_seq, page_tokens=0, 
                k_store_v=None, pool_pages=0):
     """Replay ragged ops on the ragged oracle and a libswan context.
     ops: ("append", k, v, n_new | None) | ("flush",) | ("reset", b) |
-    ("set_k", k[, k_v]) | ("decode", q).  Lengths are compared after every
+    ("fork", src, dst) | ("set_k", k[, k_v]) | ("decode", q).  Lengths are compared after every
     op, outputs after every decode."""
     import torch
 
@@ -55,6 +57,9 @@ def run_ragged(ops, R, Rv, *, B, H_kv, G, k_store, cap, max_seq, page_tokens=0, 
         elif op[0] == "reset":
             ref.reset(op[1])
             ctx.reset_sequence(op[1])
+        elif op[0] == "fork":  # the oracle's row dst becomes a copy of row src
+            ref.rows[op[2]] = copy.deepcopy(ref.rows[op[1]])
+            ctx.fork_sequence(op[1], op[2])
         elif op[0] == "set_k":
             ref.set_k(*op[1:])
             ctx.set_k(*op[1:])
@@ -243,3 +248,88 @@ def test_ragged_fp8_separate_counts_and_pool():
     ctx, ref, _ = run_ragged(ops, R, Rv, B=B, H_kv=H, G=G, k_store=40, cap=24, max_seq=900, page_tokens=P,
                              value_format="fp8_e4m3", k_store_v=24, pool_pages=pool)
     ctx.close()
+
+
+FORK_CASES = [
+    # B, H_kv, G, cap, k_store, P, fmt
+    (3, 2, 2, 32, 48, 64, "fp16"),
+    (3, 2, 1, 16, 64, 32, "fp8_e4m3"),
+    (4, 2, 8, 24, 56, 64, "fp16"),
+]
+
+
+@pytest.mark.parametrize("B,H,G,cap,ks,P,fmt", FORK_CASES)
+def test_fork_sequence_matches_oracle(B, H, G, cap, ks, P, fmt):
+    """Forked rows (swan_fork_sequence) against the oracle: the fork shares
+    the source's pages and copies its buffer, then both rows take different
+    tokens (the first appends write into the shared, partly filled last
+    page: copy on write), a fork onto a row that already holds tokens, a
+    flush, a reset and a second fork of a fork."""
+    R, Rv = _rot(H, 90 + G), _rot(H, 90 + G, synth.T_R_VO)
+    k, v = _kv(B, H, 1400, seed=91 + G)
+    q = _q(B, H * G, seed=92, scale=2.0)
+    n0 = [300] + [0] * (B - 2) + [150]
+    ops = [("append", k[:, :, :300].copy(), v[:, :, :300].copy(), n0), ("decode", q),
+           ("fork", 0, 1), ("decode", q),
+           ("append", k[:, :, 300:337].copy(), v[:, :, 300:337].copy(), [37, 21] + [5] * (B - 2)), ("decode", q),
+           ("append", k[:, :, 337:338].copy(), v[:, :, 337:338].copy(), [1] * B), ("decode", q),
+           ("fork", 1, B - 1), ("decode", q),
+           ("append", k[:, :, 338:700].copy(), v[:, :, 338:700].copy(), [362, 0] + [100] * (B - 2)), ("decode", q),
+           ("flush",), ("decode", q),
+           ("fork", B - 1, 0), ("reset", 1), ("decode", q),
+           ("append", k[:, :, 700:1300].copy(), v[:, :, 700:1300].copy(), [600, 300] + [77] * (B - 2)),
+           ("decode", q)]
+    pool = H * B * (1400 // P + 3)
+    ctx, ref, _ = run_ragged(ops, R, Rv, B=B, H_kv=H, G=G, k_store=ks, cap=cap, max_seq=1400, page_tokens=P,
+                             value_format=fmt, pool_pages=pool)
+    for b in range(B):
+        ctx.reset_sequence(b)
+    info = ctx.query(0)
+    assert info.free_pages == info.pool_pages  # every page back once no row holds it
+    ctx.close()
+
+
+def test_fork_shares_pages_and_isolates_rows():
+    """Page accounting and isolation: a fork takes no page until a row
+    writes into a shared page; the copy leaves the other row's output
+    bit for bit unchanged; forking needs a pool and two different rows."""
+    import torch
+
+    from paper_2511_18936_gb300 import swan
+    B, H, G, P, cap = 2, 2, 2, 64, 16
+    R, Rv = _rot(H, 97), _rot(H, 97, synth.T_R_VO)
+    k, v = _kv(B, H, 600, seed=98)
+    q = torch.from_numpy(_q(B, H * G, seed=99)).cuda()
+    ctx = swan.Context(torch.from_numpy(R)[None].cuda(), torch.from_numpy(Rv)[None].cuda(), num_layers=1,
+                       batch=B, n_q_heads=H * G, n_kv_heads=H, k_store=32, buffer_cap=cap, max_seq=600,
+                       page_tokens=P, pool_pages=64)
+    kt, vt = torch.from_numpy(k).cuda(), torch.from_numpy(v).cuda()
+    ctx.append(0, kt[:, :, :216].contiguous(), vt[:, :, :216].contiguous(), n_new=[216, 0])
+    free0 = ctx.query(0).free_pages                      # row 0: 200 sparse tokens, 4 pages a head
+    assert free0 == 64 - H * 4
+    ctx.fork_sequence(0, 1)
+    assert ctx.query(0).free_pages == free0              # shared, nothing copied yet
+    qq = torch.cat([q[:1], q[:1]])                       # the same query for both rows
+    out = ctx.decode(0, qq).float().cpu().numpy()
+    assert np.abs(out[0] - out[1]).max() <= TOL_OUT      # the same history (CTA splits may differ)
+    ctx.append(0, kt[:, :, 216:220].contiguous(), vt[:, :, 216:220].contiguous(), n_new=[4, 0])
+    assert ctx.query(0).free_pages == free0 - H          # row 0 copied its shared last page
+    ctx.append(0, kt[:, :, 220:224].contiguous(), vt[:, :, 220:224].contiguous(), n_new=[0, 4])
+    assert ctx.query(0).free_pages == free0 - H          # row 1 was the last holder: no copy
+    assert ctx.lengths(0) == ([204, 204], [16, 16])
+    ctx.reset_sequence(0)
+    ctx.reset_sequence(1)
+    assert ctx.query(0).free_pages == 64
+    for a, b in ((0, 0), (0, 2), (-1, 1)):
+        with pytest.raises(swan.SwanError) as e:
+            ctx.fork_sequence(a, b)
+        assert e.value.status == swan.ERR_INVALID_ARG
+    ctx.check()
+    ctx.check_guards()
+    ctx.close()
+    plain = swan.Context(torch.from_numpy(R)[None].cuda(), num_layers=1, batch=2, n_q_heads=H, n_kv_heads=H,
+                         k_store=32, buffer_cap=cap, max_seq=600)
+    with pytest.raises(swan.SwanError) as e:
+        plain.fork_sequence(0, 1)
+    assert e.value.status == swan.ERR_UNSUPPORTED
+    plain.close()

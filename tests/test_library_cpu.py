@@ -90,6 +90,7 @@ def test_null_arguments(lib):
     assert lib.swan_set_k(None, 4) == swan.ERR_INVALID_ARG
     assert lib.swan_set_kv(None, 4, 4) == swan.ERR_INVALID_ARG
     assert lib.swan_reset_sequence(None, 0) == swan.ERR_INVALID_ARG
+    assert lib.swan_fork_sequence(None, 0, 1) == swan.ERR_INVALID_ARG
     assert lib.swan_append_varlen(None, 0, None, None, 1, None) == swan.ERR_INVALID_ARG
     assert lib.swan_query_lengths(None, 0, None, None) == swan.ERR_INVALID_ARG
     assert lib.swan_debug_export_seq(None, 0, 0, 1, None, 0) == swan.ERR_INVALID_ARG

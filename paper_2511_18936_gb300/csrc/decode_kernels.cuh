@@ -468,6 +468,14 @@ __device__ __forceinline__ void finish_unit(const DecodeParams& p, int64_t c0, i
 // layer, while at 96 it took 1.72 against 1.99 ms).
 template <int MAXC>
 __host__ __device__ constexpr bool decode_two_slot() { return MAXC == 12; }
+// How many blocks ahead of use a warp asks L2 for a block's records.  Over
+// all resident warps the records in flight must stay well inside L2: at 96
+// entries read (1824 warps x 2 blocks x 18 KB = 66 MB) two blocks ahead
+// thrashed it (k 96 on the 32k layer: 1.52 ms at 2 blocks, 1.35-1.37 ms at
+// 1; k 128 1.853 -> 1.833 ms), while up to 64 entries (44 MB) two stay best
+// (k 32, 48: 1 % slower at one block).
+template <int MAXC>
+__host__ __device__ constexpr int decode_prefetch_ahead() { return MAXC > 8 ? 1 : 2; }
 // Warps per CTA of the one-head kernel: one lane-private accumulator each
 // (16 KB); for 16 chunks as many as the registers allow.
 template <int MAXC>
@@ -491,7 +499,8 @@ __host__ __device__ constexpr int decode_q_shift() { return MAXC <= 12 ? 6 : 7; 
 //   aligned region when it fits there, else after the accumulators.
 //   Lane = token; each warp walks a contiguous run of blocks.  While block g
 //   is processed, the key records of block g+1 are in flight to registers
-//   and block g+2 is being prefetched into L2.
+//   and block g+2 (g+1 for the variants that read more than 64 entries) is
+//   being prefetched into L2.
 template <int MAXC, int FMT>
 __global__ void __launch_bounds__(decode_warps<MAXC>() * 32, decode_min_ctas<MAXC>())
     decode_kernel(DecodeParams p) {
@@ -712,9 +721,9 @@ __global__ void __launch_bounds__(decode_warps<MAXC>() * 32, decode_min_ctas<MAX
           // previous block) are scored
           Chunk<FMT> vc[KS];
           load_slot(vc, 0, nchunks_v, o_vv, o_vi);
-          // two blocks ahead: into L2
+          // one or two blocks ahead: into L2
           const uint8_t* b_n2 = block_of(gi + 2);
-          prefetch_block(b_n2);
+          prefetch_block(decode_prefetch_ahead<MAXC>() == 2 ? b_n2 : b_n1);
           score_slot(kc, 0);
           s2 = valid ? ((s[0] + s[1]) + (s[2] + s[3])) * p.scale_log2 : -INFINITY;
           // the next block's key records into registers while this block's
@@ -733,7 +742,7 @@ __global__ void __launch_bounds__(decode_warps<MAXC>() * 32, decode_min_ctas<MAX
           Chunk<FMT> cy[KY];
           load_slot(cy, KS, nchunks, o_kv, o_ki);
           const uint8_t* b_n2 = block_of(gi + 2);
-          prefetch_block(b_n2);
+          prefetch_block(decode_prefetch_ahead<MAXC>() == 2 ? b_n2 : b_n1);
           score_slot(kc, 0);
           load_slot(kc, 0, nchunks_v, o_vv, o_vi);
           score_slot(cy, KS);

@@ -42,7 +42,7 @@ def _steps(B, T_list, ragged, seed):
 
 @pytest.mark.parametrize("G,fmt,ragged,cap", [(1, "fp16", False, 8), (2, "fp16", True, 8),
                                               (4, "fp8_e4m3", False, 4), (1, "fp16", True, 0),
-                                              (2, "fp8_e4m3", True, 16)])
+                                              (2, "fp8_e4m3", True, 16), (8, "fp16", True, 8)])
 def test_append_decode_equals_append_then_decode(G, fmt, ragged, cap):
     import torch
 

@@ -240,6 +240,8 @@ DECODE_CASES = [
     (3, 2, 4, 300, 0, 24, (24, 5), 32),             # no buffer at all
     (2, 2, 8, 1300, 64, 56, (56, 40, 3), 64),       # GQA G = 8 (two 16-byte q' gathers)
     (1, 2, 8, 600, 32, 128, (128, 80), 32),         # G = 8, more than 64 entries read
+    (2, 1, 8, 40, 64, 32, (32, 9), 32),             # G = 8, dense buffer only
+    (1, 2, 8, 333, 0, 40, (40, 17), 32),            # G = 8, no buffer at all
 ]
 
 

@@ -560,3 +560,24 @@ def test_runtime_value_prefix_equals_stored_split():
         split.close()
     full.check()
     full.close()
+
+
+@pytest.mark.parametrize("G,fmt", [(1, "fp16"), (4, "fp8_e4m3")])
+def test_maximum_buffer_page_and_keep_sizes(G, fmt):
+    """The largest sizes the header allows for the dense buffer (4096 tokens)
+    and a page (4096 tokens, 128 blocks), with every coordinate stored
+    (k_store 128) and read back at k 128 and below: 128 buffer groups per
+    unit, a sparse history over two pages, both kernel families."""
+    B, H, cap, P, ks = 1, 2, 4096, 4096, 128
+    L = cap + 4500
+    R, Rv = _rot(H, 140 + G), _rot(H, 140 + G, synth.T_R_VO)
+    k, v = _kv(B, H, L, seed=141)
+    q = _q(B, H * G, seed=142, scale=2.0)
+    ops = [("append", k[:, :, :5000].copy(), v[:, :, :5000].copy()), ("decode", q),
+           ("append", k[:, :, 5000:].copy(), v[:, :, 5000:].copy()), ("decode", q),
+           ("set_k", 100), ("decode", q), ("flush",), ("decode", q)]
+    ctx, ref, outs = run_ops(ops, R, Rv, B=B, H_kv=H, G=G, k_store=ks, cap=cap, page_tokens=P,
+                             value_format=fmt)
+    for got, want in outs:
+        assert np.abs(got - want).max() <= TOL_OUT
+    ctx.close()

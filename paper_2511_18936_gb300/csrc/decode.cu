@@ -1,7 +1,7 @@
 // Decode attention on the packed sparse cache (Algorithm 1, attention part;
 // Section 4.3): the query rotation q' = q R_qk, the empty-cache combine, and
-// the host launchers of the kernels in decode_kernels.cuh.
-#include "decode_kernels.cuh"
+// the host launchers of the kernels in decode_kernels.cuh and decode_mma.cuh.
+#include "decode_mma.cuh"
 
 namespace swan {
 namespace {

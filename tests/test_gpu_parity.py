@@ -506,6 +506,9 @@ ASYM_DECODE_CASES = [
     (2, 2, 1, 1000, 64, 64, 32, [(64, 32), (40, 5)], 128, "fp8_e4m3"),
     (2, 2, 4, 900, 32, 96, 16, [(96, 16), (65, 16)], 32, "fp8_e4m3"),
     (2, 2, 8, 1100, 32, 40, 80, [(40, 80), (33, 71)], 64, "fp16"),
+    # G = 8 with at most 64 entries read: scores from the key tile on the tensor cores
+    (2, 2, 8, 1100, 32, 56, 24, [(56, 24), (13, 17)], 64, "fp16"),
+    (2, 2, 8, 900, 16, 24, 56, [(24, 56), (9, 56)], 32, "fp8_e4m3"),
 ]
 
 

@@ -78,3 +78,23 @@ def test_profile_traffic_requires_matching_source_hashes(tmp_path, monkeypatch):
 
 def test_host_cores_is_the_affinity_set():
     assert bench.host_cores() == len(os.sched_getaffinity(0))
+
+
+def test_committed_profiles_are_reproducible_summaries():
+    # every ncu command a summary gives leaves the clocks alone, names only
+    # committed entry points, and every kernel file a summary hashes exists
+    import glob
+    import re
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    files = glob.glob(os.path.join(root, "profiles", "*.md"))
+    assert files
+    for path in files:
+        text = open(path).read()
+        cmds = re.findall(r"^[ \t]*ncu (?:[^\n]*\\\n)*[^\n]*", text, flags=re.M)
+        assert cmds, path
+        for cmd in cmds:
+            assert "--clock-control none" in cmd, (path, cmd)
+            assert "_work" not in cmd, (path, cmd)
+            assert re.search(r"python (bench\.py|-c)", cmd), (path, cmd)
+        for name in re.findall(r"([\w.]+\.(?:cuh|cu)) sha256\[:16\]", text):
+            assert os.path.exists(os.path.join(root, "paper_2511_18936_gb300", "csrc", name)), (path, name)
